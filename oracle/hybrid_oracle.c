@@ -1,0 +1,356 @@
+/*
+ * hybrid_oracle.c -- plain fp64 CPU oracle for block-hybrid attention.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the independent reference that the
+ * CUDA path is checked against.  Only the test suite, the smoke check and the
+ * CPU-baseline leg of the benchmark may load it.  It shares no code, header,
+ * table or helper with the CUDA library, and it never reads anything the
+ * CUDA library produced except where a caller passes such data in explicitly.
+ *
+ * Source: "Retrofitting Linear Attention into Diffusion Language Models",
+ * Section 3.1 (block-hybrid attention) and Section 2.2 (linear attention,
+ * Eq. 1).  Every routine below writes a definition of that section out
+ * literally, in double precision, with no blocking, fusion or reordering:
+ *
+ *   phi(x)   = [softmax(x W), softmax(-x W)]            (Sec. 3.1, Hedgehog map)
+ *   a_j      = exp(q . k_j / sqrt(d)),  j in active block (Sec. 3.1)
+ *   sm_num   = sum_j a_j v_j,   sm_den = sum_j a_j       (Sec. 3.1)
+ *   S_n      = S_{n-1} + sum_t phi(k_t) v_t^T            (Sec. 3.1, commit)
+ *   Z_n      = Z_{n-1} + sum_t phi(k_t)                  (Sec. 3.1, commit)
+ *   lin_num  = phi(q)^T S_{n-1},  lin_den = phi(q)^T Z_{n-1}   (Sec. 3.1)
+ *   w        = sigmoid(alpha)                            (Sec. 3.1, gate)
+ *   out      = (w sm_num + lin_num) / (w sm_den + lin_den)      (Sec. 3.1)
+ *
+ * A second route (oracle_block_attn_prefix) never forms S or Z: it sums the
+ * linear branch token by token over the explicit prefix, the left-hand form
+ * of Eq. 1.  The two routes are a mutual check (state = explicit sum).
+ *
+ * Readings of points the paper leaves open (each is listed in the design
+ * notes as well):
+ *   - W is indexed per state (key/value) head; query head h of a GQA group of
+ *     size G = Hq / Hkv uses the W and the state of head h / G.  With
+ *     Hq == Hkv this is the paper's "per query head" design.
+ *   - The gate alpha is per query head.
+ *   - No scale or temperature inside phi; 1/sqrt(d) only in the softmax branch.
+ *   - No mask inside the active block (bidirectional, all B x B pairs).
+ *   - The softmax inside phi and the exponentials of the softmax branch are
+ *     evaluated unshifted, exactly as defined; the routines refuse inputs whose
+ *     exponent arguments leave [-700, 700] (fp64 would overflow).
+ *
+ * Logical layouts (all row-major, double):
+ *   Q, O     [n_req][B][Hq][d]
+ *   K, V     [n_req][T][Hkv][d]      (T = B for the active block)
+ *   W        [Hkv][d][F]
+ *   alpha    [Hq]
+ *   S        [n_req][Hkv][2F][d]     (the paper's S in R^{2F x d})
+ *   z        [n_req][Hkv][2F]        (the paper's Z)
+ *
+ * phi_kind 0 = Hedgehog (the paper's map), 1 = identity (phi(x) = x, 2F := d;
+ * used only to pin the oracle against the plain linear-attention formula).
+ *
+ * Return value of every entry point: 0 on success, -1 on a bad argument,
+ * -2 if an exponent argument left [-700, 700].
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORACLE_EXP_LIMIT 700.0
+
+enum { PHI_HEDGEHOG = 0, PHI_IDENTITY = 1 };
+
+/* Width of phi(x): 2F for the Hedgehog map, d for the identity map. */
+static int phi_width(int phi_kind, int d, int F)
+{
+    return phi_kind == PHI_IDENTITY ? d : 2 * F;
+}
+
+/*
+ * phi(x) for one vector x in R^d with W in R^{d x F} (Sec. 3.1):
+ *   u      = x W                     (u_f = sum_e x_e W[e][f])
+ *   out[f]     = exp(u_f)  / sum_g exp(u_g)      f = 0..F-1   (softmax(xW))
+ *   out[F + f] = exp(-u_f) / sum_g exp(-u_g)     f = 0..F-1   (softmax(-xW))
+ * Returns -2 if some |u_f| exceeds the fp64 exponent limit.
+ */
+static int phi_one(int phi_kind, const double *x, const double *W, int d, int F,
+                   double *u /* scratch, F */, double *out)
+{
+    if (phi_kind == PHI_IDENTITY) {
+        for (int e = 0; e < d; ++e) out[e] = x[e];
+        return 0;
+    }
+    for (int f = 0; f < F; ++f) {
+        double acc = 0.0;
+        for (int e = 0; e < d; ++e) acc += x[e] * W[(size_t)e * F + f];
+        if (fabs(acc) > ORACLE_EXP_LIMIT) return -2;
+        u[f] = acc;
+    }
+    double sum_pos = 0.0, sum_neg = 0.0;
+    for (int f = 0; f < F; ++f) {
+        sum_pos += exp(u[f]);
+        sum_neg += exp(-u[f]);
+    }
+    for (int f = 0; f < F; ++f) {
+        out[f] = exp(u[f]) / sum_pos;
+        out[F + f] = exp(-u[f]) / sum_neg;
+    }
+    return 0;
+}
+
+/* ---------------------------------------------------------------------------
+ * Feature map on a batch of rows.
+ *   X   [n_rows][n_heads_x][d],  W [Hkv][d][F],  Phi [n_rows][n_heads_x][2F]
+ * Row head h uses W[h / (n_heads_x / Hkv)] (queries: h / G; keys: h).
+ * ------------------------------------------------------------------------- */
+int oracle_feature_map(long n_rows, int n_heads_x, int n_kv_heads, int d, int F,
+                       const double *X, const double *W, double *Phi)
+{
+    if (n_rows < 0 || n_heads_x <= 0 || n_kv_heads <= 0 || d <= 0 || F <= 0) return -1;
+    if (n_heads_x % n_kv_heads != 0) return -1;
+    const int group = n_heads_x / n_kv_heads;
+    double *u = (double *)malloc(sizeof(double) * (size_t)F);
+    if (!u) return -1;
+    int rc = 0;
+    for (long r = 0; r < n_rows && rc == 0; ++r) {
+        for (int h = 0; h < n_heads_x && rc == 0; ++h) {
+            const double *x = X + ((size_t)r * n_heads_x + h) * d;
+            const double *Wg = W + (size_t)(h / group) * d * F;
+            rc = phi_one(PHI_HEDGEHOG, x, Wg, d, F, u, Phi + ((size_t)r * n_heads_x + h) * 2 * F);
+        }
+    }
+    free(u);
+    return rc;
+}
+
+/* ---------------------------------------------------------------------------
+ * Simple static fan-out of independent (request, head) units over threads.
+ * Units never share an output element, so the split changes no result.
+ * ------------------------------------------------------------------------- */
+typedef int (*unit_fn)(void *ctx, long unit, double *scratch);
+
+typedef struct {
+    unit_fn fn;
+    void *ctx;
+    long n_units;
+    int n_threads;
+    int tid;
+    size_t scratch_doubles;
+    int rc;
+} fanout_arg;
+
+static void *fanout_worker(void *p)
+{
+    fanout_arg *a = (fanout_arg *)p;
+    double *scratch = (double *)malloc(sizeof(double) * (a->scratch_doubles ? a->scratch_doubles : 1));
+    if (!scratch) { a->rc = -1; return NULL; }
+    a->rc = 0;
+    for (long u = a->tid; u < a->n_units; u += a->n_threads) {
+        int rc = a->fn(a->ctx, u, scratch);
+        if (rc != 0) { a->rc = rc; break; }
+    }
+    free(scratch);
+    return NULL;
+}
+
+static int fanout(unit_fn fn, void *ctx, long n_units, int n_threads, size_t scratch_doubles)
+{
+    if (n_threads < 1) n_threads = 1;
+    if (n_threads > 1024) n_threads = 1024;
+    if ((long)n_threads > n_units) n_threads = n_units > 0 ? (int)n_units : 1;
+    fanout_arg *args = (fanout_arg *)calloc((size_t)n_threads, sizeof(fanout_arg));
+    pthread_t *th = (pthread_t *)calloc((size_t)n_threads, sizeof(pthread_t));
+    if (!args || !th) { free(args); free(th); return -1; }
+    for (int t = 0; t < n_threads; ++t) {
+        args[t].fn = fn; args[t].ctx = ctx; args[t].n_units = n_units;
+        args[t].n_threads = n_threads; args[t].tid = t;
+        args[t].scratch_doubles = scratch_doubles;
+    }
+    int started = 0;
+    for (int t = 1; t < n_threads; ++t) {
+        if (pthread_create(&th[t], NULL, fanout_worker, &args[t]) != 0) break;
+        started = t;
+    }
+    fanout_worker(&args[0]);
+    for (int t = 1; t <= started; ++t) pthread_join(th[t], NULL);
+    int rc = 0;
+    for (int t = 0; t < n_threads; ++t) if (args[t].rc != 0) rc = args[t].rc;
+    if (started != n_threads - 1) rc = -1;
+    free(args); free(th);
+    return rc;
+}
+
+/* ---------------------------------------------------------------------------
+ * Block commit (Sec. 3.1):  S += sum_t phi(k_t) v_t^T,   z += sum_t phi(k_t)
+ * for every (request, state head), over the T given tokens, in token order.
+ * ------------------------------------------------------------------------- */
+typedef struct {
+    int n_req, T, Hkv, d, F, phi_kind;
+    const double *K, *V, *W;
+    double *S, *z;
+} commit_ctx;
+
+static int commit_unit(void *p, long unit, double *scratch)
+{
+    const commit_ctx *c = (const commit_ctx *)p;
+    const int r = (int)(unit / c->Hkv), g = (int)(unit % c->Hkv);
+    const int d = c->d, F = c->F, P2 = phi_width(c->phi_kind, d, F);
+    double *u = scratch, *phi = scratch + F;
+    double *S = c->S + ((size_t)r * c->Hkv + g) * P2 * d;
+    double *z = c->z + ((size_t)r * c->Hkv + g) * P2;
+    const double *Wg = c->W ? c->W + (size_t)g * d * F : NULL;
+    for (int t = 0; t < c->T; ++t) {
+        const double *k = c->K + (((size_t)r * c->T + t) * c->Hkv + g) * d;
+        const double *v = c->V + (((size_t)r * c->T + t) * c->Hkv + g) * d;
+        int rc = phi_one(c->phi_kind, k, Wg, d, F, u, phi);
+        if (rc) return rc;
+        for (int f = 0; f < P2; ++f) {
+            for (int e = 0; e < d; ++e) S[(size_t)f * d + e] += phi[f] * v[e];
+            z[f] += phi[f];
+        }
+    }
+    return 0;
+}
+
+int oracle_commit(int n_req, int T, int Hkv, int d, int F, int phi_kind,
+                  const double *K, const double *V, const double *W,
+                  double *S, double *z, int n_threads)
+{
+    if (n_req < 0 || T < 0 || Hkv <= 0 || d <= 0 || F <= 0) return -1;
+    if (phi_kind != PHI_HEDGEHOG && phi_kind != PHI_IDENTITY) return -1;
+    if (phi_kind == PHI_HEDGEHOG && !W) return -1;
+    commit_ctx c = { n_req, T, Hkv, d, F, phi_kind, K, V, W, S, z };
+    const int P2 = phi_width(phi_kind, d, F);
+    return fanout(commit_unit, &c, (long)n_req * Hkv, n_threads, (size_t)F + (size_t)P2);
+}
+
+/* ---------------------------------------------------------------------------
+ * One active block, both branches, gated shared normaliser (Sec. 3.1).
+ * The cross-block branch comes either from the state (S, z) or, in the
+ * second route, from the explicit prefix tokens (Eq. 1 summed directly).
+ * ------------------------------------------------------------------------- */
+typedef struct {
+    int n_req, B, Hq, Hkv, d, F, phi_kind;
+    const double *Q, *K, *V, *W, *alpha;
+    /* route 1: state */
+    const double *S, *z;
+    /* route 2: explicit prefix */
+    const double *Kp, *Vp;
+    const int *prefix_len;
+    int P_max;
+    double *O;
+} attn_ctx;
+
+static int attn_unit(void *p, long unit, double *scratch)
+{
+    const attn_ctx *c = (const attn_ctx *)p;
+    const int r = (int)(unit / c->Hq), h = (int)(unit % c->Hq);
+    const int d = c->d, F = c->F, B = c->B;
+    const int G = c->Hq / c->Hkv, g = h / G;
+    const int P2 = phi_width(c->phi_kind, d, F);
+    const double *Wg = c->W ? c->W + (size_t)g * d * F : NULL;
+
+    double *u = scratch;                 /* F      */
+    double *phi_q = u + F;               /* P2     */
+    double *phi_k = phi_q + P2;          /* P2     */
+    double *sm_num = phi_k + P2;         /* d      */
+    double *lin_num = sm_num + d;        /* d      */
+
+    /* gate w = sigma(alpha) = 1 / (1 + exp(-alpha)); alpha = -inf gives 0, +inf gives 1 */
+    const double w = 1.0 / (1.0 + exp(-c->alpha[h]));
+
+    for (int i = 0; i < B; ++i) {
+        const double *q = c->Q + (((size_t)r * B + i) * c->Hq + h) * d;
+
+        /* within-block softmax branch: a_j = exp(q . k_j / sqrt(d)) over all j of the block */
+        double sm_den = 0.0;
+        for (int e = 0; e < d; ++e) sm_num[e] = 0.0;
+        for (int j = 0; j < B; ++j) {
+            const double *k = c->K + (((size_t)r * B + j) * c->Hkv + g) * d;
+            const double *v = c->V + (((size_t)r * B + j) * c->Hkv + g) * d;
+            double s = 0.0;
+            for (int e = 0; e < d; ++e) s += q[e] * k[e];
+            s /= sqrt((double)d);
+            if (fabs(s) > ORACLE_EXP_LIMIT) return -2;
+            const double a = exp(s);
+            for (int e = 0; e < d; ++e) sm_num[e] += a * v[e];
+            sm_den += a;
+        }
+
+        /* cross-block linear branch */
+        int rc = phi_one(c->phi_kind, q, Wg, d, F, u, phi_q);
+        if (rc) return rc;
+        double lin_den = 0.0;
+        for (int e = 0; e < d; ++e) lin_num[e] = 0.0;
+        if (c->S) {
+            /* route 1: lin_num = phi(q)^T S, lin_den = phi(q)^T z */
+            const double *S = c->S + ((size_t)r * c->Hkv + g) * P2 * d;
+            const double *z = c->z + ((size_t)r * c->Hkv + g) * P2;
+            for (int f = 0; f < P2; ++f) {
+                for (int e = 0; e < d; ++e) lin_num[e] += phi_q[f] * S[(size_t)f * d + e];
+                lin_den += phi_q[f] * z[f];
+            }
+        } else {
+            /* route 2: lin_num = sum_t (phi(q) . phi(k_t)) v_t over the prefix tokens (Eq. 1) */
+            const int P = c->prefix_len[r];
+            for (int t = 0; t < P; ++t) {
+                const double *kt = c->Kp + (((size_t)r * c->P_max + t) * c->Hkv + g) * d;
+                const double *vt = c->Vp + (((size_t)r * c->P_max + t) * c->Hkv + g) * d;
+                rc = phi_one(c->phi_kind, kt, Wg, d, F, u, phi_k);
+                if (rc) return rc;
+                double kern = 0.0;
+                for (int f = 0; f < P2; ++f) kern += phi_q[f] * phi_k[f];
+                for (int e = 0; e < d; ++e) lin_num[e] += kern * vt[e];
+                lin_den += kern;
+            }
+        }
+
+        /* gated merge through the shared normaliser */
+        double *o = c->O + (((size_t)r * B + i) * c->Hq + h) * d;
+        const double den = w * sm_den + lin_den;
+        for (int e = 0; e < d; ++e) o[e] = (w * sm_num[e] + lin_num[e]) / den;
+    }
+    return 0;
+}
+
+static int attn_check(int n_req, int B, int Hq, int Hkv, int d, int F, int phi_kind,
+                      const double *W)
+{
+    if (n_req < 0 || B <= 0 || Hq <= 0 || Hkv <= 0 || d <= 0 || F <= 0) return -1;
+    if (Hq % Hkv != 0) return -1;
+    if (phi_kind != PHI_HEDGEHOG && phi_kind != PHI_IDENTITY) return -1;
+    if (phi_kind == PHI_HEDGEHOG && !W) return -1;
+    return 0;
+}
+
+int oracle_block_attn(int n_req, int B, int Hq, int Hkv, int d, int F, int phi_kind,
+                      const double *Q, const double *K, const double *V,
+                      const double *W, const double *alpha,
+                      const double *S, const double *z, double *O, int n_threads)
+{
+    if (attn_check(n_req, B, Hq, Hkv, d, F, phi_kind, W) || !S || !z) return -1;
+    attn_ctx c;
+    memset(&c, 0, sizeof c);
+    c.n_req = n_req; c.B = B; c.Hq = Hq; c.Hkv = Hkv; c.d = d; c.F = F; c.phi_kind = phi_kind;
+    c.Q = Q; c.K = K; c.V = V; c.W = W; c.alpha = alpha; c.S = S; c.z = z; c.O = O;
+    const int P2 = phi_width(phi_kind, d, F);
+    return fanout(attn_unit, &c, (long)n_req * Hq, n_threads, (size_t)F + 2u * P2 + 2u * d);
+}
+
+int oracle_block_attn_prefix(int n_req, int B, int Hq, int Hkv, int d, int F, int phi_kind,
+                             const double *Q, const double *K, const double *V,
+                             const double *W, const double *alpha,
+                             const double *Kp, const double *Vp, const int *prefix_len,
+                             int P_max, double *O, int n_threads)
+{
+    if (attn_check(n_req, B, Hq, Hkv, d, F, phi_kind, W) || !prefix_len || P_max < 0) return -1;
+    for (int r = 0; r < n_req; ++r)
+        if (prefix_len[r] < 0 || prefix_len[r] > P_max) return -1;
+    attn_ctx c;
+    memset(&c, 0, sizeof c);
+    c.n_req = n_req; c.B = B; c.Hq = Hq; c.Hkv = Hkv; c.d = d; c.F = F; c.phi_kind = phi_kind;
+    c.Q = Q; c.K = K; c.V = V; c.W = W; c.alpha = alpha;
+    c.Kp = Kp; c.Vp = Vp; c.prefix_len = prefix_len; c.P_max = P_max; c.O = O;
+    const int P2 = phi_width(phi_kind, d, F);
+    return fanout(attn_unit, &c, (long)n_req * Hq, n_threads, (size_t)F + 2u * P2 + 2u * d);
+}

@@ -1,0 +1,65 @@
+"""Each plausible mistake, planted in a temporary copy of the oracle's C source
+(never in the oracle itself), must trip at least one pin of oracle_pins.py.
+
+This shows that the pins constrain every part of the oracle: the feature map,
+its W orientation, the softmax scale, the gate, the shared normaliser, the
+commit, the GQA head mapping and the in-block mask.  Mutants run in a
+subprocess, so a mutant that crashes counts as caught without harming the
+test process.
+"""
+import os
+import subprocess
+import sys
+
+import pytest
+
+from oracle import SOURCE, build_oracle
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+
+# (name, exact text in the oracle source, replacement)
+MUTANTS = [
+    ("softmax scale 1/d", "s /= sqrt((double)d);", "s /= (double)d;"),
+    ("softmax scale dropped", "s /= sqrt((double)d);", "s /= 1.0;"),
+    ("phi negative half sign", "out[F + f] = exp(-u[f]) / sum_neg;", "out[F + f] = exp(u[f]) / sum_neg;"),
+    ("phi negative normaliser sign", "sum_neg += exp(-u[f]);", "sum_neg += exp(u[f]);"),
+    ("phi W transposed", "acc += x[e] * W[(size_t)e * F + f];", "acc += x[e] * W[((size_t)f * d + e) % ((size_t)d * F)];"),
+    ("phi halves swapped", "out[f] = exp(u[f]) / sum_pos;\n        out[F + f] = exp(-u[f]) / sum_neg;",
+     "out[F + f] = exp(u[f]) / sum_pos;\n        out[f] = exp(-u[f]) / sum_neg;"),
+    ("gate sign", "const double w = 1.0 / (1.0 + exp(-c->alpha[h]));", "const double w = 1.0 / (1.0 + exp(c->alpha[h]));"),
+    ("gate dropped in numerator", "o[e] = (w * sm_num[e] + lin_num[e]) / den;", "o[e] = (sm_num[e] + lin_num[e]) / den;"),
+    ("gate on the wrong branch", "const double den = w * sm_den + lin_den;", "const double den = sm_den + w * lin_den;"),
+    ("separate normalisers", "o[e] = (w * sm_num[e] + lin_num[e]) / den;",
+     "o[e] = w * sm_num[e] / sm_den + (lin_den > 0 ? lin_num[e] / lin_den : 0.0);"),
+    ("z not accumulated", "z[f] += phi[f];", "z[f] += 0.0 * phi[f];"),
+    ("lin_den ignores phi(q)", "lin_den += phi_q[f] * z[f];", "lin_den += z[f];"),
+    ("state read transposed", "lin_num[e] += phi_q[f] * S[(size_t)f * d + e];",
+     "lin_num[e] += phi_q[f] * S[((size_t)e * P2 + f) % ((size_t)P2 * d)];"),
+    ("commit drops last token", "for (int t = 0; t < c->T; ++t) {", "for (int t = 0; t < c->T - 1; ++t) {"),
+    ("causal mask inside the block", "for (int j = 0; j < B; ++j) {", "for (int j = 0; j <= i; ++j) {"),
+    ("GQA mapping modulo", "const int G = c->Hq / c->Hkv, g = h / G;", "const int G = c->Hq / c->Hkv, g = h % c->Hkv;"),
+    ("prefix route skips last token", "for (int t = 0; t < P; ++t) {", "for (int t = 0; t + 1 < P; ++t) {"),
+    ("value index shifted", "for (int e = 0; e < d; ++e) sm_num[e] += a * v[e];",
+     "for (int e = 0; e < d; ++e) sm_num[e] += a * v[(e + 1) % d];"),
+]
+
+
+@pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_mutant_is_caught(tmp_path, name, old, new):
+    src = open(SOURCE).read()
+    assert src.count(old) == 1, f"mutation site for '{name}' not found exactly once"
+    mutant_src = tmp_path / "mutant.c"
+    mutant_src.write_text(src.replace(old, new))
+    lib = build_oracle(str(mutant_src), str(tmp_path / "libmutant.so"))
+    proc = subprocess.run([sys.executable, os.path.join(HERE, "oracle_pins.py"), lib],
+                          capture_output=True, text=True, timeout=300)
+    caught = proc.returncode != 0 or "FAIL" in proc.stdout
+    assert caught, f"mutant '{name}' passed every pin:\n{proc.stdout}\n{proc.stderr}"
+
+
+def test_unmutated_copy_passes(tmp_path):
+    """Control: the same harness on an unmodified copy reports no failure."""
+    lib = build_oracle(SOURCE, str(tmp_path / "libcontrol.so"))
+    proc = subprocess.run([sys.executable, os.path.join(HERE, "oracle_pins.py"), lib],
+                          capture_output=True, text=True, timeout=300)
+    assert proc.returncode == 0 and "FAIL" not in proc.stdout and "DONE" in proc.stdout, proc.stdout
