@@ -1,0 +1,454 @@
+#!/usr/bin/env python3
+"""Benchmark of the block-hybrid decoding hot path on GB300.
+
+One step = one denoising step of block-hybrid attention over the active block
+of every request (hybrid_block_attn) followed by the commit of that block into
+the per-request states (hybrid_commit_block): every stage of Section 3.1's
+per-block computation, for the batch-64 ragged-prefix GQA workload by default.
+
+Metric: active-block tokens per second = n_req * B * steps / time.
+
+Timing: CUDA events on the launching stream; W untimed warm-up steps, then
+exactly K timed steps bracketed by a barrier and torch.cuda.synchronize();
+L2 is defeated by rotating through independent buffer sets whose total size is
+more than 4x the L2.  With --gpus N (launched by torchrun) every rank runs its
+own independent batch (weak scaling, no collective on the data path) and the
+slowest rank's time is used.
+
+--impl reference times the fp64 CPU oracle instead (host cores, bounded
+sample per step), printing the same JSON line with "impl": "reference".
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "active-block tokens/sec per denoising step at batch 64; HBM GB/s vs GB300 peak"
+FALLBACK_HBM_GBS = 6800.0
+
+
+# ---------------------------------------------------------------------------
+# helpers
+# ---------------------------------------------------------------------------
+def dist_info():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def max_over_ranks(value: float, ws: int, device=None) -> float:
+    """Max of a float over all ranks (identity for a single process)."""
+    if ws <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(ws: int):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            return json.load(fh), "measured"
+    except (OSError, ValueError):
+        return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
+
+
+def source_sha(paths):
+    h = hashlib.sha256()
+    for p in paths:
+        with open(os.path.join(ROOT, p), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, workload: str):
+    """Per-launch DRAM bytes from a committed ncu summary, or None if absent or
+    taken on a different build of the kernel's source."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as fh:
+            rec = json.load(fh).get(kernel)
+    except (OSError, ValueError):
+        return None
+    if not rec or rec.get("workload") != workload:
+        return None
+    if rec.get("source_sha") != source_sha(rec.get("sources", [])):
+        return None
+    return rec.get("bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 100 ms."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    REASONS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, bus_id: str | None):
+        self.samples = []   # (t, sm_mhz, max_mhz, reasons)
+        self.proc = None
+        self.bus_id = bus_id
+        self.thread = None
+
+    def start(self):
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "100"]
+        if self.bus_id:
+            cmd += ["-i", self.bus_id]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm, mx = float(parts[1]), float(parts[2])
+            except ValueError:
+                continue
+            reasons = [n for n, v in zip(self.REASONS, parts[5:9]) if v.lower() == "active"]
+            self.samples.append((time.time(), sm, mx, reasons))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        if self.thread is not None:
+            self.thread.join(timeout=5)
+
+    def summary(self, t0, t1):
+        inside = [s for s in self.samples if t0 <= s[0] <= t1]
+        window = "timed region"
+        if not inside:
+            inside = [s for s in self.samples if t0 - 2.0 <= s[0] <= t1 + 0.5]
+            window = "timed region +-2 s (timed region shorter than the 100 ms sampling period)"
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0,
+                    "window": "no nvidia-smi samples"}
+        reasons = sorted({r for s in inside for r in s[3]})
+        return {"sm_mhz": float(np.median([s[1] for s in inside])),
+                "sm_max_mhz": float(max(s[2] for s in inside)),
+                "reasons": reasons, "samples": len(inside), "window": window}
+
+
+def bus_id_of(torch, dev):
+    try:
+        p = torch.cuda.get_device_properties(dev)
+        return f"{p.pci_domain_id:08X}:{p.pci_bus_id:02X}:{p.pci_device_id:02X}.0"
+    except Exception:  # noqa: BLE001
+        return None
+
+
+# ---------------------------------------------------------------------------
+# algorithmic bytes (per launch) of the two kernels
+# ---------------------------------------------------------------------------
+def algorithmic_bytes(wl, io_bytes):
+    n, B, Hq, Hkv, d, F = wl.n_req, wl.B, wl.Hq, wl.Hkv, wl.d, wl.F
+    q = n * B * Hq * d * io_bytes
+    kv = n * B * Hkv * d * io_bytes
+    state = n * Hkv * (2 * F * d + 2 * F) * 4
+    w = Hkv * d * F * io_bytes
+    attn = q + q + 2 * kv + state + w + Hq * 4 + n * 8          # Q, O, K, V, (S, z), W, alpha, ptrs
+    commit = 2 * kv + 2 * state + w + n * 8                      # K, V, read+write (S, z), W, ptrs
+    return {"attn": attn, "commit": commit, "q": q, "kv": kv, "state": state}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle baseline
+# ---------------------------------------------------------------------------
+def oracle_sample_step(wl, orc, n_sample, tag, W64, alpha64):
+    """One oracle step (block attention + commit) on n_sample requests."""
+    import torch
+    from paper_2608_06628_gb300 import workloads as wk
+    Q, K, V = wk.block_qkv(wl, tag, "cpu", n_req=n_sample)
+    Q64, K64, V64 = (t.to(torch.float64).numpy() for t in (Q, K, V))
+    S, z = orc.empty_state(n_sample, wl.Hkv, wl.d, wl.F)
+    t0 = time.perf_counter()
+    orc.block_attn(Q64, K64, V64, W64, alpha64, S, z)
+    orc.commit(K64, V64, W64, S, z)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(wl, budget_s=12.0):
+    """Time the oracle as it stands on the host cores: whole-batch-shaped steps
+    of the workload (n_sample requests each), repeated for about budget_s."""
+    import oracle
+    from paper_2608_06628_gb300 import workloads as wk
+    orc = oracle.load()
+    cores = oracle.default_threads()
+    W, alpha = wk.params(wl)
+    W64 = W.double().numpy()
+    alpha64 = alpha.double().numpy()
+    n_sample = min(wl.n_req, 16)
+    t_one = oracle_sample_step(wl, orc, n_sample, "cpu-probe", W64, alpha64)
+    reps = max(1, min(50, int(budget_s / max(t_one, 1e-6))))
+    tot = 0.0
+    for i in range(reps):
+        tot += oracle_sample_step(wl, orc, n_sample, ("cpu", i), W64, alpha64)
+    tokens = reps * n_sample * wl.B
+    return {"value": tokens / tot, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{reps} steps x {n_sample} of {wl.n_req} requests (block attention + commit, "
+                      f"fp64 C oracle, {cores} threads), {tot:.1f} s"}
+
+
+# ---------------------------------------------------------------------------
+# reference arm: the oracle, timed step by step
+# ---------------------------------------------------------------------------
+def run_reference(args, wl):
+    ws, rank, _ = dist_info()
+    if rank != 0:
+        return 0
+    import oracle
+    from paper_2608_06628_gb300 import workloads as wk
+    orc = oracle.load()
+    cores = oracle.default_threads()
+    W, alpha = wk.params(wl)
+    W64, alpha64 = W.double().numpy(), alpha.double().numpy()
+    t_probe = oracle_sample_step(wl, orc, 1, "ref-probe", W64, alpha64)
+    total_budget = 120.0
+    n_sample = int(max(1, min(wl.n_req, total_budget / max(1, args.steps + args.warmup) / max(t_probe, 1e-6))))
+    for i in range(args.warmup):
+        oracle_sample_step(wl, orc, n_sample, ("ref-warm", i), W64, alpha64)
+    tot = 0.0
+    for i in range(args.steps):
+        tot += oracle_sample_step(wl, orc, n_sample, ("ref", i), W64, alpha64)
+    value = args.steps * n_sample * wl.B / tot
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": workload_config(wl, None),
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": f"each step: {n_sample} of {wl.n_req} requests, block attention + commit, "
+                                   f"fp64 C oracle on {cores} host threads"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(wl, l2_note):
+    cfg = {"workload": wl.name, "n_req": wl.n_req, "block_size": wl.B, "n_q_heads": wl.Hq,
+           "n_kv_heads": wl.Hkv, "head_dim": wl.d, "feat_dim": wl.F,
+           "prefix": (f"ragged U{{{wl.prefix_min}..{wl.prefix_max}}} step {wl.B}"
+                      if wl.prefix_min != wl.prefix_max else f"{wl.prefix_min}"),
+           "k_scale": wl.k_scale, "io_dtype": str(wl.io_dtype).replace("torch.", ""),
+           "state_dtype": "float32",
+           "step": "hybrid_block_attn + hybrid_commit_block (one denoising step, then its block commit)"}
+    if l2_note:
+        cfg["l2"] = l2_note
+    return cfg
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def run_hybrid(args, wl):
+    import torch
+    ws, rank, local = dist_info()
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device(f"cuda:{local}" if ws > 1 else "cuda:0")
+    torch.cuda.set_device(dev)
+
+    from paper_2608_06628_gb300 import build
+    build.build()
+    from paper_2608_06628_gb300 import hybrid as H
+    from paper_2608_06628_gb300 import workloads as wk
+    from paper_2608_06628_gb300.state_pool import StatePool
+
+    # each rank draws its own independent batch (weak scaling)
+    if ws > 1:
+        wl = wl.with_(seed=wl.seed + 1000 * rank)
+    cfg = H.make_cfg(wl.d, wl.F, wl.Hq, wl.Hkv, wl.B, wl.io_dtype)
+    W, alpha = wk.params(wl, device=dev)
+    io_bytes = 2 if wl.io_dtype == torch.bfloat16 else 4
+    ab = algorithmic_bytes(wl, io_bytes)
+    per_set = ab["q"] * 2 + ab["kv"] * 2 + ab["state"]
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    n_sets = max(2, math.ceil(4 * l2 / per_set) + 1)
+
+    # states of set 0: ragged prefixes built by block commits
+    plen = wk.prefix_lengths(wl)
+    pool0 = StatePool(cfg, wl.n_req, dev)
+    H.hybrid_state_init(cfg, pool0.all_ptrs(), wl.n_req)
+    for b in range(int(plen.max()) // wl.B):
+        reqs = np.nonzero(plen > b * wl.B)[0]
+        K, V = wk.prefix_kv(wl, b, dev, n_req=len(reqs))
+        H.hybrid_commit_block(cfg, K, V, wl.B, W, pool0.ptr_array(reqs.tolist()), len(reqs))
+    H.hybrid_check()
+    sets = []
+    for i in range(n_sets):
+        pool = pool0 if i == 0 else StatePool(cfg, wl.n_req, dev)
+        if i:
+            pool.slab.copy_(pool0.slab)
+        Q, K, V = wk.block_qkv(wl, ("bench", i), dev)
+        sets.append(dict(pool=pool, ptrs=pool.all_ptrs(), Q=Q, K=K, V=V, O=torch.empty_like(Q)))
+    torch.cuda.synchronize()
+
+    stream = torch.cuda.current_stream(dev)
+    sh = stream.cuda_stream
+
+    def step(s):
+        H.hybrid_block_attn(cfg, s["Q"], s["K"], s["V"], W, alpha, s["ptrs"], wl.n_req, s["O"], sh, check=False)
+        H.hybrid_commit_block(cfg, s["K"], s["V"], wl.B, W, s["ptrs"], wl.n_req, sh, check=False)
+
+    clocks = ClockSampler(bus_id_of(torch, dev))
+    clocks.start()
+    time.sleep(0.3)
+    for i in range(args.warmup):
+        step(sets[i % n_sets])
+    H.hybrid_check(sh)
+
+    # timed region: K steps, events around each kernel on the launching stream
+    K_ = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K_)]
+    barrier(ws)
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    for i in range(K_):
+        s = sets[i % n_sets]
+        ev[i][0].record(stream)
+        H.hybrid_block_attn(cfg, s["Q"], s["K"], s["V"], W, alpha, s["ptrs"], wl.n_req, s["O"], sh, check=False)
+        ev[i][1].record(stream)
+        H.hybrid_commit_block(cfg, s["K"], s["V"], wl.B, W, s["ptrs"], wl.n_req, sh, check=False)
+        ev[i][2].record(stream)
+    torch.cuda.synchronize()
+    barrier(ws)
+    t_wall1 = time.time()
+    status = H.hybrid_check(sh, check=False)
+    if status != H.HYBRID_OK:
+        raise SystemExit(f"device error during the timed region: {H.hybrid_status_str(status)}")
+    elapsed_ms = ev[0][0].elapsed_time(ev[K_ - 1][2])
+    attn_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / K_
+    commit_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / K_
+    elapsed_ms = max_over_ranks(elapsed_ms, ws, dev)
+
+    # end to end through the public API: pinned host inputs in, output back out
+    hQ = sets[0]["Q"].cpu().pin_memory()
+    hK = sets[0]["K"].cpu().pin_memory()
+    hV = sets[0]["V"].cpu().pin_memory()
+    hO = torch.empty_like(hQ).pin_memory()
+    e2e_sets = [dict(s, Q=torch.empty_like(s["Q"]), K=torch.empty_like(s["K"]), V=torch.empty_like(s["V"]))
+                for s in sets]
+    for i in range(args.warmup):
+        s = e2e_sets[i % n_sets]
+        s["Q"].copy_(hQ, non_blocking=True); s["K"].copy_(hK, non_blocking=True)
+        s["V"].copy_(hV, non_blocking=True)
+        step(s)
+        hO.copy_(s["O"], non_blocking=True)
+    barrier(ws)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(K_):
+        s = e2e_sets[i % n_sets]
+        s["Q"].copy_(hQ, non_blocking=True); s["K"].copy_(hK, non_blocking=True)
+        s["V"].copy_(hV, non_blocking=True)
+        step(s)
+        hO.copy_(s["O"], non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(ws)
+    clocks.stop()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), ws, dev)
+
+    if rank != 0:
+        return 0
+    tokens = wl.n_req * wl.B * K_ * ws
+    value = tokens / (elapsed_ms * 1e-3)
+    peaks, peak_kind = measured_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    dom = "attn" if attn_ms >= commit_ms else "commit"
+    dom_ms = attn_ms if dom == "attn" else commit_ms
+    kname = {"attn": "hybrid_block_attn", "commit": "hybrid_commit_block"}[dom]
+    achieved = ab[dom] / (dom_ms * 1e-3) / 1e9
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": K_,
+        "warmup": args.warmup, "ms_per_step": elapsed_ms / K_, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if wl.io_dtype == torch.bfloat16 else "f32",
+        "data": "synthetic (seeded N(0,1) activations, random-init W ~ N(0,1/d), alpha ~ U(0,1))",
+        "config": workload_config(wl, f"{n_sets} rotating buffer sets of {per_set / 1e6:.1f} MB "
+                                      f"(> 4x the {l2 / 1e6:.0f} MB L2)"),
+        "roofline": {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": hbm,
+                     "peak_kind": f"{peak_kind} (HBM copy, MEASURED_PEAKS hbm_gbs)" if peak_kind == "measured"
+                     else "fallback 6.8 TB/s", "unit": "GB/s", "frac": achieved / hbm,
+                     "traffic": recorded_traffic(kname, wl.name),
+                     "algorithmic_bytes_per_launch": ab[dom]},
+        "kernels": {
+            "hybrid_block_attn": {"us_per_launch": attn_ms * 1e3, "bytes": ab["attn"],
+                                  "GBps": ab["attn"] / (attn_ms * 1e-3) / 1e9,
+                                  "frac_hbm": ab["attn"] / (attn_ms * 1e-3) / 1e9 / hbm},
+            "hybrid_commit_block": {"us_per_launch": commit_ms * 1e3, "bytes": ab["commit"],
+                                    "GBps": ab["commit"] / (commit_ms * 1e-3) / 1e9,
+                                    "frac_hbm": ab["commit"] / (commit_ms * 1e-3) / 1e9 / hbm},
+        },
+        "e2e": {"value": tokens / (e2e_ms * 1e-3), "unit": "tokens/s",
+                "h2d_bytes_per_step": int(hQ.numel() * hQ.element_size() + 2 * hK.numel() * hK.element_size()),
+                "d2h_bytes_per_step": int(hO.numel() * hO.element_size())},
+        "gpu_launches": 2 * K_,
+        "clocks": clocks.summary(t_wall0, t_wall1),
+    }
+    if not args.no_cpu_baseline and ws == 1:
+        line["cpu_baseline"] = cpu_baseline(wl)
+    print(json.dumps(line), flush=True)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3000)
+    ap.add_argument("--warmup", type=int, default=30)
+    ap.add_argument("--impl", choices=("hybrid", "reference"), default="hybrid")
+    ap.add_argument("--config", default="c3_bf16_b64_gqa_ragged")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    from paper_2608_06628_gb300 import workloads as wk
+    wl = wk.CONFIGS[args.config]
+    if args.impl == "reference":
+        return run_reference(args, wl)
+    return run_hybrid(args, wl)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,162 @@
+/*
+ * hybrid.h -- C ABI of the block-hybrid attention library (sm_103a).
+ *
+ * Block-hybrid attention ("Retrofitting Linear Attention into Diffusion
+ * Language Models", Section 3.1): during blockwise semi-autoregressive
+ * decoding, each query of the active block of B tokens attends
+ *   (1) to every token of its own block with exact, unmasked softmax
+ *       (a_j = exp(q.k_j / sqrt(d)); sm_num = sum_j a_j v_j; sm_den = sum_j a_j), and
+ *   (2) to all committed blocks through a fixed-size linear-attention state
+ *       S = sum_t phi(k_t) v_t^T in R^{2F x d} and z = sum_t phi(k_t) in R^{2F}
+ *       (lin_num = phi(q)^T S, lin_den = phi(q)^T z),
+ * merged through a shared normaliser with the gate w = sigmoid(alpha):
+ *       out = (w sm_num + lin_num) / (w sm_den + lin_den).
+ * The feature map is Hedgehog's: phi(x) = [softmax(xW), softmax(-xW)],
+ * W in R^{d x F}.  When a block commits, its tokens are folded into (S, z).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * Notation: n = n_req requests, B = block size, Hq query heads, Hkv state
+ * (key/value) heads, G = Hq / Hkv, d = head_dim, F = feat_dim (phi has 2F
+ * entries).
+ *
+ * Ownership: the caller allocates every buffer (inputs, outputs, states and
+ * the device array of state pointers).  The library allocates no memory in
+ * any call; it keeps one 4-byte error word per device in its own static
+ * device memory, read back by hybrid_check().
+ *
+ * Pointers: every tensor argument is a DEVICE pointer unless stated.  Tensor
+ * pointers must be 16-byte aligned (alpha: 4-byte).  d_state_ptrs is a device
+ * array of n_req device pointers, one per request, each to a state buffer of
+ * hybrid_state_bytes(cfg) bytes, 16-byte aligned.  A batch may name any
+ * subset of live requests in any order (ragged concurrent batches); the same
+ * state must not appear twice in one commit call.
+ *
+ * Streams: every call is asynchronous and ordered on the given stream
+ * (a cudaStream_t; 0 is the legacy default stream).  The calling thread's
+ * current device must own all pointers.
+ *
+ * Layouts (row-major, innermost last):
+ *   Q, O        [n][B][Hq][d]     io_dtype
+ *   K, V        [n][T][Hkv][d]    io_dtype   (T = B in hybrid_block_attn)
+ *   W           [Hkv][d][F]       io_dtype   query head h uses W[h / G]
+ *   alpha       [Hq]              float32    w_h = sigmoid(alpha[h]); +-inf allowed
+ *   state       per request: Hkv head blocks of (2F*d + 2F) float32 each.
+ *               Within a head block, S is kept transposed (S^T, d rows of 2F
+ *               features) and cut into 2F/32 tiles of d rows x 32 features
+ *               (128 bytes per row).  Logical element S[f][e] lives at float
+ *               offset
+ *                   (f/32)*32*d + e*32 + 4*(((f%32)/4) ^ (e%8)) + f%4,
+ *               i.e. each 128-byte row is stored with its eight 16-byte
+ *               granules permuted by XOR with (e mod 8).  This is the byte
+ *               image that the tensor-core kernels consume directly (a
+ *               1024-byte-aligned linear copy of a tile is a valid 128-byte-
+ *               swizzled K-major operand), so a state is streamed from HBM
+ *               with plain bulk copies.  z[f] follows at float offset
+ *               2F*d + f.  hybrid_state_unpack / hybrid_state_pack convert
+ *               to and from the logical [Hkv][2F][d] / [Hkv][2F] layout.
+ *
+ * Supported sizes: head_dim d in {64, 128}; feat_dim F in {16, 32, 64, 128,
+ * 256}; 1 <= B <= 128; 1 <= Hkv <= Hq <= 256 with Hq % Hkv == 0; io_dtype
+ * float32 or bfloat16.  The state is always float32.  Arithmetic is float32
+ * throughout; with bfloat16 inputs the block-attention contractions run on
+ * the tensor cores (bf16 and tf32 operands, float32 accumulation).
+ *
+ * Errors: argument checks run synchronously on the host and return
+ * HYBRID_ERR_INVALID_ARG (null or misaligned pointer, inconsistent sizes) or
+ * HYBRID_ERR_UNSUPPORTED (a size outside the supported set).  A failed
+ * launch returns HYBRID_ERR_CUDA.  Problems found on the device (a null or
+ * misaligned state pointer in d_state_ptrs, a wait that gave up) never trap:
+ * the affected unit is skipped, a bit is set in the device error word, and
+ * hybrid_check() reports it.
+ */
+#ifndef HYBRID_H_
+#define HYBRID_H_
+
+#include <stddef.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    HYBRID_OK = 0,
+    HYBRID_ERR_INVALID_ARG = 1,
+    HYBRID_ERR_UNSUPPORTED = 2,
+    HYBRID_ERR_CUDA = 3,
+    HYBRID_ERR_TIMEOUT = 4,   /* a bounded device-side wait gave up */
+    HYBRID_ERR_DEVICE = 5     /* a device-side argument check failed */
+} hybrid_status;
+
+typedef enum { HYBRID_F32 = 0, HYBRID_BF16 = 1 } hybrid_dtype;
+
+typedef struct {
+    int head_dim;          /* d */
+    int feat_dim;          /* F: columns of W; phi(x) has 2F entries */
+    int n_q_heads;         /* Hq */
+    int n_kv_heads;        /* Hkv: state heads (GQA group G = Hq / Hkv) */
+    int block_size;        /* B: tokens of the active block */
+    hybrid_dtype io_dtype; /* dtype of Q, K, V, O, W */
+} hybrid_cfg;
+
+/* Bytes of one request's state: Hkv * (2F*d + 2F) * 4.  Returns 0 for an
+ * invalid or unsupported cfg.  Cf. Section 3.1 (S_n in R^{2F x d},
+ * Z_n in R^{2F}); the size is independent of the number of tokens absorbed. */
+size_t hybrid_state_bytes(const hybrid_cfg *cfg);
+
+/* Zero the states of n_req requests (an empty prefix: S_0 = 0, z_0 = 0). */
+hybrid_status hybrid_state_init(const hybrid_cfg *cfg, void *const *d_state_ptrs, int n_req,
+                                 cudaStream_t stream);
+
+/* Feature map of Section 3.1: Phi = [softmax(X W_g), softmax(-X W_g)].
+ *   X    [n_rows][n_heads_x][d] io_dtype (device); row head h uses
+ *        W[h / (n_heads_x / Hkv)], so n_heads_x must be a multiple of Hkv
+ *        (pass Hq for queries, Hkv for keys).
+ *   Phi  [n_rows][n_heads_x][2F] float32 (device, written).
+ * n_rows >= 0. */
+hybrid_status hybrid_feature_map(const hybrid_cfg *cfg, const void *X, int n_rows, int n_heads_x,
+                                 const void *W, float *Phi, cudaStream_t stream);
+
+/* One denoising step of block-hybrid attention over the active block of every
+ * request (Section 3.1: in-block softmax branch, linear readout from the
+ * committed state, gated shared-normaliser merge).
+ *   Q [n][B][Hq][d], K, V [n][B][Hkv][d], W [Hkv][d][F]: inputs (io_dtype)
+ *   alpha [Hq] float32
+ *   d_state_ptrs [n]: device array of state pointers; read, never written
+ *   O [n][B][Hq][d]: output (io_dtype); must not alias an input
+ * Query head h of request r reads state head h / G of request r. */
+hybrid_status hybrid_block_attn(const hybrid_cfg *cfg, const void *Q, const void *K, const void *V,
+                                const void *W, const float *alpha, void *const *d_state_ptrs,
+                                int n_req, void *O, cudaStream_t stream);
+
+/* Block commit of Section 3.1: S += sum_t phi(k_t) v_t^T, z += sum_t phi(k_t)
+ * over the n_tok tokens of K, V [n][n_tok][Hkv][d] (io_dtype), for every
+ * request and state head.  n_tok = B folds a decoded block; any n_tok >= 0
+ * folds a prompt (prefill).  The states are updated in place. */
+hybrid_status hybrid_commit_block(const hybrid_cfg *cfg, const void *K, const void *V, int n_tok,
+                                  const void *W, void *const *d_state_ptrs, int n_req,
+                                  cudaStream_t stream);
+
+/* Convert states to / from the logical layout (device buffers):
+ *   S_logical [n][Hkv][2F][d] float32 (S[f][e] as in Section 3.1)
+ *   z_logical [n][Hkv][2F]    float32 */
+hybrid_status hybrid_state_unpack(const hybrid_cfg *cfg, void *const *d_state_ptrs, int n_req,
+                                  float *S_logical, float *z_logical, cudaStream_t stream);
+hybrid_status hybrid_state_pack(const hybrid_cfg *cfg, const float *S_logical,
+                                const float *z_logical, void *const *d_state_ptrs, int n_req,
+                                cudaStream_t stream);
+
+/* Synchronise the stream, then read and clear this device's error word.
+ * Returns HYBRID_OK, HYBRID_ERR_DEVICE (a state pointer failed its device
+ * check), HYBRID_ERR_TIMEOUT (a bounded wait gave up) or HYBRID_ERR_CUDA. */
+hybrid_status hybrid_check(cudaStream_t stream);
+
+/* Static, human-readable name of a status code. */
+const char *hybrid_status_str(hybrid_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HYBRID_H_ */

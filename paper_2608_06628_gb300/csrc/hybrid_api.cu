@@ -1,0 +1,180 @@
+// hybrid_api.cu -- the extern "C" entry points declared in include/hybrid.h:
+// argument validation, kernel selection and launch, and the device error word.
+#include <mutex>
+
+#include "hybrid_common.cuh"
+#include "hybrid_kernels.h"
+#include "hybrid_tc.h"
+
+namespace {
+
+// One error word per device, in the library's own static device memory.
+__device__ unsigned g_error_word;
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+unsigned *g_err_ptr[kMaxDevices];
+
+// Device address of this device's error word, looked up once per device
+// (with that device current, as cudaGetSymbolAddress requires).
+unsigned *error_word()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (!g_err_ptr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
+        g_err_ptr[dev] = static_cast<unsigned *>(p);
+    }
+    return g_err_ptr[dev];
+}
+
+bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+hybrid_status check_cfg(const hybrid_cfg *c)
+{
+    if (!c) return HYBRID_ERR_INVALID_ARG;
+    if (c->io_dtype != HYBRID_F32 && c->io_dtype != HYBRID_BF16) return HYBRID_ERR_UNSUPPORTED;
+    if (c->head_dim != 64 && c->head_dim != 128) return HYBRID_ERR_UNSUPPORTED;
+    const int F = c->feat_dim;
+    if (F != 16 && F != 32 && F != 64 && F != 128 && F != 256) return HYBRID_ERR_UNSUPPORTED;
+    if (c->block_size < 1 || c->block_size > 128) return HYBRID_ERR_UNSUPPORTED;
+    if (c->n_kv_heads < 1 || c->n_q_heads < 1 || c->n_q_heads > 256) return HYBRID_ERR_UNSUPPORTED;
+    if (c->n_kv_heads > c->n_q_heads || c->n_q_heads % c->n_kv_heads != 0) return HYBRID_ERR_INVALID_ARG;
+    return HYBRID_OK;
+}
+
+hybrid_status from_cuda(cudaError_t e) { return e == cudaSuccess ? HYBRID_OK : HYBRID_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+size_t hybrid_state_bytes(const hybrid_cfg *cfg)
+{
+    if (check_cfg(cfg) != HYBRID_OK) return 0;
+    return (size_t)cfg->n_kv_heads * hyb::head_floats(cfg->head_dim, cfg->feat_dim) * sizeof(float);
+}
+
+hybrid_status hybrid_state_init(const hybrid_cfg *cfg, void *const *d_state_ptrs, int n_req,
+                                cudaStream_t stream)
+{
+    hybrid_status s = check_cfg(cfg);
+    if (s != HYBRID_OK) return s;
+    if (n_req < 0) return HYBRID_ERR_INVALID_ARG;
+    if (n_req == 0) return HYBRID_OK;
+    if (!d_state_ptrs || !aligned(d_state_ptrs, 8)) return HYBRID_ERR_INVALID_ARG;
+    return from_cuda(hyb::launch_state_init(*cfg, d_state_ptrs, n_req, stream));
+}
+
+hybrid_status hybrid_feature_map(const hybrid_cfg *cfg, const void *X, int n_rows, int n_heads_x,
+                                 const void *W, float *Phi, cudaStream_t stream)
+{
+    hybrid_status s = check_cfg(cfg);
+    if (s != HYBRID_OK) return s;
+    if (n_rows < 0 || n_heads_x < 1 || n_heads_x % cfg->n_kv_heads != 0) return HYBRID_ERR_INVALID_ARG;
+    if (n_rows == 0) return HYBRID_OK;
+    if (!X || !W || !Phi || !aligned(X, 16) || !aligned(W, 16) || !aligned(Phi, 16))
+        return HYBRID_ERR_INVALID_ARG;
+    return from_cuda(hyb::launch_feature_map(cfg->io_dtype, X, n_rows, n_heads_x, cfg->n_kv_heads,
+                                             cfg->head_dim, cfg->feat_dim, W, Phi, stream));
+}
+
+hybrid_status hybrid_block_attn(const hybrid_cfg *cfg, const void *Q, const void *K, const void *V,
+                                const void *W, const float *alpha, void *const *d_state_ptrs,
+                                int n_req, void *O, cudaStream_t stream)
+{
+    hybrid_status s = check_cfg(cfg);
+    if (s != HYBRID_OK) return s;
+    if (n_req < 0) return HYBRID_ERR_INVALID_ARG;
+    if (n_req == 0) return HYBRID_OK;
+    if (!Q || !K || !V || !W || !alpha || !d_state_ptrs || !O) return HYBRID_ERR_INVALID_ARG;
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(W, 16) || !aligned(O, 16) ||
+        !aligned(alpha, 4) || !aligned(d_state_ptrs, 8))
+        return HYBRID_ERR_INVALID_ARG;
+    unsigned *err = error_word();
+    if (!err) return HYBRID_ERR_CUDA;
+    if (hyb::tc_attn_supported(*cfg))
+        return from_cuda(hyb::launch_attn_tc(*cfg, Q, K, V, W, alpha, d_state_ptrs, n_req, O, err, stream));
+    return from_cuda(hyb::launch_attn_generic(*cfg, Q, K, V, W, alpha, d_state_ptrs, n_req, O, err, stream));
+}
+
+hybrid_status hybrid_commit_block(const hybrid_cfg *cfg, const void *K, const void *V, int n_tok,
+                                  const void *W, void *const *d_state_ptrs, int n_req,
+                                  cudaStream_t stream)
+{
+    hybrid_status s = check_cfg(cfg);
+    if (s != HYBRID_OK) return s;
+    if (n_req < 0 || n_tok < 0) return HYBRID_ERR_INVALID_ARG;
+    if (n_req == 0 || n_tok == 0) return HYBRID_OK;
+    if (!K || !V || !W || !d_state_ptrs) return HYBRID_ERR_INVALID_ARG;
+    if (!aligned(K, 16) || !aligned(V, 16) || !aligned(W, 16) || !aligned(d_state_ptrs, 8))
+        return HYBRID_ERR_INVALID_ARG;
+    unsigned *err = error_word();
+    if (!err) return HYBRID_ERR_CUDA;
+    return from_cuda(hyb::launch_commit_generic(*cfg, K, V, n_tok, W, d_state_ptrs, n_req, err, stream));
+}
+
+hybrid_status hybrid_state_unpack(const hybrid_cfg *cfg, void *const *d_state_ptrs, int n_req,
+                                  float *S_logical, float *z_logical, cudaStream_t stream)
+{
+    hybrid_status s = check_cfg(cfg);
+    if (s != HYBRID_OK) return s;
+    if (n_req < 0) return HYBRID_ERR_INVALID_ARG;
+    if (n_req == 0) return HYBRID_OK;
+    if (!d_state_ptrs || !S_logical || !z_logical || !aligned(d_state_ptrs, 8) ||
+        !aligned(S_logical, 4) || !aligned(z_logical, 4))
+        return HYBRID_ERR_INVALID_ARG;
+    unsigned *err = error_word();
+    if (!err) return HYBRID_ERR_CUDA;
+    return from_cuda(hyb::launch_state_unpack(*cfg, d_state_ptrs, n_req, S_logical, z_logical, err, stream));
+}
+
+hybrid_status hybrid_state_pack(const hybrid_cfg *cfg, const float *S_logical,
+                                const float *z_logical, void *const *d_state_ptrs, int n_req,
+                                cudaStream_t stream)
+{
+    hybrid_status s = check_cfg(cfg);
+    if (s != HYBRID_OK) return s;
+    if (n_req < 0) return HYBRID_ERR_INVALID_ARG;
+    if (n_req == 0) return HYBRID_OK;
+    if (!d_state_ptrs || !S_logical || !z_logical || !aligned(d_state_ptrs, 8) ||
+        !aligned(S_logical, 4) || !aligned(z_logical, 4))
+        return HYBRID_ERR_INVALID_ARG;
+    unsigned *err = error_word();
+    if (!err) return HYBRID_ERR_CUDA;
+    return from_cuda(hyb::launch_state_pack(*cfg, S_logical, z_logical, d_state_ptrs, n_req, err, stream));
+}
+
+hybrid_status hybrid_check(cudaStream_t stream)
+{
+    unsigned *err = error_word();
+    if (!err) return HYBRID_ERR_CUDA;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return HYBRID_ERR_CUDA;
+    unsigned word = 0;
+    if (cudaMemcpy(&word, err, sizeof word, cudaMemcpyDeviceToHost) != cudaSuccess) return HYBRID_ERR_CUDA;
+    if (word != 0) {
+        const unsigned zero = 0;
+        if (cudaMemcpy(err, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess)
+            return HYBRID_ERR_CUDA;
+    }
+    if (word & hyb::ERR_WAIT_TIMEOUT) return HYBRID_ERR_TIMEOUT;
+    if (word & hyb::ERR_BAD_STATE_PTR) return HYBRID_ERR_DEVICE;
+    return HYBRID_OK;
+}
+
+const char *hybrid_status_str(hybrid_status status)
+{
+    switch (status) {
+    case HYBRID_OK: return "HYBRID_OK";
+    case HYBRID_ERR_INVALID_ARG: return "HYBRID_ERR_INVALID_ARG: invalid argument";
+    case HYBRID_ERR_UNSUPPORTED: return "HYBRID_ERR_UNSUPPORTED: size or dtype outside the supported set";
+    case HYBRID_ERR_CUDA: return "HYBRID_ERR_CUDA: CUDA runtime error";
+    case HYBRID_ERR_TIMEOUT: return "HYBRID_ERR_TIMEOUT: a bounded device wait gave up";
+    case HYBRID_ERR_DEVICE: return "HYBRID_ERR_DEVICE: a device-side argument check failed";
+    }
+    return "HYBRID_ERR_UNKNOWN";
+}
+
+}  // extern "C"

@@ -1,0 +1,273 @@
+"""CUDA path vs the fp64 oracle, element by element, through the C ABI.
+
+Sizes span several tiles and ragged tails while the oracle still finishes in
+seconds.  Tolerances (written in gpu_harness.TOL): fp32 I/O rel-L2 <= 1e-5 and
+max-abs <= 1e-4; bf16 I/O with fp32 state rel-L2 <= 1e-2, for outputs and for
+committed states alike.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from gpu_harness import Pair, assert_parity, h64, rel_l2
+from paper_2608_06628_gb300 import hybrid as H
+from paper_2608_06628_gb300 import workloads as wk
+from paper_2608_06628_gb300.state_pool import StatePool
+
+pytestmark = pytest.mark.gpu
+
+BF16, F32 = torch.bfloat16, torch.float32
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _device():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_06628_gb300 import build
+    build.build()
+    torch.cuda.set_device(0)
+
+
+def W_(name, dt, n, Hq, Hkv, d, F, B, seed, pmin=0, pmax=0, k_scale=1.0):
+    return wk.Workload(name, dt, n, Hq, Hkv, d, F, B, seed, pmin, pmax, k_scale)
+
+
+# small cases: (workload, explicit ragged prefix lengths)
+SMALL = [
+    (wk.C1, None),
+    (W_("mha_bf16", BF16, 3, 4, 4, 128, 128, 32, 11), [64, 0, 96]),
+    (W_("gqa4_bf16", BF16, 5, 8, 2, 128, 128, 32, 12), [0, 32, 96, 160, 256]),
+    (W_("f256_b64_k8_bf16", BF16, 3, 2, 2, 128, 256, 64, 13, k_scale=8.0), [0, 128, 384]),
+    (W_("d64_f64_bf16", BF16, 4, 4, 2, 64, 64, 32, 14), [32, 64, 0, 128]),
+    (W_("d64_f16_b16_f32", F32, 3, 2, 1, 64, 16, 16, 15), [16, 48, 0]),
+    (W_("f32_b48_ragged_rows", F32, 2, 3, 3, 128, 32, 48, 16), [96, 48]),
+    (W_("bf16_b48_f32feat", BF16, 2, 4, 4, 128, 32, 48, 17), [48, 144]),
+    (W_("bf16_g8_b32_generic", BF16, 2, 8, 1, 128, 64, 32, 18), [64, 32]),
+    (W_("bf16_b16_g2", BF16, 3, 4, 2, 128, 128, 16, 19), [16, 0, 80]),
+    (W_("bf16_b64_g2", BF16, 2, 4, 2, 64, 128, 64, 20), [128, 64]),
+    (W_("f32_mha_f128", F32, 2, 2, 2, 128, 128, 32, 21), [64, 32]),
+]
+
+
+def _plen(wl, plen):
+    return wk.prefix_lengths(wl) if plen is None else np.asarray(plen, dtype=np.int64)
+
+
+@pytest.mark.parametrize("wl,plen", SMALL, ids=[w.name for w, _ in SMALL])
+def test_commit_then_step_parity(wl, plen):
+    pair = Pair(wl)
+    plen = _plen(wl, plen)
+    pair.build_prefixes(plen)
+    S, z = pair.gpu_state()
+    assert_parity(S, pair.S, wl.io_dtype, "prefix state S")
+    assert_parity(z, pair.z, wl.io_dtype, "prefix state z")
+    Q, K, V = wk.block_qkv(wl, "step", pair.dev)
+    got, want, _ = pair.step(Q, K, V)
+    assert_parity(got, want, wl.io_dtype, "block attention output")
+    # fold the active block in (the final denoising step's K/V) and compare the state
+    pair.commit(K, V)
+    S, z = pair.gpu_state()
+    assert_parity(S, pair.S, wl.io_dtype, "post-commit state S")
+    assert_parity(z, pair.z, wl.io_dtype, "post-commit state z")
+    # a second step against the grown state
+    Q2, K2, V2 = wk.block_qkv(wl, "step2", pair.dev)
+    got, want, _ = pair.step(Q2, K2, V2)
+    assert_parity(got, want, wl.io_dtype, "second step output")
+
+
+@pytest.mark.parametrize("dt", [F32, BF16])
+@pytest.mark.parametrize("d,F,nh,Hkv", [(64, 16, 2, 1), (128, 128, 16, 4), (128, 256, 3, 3), (64, 64, 4, 4)])
+def test_feature_map_parity(dt, d, F, nh, Hkv):
+    import oracle
+    g = torch.Generator(device="cuda").manual_seed(d * 1000 + F + nh)
+    n_rows = 37
+    X = (torch.randn((n_rows, nh, d), generator=g, device="cuda") * 1.5).to(dt)
+    W = (torch.randn((Hkv, d, F), generator=g, device="cuda") / math.sqrt(d)).to(dt)
+    cfg = H.make_cfg(d, F, nh, Hkv, 32, dt)
+    Phi = torch.empty((n_rows, nh, 2 * F), dtype=torch.float32, device="cuda")
+    H.hybrid_feature_map(cfg, X, n_rows, nh, W, Phi)
+    H.hybrid_check()
+    want = oracle.load().feature_map(h64(X), h64(W))
+    # phi is computed and returned in float32 from exactly representable inputs
+    assert_parity(h64(Phi), want, F32, "phi")
+
+
+def test_state_layout_matches_header_formula():
+    """pack/unpack round trip is exact, and the raw bytes follow the documented
+    offset formula (f/32)*32*d + e*32 + 4*(((f%32)/4) ^ (e%8)) + f%4, z at 2F*d + f."""
+    d, F, Hkv = 64, 32, 2
+    cfg = H.make_cfg(d, F, 2, Hkv, 16, F32)
+    pool = StatePool(cfg, 3, "cuda")
+    ptrs = pool.all_ptrs()
+    g = torch.Generator(device="cuda").manual_seed(5)
+    S = torch.randn((3, Hkv, 2 * F, d), generator=g, device="cuda")
+    z = torch.randn((3, Hkv, 2 * F), generator=g, device="cuda")
+    H.hybrid_state_pack(cfg, S, z, ptrs, 3)
+    S2, z2 = torch.empty_like(S), torch.empty_like(z)
+    H.hybrid_state_unpack(cfg, ptrs, 3, S2, z2)
+    H.hybrid_check()
+    assert torch.equal(S, S2) and torch.equal(z, z2)
+    raw = pool.slab.view(3, Hkv, -1).cpu().numpy()
+    Sh, zh = S.cpu().numpy(), z.cpu().numpy()
+    f = np.arange(2 * F)[:, None]
+    e = np.arange(d)[None, :]
+    off = (f // 32) * 32 * d + e * 32 + 4 * (((f % 32) // 4) ^ (e % 8)) + f % 4
+    for r in range(3):
+        for h in range(Hkv):
+            assert np.array_equal(raw[r, h][off], Sh[r, h])
+            assert np.array_equal(raw[r, h][2 * F * d + np.arange(2 * F)], zh[r, h])
+
+
+def test_state_init_zeroes():
+    cfg = H.make_cfg(128, 128, 16, 4, 32, BF16)
+    pool = StatePool(cfg, 4, "cuda")
+    pool.slab.fill_(7.0)
+    H.hybrid_state_init(cfg, pool.ptr_array([0, 2]), 2)
+    H.hybrid_check()
+    n = pool.slot_bytes // 4
+    assert torch.count_nonzero(pool.slab[:n]) == 0
+    assert torch.all(pool.slab[n:2 * n] == 7.0)
+    assert torch.count_nonzero(pool.slab[2 * n:3 * n]) == 0
+
+
+# ---------------------------------------------------------------------------
+# edge cases
+# ---------------------------------------------------------------------------
+EDGE_WL = [W_("edge_gqa_bf16", BF16, 3, 8, 2, 128, 128, 32, 31),
+           W_("edge_f32", F32, 2, 2, 2, 64, 64, 16, 32)]
+
+
+@pytest.mark.parametrize("wl", EDGE_WL, ids=[w.name for w in EDGE_WL])
+def test_gate_limits(wl):
+    pair = Pair(wl)
+    pair.build_prefixes(np.full(wl.n_req, 2 * wl.B))
+    Q, K, V = wk.block_qkv(wl, "gate", pair.dev)
+    for a in (math.inf, -math.inf, 30.0, -30.0, 0.0):
+        alpha = torch.full((wl.Hq,), a, dtype=torch.float32, device=pair.dev)
+        got, want, _ = pair.step(Q, K, V, alpha)
+        assert_parity(got, want, wl.io_dtype, f"alpha={a}")
+
+
+@pytest.mark.parametrize("wl", EDGE_WL, ids=[w.name for w in EDGE_WL])
+def test_empty_prefix_is_block_softmax(wl):
+    pair = Pair(wl)
+    Q, K, V = wk.block_qkv(wl, "empty", pair.dev)
+    got, want, O = pair.step(Q, K, V)
+    assert_parity(got, want, wl.io_dtype, "empty prefix")
+    G = wl.Hq // wl.Hkv
+    q = Q.float().permute(0, 2, 1, 3)
+    k = K.float().repeat_interleave(G, dim=2).permute(0, 2, 1, 3)
+    v = V.float().repeat_interleave(G, dim=2).permute(0, 2, 1, 3)
+    ref = torch.nn.functional.scaled_dot_product_attention(q, k, v).permute(0, 2, 1, 3)
+    assert rel_l2(h64(O), h64(ref)) <= (1e-5 if wl.io_dtype == F32 else 1e-2)
+
+
+@pytest.mark.parametrize("wl", EDGE_WL, ids=[w.name for w in EDGE_WL])
+def test_values_one_give_one(wl):
+    pair = Pair(wl)
+    reqs = np.arange(wl.n_req)
+    for b in range(3):
+        K, _ = wk.prefix_kv(wl, b, pair.dev)
+        pair.commit(K, torch.ones_like(K), reqs)
+    Q, K, _ = wk.block_qkv(wl, "ones", pair.dev)
+    got, want, O = pair.step(Q, K, torch.ones_like(K))
+    assert np.max(np.abs(h64(O) - 1.0)) <= (1e-5 if wl.io_dtype == F32 else 4e-3)
+
+
+@pytest.mark.parametrize("wl", EDGE_WL, ids=[w.name for w in EDGE_WL])
+def test_tied_keys(wl):
+    """All keys equal: the in-block softmax is uniform (every score ties)."""
+    pair = Pair(wl)
+    pair.build_prefixes(np.full(wl.n_req, wl.B))
+    Q, K, V = wk.block_qkv(wl, "ties", pair.dev)
+    K = K[:, :1].expand_as(K).contiguous()
+    got, want, _ = pair.step(Q, K, V)
+    assert_parity(got, want, wl.io_dtype, "tied keys")
+
+
+def test_permuted_and_subset_pointer_arrays():
+    """A batch may list any subset of states in any order: the output of a
+    request depends only on its own state pointer."""
+    wl = W_("perm_bf16", BF16, 6, 8, 2, 128, 128, 32, 41)
+    pair = Pair(wl)
+    pair.build_prefixes(np.array([32, 64, 96, 128, 160, 192]))
+    Q, K, V = wk.block_qkv(wl, "perm", pair.dev)
+    O = torch.empty_like(Q)
+    H.hybrid_block_attn(pair.cfg, Q, K, V, pair.W, pair.alpha, pair.ptrs, wl.n_req, O)
+    order = [4, 1, 5]
+    idx = torch.as_tensor(order, device=pair.dev)
+    O2 = torch.empty_like(Q[idx])
+    H.hybrid_block_attn(pair.cfg, Q[idx].contiguous(), K[idx].contiguous(), V[idx].contiguous(),
+                        pair.W, pair.alpha, pair.pool.ptr_array(order), len(order), O2)
+    H.hybrid_check()
+    assert torch.equal(O[idx], O2)
+
+
+def test_deterministic():
+    wl = W_("det_bf16", BF16, 4, 16, 4, 128, 128, 32, 42)
+    pair = Pair(wl)
+    pair.build_prefixes(np.array([64, 32, 0, 96]))
+    Q, K, V = wk.block_qkv(wl, "det", pair.dev)
+    O1, O2 = torch.empty_like(Q), torch.empty_like(Q)
+    H.hybrid_block_attn(pair.cfg, Q, K, V, pair.W, pair.alpha, pair.ptrs, wl.n_req, O1)
+    H.hybrid_block_attn(pair.cfg, Q, K, V, pair.W, pair.alpha, pair.ptrs, wl.n_req, O2)
+    H.hybrid_check()
+    assert torch.equal(O1, O2)
+    # commits are deterministic too: two pools, same commits, identical bytes
+    pair2 = Pair(wl)
+    pair2.build_prefixes(np.array([64, 32, 0, 96]))
+    torch.cuda.synchronize()
+    assert torch.equal(pair.pool.slab, pair2.pool.slab)
+
+
+def test_state_copy_out_and_back_resumes():
+    """The state is the resumable object: copying a state's bytes out and back
+    (e.g. to host memory) gives identical subsequent outputs."""
+    wl = W_("resume_bf16", BF16, 2, 4, 4, 128, 128, 32, 43)
+    pair = Pair(wl)
+    pair.build_prefixes(np.array([96, 64]))
+    saved = pair.pool.slab.cpu().clone()
+    Q, K, V = wk.block_qkv(wl, "resume", pair.dev)
+    O1 = torch.empty_like(Q)
+    H.hybrid_block_attn(pair.cfg, Q, K, V, pair.W, pair.alpha, pair.ptrs, wl.n_req, O1)
+    pair.pool.slab.fill_(0.0)
+    pair.pool.slab.copy_(saved.to(pair.dev))
+    O2 = torch.empty_like(Q)
+    H.hybrid_block_attn(pair.cfg, Q, K, V, pair.W, pair.alpha, pair.ptrs, wl.n_req, O2)
+    H.hybrid_check()
+    assert torch.equal(O1, O2)
+
+
+def test_bad_state_pointer_is_reported_not_faulted():
+    """A null or misaligned entry in d_state_ptrs is skipped on the device and
+    reported by hybrid_check; the context stays usable."""
+    wl = W_("badptr_bf16", BF16, 3, 4, 4, 128, 128, 32, 44)
+    pair = Pair(wl)
+    Q, K, V = wk.block_qkv(wl, "bad", pair.dev)
+    good = pair.pool.ptr_array([0, 1, 2])
+    for bad_value in (0, pair.pool.slot_ptr(1) + 4):
+        ptrs = good.clone()
+        ptrs[1] = bad_value
+        O = torch.zeros_like(Q)
+        H.hybrid_block_attn(pair.cfg, Q, K, V, pair.W, pair.alpha, ptrs, 3, O)
+        assert H.hybrid_check(check=False) == H.HYBRID_ERR_DEVICE
+        H.hybrid_commit_block(pair.cfg, K, V, wl.B, pair.W, ptrs, 3)
+        assert H.hybrid_check(check=False) == H.HYBRID_ERR_DEVICE
+    # the error word was cleared and the device still works
+    O = torch.empty_like(Q)
+    H.hybrid_block_attn(pair.cfg, Q, K, V, pair.W, pair.alpha, good, 3, O)
+    assert H.hybrid_check(check=False) == H.HYBRID_OK
+
+
+def test_prefill_commit_long_ragged():
+    """Prompt prefill: commits of many tokens (T not a multiple of 32) in one call
+    equal the same tokens committed in B-sized pieces."""
+    wl = W_("prefill_bf16", BF16, 3, 4, 2, 128, 64, 32, 45)
+    pair = Pair(wl)
+    K, V = wk.prefix_kv(wl, 0, pair.dev, n_tok=161)
+    pair.commit(K, V)
+    S, z = pair.gpu_state()
+    assert_parity(S, pair.S, BF16, "prefill S")
+    assert_parity(z, pair.z, BF16, "prefill z")
