@@ -1,15 +1,448 @@
-// hybrid_tc.cu -- tensor-core (tcgen05) block-attention kernel.
+// hybrid_tc.cu -- block-hybrid attention on the 5th-generation tensor cores.
+//
+// One CTA per (request r, state head g).  Its M = G*B query rows (the G query
+// heads of the group times the B tokens of the active block, padded to 128)
+// share the state (S_g, z_g) of Section 3.1 of "Retrofitting Linear Attention
+// into Diffusion Language Models", so the state is streamed from HBM once per
+// group.  Contractions (tcgen05.mma, accumulators in Tensor Memory):
+//   U      = Q W_g              bf16 x bf16 -> f32   (feature-map projection)
+//   scores = Q K^T              bf16 x bf16 -> f32   (in-block softmax logits)
+//   D_lin  = phi(Q) S_g         tf32 x tf32 -> f32   (linear readout; phi(Q) in TMEM)
+//   D_s    = P V                bf16 x bf16 -> f32   (softmax numerator)
+// Per-row work (one thread per TMEM lane/row, two threads per row splitting
+// the columns): phi = [softmax(U), softmax(-U)], lin_den = phi . z_g, the
+// in-block softmax statistics, and the gated shared-normaliser merge.
+//
+// The state arrives by 1-D bulk copies: its HBM layout (hybrid.h) is already
+// the 128-byte-swizzled K-major operand image, so each 32-feature tile is one
+// copy straight into an MMA-ready buffer.  Q, K, V and W are gathered with
+// 16-byte cp.async into their swizzled operand layouts.
 #include "hybrid_common.cuh"
 #include "hybrid_tc.h"
+#include "tc_ptx.cuh"
 
 namespace hyb {
 
-bool tc_attn_supported(const hybrid_cfg &) { return false; }
+namespace {
 
-cudaError_t launch_attn_tc(const hybrid_cfg &, const void *, const void *, const void *, const void *,
-                           const float *, void *const *, int, void *, unsigned *, cudaStream_t)
+constexpr int kThreads = 256;
+constexpr uint32_t kColA = 0;     // U, then phi = [phi+, phi-]  (2F <= 256 columns)
+constexpr uint32_t kColD = 256;   // D_lin (d columns)
+constexpr uint32_t kColS = 384;   // scores (B columns), then D_s (d columns)
+constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s per bounded wait
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr int kSmemLimit = 232448;            // 227 KB opt-in per CTA
+constexpr int kOneCtaPerSm = 118 * 1024;      // request at least this much: 1 CTA / SM (TMEM 512 cols)
+
+struct TcAttnArgs {
+    const __nv_bfloat16 *Q, *K, *V, *W;
+    const float *alpha;
+    void *const *states;
+    __nv_bfloat16 *O;
+    unsigned *err;
+    int B, Hq, Hkv, G, d, F;
+    int n_slots;
+    float scale_log2;   // log2(e) / sqrt(d)
+    float inv_sqrt_d;
+    uint32_t off_q, off_w, off_k, off_v, off_p, off_z, off_bar;
+};
+
+struct Layout {
+    uint32_t off_q, off_w, off_k, off_v, off_p, off_z, off_bar, bytes;
+    int n_slots;
+};
+
+Layout make_layout(int d, int F, int B)
 {
-    return cudaErrorNotSupported;
+    Layout L{};
+    const uint32_t chunk = (uint32_t)d * 128;
+    const int NC = 2 * F / 32;
+    const uint32_t q = (uint32_t)d * 256, w = (uint32_t)d * F * 2, k = (uint32_t)B * d * 2,
+                   v = (uint32_t)B * d * 2, p = 128u * B * 2, z = ((uint32_t)2 * F * 4 + 1023) & ~1023u;
+    const uint32_t fixed = q + w + k + v + p + z + 1024 /*barriers*/ + 1024 /*alignment slack*/;
+    int slots = (int)((kSmemLimit - (int)fixed) / (int)chunk);
+    if (slots > NC) slots = NC;
+    L.n_slots = slots;
+    uint32_t off = (uint32_t)slots * chunk;
+    L.off_q = off; off += q;
+    L.off_w = off; off += w;
+    L.off_k = off; off += k;
+    L.off_v = off; off += v;
+    L.off_p = off; off += p;
+    L.off_z = off; off += z;
+    L.off_bar = off; off += 1024;
+    L.bytes = off + 1024;
+    if ((int)L.bytes < kOneCtaPerSm) L.bytes = kOneCtaPerSm;
+    return L;
+}
+
+__device__ __forceinline__ float tf32_round(float x)
+{
+    uint32_t r;
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+    return __uint_as_float(r);
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b)
+{
+    const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+__global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__ TcAttnArgs a)
+{
+    using namespace ptx;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int r = blockIdx.x / a.Hkv, g = blockIdx.x % a.Hkv;
+    const int d = a.d, F = a.F, B = a.B, G = a.G;
+    const int NC = (2 * F) / 32;
+    const int Mv = G * B;
+    const uint32_t chunk_bytes = (uint32_t)d * 128;
+
+    const float *state = reinterpret_cast<const float *>(a.states[r]);
+    if (!state_ptr_ok(state)) {
+        if (tid == 0) raise_error(a.err, ERR_BAD_STATE_PTR);
+        return;
+    }
+    const float *Sg = state + (size_t)g * head_floats(d, F);
+    const float *zg = Sg + (size_t)2 * F * d;
+
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + a.off_bar);
+    uint64_t *full = bars;
+    uint64_t *empty = bars + a.n_slots;
+    uint64_t *bar_z = bars + 2 * a.n_slots;
+    uint64_t *bar_u = bar_z + 1;
+    uint64_t *bar_d = bar_z + 2;
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_z + 3);
+    int *fail = reinterpret_cast<int *>(tmem_holder + 1);
+    int *issued = fail + 1;   // S chunks issued so far (for draining after a failure)
+
+    if (tid == 0) {
+        for (int i = 0; i < 2 * a.n_slots + 3; ++i) mbar_init(&bars[i], 1);
+        *fail = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(tmem_holder, 512);
+        tmem_relinquish();
+    }
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_holder;
+
+    // ---- producer: z and the first S tiles (bulk copies of the state image)
+    if (tid == 0) {
+        mbar_arrive_expect_tx(bar_z, 2 * F * 4);
+        bulk_g2s(smem + a.off_z, zg, 2 * F * 4, bar_z);
+        const int pre = NC < a.n_slots ? NC : a.n_slots;
+        for (int c = 0; c < pre; ++c) {
+            mbar_arrive_expect_tx(&full[c], chunk_bytes);
+            bulk_g2s(smem + (size_t)c * chunk_bytes, Sg + (size_t)c * 32 * d, chunk_bytes, &full[c]);
+        }
+        *issued = pre;
+    }
+    // ---- Q, K, V, W into their operand layouts (16-byte cp.async)
+    {
+        const int gpr = d / 8;
+        for (int idx = tid; idx < Mv * gpr; idx += kThreads) {
+            const int i = idx / gpr, c = idx % gpr;
+            const int t = i / G, hh = i % G;
+            const __nv_bfloat16 *src = a.Q + (((size_t)r * B + t) * a.Hq + g * G + hh) * d + 8 * c;
+            cp_async16(smem + a.off_q + (c >> 3) * (128 * 128) + i * 128 + (((c & 7) ^ (i & 7)) << 4), src);
+        }
+        for (int idx = tid; idx < B * gpr; idx += kThreads) {
+            const int j = idx / gpr, c = idx % gpr;
+            const size_t so = (((size_t)r * B + j) * a.Hkv + g) * d + 8 * c;
+            cp_async16(smem + a.off_k + (c >> 3) * (B * 128) + j * 128 + (((c & 7) ^ (j & 7)) << 4), a.K + so);
+            cp_async16(smem + a.off_v + (j >> 3) * ((d / 64) * 1024) + (c >> 3) * 1024 + (j & 7) * 128 +
+                           (((c & 7) ^ (j & 7)) << 4),
+                       a.V + so);
+        }
+        const int gw = F / 8;
+        for (int idx = tid; idx < d * gw; idx += kThreads) {
+            const int e = idx / gw, c = idx % gw;
+            cp_async16(smem + a.off_w + (e >> 3) * ((F / 64) * 1024) + (c >> 3) * 1024 + (e & 7) * 128 +
+                           (((c & 7) ^ (e & 7)) << 4),
+                       a.W + ((size_t)g * d + e) * F + 8 * c);
+        }
+    }
+    cp_async_wait_all();
+    fence_proxy_async_smem();
+    __syncthreads();
+
+    // ---- U = Q W_g and scores = Q K^T
+    if (tid == 0) {
+        tc_fence_after();
+        const uint32_t q_u = smem_u32(smem + a.off_q), w_u = smem_u32(smem + a.off_w),
+                       k_u = smem_u32(smem + a.off_k);
+        const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
+        const uint32_t idS = instr_desc(FMT_BF16, FMT_BF16, false, false, 128, B);
+        for (int k = 0; k < d / 16; ++k) {
+            const uint64_t ad = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
+            const uint64_t bw = smem_desc(w_u + 2 * k * ((F / 64) * 1024), 1024, (F / 64) * 1024, SWZ_128B);
+            const uint64_t bk = smem_desc(k_u + (k >> 2) * (B * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
+            mma_bf16_ss(tmem + kColA, ad, bw, idU, k > 0);
+            mma_bf16_ss(tmem + kColS, ad, bk, idS, k > 0);
+        }
+        mma_commit(bar_u);
+    }
+    if (!mbar_wait(bar_u, 0, kWaitNs)) atomicOr(fail, 1);
+    tc_fence_after();
+
+    // Q is no longer read by the tensor cores: its buffer holds the row statistics.
+    float *stat = reinterpret_cast<float *>(smem + a.off_q);   // [3][128] m, l, lin_den
+    float *ex = stat + 3 * 128;                                 // [8][2][128] exchange
+    const int q4 = warp & 3, half = warp >> 2;
+    const int row = 32 * q4 + lane;
+    const uint32_t lane_off = (uint32_t)(32 * q4) << 16;
+    const bool valid = row < Mv;
+    const int nsc = B / 16;       // 16-column chunks of scores; chunk k -> half k % 2
+    const int nfc = F / 32;       // 32-column chunks of U;      chunk k -> half k % 2
+
+    // ---- round 1: local extrema
+    {
+        float ms = -INFINITY, mx = -INFINITY, mn = INFINITY;
+        for (int k = half; k < nsc; k += 2) {
+            float v[16];
+            tmem_ld16(tmem + lane_off + kColS + 16 * k, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) ms = fmaxf(ms, v[i]);
+        }
+        for (int k = half; k < nfc; k += 2) {
+            float v[32];
+            tmem_ld32(tmem + lane_off + kColA + 32 * k, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, v[i]); mn = fminf(mn, v[i]); }
+        }
+        ex[0 * 256 + half * 128 + row] = ms;
+        ex[1 * 256 + half * 128 + row] = mx;
+        ex[2 * 256 + half * 128 + row] = mn;
+    }
+    __syncthreads();
+    if (!mbar_wait(bar_z, 0, kWaitNs)) atomicOr(fail, 1);
+
+    // ---- round 2: exponentials, P, unnormalised phi halves, partial sums
+    {
+        const float m_raw = fmaxf(ex[0 * 256 + row], ex[0 * 256 + 128 + row]);
+        const float mx = fmaxf(ex[1 * 256 + row], ex[1 * 256 + 128 + row]);
+        const float mn = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]);
+        float l = 0.f, sp = 0.f, sn = 0.f, lp = 0.f, ln = 0.f;
+        for (int k = half; k < nsc; k += 2) {
+            float v[16];
+            tmem_ld16(tmem + lane_off + kColS + 16 * k, v);
+            tmem_wait_ld();
+            uint32_t pk[8];
+#pragma unroll
+            for (int i = 0; i < 16; i += 2) {
+                const float p0 = exp2f((v[i] - m_raw) * a.scale_log2);
+                const float p1 = exp2f((v[i + 1] - m_raw) * a.scale_log2);
+                pk[i / 2] = pack_bf16x2(p0, p1);
+                const __nv_bfloat162 b2 = *reinterpret_cast<const __nv_bfloat162 *>(&pk[i / 2]);
+                l += __low2float(b2) + __high2float(b2);   // sum what the MMA will use
+            }
+            // P is K-major without swizzle: core matrices of 8 rows x 16 bytes
+            uint8_t *prow = smem + a.off_p + (row >> 3) * (B / 8) * 128 + (row & 7) * 16;
+            *reinterpret_cast<uint4 *>(prow + (2 * k) * 128) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            *reinterpret_cast<uint4 *>(prow + (2 * k + 1) * 128) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+        }
+        const float *zs = reinterpret_cast<const float *>(smem + a.off_z);
+        const float mxl = mx * kLog2e, mnl = mn * kLog2e;
+        for (int k = half; k < nfc; k += 2) {
+            float u[32], ep[32], en[32];
+            tmem_ld32(tmem + lane_off + kColA + 32 * k, u);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                ep[i] = exp2f(fmaf(u[i], kLog2e, -mxl));
+                en[i] = exp2f(fmaf(-u[i], kLog2e, mnl));
+                sp += ep[i];
+                sn += en[i];
+                lp = fmaf(ep[i], zs[32 * k + i], lp);
+                ln = fmaf(en[i], zs[F + 32 * k + i], ln);
+            }
+            tmem_st32(tmem + lane_off + kColA + 32 * k, ep);
+            tmem_st32(tmem + lane_off + kColA + F + 32 * k, en);
+        }
+        ex[3 * 256 + half * 128 + row] = l;
+        ex[4 * 256 + half * 128 + row] = sp;
+        ex[5 * 256 + half * 128 + row] = sn;
+        ex[6 * 256 + half * 128 + row] = lp;
+        ex[7 * 256 + half * 128 + row] = ln;
+        if (half == 0) stat[row] = m_raw * a.inv_sqrt_d;
+        tmem_wait_st();
+    }
+    __syncthreads();
+
+    // ---- round 3: normalise phi in place (rounded to tf32), row statistics
+    {
+        const float sp = ex[4 * 256 + row] + ex[4 * 256 + 128 + row];
+        const float sn = ex[5 * 256 + row] + ex[5 * 256 + 128 + row];
+        const float isp = 1.f / sp, isn = 1.f / sn;
+        for (int k = half; k < nfc; k += 2) {
+            float v[32];
+            tmem_ld32(tmem + lane_off + kColA + 32 * k, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = tf32_round(v[i] * isp);
+            tmem_st32(tmem + lane_off + kColA + 32 * k, v);
+            tmem_ld32(tmem + lane_off + kColA + F + 32 * k, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = tf32_round(v[i] * isn);
+            tmem_st32(tmem + lane_off + kColA + F + 32 * k, v);
+        }
+        if (half == 0) {
+            stat[128 + row] = ex[3 * 256 + row] + ex[3 * 256 + 128 + row];
+            const float lp = ex[6 * 256 + row] + ex[6 * 256 + 128 + row];
+            const float ln = ex[7 * 256 + row] + ex[7 * 256 + 128 + row];
+            stat[256 + row] = lp * isp + ln * isn;
+        }
+        tmem_wait_st();
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+
+    // ---- readout D_lin = phi(Q) S_g over the 2F/32 state tiles, then D_s = P V
+    if (tid == 0) {
+        bool ok = *fail == 0;
+        if (ok) {
+            tc_fence_after();
+            const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
+            for (int c = 0; c < NC && ok; ++c) {
+                const int slot = c % a.n_slots;
+                const uint32_t ph = (uint32_t)(c / a.n_slots) & 1u;
+                if (!mbar_wait(&full[slot], ph, kWaitNs)) { ok = false; break; }
+                const uint32_t s_u = smem_u32(smem + (size_t)slot * chunk_bytes);
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)
+                    mma_tf32_ts(tmem + kColD, tmem + kColA + 32 * c + 8 * kk,
+                                smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B), idR, (c | kk) != 0);
+                if (c + a.n_slots < NC) {
+                    // refill this slot once the tensor cores have read it
+                    mma_commit(&empty[slot]);
+                    if (!mbar_wait(&empty[slot], ph, kWaitNs)) { ok = false; break; }
+                    mbar_arrive_expect_tx(&full[slot], chunk_bytes);
+                    bulk_g2s(smem + (size_t)slot * chunk_bytes, Sg + (size_t)(c + a.n_slots) * 32 * d,
+                             chunk_bytes, &full[slot]);
+                    *issued = c + a.n_slots + 1;
+                }
+            }
+            if (ok) {
+                const uint32_t p_u = smem_u32(smem + a.off_p), v_u = smem_u32(smem + a.off_v);
+                const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
+                for (int k = 0; k < B / 16; ++k) {
+                    const uint64_t ad = smem_desc(p_u + k * 256, 128, (B / 8) * 128, SWZ_NONE);
+                    const uint64_t bd = smem_desc(v_u + 2 * k * ((d / 64) * 1024), 1024, (d / 64) * 1024, SWZ_128B);
+                    mma_bf16_ss(tmem + kColS, ad, bd, idP, k > 0);
+                }
+                mma_commit(bar_d);
+            }
+        }
+        if (!ok) {
+            atomicOr(fail, 1);
+            mbar_arrive(bar_d);   // release the waiting threads
+        }
+    }
+    if (!mbar_wait(bar_d, 0, kWaitNs)) atomicOr(fail, 1);
+    tc_fence_after();
+    __syncthreads();
+    const bool failed = *fail != 0;
+
+    // ---- epilogue: out = ws * D_s + wl * D_lin, stored as bf16
+    if (!failed) {
+        const int dh = d / 2;
+        const float m = stat[row], l = stat[128 + row], ld = stat[256 + row];
+        const int t = row / G, hh = row % G;
+        MergeWeights mw{0.f, 0.f};
+        if (valid) mw = merge_weights(log_sigmoid(a.alpha[g * G + hh]), m, l, ld);
+        __nv_bfloat16 *orow = a.O + (((size_t)r * B + t) * a.Hq + g * G + hh) * d + half * dh;
+        for (int c0 = 0; c0 < dh; c0 += 32) {
+            float dl[32], ds[32];
+            tmem_ld32(tmem + lane_off + kColD + half * dh + c0, dl);
+            tmem_ld32(tmem + lane_off + kColS + half * dh + c0, ds);
+            tmem_wait_ld();
+            if (valid) {
+                uint32_t pk[16];
+#pragma unroll
+                for (int i = 0; i < 32; i += 2) {
+                    const float o0 = mw.ws * ds[i] + (mw.wl == 0.f ? 0.f : mw.wl * dl[i]);
+                    const float o1 = mw.ws * ds[i + 1] + (mw.wl == 0.f ? 0.f : mw.wl * dl[i + 1]);
+                    pk[i / 2] = pack_bf16x2(o0, o1);
+                }
+                uint4 *dst = reinterpret_cast<uint4 *>(orow + c0);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+            }
+        }
+    } else if (tid == 0) {
+        raise_error(a.err, ERR_WAIT_TIMEOUT);
+        // drain bulk copies that may still be landing in this CTA's shared memory
+        mbar_wait(bar_z, 0, kWaitNs);
+        for (int c = 0; c < *issued; ++c)
+            mbar_wait(&full[c % a.n_slots], (uint32_t)(c / a.n_slots) & 1u, kWaitNs);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+}  // namespace
+
+bool tc_attn_supported(const hybrid_cfg &c)
+{
+    if (c.io_dtype != HYBRID_BF16) return false;
+    if (c.head_dim != 64 && c.head_dim != 128) return false;
+    if (c.feat_dim != 64 && c.feat_dim != 128) return false;
+    if (c.block_size % 16 != 0) return false;
+    const int G = c.n_q_heads / c.n_kv_heads;
+    if (G * c.block_size > 128) return false;
+    const Layout L = make_layout(c.head_dim, c.feat_dim, c.block_size);
+    return L.n_slots >= 1 && (int)L.bytes <= kSmemLimit;
+}
+
+cudaError_t launch_attn_tc(const hybrid_cfg &c, const void *Q, const void *K, const void *V, const void *W,
+                           const float *alpha, void *const *states, int n_req, void *O, unsigned *err,
+                           cudaStream_t st)
+{
+    const Layout L = make_layout(c.head_dim, c.feat_dim, c.block_size);
+    TcAttnArgs a;
+    a.Q = static_cast<const __nv_bfloat16 *>(Q);
+    a.K = static_cast<const __nv_bfloat16 *>(K);
+    a.V = static_cast<const __nv_bfloat16 *>(V);
+    a.W = static_cast<const __nv_bfloat16 *>(W);
+    a.alpha = alpha;
+    a.states = states;
+    a.O = static_cast<__nv_bfloat16 *>(O);
+    a.err = err;
+    a.B = c.block_size;
+    a.Hq = c.n_q_heads;
+    a.Hkv = c.n_kv_heads;
+    a.G = c.n_q_heads / c.n_kv_heads;
+    a.d = c.head_dim;
+    a.F = c.feat_dim;
+    a.n_slots = L.n_slots;
+    a.inv_sqrt_d = 1.f / sqrtf((float)c.head_dim);
+    a.scale_log2 = kLog2e * a.inv_sqrt_d;
+    a.off_q = L.off_q;
+    a.off_w = L.off_w;
+    a.off_k = L.off_k;
+    a.off_v = L.off_v;
+    a.off_p = L.off_p;
+    a.off_z = L.off_z;
+    a.off_bar = L.off_bar;
+    cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.bytes);
+    if (e != cudaSuccess) return e;
+    const long long blocks = (long long)n_req * c.n_kv_heads;
+    k_attn_tc<<<(unsigned)blocks, kThreads, L.bytes, st>>>(a);
+    return cudaGetLastError();
 }
 
 }  // namespace hyb
