@@ -212,7 +212,7 @@ def cpu_baseline(wl, budget_s=12.0):
     alpha64 = alpha.double().numpy()
     n_sample = min(wl.n_req, 16)
     t_one = oracle_sample_step(wl, orc, n_sample, "cpu-probe", W64, alpha64)
-    reps = max(1, min(50, int(budget_s / max(t_one, 1e-6))))
+    reps = max(1, min(10000, int(budget_s / max(t_one, 1e-6))))
     tot = 0.0
     for i in range(reps):
         tot += oracle_sample_step(wl, orc, n_sample, ("cpu", i), W64, alpha64)
