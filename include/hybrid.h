@@ -130,6 +130,19 @@ hybrid_status hybrid_block_attn(const hybrid_cfg *cfg, const void *Q, const void
                                 const void *W, const float *alpha, void *const *d_state_ptrs,
                                 int n_req, void *O, cudaStream_t stream);
 
+/* One denoising step followed by the commit of the same block, in one pass
+ * over the states (Section 3.1's step and state update; the paper's serving
+ * section computes both in a single kernel launch).  O is computed from the
+ * pre-commit state, then the block's K, V are folded into (S, z): equivalent to
+ * hybrid_block_attn followed by hybrid_commit_block with n_tok = B, reading
+ * and writing each state element once.  Arguments and layouts as in
+ * hybrid_block_attn; the states are updated in place, so d_state_ptrs must not
+ * name the same state twice. */
+hybrid_status hybrid_block_attn_commit(const hybrid_cfg *cfg, const void *Q, const void *K,
+                                       const void *V, const void *W, const float *alpha,
+                                       void *const *d_state_ptrs, int n_req, void *O,
+                                       cudaStream_t stream);
+
 /* Block commit of Section 3.1: S += sum_t phi(k_t) v_t^T, z += sum_t phi(k_t)
  * over the n_tok tokens of K, V [n][n_tok][Hkv][d] (io_dtype), for every
  * request and state head.  n_tok = B folds a decoded block; any n_tok >= 0

@@ -95,9 +95,33 @@ hybrid_status hybrid_block_attn(const hybrid_cfg *cfg, const void *Q, const void
         return HYBRID_ERR_INVALID_ARG;
     unsigned *err = error_word();
     if (!err) return HYBRID_ERR_CUDA;
+    if (hyb::fused_supported(*cfg, false))
+        return from_cuda(hyb::launch_fused(*cfg, false, Q, K, V, W, alpha, d_state_ptrs, n_req, O, err, stream));
     if (hyb::tc_attn_supported(*cfg))
         return from_cuda(hyb::launch_attn_tc(*cfg, Q, K, V, W, alpha, d_state_ptrs, n_req, O, err, stream));
     return from_cuda(hyb::launch_attn_generic(*cfg, Q, K, V, W, alpha, d_state_ptrs, n_req, O, err, stream));
+}
+
+hybrid_status hybrid_block_attn_commit(const hybrid_cfg *cfg, const void *Q, const void *K, const void *V,
+                                       const void *W, const float *alpha, void *const *d_state_ptrs,
+                                       int n_req, void *O, cudaStream_t stream)
+{
+    hybrid_status s = check_cfg(cfg);
+    if (s != HYBRID_OK) return s;
+    if (n_req < 0) return HYBRID_ERR_INVALID_ARG;
+    if (n_req == 0) return HYBRID_OK;
+    if (!Q || !K || !V || !W || !alpha || !d_state_ptrs || !O) return HYBRID_ERR_INVALID_ARG;
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(W, 16) || !aligned(O, 16) ||
+        !aligned(alpha, 4) || !aligned(d_state_ptrs, 8))
+        return HYBRID_ERR_INVALID_ARG;
+    unsigned *err = error_word();
+    if (!err) return HYBRID_ERR_CUDA;
+    if (hyb::fused_supported(*cfg, true))
+        return from_cuda(hyb::launch_fused(*cfg, true, Q, K, V, W, alpha, d_state_ptrs, n_req, O, err, stream));
+    // other shapes: the step, then the commit, on the same stream
+    s = hybrid_block_attn(cfg, Q, K, V, W, alpha, d_state_ptrs, n_req, O, stream);
+    if (s != HYBRID_OK) return s;
+    return hybrid_commit_block(cfg, K, V, cfg->block_size, W, d_state_ptrs, n_req, stream);
 }
 
 hybrid_status hybrid_commit_block(const hybrid_cfg *cfg, const void *K, const void *V, int n_tok,

@@ -271,3 +271,54 @@ def test_prefill_commit_long_ragged():
     S, z = pair.gpu_state()
     assert_parity(S, pair.S, BF16, "prefill S")
     assert_parity(z, pair.z, BF16, "prefill z")
+
+
+# ---------------------------------------------------------------------------
+# fused step + commit (hybrid_block_attn_commit)
+# ---------------------------------------------------------------------------
+FUSED = [
+    (W_("fused_gqa4", BF16, 5, 8, 2, 128, 128, 32, 51), [0, 32, 96, 160, 256]),
+    (W_("fused_mha_d64_f64", BF16, 3, 4, 4, 64, 64, 32, 52), [64, 0, 32]),
+    (W_("fused_gqa4_many_units", BF16, 40, 16, 4, 128, 128, 32, 53), None),   # 160 units > 152 SMs
+    (W_("fused_b16_fallback", BF16, 3, 4, 2, 128, 128, 16, 54), [16, 0, 48]),  # B != 32: step + commit
+]
+
+
+@pytest.mark.parametrize("wl,plen", FUSED, ids=[w.name for w, _ in FUSED])
+def test_fused_step_commit_parity(wl, plen):
+    pair = Pair(wl)
+    plen = (np.arange(wl.n_req) % 5) * wl.B if plen is None else np.asarray(plen, dtype=np.int64)
+    pair.build_prefixes(plen)
+    for step in range(3):   # three consecutive committing steps
+        Q, K, V = wk.block_qkv(wl, ("fused", step), pair.dev)
+        O = torch.empty_like(Q)
+        H.hybrid_block_attn_commit(pair.cfg, Q, K, V, pair.W, pair.alpha, pair.ptrs, wl.n_req, O)
+        H.hybrid_check()
+        t = torch.as_tensor(pair.tracked, device=Q.device)
+        want = pair.orc.block_attn(h64(Q[t]), h64(K[t]), h64(V[t]), pair.W64, pair.alpha64,
+                                   pair.S, pair.z)
+        assert_parity(h64(O[t]), want, wl.io_dtype, f"fused output, step {step}")
+        pair.orc.commit(h64(K[t]), h64(V[t]), pair.W64, pair.S, pair.z)
+        S, z = pair.gpu_state()
+        assert_parity(S, pair.S, wl.io_dtype, f"fused state S, step {step}")
+        assert_parity(z, pair.z, wl.io_dtype, f"fused state z, step {step}")
+
+
+def test_fused_matches_separate_calls():
+    """hybrid_block_attn_commit equals hybrid_block_attn then hybrid_commit_block
+    (both within the bf16 tolerance of each other)."""
+    wl = W_("fused_vs_separate", BF16, 6, 16, 4, 128, 128, 32, 55)
+    a, b = Pair(wl), Pair(wl)
+    plen = np.array([32, 64, 0, 128, 96, 32])
+    a.build_prefixes(plen)
+    b.build_prefixes(plen)
+    Q, K, V = wk.block_qkv(wl, "fvs", a.dev)
+    O1, O2 = torch.empty_like(Q), torch.empty_like(Q)
+    H.hybrid_block_attn_commit(a.cfg, Q, K, V, a.W, a.alpha, a.ptrs, wl.n_req, O1)
+    H.hybrid_block_attn(b.cfg, Q, K, V, b.W, b.alpha, b.ptrs, wl.n_req, O2)
+    H.hybrid_commit_block(b.cfg, K, V, wl.B, b.W, b.ptrs, wl.n_req)
+    H.hybrid_check()
+    assert rel_l2(h64(O1), h64(O2)) <= 1e-2
+    Sa, za = a.gpu_state()
+    Sb, zb = b.gpu_state()
+    assert rel_l2(Sa, Sb) <= 1e-3 and rel_l2(za, zb) <= 1e-4
