@@ -1,5 +1,6 @@
 // hybrid_api.cu -- the extern "C" entry points declared in include/hybrid.h:
 // argument validation, kernel selection and launch, and the device error word.
+#include <atomic>
 #include <mutex>
 
 #include "hybrid_common.cuh"
@@ -13,7 +14,7 @@ __device__ unsigned g_error_word;
 
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
-unsigned *g_err_ptr[kMaxDevices];
+std::atomic<unsigned *> g_err_ptr[kMaxDevices];
 
 // Device address of this device's error word, looked up once per device
 // (with that device current, as cudaGetSymbolAddress requires).
@@ -21,13 +22,17 @@ unsigned *error_word()
 {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    unsigned *p = g_err_ptr[dev].load(std::memory_order_acquire);
+    if (p) return p;
     std::lock_guard<std::mutex> lock(g_mu);
-    if (!g_err_ptr[dev]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
-        g_err_ptr[dev] = static_cast<unsigned *>(p);
+    p = g_err_ptr[dev].load(std::memory_order_relaxed);
+    if (!p) {
+        void *sym = nullptr;
+        if (cudaGetSymbolAddress(&sym, g_error_word) != cudaSuccess) return nullptr;
+        p = static_cast<unsigned *>(sym);
+        g_err_ptr[dev].store(p, std::memory_order_release);
     }
-    return g_err_ptr[dev];
+    return p;
 }
 
 bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }

@@ -14,8 +14,13 @@
 //              copies, through an NS-slot ring (the state layout is the MMA
 //              operand image, see hybrid.h).
 //   warp 1     MMA issuer (one thread).
-//   warps 2-3  producers: Q, W, K (region X) and V of the next unit by cp.async;
-//              V^T in f32 (commit operand) into region X once Q, W, K are spent.
+//   warp 2     producer: TMA of Q, W, K (region X) and V of the next unit; V^T in
+//              f32 (commit operand) into region X once Q, W, K are spent.
+//   warp 3     storer: TMA stores of the output tile and, with the commit, bulk
+//              stores of the updated state tiles and z, releasing ring slots
+//              once they have been read out.  The output tile (128 rows x d
+//              bf16) is staged in the ring slots of the unit's last two state
+//              tiles, which are held back for it.
 //   warps 4-11 math: row statistics and phi(Q) (one thread per TMEM lane and
 //              column half), P, phi(K)^T, the state-tile update and the output.
 // Tensor Memory (512 columns):
@@ -35,6 +40,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "hybrid_common.cuh"
@@ -50,7 +56,6 @@ using bf16 = __nv_bfloat16;
 constexpr int kWarps = 12;
 constexpr int kThreads = kWarps * 32;
 constexpr int kMathThreads = 256;
-constexpr int kProdThreads = 64;
 constexpr uint32_t kColA = 0, kColD0 = 256;
 constexpr int kMaxSlots = 16;
 constexpr uint64_t kWaitNs = 1000000000ull;
@@ -58,10 +63,9 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kSmemLimit = 232448;
 constexpr int kOneCtaPerSm = 118 * 1024;
 constexpr uint32_t kBarMath = 1;
-constexpr uint32_t kBarProd = 2;
 
 struct FusedArgs {
-    CUtensorMap tmQ, tmK, tmV, tmW;   // Q [n*B][Hq][d], K and V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
+    CUtensorMap tmQ, tmK, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], K and V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
     const bf16 *Q, *K, *V, *W;
     const float *alpha;
     void *const *states;
@@ -157,10 +161,7 @@ __device__ __forceinline__ bool math_sync_failed(bool local_fail)
 {
     return group_sync_failed(kBarMath, kMathThreads, local_fail);
 }
-__device__ __forceinline__ bool prod_sync_failed(bool local_fail)
-{
-    return group_sync_failed(kBarProd, kProdThreads, local_fail);
-}
+
 
 // Reduce 16 per-lane values across the 32 lanes of a warp (op = add / max /
 // min) by halving the set each step; on return lane L holds the total of
@@ -241,6 +242,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int d = a.d, F = a.F, B = a.B, G = a.G, NS = a.NS;
     const int NC = (2 * F) / 32;
+    // with the commit, the output tile is staged in the slots of tiles ocm, ocm + 1
+    const int ocm = NC > NS ? NC - NS : 0;
     const uint32_t chunk_bytes = (uint32_t)d * 128;
     const int per = a.n_units / (int)gridDim.x, rem = a.n_units % (int)gridDim.x;
     const int u_begin = (int)blockIdx.x * per + min((int)blockIdx.x, rem);
@@ -265,7 +268,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint64_t *efree = phiready + 1;
     uint64_t *rdone = efree + 1;
     uint64_t *mmadone = rdone + 1;
-    const int n_bars = 2 * NS + 14 + 10;
+    uint64_t *tready = mmadone + 1;  // [2] math -> storer: a feature half of the tiles is updated
+    uint64_t *zdone = tready + 2;    // math -> storer: z is updated
+    uint64_t *ofree = zdone + 1;     // the last two slots of the unit may take the output tile
+    uint64_t *ostaged = ofree + 1;   // math -> storer: the output tile is in the slots
+    const int n_bars = 2 * NS + 14 + 15;
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + n_bars);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
@@ -373,7 +380,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     for (int kk = 0; kk < 4; ++kk)
                         mma_tf32_ts(dcol, tmem + kColA + 32 * c + 8 * kk, smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B),
                                     idR, (c | kk) != 0);
-                    if (!kCommit) mma_commit(&empty[slot]);
+                    if (!kCommit) {
+                        if (c < NC - 2) mma_commit(&empty[slot]);
+                        else if (c == NC - 1) mma_commit(ofree);
+                    }
                     if (kCommit && c == NC / 2 - 1) {
                         // phi+ has been read: its columns take dS^T for features [0, F);
                         // dS^T for [F, 2F) goes to the idle output accumulator
@@ -408,9 +418,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             mma_commit(mmadone);
             mbar_wait(mmadone, 0, kWaitNs);
         }
-    } else if (warp < 4) {
-        // ------------------------------------------------------------ producers
-        const int pt = tid - 64;
+    } else if (warp == 2) {
+        // ------------------------------------------------------------- producer
         uint32_t kp = 0;
         for (int u = u_begin; u < u_end; ++u) {
             if (!unit_state(a, u)) continue;
@@ -420,16 +429,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 // region X is free once the previous unit's last use of it has completed
                 ok = kCommit ? wait_bar(&dsready[1], (kp - 1) & 1u, fail) : wait_bar(xfree, (kp - 1) & 1u, fail);
             }
-            if (prod_sync_failed(!ok)) break;
-            if (pt == 0) tma_x(a, smem, r, g, xfull);
+            if (__any_sync(0xffffffffu, !ok)) break;
+            if (lane == 0) tma_x(a, smem, r, g, xfull);
             if (kp > 0) ok = wait_bar(vfree, (kp - 1) & 1u, fail);
-            if (prod_sync_failed(!ok)) break;
-            if (pt == 0) tma_v(a, smem, r, g, vfull);
+            if (__any_sync(0xffffffffu, !ok)) break;
+            if (lane == 0) tma_v(a, smem, r, g, vfull);
             if (kCommit) {
                 // V^T in f32 into region X once this unit's first MMA group is done with it
                 ok = wait_bar(xfree, kp & 1u, fail);
-                if (prod_sync_failed(!ok)) break;
-                for (int idx = pt; idx < 16 * 32; idx += kProdThreads) {
+                if (__any_sync(0xffffffffu, !ok)) break;
+                for (int idx = lane; idx < 16 * 32; idx += 32) {
                     const int eg = idx >> 5, t = idx & 31;     // 8 rows e = 8*eg .. 8*eg+7, column t
                     float v[8];
                     if (eg * 8 < d) {
@@ -449,10 +458,62 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     }
                 }
                 fence_proxy_async_smem();
-                if (prod_sync_failed(false)) break;
-                if (pt == 0) mbar_arrive(vtready);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(vtready);
             }
             ++kp;
+        }
+    } else if (warp == 3) {
+        // --------------------------------------------------------------- storer
+        if (lane == 0) {
+            uint32_t q = 0, kp = 0;
+            for (int u = u_begin; u < u_end; ++u) {
+                float *Sg = unit_state(a, u);
+                if (!Sg) continue;
+                const int r = u / a.Hkv, g = u % a.Hkv;
+                bool ok = true;
+                if (kCommit) {
+                    const int zb = kp & 1;
+                    if (!wait_bar(zdone, kp & 1u, fail)) break;
+                    bulk_s2g(Sg + (size_t)2 * F * d, zbuf0 + zb * zstride, 2 * F * 4);
+                    bulk_commit();
+                    bulk_wait_read_all();
+                    mbar_arrive(&zempty[zb]);
+                    for (int h = 0; h < 2 && ok; ++h) {
+                        if (!wait_bar(&tready[h], kp & 1u, fail)) { ok = false; break; }
+                        for (int c = h * NC / 2; c < (h + 1) * NC / 2; ++c)
+                            bulk_s2g(Sg + (size_t)c * 32 * d, ring + (size_t)((q + c) % NS) * chunk_bytes, chunk_bytes);
+                        bulk_commit();
+                        bulk_wait_read_all();
+                        // with the commit, two slots of the first half are held for the
+                        // output tile: tiles oc and oc + 1, whose slots no later tile of
+                        // this unit reuses
+                        for (int c = h * NC / 2; c < (h + 1) * NC / 2; ++c)
+                            if (h == 1 || c < ocm || c > ocm + 1) mbar_arrive(&empty[(q + c) % NS]);
+                        if (h == 0) mbar_arrive(ofree);
+                    }
+                    if (!ok) break;
+                }
+                // output tile: two TMA boxes from the two held-back slots
+                if (!wait_bar(ostaged, kp & 1u, fail)) break;
+                const int oc = kCommit ? ocm : NC - 2;   // first of the two slots holding the output
+                uint8_t *s0 = ring + (size_t)((q + oc) % NS) * chunk_bytes;
+                uint8_t *s1 = ring + (size_t)((q + oc + 1) % NS) * chunk_bytes;
+                if (d == 128) {
+                    tma_store_3d(&a.tmO, 0, g * G, r * B, s0);
+                    tma_store_3d(&a.tmO, 64, g * G, r * B, s1);
+                } else {
+                    tma_store_3d(&a.tmO, 0, g * G, r * B, s0);
+                    tma_store_3d(&a.tmO, 0, g * G, r * B + B / 2, s1);
+                }
+                bulk_commit();
+                bulk_wait_read_all();
+                mbar_arrive(&empty[(q + oc) % NS]);
+                mbar_arrive(&empty[(q + oc + 1) % NS]);
+                q += NC;
+                ++kp;
+            }
+            bulk_wait_all();
         }
     } else {
         // ------------------------------------------------------------- math
@@ -476,8 +537,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 if (mt == 0) raise_error(a.err, ERR_BAD_STATE_PTR);
                 continue;
             }
-            const int g = u % a.Hkv, r = u / a.Hkv;
+            const int g = u % a.Hkv;
             const int zb = kp & 1;
+            // gate of this row's query head, loaded now so the latency overlaps the first rounds
+            const float alpha_row = valid ? a.alpha[g * G + row % G] : 0.f;
             float *zs = zbuf0 + zb * zstride;
             const uint32_t dcol = tmem + kColD0 + 128 * (kp & 1);
             float *den = den_s + 128 * (kp & 1);
@@ -630,7 +693,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 const float ln = ex[7 * 256 + row] + ex[7 * 256 + 128 + row];
                 const float lin_den = lp / sp + ln / sn;
                 const int hh = row % G;
-                const float lw = valid ? log_sigmoid(a.alpha[g * G + hh]) : 0.f;
+                const float lw = valid ? log_sigmoid(alpha_row) : 0.f;
                 const float log_s = lw + m_raw * a.scale + logf(l);   // log(w sm_den)
                 const float log_l = logf(lin_den);                      // log(lin_den), -inf if empty
                 const float sig = fmaxf(fmaxf(log_s, log_l), -60.f);
@@ -638,17 +701,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 const float cpos = lin_den > 0.f ? esig / sp : 0.f;
                 const float cneg = lin_den > 0.f ? esig / sn : 0.f;
                 for (int k = half; k < nfc; k += 2) {
-                    float v[32];
+                    float v[32], w[32];
                     tmem_ld32(tmem + lane_off + kColA + 32 * k, v);
+                    tmem_ld32(tmem + lane_off + kColA + F + 32 * k, w);
                     tmem_wait_ld();
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] *= cpos;
+                    for (int i = 0; i < 32; ++i) { v[i] *= cpos; w[i] *= cneg; }
                     tmem_st32(tmem + lane_off + kColA + 32 * k, v);
-                    tmem_ld32(tmem + lane_off + kColA + F + 32 * k, v);
-                    tmem_wait_ld();
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] *= cneg;
-                    tmem_st32(tmem + lane_off + kColA + F + 32 * k, v);
+                    tmem_st32(tmem + lane_off + kColA + F + 32 * k, w);
                 }
                 // P' = w e^(s - sigma): K-major, no swizzle (8-row x 16-byte core matrices)
                 const float pofs = (lw - sig) * kLog2e;
@@ -671,19 +731,24 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     uint8_t *rp = pt_s + row * 128;
                     uint8_t *rn = pt_s + (F + row) * 128;
                     float dzp = 0.f, dzn = 0.f;
+                    float4 x[4], y[4], a4[4], b4[4];
 #pragma unroll
                     for (int gq = 0; gq < 4; ++gq) {
                         const int gi = 4 * half + gq;
-                        float4 *pp = reinterpret_cast<float4 *>(rp + ((gi ^ (row & 7)) << 4));
-                        float4 *pn = reinterpret_cast<float4 *>(rn + ((gi ^ ((F + row) & 7)) << 4));
-                        const float4 a4 = ip[gq], b4 = in[gq];
-                        float4 x = *pp, y = *pn;
-                        x.x *= a4.x; x.y *= a4.y; x.z *= a4.z; x.w *= a4.w;
-                        y.x *= b4.x; y.y *= b4.y; y.z *= b4.z; y.w *= b4.w;
-                        *pp = x;
-                        *pn = y;
-                        dzp += (x.x + x.y) + (x.z + x.w);
-                        dzn += (y.x + y.y) + (y.z + y.w);
+                        x[gq] = *reinterpret_cast<const float4 *>(rp + ((gi ^ (row & 7)) << 4));
+                        y[gq] = *reinterpret_cast<const float4 *>(rn + ((gi ^ ((F + row) & 7)) << 4));
+                        a4[gq] = ip[gq];
+                        b4[gq] = in[gq];
+                    }
+#pragma unroll
+                    for (int gq = 0; gq < 4; ++gq) {
+                        const int gi = 4 * half + gq;
+                        x[gq].x *= a4[gq].x; x[gq].y *= a4[gq].y; x[gq].z *= a4[gq].z; x[gq].w *= a4[gq].w;
+                        y[gq].x *= b4[gq].x; y[gq].y *= b4[gq].y; y[gq].z *= b4[gq].z; y[gq].w *= b4[gq].w;
+                        *reinterpret_cast<float4 *>(rp + ((gi ^ (row & 7)) << 4)) = x[gq];
+                        *reinterpret_cast<float4 *>(rn + ((gi ^ ((F + row) & 7)) << 4)) = y[gq];
+                        dzp += (x[gq].x + x[gq].y) + (x[gq].z + x[gq].w);
+                        dzn += (y[gq].x + y[gq].y) + (y[gq].z + y[gq].w);
                     }
                     atomicAdd(&zs[row], dzp);
                     atomicAdd(&zs[F + row], dzn);
@@ -697,11 +762,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 mbar_arrive(phiready);
                 if (kCommit) {
                     mbar_arrive(vtready);
-                    bulk_s2g(Sg + (size_t)2 * F * d, zs, 2 * F * 4);
-                    bulk_commit();
-                    bulk_wait_read_all();
+                    mbar_arrive(zdone);
+                } else {
+                    mbar_arrive(&zempty[zb]);
                 }
-                mbar_arrive(&zempty[zb]);
             }
 
             // ---- state update: S^T tile rows += dS^T rows (per feature half), then store
@@ -721,77 +785,81 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                         const int slot = (q + c) % NS;
                         float v[32];
                         tmem_ld32((h == 0 ? tmem + kColA : dother) + lane_off + fl, v);
+                        uint8_t *rowp = ring + (size_t)slot * chunk_bytes + e * 128;
+                        float4 s[8];
+                        if (e < d) {
+#pragma unroll
+                            for (int gq = 0; gq < 8; ++gq) s[gq] = *reinterpret_cast<const float4 *>(rowp + ((gq ^ (e & 7)) << 4));
+                        }
                         tmem_wait_ld();
                         if (ok && e < d) {
-                            uint8_t *rowp = ring + (size_t)slot * chunk_bytes + e * 128;
 #pragma unroll
                             for (int gq = 0; gq < 8; ++gq) {
-                                float4 *p = reinterpret_cast<float4 *>(rowp + ((gq ^ (e & 7)) << 4));
-                                float4 s = *p;
-                                s.x += v[4 * gq];
-                                s.y += v[4 * gq + 1];
-                                s.z += v[4 * gq + 2];
-                                s.w += v[4 * gq + 3];
-                                *p = s;
+                                s[gq].x += v[4 * gq];
+                                s[gq].y += v[4 * gq + 1];
+                                s[gq].z += v[4 * gq + 2];
+                                s[gq].w += v[4 * gq + 3];
                             }
+#pragma unroll
+                            for (int gq = 0; gq < 8; ++gq) *reinterpret_cast<float4 *>(rowp + ((gq ^ (e & 7)) << 4)) = s[gq];
                         }
                     }
                     fence_proxy_async_smem();
                     tc_fence_before();
                     if (math_sync_failed(!ok)) { brk = true; break; }
                     if (mt == 0) {
-                        for (int c = h * NC / 2; c < (h + 1) * NC / 2; ++c)
-                            bulk_s2g(Sg + (size_t)c * 32 * d, ring + (size_t)((q + c) % NS) * chunk_bytes, chunk_bytes);
-                        bulk_commit();
-                        if (h == 0) {
-                            // release the first half's slots as soon as their tiles are read
-                            bulk_wait_read_all();
-                            for (int c = 0; c < NC / 2; ++c) mbar_arrive(&empty[(q + c) % NS]);
-                        } else {
-                            mbar_arrive(efree);
-                        }
+                        mbar_arrive(&tready[h]);
+                        if (h == 1) mbar_arrive(efree);
                     }
                 }
                 if (brk) break;
             }
 
-            // ---- output epilogue: out = D / den
+            // ---- output epilogue: out = D / den, staged as the TMA box image in the
+            // unit's last two ring slots (row i = t*G + hh, 128-byte swizzle)
             ok = wait_bar(&dready[kp & 1], (kp >> 1) & 1u, fail);
+            if (ok) ok = wait_bar(ofree, kp & 1u, fail);
             tc_fence_after();
-            if (kCommit && mt == 0) {
-                bulk_wait_read_all();
-                for (int c = NC / 2; c < NC; ++c) mbar_arrive(&empty[(q + c) % NS]);
-            }
             {
                 const int dh = d / 2;
                 const float inv = 1.f / den[row];
-                const int t = row / G, hh = row % G;
-                bf16 *orow = a.O + (((size_t)r * B + t) * a.Hq + g * G + hh) * d + half * dh;
-                for (int c0 = 0; c0 < dh; c0 += 32) {
-                    float v[32];
-                    tmem_ld32(dcol + lane_off + half * dh + c0, v);
-                    tmem_wait_ld();
-                    if (ok && valid) {
+                float v[2][32];
+                tmem_ld32(dcol + lane_off + half * dh, v[0]);
+                if (dh > 32) tmem_ld32(dcol + lane_off + half * dh + 32, v[1]);
+                tmem_wait_ld();
+                if (ok && valid) {
+                    // d = 128: column half -> slot; d = 64: token half -> slot (one 64-column atom)
+                    const int rows_half = G * B / 2;
+                    const int sidx = d == 128 ? half : (row >= rows_half ? 1 : 0);
+                    const int srow = d == 128 ? row : row - sidx * rows_half;
+                    const int oc = kCommit ? ocm : NC - 2;
+                    uint8_t *base = ring + (size_t)((q + oc + sidx) % NS) * chunk_bytes + srow * 128;
+#pragma unroll
+                    for (int hc = 0; hc < 2; ++hc) {
+                        if (hc * 32 >= dh) break;
                         uint32_t pk[16];
 #pragma unroll
-                        for (int i = 0; i < 32; i += 2) pk[i / 2] = pack_bf16x2(v[i] * inv, v[i + 1] * inv);
-                        uint4 *dst = reinterpret_cast<uint4 *>(orow + c0);
+                        for (int i = 0; i < 32; i += 2) pk[i / 2] = pack_bf16x2(v[hc][i] * inv, v[hc][i + 1] * inv);
 #pragma unroll
-                        for (int i = 0; i < 4; ++i)
-                            dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                        for (int i = 0; i < 4; ++i) {
+                            const int gi = 4 * hc + i + (d == 128 ? 0 : 4 * half);   // 16-byte granule in the 128-byte row
+                            *reinterpret_cast<uint4 *>(base + ((gi ^ (srow & 7)) << 4)) =
+                                make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                        }
                     }
                 }
             }
+            fence_proxy_async_smem();
             tc_fence_before();
             if (math_sync_failed(!ok)) break;
-            if (mt == 0) mbar_arrive(&dfree[kp & 1]);
+            if (mt == 0) {
+                mbar_arrive(ostaged);
+                mbar_arrive(&dfree[kp & 1]);
+            }
             q += NC;
             ++kp;
         }
-        if (mt == 0) {
-            bulk_wait_all();
-            if (*fail) raise_error(a.err, ERR_WAIT_TIMEOUT);
-        }
+        if (mt == 0 && *fail) raise_error(a.err, ERR_WAIT_TIMEOUT);
     }
 
     __syncthreads();
@@ -857,7 +925,7 @@ bool fused_supported(const hybrid_cfg &c, bool commit)
     const FLayout L = make_flayout(c.head_dim, c.feat_dim, c.block_size);
     const int NC = 2 * c.feat_dim / 32;
     // the commit keeps the first feature half resident while the second streams
-    if (L.NS < (commit ? NC / 2 + 2 : 2)) return false;
+    if (L.NS < (commit ? NC / 2 + 2 : 4)) return false;
     // region X must also hold V^T and phi(K)^T for the commit
     if (commit && (uint32_t)(128 * 128 + 2 * c.feat_dim * 128) > L.off_vb - L.off_q) return false;
     return (int)L.bytes <= kSmemLimit;
@@ -884,6 +952,9 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
         const cuuint32_t bw[2] = {64, (cuuint32_t)d};
         if (!encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !encode_bf16(&a.tmK, K, 3, dk, sk, bk) ||
             !encode_bf16(&a.tmV, V, 3, dk, sk, bk) || !encode_bf16(&a.tmW, W, 2, dw, sw, bw))
+            return cudaErrorInvalidValue;
+        const cuuint32_t bo[3] = {64, (cuuint32_t)G, (cuuint32_t)(d == 128 ? B : B / 2)};
+        if (!encode_bf16(&a.tmO, O, 3, dq, sq, bo))
             return cudaErrorInvalidValue;
     }
     a.Q = static_cast<const bf16 *>(Q);
@@ -912,16 +983,20 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
     a.off_st = L.off_st;
     a.off_bar = L.off_bar;
     const int grid = a.n_units < sm_count() ? a.n_units : sm_count();
-    cudaError_t e;
-    if (commit) {
-        e = cudaFuncSetAttribute(k_fused<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.bytes);
+    // opt in to the full shared memory once per device and kernel (the attribute
+    // is set to the maximum, so every layout fits)
+    static std::atomic<unsigned long long> opted[2];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    const unsigned long long bit = 1ull << dev;
+    if (!(opted[commit].load(std::memory_order_acquire) & bit)) {
+        const cudaError_t e = commit ? cudaFuncSetAttribute(k_fused<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit)
+                                     : cudaFuncSetAttribute(k_fused<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
         if (e != cudaSuccess) return e;
-        k_fused<true><<<grid, kThreads, L.bytes, st>>>(a);
-    } else {
-        e = cudaFuncSetAttribute(k_fused<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.bytes);
-        if (e != cudaSuccess) return e;
-        k_fused<false><<<grid, kThreads, L.bytes, st>>>(a);
+        opted[commit].fetch_or(bit, std::memory_order_release);
     }
+    if (commit) k_fused<true><<<grid, kThreads, L.bytes, st>>>(a);
+    else k_fused<false><<<grid, kThreads, L.bytes, st>>>(a);
     return cudaGetLastError();
 }
 
