@@ -8,35 +8,44 @@
 // every state tile is read once, used for the readout with the pre-commit
 // state, updated with this block's phi(k) v^T and written back.
 //
-// Work unit = (request r, state head g).  One CTA per SM loops over a
-// contiguous range of units.  Warp roles (12 warps):
+// Work unit = (request r, state head g): the G*B query rows of the unit share
+// one state.  One CTA per SM loops over a contiguous range of units.  Warp
+// roles (12 warps):
 //   warp 0     S producer: z and the 2F/32 state tiles of each unit, by 1-D bulk
 //              copies, through an NS-slot ring (the state layout is the MMA
 //              operand image, see hybrid.h).
-//   warp 1     MMA issuer (one thread).
-//   warp 2     producer: TMA of Q, W, K (region X) and V of the next unit; V^T in
-//              f32 (commit operand) into region X once Q, W, K are spent.
+//   warp 1     MMA issuer (one thread); owns the Tensor Memory allocation.
+//   warp 2     producer: TMA of Q and W, the transposed key tile K^T (built by
+//              the warp from global memory) and V, one unit ahead.
 //   warp 3     storer: TMA stores of the output tile and, with the commit, bulk
-//              stores of the updated state tiles and z, releasing ring slots
-//              once they have been read out.  The output tile (128 rows x d
-//              bf16) is staged in the ring slots of the unit's last two state
-//              tiles, which are held back for it.
-//   warps 4-11 math: row statistics and phi(Q) (one thread per TMEM lane and
-//              column half), P, phi(K)^T, the state-tile update and the output.
-// Tensor Memory (512 columns):
-//   [0,256)    U = Q W, then phi(Q) = [phi+, phi-] (A operand of the readout);
-//              with the commit, each half is reused for dS^T = V^T phi(K)^T of
-//              the same features once the readout has consumed it.
-//   [256,384), [384,512)  two output accumulators (alternating units): first
-//              the scores Q K^T (and U_k^T = W^T K^T), then
-//              D = phi'(Q) S + P' V, the merged numerator.
-// Merge: with sigma = log of the larger branch mass, phi' = phi e^-sigma and
-// P' = w e^(s - sigma), so D / den = (w sm_num + lin_num) / (w sm_den + lin_den)
-// exactly, with den = e^(log lin_den - sigma) + e^(log(w sm_den) - sigma) in [1, 2].
+//              stores of the updated state tiles and z.
+//   warps 4-11 math: two threads per query row (one per TMEM lane and "part");
+//              a part owns every other 32-feature chunk of each half of phi.
+//
+// Per unit the tensor cores run
+//   g1   [U | scores] = Q [W | K^T]  (one N = F + B product; U = Q W)
+//        and, with the commit, U_k^T = W^T K^T (phi of the block's keys)
+//   PV   D  = P' V                    (P' = w e^(s - sigma), bf16)
+//   R+   D += phi+'(Q) S+             (tf32, A operand in Tensor Memory)
+//   R-   D += phi-'(Q) S-
+//   dS   dS^T = V^T phi(K)^T per feature half (commit; bf16)
+// and the math warps compute the row statistics, phi(Q) and P' between g1
+// and PV, and out = D / den afterwards.  Merge: with sigma the log of the
+// larger branch mass, phi' = phi e^-sigma and P' = w e^(s - sigma), so
+// D / den = (w sm_num + lin_num) / (w sm_den + lin_den) exactly, with
+// den = e^(log lin_den - sigma) + e^(log(w sm_den) - sigma) in [1, 2].
+//
+// Overlap between units (step only): Tensor Memory holds two unit slots of
+// 256 columns, [phi | D] each, so the next unit's g1 runs between this unit's
+// R+ and R-.  A unit's phi+ and phi- share its F phi columns: phi- is held in
+// registers until R+ has consumed phi+.  With the commit the phi columns hold
+// both halves ([0, 2F)) and dS^T of the two halves reuses the phi+ columns and
+// the idle output accumulator; units then follow one another on the tensor
+// cores, the math of one overlapping the MMAs of the other.
 //
 // MMA cost note: on this part a tcgen05.mma with M = 128 costs about the same
 // time for any N up to 128-256, so contractions are shaped for few, wide
-// instructions (dS^T as two N = F products rather than per-tile N = 32 ones).
+// instructions (the scores ride along with U; dS^T is two N = F products).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -56,58 +65,60 @@ using bf16 = __nv_bfloat16;
 constexpr int kWarps = 12;
 constexpr int kThreads = kWarps * 32;
 constexpr int kMathThreads = 256;
-constexpr uint32_t kColA = 0, kColD0 = 256;
 constexpr int kMaxSlots = 16;
 constexpr uint64_t kWaitNs = 1000000000ull;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kSmemLimit = 232448;
 constexpr int kOneCtaPerSm = 118 * 1024;
-constexpr uint32_t kBarMath = 1;
+constexpr uint32_t kBarMath = 1;      // named barrier over the 256 math threads
+constexpr uint32_t kBarPair = 2;      // 2..5: the two math warps of one TMEM lane quarter
+constexpr uint32_t kStatBytes = 14 * 1024;
 
 struct FusedArgs {
-    CUtensorMap tmQ, tmK, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], K and V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
-    const bf16 *Q, *K, *V, *W;
+    CUtensorMap tmQ, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
+    const bf16 *K;
     const float *alpha;
     void *const *states;
-    bf16 *O;
     unsigned *err;
     int n_units, B, Hq, Hkv, G, d, F, NS;
     float scale;
-    uint32_t off_q, off_w, off_k, off_vb, off_p, off_z, off_st, off_bar;
+    uint32_t off_q, off_wk, off_vb, off_p, off_pk, off_z, off_st, off_bar;
 };
 
-// Shared memory: [ring NS x d*128][X: Q | W | K][Vb][P][z x2][stats][barriers].
-// With the commit, V^T (128 x 32 f32) and phi(K)^T (2F x 32 f32) reuse region X
-// after the unit's first MMA group has consumed Q, W and K.  Q, K, V and W land
-// by TMA with the 128-byte swizzle: Q as two 64-column atoms of 128 rows
-// (16 KB apart), K as two atoms of B rows, V as two 64-column atoms of B rows
-// (MN-major B operand: j-groups 1 KB apart, atoms B*128 apart), W as F/64
-// atoms of d rows (MN-major: e-groups 1 KB apart, atoms d*128 apart).
+// Shared memory: [ring NS x d*128][Q][W | K^T][V][P'][phi(K) (commit)][z x2][stats][barriers].
+// Q, V and W land by TMA with the 128-byte swizzle: Q as d/64 atoms of 128 rows
+// (16 KB apart; rows t*G + h), V as d/64 atoms of B rows (MN-major operand:
+// 8-row groups 1 KB apart, atoms B*128 apart), W as F/64 atoms of d rows
+// (MN-major: e-groups 1 KB apart, atoms d*128 apart) followed by the K^T atom
+// (row e holds K[0..B)[e]), so that [W | K^T] is one MN-major B operand.
 struct FLayout {
-    uint32_t off_q, off_w, off_k, off_vb, off_p, off_z, off_st, off_bar, bytes;
+    uint32_t off_q, off_wk, off_vb, off_p, off_pk, off_z, off_st, off_bar, bytes;
     int NS;
 };
 
-FLayout make_flayout(int d, int F, int B)
+FLayout make_flayout(int d, int F, int B, bool commit)
 {
     FLayout L{};
     const uint32_t chunk = (uint32_t)d * 128;
     const uint32_t zb = (((uint32_t)2 * F * 4) + 1023) & ~1023u;
-    const uint32_t q = (uint32_t)d * 256, w = (uint32_t)d * (F < 128 ? 128 : F) * 2, k = (uint32_t)B * d * 2,
-                   vb = (uint32_t)B * d * 2, p = 128u * B * 2;
-    const uint32_t st = 16 * 1024, bar = 1024;
-    const uint32_t fixed = q + w + k + vb + p + 2 * zb + st + bar + 1024;
+    const uint32_t q = (uint32_t)d * 256;
+    const uint32_t wk = (uint32_t)(F / 64 + 1) * d * 128;
+    const uint32_t vb = (((uint32_t)B * d * 2) + 1023) & ~1023u;
+    const uint32_t p = (((uint32_t)128 * B * 2) + 1023) & ~1023u;
+    const uint32_t pk = commit ? ((((uint32_t)(2 * F / 64) * B * 128) + 1023) & ~1023u) : 0u;
+    const uint32_t bar = 1024;
+    const uint32_t fixed = q + wk + vb + p + pk + 2 * zb + kStatBytes + bar + 1024;
     int ns = ((int)kSmemLimit - (int)fixed) / (int)chunk;
     if (ns > kMaxSlots) ns = kMaxSlots;
     L.NS = ns;
     uint32_t off = (uint32_t)(ns > 0 ? ns : 0) * chunk;
     L.off_q = off; off += q;
-    L.off_w = off; off += w;
-    L.off_k = off; off += k;
+    L.off_wk = off; off += wk;
     L.off_vb = off; off += vb;
     L.off_p = off; off += p;
+    L.off_pk = off; off += pk;
     L.off_z = off; off += 2 * zb;
-    L.off_st = off; off += st;
+    L.off_st = off; off += kStatBytes;
     L.off_bar = off; off += bar;
     L.bytes = off + 1024;
     if ((int)L.bytes < kOneCtaPerSm) L.bytes = kOneCtaPerSm;
@@ -142,8 +153,8 @@ __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, volatil
     }
 }
 
-// Barrier over one warp group that also ORs a failure flag across it, so that
-// every thread of the group takes the same branch afterwards.
+// Barrier over a group of warps that also ORs a failure flag across it, so
+// that every thread of the group takes the same branch afterwards.
 __device__ __forceinline__ bool group_sync_failed(uint32_t id, uint32_t nthreads, bool local_fail)
 {
     uint32_t r;
@@ -157,11 +168,6 @@ __device__ __forceinline__ bool group_sync_failed(uint32_t id, uint32_t nthreads
         : "memory");
     return r != 0;
 }
-__device__ __forceinline__ bool math_sync_failed(bool local_fail)
-{
-    return group_sync_failed(kBarMath, kMathThreads, local_fail);
-}
-
 
 // Reduce 16 per-lane values across the 32 lanes of a warp (op = add / max /
 // min) by halving the set each step; on return lane L holds the total of
@@ -212,25 +218,50 @@ __device__ __forceinline__ float *unit_state(const FusedArgs &a, int u)
     return st + (size_t)g * head_floats(a.d, a.F);
 }
 
-// TMA of unit (r, g)'s Q, W, K into region X (one thread), completing on bar.
-__device__ __forceinline__ void tma_x(const FusedArgs &a, uint8_t *smem, int r, int g, uint64_t *bar)
+// Transposed key tile of a unit into the K^T atom (one warp): row e holds
+// K[t][e] for t < B, 128-byte swizzled like the W atoms before it.  Lane =
+// (token pair, parity of the 8-dim group), so each store instruction writes
+// 16 consecutive words of one row.  The loads are issued first (kt_load, into
+// registers, before the region is free) and the stores later (kt_store).
+struct KtRegs {
+    uint4 r0[8], r1[8];
+};
+__device__ __forceinline__ void kt_load(const FusedArgs &a, KtRegs &k, int r, int g, int lane)
 {
-    using namespace ptx;
-    const int d = a.d, F = a.F, B = a.B, G = a.G;
-    const uint32_t bytes = (uint32_t)(d / 64) * (G * B * 128) + (uint32_t)(F / 64) * (d * 128) + (uint32_t)(d / 64) * (B * 128);
-    mbar_arrive_expect_tx(bar, bytes);
-    for (int e = 0; e < d / 64; ++e) {
-        tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, bar);
-        tma_load_3d(smem + a.off_k + e * (B * 128), &a.tmK, 64 * e, g, r * B, bar);
-    }
-    for (int f = 0; f < F / 64; ++f) tma_load_2d(smem + a.off_w + f * (d * 128), &a.tmW, 64 * f, g * d, bar);
-}
-__device__ __forceinline__ void tma_v(const FusedArgs &a, uint8_t *smem, int r, int g, uint64_t *bar)
-{
-    using namespace ptx;
     const int d = a.d, B = a.B;
-    mbar_arrive_expect_tx(bar, (uint32_t)(d / 64) * (B * 128));
-    for (int e = 0; e < d / 64; ++e) tma_load_3d(smem + a.off_vb + e * (B * 128), &a.tmV, 64 * e, g, r * B, bar);
+    const int tp = lane & 15, eh = lane >> 4;
+    if (2 * tp >= B) return;
+    const size_t tstride = (size_t)a.Hkv * d;
+    const uint4 *k0 = reinterpret_cast<const uint4 *>(a.K + ((size_t)r * B * a.Hkv + g) * d + (size_t)(2 * tp) * tstride);
+    const uint4 *k1 = reinterpret_cast<const uint4 *>(reinterpret_cast<const bf16 *>(k0) + tstride);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const int ec = eh + 2 * i;
+        if (ec < d / 8) {
+            k.r0[i] = __ldg(k0 + ec);
+            k.r1[i] = __ldg(k1 + ec);
+        }
+    }
+}
+__device__ __forceinline__ void kt_store(const FusedArgs &a, const KtRegs &k, uint8_t *kt, int lane)
+{
+    const int d = a.d, B = a.B;
+    const int tp = lane & 15, eh = lane >> 4;
+    if (2 * tp >= B) return;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const int ec = eh + 2 * i;
+        if (ec >= d / 8) break;
+        const uint32_t w0[4] = {k.r0[i].x, k.r0[i].y, k.r0[i].z, k.r0[i].w};
+        const uint32_t w1[4] = {k.r1[i].x, k.r1[i].y, k.r1[i].z, k.r1[i].w};
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const uint32_t lo = (w0[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
+            const uint32_t hi = (w1[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
+            const int e = 8 * ec + j;
+            *reinterpret_cast<uint32_t *>(kt + e * 128 + ((((tp >> 2) ^ (e & 7))) << 4) + (tp & 3) * 4) = lo | (hi << 16);
+        }
+    }
 }
 
 template <bool kCommit>
@@ -241,9 +272,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int d = a.d, F = a.F, B = a.B, G = a.G, NS = a.NS;
-    const int NC = (2 * F) / 32;
-    // with the commit, the output tile is staged in the slots of tiles ocm, ocm + 1
-    const int ocm = NC > NS ? NC - NS : 0;
+    const int NCH = F / 32;          // 32-feature chunks (state tiles) per half of phi
+    const int NC = 2 * NCH;          // state tiles per unit
+    // the output tile is staged in the slots of tiles ocm, ocm + 1 of its unit:
+    // with the commit, first-half tiles that no later tile of the unit reuses;
+    // without, the last two
+    const int ocm = kCommit ? (NC > NS ? NC - NS : 0) : NC - 2;
     const uint32_t chunk_bytes = (uint32_t)d * 128;
     const int per = a.n_units / (int)gridDim.x, rem = a.n_units % (int)gridDim.x;
     const int u_begin = (int)blockIdx.x * per + min((int)blockIdx.x, rem);
@@ -252,35 +286,44 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + a.off_bar);
     uint64_t *full = bars;
     uint64_t *empty = full + NS;
-    uint64_t *zfull = empty + NS;
-    uint64_t *zempty = zfull + 2;
-    uint64_t *dready = zempty + 2;   // [2]
-    uint64_t *dfree = dready + 2;    // [2]
-    uint64_t *hread = dfree + 2;     // [2]
-    uint64_t *dsready = hread + 2;   // [2]
-    uint64_t *xfull = dsready + 2;
+    uint64_t *zfull = empty + NS;     // [2]
+    uint64_t *zempty = zfull + 2;     // [2]
+    uint64_t *dready = zempty + 2;    // [2] MMA -> math: the unit's output accumulator is complete
+    uint64_t *dfree = dready + 2;     // [2] math -> MMA: the output accumulator has been read
+    uint64_t *dsready = dfree + 2;    // [2] MMA -> math: dS^T of a feature half is in Tensor Memory
+    uint64_t *tready = dsready + 2;   // [2] math -> storer: a feature half of the tiles is updated
+    uint64_t *xfull = tready + 2;     // Q, W (TMA) and K^T (producer warp) are in place
     uint64_t *xfree = xfull + 1;
     uint64_t *vfull = xfree + 1;
     uint64_t *vfree = vfull + 1;
-    uint64_t *vtready = vfree + 1;
-    uint64_t *uready = vtready + 1;
-    uint64_t *phiready = uready + 1;
-    uint64_t *efree = phiready + 1;
-    uint64_t *rdone = efree + 1;
-    uint64_t *mmadone = rdone + 1;
-    uint64_t *tready = mmadone + 1;  // [2] math -> storer: a feature half of the tiles is updated
-    uint64_t *zdone = tready + 2;    // math -> storer: z is updated
-    uint64_t *ofree = zdone + 1;     // the last two slots of the unit may take the output tile
-    uint64_t *ostaged = ofree + 1;   // math -> storer: the output tile is in the slots
-    const int n_bars = 2 * NS + 14 + 15;
+    uint64_t *uready = vfree + 1;     // MMA -> math: g1 done
+    uint64_t *phip = uready + 1;      // math -> MMA: phi+ (with the commit: all of phi, phi(K)) and P'
+    uint64_t *phim = phip + 1;        // math -> MMA: phi- (step only)
+    uint64_t *pread = phim + 1;       // MMA -> math: R+ has consumed phi+ (step only)
+    uint64_t *efree = pread + 1;      // math -> MMA: dS^T has been consumed (commit)
+    uint64_t *zdone = efree + 1;      // math -> storer: z is updated (commit)
+    uint64_t *ofree = zdone + 1;      // storer -> math: the output slots may be written (commit)
+    uint64_t *ostaged = ofree + 1;    // math -> storer: the output tile is in its slots
+    uint64_t *mmadone = ostaged + 1;
+    const int n_bars = 2 * NS + 12 + 13;
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + n_bars);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
     if (tid == 0) {
-        for (int i = 0; i < n_bars; ++i) {
-            uint64_t *b = &bars[i];
-            const uint32_t cnt = b == vtready ? 2u : 1u;
-            mbar_init(b, cnt);
+        for (int i = 0; i < n_bars; ++i) mbar_init(&bars[i], 1);
+        mbar_init(xfull, 2);
+        mbar_init(phip, 8);
+        mbar_init(phim, 8);
+        mbar_init(efree, 8);
+        mbar_init(zdone, 8);
+        mbar_init(ostaged, 8);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&dfree[i], 8);
+            mbar_init(&tready[i], 8);
+        }
+        if (!kCommit) {
+            mbar_init(&zempty[0], 8);
+            mbar_init(&zempty[1], 8);
         }
         *fail = 0;
         fence_mbar_init();
@@ -295,8 +338,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint8_t *ring = smem;
     float *zbuf0 = reinterpret_cast<float *>(smem + a.off_z);
     const int zstride = ((2 * F * 4 + 1023) & ~1023) / 4;
-    uint8_t *vt_s = smem + a.off_q;                     // V^T: 128 rows x 128 B (commit)
-    uint8_t *pt_s = smem + a.off_q + 128 * 128;         // phi(K)^T: 2F rows x 128 B (commit)
 
     if (warp == 0) {
         // ------------------------------------------------------- S producer
@@ -314,6 +355,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 mbar_arrive_expect_tx(&zfull[zb], 2 * F * 4);
                 bulk_g2s(zbuf0 + zb * zstride, Sg + (size_t)2 * F * d, 2 * F * 4, &zfull[zb]);
                 ++issued_z[zb];
+                // at start-up every SM asks for its first unit at once: let Q, W and K
+                // (needed first) arrive before the state tiles (needed after g1 and phi)
+                if (kp == 0 && !wait_bar(xfull, 0, fail)) break;
                 for (int c = 0; c < NC; ++c, ++q) {
                     const int slot = q % NS;
                     if (!wait_bar(&empty[slot], ((q / NS) & 1u) ^ 1u, fail)) { ok = false; break; }
@@ -333,87 +377,123 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     } else if (warp == 1) {
         // ------------------------------------------------------- MMA issuer
         if (lane == 0) {
-            const uint32_t q_u = smem_u32(smem + a.off_q), w_u = smem_u32(smem + a.off_w),
-                           k_u = smem_u32(smem + a.off_k), vb_u = smem_u32(smem + a.off_vb),
-                           vt_u = smem_u32(vt_s), pt_u = smem_u32(pt_s), p_u = smem_u32(smem + a.off_p),
-                           ring_u = smem_u32(ring);
-            const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
-            const uint32_t idS = instr_desc(FMT_BF16, FMT_BF16, false, false, 128, B);
-            const uint32_t idK = instr_desc(FMT_BF16, FMT_BF16, true, false, 128, B);
+            const uint32_t q_u = smem_u32(smem + a.off_q), wk_u = smem_u32(smem + a.off_wk),
+                           vb_u = smem_u32(smem + a.off_vb), p_u = smem_u32(smem + a.off_p),
+                           pk_u = smem_u32(smem + a.off_pk), ring_u = smem_u32(ring);
+            const uint32_t kt_u = wk_u + (uint32_t)(F / 64) * d * 128;
+            const uint32_t idUS = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F + B);
+            const uint32_t idKT = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, B);
             const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
-            const uint32_t idDS = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, F);
             const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
-            uint32_t q = 0, kp = 0;
-            bool ok = true;
-            for (int u = u_begin; u < u_end && ok; ++u) {
-                if (!unit_state(a, u)) continue;
-                const uint32_t dcol = tmem + kColD0 + 128 * (kp & 1);
-                const uint32_t dother = tmem + kColD0 + 128 * ((kp + 1) & 1);
-                if (!wait_bar(xfull, kp & 1u, fail)) break;
-                if (kp > 0) {
-                    // Tensor Memory of the previous unit: phi columns (and, with the
-                    // commit, the dS^T halves) must be consumed before U is rewritten
-                    if (kCommit) { if (!wait_bar(efree, (kp - 1) & 1u, fail)) break; }
-                    else { if (!wait_bar(rdone, (kp - 1) & 1u, fail)) break; }
-                }
-                if (kp > 1 && !wait_bar(&dfree[kp & 1], ((kp - 2) >> 1) & 1u, fail)) break;
-                tc_fence_after();
-                // group 1: U = Q W, scores = Q K^T, U_k^T = W^T K^T
+            const uint32_t idDS = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, F);
+            // g1: [U | scores] at column ucol, and (commit) U_k^T at column kcol
+            auto g1 = [&](uint32_t ucol, uint32_t kcol) {
                 for (int k = 0; k < d / 16; ++k) {
                     const uint64_t aq = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
-                    const uint64_t bw = smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
-                    const uint64_t bk = smem_desc(k_u + (k >> 2) * (B * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
-                    mma_bf16_ss(tmem + kColA, aq, bw, idU, k > 0);
-                    mma_bf16_ss(dcol, aq, bk, idS, k > 0);
-                    if (kCommit) mma_bf16_ss(dcol + B, bw, bk, idK, k > 0);
-                }
-                mma_commit(uready);
-                mma_commit(xfree);
-                // group 2: readout over the state tiles, dS^T per feature half, then P V
-                if (!wait_bar(phiready, kp & 1u, fail)) break;
-                tc_fence_after();
-                for (int c = 0; c < NC; ++c, ++q) {
-                    const int slot = q % NS;
-                    if (!wait_bar(&full[slot], (q / NS) & 1u, fail)) { ok = false; break; }
-                    const uint32_t s_u = ring_u + slot * chunk_bytes;
-#pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
-                        mma_tf32_ts(dcol, tmem + kColA + 32 * c + 8 * kk, smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B),
-                                    idR, (c | kk) != 0);
-                    if (!kCommit) {
-                        if (c < NC - 2) mma_commit(&empty[slot]);
-                        else if (c == NC - 1) mma_commit(ofree);
-                    }
-                    if (kCommit && c == NC / 2 - 1) {
-                        // phi+ has been read: its columns take dS^T for features [0, F);
-                        // dS^T for [F, 2F) goes to the idle output accumulator
-                        mma_commit(&hread[0]);
-                        if (!wait_bar(&hread[0], kp & 1u, fail)) { ok = false; break; }
-                        if (!wait_bar(vtready, kp & 1u, fail)) { ok = false; break; }
-                        if (kp > 0 && !wait_bar(&dfree[(kp + 1) & 1], ((kp - 1) >> 1) & 1u, fail)) { ok = false; break; }
-                        tc_fence_after();
-#pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-#pragma unroll
-                            for (int kk = 0; kk < 4; ++kk)
-                                mma_tf32_ss(h == 0 ? tmem + kColA : dother, smem_desc(vt_u + 32 * kk, 16, 1024, SWZ_128B),
-                                            smem_desc(pt_u + h * F * 128 + 32 * kk, 16, 1024, SWZ_128B), idDS, kk != 0);
-                            mma_commit(&dsready[h]);
-                        }
+                    const uint64_t bwk = smem_desc(wk_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
+                    mma_bf16_ss(tmem + ucol, aq, bwk, idUS, k > 0);
+                    if (kCommit) {
+                        const uint64_t bkt = smem_desc(kt_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
+                        mma_bf16_ss(tmem + kcol, bwk, bkt, idKT, k > 0);
                     }
                 }
-                if (!ok) break;
-                mma_commit(rdone);
-                if (!wait_bar(vfull, kp & 1u, fail)) break;
-                tc_fence_after();
+            };
+            auto pv = [&](uint32_t dcol) {
                 for (int k = 0; k < B / 16; ++k) {
                     const uint64_t ap = smem_desc(p_u + k * 256, 128, (B / 8) * 128, SWZ_NONE);
                     const uint64_t bv = smem_desc(vb_u + 2 * k * 1024, B * 128, 1024, SWZ_128B);
-                    mma_bf16_ss(dcol, ap, bv, idP, 1);
+                    mma_bf16_ss(tmem + dcol, ap, bv, idP, k > 0);
                 }
-                mma_commit(&dready[kp & 1]);
-                mma_commit(vfree);
-                ++kp;
+            };
+            // readout of state tile c (global tile counter qt + c) with phi columns acol
+            auto readout = [&](uint32_t dcol, uint32_t acol, uint32_t qc) -> int {
+                const int slot = qc % NS;
+                if (!wait_bar(&full[slot], (qc / NS) & 1u, fail)) return -1;
+                tc_fence_after();
+                const uint32_t s_u = ring_u + slot * chunk_bytes;
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)
+                    mma_tf32_ts(tmem + dcol, tmem + acol + 8 * kk, smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B), idR, 1);
+                return slot;
+            };
+            auto ds = [&](uint32_t dcol, int h) {
+                for (int ks = 0; ks < B / 16; ++ks) {
+                    const uint64_t av = smem_desc(vb_u + ks * 2048, B * 128, 1024, SWZ_128B);
+                    const uint64_t bp = smem_desc(pk_u + (uint32_t)h * (F / 64) * (B * 128) + ks * 2048, B * 128, 1024,
+                                                  SWZ_128B);
+                    mma_bf16_ss(tmem + dcol, av, bp, idDS, ks > 0);
+                }
+            };
+            uint32_t kp = 0, qt = 0, prev_qt = 0;
+            bool ok = true;
+            if (!kCommit) {
+                // R- of the previous unit: its phi- sits in the phi columns R+ has consumed
+                auto tail = [&](uint32_t ik, uint32_t iq) -> bool {
+                    const uint32_t T = (ik & 1) * 256;
+                    if (!wait_bar(phim, ik & 1u, fail)) return false;
+                    tc_fence_after();
+                    for (int c = NCH; c < NC; ++c) {
+                        const int slot = readout(T + 128, T + 32 * (c - NCH), iq + c);
+                        if (slot < 0) return false;
+                        if (c < ocm) mma_commit(&empty[slot]);
+                    }
+                    mma_commit(&dready[ik & 1]);
+                    return true;
+                };
+                for (int u = u_begin; u < u_end; ++u) {
+                    if (!unit_state(a, u)) continue;
+                    const uint32_t T = (kp & 1) * 256;
+                    if (!wait_bar(xfull, kp & 1u, fail)) { ok = false; break; }
+                    if (kp >= 2 && !wait_bar(&dfree[kp & 1], ((kp - 2) >> 1) & 1u, fail)) { ok = false; break; }
+                    tc_fence_after();
+                    g1(T, 0);
+                    mma_commit(uready);
+                    mma_commit(xfree);
+                    if (kp >= 1 && !tail(kp - 1, prev_qt)) { ok = false; break; }
+                    if (!wait_bar(phip, kp & 1u, fail) || !wait_bar(vfull, kp & 1u, fail)) { ok = false; break; }
+                    tc_fence_after();
+                    pv(T + 128);
+                    mma_commit(vfree);
+                    for (int c = 0; c < NCH; ++c) {
+                        const int slot = readout(T + 128, T + 32 * c, qt + c);
+                        if (slot < 0) { ok = false; break; }
+                        mma_commit(&empty[slot]);
+                    }
+                    if (!ok) break;
+                    mma_commit(pread);
+                    prev_qt = qt;
+                    qt += NC;
+                    ++kp;
+                }
+                if (ok && kp >= 1) tail(kp - 1, prev_qt);
+            } else {
+                for (int u = u_begin; u < u_end; ++u) {
+                    if (!unit_state(a, u)) continue;
+                    const uint32_t D = 256 + 128 * (kp & 1), Do = 256 + 128 * ((kp + 1) & 1);
+                    if (!wait_bar(xfull, kp & 1u, fail)) { ok = false; break; }
+                    if (kp >= 1 && !wait_bar(efree, (kp - 1) & 1u, fail)) { ok = false; break; }
+                    if (kp >= 2 && !wait_bar(&dfree[kp & 1], ((kp - 2) >> 1) & 1u, fail)) { ok = false; break; }
+                    tc_fence_after();
+                    g1(0, D);
+                    mma_commit(uready);
+                    mma_commit(xfree);
+                    // phip also covers phi-, phi(K) and the previous unit's epilogue
+                    if (!wait_bar(phip, kp & 1u, fail) || !wait_bar(vfull, kp & 1u, fail)) { ok = false; break; }
+                    tc_fence_after();
+                    pv(D);
+                    for (int c = 0; c < NCH && ok; ++c) ok = readout(D, 32 * c, qt + c) >= 0;
+                    if (!ok) break;
+                    ds(0, 0);   // dS^T of phi+ features into the phi+ columns R+ has consumed
+                    mma_commit(&dsready[0]);
+                    for (int c = NCH; c < NC && ok; ++c) ok = readout(D, F + 32 * (c - NCH), qt + c) >= 0;
+                    if (!ok) break;
+                    ds(Do, 1);  // dS^T of phi- features into the idle output accumulator
+                    mma_commit(&dsready[1]);
+                    mma_commit(&dready[kp & 1]);
+                    mma_commit(vfree);
+                    qt += NC;
+                    ++kp;
+                }
             }
             mma_commit(mmadone);
             mbar_wait(mmadone, 0, kWaitNs);
@@ -421,47 +501,43 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     } else if (warp == 2) {
         // ------------------------------------------------------------- producer
         uint32_t kp = 0;
+        int nx = 0, nv = 0;
+        const uint32_t xbytes = (uint32_t)(d / 64) * (G * B * 128) + (uint32_t)(F / 64) * (d * 128);
+        uint8_t *kt = smem + a.off_wk + (F / 64) * d * 128;
         for (int u = u_begin; u < u_end; ++u) {
             if (!unit_state(a, u)) continue;
             const int r = u / a.Hkv, g = u % a.Hkv;
+            KtRegs kr;
+            kt_load(a, kr, r, g, lane);   // in flight while the region drains
             bool ok = true;
-            if (kp > 0) {
-                // region X is free once the previous unit's last use of it has completed
-                ok = kCommit ? wait_bar(&dsready[1], (kp - 1) & 1u, fail) : wait_bar(xfree, (kp - 1) & 1u, fail);
-            }
+            if (kp > 0) ok = wait_bar(xfree, (kp - 1) & 1u, fail);
             if (__any_sync(0xffffffffu, !ok)) break;
-            if (lane == 0) tma_x(a, smem, r, g, xfull);
+            if (lane == 0) {
+                mbar_arrive_expect_tx(xfull, xbytes);
+                for (int e = 0; e < d / 64; ++e)
+                    tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xfull);
+                for (int f = 0; f < F / 64; ++f)
+                    tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xfull);
+            }
+            kt_store(a, kr, kt, lane);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(xfull);
+            ++nx;
             if (kp > 0) ok = wait_bar(vfree, (kp - 1) & 1u, fail);
             if (__any_sync(0xffffffffu, !ok)) break;
-            if (lane == 0) tma_v(a, smem, r, g, vfull);
-            if (kCommit) {
-                // V^T in f32 into region X once this unit's first MMA group is done with it
-                ok = wait_bar(xfree, kp & 1u, fail);
-                if (__any_sync(0xffffffffu, !ok)) break;
-                for (int idx = lane; idx < 16 * 32; idx += 32) {
-                    const int eg = idx >> 5, t = idx & 31;     // 8 rows e = 8*eg .. 8*eg+7, column t
-                    float v[8];
-                    if (eg * 8 < d) {
-                        const uint4 raw = *reinterpret_cast<const uint4 *>(
-                            a.V + (((size_t)r * B + t) * a.Hkv + g) * d + 8 * eg);
-                        const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) { v[2 * i] = __low2float(b2[i]); v[2 * i + 1] = __high2float(b2[i]); }
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) v[i] = 0.f;
-                    }
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const int e = 8 * eg + i;
-                        *(reinterpret_cast<float *>(vt_s + e * 128 + ((((t >> 2) ^ (e & 7))) << 4)) + (t & 3)) = v[i];
-                    }
-                }
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(vtready);
+            if (lane == 0) {
+                mbar_arrive_expect_tx(vfull, (uint32_t)(d / 64) * (B * 128));
+                for (int e = 0; e < d / 64; ++e)
+                    tma_load_3d(smem + a.off_vb + e * (B * 128), &a.tmV, 64 * e, g, r * B, vfull);
             }
+            ++nv;
             ++kp;
+        }
+        if (lane == 0 && *fail) {
+            // let copies in flight land before the CTA exits
+            if (nx) mbar_wait(xfull, (uint32_t)(nx - 1) & 1u, kWaitNs);
+            if (nv) mbar_wait(vfull, (uint32_t)(nv - 1) & 1u, kWaitNs);
         }
     } else if (warp == 3) {
         // --------------------------------------------------------------- storer
@@ -481,24 +557,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     mbar_arrive(&zempty[zb]);
                     for (int h = 0; h < 2 && ok; ++h) {
                         if (!wait_bar(&tready[h], kp & 1u, fail)) { ok = false; break; }
-                        for (int c = h * NC / 2; c < (h + 1) * NC / 2; ++c)
+                        for (int c = h * NCH; c < (h + 1) * NCH; ++c)
                             bulk_s2g(Sg + (size_t)c * 32 * d, ring + (size_t)((q + c) % NS) * chunk_bytes, chunk_bytes);
                         bulk_commit();
                         bulk_wait_read_all();
-                        // with the commit, two slots of the first half are held for the
-                        // output tile: tiles oc and oc + 1, whose slots no later tile of
-                        // this unit reuses
-                        for (int c = h * NC / 2; c < (h + 1) * NC / 2; ++c)
-                            if (h == 1 || c < ocm || c > ocm + 1) mbar_arrive(&empty[(q + c) % NS]);
+                        for (int c = h * NCH; c < (h + 1) * NCH; ++c)
+                            if (c < ocm || c > ocm + 1) mbar_arrive(&empty[(q + c) % NS]);
                         if (h == 0) mbar_arrive(ofree);
                     }
                     if (!ok) break;
                 }
                 // output tile: two TMA boxes from the two held-back slots
                 if (!wait_bar(ostaged, kp & 1u, fail)) break;
-                const int oc = kCommit ? ocm : NC - 2;   // first of the two slots holding the output
-                uint8_t *s0 = ring + (size_t)((q + oc) % NS) * chunk_bytes;
-                uint8_t *s1 = ring + (size_t)((q + oc + 1) % NS) * chunk_bytes;
+                uint8_t *s0 = ring + (size_t)((q + ocm) % NS) * chunk_bytes;
+                uint8_t *s1 = ring + (size_t)((q + ocm + 1) % NS) * chunk_bytes;
                 if (d == 128) {
                     tma_store_3d(&a.tmO, 0, g * G, r * B, s0);
                     tma_store_3d(&a.tmO, 64, g * G, r * B, s1);
@@ -508,8 +580,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 }
                 bulk_commit();
                 bulk_wait_read_all();
-                mbar_arrive(&empty[(q + oc) % NS]);
-                mbar_arrive(&empty[(q + oc + 1) % NS]);
+                mbar_arrive(&empty[(q + ocm) % NS]);
+                mbar_arrive(&empty[(q + ocm + 1) % NS]);
                 q += NC;
                 ++kp;
             }
@@ -518,19 +590,69 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     } else {
         // ------------------------------------------------------------- math
         const int mt = tid - 128;
-        const int q4 = warp & 3, half = (warp - 4) >> 2;
+        const int q4 = warp & 3, part = (warp - 4) >> 2;
         const int row = 32 * q4 + lane;
         const uint32_t lane_off = (uint32_t)(32 * q4) << 16;
-        const int nsc = B / 16, nfc = F / 32;
+        const bool two = NCH >= 4;          // a part owns chunks part and part + 2 of each half
+        const bool has_sc = part < B / 16;  // score columns [16 part, 16 part + 16)
         const int Mv = G * B;
         const bool valid = row < Mv;
         const bool fval = row < F;
-        float *ex = reinterpret_cast<float *>(smem + a.off_st);   // [8 slots][2 halves][128 rows]
-        float *den_s = ex + 8 * 256;                                // [2][128]
-        float *tk = den_s + 256;                                    // token stats (commit) [8][32][4]
+        float *xa = reinterpret_cast<float *>(smem + a.off_st);   // [part][ms, mx, mn][128]
+        float *xb = xa + 6 * 128;                                  // [part][l, sp, sn, lp, ln][128]
+        float *tk = xb + 10 * 128;                                 // token statistics (commit)
+        uint8_t *pkb = smem + a.off_pk;
         const float scale_l2 = a.scale * kLog2e;
         const int tok = reduce16_token(lane);
-        uint32_t q = 0, kp = 0;
+        const uint32_t pair_bar = kBarPair + q4;
+        // one exchange point: pair barrier for the step, all math warps with the commit
+        auto sync_failed = [&](bool local_fail) -> bool {
+            return kCommit ? group_sync_failed(kBarMath, kMathThreads, local_fail)
+                           : group_sync_failed(pair_bar, 64, local_fail);
+        };
+
+        // out = D / den, staged as the TMA box image in the unit's held-back ring
+        // slots (row i = t*G + hh, 128-byte swizzle)
+        auto epilogue = [&](uint32_t ek, uint32_t eq, float inv) -> bool {
+            const uint32_t dcol = kCommit ? 256 + 128 * (ek & 1) : (ek & 1) * 256 + 128;
+            bool ok = wait_bar(&dready[ek & 1], (ek >> 1) & 1u, fail);
+            if (kCommit && ok) ok = wait_bar(ofree, ek & 1u, fail);
+            tc_fence_after();
+            const int dh = d / 2;
+            // d = 128: column half -> slot; d = 64: token half -> slot (one 64-column atom)
+            const int rows_half = G * B / 2;
+            const int sidx = d == 128 ? part : (row >= rows_half ? 1 : 0);
+            const int srow = d == 128 ? row : row - sidx * rows_half;
+            uint8_t *base = ring + (size_t)((eq + ocm + sidx) % NS) * chunk_bytes + srow * 128;
+            for (int hc = 0; hc < dh / 32; ++hc) {
+                float v[32];
+                tmem_ld32(tmem + dcol + lane_off + part * dh + 32 * hc, v);
+                tmem_wait_ld();
+                if (ok && valid) {
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int i = 0; i < 32; i += 2) pk[i / 2] = pack_bf16x2(v[i] * inv, v[i + 1] * inv);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const int gi = 4 * hc + i + (d == 128 ? 0 : 4 * part);   // 16-byte granule in the row
+                        *reinterpret_cast<uint4 *>(base + ((gi ^ (srow & 7)) << 4)) =
+                            make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                    }
+                }
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0 && ok) {
+                mbar_arrive(ostaged);
+                mbar_arrive(&dfree[ek & 1]);
+            }
+            return ok;
+        };
+
+        uint32_t q = 0, kp = 0, prev_q = 0;
+        float prev_inv = 0.f;   // 1 / den of the unit whose output is still pending (step)
+        bool ok = true;
         for (int u = u_begin; u < u_end; ++u) {
             float *Sg = unit_state(a, u);
             if (!Sg) {
@@ -539,48 +661,53 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             }
             const int g = u % a.Hkv;
             const int zb = kp & 1;
-            // gate of this row's query head, loaded now so the latency overlaps the first rounds
+            // gate of this row's query head, loaded now so the latency overlaps the first phase
             const float alpha_row = valid ? a.alpha[g * G + row % G] : 0.f;
             float *zs = zbuf0 + zb * zstride;
-            const uint32_t dcol = tmem + kColD0 + 128 * (kp & 1);
-            float *den = den_s + 128 * (kp & 1);
-            bool ok = wait_bar(uready, kp & 1u, fail);
-            tc_fence_after();
+            const uint32_t T = kCommit ? 0u : (kp & 1) * 256;
+            const uint32_t pcol = tmem + T + lane_off;                         // phi+ (and U)
+            const uint32_t mcol = tmem + (kCommit ? (uint32_t)F : T) + lane_off;   // phi-
+            const uint32_t scol = tmem + T + F + lane_off;                     // scores
+            const uint32_t kcol = tmem + 256 + 128 * (kp & 1) + lane_off;      // U_k^T (commit)
 
-            // ---- round 1: row extrema; per-token extrema of U_k^T (features on lanes)
-            {
-                float ms = -INFINITY, mx = -INFINITY, mn = INFINITY;
-                for (int k = half; k < nsc; k += 2) {
-                    float v[16];
-                    tmem_ld16(dcol + lane_off + 16 * k, v);
-                    tmem_wait_ld();
+            // ---- phase A: row extrema of U and of the scores (U kept in registers)
+            bool bad = !wait_bar(uready, kp & 1u, fail);
+            tc_fence_after();
+            float sc[16], u0[32], u1[32], uk[16];
+            if (kCommit) {
+                // per-token extrema of U_k^T over this warp's 32 features (features on lanes)
+                tmem_ld16(kcol + 16 * part, uk);
+                tmem_wait_ld();
+                float vmx[16], vmn[16];
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) ms = fmaxf(ms, v[i]);
-                }
-                for (int k = half; k < nfc; k += 2) {
-                    float v[32];
-                    tmem_ld32(tmem + lane_off + kColA + 32 * k, v);
-                    tmem_wait_ld();
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, v[i]); mn = fminf(mn, v[i]); }
-                }
-                ex[(0 * 2 + half) * 128 + row] = ms;
-                ex[(1 * 2 + half) * 128 + row] = mx;
-                ex[(2 * 2 + half) * 128 + row] = mn;
-                if (kCommit) {
-                    float uk[16], vmx[16], vmn[16];
-                    tmem_ld16(dcol + B + lane_off + 16 * half, uk);
-                    tmem_wait_ld();
-#pragma unroll
-                    for (int t = 0; t < 16; ++t) { vmx[t] = fval ? uk[t] : -INFINITY; vmn[t] = fval ? uk[t] : INFINITY; }
-                    const float rmx = warp_reduce16<1>(vmx, lane), rmn = warp_reduce16<2>(vmn, lane);
-                    if (!(lane & 1)) {
-                        tk[(0 * 32 + 16 * half + tok) * 4 + q4] = rmx;
-                        tk[(1 * 32 + 16 * half + tok) * 4 + q4] = rmn;
-                    }
+                for (int t = 0; t < 16; ++t) { vmx[t] = fval ? uk[t] : -INFINITY; vmn[t] = fval ? uk[t] : INFINITY; }
+                const float rmx = warp_reduce16<1>(vmx, lane), rmn = warp_reduce16<2>(vmn, lane);
+                if (!(lane & 1)) {
+                    tk[(0 * 32 + 16 * part + tok) * 4 + q4] = rmx;
+                    tk[(1 * 32 + 16 * part + tok) * 4 + q4] = rmn;
                 }
             }
-            if (math_sync_failed(!ok)) break;
+            if (has_sc) tmem_ld16(scol + 16 * part, sc);
+            tmem_ld32(pcol + 32 * part, u0);
+            if (two) tmem_ld32(pcol + 32 * (part + 2), u1);
+            tmem_wait_ld();
+            {
+                float ms = -INFINITY, mx = -INFINITY, mn = INFINITY;
+                if (has_sc) {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) ms = fmaxf(ms, sc[i]);
+                }
+#pragma unroll
+                for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, u0[i]); mn = fminf(mn, u0[i]); }
+                if (two) {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, u1[i]); mn = fminf(mn, u1[i]); }
+                }
+                xa[(part * 3 + 0) * 128 + row] = ms;
+                xa[(part * 3 + 1) * 128 + row] = mx;
+                xa[(part * 3 + 2) * 128 + row] = mn;
+            }
+            if (sync_failed(bad)) { ok = false; break; }
             if (kCommit) {
                 if (mt < 64) {   // combine the four feature quarters per token
                     const int t = mt & 31, s = mt >> 5;
@@ -588,61 +715,67 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     tk[(4 + s) * 128 + t] = s == 0 ? fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w))
                                                    : fminf(fminf(v.x, v.y), fminf(v.z, v.w));
                 }
-                if (math_sync_failed(false)) break;
+                if (sync_failed(false)) { ok = false; break; }
             }
-            ok = wait_bar(&zfull[zb], (kp >> 1) & 1u, fail);
+            const float ms = fmaxf(xa[0 * 128 + row], xa[3 * 128 + row]);
+            const float mx = fmaxf(xa[1 * 128 + row], xa[4 * 128 + row]);
+            const float mn = fminf(xa[2 * 128 + row], xa[5 * 128 + row]);
 
-            // ---- round 2: exponentials and partial sums
-            const float m_raw = fmaxf(ex[0 * 256 + row], ex[0 * 256 + 128 + row]);
+            // ---- phase B: exponentials; phi+ unnormalised into Tensor Memory, phi- kept
+            bad = !wait_bar(&zfull[zb], (kp >> 1) & 1u, fail);
+            float epk[16], enk[16];
             {
-                const float mx = fmaxf(ex[1 * 256 + row], ex[1 * 256 + 128 + row]);
-                const float mn = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]);
-                const float mxl = mx * kLog2e, mnl = mn * kLog2e, ml = m_raw * scale_l2;
+                const float mxl = mx * kLog2e, mnl = mn * kLog2e, ml = ms * scale_l2;
                 float l = 0.f, sp = 0.f, sn = 0.f, lp = 0.f, ln = 0.f;
-                for (int k = half; k < nsc; k += 2) {
-                    float v[16];
-                    tmem_ld16(dcol + lane_off + 16 * k, v);
-                    tmem_wait_ld();
+                if (has_sc) {
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) l += ex2(fmaf(v[i], scale_l2, -ml));
+                    for (int i = 0; i < 16; ++i) l += ex2(fmaf(sc[i], scale_l2, -ml));
                 }
-                for (int k = half; k < nfc; k += 2) {
-                    float uu[32], ep[32], en[32];
-                    tmem_ld32(tmem + lane_off + kColA + 32 * k, uu);
-                    tmem_wait_ld();
+                auto exps = [&](float (&uu)[32], int k) {
+                    float ep[32];
                     const float4 *zp = reinterpret_cast<const float4 *>(zs + 32 * k);
                     const float4 *zn = reinterpret_cast<const float4 *>(zs + F + 32 * k);
 #pragma unroll
                     for (int i4 = 0; i4 < 8; ++i4) {
                         const float4 a4 = zp[i4], b4 = zn[i4];
-                        const float za[4] = {a4.x, a4.y, a4.z, a4.w}, zb4[4] = {b4.x, b4.y, b4.z, b4.w};
+                        const float za[4] = {a4.x, a4.y, a4.z, a4.w}, zn4[4] = {b4.x, b4.y, b4.z, b4.w};
 #pragma unroll
                         for (int j = 0; j < 4; ++j) {
                             const int i = 4 * i4 + j;
-                            ep[i] = ex2(fmaf(uu[i], kLog2e, -mxl));
-                            en[i] = ex2(fmaf(-uu[i], kLog2e, mnl));
-                            sp += ep[i];
-                            sn += en[i];
-                            lp = fmaf(ep[i], za[j], lp);
-                            ln = fmaf(en[i], zb4[j], ln);
+                            const float e = ex2(fmaf(uu[i], kLog2e, -mxl));
+                            const float en = ex2(fmaf(-uu[i], kLog2e, mnl));
+                            ep[i] = e;
+                            uu[i] = en;
+                            sp += e;
+                            sn += en;
+                            lp = fmaf(e, za[j], lp);
+                            ln = fmaf(en, zn4[j], ln);
                         }
                     }
-                    tmem_st32(tmem + lane_off + kColA + 32 * k, ep);
-                    tmem_st32(tmem + lane_off + kColA + F + 32 * k, en);
-                }
-                ex[(3 * 2 + half) * 128 + row] = l;
-                ex[(4 * 2 + half) * 128 + row] = sp;
-                ex[(5 * 2 + half) * 128 + row] = sn;
-                ex[(6 * 2 + half) * 128 + row] = lp;
-                ex[(7 * 2 + half) * 128 + row] = ln;
+                    tmem_st32(pcol + 32 * k, ep);
+                    // with the commit phi- has its own columns (the scores there are in
+                    // registers by now): store it unnormalised as well
+                    if (kCommit) tmem_st32(mcol + 32 * k, uu);
+                };
                 if (kCommit) {
-                    // unnormalised phi(K) into the phi(K)^T tile (row f, this half's 16 token
-                    // columns), per-token partial sums over this warp's features
-                    float uk[16], ep16[16], en16[16];
-                    tmem_ld16(dcol + B + lane_off + 16 * half, uk);
+                    // U is reloaded rather than kept since phase A (register pressure)
+#pragma unroll 1
+                    for (int k = part; k < NCH; k += 2) {
+                        float uu[32];
+                        tmem_ld32(pcol + 32 * k, uu);
+                        tmem_wait_ld();
+                        exps(uu, k);
+                    }
+                } else {
+                    exps(u0, part);
+                    if (two) exps(u1, part + 2);
+                }
+                if (kCommit) {
+                    // unnormalised phi(K) of this half's 16 tokens; per-token sums over the warp's features
+                    tmem_ld16(kcol + 16 * part, uk);
                     tmem_wait_ld();
-                    const float4 *tmx = reinterpret_cast<const float4 *>(&tk[4 * 128 + 16 * half]);
-                    const float4 *tmn = reinterpret_cast<const float4 *>(&tk[5 * 128 + 16 * half]);
+                    const float4 *tmx = reinterpret_cast<const float4 *>(&tk[4 * 128 + 16 * part]);
+                    const float4 *tmn = reinterpret_cast<const float4 *>(&tk[5 * 128 + 16 * part]);
 #pragma unroll
                     for (int t4 = 0; t4 < 4; ++t4) {
                         const float4 x = tmx[t4], y = tmn[t4];
@@ -650,215 +783,195 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
 #pragma unroll
                         for (int j = 0; j < 4; ++j) {
                             const int t = 4 * t4 + j;
-                            ep16[t] = fval ? ex2((uk[t] - kx[j]) * kLog2e) : 0.f;
-                            en16[t] = fval ? ex2((kn[j] - uk[t]) * kLog2e) : 0.f;
+                            epk[t] = fval ? ex2((uk[t] - kx[j]) * kLog2e) : 0.f;
+                            enk[t] = fval ? ex2((kn[j] - uk[t]) * kLog2e) : 0.f;
                         }
                     }
-                    if (fval) {
-                        uint8_t *rp = pt_s + row * 128;
-                        uint8_t *rn = pt_s + (F + row) * 128;
+                    float sr[16];
 #pragma unroll
-                        for (int gq = 0; gq < 4; ++gq) {
-                            const int gi = 4 * half + gq;
-                            *reinterpret_cast<float4 *>(rp + ((gi ^ (row & 7)) << 4)) =
-                                make_float4(ep16[4 * gq], ep16[4 * gq + 1], ep16[4 * gq + 2], ep16[4 * gq + 3]);
-                            *reinterpret_cast<float4 *>(rn + ((gi ^ ((F + row) & 7)) << 4)) =
-                                make_float4(en16[4 * gq], en16[4 * gq + 1], en16[4 * gq + 2], en16[4 * gq + 3]);
-                        }
-                    }
-                    const float rsp = warp_reduce16<0>(ep16, lane), rsn = warp_reduce16<0>(en16, lane);
+                    for (int t = 0; t < 16; ++t) sr[t] = epk[t];
+                    const float rsp = warp_reduce16<0>(sr, lane);
+#pragma unroll
+                    for (int t = 0; t < 16; ++t) sr[t] = enk[t];
+                    const float rsn = warp_reduce16<0>(sr, lane);
                     if (!(lane & 1)) {
-                        tk[(2 * 32 + 16 * half + tok) * 4 + q4] = rsp;
-                        tk[(3 * 32 + 16 * half + tok) * 4 + q4] = rsn;
+                        tk[(2 * 32 + 16 * part + tok) * 4 + q4] = rsp;
+                        tk[(3 * 32 + 16 * part + tok) * 4 + q4] = rsn;
                     }
                 }
+                xb[(part * 5 + 0) * 128 + row] = l;
+                xb[(part * 5 + 1) * 128 + row] = sp;
+                xb[(part * 5 + 2) * 128 + row] = sn;
+                xb[(part * 5 + 3) * 128 + row] = lp;
+                xb[(part * 5 + 4) * 128 + row] = ln;
                 tmem_wait_st();
             }
-            if (math_sync_failed(!ok)) break;
+            if (!kCommit) {
+                // z has been read
+                __syncwarp();
+                if (lane == 0 && !bad) mbar_arrive(&zempty[zb]);
+            }
+            if (sync_failed(bad)) { ok = false; break; }
             if (kCommit) {
                 if (mt < 64) {   // per-token normalisers of phi(K)
                     const int t = mt & 31, s = mt >> 5;
                     const float4 v = *reinterpret_cast<const float4 *>(&tk[((2 + s) * 32 + t) * 4]);
                     tk[(6 + s) * 128 + t] = 1.f / ((v.x + v.y) + (v.z + v.w));
                 }
-                if (math_sync_failed(false)) break;
+                if (sync_failed(false)) { ok = false; break; }
             }
 
-            // ---- round 3: sigma, scaled phi(Q) in place, P', den; phi(K) normalised, z update
+            // ---- phase C: sigma, phi+ scaled in place, P', den; commit: phi-, phi(K), z
+            float cneg, inv_den;
             {
-                const float l = ex[3 * 256 + row] + ex[3 * 256 + 128 + row];
-                const float sp = ex[4 * 256 + row] + ex[4 * 256 + 128 + row];
-                const float sn = ex[5 * 256 + row] + ex[5 * 256 + 128 + row];
-                const float lp = ex[6 * 256 + row] + ex[6 * 256 + 128 + row];
-                const float ln = ex[7 * 256 + row] + ex[7 * 256 + 128 + row];
+                const float l = xb[0 * 128 + row] + xb[5 * 128 + row];
+                const float sp = xb[1 * 128 + row] + xb[6 * 128 + row];
+                const float sn = xb[2 * 128 + row] + xb[7 * 128 + row];
+                const float lp = xb[3 * 128 + row] + xb[8 * 128 + row];
+                const float ln = xb[4 * 128 + row] + xb[9 * 128 + row];
                 const float lin_den = lp / sp + ln / sn;
-                const int hh = row % G;
                 const float lw = valid ? log_sigmoid(alpha_row) : 0.f;
-                const float log_s = lw + m_raw * a.scale + logf(l);   // log(w sm_den)
-                const float log_l = logf(lin_den);                      // log(lin_den), -inf if empty
+                const float log_s = lw + ms * a.scale + logf(l);   // log(w sm_den)
+                const float log_l = logf(lin_den);                   // log(lin_den), -inf if empty
                 const float sig = fmaxf(fmaxf(log_s, log_l), -60.f);
                 const float esig = expf(-sig);
                 const float cpos = lin_den > 0.f ? esig / sp : 0.f;
-                const float cneg = lin_den > 0.f ? esig / sn : 0.f;
-                for (int k = half; k < nfc; k += 2) {
-                    float v[32], w[32];
-                    tmem_ld32(tmem + lane_off + kColA + 32 * k, v);
-                    tmem_ld32(tmem + lane_off + kColA + F + 32 * k, w);
+                cneg = lin_den > 0.f ? esig / sn : 0.f;
+                auto scale_chunk = [&](uint32_t col, float c) {
+                    float v[32];
+                    tmem_ld32(col, v);
                     tmem_wait_ld();
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) { v[i] *= cpos; w[i] *= cneg; }
-                    tmem_st32(tmem + lane_off + kColA + 32 * k, v);
-                    tmem_st32(tmem + lane_off + kColA + F + 32 * k, w);
+                    for (int i = 0; i < 32; ++i) v[i] *= c;
+                    tmem_st32(col, v);
+                };
+                scale_chunk(pcol + 32 * part, cpos);
+                if (two) scale_chunk(pcol + 32 * (part + 2), cpos);
+                if (kCommit) {
+                    scale_chunk(mcol + 32 * part, cneg);
+                    if (two) scale_chunk(mcol + 32 * (part + 2), cneg);
                 }
-                // P' = w e^(s - sigma): K-major, no swizzle (8-row x 16-byte core matrices)
-                const float pofs = (lw - sig) * kLog2e;
-                for (int k = half; k < nsc; k += 2) {
-                    float v[16];
-                    tmem_ld16(dcol + lane_off + 16 * k, v);
-                    tmem_wait_ld();
+                if (has_sc) {
+                    // P' = w e^(s - sigma): K-major, no swizzle (8-row x 16-byte core matrices)
+                    const float pofs = (lw - sig) * kLog2e;
                     uint32_t pk[8];
 #pragma unroll
                     for (int i = 0; i < 16; i += 2)
-                        pk[i / 2] = pack_bf16x2(ex2(fmaf(v[i], scale_l2, pofs)), ex2(fmaf(v[i + 1], scale_l2, pofs)));
+                        pk[i / 2] = pack_bf16x2(ex2(fmaf(sc[i], scale_l2, pofs)), ex2(fmaf(sc[i + 1], scale_l2, pofs)));
                     uint8_t *prow = smem + a.off_p + (row >> 3) * (B / 8) * 128 + (row & 7) * 16;
-                    *reinterpret_cast<uint4 *>(prow + (2 * k) * 128) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-                    *reinterpret_cast<uint4 *>(prow + (2 * k + 1) * 128) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+                    *reinterpret_cast<uint4 *>(prow + (2 * part) * 128) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                    *reinterpret_cast<uint4 *>(prow + (2 * part + 1) * 128) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                 }
-                if (half == 0) den[row] = expf(log_l - sig) + expf(log_s - sig);
-                if (kCommit && fval) {
-                    const float4 *ip = reinterpret_cast<const float4 *>(&tk[6 * 128 + 16 * half]);
-                    const float4 *in = reinterpret_cast<const float4 *>(&tk[7 * 128 + 16 * half]);
-                    uint8_t *rp = pt_s + row * 128;
-                    uint8_t *rn = pt_s + (F + row) * 128;
-                    float dzp = 0.f, dzn = 0.f;
-                    float4 x[4], y[4], a4[4], b4[4];
+                inv_den = 1.f / (expf(log_l - sig) + expf(log_s - sig));
+                if (kCommit) {
+                    // phi(K) normalised, as the bf16 MN-major operand [token][feature]
+                    // (64-feature atoms of B rows), and this row's share of z += sum_t phi(k_t)
+                    if (fval) {
+                        const float4 *ip = reinterpret_cast<const float4 *>(&tk[6 * 128 + 16 * part]);
+                        const float4 *in = reinterpret_cast<const float4 *>(&tk[7 * 128 + 16 * part]);
+                        float dzp = 0.f, dzn = 0.f;
+                        const int fp = row, fn = F + row;
+                        uint8_t *bp = pkb + (fp >> 6) * (B * 128) + ((fp & 7) << 1);
+                        uint8_t *bn = pkb + (fn >> 6) * (B * 128) + ((fn & 7) << 1);
+                        const int gp = (fp & 63) >> 3, gn = (fn & 63) >> 3;
 #pragma unroll
-                    for (int gq = 0; gq < 4; ++gq) {
-                        const int gi = 4 * half + gq;
-                        x[gq] = *reinterpret_cast<const float4 *>(rp + ((gi ^ (row & 7)) << 4));
-                        y[gq] = *reinterpret_cast<const float4 *>(rn + ((gi ^ ((F + row) & 7)) << 4));
-                        a4[gq] = ip[gq];
-                        b4[gq] = in[gq];
-                    }
+                        for (int t4 = 0; t4 < 4; ++t4) {
+                            const float4 x = ip[t4], y = in[t4];
+                            const float ix[4] = {x.x, x.y, x.z, x.w}, iy[4] = {y.x, y.y, y.z, y.w};
 #pragma unroll
-                    for (int gq = 0; gq < 4; ++gq) {
-                        const int gi = 4 * half + gq;
-                        x[gq].x *= a4[gq].x; x[gq].y *= a4[gq].y; x[gq].z *= a4[gq].z; x[gq].w *= a4[gq].w;
-                        y[gq].x *= b4[gq].x; y[gq].y *= b4[gq].y; y[gq].z *= b4[gq].z; y[gq].w *= b4[gq].w;
-                        *reinterpret_cast<float4 *>(rp + ((gi ^ (row & 7)) << 4)) = x[gq];
-                        *reinterpret_cast<float4 *>(rn + ((gi ^ ((F + row) & 7)) << 4)) = y[gq];
-                        dzp += (x[gq].x + x[gq].y) + (x[gq].z + x[gq].w);
-                        dzn += (y[gq].x + y[gq].y) + (y[gq].z + y[gq].w);
+                            for (int j = 0; j < 4; ++j) {
+                                const int tl = 4 * t4 + j, t = 16 * part + tl;
+                                const float vp = epk[tl] * ix[j], vn = enk[tl] * iy[j];
+                                dzp += vp;
+                                dzn += vn;
+                                *reinterpret_cast<bf16 *>(bp + t * 128 + ((gp ^ (t & 7)) << 4)) = __float2bfloat16_rn(vp);
+                                *reinterpret_cast<bf16 *>(bn + t * 128 + ((gn ^ (t & 7)) << 4)) = __float2bfloat16_rn(vn);
+                            }
+                        }
+                        atomicAdd(&zs[fp], dzp);
+                        atomicAdd(&zs[fn], dzn);
                     }
-                    atomicAdd(&zs[row], dzp);
-                    atomicAdd(&zs[F + row], dzn);
                 }
                 tmem_wait_st();
             }
-            fence_proxy_async_smem();
             tc_fence_before();
-            if (math_sync_failed(!ok)) break;
-            if (mt == 0) {
-                mbar_arrive(phiready);
-                if (kCommit) {
-                    mbar_arrive(vtready);
-                    mbar_arrive(zdone);
-                } else {
-                    mbar_arrive(&zempty[zb]);
-                }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(phip);
+                if (kCommit) mbar_arrive(zdone);
             }
 
-            // ---- state update: S^T tile rows += dS^T rows (per feature half), then store
-            if (kCommit) {
+            if (!kCommit) {
+                // previous unit's output, while R+ of this one runs
+                if (kp >= 1) bad = !epilogue(kp - 1, prev_q, prev_inv);
+                // ---- phase D: phi- into the phi columns once R+ has consumed phi+
+                bad = !wait_bar(pread, kp & 1u, fail) || bad;
+                tc_fence_after();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) u0[i] *= cneg;
+                tmem_st32(pcol + 32 * part, u0);
+                if (two) {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) u1[i] *= cneg;
+                    tmem_st32(pcol + 32 * (part + 2), u1);
+                }
+                tmem_wait_st();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0 && !bad) mbar_arrive(phim);
+            } else {
+                // ---- state update: S^T tile rows += dS^T rows (per feature half), then store
                 const int e = row;
-                const int fpt = F / 2;   // features per thread within a half
-                bool brk = false;
-                const uint32_t dother = tmem + kColD0 + 128 * ((kp + 1) & 1);
+#pragma unroll 1
                 for (int h = 0; h < 2; ++h) {
-                    ok = wait_bar(&dsready[h], kp & 1u, fail);
-                    // the second half's tiles are modified only after the readout has read them
-                    if (h == 1 && ok) ok = wait_bar(rdone, kp & 1u, fail);
+                    bool bad2 = !wait_bar(&dsready[h], kp & 1u, fail);
                     tc_fence_after();
-                    for (int j = 0; j < fpt / 32; ++j) {
-                        const int fl = half * fpt + 32 * j;           // feature offset within the half
-                        const int c = (h * F + fl) / 32;              // state tile
-                        const int slot = (q + c) % NS;
-                        float v[32];
-                        tmem_ld32((h == 0 ? tmem + kColA : dother) + lane_off + fl, v);
+                    const uint32_t src = (h == 0 ? tmem : tmem + 256 + 128 * ((kp + 1) & 1)) + lane_off;
+                    auto upd = [&](int k) {
+                        const int slot = (q + h * NCH + k) % NS;
                         uint8_t *rowp = ring + (size_t)slot * chunk_bytes + e * 128;
-                        float4 s[8];
-                        if (e < d) {
+#pragma unroll 1
+                        for (int hh = 0; hh < 2; ++hh) {   // 16 features (4 granules) at a time
+                            float v[16];
+                            tmem_ld16(src + 32 * k + 16 * hh, v);
+                            float4 s4[4];
+                            if (e < d) {
 #pragma unroll
-                            for (int gq = 0; gq < 8; ++gq) s[gq] = *reinterpret_cast<const float4 *>(rowp + ((gq ^ (e & 7)) << 4));
-                        }
-                        tmem_wait_ld();
-                        if (ok && e < d) {
-#pragma unroll
-                            for (int gq = 0; gq < 8; ++gq) {
-                                s[gq].x += v[4 * gq];
-                                s[gq].y += v[4 * gq + 1];
-                                s[gq].z += v[4 * gq + 2];
-                                s[gq].w += v[4 * gq + 3];
+                                for (int gq = 0; gq < 4; ++gq)
+                                    s4[gq] = *reinterpret_cast<const float4 *>(rowp + (((4 * hh + gq) ^ (e & 7)) << 4));
                             }
+                            tmem_wait_ld();
+                            if (!bad2 && e < d) {
 #pragma unroll
-                            for (int gq = 0; gq < 8; ++gq) *reinterpret_cast<float4 *>(rowp + ((gq ^ (e & 7)) << 4)) = s[gq];
+                                for (int gq = 0; gq < 4; ++gq) {
+                                    s4[gq].x += v[4 * gq];
+                                    s4[gq].y += v[4 * gq + 1];
+                                    s4[gq].z += v[4 * gq + 2];
+                                    s4[gq].w += v[4 * gq + 3];
+                                    *reinterpret_cast<float4 *>(rowp + (((4 * hh + gq) ^ (e & 7)) << 4)) = s4[gq];
+                                }
+                            }
                         }
-                    }
+                    };
+#pragma unroll 1
+                    for (int k = part; k < NCH; k += 2) upd(k);
                     fence_proxy_async_smem();
                     tc_fence_before();
-                    if (math_sync_failed(!ok)) { brk = true; break; }
-                    if (mt == 0) {
+                    __syncwarp();
+                    if (lane == 0 && !bad2) {
                         mbar_arrive(&tready[h]);
                         if (h == 1) mbar_arrive(efree);
                     }
                 }
-                if (brk) break;
+                epilogue(kp, q, inv_den);
             }
-
-            // ---- output epilogue: out = D / den, staged as the TMA box image in the
-            // unit's last two ring slots (row i = t*G + hh, 128-byte swizzle)
-            ok = wait_bar(&dready[kp & 1], (kp >> 1) & 1u, fail);
-            if (ok) ok = wait_bar(ofree, kp & 1u, fail);
-            tc_fence_after();
-            {
-                const int dh = d / 2;
-                const float inv = 1.f / den[row];
-                float v[2][32];
-                tmem_ld32(dcol + lane_off + half * dh, v[0]);
-                if (dh > 32) tmem_ld32(dcol + lane_off + half * dh + 32, v[1]);
-                tmem_wait_ld();
-                if (ok && valid) {
-                    // d = 128: column half -> slot; d = 64: token half -> slot (one 64-column atom)
-                    const int rows_half = G * B / 2;
-                    const int sidx = d == 128 ? half : (row >= rows_half ? 1 : 0);
-                    const int srow = d == 128 ? row : row - sidx * rows_half;
-                    const int oc = kCommit ? ocm : NC - 2;
-                    uint8_t *base = ring + (size_t)((q + oc + sidx) % NS) * chunk_bytes + srow * 128;
-#pragma unroll
-                    for (int hc = 0; hc < 2; ++hc) {
-                        if (hc * 32 >= dh) break;
-                        uint32_t pk[16];
-#pragma unroll
-                        for (int i = 0; i < 32; i += 2) pk[i / 2] = pack_bf16x2(v[hc][i] * inv, v[hc][i + 1] * inv);
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            const int gi = 4 * hc + i + (d == 128 ? 0 : 4 * half);   // 16-byte granule in the 128-byte row
-                            *reinterpret_cast<uint4 *>(base + ((gi ^ (srow & 7)) << 4)) =
-                                make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-                        }
-                    }
-                }
-            }
-            fence_proxy_async_smem();
-            tc_fence_before();
-            if (math_sync_failed(!ok)) break;
-            if (mt == 0) {
-                mbar_arrive(ostaged);
-                mbar_arrive(&dfree[kp & 1]);
-            }
+            prev_q = q;
+            prev_inv = inv_den;
             q += NC;
             ++kp;
         }
+        if (!kCommit && ok && kp >= 1) epilogue(kp - 1, prev_q, prev_inv);
         if (mt == 0 && *fail) raise_error(a.err, ERR_WAIT_TIMEOUT);
     }
 
@@ -918,16 +1031,16 @@ bool fused_supported(const hybrid_cfg &c, bool commit)
     if (c.io_dtype != HYBRID_BF16) return false;
     if (c.head_dim != 64 && c.head_dim != 128) return false;
     if (c.feat_dim != 64 && c.feat_dim != 128) return false;
-    if (c.block_size % 16 != 0) return false;
+    // scores ride in one 16-column chunk per part; the K^T atom holds B <= 64 tokens
+    if (c.block_size != 16 && c.block_size != 32) return false;
     const int G = c.n_q_heads / c.n_kv_heads;
     if (G * c.block_size > 128) return false;
     if (commit && c.block_size != 32) return false;
-    const FLayout L = make_flayout(c.head_dim, c.feat_dim, c.block_size);
-    const int NC = 2 * c.feat_dim / 32;
-    // the commit keeps the first feature half resident while the second streams
-    if (L.NS < (commit ? NC / 2 + 2 : 4)) return false;
-    // region X must also hold V^T and phi(K)^T for the commit
-    if (commit && (uint32_t)(128 * 128 + 2 * c.feat_dim * 128) > L.off_vb - L.off_q) return false;
+    const FLayout L = make_flayout(c.head_dim, c.feat_dim, c.block_size, commit);
+    const int NCH = c.feat_dim / 32;
+    // step: the last two tiles of a unit are held for the output; commit: the
+    // first half stays resident until updated and two of its slots take the output
+    if (L.NS < (commit ? NCH + 2 : 4)) return false;
     return (int)L.bytes <= kSmemLimit;
 }
 
@@ -935,7 +1048,7 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
                          const void *W, const float *alpha, void *const *states, int n_req, void *O,
                          unsigned *err, cudaStream_t st)
 {
-    const FLayout L = make_flayout(c.head_dim, c.feat_dim, c.block_size);
+    const FLayout L = make_flayout(c.head_dim, c.feat_dim, c.block_size, commit);
     FusedArgs a;
     {
         const int d = c.head_dim, F = c.feat_dim, B = c.block_size, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
@@ -944,26 +1057,20 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
         const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)Hq, rows};
         const cuuint64_t sq[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hq * d * 2};
         const cuuint32_t bq[3] = {64, (cuuint32_t)G, (cuuint32_t)B};
-        const cuuint64_t dk[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, rows};
-        const cuuint64_t sk[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
-        const cuuint32_t bk[3] = {64, 1, (cuuint32_t)B};
+        const cuuint64_t dv[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, rows};
+        const cuuint64_t sv[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
+        const cuuint32_t bv[3] = {64, 1, (cuuint32_t)B};
         const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
         const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
         const cuuint32_t bw[2] = {64, (cuuint32_t)d};
-        if (!encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !encode_bf16(&a.tmK, K, 3, dk, sk, bk) ||
-            !encode_bf16(&a.tmV, V, 3, dk, sk, bk) || !encode_bf16(&a.tmW, W, 2, dw, sw, bw))
-            return cudaErrorInvalidValue;
         const cuuint32_t bo[3] = {64, (cuuint32_t)G, (cuuint32_t)(d == 128 ? B : B / 2)};
-        if (!encode_bf16(&a.tmO, O, 3, dq, sq, bo))
+        if (!encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !encode_bf16(&a.tmV, V, 3, dv, sv, bv) ||
+            !encode_bf16(&a.tmW, W, 2, dw, sw, bw) || !encode_bf16(&a.tmO, O, 3, dq, sq, bo))
             return cudaErrorInvalidValue;
     }
-    a.Q = static_cast<const bf16 *>(Q);
     a.K = static_cast<const bf16 *>(K);
-    a.V = static_cast<const bf16 *>(V);
-    a.W = static_cast<const bf16 *>(W);
     a.alpha = alpha;
     a.states = states;
-    a.O = static_cast<bf16 *>(O);
     a.err = err;
     a.n_units = n_req * c.n_kv_heads;
     a.B = c.block_size;
@@ -975,10 +1082,10 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
     a.NS = L.NS;
     a.scale = 1.f / sqrtf((float)c.head_dim);
     a.off_q = L.off_q;
-    a.off_w = L.off_w;
-    a.off_k = L.off_k;
+    a.off_wk = L.off_wk;
     a.off_vb = L.off_vb;
     a.off_p = L.off_p;
+    a.off_pk = L.off_pk;
     a.off_z = L.off_z;
     a.off_st = L.off_st;
     a.off_bar = L.off_bar;
