@@ -28,20 +28,21 @@
 //   PV   D  = P' V                    (P' = w e^(s - sigma), bf16)
 //   R+   D += phi+'(Q) S+             (tf32, A operand in Tensor Memory)
 //   R-   D += phi-'(Q) S-
-//   dS   dS^T = V^T phi(K)^T per feature half (commit; bf16)
+//   dS   dS^T = V^T phi(K)^T per feature half (commit; bf16 from the TMA'd V)
 // and the math warps compute the row statistics, phi(Q) and P' between g1
 // and PV, and out = D / den afterwards.  Merge: with sigma the log of the
 // larger branch mass, phi' = phi e^-sigma and P' = w e^(s - sigma), so
 // D / den = (w sm_num + lin_num) / (w sm_den + lin_den) exactly, with
 // den = e^(log lin_den - sigma) + e^(log(w sm_den) - sigma) in [1, 2].
 //
-// Overlap between units (step only): Tensor Memory holds two unit slots of
-// 256 columns, [phi | D] each, so the next unit's g1 runs between this unit's
-// R+ and R-.  A unit's phi+ and phi- share its F phi columns: phi- is held in
-// registers until R+ has consumed phi+.  With the commit the phi columns hold
-// both halves ([0, 2F)) and dS^T of the two halves reuses the phi+ columns and
-// the idle output accumulator; units then follow one another on the tensor
-// cores, the math of one overlapping the MMAs of the other.
+// A unit's phi+ and phi- share its F phi columns: phi- waits in registers until
+// R+ has consumed phi+.  Step: Tensor Memory holds two unit slots of 256
+// columns, [phi | D] each, so the next unit's g1 runs between this unit's R+
+// and R- and its feature map overlaps R-.  Commit: [D | phi | dS+ | dS-];
+// dS^T is formed before the readout, so each half's tiles are updated in
+// shared memory (and written back by the storer) as soon as the readout has
+// consumed them; V, P' and phi(K) then share the Q region, so all 2F/32 state
+// tiles of a unit fit in the ring.
 //
 // MMA cost note: on this part a tcgen05.mma with M = 128 costs about the same
 // time for any N up to 128-256, so contractions are shaped for few, wide
@@ -73,6 +74,8 @@ constexpr int kOneCtaPerSm = 118 * 1024;
 constexpr uint32_t kBarMath = 1;      // named barrier over the 256 math threads
 constexpr uint32_t kBarPair = 2;      // 2..5: the two math warps of one TMEM lane quarter
 constexpr uint32_t kStatBytes = 14 * 1024;
+// Tensor Memory columns with the commit (F <= 128, d <= 128)
+constexpr uint32_t kCmD = 0, kCmP = 128, kCmDSp = 256, kCmK = 288, kCmDSm = 384;
 
 struct FusedArgs {
     CUtensorMap tmQ, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
@@ -107,16 +110,25 @@ FLayout make_flayout(int d, int F, int B, bool commit)
     const uint32_t p = (((uint32_t)128 * B * 2) + 1023) & ~1023u;
     const uint32_t pk = commit ? ((((uint32_t)(2 * F / 64) * B * 128) + 1023) & ~1023u) : 0u;
     const uint32_t bar = 1024;
-    const uint32_t fixed = q + wk + vb + p + pk + 2 * zb + kStatBytes + bar + 1024;
+    // with the commit, V, P' and phi(K) live in the Q region once g1 has read Q
+    // (the next unit's Q is loaded after the unit's dS^T and P V are done)
+    const bool overlay = commit && vb + p + pk <= q;
+    const uint32_t fixed = q + wk + (overlay ? 0u : vb + p + pk) + 2 * zb + kStatBytes + bar + 1024;
     int ns = ((int)kSmemLimit - (int)fixed) / (int)chunk;
     if (ns > kMaxSlots) ns = kMaxSlots;
     L.NS = ns;
     uint32_t off = (uint32_t)(ns > 0 ? ns : 0) * chunk;
     L.off_q = off; off += q;
     L.off_wk = off; off += wk;
-    L.off_vb = off; off += vb;
-    L.off_p = off; off += p;
-    L.off_pk = off; off += pk;
+    if (overlay) {
+        L.off_vb = L.off_q;
+        L.off_p = L.off_q + vb;
+        L.off_pk = L.off_q + vb + p;
+    } else {
+        L.off_vb = off; off += vb;
+        L.off_p = off; off += p;
+        L.off_pk = off; off += pk;
+    }
     L.off_z = off; off += 2 * zb;
     L.off_st = off; off += kStatBytes;
     L.off_bar = off; off += bar;
@@ -169,47 +181,45 @@ __device__ __forceinline__ bool group_sync_failed(uint32_t id, uint32_t nthreads
     return r != 0;
 }
 
-// Reduce 16 per-lane values across the 32 lanes of a warp (op = add / max /
-// min) by halving the set each step; on return lane L holds the total of
-// value index tok(L) = 8*b4 + 4*b3 + 2*b2 + b1 (b_i = bit i of L).
 template <int kOp>
 __device__ __forceinline__ float comb(float a, float b)
 {
     return kOp == 0 ? a + b : (kOp == 1 ? fmaxf(a, b) : fminf(a, b));
 }
+// Reduce 32 per-lane values across the 32 lanes of a warp (op = add / max /
+// min) by halving the set each step (31 shuffles); on return lane L holds the
+// total of value index L.
 template <int kOp>
-__device__ __forceinline__ float warp_reduce16(float (&v)[16], int lane)
+__device__ __forceinline__ float warp_reduce32(float (&v)[32], int lane)
 {
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
+    for (int i = 0; i < 16; ++i) {
         const bool up = lane & 16;
-        const float send = up ? v[i] : v[i + 8], keep = up ? v[i + 8] : v[i];
+        const float send = up ? v[i] : v[i + 16], keep = up ? v[i + 16] : v[i];
         v[i] = comb<kOp>(keep, __shfl_xor_sync(0xffffffffu, send, 16));
     }
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < 8; ++i) {
         const bool up = lane & 8;
-        const float send = up ? v[i] : v[i + 4], keep = up ? v[i + 4] : v[i];
+        const float send = up ? v[i] : v[i + 8], keep = up ? v[i + 8] : v[i];
         v[i] = comb<kOp>(keep, __shfl_xor_sync(0xffffffffu, send, 8));
     }
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < 4; ++i) {
         const bool up = lane & 4;
-        const float send = up ? v[i] : v[i + 2], keep = up ? v[i + 2] : v[i];
+        const float send = up ? v[i] : v[i + 4], keep = up ? v[i + 4] : v[i];
         v[i] = comb<kOp>(keep, __shfl_xor_sync(0xffffffffu, send, 4));
     }
-    {
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
         const bool up = lane & 2;
-        const float send = up ? v[0] : v[1], keep = up ? v[1] : v[0];
-        v[0] = comb<kOp>(keep, __shfl_xor_sync(0xffffffffu, send, 2));
+        const float send = up ? v[i] : v[i + 2], keep = up ? v[i + 2] : v[i];
+        v[i] = comb<kOp>(keep, __shfl_xor_sync(0xffffffffu, send, 2));
     }
-    return comb<kOp>(v[0], __shfl_xor_sync(0xffffffffu, v[0], 1));
+    const bool up = lane & 1;
+    const float send = up ? v[0] : v[1], keep = up ? v[1] : v[0];
+    return comb<kOp>(keep, __shfl_xor_sync(0xffffffffu, send, 1));
 }
-__device__ __forceinline__ int reduce16_token(int lane)
-{
-    return ((lane >> 4) & 1) * 8 + ((lane >> 3) & 1) * 4 + ((lane >> 2) & 1) * 2 + ((lane >> 1) & 1);
-}
-
 __device__ __forceinline__ float *unit_state(const FusedArgs &a, int u)
 {
     const int r = u / a.Hkv, g = u % a.Hkv;
@@ -290,22 +300,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint64_t *zempty = zfull + 2;     // [2]
     uint64_t *dready = zempty + 2;    // [2] MMA -> math: the unit's output accumulator is complete
     uint64_t *dfree = dready + 2;     // [2] math -> MMA: the output accumulator has been read
-    uint64_t *dsready = dfree + 2;    // [2] MMA -> math: dS^T of a feature half is in Tensor Memory
-    uint64_t *tready = dsready + 2;   // [2] math -> storer: a feature half of the tiles is updated
+    uint64_t *tready = dfree + 2;     // [2] math -> storer: a feature half of the tiles is updated
     uint64_t *xfull = tready + 2;     // Q, W (TMA) and K^T (producer warp) are in place
     uint64_t *xfree = xfull + 1;
     uint64_t *vfull = xfree + 1;
     uint64_t *vfree = vfull + 1;
     uint64_t *uready = vfree + 1;     // MMA -> math: g1 done
-    uint64_t *phip = uready + 1;      // math -> MMA: phi+ (with the commit: all of phi, phi(K)) and P'
-    uint64_t *phim = phip + 1;        // math -> MMA: phi- (step only)
-    uint64_t *pread = phim + 1;       // MMA -> math: R+ has consumed phi+ (step only)
-    uint64_t *efree = pread + 1;      // math -> MMA: dS^T has been consumed (commit)
+    uint64_t *phip = uready + 1;      // math -> MMA: phi+ and P' (with the commit also phi(K))
+    uint64_t *phim = phip + 1;        // math -> MMA: phi- in the phi columns
+    uint64_t *pread = phim + 1;       // MMA -> math: R+ has consumed phi+ (and dS^T is formed)
+    uint64_t *efree = pread + 1;      // math -> MMA: the first-half update has read dS+ (commit)
     uint64_t *zdone = efree + 1;      // math -> storer: z is updated (commit)
     uint64_t *ofree = zdone + 1;      // storer -> math: the output slots may be written (commit)
     uint64_t *ostaged = ofree + 1;    // math -> storer: the output tile is in its slots
     uint64_t *mmadone = ostaged + 1;
-    const int n_bars = 2 * NS + 12 + 13;
+    const int n_bars = 2 * NS + 10 + 13;
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + n_bars);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
@@ -467,28 +476,33 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 }
                 if (ok && kp >= 1) tail(kp - 1, prev_qt);
             } else {
+                // Tensor Memory: [0,128) D, [128,128+F) phi (U, then phi+, then phi-),
+                // scores after U, [256,256+F) dS+ (U_k^T at 288 until then),
+                // [384,384+F) dS-.  dS^T is formed before the readout, so each half's
+                // tiles can be updated as soon as that half has been read out.
                 for (int u = u_begin; u < u_end; ++u) {
                     if (!unit_state(a, u)) continue;
-                    const uint32_t D = 256 + 128 * (kp & 1), Do = 256 + 128 * ((kp + 1) & 1);
                     if (!wait_bar(xfull, kp & 1u, fail)) { ok = false; break; }
+                    // U_k^T and the scores land in the dS+ columns: the previous unit's
+                    // first-half update must have read them (its R- precedes in issue order)
                     if (kp >= 1 && !wait_bar(efree, (kp - 1) & 1u, fail)) { ok = false; break; }
-                    if (kp >= 2 && !wait_bar(&dfree[kp & 1], ((kp - 2) >> 1) & 1u, fail)) { ok = false; break; }
                     tc_fence_after();
-                    g1(0, D);
+                    g1(kCmP, kCmK);
                     mma_commit(uready);
                     mma_commit(xfree);
-                    // phip also covers phi-, phi(K) and the previous unit's epilogue
+                    // phip also covers the previous unit's output epilogue and second-half update
                     if (!wait_bar(phip, kp & 1u, fail) || !wait_bar(vfull, kp & 1u, fail)) { ok = false; break; }
                     tc_fence_after();
-                    pv(D);
-                    for (int c = 0; c < NCH && ok; ++c) ok = readout(D, 32 * c, qt + c) >= 0;
+                    ds(kCmDSp, 0);
+                    ds(kCmDSm, 1);
+                    pv(kCmD);
+                    for (int c = 0; c < NCH && ok; ++c) ok = readout(kCmD, kCmP + 32 * c, qt + c) >= 0;
                     if (!ok) break;
-                    ds(0, 0);   // dS^T of phi+ features into the phi+ columns R+ has consumed
-                    mma_commit(&dsready[0]);
-                    for (int c = NCH; c < NC && ok; ++c) ok = readout(D, F + 32 * (c - NCH), qt + c) >= 0;
+                    mma_commit(pread);
+                    if (!wait_bar(phim, kp & 1u, fail)) { ok = false; break; }
+                    tc_fence_after();
+                    for (int c = NCH; c < NC && ok; ++c) ok = readout(kCmD, kCmP + 32 * (c - NCH), qt + c) >= 0;
                     if (!ok) break;
-                    ds(Do, 1);  // dS^T of phi- features into the idle output accumulator
-                    mma_commit(&dsready[1]);
                     mma_commit(&dready[kp & 1]);
                     mma_commit(vfree);
                     qt += NC;
@@ -514,17 +528,25 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
                 mbar_arrive_expect_tx(xfull, xbytes);
-                for (int e = 0; e < d / 64; ++e)
-                    tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xfull);
                 for (int f = 0; f < F / 64; ++f)
                     tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xfull);
             }
             kt_store(a, kr, kt, lane);
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(xfull);
+            // with the commit the Q region holds the previous unit's V, P' and phi(K)
+            // until its dS^T and P V have run
+            if (kCommit && kp > 0) ok = wait_bar(pread, (kp - 1) & 1u, fail);
+            if (__any_sync(0xffffffffu, !ok)) break;
+            if (lane == 0) {
+                for (int e = 0; e < d / 64; ++e)
+                    tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xfull);
+                mbar_arrive(xfull);
+            }
             ++nx;
-            if (kp > 0) ok = wait_bar(vfree, (kp - 1) & 1u, fail);
+            // V: after the previous unit's P V (step), after this unit's g1 has read
+            // Q (commit: V shares the Q region)
+            ok = kCommit ? wait_bar(xfree, kp & 1u, fail) : (kp == 0 || wait_bar(vfree, (kp - 1) & 1u, fail));
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
                 mbar_arrive_expect_tx(vfull, (uint32_t)(d / 64) * (B * 128));
@@ -603,7 +625,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         float *tk = xb + 10 * 128;                                 // token statistics (commit)
         uint8_t *pkb = smem + a.off_pk;
         const float scale_l2 = a.scale * kLog2e;
-        const int tok = reduce16_token(lane);
         const uint32_t pair_bar = kBarPair + q4;
         // one exchange point: pair barrier for the step, all math warps with the commit
         auto sync_failed = [&](bool local_fail) -> bool {
@@ -614,7 +635,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         // out = D / den, staged as the TMA box image in the unit's held-back ring
         // slots (row i = t*G + hh, 128-byte swizzle)
         auto epilogue = [&](uint32_t ek, uint32_t eq, float inv) -> bool {
-            const uint32_t dcol = kCommit ? 256 + 128 * (ek & 1) : (ek & 1) * 256 + 128;
+            const uint32_t dcol = kCommit ? kCmD : (ek & 1) * 256 + 128;
             bool ok = wait_bar(&dready[ek & 1], (ek >> 1) & 1u, fail);
             if (kCommit && ok) ok = wait_bar(ofree, ek & 1u, fail);
             tc_fence_after();
@@ -664,28 +685,27 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             // gate of this row's query head, loaded now so the latency overlaps the first phase
             const float alpha_row = valid ? a.alpha[g * G + row % G] : 0.f;
             float *zs = zbuf0 + zb * zstride;
-            const uint32_t T = kCommit ? 0u : (kp & 1) * 256;
-            const uint32_t pcol = tmem + T + lane_off;                         // phi+ (and U)
-            const uint32_t mcol = tmem + (kCommit ? (uint32_t)F : T) + lane_off;   // phi-
-            const uint32_t scol = tmem + T + F + lane_off;                     // scores
-            const uint32_t kcol = tmem + 256 + 128 * (kp & 1) + lane_off;      // U_k^T (commit)
+            const uint32_t T = (kp & 1) * 256;
+            const uint32_t pcol = tmem + (kCommit ? kCmP : T) + lane_off;       // U, phi+, phi-
+            const uint32_t scol = pcol + F;                                    // scores
+            const uint32_t kcol = tmem + kCmK + lane_off;                      // U_k^T (commit)
 
-            // ---- phase A: row extrema of U and of the scores (U kept in registers)
+            // ---- phase A: row extrema of U and of the scores (U kept in registers);
+            // commit: per-token extrema of U_k^T over this warp's 32 features
             bool bad = !wait_bar(uready, kp & 1u, fail);
             tc_fence_after();
-            float sc[16], u0[32], u1[32], uk[16];
+            float sc[16], u0[32], u1[32];
             if (kCommit) {
-                // per-token extrema of U_k^T over this warp's 32 features (features on lanes)
-                tmem_ld16(kcol + 16 * part, uk);
+                // phi(K): thread (feature row, part) owns feature part*F + row of every
+                // token; part 0 needs the per-token max of U_k over features, part 1
+                // the min (features on lanes: reduce over the warp, then the quarters)
+                float uk[32];
+                tmem_ld32(kcol, uk);
                 tmem_wait_ld();
-                float vmx[16], vmn[16];
 #pragma unroll
-                for (int t = 0; t < 16; ++t) { vmx[t] = fval ? uk[t] : -INFINITY; vmn[t] = fval ? uk[t] : INFINITY; }
-                const float rmx = warp_reduce16<1>(vmx, lane), rmn = warp_reduce16<2>(vmn, lane);
-                if (!(lane & 1)) {
-                    tk[(0 * 32 + 16 * part + tok) * 4 + q4] = rmx;
-                    tk[(1 * 32 + 16 * part + tok) * 4 + q4] = rmn;
-                }
+                for (int t = 0; t < 32; ++t) uk[t] = fval ? (part == 0 ? uk[t] : -uk[t]) : -INFINITY;
+                const float ext = warp_reduce32<1>(uk, lane);
+                tk[(part * 32 + lane) * 4 + q4] = ext;   // max of +-U_k for token lane
             }
             if (has_sc) tmem_ld16(scol + 16 * part, sc);
             tmem_ld32(pcol + 32 * part, u0);
@@ -708,22 +728,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 xa[(part * 3 + 2) * 128 + row] = mn;
             }
             if (sync_failed(bad)) { ok = false; break; }
-            if (kCommit) {
-                if (mt < 64) {   // combine the four feature quarters per token
-                    const int t = mt & 31, s = mt >> 5;
-                    const float4 v = *reinterpret_cast<const float4 *>(&tk[(s * 32 + t) * 4]);
-                    tk[(4 + s) * 128 + t] = s == 0 ? fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w))
-                                                   : fminf(fminf(v.x, v.y), fminf(v.z, v.w));
-                }
-                if (sync_failed(false)) { ok = false; break; }
-            }
             const float ms = fmaxf(xa[0 * 128 + row], xa[3 * 128 + row]);
             const float mx = fmaxf(xa[1 * 128 + row], xa[4 * 128 + row]);
             const float mn = fminf(xa[2 * 128 + row], xa[5 * 128 + row]);
 
             // ---- phase B: exponentials; phi+ unnormalised into Tensor Memory, phi- kept
+            // in registers until R+ has consumed phi+; commit: unnormalised phi(K)
             bad = !wait_bar(&zfull[zb], (kp >> 1) & 1u, fail);
-            float epk[16], enk[16];
+            float ek[32];   // commit: unnormalised phi(K) of feature part*F + row, per token
             {
                 const float mxl = mx * kLog2e, mnl = mn * kLog2e, ml = ms * scale_l2;
                 float l = 0.f, sp = 0.f, sn = 0.f, lp = 0.f, ln = 0.f;
@@ -753,51 +765,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                         }
                     }
                     tmem_st32(pcol + 32 * k, ep);
-                    // with the commit phi- has its own columns (the scores there are in
-                    // registers by now): store it unnormalised as well
-                    if (kCommit) tmem_st32(mcol + 32 * k, uu);
                 };
+                exps(u0, part);
+                if (two) exps(u1, part + 2);
                 if (kCommit) {
-                    // U is reloaded rather than kept since phase A (register pressure)
-#pragma unroll 1
-                    for (int k = part; k < NCH; k += 2) {
-                        float uu[32];
-                        tmem_ld32(pcol + 32 * k, uu);
-                        tmem_wait_ld();
-                        exps(uu, k);
-                    }
-                } else {
-                    exps(u0, part);
-                    if (two) exps(u1, part + 2);
-                }
-                if (kCommit) {
-                    // unnormalised phi(K) of this half's 16 tokens; per-token sums over the warp's features
-                    tmem_ld16(kcol + 16 * part, uk);
+                    // unnormalised phi(K) of this thread's feature for every token
+                    float uk[32];
+                    tmem_ld32(kcol, uk);
                     tmem_wait_ld();
-                    const float4 *tmx = reinterpret_cast<const float4 *>(&tk[4 * 128 + 16 * part]);
-                    const float4 *tmn = reinterpret_cast<const float4 *>(&tk[5 * 128 + 16 * part]);
 #pragma unroll
-                    for (int t4 = 0; t4 < 4; ++t4) {
-                        const float4 x = tmx[t4], y = tmn[t4];
-                        const float kx[4] = {x.x, x.y, x.z, x.w}, kn[4] = {y.x, y.y, y.z, y.w};
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) {
-                            const int t = 4 * t4 + j;
-                            epk[t] = fval ? ex2((uk[t] - kx[j]) * kLog2e) : 0.f;
-                            enk[t] = fval ? ex2((kn[j] - uk[t]) * kLog2e) : 0.f;
-                        }
+                    for (int t = 0; t < 32; ++t) {
+                        const float4 x = *reinterpret_cast<const float4 *>(&tk[(part * 32 + t) * 4]);
+                        const float m = fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w));
+                        ek[t] = fval ? ex2(((part == 0 ? uk[t] : -uk[t]) - m) * kLog2e) : 0.f;
+                        uk[t] = ek[t];
                     }
-                    float sr[16];
-#pragma unroll
-                    for (int t = 0; t < 16; ++t) sr[t] = epk[t];
-                    const float rsp = warp_reduce16<0>(sr, lane);
-#pragma unroll
-                    for (int t = 0; t < 16; ++t) sr[t] = enk[t];
-                    const float rsn = warp_reduce16<0>(sr, lane);
-                    if (!(lane & 1)) {
-                        tk[(2 * 32 + 16 * part + tok) * 4 + q4] = rsp;
-                        tk[(3 * 32 + 16 * part + tok) * 4 + q4] = rsn;
-                    }
+                    const float ssum = warp_reduce32<0>(uk, lane);
+                    tk[((2 + part) * 32 + lane) * 4 + q4] = ssum;
                 }
                 xb[(part * 5 + 0) * 128 + row] = l;
                 xb[(part * 5 + 1) * 128 + row] = sp;
@@ -812,16 +796,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 if (lane == 0 && !bad) mbar_arrive(&zempty[zb]);
             }
             if (sync_failed(bad)) { ok = false; break; }
-            if (kCommit) {
-                if (mt < 64) {   // per-token normalisers of phi(K)
-                    const int t = mt & 31, s = mt >> 5;
-                    const float4 v = *reinterpret_cast<const float4 *>(&tk[((2 + s) * 32 + t) * 4]);
-                    tk[(6 + s) * 128 + t] = 1.f / ((v.x + v.y) + (v.z + v.w));
-                }
-                if (sync_failed(false)) { ok = false; break; }
-            }
 
-            // ---- phase C: sigma, phi+ scaled in place, P', den; commit: phi-, phi(K), z
+            // ---- phase C: sigma, phi+ scaled in place, P', den; commit: phi(K), z
             float cneg, inv_den;
             {
                 const float l = xb[0 * 128 + row] + xb[5 * 128 + row];
@@ -837,20 +813,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 const float esig = expf(-sig);
                 const float cpos = lin_den > 0.f ? esig / sp : 0.f;
                 cneg = lin_den > 0.f ? esig / sn : 0.f;
-                auto scale_chunk = [&](uint32_t col, float c) {
+                auto scale_chunk = [&](uint32_t col) {
                     float v[32];
                     tmem_ld32(col, v);
                     tmem_wait_ld();
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] *= c;
+                    for (int i = 0; i < 32; ++i) v[i] *= cpos;
                     tmem_st32(col, v);
                 };
-                scale_chunk(pcol + 32 * part, cpos);
-                if (two) scale_chunk(pcol + 32 * (part + 2), cpos);
-                if (kCommit) {
-                    scale_chunk(mcol + 32 * part, cneg);
-                    if (two) scale_chunk(mcol + 32 * (part + 2), cneg);
-                }
+                scale_chunk(pcol + 32 * part);
+                if (two) scale_chunk(pcol + 32 * (part + 2));
                 if (has_sc) {
                     // P' = w e^(s - sigma): K-major, no swizzle (8-row x 16-byte core matrices)
                     const float pofs = (lw - sig) * kLog2e;
@@ -865,32 +837,24 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 inv_den = 1.f / (expf(log_l - sig) + expf(log_s - sig));
                 if (kCommit) {
                     // phi(K) normalised, as the bf16 MN-major operand [token][feature]
-                    // (64-feature atoms of B rows), and this row's share of z += sum_t phi(k_t)
-                    if (fval) {
-                        const float4 *ip = reinterpret_cast<const float4 *>(&tk[6 * 128 + 16 * part]);
-                        const float4 *in = reinterpret_cast<const float4 *>(&tk[7 * 128 + 16 * part]);
-                        float dzp = 0.f, dzn = 0.f;
-                        const int fp = row, fn = F + row;
-                        uint8_t *bp = pkb + (fp >> 6) * (B * 128) + ((fp & 7) << 1);
-                        uint8_t *bn = pkb + (fn >> 6) * (B * 128) + ((fn & 7) << 1);
-                        const int gp = (fp & 63) >> 3, gn = (fn & 63) >> 3;
-#pragma unroll
-                        for (int t4 = 0; t4 < 4; ++t4) {
-                            const float4 x = ip[t4], y = in[t4];
-                            const float ix[4] = {x.x, x.y, x.z, x.w}, iy[4] = {y.x, y.y, y.z, y.w};
-#pragma unroll
-                            for (int j = 0; j < 4; ++j) {
-                                const int tl = 4 * t4 + j, t = 16 * part + tl;
-                                const float vp = epk[tl] * ix[j], vn = enk[tl] * iy[j];
-                                dzp += vp;
-                                dzn += vn;
-                                *reinterpret_cast<bf16 *>(bp + t * 128 + ((gp ^ (t & 7)) << 4)) = __float2bfloat16_rn(vp);
-                                *reinterpret_cast<bf16 *>(bn + t * 128 + ((gn ^ (t & 7)) << 4)) = __float2bfloat16_rn(vn);
-                            }
-                        }
-                        atomicAdd(&zs[fp], dzp);
-                        atomicAdd(&zs[fn], dzn);
+                    // (64-feature atoms of B rows), and z[part*F + row] += sum_t phi(k_t)
+                    // (this thread is the only writer); lane t holds token t's normaliser
+                    float inv_l;
+                    {
+                        const float4 v = *reinterpret_cast<const float4 *>(&tk[((2 + part) * 32 + lane) * 4]);
+                        inv_l = 1.f / ((v.x + v.y) + (v.z + v.w));
                     }
+                    const int f = part * F + row;
+                    uint8_t *bf = pkb + (f >> 6) * (B * 128) + ((f & 7) << 1);
+                    const int gf = (f & 63) >> 3;
+                    float dz = 0.f;
+#pragma unroll
+                    for (int t = 0; t < 32; ++t) {
+                        const float v = ek[t] * __shfl_sync(0xffffffffu, inv_l, t);
+                        dz += v;
+                        if (fval) *reinterpret_cast<bf16 *>(bf + t * 128 + ((gf ^ (t & 7)) << 4)) = __float2bfloat16_rn(v);
+                    }
+                    if (fval) zs[f] += dz;
                 }
                 tmem_wait_st();
             }
@@ -902,32 +866,34 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 if (kCommit) mbar_arrive(zdone);
             }
 
-            if (!kCommit) {
-                // previous unit's output, while R+ of this one runs
-                if (kp >= 1) bad = !epilogue(kp - 1, prev_q, prev_inv);
-                // ---- phase D: phi- into the phi columns once R+ has consumed phi+
-                bad = !wait_bar(pread, kp & 1u, fail) || bad;
-                tc_fence_after();
+            // previous unit's output, while R+ of this one runs (step)
+            if (!kCommit && kp >= 1) bad = !epilogue(kp - 1, prev_q, prev_inv);
+            // ---- phase D: phi- into the phi columns once R+ has consumed phi+
+            bad = !wait_bar(pread, kp & 1u, fail) || bad;
+            tc_fence_after();
 #pragma unroll
-                for (int i = 0; i < 32; ++i) u0[i] *= cneg;
-                tmem_st32(pcol + 32 * part, u0);
-                if (two) {
+            for (int i = 0; i < 32; ++i) u0[i] *= cneg;
+            tmem_st32(pcol + 32 * part, u0);
+            if (two) {
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) u1[i] *= cneg;
-                    tmem_st32(pcol + 32 * (part + 2), u1);
-                }
-                tmem_wait_st();
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0 && !bad) mbar_arrive(phim);
-            } else {
-                // ---- state update: S^T tile rows += dS^T rows (per feature half), then store
+                for (int i = 0; i < 32; ++i) u1[i] *= cneg;
+                tmem_st32(pcol + 32 * (part + 2), u1);
+            }
+            tmem_wait_st();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0 && !bad) mbar_arrive(phim);
+
+            if (kCommit) {
+                // ---- state update: S^T tile rows += dS^T rows, a feature half as soon as
+                // the readout has consumed its tiles (first half now, second after R-)
                 const int e = row;
 #pragma unroll 1
                 for (int h = 0; h < 2; ++h) {
-                    bool bad2 = !wait_bar(&dsready[h], kp & 1u, fail);
+                    bool bad2 = bad;
+                    if (h == 1) bad2 = !wait_bar(&dready[kp & 1], (kp >> 1) & 1u, fail);
                     tc_fence_after();
-                    const uint32_t src = (h == 0 ? tmem : tmem + 256 + 128 * ((kp + 1) & 1)) + lane_off;
+                    const uint32_t src = tmem + (h == 0 ? kCmDSp : kCmDSm) + lane_off;
                     auto upd = [&](int k) {
                         const int slot = (q + h * NCH + k) % NS;
                         uint8_t *rowp = ring + (size_t)slot * chunk_bytes + e * 128;
@@ -961,7 +927,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     __syncwarp();
                     if (lane == 0 && !bad2) {
                         mbar_arrive(&tready[h]);
-                        if (h == 1) mbar_arrive(efree);
+                        if (h == 0) mbar_arrive(efree);
                     }
                 }
                 epilogue(kp, q, inv_den);
