@@ -63,6 +63,12 @@ def max_over_ranks(value: float, ws: int, device=None) -> float:
     return float(t.item())
 
 
+def rank_workload(wl, rank: int):
+    """The batch rank `rank` draws: every rank has its own independent requests
+    (weak scaling; no data is exchanged between ranks)."""
+    return wl.with_(seed=wl.seed + 1000 * rank) if rank else wl
+
+
 def barrier(ws: int):
     if ws > 1:
         import torch.distributed as dist
@@ -294,8 +300,7 @@ def run_hybrid(args, wl):
     from paper_2608_06628_gb300.state_pool import StatePool
 
     # each rank draws its own independent batch (weak scaling)
-    if ws > 1:
-        wl = wl.with_(seed=wl.seed + 1000 * rank)
+    wl = rank_workload(wl, rank)
     cfg = H.make_cfg(wl.d, wl.F, wl.Hq, wl.Hkv, wl.B, wl.io_dtype)
     W, alpha = wk.params(wl, device=dev)
     io_bytes = 2 if wl.io_dtype == torch.bfloat16 else 4
@@ -394,21 +399,32 @@ def run_hybrid(args, wl):
     torch.cuda.synchronize()
     direct_ms = (evs[0][0].elapsed_time(evs[-1][1])) / len(evs)
 
-    # context (not part of the value): the step split into its two separate launches
-    def attn_only(s):
-        H.hybrid_block_attn(cfg, s["Q"], s["K"], s["V"], W, alpha, s["ptrs"], wl.n_req, s["O"], sh, check=False)
+    # context (not part of the value): the step split into its two separate
+    # launches, each replayed from a CUDA graph like the timed steps
+    def attn_only(s, st):
+        H.hybrid_block_attn(cfg, s["Q"], s["K"], s["V"], W, alpha, s["ptrs"], wl.n_req, s["O"], st, check=False)
 
-    def commit_only(s):
-        H.hybrid_commit_block(cfg, s["K"], s["V"], wl.B, W, s["ptrs"], wl.n_req, sh, check=False)
+    def commit_only(s, st):
+        H.hybrid_commit_block(cfg, s["K"], s["V"], wl.B, W, s["ptrs"], wl.n_req, st, check=False)
 
-    n_ctx = max(3, min(K_, 200))
-    for fn in (attn_only, commit_only):
-        timed(fn, 3)
-    ev_a = timed(attn_only, n_ctx)
-    ev_c = timed(commit_only, n_ctx)
-    torch.cuda.synchronize()
-    attn_ms = sum(a.elapsed_time(b) for a, b in ev_a) / n_ctx
-    commit_ms = sum(a.elapsed_time(b) for a, b in ev_c) / n_ctx
+    def graph_ms(fn, n_rep=max(1, min(K_, 200) // n_sets)):
+        g_ = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_, stream=side):
+            for i in range(n_sets):
+                fn(sets[i], side.cuda_stream)
+        torch.cuda.synchronize()
+        g_.replay()
+        torch.cuda.synchronize()
+        a_, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a_.record(stream)
+        for _ in range(n_rep):
+            g_.replay()
+        b_.record(stream)
+        torch.cuda.synchronize()
+        return a_.elapsed_time(b_) / (n_rep * n_sets)
+
+    attn_ms = graph_ms(attn_only)
+    commit_ms = graph_ms(commit_only)
 
     # end to end through the public API: pinned host inputs in, output back out
     hQ = sets[0]["Q"].cpu().pin_memory()
