@@ -22,8 +22,9 @@
  *
  * Ownership: the caller allocates every buffer (inputs, outputs, states and
  * the device array of state pointers).  The library allocates no memory in
- * any call; it keeps one 4-byte error word per device in its own static
- * device memory, read back by hybrid_check().
+ * any call.  Its own static device memory, per device, is one 4-byte error word
+ * (read back by hybrid_check()) and the HYBRID_LOGICAL_SCRATCH_BYTES scratch
+ * array used only by hybrid_block_attn_commit_logical().
  *
  * Pointers: every tensor argument is a DEVICE pointer unless stated.  Tensor
  * pointers must be 16-byte aligned (alpha: 4-byte).  d_state_ptrs is a device
@@ -142,6 +143,32 @@ hybrid_status hybrid_block_attn_commit(const hybrid_cfg *cfg, const void *Q, con
                                        const void *V, const void *W, const float *alpha,
                                        void *const *d_state_ptrs, int n_req, void *O,
                                        cudaStream_t stream);
+
+/* Bytes of the library's static scratch for hybrid_block_attn_commit_logical
+ * (64 MiB, part of the library's device image on every device it runs on). */
+#define HYBRID_LOGICAL_SCRATCH_BYTES (64u << 20)
+
+/* hybrid_block_attn_commit on states held in the LOGICAL layout (the paper has
+ * no counterpart: this is an interface convenience for callers that keep
+ * S [n][Hkv][2F][d] and z [n][Hkv][2F] float32 themselves, e.g. states moved in
+ * from another framework).  One call packs the n_req states into the library's
+ * static scratch (operand-image layout, plus the state-pointer array), runs the
+ * fused step and commit there, and unpacks the updated states back in place:
+ *   Q, K, V, W, alpha, O  as in hybrid_block_attn (device pointers)
+ *   S_logical, z_logical  device, read and overwritten with the committed state
+ * It allocates nothing.  Errors: HYBRID_ERR_UNSUPPORTED when
+ * ceil256(8 n_req) + n_req * hybrid_state_bytes(cfg) exceeds
+ * HYBRID_LOGICAL_SCRATCH_BYTES (c3: 64 requests x 528 KB fit); otherwise as
+ * hybrid_block_attn_commit.
+ * Races: the scratch is one per device and shared by every caller, so two calls
+ * must not overlap on a device (issue them on one stream, or synchronise).
+ * Set-up: the first call on a device looks the scratch address up with the CUDA
+ * runtime; make that call (n_req = 0 is enough) before capturing this entry
+ * point in a CUDA graph. */
+hybrid_status hybrid_block_attn_commit_logical(const hybrid_cfg *cfg, const void *Q, const void *K,
+                                               const void *V, const void *W, const float *alpha,
+                                               float *S_logical, float *z_logical, int n_req, void *O,
+                                               cudaStream_t stream);
 
 /* Block commit of Section 3.1: S += sum_t phi(k_t) v_t^T, z += sum_t phi(k_t)
  * over the n_tok tokens of K, V [n][n_tok][Hkv][d] (io_dtype), for every

@@ -35,6 +35,37 @@ unsigned *error_word()
     return p;
 }
 
+// Scratch of hybrid_block_attn_commit_logical: the pointer array and the packed
+// (operand-image) states of one call, in the library's own static device memory.
+constexpr size_t kScratchBytes = (size_t)HYBRID_LOGICAL_SCRATCH_BYTES;
+__device__ __align__(256) unsigned char g_scratch[kScratchBytes];
+std::atomic<unsigned char *> g_scratch_ptr[kMaxDevices];
+
+// Device address of this device's scratch, looked up once per device.
+unsigned char *scratch()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    unsigned char *p = g_scratch_ptr[dev].load(std::memory_order_acquire);
+    if (p) return p;
+    std::lock_guard<std::mutex> lock(g_mu);
+    p = g_scratch_ptr[dev].load(std::memory_order_relaxed);
+    if (!p) {
+        void *sym = nullptr;
+        if (cudaGetSymbolAddress(&sym, g_scratch) != cudaSuccess) return nullptr;
+        p = static_cast<unsigned char *>(sym);
+        g_scratch_ptr[dev].store(p, std::memory_order_release);
+    }
+    return p;
+}
+
+// ptrs[i] = base + i * stride (the state pointers of the scratch slots).
+__global__ void k_fill_ptrs(void **ptrs, unsigned char *base, size_t stride, int n)
+{
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) ptrs[i] = base + (size_t)i * stride;
+}
+
 bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
 hybrid_status check_cfg(const hybrid_cfg *c)
@@ -127,6 +158,33 @@ hybrid_status hybrid_block_attn_commit(const hybrid_cfg *cfg, const void *Q, con
     s = hybrid_block_attn(cfg, Q, K, V, W, alpha, d_state_ptrs, n_req, O, stream);
     if (s != HYBRID_OK) return s;
     return hybrid_commit_block(cfg, K, V, cfg->block_size, W, d_state_ptrs, n_req, stream);
+}
+
+hybrid_status hybrid_block_attn_commit_logical(const hybrid_cfg *cfg, const void *Q, const void *K,
+                                               const void *V, const void *W, const float *alpha,
+                                               float *S_logical, float *z_logical, int n_req, void *O,
+                                               cudaStream_t stream)
+{
+    hybrid_status s = check_cfg(cfg);
+    if (s != HYBRID_OK) return s;
+    if (n_req < 0) return HYBRID_ERR_INVALID_ARG;
+    // the scratch address is looked up here, also for n_req = 0 (set-up call)
+    unsigned char *base = scratch();
+    if (!base) return HYBRID_ERR_CUDA;
+    if (n_req == 0) return HYBRID_OK;
+    if (!S_logical || !z_logical || !aligned(S_logical, 4) || !aligned(z_logical, 4)) return HYBRID_ERR_INVALID_ARG;
+    const size_t sb = hybrid_state_bytes(cfg);   // a multiple of 16 bytes
+    const size_t ptr_bytes = ((size_t)n_req * sizeof(void *) + 255) & ~(size_t)255;
+    if (sb == 0 || (size_t)n_req > (kScratchBytes - ptr_bytes) / sb) return HYBRID_ERR_UNSUPPORTED;
+    void **d_ptrs = reinterpret_cast<void **>(base);
+    unsigned char *states = base + ptr_bytes;
+    k_fill_ptrs<<<(n_req + 127) / 128, 128, 0, stream>>>(d_ptrs, states, sb, n_req);
+    if (cudaGetLastError() != cudaSuccess) return HYBRID_ERR_CUDA;
+    s = hybrid_state_pack(cfg, S_logical, z_logical, d_ptrs, n_req, stream);
+    if (s != HYBRID_OK) return s;
+    s = hybrid_block_attn_commit(cfg, Q, K, V, W, alpha, d_ptrs, n_req, O, stream);
+    if (s != HYBRID_OK) return s;
+    return hybrid_state_unpack(cfg, d_ptrs, n_req, S_logical, z_logical, stream);
 }
 
 hybrid_status hybrid_commit_block(const hybrid_cfg *cfg, const void *K, const void *V, int n_tok,

@@ -25,7 +25,7 @@ HYBRID_BF16 = 1
 
 EXPORTED = (
     "hybrid_state_bytes", "hybrid_state_init", "hybrid_feature_map", "hybrid_block_attn",
-    "hybrid_block_attn_commit", "hybrid_commit_block", "hybrid_state_unpack", "hybrid_state_pack", "hybrid_check",
+    "hybrid_block_attn_commit", "hybrid_block_attn_commit_logical", "hybrid_commit_block", "hybrid_state_unpack", "hybrid_state_pack", "hybrid_check",
     "hybrid_status_str",
 )
 
@@ -72,6 +72,7 @@ def lib(path: str | None = None):
     L.hybrid_feature_map.argtypes = [cfgp, P, I, I, P, P, P]
     L.hybrid_block_attn.argtypes = [cfgp, P, P, P, P, P, P, I, P, P]
     L.hybrid_block_attn_commit.argtypes = [cfgp, P, P, P, P, P, P, I, P, P]
+    L.hybrid_block_attn_commit_logical.argtypes = [cfgp, P, P, P, P, P, P, P, I, P, P]
     L.hybrid_commit_block.argtypes = [cfgp, P, P, I, P, P, I, P]
     L.hybrid_state_unpack.argtypes = [cfgp, P, I, P, P, P]
     L.hybrid_state_pack.argtypes = [cfgp, P, P, P, I, P]
@@ -146,6 +147,14 @@ def hybrid_block_attn_commit(cfg, Q, K, V, W, alpha, state_ptrs, n_req, O, strea
                                         _ptr(alpha), _ptr(state_ptrs), int(n_req), _ptr(O),
                                         _stream(stream))
     return _ret(st, "hybrid_block_attn_commit", check)
+
+
+def hybrid_block_attn_commit_logical(cfg, Q, K, V, W, alpha, S_logical, z_logical, n_req, O, stream=None,
+                                     check=True):
+    st = lib().hybrid_block_attn_commit_logical(ctypes.byref(cfg), _ptr(Q), _ptr(K), _ptr(V), _ptr(W),
+                                                _ptr(alpha), _ptr(S_logical), _ptr(z_logical), int(n_req),
+                                                _ptr(O), _stream(stream))
+    return _ret(st, "hybrid_block_attn_commit_logical", check)
 
 
 def hybrid_commit_block(cfg, K, V, n_tok, W, state_ptrs, n_req, stream=None, check=True):
