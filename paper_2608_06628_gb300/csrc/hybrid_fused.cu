@@ -343,6 +343,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     }
     __syncthreads();
     tc_fence_after();
+    // launched with programmatic stream serialisation: the set-up above may run
+    // while the previous kernel of the stream drains; nothing below touches
+    // global memory before that kernel has completed
+    if (tid == 0) griddep_launch_dependents();
+    griddep_wait();
     const uint32_t tmem = *tmem_holder;
     uint8_t *ring = smem;
     float *zbuf0 = reinterpret_cast<float *>(smem + a.off_z);
@@ -1068,9 +1073,17 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
         if (e != cudaSuccess) return e;
         opted[commit].fetch_or(bit, std::memory_order_release);
     }
-    if (commit) k_fused<true><<<grid, kThreads, L.bytes, st>>>(a);
-    else k_fused<false><<<grid, kThreads, L.bytes, st>>>(a);
-    return cudaGetLastError();
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid);
+    lc.blockDim = dim3(kThreads);
+    lc.dynamicSmemBytes = L.bytes;
+    lc.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 1;
+    return commit ? cudaLaunchKernelEx(&lc, k_fused<true>, a) : cudaLaunchKernelEx(&lc, k_fused<false>, a);
 }
 
 }  // namespace hyb
