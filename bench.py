@@ -109,7 +109,7 @@ def recorded_traffic(kernel: str, workload: str):
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons, sampled every 100 ms."""
+    """nvidia-smi clocks and throttle reasons, sampled every 50 ms."""
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
@@ -122,7 +122,7 @@ class ClockSampler:
         self.thread = None
 
     def start(self):
-        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "100"]
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "50"]
         if self.bus_id:
             cmd += ["-i", self.bus_id]
         try:
@@ -160,7 +160,7 @@ class ClockSampler:
         window = "timed region"
         if not inside:
             inside = [s for s in self.samples if t0 - 2.0 <= s[0] <= t1 + 0.5]
-            window = "timed region +-2 s (timed region shorter than the 100 ms sampling period)"
+            window = "timed region +-2 s (timed region shorter than the 50 ms sampling period)"
         if not inside:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0,
                     "window": "no nvidia-smi samples"}
@@ -506,8 +506,8 @@ def run_hybrid(args, wl):
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=3000)
-    ap.add_argument("--warmup", type=int, default=30)
+    ap.add_argument("--steps", type=int, default=30000)
+    ap.add_argument("--warmup", type=int, default=50)
     ap.add_argument("--impl", choices=("hybrid", "reference"), default="hybrid")
     ap.add_argument("--config", default="c3_bf16_b64_gqa_ragged")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -318,6 +318,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + n_bars);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
+    if (warp == 2 && lane == 0) {
+        prefetch_tensormap(&a.tmQ);
+        prefetch_tensormap(&a.tmW);
+        prefetch_tensormap(&a.tmV);
+    }
+    if (warp == 3 && lane == 0) prefetch_tensormap(&a.tmO);
     if (tid == 0) {
         for (int i = 0; i < n_bars; ++i) mbar_init(&bars[i], 1);
         mbar_init(xfull, 2);
@@ -777,12 +783,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     // unnormalised phi(K) of this thread's feature for every token
                     float uk[32];
                     tmem_ld32(kcol, uk);
+                    // lane t combines token t's extremum over the four feature quarters
+                    float m_l;
+                    {
+                        const float4 x = *reinterpret_cast<const float4 *>(&tk[(part * 32 + lane) * 4]);
+                        m_l = fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w)) * kLog2e;
+                    }
                     tmem_wait_ld();
+                    const float sgn = part == 0 ? kLog2e : -kLog2e;
 #pragma unroll
                     for (int t = 0; t < 32; ++t) {
-                        const float4 x = *reinterpret_cast<const float4 *>(&tk[(part * 32 + t) * 4]);
-                        const float m = fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w));
-                        ek[t] = fval ? ex2(((part == 0 ? uk[t] : -uk[t]) - m) * kLog2e) : 0.f;
+                        const float m = __shfl_sync(0xffffffffu, m_l, t);
+                        ek[t] = fval ? ex2(fmaf(uk[t], sgn, -m)) : 0.f;
                         uk[t] = ek[t];
                     }
                     const float ssum = warp_reduce32<0>(uk, lane);

@@ -230,6 +230,12 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float (&v)[32])
         : "memory");
 }
 
+// Bring a tensor-map descriptor (kernel parameter) into the descriptor cache.
+__device__ __forceinline__ void prefetch_tensormap(const void *tmap)
+{
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
+}
+
 // Programmatic dependent launch: let the next kernel of the stream start its
 // prologue once every CTA of this grid has signalled (or exited), and wait
 // until the previous grid has completed and its writes are visible.
