@@ -33,7 +33,10 @@
 // and PV, and out = D / den afterwards.  Merge: with sigma the log of the
 // larger branch mass, phi' = phi e^-sigma and P' = w e^(s - sigma), so
 // D / den = (w sm_num + lin_num) / (w sm_den + lin_den) exactly, with
-// den = e^(log lin_den - sigma) + e^(log(w sm_den) - sigma) in [1, 2].
+// den = e^(log lin_den - sigma) + e^(log(w sm_den) - sigma) in [1, 2].  While
+// the unshifted softmax mass w sp e^s of a warp's rows stays below e^60, the
+// kernel accumulates D / kappa (kappa = e^-sigma / sp) instead, so phi+ needs
+// no rescaling in Tensor Memory; kappa is folded into 1 / den.
 //
 // A unit's phi+ and phi- share its F phi columns: phi- waits in registers until
 // R+ has consumed phi+.  Step: Tensor Memory holds two unit slots of 256
@@ -285,8 +288,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     const int NCH = F / 32;          // 32-feature chunks (state tiles) per half of phi
     const int NC = 2 * NCH;          // state tiles per unit
     // the output tile is staged in the slots of tiles ocm, ocm + 1 of its unit:
-    // with the commit, first-half tiles that no later tile of the unit reuses;
-    // without, the last two
+    // with the commit, first-half tiles that no later tile of the unit reuses
+    // (drained before the epilogue); without, the last two
     const int ocm = kCommit ? (NC > NS ? NC - NS : 0) : NC - 2;
     const uint32_t chunk_bytes = (uint32_t)d * 128;
     const int per = a.n_units / (int)gridDim.x, rem = a.n_units % (int)gridDim.x;
@@ -828,21 +831,36 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 const float log_l = logf(lin_den);                   // log(lin_den), -inf if empty
                 const float sig = fmaxf(fmaxf(log_s, log_l), -60.f);
                 const float esig = expf(-sig);
-                const float cpos = lin_den > 0.f ? esig / sp : 0.f;
-                cneg = lin_den > 0.f ? esig / sn : 0.f;
-                auto scale_chunk = [&](uint32_t col) {
-                    float v[32];
-                    tmem_ld32(col, v);
-                    tmem_wait_ld();
+                // Accumulate D / kappa with kappa = e^-sigma / sp: phi+ then stays
+                // unnormalised in Tensor Memory (no rescale pass) and phi- (in
+                // registers) and P' absorb the factor (phi- x sp/sn, P' = w sp e^s).
+                // This needs the unshifted softmax mass w sp e^(s) inside float
+                // range; a warp with any row beyond e^60 rescales phi+ instead.
+                const bool fast = __all_sync(0xffffffffu, !(lw + ms * a.scale + logf(sp) > 60.f));
+                float kappa, pofs;
+                if (fast) {
+                    kappa = esig / sp;
+                    cneg = lin_den > 0.f ? sp / sn : 0.f;
+                    pofs = (lw + logf(sp)) * kLog2e;
+                } else {
+                    const float cpos = lin_den > 0.f ? esig / sp : 0.f;
+                    cneg = lin_den > 0.f ? esig / sn : 0.f;
+                    kappa = 1.f;
+                    pofs = (lw - sig) * kLog2e;
+                    auto scale_chunk = [&](uint32_t col) {
+                        float v[32];
+                        tmem_ld32(col, v);
+                        tmem_wait_ld();
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] *= cpos;
-                    tmem_st32(col, v);
-                };
-                scale_chunk(pcol + 32 * part);
-                if (two) scale_chunk(pcol + 32 * (part + 2));
+                        for (int i = 0; i < 32; ++i) v[i] *= cpos;
+                        tmem_st32(col, v);
+                    };
+                    scale_chunk(pcol + 32 * part);
+                    if (two) scale_chunk(pcol + 32 * (part + 2));
+                }
                 if (has_sc) {
-                    // P' = w e^(s - sigma): K-major, no swizzle (8-row x 16-byte core matrices)
-                    const float pofs = (lw - sig) * kLog2e;
+                    // P' (w e^(s - sigma), or w sp e^s on the fast path): K-major, no swizzle
+                    // (8-row x 16-byte core matrices)
                     uint32_t pk[8];
 #pragma unroll
                     for (int i = 0; i < 16; i += 2)
@@ -851,7 +869,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     *reinterpret_cast<uint4 *>(prow + (2 * part) * 128) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
                     *reinterpret_cast<uint4 *>(prow + (2 * part + 1) * 128) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                 }
-                inv_den = 1.f / (expf(log_l - sig) + expf(log_s - sig));
+                inv_den = kappa / (expf(log_l - sig) + expf(log_s - sig));
                 if (kCommit) {
                     // phi(K) normalised, as the bf16 MN-major operand [token][feature]
                     // (64-feature atoms of B rows), and z[part*F + row] += sum_t phi(k_t)

@@ -136,6 +136,7 @@ def test_state_init_zeroes():
 # edge cases
 # ---------------------------------------------------------------------------
 EDGE_WL = [W_("edge_gqa_bf16", BF16, 3, 8, 2, 128, 128, 32, 31),
+           W_("edge_gqa_k24_bf16", BF16, 3, 8, 2, 128, 128, 32, 33, k_scale=24.0),
            W_("edge_f32", F32, 2, 2, 2, 64, 64, 16, 32)]
 
 
@@ -281,6 +282,8 @@ FUSED = [
     (W_("fused_mha_d64_f64", BF16, 3, 4, 4, 64, 64, 32, 52), [64, 0, 32]),
     (W_("fused_gqa4_many_units", BF16, 40, 16, 4, 128, 128, 32, 53), None),   # 160 units > 152 SMs
     (W_("fused_b16_fallback", BF16, 3, 4, 2, 128, 128, 16, 54), [16, 0, 48]),  # B != 32: step + commit
+    # keys x24: scores near 60 make some warps take the exact phi+ rescale
+    (W_("fused_gqa4_k24", BF16, 3, 8, 2, 128, 128, 32, 56, k_scale=24.0), [32, 0, 96]),
 ]
 
 
