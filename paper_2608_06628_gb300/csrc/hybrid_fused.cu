@@ -18,7 +18,7 @@
 //   warp 2     producer: TMA of Q and W, the transposed key tile K^T (built by
 //              the warp from global memory) and V, one unit ahead.
 //   warp 3     storer: TMA stores of the output tile and, with the commit, bulk
-//              stores of the updated state tiles and z.
+//              reduce-adds of the dS^T tiles into the state, and the store of z.
 //   warps 4-11 math: two threads per query row (one per TMEM lane and "part");
 //              a part owns every other 32-feature chunk of each half of phi.
 //
@@ -594,7 +594,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     for (int h = 0; h < 2 && ok; ++h) {
                         if (!wait_bar(&tready[h], kp & 1u, fail)) { ok = false; break; }
                         for (int c = h * NCH; c < (h + 1) * NCH; ++c)
-                            bulk_s2g(Sg + (size_t)c * 32 * d, ring + (size_t)((q + c) % NS) * chunk_bytes, chunk_bytes);
+                            bulk_reduce_add_f32(Sg + (size_t)c * 32 * d, ring + (size_t)((q + c) % NS) * chunk_bytes,
+                                                chunk_bytes);
                         bulk_commit();
                         bulk_wait_read_all();
                         for (int c = h * NCH; c < (h + 1) * NCH; ++c)
@@ -920,8 +921,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             if (lane == 0 && !bad) mbar_arrive(phim);
 
             if (kCommit) {
-                // ---- state update: S^T tile rows += dS^T rows, a feature half as soon as
-                // the readout has consumed its tiles (first half now, second after R-)
+                // ---- state update: S^T += dS^T for a feature half as soon as the readout
+                // has consumed its tiles (first half now, second after R-): dS^T rows go
+                // into the tiles' slots and the storer adds them into the state by
+                // bulk reductions (float32 add at L2)
                 const int e = row;
 #pragma unroll 1
                 for (int h = 0; h < 2; ++h) {
@@ -930,29 +933,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     tc_fence_after();
                     const uint32_t src = tmem + (h == 0 ? kCmDSp : kCmDSm) + lane_off;
                     auto upd = [&](int k) {
-                        const int slot = (q + h * NCH + k) % NS;
-                        uint8_t *rowp = ring + (size_t)slot * chunk_bytes + e * 128;
-#pragma unroll 1
-                        for (int hh = 0; hh < 2; ++hh) {   // 16 features (4 granules) at a time
-                            float v[16];
-                            tmem_ld16(src + 32 * k + 16 * hh, v);
-                            float4 s4[4];
-                            if (e < d) {
+                        // the readout has consumed the tile: its slot now takes dS^T,
+                        // which the storer adds into the state in global memory
+                        uint8_t *rowp = ring + (size_t)((q + h * NCH + k) % NS) * chunk_bytes + e * 128;
+                        float v[32];
+                        tmem_ld32(src + 32 * k, v);
+                        tmem_wait_ld();
+                        if (!bad2 && e < d) {
 #pragma unroll
-                                for (int gq = 0; gq < 4; ++gq)
-                                    s4[gq] = *reinterpret_cast<const float4 *>(rowp + (((4 * hh + gq) ^ (e & 7)) << 4));
-                            }
-                            tmem_wait_ld();
-                            if (!bad2 && e < d) {
-#pragma unroll
-                                for (int gq = 0; gq < 4; ++gq) {
-                                    s4[gq].x += v[4 * gq];
-                                    s4[gq].y += v[4 * gq + 1];
-                                    s4[gq].z += v[4 * gq + 2];
-                                    s4[gq].w += v[4 * gq + 3];
-                                    *reinterpret_cast<float4 *>(rowp + (((4 * hh + gq) ^ (e & 7)) << 4)) = s4[gq];
-                                }
-                            }
+                            for (int gq = 0; gq < 8; ++gq)
+                                *reinterpret_cast<float4 *>(rowp + ((gq ^ (e & 7)) << 4)) =
+                                    make_float4(v[4 * gq], v[4 * gq + 1], v[4 * gq + 2], v[4 * gq + 3]);
                         }
                     };
 #pragma unroll 1

@@ -123,6 +123,15 @@ __device__ __forceinline__ void bulk_s2g(void *dst, const void *src, uint32_t by
                  "r"(bytes)
                  : "memory");
 }
+// global[dst, dst + bytes) += shared[src, ...) as float32, element-wise, by the
+// bulk-copy engine (a reduction at L2); both addresses 16-byte aligned, bytes a
+// multiple of 16; completes as a bulk group like bulk_s2g.
+__device__ __forceinline__ void bulk_reduce_add_f32(void *dst, const void *src, uint32_t bytes)
+{
+    asm volatile("cp.reduce.async.bulk.global.shared::cta.bulk_group.add.f32 [%0], [%1], %2;" ::"l"(dst),
+                 "r"(smem_u32(src)), "r"(bytes)
+                 : "memory");
+}
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
