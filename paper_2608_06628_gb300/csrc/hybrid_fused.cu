@@ -593,14 +593,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     mbar_arrive(&zempty[zb]);
                     for (int h = 0; h < 2 && ok; ++h) {
                         if (!wait_bar(&tready[h], kp & 1u, fail)) { ok = false; break; }
-                        for (int c = h * NCH; c < (h + 1) * NCH; ++c)
+                        // one bulk group per tile; the two output slots (first in
+                        // the first half) are freed as soon as their reductions have read them
+                        for (int c = h * NCH; c < (h + 1) * NCH; ++c) {
                             bulk_reduce_add_f32(Sg + (size_t)c * 32 * d, ring + (size_t)((q + c) % NS) * chunk_bytes,
                                                 chunk_bytes);
-                        bulk_commit();
+                            bulk_commit();
+                        }
+                        if (h == 0) {
+                            // groups issued after the two output tiles: NCH - ocm - 2
+                            if (NCH - ocm - 2 >= 2) bulk_wait_read_2();
+                            else bulk_wait_read_all();
+                            mbar_arrive(ofree);
+                        }
                         bulk_wait_read_all();
                         for (int c = h * NCH; c < (h + 1) * NCH; ++c)
                             if (c < ocm || c > ocm + 1) mbar_arrive(&empty[(q + c) % NS]);
-                        if (h == 0) mbar_arrive(ofree);
                     }
                     if (!ok) break;
                 }
