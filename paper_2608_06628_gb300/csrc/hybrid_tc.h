@@ -25,4 +25,10 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
                          const void *W, const float *alpha, void *const *states, int n_req, void *O,
                          unsigned *err, cudaStream_t st);
 
+// Commit / prefill as a reduction (hybrid_commit_red.cu): S += dS and z += dz are
+// added into the state in global memory by bulk reduce-adds; any n_tok >= 1.
+bool commit_red_supported(const hybrid_cfg &c);
+cudaError_t launch_commit_red(const hybrid_cfg &c, const void *K, const void *V, int n_tok, const void *W,
+                              void *const *states, int n_req, unsigned *err, cudaStream_t st);
+
 }  // namespace hyb
