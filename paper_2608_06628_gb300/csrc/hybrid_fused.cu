@@ -180,13 +180,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint64_t *uready = vfree + 1;     // MMA -> math: g1 done
     uint64_t *phip = uready + 1;      // math -> MMA: phi+ and P' (with the commit also phi(K))
     uint64_t *phim = phip + 1;        // math -> MMA: phi- in the phi columns
-    uint64_t *pread = phim + 1;       // MMA -> math: R+ has consumed phi+ (and dS^T is formed)
-    uint64_t *efree = pread + 1;      // math -> MMA: the first-half update has read dS+ (commit)
+    uint64_t *pread = phim + 1;       // MMA -> math: R+ has consumed phi+
+    uint64_t *pready = pread + 1;     // math -> MMA: P' (and, with the commit, phi(K)) is written
+    uint64_t *dsdone = pready + 1;    // MMA -> math: dS^T is formed (commit)
+    uint64_t *efree = dsdone + 1;     // math -> MMA: the first-half update has read dS+ (commit)
     uint64_t *zdone = efree + 1;      // math -> storer: z is updated (commit)
     uint64_t *ofree = zdone + 1;      // storer -> math: the output slots may be written (commit)
     uint64_t *ostaged = ofree + 1;    // math -> storer: the output tile is in its slots
     uint64_t *mmadone = ostaged + 1;
-    const int n_bars = 2 * NS + 10 + 13;
+    const int n_bars = 2 * NS + 10 + 15;
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + n_bars);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
@@ -201,6 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         mbar_init(xfull, 2);
         mbar_init(phip, 8);
         mbar_init(phim, 8);
+        mbar_init(pready, 8);
         mbar_init(efree, 8);
         mbar_init(zdone, 8);
         mbar_init(ostaged, 8);
@@ -290,22 +293,25 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     }
                 }
             };
+            // P'V accumulates onto the phi+ readout
             auto pv = [&](uint32_t dcol) {
                 for (int k = 0; k < B / 16; ++k) {
                     const uint64_t ap = smem_desc(p_u + k * 256, 128, (B / 8) * 128, SWZ_NONE);
                     const uint64_t bv = smem_desc(vb_u + 2 * k * 1024, B * 128, 1024, SWZ_128B);
-                    mma_bf16_ss(tmem + dcol, ap, bv, idP, k > 0);
+                    mma_bf16_ss(tmem + dcol, ap, bv, idP, 1);
                 }
             };
             // readout of state tile c (global tile counter qt + c) with phi columns acol
-            auto readout = [&](uint32_t dcol, uint32_t acol, uint32_t qc) -> int {
+            // (first: the tile's first MMA initialises the accumulator)
+            auto readout = [&](uint32_t dcol, uint32_t acol, uint32_t qc, bool first = false) -> int {
                 const int slot = qc % NS;
                 if (!wait_bar(&full[slot], (qc / NS) & 1u, fail)) return -1;
                 tc_fence_after();
                 const uint32_t s_u = ring_u + slot * chunk_bytes;
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk)
-                    mma_tf32_ts(tmem + dcol, tmem + acol + 8 * kk, smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B), idR, 1);
+                    mma_tf32_ts(tmem + dcol, tmem + acol + 8 * kk, smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B), idR,
+                                !(first && kk == 0));
                 return slot;
             };
             auto ds = [&](uint32_t dcol, int h) {
@@ -332,6 +338,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     mma_commit(&dready[ik & 1]);
                     return true;
                 };
+                // P'V and R- of the previous unit: its P' and phi- come last
+                auto finish = [&](uint32_t ik, uint32_t iq) -> bool {
+                    if (!wait_bar(pready, ik & 1u, fail) || !wait_bar(vfull, ik & 1u, fail)) return false;
+                    tc_fence_after();
+                    pv((ik & 1) * 256 + 128);
+                    mma_commit(vfree);
+                    return tail(ik, iq);
+                };
                 for (int u = u_begin; u < u_end; ++u) {
                     if (!unit_state(a, u)) continue;
                     const uint32_t T = (kp & 1) * 256;
@@ -341,13 +355,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     g1(T, 0);
                     mma_commit(uready);
                     mma_commit(xfree);
-                    if (kp >= 1 && !tail(kp - 1, prev_qt)) { ok = false; break; }
-                    if (!wait_bar(phip, kp & 1u, fail) || !wait_bar(vfull, kp & 1u, fail)) { ok = false; break; }
+                    if (kp >= 1 && !finish(kp - 1, prev_qt)) { ok = false; break; }
+                    if (!wait_bar(phip, kp & 1u, fail)) { ok = false; break; }
                     tc_fence_after();
-                    pv(T + 128);
-                    mma_commit(vfree);
                     for (int c = 0; c < NCH; ++c) {
-                        const int slot = readout(T + 128, T + 32 * c, qt + c);
+                        const int slot = readout(T + 128, T + 32 * c, qt + c, c == 0);
                         if (slot < 0) { ok = false; break; }
                         mma_commit(&empty[slot]);
                     }
@@ -357,7 +369,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     qt += NC;
                     ++kp;
                 }
-                if (ok && kp >= 1) tail(kp - 1, prev_qt);
+                if (ok && kp >= 1) finish(kp - 1, prev_qt);
             } else {
                 // Tensor Memory: [0,128) D, [128,128+F) phi (U, then phi+, then phi-),
                 // scores after U, [256,256+F) dS+ (U_k^T at 288 until then),
@@ -374,14 +386,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     mma_commit(uready);
                     mma_commit(xfree);
                     // phip also covers the previous unit's output epilogue and second-half update
-                    if (!wait_bar(phip, kp & 1u, fail) || !wait_bar(vfull, kp & 1u, fail)) { ok = false; break; }
+                    if (!wait_bar(phip, kp & 1u, fail)) { ok = false; break; }
+                    tc_fence_after();
+                    for (int c = 0; c < NCH && ok; ++c) ok = readout(kCmD, kCmP + 32 * c, qt + c, c == 0) >= 0;
+                    if (!ok) break;
+                    mma_commit(pread);
+                    if (!wait_bar(pready, kp & 1u, fail) || !wait_bar(vfull, kp & 1u, fail)) { ok = false; break; }
                     tc_fence_after();
                     ds(kCmDSp, 0);
                     ds(kCmDSm, 1);
                     pv(kCmD);
-                    for (int c = 0; c < NCH && ok; ++c) ok = readout(kCmD, kCmP + 32 * c, qt + c) >= 0;
-                    if (!ok) break;
-                    mma_commit(pread);
+                    mma_commit(dsdone);
                     if (!wait_bar(phim, kp & 1u, fail)) { ok = false; break; }
                     tc_fence_after();
                     for (int c = NCH; c < NC && ok; ++c) ok = readout(kCmD, kCmP + 32 * (c - NCH), qt + c) >= 0;
@@ -419,7 +434,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             __syncwarp();
             // with the commit the Q region holds the previous unit's V, P' and phi(K)
             // until its dS^T and P V have run
-            if (kCommit && kp > 0) ok = wait_bar(pread, (kp - 1) & 1u, fail);
+            if (kCommit && kp > 0) ok = wait_bar(dsdone, (kp - 1) & 1u, fail);
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
                 for (int e = 0; e < d / 64; ++e)
@@ -513,8 +528,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         const bool valid = row < Mv;
         const bool fval = row < F;
         float *xa = reinterpret_cast<float *>(smem + a.off_st);   // [part][ms, mx, mn][128]
-        float *xb = xa + 6 * 128;                                  // [part][l, sp, sn, lp, ln][128]
-        float *tk = xb + 10 * 128;                                 // token statistics (commit)
+        float *xs = xa + 6 * 128;                                  // [part][sp][128]
+        float *xb = xs + 2 * 128;                                  // [part][l, lp, sn, ln][128]
+        float *tk = xb + 8 * 128;                                  // token statistics (commit)
         uint8_t *pkb = smem + a.off_pk;
         const float scale_l2 = a.scale * kLog2e;
         const uint32_t pair_bar = kBarPair + q4;
@@ -624,42 +640,78 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             const float mx = fmaxf(xa[1 * 128 + row], xa[4 * 128 + row]);
             const float mn = fminf(xa[2 * 128 + row], xa[5 * 128 + row]);
 
-            // ---- phase B: exponentials; phi+ unnormalised into Tensor Memory, phi- kept
-            // in registers until R+ has consumed phi+; commit: unnormalised phi(K)
+            // ---- phase B1: phi+ (unnormalised) into Tensor Memory; once the row sums are
+            // exchanged, R+ may start on it (unless the warp needs the exact rescale)
             bad = !wait_bar(&zfull[zb], (kp >> 1) & 1u, fail);
-            float ek[32];   // commit: unnormalised phi(K) of feature part*F + row, per token
+            const float mxl = mx * kLog2e, mnl = mn * kLog2e, ml = ms * scale_l2;
+            const float lw = valid ? log_sigmoid(alpha_row) : 0.f;
+            float lp = 0.f;
             {
-                const float mxl = mx * kLog2e, mnl = mn * kLog2e, ml = ms * scale_l2;
-                float l = 0.f, sp = 0.f, sn = 0.f, lp = 0.f, ln = 0.f;
-                if (has_sc) {
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) l += ex2(fmaf(sc[i], scale_l2, -ml));
-                }
-                auto exps = [&](float (&uu)[32], int k) {
+                float sp = 0.f;
+                auto expp = [&](const float (&uu)[32], int k) {
                     float ep[32];
                     const float4 *zp = reinterpret_cast<const float4 *>(zs + 32 * k);
-                    const float4 *zn = reinterpret_cast<const float4 *>(zs + F + 32 * k);
 #pragma unroll
                     for (int i4 = 0; i4 < 8; ++i4) {
-                        const float4 a4 = zp[i4], b4 = zn[i4];
-                        const float za[4] = {a4.x, a4.y, a4.z, a4.w}, zn4[4] = {b4.x, b4.y, b4.z, b4.w};
+                        const float4 a4 = zp[i4];
+                        const float za[4] = {a4.x, a4.y, a4.z, a4.w};
 #pragma unroll
                         for (int j = 0; j < 4; ++j) {
                             const int i = 4 * i4 + j;
                             const float e = ex2(fmaf(uu[i], kLog2e, -mxl));
-                            const float en = ex2(fmaf(-uu[i], kLog2e, mnl));
                             ep[i] = e;
-                            uu[i] = en;
                             sp += e;
-                            sn += en;
                             lp = fmaf(e, za[j], lp);
-                            ln = fmaf(en, zn4[j], ln);
                         }
                     }
                     tmem_st32(pcol + 32 * k, ep);
                 };
-                exps(u0, part);
-                if (two) exps(u1, part + 2);
+                expp(u0, part);
+                if (two) expp(u1, part + 2);
+                xs[part * 128 + row] = sp;
+            }
+            if (sync_failed(bad)) { ok = false; break; }
+            const float sp = xs[row] + xs[128 + row];
+            // Accumulate D / kappa with kappa = e^-sigma / sp: phi+ then stays
+            // unnormalised in Tensor Memory (no rescale pass) and phi- (in registers)
+            // and P' absorb the factor (phi- x sp/sn, P' = w sp e^s).  This needs the
+            // unshifted softmax mass w sp e^(s) inside float range; a warp with any row
+            // beyond e^60 rescales phi+ exactly once sigma is known (phase C).
+            const bool fast = __all_sync(0xffffffffu, !(lw + ms * a.scale + logf(sp) > 60.f));
+            if (fast) {
+                tmem_wait_st();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(phip);
+            }
+
+            // ---- phase B2: phi- (kept in registers until R+ has consumed phi+), the
+            // score sums; commit: unnormalised phi(K)
+            float ek[32];   // commit: unnormalised phi(K) of feature part*F + row, per token
+            {
+                float l = 0.f, sn = 0.f, ln = 0.f;
+                if (has_sc) {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) l += ex2(fmaf(sc[i], scale_l2, -ml));
+                }
+                auto expm = [&](float (&uu)[32], int k) {
+                    const float4 *zn = reinterpret_cast<const float4 *>(zs + F + 32 * k);
+#pragma unroll
+                    for (int i4 = 0; i4 < 8; ++i4) {
+                        const float4 b4 = zn[i4];
+                        const float zn4[4] = {b4.x, b4.y, b4.z, b4.w};
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const int i = 4 * i4 + j;
+                            const float en = ex2(fmaf(-uu[i], kLog2e, mnl));
+                            uu[i] = en;
+                            sn += en;
+                            ln = fmaf(en, zn4[j], ln);
+                        }
+                    }
+                };
+                expm(u0, part);
+                if (two) expm(u1, part + 2);
                 if (kCommit) {
                     // unnormalised phi(K) of this thread's feature for every token
                     float uk[32];
@@ -681,12 +733,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     const float ssum = warp_reduce32<0>(uk, lane);
                     tk[((2 + part) * 32 + lane) * 4 + q4] = ssum;
                 }
-                xb[(part * 5 + 0) * 128 + row] = l;
-                xb[(part * 5 + 1) * 128 + row] = sp;
-                xb[(part * 5 + 2) * 128 + row] = sn;
-                xb[(part * 5 + 3) * 128 + row] = lp;
-                xb[(part * 5 + 4) * 128 + row] = ln;
-                tmem_wait_st();
+                xb[(part * 4 + 0) * 128 + row] = l;
+                xb[(part * 4 + 1) * 128 + row] = lp;
+                xb[(part * 4 + 2) * 128 + row] = sn;
+                xb[(part * 4 + 3) * 128 + row] = ln;
             }
             if (!kCommit) {
                 // z has been read
@@ -695,26 +745,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             }
             if (sync_failed(bad)) { ok = false; break; }
 
-            // ---- phase C: sigma, phi+ scaled in place, P', den; commit: phi(K), z
+            // ---- phase C: sigma, P', den (and, off the fast path, phi+ rescaled);
+            // commit: phi(K), z
             float cneg, inv_den;
             {
-                const float l = xb[0 * 128 + row] + xb[5 * 128 + row];
-                const float sp = xb[1 * 128 + row] + xb[6 * 128 + row];
-                const float sn = xb[2 * 128 + row] + xb[7 * 128 + row];
-                const float lp = xb[3 * 128 + row] + xb[8 * 128 + row];
-                const float ln = xb[4 * 128 + row] + xb[9 * 128 + row];
-                const float lin_den = lp / sp + ln / sn;
-                const float lw = valid ? log_sigmoid(alpha_row) : 0.f;
+                const float l = xb[0 * 128 + row] + xb[4 * 128 + row];
+                const float lpf = xb[1 * 128 + row] + xb[5 * 128 + row];
+                const float sn = xb[2 * 128 + row] + xb[6 * 128 + row];
+                const float ln = xb[3 * 128 + row] + xb[7 * 128 + row];
+                const float lin_den = lpf / sp + ln / sn;
                 const float log_s = lw + ms * a.scale + logf(l);   // log(w sm_den)
                 const float log_l = logf(lin_den);                   // log(lin_den), -inf if empty
                 const float sig = fmaxf(fmaxf(log_s, log_l), -60.f);
                 const float esig = expf(-sig);
-                // Accumulate D / kappa with kappa = e^-sigma / sp: phi+ then stays
-                // unnormalised in Tensor Memory (no rescale pass) and phi- (in
-                // registers) and P' absorb the factor (phi- x sp/sn, P' = w sp e^s).
-                // This needs the unshifted softmax mass w sp e^(s) inside float
-                // range; a warp with any row beyond e^60 rescales phi+ instead.
-                const bool fast = __all_sync(0xffffffffu, !(lw + ms * a.scale + logf(sp) > 60.f));
                 float kappa, pofs;
                 if (fast) {
                     kappa = esig / sp;
@@ -735,7 +778,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     };
                     scale_chunk(pcol + 32 * part);
                     if (two) scale_chunk(pcol + 32 * (part + 2));
+                    tmem_wait_st();
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(phip);
                 }
+                // step: the previous unit's P'V (issued after this unit's g1) has read P'
+                if (!kCommit && kp >= 1) bad = !wait_bar(vfree, (kp - 1) & 1u, fail) || bad;
                 if (has_sc) {
                     // P' (w e^(s - sigma), or w sp e^s on the fast path): K-major, no swizzle
                     // (8-row x 16-byte core matrices)
@@ -769,13 +818,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     }
                     if (fval) zs[f] += dz;
                 }
-                tmem_wait_st();
             }
-            tc_fence_before();
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {
-                mbar_arrive(phip);
+                mbar_arrive(pready);
                 if (kCommit) mbar_arrive(zdone);
             }
 
@@ -805,8 +852,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 const int e = row;
 #pragma unroll 1
                 for (int h = 0; h < 2; ++h) {
-                    bool bad2 = bad;
-                    if (h == 1) bad2 = !wait_bar(&dready[kp & 1], (kp >> 1) & 1u, fail);
+                    const bool bad2 = h == 0 ? !wait_bar(dsdone, kp & 1u, fail) || bad
+                                             : !wait_bar(&dready[kp & 1], (kp >> 1) & 1u, fail);
                     tc_fence_after();
                     const uint32_t src = tmem + (h == 0 ? kCmDSp : kCmDSm) + lane_off;
                     auto upd = [&](int k) {
