@@ -202,8 +202,6 @@ hybrid_status hybrid_commit_block(const hybrid_cfg *cfg, const void *K, const vo
     if (!err) return HYBRID_ERR_CUDA;
     if (hyb::commit_red_supported(*cfg))
         return from_cuda(hyb::launch_commit_red(*cfg, K, V, n_tok, W, d_state_ptrs, n_req, err, stream));
-    if (hyb::tc_commit_supported(*cfg))
-        return from_cuda(hyb::launch_commit_tc(*cfg, K, V, n_tok, W, d_state_ptrs, n_req, err, stream));
     return from_cuda(hyb::launch_commit_generic(*cfg, K, V, n_tok, W, d_state_ptrs, n_req, err, stream));
 }
 

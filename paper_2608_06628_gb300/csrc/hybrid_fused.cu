@@ -22,15 +22,16 @@
 //   warps 4-11 math: two threads per query row (one per TMEM lane and "part");
 //              a part owns every other 32-feature chunk of each half of phi.
 //
-// Per unit the tensor cores run
+// Per unit the tensor cores run, in this order,
 //   g1   [U | scores] = Q [W | K^T]  (one N = F + B product; U = Q W)
 //        and, with the commit, U_k^T = W^T K^T (phi of the block's keys)
-//   PV   D  = P' V                    (P' = w e^(s - sigma), bf16)
-//   R+   D += phi+'(Q) S+             (tf32, A operand in Tensor Memory)
-//   R-   D += phi-'(Q) S-
+//   R+   D  = phi+'(Q) S+             (tf32, A operand in Tensor Memory)
 //   dS   dS^T = V^T phi(K)^T per feature half (commit; bf16 from the TMA'd V)
-// and the math warps compute the row statistics, phi(Q) and P' between g1
-// and PV, and out = D / den afterwards.  Merge: with sigma the log of the
+//   PV   D += P' V                    (P' = w e^(s - sigma), bf16)
+//   R-   D += phi-'(Q) S-
+// The math warps publish phi+ as soon as its exponentials are in Tensor
+// Memory (R+ then overlaps the rest of the feature map), then compute phi-,
+// the row statistics, P' and phi(K), and out = D / den after R-.  Merge: with sigma the log of the
 // larger branch mass, phi' = phi e^-sigma and P' = w e^(s - sigma), so
 // D / den = (w sm_num + lin_num) / (w sm_den + lin_den) exactly, with
 // den = e^(log lin_den - sigma) + e^(log(w sm_den) - sigma) in [1, 2].  While
@@ -41,11 +42,12 @@
 // A unit's phi+ and phi- share its F phi columns: phi- waits in registers until
 // R+ has consumed phi+.  Step: Tensor Memory holds two unit slots of 256
 // columns, [phi | D] each, so the next unit's g1 runs between this unit's R+
-// and R- and its feature map overlaps R-.  Commit: [D | phi | dS+ | dS-];
-// dS^T is formed before the readout, so each half's tiles are updated in
-// shared memory (and written back by the storer) as soon as the readout has
-// consumed them; V, P' and phi(K) then share the Q region, so all 2F/32 state
-// tiles of a unit fit in the ring.
+// and R- and its feature map overlaps R-.  Commit: [D | phi | dS+ | dS-]; once
+// a half's tiles have been read out, their ring slots take that half's dS^T
+// rows and the storer adds them into the state in global memory by bulk
+// reduce-adds (the float32 add happens at L2), so the SM never writes a state
+// tile back.  V, P' and phi(K) share the Q region once g1 has consumed Q, so
+// all 2F/32 state tiles of a unit fit in the ring.
 //
 // MMA cost note: on this part a tcgen05.mma with M = 128 costs about the same
 // time for any N up to 128-256, so contractions are shaped for few, wide
@@ -373,8 +375,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             } else {
                 // Tensor Memory: [0,128) D, [128,128+F) phi (U, then phi+, then phi-),
                 // scores after U, [256,256+F) dS+ (U_k^T at 288 until then),
-                // [384,384+F) dS-.  dS^T is formed before the readout, so each half's
-                // tiles can be updated as soon as that half has been read out.
+                // [384,384+F) dS-.  dS^T follows R+, so the first half's tiles are
+                // free for their increments as soon as dS^T is in Tensor Memory.
                 for (int u = u_begin; u < u_end; ++u) {
                     if (!unit_state(a, u)) continue;
                     if (!wait_bar(xfull, kp & 1u, fail)) { ok = false; break; }

@@ -13,11 +13,6 @@ cudaError_t launch_attn_tc(const hybrid_cfg &c, const void *Q, const void *K, co
                            const void *W, const float *alpha, void *const *states, int n_req,
                            void *O, unsigned *err, cudaStream_t st);
 
-// True when hybrid_commit_block for this cfg runs on the tcgen05 kernel.
-bool tc_commit_supported(const hybrid_cfg &c);
-cudaError_t launch_commit_tc(const hybrid_cfg &c, const void *K, const void *V, int n_tok, const void *W,
-                             void *const *states, int n_req, unsigned *err, cudaStream_t st);
-
 // Persistent warp-specialised step kernel (hybrid_fused.cu); commit = true also
 // folds the block's K/V into the state in the same pass.
 bool fused_supported(const hybrid_cfg &c, bool commit);
