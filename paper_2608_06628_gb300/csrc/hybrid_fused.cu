@@ -159,9 +159,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     const int NCH = F / 32;          // 32-feature chunks (state tiles) per half of phi
     const int NC = 2 * NCH;          // state tiles per unit
     // the output tile is staged in the slots of tiles ocm, ocm + 1 of its unit:
-    // with the commit, first-half tiles that no later tile of the unit reuses
-    // (drained before the epilogue); without, the last two
-    const int ocm = kCommit ? (NC > NS ? NC - NS : 0) : NC - 2;
+    // with the commit, the first two second-half tiles (their increments are
+    // reduce-added before the epilogue), so the next unit's first-half tiles,
+    // needed first, can enter the ring early; if a unit has more tiles than the
+    // ring, first-half tiles that no later tile of the unit reuses; without the
+    // commit, the last two
+    const int ocm = kCommit ? (NC > NS ? NC - NS : NCH) : NC - 2;
     const uint32_t chunk_bytes = (uint32_t)d * 128;
     const int per = a.n_units / (int)gridDim.x, rem = a.n_units % (int)gridDim.x;
     const int u_begin = (int)blockIdx.x * per + min((int)blockIdx.x, rem);
@@ -426,21 +429,27 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             bool ok = true;
             if (kp > 0) ok = wait_bar(xfree, (kp - 1) & 1u, fail);
             if (__any_sync(0xffffffffu, !ok)) break;
+            // with the commit the Q region holds the previous unit's V, P' and phi(K)
+            // until its dS^T and P V have run (Q then follows K^T, which measured
+            // faster at start-up too); otherwise Q goes with W, before K^T
+            const bool q_early = !kCommit;
             if (lane == 0) {
                 mbar_arrive_expect_tx(xfull, xbytes);
+                if (q_early)
+                    for (int e = 0; e < d / 64; ++e)
+                        tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xfull);
                 for (int f = 0; f < F / 64; ++f)
                     tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xfull);
             }
             kt_store(kr, d, kt, lane);
             fence_proxy_async_smem();
             __syncwarp();
-            // with the commit the Q region holds the previous unit's V, P' and phi(K)
-            // until its dS^T and P V have run
-            if (kCommit && kp > 0) ok = wait_bar(dsdone, (kp - 1) & 1u, fail);
+            if (!q_early && kp > 0) ok = wait_bar(dsdone, (kp - 1) & 1u, fail);
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
-                for (int e = 0; e < d / 64; ++e)
-                    tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xfull);
+                if (!q_early)
+                    for (int e = 0; e < d / 64; ++e)
+                        tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xfull);
                 mbar_arrive(xfull);
             }
             ++nx;
@@ -479,16 +488,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     mbar_arrive(&zempty[zb]);
                     for (int h = 0; h < 2 && ok; ++h) {
                         if (!wait_bar(&tready[h], kp & 1u, fail)) { ok = false; break; }
-                        // one bulk group per tile; the two output slots (first in
-                        // the first half) are freed as soon as their reductions have read them
+                        // one bulk group per tile; the two output slots are freed as
+                        // soon as their reductions have read them
                         for (int c = h * NCH; c < (h + 1) * NCH; ++c) {
                             bulk_reduce_add_f32(Sg + (size_t)c * 32 * d, ring + (size_t)((q + c) % NS) * chunk_bytes,
                                                 chunk_bytes);
                             bulk_commit();
                         }
-                        if (h == 0) {
-                            // groups issued after the two output tiles: NCH - ocm - 2
-                            if (NCH - ocm - 2 >= 2) bulk_wait_read_2();
+                        if (h == ocm / NCH) {
+                            // the output slots may be written once their reductions have read them
+                            if ((h + 1) * NCH - (ocm + 2) >= 2) bulk_wait_read_2();
                             else bulk_wait_read_all();
                             mbar_arrive(ofree);
                         }
