@@ -79,6 +79,9 @@ constexpr uint32_t kBarPair = 2;      // 2..5: the two math warps of one TMEM la
 constexpr uint32_t kStatBytes = 14 * 1024;
 // Tensor Memory columns with the commit (F <= 128, d <= 128)
 constexpr uint32_t kCmD = 0, kCmP = 128, kCmDSp = 256, kCmK = 288, kCmDSm = 384;
+// unnormalised phi(K) parked between the two exchanges of the math warps (free
+// columns until dS+ is formed)
+constexpr uint32_t kCmEK = 320;
 
 struct FusedArgs {
     CUtensorMap tmQ, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
@@ -698,10 +701,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
 
             // ---- phase B2: phi- (kept in registers until R+ has consumed phi+), the
             // score sums; commit: unnormalised phi(K)
-            float ek[32];   // commit: unnormalised phi(K) of feature part*F + row, per token
             {
                 float l = 0.f, sn = 0.f, ln = 0.f;
                 if (has_sc) {
+                    if (kCommit) {
+                        tmem_ld16(scol + 16 * part, sc);
+                        tmem_wait_ld();
+                    }
 #pragma unroll
                     for (int i = 0; i < 16; ++i) l += ex2(fmaf(sc[i], scale_l2, -ml));
                 }
@@ -738,9 +744,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
 #pragma unroll
                     for (int t = 0; t < 32; ++t) {
                         const float m = __shfl_sync(0xffffffffu, m_l, t);
-                        ek[t] = fval ? ex2(fmaf(uk[t], sgn, -m)) : 0.f;
-                        uk[t] = ek[t];
+                        uk[t] = fval ? ex2(fmaf(uk[t], sgn, -m)) : 0.f;
                     }
+                    // parked in Tensor Memory until the token sums are exchanged
+                    tmem_st32(tmem + kCmEK + 32 * part + lane_off, uk);
                     const float ssum = warp_reduce32<0>(uk, lane);
                     tk[((2 + part) * 32 + lane) * 4 + q4] = ssum;
                 }
@@ -799,6 +806,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 if (has_sc) {
                     // P' (w e^(s - sigma), or w sp e^s on the fast path): K-major, no swizzle
                     // (8-row x 16-byte core matrices)
+                    if (kCommit) {
+                        tmem_ld16(scol + 16 * part, sc);
+                        tmem_wait_ld();
+                    }
                     uint32_t pk[8];
 #pragma unroll
                     for (int i = 0; i < 16; i += 2)
@@ -817,6 +828,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                         const float4 v = *reinterpret_cast<const float4 *>(&tk[((2 + part) * 32 + lane) * 4]);
                         inv_l = 1.f / ((v.x + v.y) + (v.z + v.w));
                     }
+                    float ek[32];   // unnormalised phi(K) of feature part*F + row, per token
+                    tmem_wait_st();
+                    tmem_ld32(tmem + kCmEK + 32 * part + lane_off, ek);
+                    tmem_wait_ld();
                     const int f = part * F + row;
                     uint8_t *bf = pkb + (f >> 6) * (B * 128) + ((f & 7) << 1);
                     const int gf = (f & 63) >> 3;

@@ -132,21 +132,27 @@ __device__ __forceinline__ void kt_load(const bf16 *K, size_t tok0, int nt, int 
         }
     }
 }
-__device__ __forceinline__ void kt_store(const KtRegs &k, int d, uint8_t *kt, int lane)
+__device__ __forceinline__ void kt_store(const KtRegs &k, int d, uint8_t *kt_in, int lane)
 {
+    // the base is made opaque so the 64 store addresses, which depend only on
+    // the lane, are formed at the stores rather than kept live across a caller's loop
+    uint8_t *kt = kt_in;
+    asm volatile("" : "+l"(kt));
     const int tp = lane & 15, eh = lane >> 4;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
         const int ec = eh + 2 * i;
-        if (ec >= d / 8) break;
-        const uint32_t w0[4] = {k.r0[i].x, k.r0[i].y, k.r0[i].z, k.r0[i].w};
-        const uint32_t w1[4] = {k.r1[i].x, k.r1[i].y, k.r1[i].z, k.r1[i].w};
+        if (ec < d / 8) {
+            const uint32_t w0[4] = {k.r0[i].x, k.r0[i].y, k.r0[i].z, k.r0[i].w};
+            const uint32_t w1[4] = {k.r1[i].x, k.r1[i].y, k.r1[i].z, k.r1[i].w};
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            const uint32_t lo = (w0[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
-            const uint32_t hi = (w1[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
-            const int e = 8 * ec + j;
-            *reinterpret_cast<uint32_t *>(kt + e * 128 + ((((tp >> 2) ^ (e & 7))) << 4) + (tp & 3) * 4) = lo | (hi << 16);
+            for (int j = 0; j < 8; ++j) {
+                const uint32_t lo = (w0[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
+                const uint32_t hi = (w1[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
+                const int e = 8 * ec + j;
+                *reinterpret_cast<uint32_t *>(kt + e * 128 + ((((tp >> 2) ^ (e & 7))) << 4) + (tp & 3) * 4) =
+                    lo | (hi << 16);
+            }
         }
     }
 }
