@@ -431,12 +431,18 @@ def run_hybrid(args, wl):
     # steps are pipelined over three streams (copy in, compute, copy out) so the
     # next step's inputs and the previous step's output move while a step runs;
     # the sequence is captured once in a CUDA graph and replayed.
-    hQ = sets[0]["Q"].cpu().pin_memory()
-    hK = sets[0]["K"].cpu().pin_memory()
-    hV = sets[0]["V"].cpu().pin_memory()
-    hO = [torch.empty_like(hQ).pin_memory() for _ in range(2)]
-    e2e_sets = [dict(s, Q=torch.empty_like(s["Q"]), K=torch.empty_like(s["K"]), V=torch.empty_like(s["V"]))
-                for s in sets]
+    # a step's Q, K and V sit back to back in one pinned host buffer and one
+    # device buffer, so each step's input is one copy
+    q0, k0, v0 = sets[0]["Q"], sets[0]["K"], sets[0]["V"]
+    nq, nk = q0.numel(), k0.numel()
+    hQKV = torch.cat([q0.reshape(-1), k0.reshape(-1), v0.reshape(-1)]).cpu().pin_memory()
+    hO = [torch.empty(q0.shape, dtype=q0.dtype).pin_memory() for _ in range(2)]
+
+    def split_qkv(buf):
+        return dict(Q=buf[:nq].view(q0.shape), K=buf[nq:nq + nk].view(k0.shape), V=buf[nq + nk:].view(v0.shape))
+
+    e2e_bufs = [torch.empty_like(hQKV, device=dev) for _ in sets]
+    e2e_sets = [dict(s, **split_qkv(b)) for s, b in zip(sets, e2e_bufs)]
     n_e2e = 2 * n_sets
     cin, cout = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
     g_e2e = torch.cuda.CUDAGraph()
@@ -451,9 +457,7 @@ def run_hybrid(args, wl):
             if i >= n_sets:
                 cin.wait_event(ev_out[i - n_sets])   # the set's previous step has finished with it
             with torch.cuda.stream(cin):
-                s["Q"].copy_(hQ, non_blocking=True)
-                s["K"].copy_(hK, non_blocking=True)
-                s["V"].copy_(hV, non_blocking=True)
+                e2e_bufs[i % n_sets].copy_(hQKV, non_blocking=True)
             ev_in[i].record(cin)
             side.wait_event(ev_in[i])
             H.hybrid_block_attn_commit(cfg, s["Q"], s["K"], s["V"], W, alpha, s["ptrs"], wl.n_req, s["O"],
@@ -520,7 +524,7 @@ def run_hybrid(args, wl):
         },
         "e2e": {"value": wl.n_req * wl.B * e2e_steps * ws / (e2e_ms * 1e-3), "unit": "tokens/s",
                 "steps": e2e_steps, "pipelined": "copy-in / step / copy-out on three streams, graph-replayed",
-                "h2d_bytes_per_step": int(hQ.numel() * hQ.element_size() + 2 * hK.numel() * hK.element_size()),
+                "h2d_bytes_per_step": int(hQKV.numel() * hQKV.element_size()),
                 "d2h_bytes_per_step": int(hO[0].numel() * hO[0].element_size())},
         "gpu_launches": K_,
         "clocks": clocks.summary(t_wall0, t_wall1),
