@@ -186,17 +186,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint64_t *vfull = xfree + 1;
     uint64_t *vfree = vfull + 1;
     uint64_t *uready = vfree + 1;     // MMA -> math: g1 done
-    uint64_t *phip = uready + 1;      // math -> MMA: phi+ and P' (with the commit also phi(K))
+    uint64_t *phip = uready + 1;      // math -> MMA: phi+ is in the phi columns
     uint64_t *phim = phip + 1;        // math -> MMA: phi- in the phi columns
     uint64_t *pread = phim + 1;       // MMA -> math: R+ has consumed phi+
-    uint64_t *pready = pread + 1;     // math -> MMA: P' (and, with the commit, phi(K)) is written
-    uint64_t *dsdone = pready + 1;    // MMA -> math: dS^T is formed (commit)
-    uint64_t *efree = dsdone + 1;     // math -> MMA: the first-half update has read dS+ (commit)
+    uint64_t *pready = pread + 1;     // math -> MMA: P' is written
+    uint64_t *kready = pready + 1;    // math -> MMA: phi(K) is written (commit)
+    uint64_t *dsdone = kready + 1;    // MMA -> math: dS^T is formed (commit)
+    uint64_t *pvdone = dsdone + 1;    // MMA -> producer: P V has read V and P' (commit)
+    uint64_t *efree = pvdone + 1;     // math -> MMA: the first-half update has read dS+ (commit)
     uint64_t *zdone = efree + 1;      // math -> storer: z is updated (commit)
     uint64_t *ofree = zdone + 1;      // storer -> math: the output slots may be written (commit)
     uint64_t *ostaged = ofree + 1;    // math -> storer: the output tile is in its slots
     uint64_t *mmadone = ostaged + 1;
-    const int n_bars = 2 * NS + 10 + 15;
+    const int n_bars = 2 * NS + 10 + 17;
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + n_bars);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
@@ -212,6 +214,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         mbar_init(phip, 8);
         mbar_init(phim, 8);
         mbar_init(pready, 8);
+        mbar_init(kready, 8);
         mbar_init(efree, 8);
         mbar_init(zdone, 8);
         mbar_init(ostaged, 8);
@@ -399,12 +402,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     for (int c = 0; c < NCH && ok; ++c) ok = readout(kCmD, kCmP + 32 * c, qt + c, c == 0) >= 0;
                     if (!ok) break;
                     mma_commit(pread);
-                    if (!wait_bar(pready, kp & 1u, fail) || !wait_bar(vfull, kp & 1u, fail)) { ok = false; break; }
+                    if (!wait_bar(kready, kp & 1u, fail) || !wait_bar(vfull, kp & 1u, fail)) { ok = false; break; }
                     tc_fence_after();
                     ds(kCmDSp, 0);
                     ds(kCmDSm, 1);
-                    pv(kCmD);
                     mma_commit(dsdone);
+                    if (!wait_bar(pready, kp & 1u, fail)) { ok = false; break; }
+                    tc_fence_after();
+                    pv(kCmD);
+                    mma_commit(pvdone);
                     if (!wait_bar(phim, kp & 1u, fail)) { ok = false; break; }
                     tc_fence_after();
                     for (int c = NCH; c < NC && ok; ++c) ok = readout(kCmD, kCmP + 32 * (c - NCH), qt + c) >= 0;
@@ -447,7 +453,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             kt_store(kr, d, kt, lane);
             fence_proxy_async_smem();
             __syncwarp();
-            if (!q_early && kp > 0) ok = wait_bar(dsdone, (kp - 1) & 1u, fail);
+            if (!q_early && kp > 0) ok = wait_bar(pvdone, (kp - 1) & 1u, fail);
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
                 if (!q_early)
@@ -767,6 +773,43 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             // commit: phi(K), z
             float cneg, inv_den;
             {
+                // with the commit the scores share the dS+ columns, which dS^T may
+                // overwrite once phi(K) is signalled: P' takes them from registers
+                if (kCommit && has_sc) tmem_ld16(scol + 16 * part, sc);
+                if (kCommit) {
+                    // phi(K) normalised, as the bf16 MN-major operand [token][feature]
+                    // (64-feature atoms of B rows), and z[part*F + row] += sum_t phi(k_t)
+                    // (this thread is the only writer); lane t holds token t's normaliser
+                    float inv_l;
+                    {
+                        const float4 v = *reinterpret_cast<const float4 *>(&tk[((2 + part) * 32 + lane) * 4]);
+                        inv_l = 1.f / ((v.x + v.y) + (v.z + v.w));
+                    }
+                    float ek[32];   // unnormalised phi(K) of feature part*F + row, per token
+                    tmem_wait_st();
+                    tmem_ld32(tmem + kCmEK + 32 * part + lane_off, ek);
+                    tmem_wait_ld();
+                    const int f = part * F + row;
+                    uint8_t *bf = pkb + (f >> 6) * (B * 128) + ((f & 7) << 1);
+                    const int gf = (f & 63) >> 3;
+                    float dz = 0.f;
+#pragma unroll
+                    for (int t = 0; t < 32; ++t) {
+                        const float v = ek[t] * __shfl_sync(0xffffffffu, inv_l, t);
+                        dz += v;
+                        if (fval) *reinterpret_cast<bf16 *>(bf + t * 128 + ((gf ^ (t & 7)) << 4)) = __float2bfloat16_rn(v);
+                    }
+                    if (fval) zs[f] += dz;
+                    // dS^T may be formed while P' is computed (it overwrites the
+                    // scores and U_k^T this thread has read from Tensor Memory)
+                    fence_proxy_async_smem();
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) {
+                        mbar_arrive(kready);
+                        mbar_arrive(zdone);
+                    }
+                }
                 const float l = xb[0 * 128 + row] + xb[4 * 128 + row];
                 const float lpf = xb[1 * 128 + row] + xb[5 * 128 + row];
                 const float sn = xb[2 * 128 + row] + xb[6 * 128 + row];
@@ -806,10 +849,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 if (has_sc) {
                     // P' (w e^(s - sigma), or w sp e^s on the fast path): K-major, no swizzle
                     // (8-row x 16-byte core matrices)
-                    if (kCommit) {
-                        tmem_ld16(scol + 16 * part, sc);
-                        tmem_wait_ld();
-                    }
                     uint32_t pk[8];
 #pragma unroll
                     for (int i = 0; i < 16; i += 2)
@@ -819,38 +858,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     *reinterpret_cast<uint4 *>(prow + (2 * part + 1) * 128) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                 }
                 inv_den = kappa / (expf(log_l - sig) + expf(log_s - sig));
-                if (kCommit) {
-                    // phi(K) normalised, as the bf16 MN-major operand [token][feature]
-                    // (64-feature atoms of B rows), and z[part*F + row] += sum_t phi(k_t)
-                    // (this thread is the only writer); lane t holds token t's normaliser
-                    float inv_l;
-                    {
-                        const float4 v = *reinterpret_cast<const float4 *>(&tk[((2 + part) * 32 + lane) * 4]);
-                        inv_l = 1.f / ((v.x + v.y) + (v.z + v.w));
-                    }
-                    float ek[32];   // unnormalised phi(K) of feature part*F + row, per token
-                    tmem_wait_st();
-                    tmem_ld32(tmem + kCmEK + 32 * part + lane_off, ek);
-                    tmem_wait_ld();
-                    const int f = part * F + row;
-                    uint8_t *bf = pkb + (f >> 6) * (B * 128) + ((f & 7) << 1);
-                    const int gf = (f & 63) >> 3;
-                    float dz = 0.f;
-#pragma unroll
-                    for (int t = 0; t < 32; ++t) {
-                        const float v = ek[t] * __shfl_sync(0xffffffffu, inv_l, t);
-                        dz += v;
-                        if (fval) *reinterpret_cast<bf16 *>(bf + t * 128 + ((gf ^ (t & 7)) << 4)) = __float2bfloat16_rn(v);
-                    }
-                    if (fval) zs[f] += dz;
-                }
             }
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(pready);
-                if (kCommit) mbar_arrive(zdone);
-            }
+            if (lane == 0) mbar_arrive(pready);
 
             // previous unit's output, while R+ of this one runs (step)
             if (!kCommit && kp >= 1) bad = !epilogue(kp - 1, prev_q, prev_inv);
