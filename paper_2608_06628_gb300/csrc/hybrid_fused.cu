@@ -31,7 +31,8 @@
 //   R-   D += phi-'(Q) S-
 // The math warps publish phi+ as soon as its exponentials are in Tensor
 // Memory (R+ then overlaps the rest of the feature map), then compute phi-,
-// the row statistics, P' and phi(K), and out = D / den after R-.  Merge: with sigma the log of the
+// the row statistics, phi(K) (signalled first, so dS^T is formed meanwhile)
+// and P', and out = D / den after R-.  Merge: with sigma the log of the
 // larger branch mass, phi' = phi e^-sigma and P' = w e^(s - sigma), so
 // D / den = (w sm_num + lin_num) / (w sm_den + lin_den) exactly, with
 // den = e^(log lin_den - sigma) + e^(log(w sm_den) - sigma) in [1, 2].  While
