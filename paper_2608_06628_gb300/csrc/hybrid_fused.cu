@@ -400,9 +400,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     // phip also covers the previous unit's output epilogue and second-half update
                     if (!wait_bar(phip, kp & 1u, fail)) { ok = false; break; }
                     tc_fence_after();
-                    for (int c = 0; c < NCH && ok; ++c) ok = readout(kCmD, kCmP + 32 * c, qt + c, c == 0) >= 0;
+                    for (int c = 0; c < NCH && ok; ++c) ok = readout(kCmD, kCmDSm + 32 * c, qt + c, c == 0) >= 0;
                     if (!ok) break;
-                    mma_commit(pread);
                     if (!wait_bar(kready, kp & 1u, fail) || !wait_bar(vfull, kp & 1u, fail)) { ok = false; break; }
                     tc_fence_after();
                     ds(kCmDSp, 0);
@@ -618,6 +617,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             const uint32_t pcol = tmem + (kCommit ? kCmP : T) + lane_off;       // U, phi+, phi-
             const uint32_t scol = pcol + F;                                    // scores
             const uint32_t kcol = tmem + kCmK + lane_off;                      // U_k^T (commit)
+            // phi+: with the commit in the dS- columns (free until dS^T is formed), so U
+            // stays in place for phi- and no thread holds U in registers; the step keeps
+            // U in registers and writes phi+ over it
+            const uint32_t ppcol = kCommit ? tmem + kCmDSm + lane_off : pcol;
 
             // ---- phase A: row extrema of U and of the scores (U kept in registers);
             // commit: per-token extrema of U_k^T over this warp's 32 features
@@ -637,8 +640,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 tk[(part * 32 + lane) * 4 + q4] = ext;   // max of +-U_k for token lane
             }
             if (has_sc) tmem_ld16(scol + 16 * part, sc);
-            tmem_ld32(pcol + 32 * part, u0);
-            if (two) tmem_ld32(pcol + 32 * (part + 2), u1);
+            if (!kCommit) {
+                tmem_ld32(pcol + 32 * part, u0);
+                if (two) tmem_ld32(pcol + 32 * (part + 2), u1);
+            }
             tmem_wait_ld();
             {
                 float ms = -INFINITY, mx = -INFINITY, mn = INFINITY;
@@ -646,11 +651,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
 #pragma unroll
                     for (int i = 0; i < 16; ++i) ms = fmaxf(ms, sc[i]);
                 }
+                if (kCommit) {
+                    // this thread's 32-feature chunks of U, one at a time
+#pragma unroll 1
+                    for (int k = part; k < NCH; k += 2) {
+                        float x[32];
+                        tmem_ld32(pcol + 32 * k, x);
+                        tmem_wait_ld();
 #pragma unroll
-                for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, u0[i]); mn = fminf(mn, u0[i]); }
-                if (two) {
+                        for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, x[i]); mn = fminf(mn, x[i]); }
+                    }
+                } else {
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, u1[i]); mn = fminf(mn, u1[i]); }
+                    for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, u0[i]); mn = fminf(mn, u0[i]); }
+                    if (two) {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, u1[i]); mn = fminf(mn, u1[i]); }
+                    }
                 }
                 xa[(part * 3 + 0) * 128 + row] = ms;
                 xa[(part * 3 + 1) * 128 + row] = mx;
@@ -685,10 +702,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                             lp = fmaf(e, za[j], lp);
                         }
                     }
-                    tmem_st32(pcol + 32 * k, ep);
+                    tmem_st32(ppcol + 32 * k, ep);
                 };
-                expp(u0, part);
-                if (two) expp(u1, part + 2);
+                if (kCommit) {
+#pragma unroll 1
+                    for (int k = part; k < NCH; k += 2) {
+                        float x[32];
+                        tmem_ld32(pcol + 32 * k, x);
+                        tmem_wait_ld();
+                        expp(x, k);
+                    }
+                } else {
+                    expp(u0, part);
+                    if (two) expp(u1, part + 2);
+                }
                 xs[part * 128 + row] = sp;
             }
             if (sync_failed(bad)) { ok = false; break; }
@@ -734,8 +761,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                         }
                     }
                 };
-                expm(u0, part);
-                if (two) expm(u1, part + 2);
+                if (kCommit) {
+                    // phi- (unscaled) over U in its columns; scaled by cneg in phase D
+#pragma unroll 1
+                    for (int k = part; k < NCH; k += 2) {
+                        float x[32];
+                        tmem_ld32(pcol + 32 * k, x);
+                        tmem_wait_ld();
+                        expm(x, k);
+                        tmem_st32(pcol + 32 * k, x);
+                    }
+                } else {
+                    expm(u0, part);
+                    if (two) expm(u1, part + 2);
+                }
                 if (kCommit) {
                     // unnormalised phi(K) of this thread's feature for every token
                     float uk[32];
@@ -838,8 +877,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                         for (int i = 0; i < 32; ++i) v[i] *= cpos;
                         tmem_st32(col, v);
                     };
-                    scale_chunk(pcol + 32 * part);
-                    if (two) scale_chunk(pcol + 32 * (part + 2));
+                    scale_chunk(ppcol + 32 * part);
+                    if (two) scale_chunk(ppcol + 32 * (part + 2));
                     tmem_wait_st();
                     tc_fence_before();
                     __syncwarp();
@@ -866,16 +905,30 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
 
             // previous unit's output, while R+ of this one runs (step)
             if (!kCommit && kp >= 1) bad = !epilogue(kp - 1, prev_q, prev_inv);
-            // ---- phase D: phi- into the phi columns once R+ has consumed phi+
-            bad = !wait_bar(pread, kp & 1u, fail) || bad;
-            tc_fence_after();
+            // ---- phase D: phi- scaled by cneg in the phi columns (step: once R+ has
+            // consumed phi+ there)
+            if (kCommit) {
+                tmem_wait_st();
+#pragma unroll 1
+                for (int k = part; k < NCH; k += 2) {
+                    float x[32];
+                    tmem_ld32(pcol + 32 * k, x);
+                    tmem_wait_ld();
 #pragma unroll
-            for (int i = 0; i < 32; ++i) u0[i] *= cneg;
-            tmem_st32(pcol + 32 * part, u0);
-            if (two) {
+                    for (int i = 0; i < 32; ++i) x[i] *= cneg;
+                    tmem_st32(pcol + 32 * k, x);
+                }
+            } else {
+                bad = !wait_bar(pread, kp & 1u, fail) || bad;
+                tc_fence_after();
 #pragma unroll
-                for (int i = 0; i < 32; ++i) u1[i] *= cneg;
-                tmem_st32(pcol + 32 * (part + 2), u1);
+                for (int i = 0; i < 32; ++i) u0[i] *= cneg;
+                tmem_st32(pcol + 32 * part, u0);
+                if (two) {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) u1[i] *= cneg;
+                    tmem_st32(pcol + 32 * (part + 2), u1);
+                }
             }
             tmem_wait_st();
             tc_fence_before();
