@@ -1003,8 +1003,9 @@ bool fused_supported(const hybrid_cfg &c, bool commit)
     if (commit && c.block_size != 32) return false;
     const FLayout L = make_flayout(c.head_dim, c.feat_dim, c.block_size, commit);
     const int NCH = c.feat_dim / 32;
-    // step: the last two tiles of a unit are held for the output; commit: the
-    // first half stays resident until updated and two of its slots take the output
+    // step: the last two tiles of a unit are held for the output; commit: a ring
+    // shorter than a unit stages the output in first-half slots that no later tile
+    // of the unit reuses, which needs NCH + 2 slots
     if (L.NS < (commit ? NCH + 2 : 4)) return false;
     return (int)L.bytes <= kSmemLimit;
 }

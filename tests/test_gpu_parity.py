@@ -284,6 +284,10 @@ FUSED = [
     (W_("fused_b16_fallback", BF16, 3, 4, 2, 128, 128, 16, 54), [16, 0, 48]),  # B != 32: step + commit
     # keys x24: scores near 60 make some warps take the exact phi+ rescale
     (W_("fused_gqa4_k24", BF16, 3, 8, 2, 128, 128, 32, 56, k_scale=24.0), [32, 0, 96]),
+    # F = 64: one 32-feature chunk per part, the output takes the whole second half
+    (W_("fused_d128_f64", BF16, 4, 8, 4, 128, 64, 32, 57), [0, 64, 32, 96]),
+    # d = 64, F = 128: a ring longer than a unit; 192 units, two or more per CTA
+    (W_("fused_d64_f128_many", BF16, 48, 16, 4, 64, 128, 32, 58), None),
 ]
 
 
