@@ -231,6 +231,95 @@ def cpu_baseline(wl, budget_s=12.0):
                       f"fp64 C oracle, {cores} threads), {tot:.1f} s"}
 
 
+def small_config_context(dev, warmup=5, iters=20):
+    """Context for the two small configurations (not part of the value): the
+    per-call device time of the call the tests make on them, replayed from a CUDA
+    graph and launched directly (median of iters after warmup), and the oracle's
+    one-thread time for the same call.  c1 (fp32, one request) is latency-bound
+    and uses one buffer set; c2 rotates enough sets that each call misses L2."""
+    import torch
+    import oracle
+    from paper_2608_06628_gb300 import hybrid as H
+    from paper_2608_06628_gb300 import workloads as wk
+    from paper_2608_06628_gb300.state_pool import StatePool
+    orc = oracle.load()
+    out = {}
+    for wl, fused in ((wk.C1, False), (wk.C2, True)):
+        cfg = H.make_cfg(wl.d, wl.F, wl.Hq, wl.Hkv, wl.B, wl.io_dtype)
+        W, alpha = wk.params(wl, device=dev)
+        io_bytes = 2 if wl.io_dtype == torch.bfloat16 else 4
+        ab = algorithmic_bytes(wl, io_bytes)
+        l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+        per_set = ab["q"] * 2 + ab["kv"] * 2 + ab["state"]
+        n_sets = 1 if not fused else max(2, math.ceil(4 * l2 / per_set) + 1)
+        plen = wk.prefix_lengths(wl)
+        pool0 = StatePool(cfg, wl.n_req, dev)
+        H.hybrid_state_init(cfg, pool0.all_ptrs(), wl.n_req)
+        for b in range(int(plen.max()) // wl.B):
+            reqs = np.nonzero(plen > b * wl.B)[0]
+            K, V = wk.prefix_kv(wl, b, dev, n_req=len(reqs))
+            H.hybrid_commit_block(cfg, K, V, wl.B, W, pool0.ptr_array(reqs.tolist()), len(reqs))
+        H.hybrid_check()
+        sets = []
+        for i in range(n_sets):
+            pool = pool0 if i == 0 else StatePool(cfg, wl.n_req, dev)
+            if i:
+                pool.slab.copy_(pool0.slab)
+            Q, K, V = wk.block_qkv(wl, ("ctx", i), dev)
+            sets.append(dict(pool=pool, ptrs=pool.all_ptrs(), Q=Q, K=K, V=V, O=torch.empty_like(Q)))
+        fn = H.hybrid_block_attn_commit if fused else H.hybrid_block_attn
+        stream = torch.cuda.current_stream(dev)
+
+        def call(s, st):
+            fn(cfg, s["Q"], s["K"], s["V"], W, alpha, s["ptrs"], wl.n_req, s["O"], st, check=False)
+
+        for i in range(warmup):
+            call(sets[i % n_sets], stream.cuda_stream)
+        H.hybrid_check()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(iters)]
+        for i in range(iters):
+            evs[i][0].record(stream)
+            call(sets[i % n_sets], stream.cuda_stream)
+            evs[i][1].record(stream)
+        torch.cuda.synchronize()
+        direct = sorted(a.elapsed_time(b) for a, b in evs)[iters // 2]
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(stream)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=side):
+            for i in range(iters):
+                call(sets[i % n_sets], side.cuda_stream)
+        torch.cuda.synchronize()
+        g.replay()
+        torch.cuda.synchronize()
+        a_, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a_.record(stream)
+        g.replay()
+        b_.record(stream)
+        torch.cuda.synchronize()
+        graph_ms = a_.elapsed_time(b_) / iters
+        status = H.hybrid_check(check=False)
+        if status != H.HYBRID_OK:
+            raise SystemExit(f"device error in the small-config context: {H.hybrid_status_str(status)}")
+        # the oracle's cost does not depend on the state's values: time it on empty states
+        Wc, alc = wk.params(wl)
+        W64, al64 = Wc.double().numpy(), alc.double().numpy()
+        Q, K, V = wk.block_qkv(wl, "ctx-oracle", "cpu")
+        Q64, K64, V64 = (t.to(torch.float64).numpy() for t in (Q, K, V))
+        S, z = orc.empty_state(wl.n_req, wl.Hkv, wl.d, wl.F)
+        t0 = time.perf_counter()
+        orc.block_attn(Q64, K64, V64, W64, al64, S, z, n_threads=1)
+        if fused:
+            orc.commit(K64, V64, W64, S, z, n_threads=1)
+        t_orc = time.perf_counter() - t0
+        nbytes = ab["fused"] if fused else ab["attn"]
+        out[wl.name] = {"call": fn.__name__, "graph_us": graph_ms * 1e3, "direct_us_median": direct * 1e3,
+                        "algorithmic_bytes": nbytes, "buffer_sets": n_sets,
+                        "tokens_per_s_graph": wl.n_req * wl.B / (graph_ms * 1e-3),
+                        "oracle_1thread_us": t_orc * 1e6}
+    return out
+
+
 # ---------------------------------------------------------------------------
 # reference arm: the oracle, timed step by step
 # ---------------------------------------------------------------------------
@@ -529,6 +618,8 @@ def run_hybrid(args, wl):
         "gpu_launches": K_,
         "clocks": clocks.summary(t_wall0, t_wall1),
     }
+    if not args.no_small_configs and ws == 1:
+        line["small_configs"] = small_config_context(dev)
     if not args.no_cpu_baseline and ws == 1:
         line["cpu_baseline"] = cpu_baseline(wl)
     print(json.dumps(line), flush=True)
@@ -546,6 +637,8 @@ def main(argv=None):
     ap.add_argument("--impl", choices=("hybrid", "reference"), default="hybrid")
     ap.add_argument("--config", default="c3_bf16_b64_gqa_ragged")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-small-configs", action="store_true",
+                    help="skip the c1/c2 context timings (graph and direct launches, 1-thread oracle)")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
