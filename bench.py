@@ -320,6 +320,54 @@ def small_config_context(dev, warmup=5, iters=20):
     return out
 
 
+def prefill_context(dev, wl, T=4096, warmup=2, iters=5):
+    """Context (not part of the value): one prompt prefill of T tokens into every
+    request's state at the workload's shape (hybrid_commit_block with n_tok = T),
+    median device time of iters calls after warmup.  Traffic is K + V + the state
+    read and written once; flops are U_k^T = W^T K^T (2FdT per unit) and
+    dS^T = V^T phi(K)^T (4FdT per unit)."""
+    import torch
+    from paper_2608_06628_gb300 import hybrid as H
+    from paper_2608_06628_gb300 import workloads as wk
+    from paper_2608_06628_gb300.state_pool import StatePool
+    cfg = H.make_cfg(wl.d, wl.F, wl.Hq, wl.Hkv, wl.B, wl.io_dtype)
+    W, _ = wk.params(wl, device=dev)
+    pool = StatePool(cfg, wl.n_req, dev)
+    ptrs = pool.all_ptrs()
+    H.hybrid_state_init(cfg, ptrs, wl.n_req)
+    g = torch.Generator(device=dev).manual_seed(4096)
+    shape = (wl.n_req, T, wl.Hkv, wl.d)
+    K = torch.randn(shape, generator=g, device=dev, dtype=torch.float32).to(wl.io_dtype)
+    V = torch.randn(shape, generator=g, device=dev, dtype=torch.float32).to(wl.io_dtype)
+    stream = torch.cuda.current_stream(dev)
+    for _ in range(warmup):
+        H.hybrid_commit_block(cfg, K, V, T, W, ptrs, wl.n_req, stream.cuda_stream, check=False)
+    H.hybrid_check()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(iters)]
+    for a_, b_ in evs:
+        a_.record(stream)
+        H.hybrid_commit_block(cfg, K, V, T, W, ptrs, wl.n_req, stream.cuda_stream, check=False)
+        b_.record(stream)
+    torch.cuda.synchronize()
+    status = H.hybrid_check(check=False)
+    if status != H.HYBRID_OK:
+        raise SystemExit(f"device error in the prefill context: {H.hybrid_status_str(status)}")
+    ms = sorted(a_.elapsed_time(b_) for a_, b_ in evs)[iters // 2]
+    io = K.element_size()
+    units = wl.n_req * wl.Hkv
+    nbytes = 2 * K.numel() * io + 2 * units * (2 * wl.F * wl.d + 2 * wl.F) * 4 + wl.Hkv * wl.d * wl.F * io
+    flops = 6.0 * wl.F * wl.d * T * units
+    peaks, _ = measured_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    bf16 = float(peaks.get("bf16_tflops", 1900.0))
+    del K, V
+    return {"call": "hybrid_commit_block", "tokens_per_request": T, "us": ms * 1e3,
+            "algorithmic_bytes": nbytes, "GBps": nbytes / (ms * 1e-3) / 1e9,
+            "frac_hbm": nbytes / (ms * 1e-3) / 1e9 / hbm,
+            "TFLOPs": flops / (ms * 1e-3) / 1e12, "frac_bf16_peak": flops / (ms * 1e-3) / 1e12 / bf16,
+            "prompt_tokens_per_s": wl.n_req * T / (ms * 1e-3)}
+
+
 # ---------------------------------------------------------------------------
 # reference arm: the oracle, timed step by step
 # ---------------------------------------------------------------------------
@@ -620,6 +668,7 @@ def run_hybrid(args, wl):
     }
     if not args.no_small_configs and ws == 1:
         line["small_configs"] = small_config_context(dev)
+        line["prefill_context"] = prefill_context(dev, wl)
     if not args.no_cpu_baseline and ws == 1:
         line["cpu_baseline"] = cpu_baseline(wl)
     print(json.dumps(line), flush=True)

@@ -187,6 +187,10 @@ hybrid_status hybrid_block_attn_commit_logical(const hybrid_cfg *cfg, const void
     return hybrid_state_unpack(cfg, d_ptrs, n_req, S_logical, z_logical, stream);
 }
 
+// Commits of more tokens than this run the prefill kernel (measured crossover
+// on the batch-64 shape: 64 tokens per request).
+constexpr int kPrefillMinTokens = 64;
+
 hybrid_status hybrid_commit_block(const hybrid_cfg *cfg, const void *K, const void *V, int n_tok,
                                   const void *W, void *const *d_state_ptrs, int n_req,
                                   cudaStream_t stream)
@@ -200,6 +204,10 @@ hybrid_status hybrid_commit_block(const hybrid_cfg *cfg, const void *K, const vo
         return HYBRID_ERR_INVALID_ARG;
     unsigned *err = error_word();
     if (!err) return HYBRID_ERR_CUDA;
+    // block commits (a few dozen tokens) run the per-unit reduction kernel; longer
+    // prompts the token-major prefill kernel, which balances chunks across SMs
+    if (n_tok > kPrefillMinTokens && hyb::prefill_supported(*cfg))
+        return from_cuda(hyb::launch_prefill(*cfg, K, V, n_tok, W, d_state_ptrs, n_req, err, stream));
     if (hyb::commit_red_supported(*cfg))
         return from_cuda(hyb::launch_commit_red(*cfg, K, V, n_tok, W, d_state_ptrs, n_req, err, stream));
     return from_cuda(hyb::launch_commit_generic(*cfg, K, V, n_tok, W, d_state_ptrs, n_req, err, stream));

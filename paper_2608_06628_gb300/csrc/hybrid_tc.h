@@ -23,6 +23,12 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
 // Commit / prefill as a reduction (hybrid_commit_red.cu): S += dS and z += dz are
 // added into the state in global memory by bulk reduce-adds; any n_tok >= 1.
 bool commit_red_supported(const hybrid_cfg &c);
+// Commit / prefill with the key feature map computed token-major
+// (hybrid_prefill.cu): 128-token chunks, ranges of chunks balanced across SMs,
+// increments added by bulk reduce-adds; any n_tok >= 1.
+bool prefill_supported(const hybrid_cfg &c);
+cudaError_t launch_prefill(const hybrid_cfg &c, const void *K, const void *V, int n_tok, const void *W,
+                           void *const *states, int n_req, unsigned *err, cudaStream_t st);
 cudaError_t launch_commit_red(const hybrid_cfg &c, const void *K, const void *V, int n_tok, const void *W,
                               void *const *states, int n_req, unsigned *err, cudaStream_t st);
 

@@ -262,6 +262,31 @@ def test_bad_state_pointer_is_reported_not_faulted():
     assert H.hybrid_check(check=False) == H.HYBRID_OK
 
 
+PREFILL = [
+    # 6 units x 8 chunks: every unit's chunks are spread over 8 CTAs and combined
+    # by the reduce-adds, on top of a prefix already in the state
+    (W_("prefill_split_runs", BF16, 3, 4, 2, 128, 128, 32, 46), 1000, 64),
+    # 80 units x 3 chunks on 152 CTAs: ranges cross unit boundaries; 44-token tail
+    (W_("prefill_cross_units", BF16, 20, 8, 4, 128, 128, 32, 47), 300, 0),
+    # d = F = 64, a one-token last chunk
+    (W_("prefill_d64_f64", BF16, 4, 4, 4, 64, 64, 32, 48), 257, 32),
+]
+
+
+@pytest.mark.parametrize("wl,T,prefix", PREFILL, ids=[w.name for w, _, _ in PREFILL])
+def test_prefill_split_across_ctas(wl, T, prefix):
+    """Long prompt prefills (hybrid_commit_block with n_tok = T) against the
+    oracle, the state holding an earlier prefix of `prefix` tokens."""
+    pair = Pair(wl)
+    if prefix:
+        pair.build_prefixes(np.full(wl.n_req, prefix, dtype=np.int64))
+    K, V = wk.prefix_kv(wl, 1, pair.dev, n_tok=T)
+    pair.commit(K, V)
+    S, z = pair.gpu_state()
+    assert_parity(S, pair.S, BF16, f"prefill {T} S")
+    assert_parity(z, pair.z, BF16, f"prefill {T} z")
+
+
 def test_prefill_commit_long_ragged():
     """Prompt prefill: commits of many tokens (T not a multiple of 32) in one call
     equal the same tokens committed in B-sized pieces."""
