@@ -11,6 +11,7 @@ marshals numpy float64 arrays in and out.
 
 Logical layouts (row-major):
     Q, O   [n_req, B, Hq, d]       K, V  [n_req, T, Hkv, d]
+    training form: Q, O, dO [n_seq, L, Hq, d], K, V [n_seq, L, Hkv, d]
     W      [Hkv, d, F]             alpha [Hq]
     S      [n_req, Hkv, 2F, d]     z     [n_req, Hkv, 2F]
 """
@@ -86,8 +87,11 @@ class Oracle:
         lib.oracle_block_attn.argtypes = [I, I, I, I, I, I, I, D, D, D, D, D, D, D, D, I]
         lib.oracle_block_attn_prefix.argtypes = [I, I, I, I, I, I, I, D, D, D, D, D, D, D,
                                                  ctypes.POINTER(ctypes.c_int), I, D, I]
+        lib.oracle_train_forward.argtypes = [I, I, I, I, I, I, I, D, D, D, D, D, D, I]
+        lib.oracle_train_backward.argtypes = [I, I, I, I, I, I, I, D, D, D, D, D, D, D, D, I]
         for fn in (lib.oracle_feature_map, lib.oracle_commit, lib.oracle_block_attn,
-                   lib.oracle_block_attn_prefix):
+                   lib.oracle_block_attn_prefix, lib.oracle_train_forward,
+                   lib.oracle_train_backward):
             fn.restype = ctypes.c_int
         self.lib = lib
 
@@ -179,6 +183,34 @@ class Oracle:
             _dptr(O), n_threads or default_threads())
         self._check(rc, "block_attn_prefix")
         return O
+
+    # -- training form (Stage 1 attention transfer) ---------------------------
+    def train_forward(self, Q, K, V, W, alpha, B, n_threads=None):
+        """Every block of each sequence against the state of the blocks before
+        it.  Q [n_seq, L, Hq, d], K, V [n_seq, L, Hkv, d] -> O [n_seq, L, Hq, d]."""
+        Q, K, V, W, alpha = (_f64(a, "") for a in (Q, K, V, W, alpha))
+        n_seq, L, Hq, d = Q.shape
+        Hkv, F = K.shape[2], W.shape[2]
+        O = np.zeros_like(Q)
+        rc = self.lib.oracle_train_forward(n_seq, L, B, Hq, Hkv, d, F, _dptr(Q), _dptr(K),
+                                           _dptr(V), _dptr(W), _dptr(alpha), _dptr(O),
+                                           n_threads or default_threads())
+        self._check(rc, "train_forward")
+        return O
+
+    def train_backward(self, Q, K, V, W, alpha, dO, B, n_threads=None):
+        """Gradient of sum(dO * O) with respect to W [Hkv, d, F] and alpha [Hq]."""
+        Q, K, V, W, alpha, dO = (_f64(a, "") for a in (Q, K, V, W, alpha, dO))
+        n_seq, L, Hq, d = Q.shape
+        Hkv, F = K.shape[2], W.shape[2]
+        dW = np.zeros_like(W)
+        dalpha = np.zeros_like(alpha)
+        rc = self.lib.oracle_train_backward(n_seq, L, B, Hq, Hkv, d, F, _dptr(Q), _dptr(K),
+                                            _dptr(V), _dptr(W), _dptr(alpha), _dptr(dO),
+                                            _dptr(dW), _dptr(dalpha),
+                                            n_threads or default_threads())
+        self._check(rc, "train_backward")
+        return dW, dalpha
 
 
 _default = None

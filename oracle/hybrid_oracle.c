@@ -21,6 +21,11 @@
  *   w        = sigmoid(alpha)                            (Sec. 3.1, gate)
  *   out      = (w sm_num + lin_num) / (w sm_den + lin_den)      (Sec. 3.1)
  *
+ * The training form (Sec. 3.2, Stage 1) applies the same definitions to every
+ * block of a sequence (oracle_train_forward) and writes out, by the chain
+ * rule, the gradient of sum(dO * O) with respect to W and alpha
+ * (oracle_train_backward).
+ *
  * A second route (oracle_block_attn_prefix) never forms S or Z: it sums the
  * linear branch token by token over the explicit prefix, the left-hand form
  * of Eq. 1.  The two routes are a mutual check (state = explicit sum).
@@ -353,4 +358,291 @@ int oracle_block_attn_prefix(int n_req, int B, int Hq, int Hkv, int d, int F, in
     c.Kp = Kp; c.Vp = Vp; c.prefix_len = prefix_len; c.P_max = P_max; c.O = O;
     const int P2 = phi_width(phi_kind, d, F);
     return fanout(attn_unit, &c, (long)n_req * Hq, n_threads, (size_t)F + 2u * P2 + 2u * d);
+}
+
+/* ===========================================================================
+ * Training form (Sec. 3.2, Stage 1 attention transfer).
+ *
+ * A training sequence of L = n_blk * B tokens is cut into blocks B_0, B_1, ...
+ * of B tokens.  Teacher forcing gives every block its queries, keys and
+ * values; block n attends to itself with the exact softmax branch and to the
+ * blocks before it through S_{n-1}, Z_{n-1} (Sec. 3.1 applied to each block of
+ * the sequence; S_{-1} = 0).  Stage 1 trains only psi = {W, alpha}.
+ *
+ * Layouts: Q, O, dO [n_seq][L][Hq][d];  K, V [n_seq][L][Hkv][d];
+ *          W, dW [Hkv][d][F];  alpha, dalpha [Hq].
+ * ------------------------------------------------------------------------- */
+typedef struct {
+    int n_seq, L, B, Hq, Hkv, d, F;
+    const double *Q, *K, *V, *W, *alpha, *dO;
+    double *O;
+    double *dW_part;       /* [n_seq * Hkv][d][F]  one slot per unit */
+    double *dw_part;       /* [n_seq * Hq]          d loss / d w per (sequence, head) */
+} train_ctx;
+
+/* Forward for one (sequence, query head): block by block, the outputs of the
+ * block's queries against the state of the earlier blocks, then the commit
+ * of the block into that state. */
+static int train_fwd_unit(void *p, long unit, double *scratch)
+{
+    const train_ctx *c = (const train_ctx *)p;
+    const int s = (int)(unit / c->Hq), h = (int)(unit % c->Hq);
+    const int d = c->d, F = c->F, B = c->B, P2 = 2 * F;
+    const int G = c->Hq / c->Hkv, g = h / G;
+    const double *Wg = c->W + (size_t)g * d * F;
+    double *S = scratch;                      /* P2 * d */
+    double *z = S + (size_t)P2 * d;           /* P2     */
+    double *u = z + P2;                       /* F      */
+    double *phi = u + F;                      /* P2     */
+    double *num = phi + P2;                   /* d      */
+    for (size_t i = 0; i < (size_t)P2 * d + P2; ++i) S[i] = 0.0;
+    const double w = 1.0 / (1.0 + exp(-c->alpha[h]));
+    const int n_blk = c->L / B;
+    for (int n = 0; n < n_blk; ++n) {
+        for (int i = 0; i < B; ++i) {
+            const size_t ti = (size_t)s * c->L + (size_t)n * B + i;
+            const double *q = c->Q + (ti * c->Hq + h) * d;
+            double sm_den = 0.0;
+            for (int e = 0; e < d; ++e) num[e] = 0.0;
+            for (int j = 0; j < B; ++j) {
+                const size_t tj = (size_t)s * c->L + (size_t)n * B + j;
+                const double *k = c->K + (tj * c->Hkv + g) * d;
+                const double *v = c->V + (tj * c->Hkv + g) * d;
+                double sc = 0.0;
+                for (int e = 0; e < d; ++e) sc += q[e] * k[e];
+                sc /= sqrt((double)d);
+                if (fabs(sc) > ORACLE_EXP_LIMIT) return -2;
+                const double a = exp(sc);
+                for (int e = 0; e < d; ++e) num[e] += w * a * v[e];
+                sm_den += a;
+            }
+            int rc = phi_one(PHI_HEDGEHOG, q, Wg, d, F, u, phi);
+            if (rc) return rc;
+            double lin_den = 0.0;
+            for (int f = 0; f < P2; ++f) {
+                for (int e = 0; e < d; ++e) num[e] += phi[f] * S[(size_t)f * d + e];
+                lin_den += phi[f] * z[f];
+            }
+            double *o = c->O + (ti * c->Hq + h) * d;
+            const double den = w * sm_den + lin_den;
+            for (int e = 0; e < d; ++e) o[e] = num[e] / den;
+        }
+        for (int t = 0; t < B; ++t) {
+            const size_t tt = (size_t)s * c->L + (size_t)n * B + t;
+            const double *k = c->K + (tt * c->Hkv + g) * d;
+            const double *v = c->V + (tt * c->Hkv + g) * d;
+            int rc = phi_one(PHI_HEDGEHOG, k, Wg, d, F, u, phi);
+            if (rc) return rc;
+            for (int f = 0; f < P2; ++f) {
+                for (int e = 0; e < d; ++e) S[(size_t)f * d + e] += phi[f] * v[e];
+                z[f] += phi[f];
+            }
+        }
+    }
+    return 0;
+}
+
+/* Reverse mode through phi(x) = [softmax(u), softmax(-u)], u = x W, for one
+ * vector: given g = dL/dphi (2F), add dL/dW[e][f] = x[e] * du[f] into dW, with
+ *   du = p+ (g+ - <g+, p+>) - p- (g- - <g-, p->),   p+- = softmax(+-u). */
+static void phi_backward_add(const double *x, const double *phi, const double *gphi, int d, int F,
+                             double *du /* scratch, F */, double *dW)
+{
+    double dot_pos = 0.0, dot_neg = 0.0;
+    for (int f = 0; f < F; ++f) {
+        dot_pos += gphi[f] * phi[f];
+        dot_neg += gphi[F + f] * phi[F + f];
+    }
+    for (int f = 0; f < F; ++f)
+        du[f] = phi[f] * (gphi[f] - dot_pos) - phi[F + f] * (gphi[F + f] - dot_neg);
+    for (int e = 0; e < d; ++e)
+        for (int f = 0; f < F; ++f) dW[(size_t)e * F + f] += x[e] * du[f];
+}
+
+/* Backward for one (sequence, state head g): the gradient of sum(dO * O) with
+ * respect to W_g and to the gates w_h of the G query heads of the group.
+ * Per query row i of block n (N = numerator, D = denominator of the merge):
+ *   dN = g / D,   dD = -(g . o) / D,            g = dO row, o = N / D
+ *   dw_h    += dN . sm_num + dD sm_den
+ *   dphi(q)  = S_{n-1} dN + Z_{n-1} dD,    dS_{n-1} += phi(q) dN^T,  dZ_{n-1} += phi(q) dD
+ * and, since S_{n-1} = sum_{m < n} sum_{t in B_m} phi(k_t) v_t^T, a key t of
+ * block m receives  dphi(k_t) = (sum_{n > m} dS_{n-1}) v_t + sum_{n > m} dZ_{n-1}. */
+static int train_bwd_unit(void *p, long unit, double *scratch)
+{
+    const train_ctx *c = (const train_ctx *)p;
+    const int s = (int)(unit / c->Hkv), g = (int)(unit % c->Hkv);
+    const int d = c->d, F = c->F, B = c->B, P2 = 2 * F;
+    const int G = c->Hq / c->Hkv, n_blk = c->L / B;
+    const size_t st = (size_t)P2 * d + P2;    /* one (S, Z) pair */
+    const double *Wg = c->W + (size_t)g * d * F;
+    double *Spre = scratch;                   /* n_blk states: S_{n-1}, Z_{n-1} for block n */
+    double *dSpre = Spre + (size_t)n_blk * st;/* n_blk gradients of those states */
+    double *u = dSpre + (size_t)n_blk * st;   /* F  */
+    double *phi = u + F;                      /* P2 */
+    double *gphi = phi + P2;                  /* P2 */
+    double *sm_num = gphi + P2;               /* d  */
+    double *o = sm_num + d;                   /* d  */
+    double *dN = o + d;                       /* d  */
+    double *du = dN + d;                      /* F  */
+    double *acc = du + F;                     /* st: running sum of dS over later blocks */
+    double *dW = c->dW_part + (size_t)unit * d * F;
+    for (size_t i = 0; i < (size_t)n_blk * st; ++i) { Spre[i] = 0.0; dSpre[i] = 0.0; }
+    for (size_t i = 0; i < (size_t)d * F; ++i) dW[i] = 0.0;
+
+    /* prefix states: S_{n-1} = S_{n-2} + commit(B_{n-1}) */
+    for (int n = 1; n < n_blk; ++n) {
+        double *Sn = Spre + (size_t)n * st, *zn = Sn + (size_t)P2 * d;
+        const double *Sp = Spre + (size_t)(n - 1) * st;
+        for (size_t i = 0; i < st; ++i) Sn[i] = Sp[i];
+        for (int t = 0; t < B; ++t) {
+            const size_t tt = (size_t)s * c->L + (size_t)(n - 1) * B + t;
+            const double *k = c->K + (tt * c->Hkv + g) * d;
+            const double *v = c->V + (tt * c->Hkv + g) * d;
+            int rc = phi_one(PHI_HEDGEHOG, k, Wg, d, F, u, phi);
+            if (rc) return rc;
+            for (int f = 0; f < P2; ++f) {
+                for (int e = 0; e < d; ++e) Sn[(size_t)f * d + e] += phi[f] * v[e];
+                zn[f] += phi[f];
+            }
+        }
+    }
+
+    /* query side */
+    for (int hl = 0; hl < G; ++hl) {
+        const int h = g * G + hl;
+        const double w = 1.0 / (1.0 + exp(-c->alpha[h]));
+        double dw = 0.0;
+        for (int n = 0; n < n_blk; ++n) {
+            const double *S = Spre + (size_t)n * st, *z = S + (size_t)P2 * d;
+            double *dS = dSpre + (size_t)n * st, *dz = dS + (size_t)P2 * d;
+            for (int i = 0; i < B; ++i) {
+                const size_t ti = (size_t)s * c->L + (size_t)n * B + i;
+                const double *q = c->Q + (ti * c->Hq + h) * d;
+                const double *gr = c->dO + (ti * c->Hq + h) * d;
+                double sm_den = 0.0;
+                for (int e = 0; e < d; ++e) sm_num[e] = 0.0;
+                for (int j = 0; j < B; ++j) {
+                    const size_t tj = (size_t)s * c->L + (size_t)n * B + j;
+                    const double *k = c->K + (tj * c->Hkv + g) * d;
+                    const double *v = c->V + (tj * c->Hkv + g) * d;
+                    double sc = 0.0;
+                    for (int e = 0; e < d; ++e) sc += q[e] * k[e];
+                    sc /= sqrt((double)d);
+                    if (fabs(sc) > ORACLE_EXP_LIMIT) return -2;
+                    const double a = exp(sc);
+                    for (int e = 0; e < d; ++e) sm_num[e] += a * v[e];
+                    sm_den += a;
+                }
+                int rc = phi_one(PHI_HEDGEHOG, q, Wg, d, F, u, phi);
+                if (rc) return rc;
+                double lin_den = 0.0;
+                for (int e = 0; e < d; ++e) o[e] = w * sm_num[e];
+                for (int f = 0; f < P2; ++f) {
+                    for (int e = 0; e < d; ++e) o[e] += phi[f] * S[(size_t)f * d + e];
+                    lin_den += phi[f] * z[f];
+                }
+                const double D = w * sm_den + lin_den;
+                double go = 0.0;
+                for (int e = 0; e < d; ++e) {
+                    o[e] /= D;
+                    go += gr[e] * o[e];
+                }
+                const double dD = -go / D;
+                for (int e = 0; e < d; ++e) dN[e] = gr[e] / D;
+                for (int e = 0; e < d; ++e) dw += dN[e] * sm_num[e];
+                dw += dD * sm_den;
+                for (int f = 0; f < P2; ++f) {
+                    double acc_f = z[f] * dD;
+                    for (int e = 0; e < d; ++e) acc_f += S[(size_t)f * d + e] * dN[e];
+                    gphi[f] = acc_f;
+                    for (int e = 0; e < d; ++e) dS[(size_t)f * d + e] += phi[f] * dN[e];
+                    dz[f] += phi[f] * dD;
+                }
+                phi_backward_add(q, phi, gphi, d, F, du, dW);
+            }
+        }
+        c->dw_part[(size_t)s * c->Hq + h] = dw;
+    }
+
+    /* key side: block m gets the sum of dS_{n-1} over the later blocks n > m */
+    for (size_t i = 0; i < st; ++i) acc[i] = 0.0;
+    for (int m = n_blk - 1; m >= 0; --m) {
+        if (m + 1 < n_blk) {
+            const double *dS = dSpre + (size_t)(m + 1) * st;
+            for (size_t i = 0; i < st; ++i) acc[i] += dS[i];
+        }
+        const double *dz = acc + (size_t)P2 * d;
+        for (int t = 0; t < B; ++t) {
+            const size_t tt = (size_t)s * c->L + (size_t)m * B + t;
+            const double *k = c->K + (tt * c->Hkv + g) * d;
+            const double *v = c->V + (tt * c->Hkv + g) * d;
+            int rc = phi_one(PHI_HEDGEHOG, k, Wg, d, F, u, phi);
+            if (rc) return rc;
+            for (int f = 0; f < P2; ++f) {
+                double acc_f = dz[f];
+                for (int e = 0; e < d; ++e) acc_f += acc[(size_t)f * d + e] * v[e];
+                gphi[f] = acc_f;
+            }
+            phi_backward_add(k, phi, gphi, d, F, du, dW);
+        }
+    }
+    return 0;
+}
+
+static int train_check(int n_seq, int L, int B, int Hq, int Hkv, int d, int F)
+{
+    if (n_seq < 0 || L < 0 || B <= 0 || Hq <= 0 || Hkv <= 0 || d <= 0 || F <= 0) return -1;
+    if (Hq % Hkv != 0 || L % B != 0) return -1;
+    return 0;
+}
+
+int oracle_train_forward(int n_seq, int L, int B, int Hq, int Hkv, int d, int F,
+                         const double *Q, const double *K, const double *V,
+                         const double *W, const double *alpha, double *O, int n_threads)
+{
+    if (train_check(n_seq, L, B, Hq, Hkv, d, F) || !W) return -1;
+    train_ctx c;
+    memset(&c, 0, sizeof c);
+    c.n_seq = n_seq; c.L = L; c.B = B; c.Hq = Hq; c.Hkv = Hkv; c.d = d; c.F = F;
+    c.Q = Q; c.K = K; c.V = V; c.W = W; c.alpha = alpha; c.O = O;
+    const size_t P2 = 2u * (size_t)F;
+    return fanout(train_fwd_unit, &c, (long)n_seq * Hq, n_threads,
+                  P2 * d + 2 * P2 + (size_t)F + (size_t)d);
+}
+
+/* dW [Hkv][d][F] and dalpha [Hq] of sum(dO * O); dalpha_h = dw_h * w_h (1 - w_h). */
+int oracle_train_backward(int n_seq, int L, int B, int Hq, int Hkv, int d, int F,
+                          const double *Q, const double *K, const double *V,
+                          const double *W, const double *alpha, const double *dO,
+                          double *dW, double *dalpha, int n_threads)
+{
+    if (train_check(n_seq, L, B, Hq, Hkv, d, F) || !W || !dO || !dW || !dalpha) return -1;
+    const size_t P2 = 2u * (size_t)F, st = P2 * d + P2;
+    const int n_blk = B > 0 ? L / B : 0;
+    train_ctx c;
+    memset(&c, 0, sizeof c);
+    c.n_seq = n_seq; c.L = L; c.B = B; c.Hq = Hq; c.Hkv = Hkv; c.d = d; c.F = F;
+    c.Q = Q; c.K = K; c.V = V; c.W = W; c.alpha = alpha; c.dO = dO;
+    c.dW_part = (double *)calloc((size_t)n_seq * Hkv * d * F + 1, sizeof(double));
+    c.dw_part = (double *)calloc((size_t)n_seq * Hq + 1, sizeof(double));
+    if (!c.dW_part || !c.dw_part) { free(c.dW_part); free(c.dw_part); return -1; }
+    int rc = fanout(train_bwd_unit, &c, (long)n_seq * Hkv, n_threads,
+                    2 * (size_t)n_blk * st + 3 * P2 + 3 * (size_t)d + 2 * (size_t)F + st);
+    if (rc == 0) {
+        for (int g = 0; g < Hkv; ++g)
+            for (size_t i = 0; i < (size_t)d * F; ++i) {
+                double a = 0.0;
+                for (int s = 0; s < n_seq; ++s) a += c.dW_part[((size_t)s * Hkv + g) * d * F + i];
+                dW[(size_t)g * d * F + i] = a;
+            }
+        for (int h = 0; h < Hq; ++h) {
+            const double w = 1.0 / (1.0 + exp(-alpha[h]));
+            double a = 0.0;
+            for (int s = 0; s < n_seq; ++s) a += c.dw_part[(size_t)s * Hq + h];
+            dalpha[h] = a * w * (1.0 - w);
+        }
+    }
+    free(c.dW_part);
+    free(c.dw_part);
+    return rc;
 }

@@ -410,6 +410,106 @@ def pin_large_keys(orc):
             assert np.all(O1[r, :, h] >= vals.min(0) - 1e-9), "convexity (min)"
 
 
+# --------------------------------------------------------------------------
+# Training form (Sec. 3.2, Stage 1): every block of a sequence against the
+# state of the blocks before it, and the gradient with respect to W and alpha.
+# --------------------------------------------------------------------------
+def _train_problem(rng, n_seq=2, n_blk=3, B=2, Hq=4, Hkv=2, d=4, F=3):
+    L = n_blk * B
+    return dict(
+        Q=rng.standard_normal((n_seq, L, Hq, d)),
+        K=rng.standard_normal((n_seq, L, Hkv, d)),
+        V=rng.standard_normal((n_seq, L, Hkv, d)),
+        W=rng.standard_normal((Hkv, d, F)) / math.sqrt(d),
+        alpha=rng.uniform(-1.0, 1.5, Hq),
+        dO=rng.standard_normal((n_seq, L, Hq, d)),
+        B=B, n_blk=n_blk)
+
+
+def pin_train_forward_is_prefix_route(orc):
+    """Block n of a training sequence is one block-hybrid step whose linear
+    branch is summed token by token over the n*B earlier tokens (Eq. 1 route,
+    which never forms a state)."""
+    p = _train_problem(_rng(31), n_seq=2, n_blk=4, B=3, Hq=4, Hkv=2, d=5, F=3)
+    B = p["B"]
+    O = orc.train_forward(p["Q"], p["K"], p["V"], p["W"], p["alpha"], B)
+    for n in range(p["n_blk"]):
+        blk = slice(n * B, (n + 1) * B)
+        On = orc.block_attn_prefix(p["Q"][:, blk], p["K"][:, blk], p["V"][:, blk], p["W"],
+                                   p["alpha"], p["K"], p["V"], [n * B] * 2)
+        _close(O[:, blk], On, rtol=1e-11, atol=1e-12, what=f"training block {n}")
+
+
+def _train_loss(orc, p, W, alpha):
+    O = orc.train_forward(p["Q"], p["K"], p["V"], W, alpha, p["B"], n_threads=1)
+    return float(np.sum(p["dO"] * O))
+
+
+def pin_train_backward_finite_differences(orc):
+    """dW and dalpha are the derivatives of sum(dO * O): central differences of
+    the training forward, element by element."""
+    p = _train_problem(_rng(32))
+    dW, dalpha = orc.train_backward(p["Q"], p["K"], p["V"], p["W"], p["alpha"], p["dO"], p["B"])
+    h = 1e-6
+    fd_W = np.zeros_like(p["W"])
+    for idx in np.ndindex(*p["W"].shape):
+        Wp, Wm = p["W"].copy(), p["W"].copy()
+        Wp[idx] += h
+        Wm[idx] -= h
+        fd_W[idx] = (_train_loss(orc, p, Wp, p["alpha"]) - _train_loss(orc, p, Wm, p["alpha"])) / (2 * h)
+    fd_a = np.zeros_like(p["alpha"])
+    for i in range(p["alpha"].size):
+        ap, am = p["alpha"].copy(), p["alpha"].copy()
+        ap[i] += h
+        am[i] -= h
+        fd_a[i] = (_train_loss(orc, p, p["W"], ap) - _train_loss(orc, p, p["W"], am)) / (2 * h)
+    _close(dW, fd_W, rtol=1e-6, atol=1e-7, what="dW vs central differences")
+    _close(dalpha, fd_a, rtol=1e-6, atol=1e-7, what="dalpha vs central differences")
+    assert np.abs(fd_W).max() > 1e-3 and np.abs(fd_a).max() > 1e-3, "degenerate problem"
+
+
+def pin_train_backward_single_block(orc):
+    """With one block per sequence no query has a prefix: O is the in-block
+    softmax alone, independent of W and alpha, so both gradients are zero
+    (dW exactly: every state and state gradient is zero; dalpha to rounding,
+    as the two terms of dw cancel)."""
+    p = _train_problem(_rng(33), n_blk=1, B=4)
+    dW, dalpha = orc.train_backward(p["Q"], p["K"], p["V"], p["W"], p["alpha"], p["dO"], p["B"])
+    assert np.all(dW == 0.0) and np.abs(dalpha).max() < 1e-12, "gradients without any prefix"
+
+
+def pin_train_backward_constant_values(orc):
+    """V = 1 everywhere makes every output exactly 1 for any W and alpha (the
+    attention mass sums to one), so both gradients vanish."""
+    p = _train_problem(_rng(34), n_blk=4)
+    p["V"] = np.ones_like(p["V"])
+    dW, dalpha = orc.train_backward(p["Q"], p["K"], p["V"], p["W"], p["alpha"], p["dO"], p["B"])
+    assert np.abs(dW).max() < 1e-12 and np.abs(dalpha).max() < 1e-12, "gradients with V = 1"
+
+
+def pin_train_backward_linear_in_dO(orc):
+    """The gradient of sum(dO * O) is linear in dO."""
+    p = _train_problem(_rng(35))
+    rng = _rng(36)
+    d1, d2 = p["dO"], rng.standard_normal(p["dO"].shape)
+    args = (p["Q"], p["K"], p["V"], p["W"], p["alpha"])
+    g1 = orc.train_backward(*args, d1, p["B"])
+    g2 = orc.train_backward(*args, d2, p["B"])
+    g3 = orc.train_backward(*args, 2.0 * d1 - 3.0 * d2, p["B"])
+    for a, b, c, what in zip(g1, g2, g3, ("dW", "dalpha")):
+        _close(c, 2.0 * a - 3.0 * b, rtol=1e-10, atol=1e-12, what=f"{what} linear in dO")
+
+
+def pin_train_backward_saturated_gate(orc):
+    """w = sigmoid(alpha) is flat at alpha = +inf: dalpha is zero there, and dW
+    is the gradient of the model whose gate is exactly 1."""
+    p = _train_problem(_rng(37))
+    a = p["alpha"].copy()
+    a[1] = np.inf
+    dW, dalpha = orc.train_backward(p["Q"], p["K"], p["V"], p["W"], a, p["dO"], p["B"])
+    assert dalpha[1] == 0.0 and np.all(np.isfinite(dW)), "saturated gate"
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]
 
 

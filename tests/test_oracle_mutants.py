@@ -41,6 +41,21 @@ MUTANTS = [
     ("prefix route skips last token", "for (int t = 0; t < P; ++t) {", "for (int t = 0; t + 1 < P; ++t) {"),
     ("value index shifted", "for (int e = 0; e < d; ++e) sm_num[e] += a * v[e];",
      "for (int e = 0; e < d; ++e) sm_num[e] += a * v[(e + 1) % d];"),
+    # training form (Stage 1): forward over a sequence and the gradient of W, alpha
+    ("train forward gate dropped", "num[e] += w * a * v[e];", "num[e] += a * v[e];"),
+    ("train forward sees own block", "        for (int t = 0; t < B; ++t) {\n            const size_t tt = (size_t)s * c->L + (size_t)n * B + t;",
+     "        for (int t = 0; t < B && n < 0; ++t) {\n            const size_t tt = (size_t)s * c->L + (size_t)n * B + t;"),
+    ("train dD sign", "const double dD = -go / D;", "const double dD = go / D;"),
+    ("train z gradient dropped", "double acc_f = z[f] * dD;", "double acc_f = 0.0 * dD;"),
+    ("train phi backward negative half sign", "- phi[F + f] * (gphi[F + f] - dot_neg);",
+     "+ phi[F + f] * (gphi[F + f] - dot_neg);"),
+    ("train key side uses its own block", "const double *dS = dSpre + (size_t)(m + 1) * st;",
+     "const double *dS = dSpre + (size_t)m * st;"),
+    ("train key gradient ignores values", "acc_f += acc[(size_t)f * d + e] * v[e];",
+     "acc_f += acc[(size_t)f * d + e];"),
+    ("train dalpha without the sigmoid slope", "dalpha[h] = a * w * (1.0 - w);", "dalpha[h] = a;"),
+    ("train state gradient of own block", "dS[(size_t)f * d + e] += phi[f] * dN[e];",
+     "dS[(size_t)f * d + e] += phi[f] * dN[(e + 1) % d];"),
 ]
 
 
