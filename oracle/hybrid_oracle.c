@@ -104,6 +104,78 @@ static int phi_one(int phi_kind, const double *x, const double *W, int d, int F,
 }
 
 /* ---------------------------------------------------------------------------
+ * The definitions of Sec. 3.1 that every route below shares, one routine each.
+ * ------------------------------------------------------------------------- */
+
+/* Gate w = sigma(alpha) = 1 / (1 + exp(-alpha)); alpha = -inf gives 0, +inf gives 1. */
+static double gate(double alpha)
+{
+    return 1.0 / (1.0 + exp(-alpha));
+}
+
+/* GQA: query head h reads the state (and W) of state head h / G, G = Hq / Hkv. */
+static int group_of(int h, int Hq, int Hkv)
+{
+    const int G = Hq / Hkv;
+    return h / G;
+}
+
+/* Within-block softmax branch for one query q over the B keys / values of
+ * its block (row j at K + j*stride, V + j*stride):
+ *   a_j = exp(q . k_j / sqrt(d)),  sm_num = sum_j a_j v_j,  sm_den = sum_j a_j. */
+static int softmax_branch(const double *q, const double *K, const double *V, size_t stride, int B,
+                          int d, double *sm_num, double *sm_den_out)
+{
+    double sm_den = 0.0;
+    for (int e = 0; e < d; ++e) sm_num[e] = 0.0;
+    for (int j = 0; j < B; ++j) {
+        const double *k = K + (size_t)j * stride;
+        const double *v = V + (size_t)j * stride;
+        double s = 0.0;
+        for (int e = 0; e < d; ++e) s += q[e] * k[e];
+        s /= sqrt((double)d);
+        if (fabs(s) > ORACLE_EXP_LIMIT) return -2;
+        const double a = exp(s);
+        for (int e = 0; e < d; ++e) sm_num[e] += a * v[e];
+        sm_den += a;
+    }
+    *sm_den_out = sm_den;
+    return 0;
+}
+
+/* Cross-block branch read from the state: lin_num = phi(q)^T S, lin_den = phi(q)^T z. */
+static void linear_branch(const double *phi_q, const double *S, const double *z, int P2, int d,
+                          double *lin_num, double *lin_den_out)
+{
+    double lin_den = 0.0;
+    for (int e = 0; e < d; ++e) lin_num[e] = 0.0;
+    for (int f = 0; f < P2; ++f) {
+        for (int e = 0; e < d; ++e) lin_num[e] += phi_q[f] * S[(size_t)f * d + e];
+        lin_den += phi_q[f] * z[f];
+    }
+    *lin_den_out = lin_den;
+}
+
+/* Gated shared normaliser: out = (w sm_num + lin_num) / (w sm_den + lin_den);
+ * returns the denominator. */
+static double merge(double w, const double *sm_num, double sm_den, const double *lin_num,
+                    double lin_den, int d, double *o)
+{
+    const double den = w * sm_den + lin_den;
+    for (int e = 0; e < d; ++e) o[e] = (w * sm_num[e] + lin_num[e]) / den;
+    return den;
+}
+
+/* Commit of one token: S += phi(k) v^T, z += phi(k). */
+static void commit_token(const double *phi, const double *v, int P2, int d, double *S, double *z)
+{
+    for (int f = 0; f < P2; ++f) {
+        for (int e = 0; e < d; ++e) S[(size_t)f * d + e] += phi[f] * v[e];
+        z[f] += phi[f];
+    }
+}
+
+/* ---------------------------------------------------------------------------
  * Feature map on a batch of rows.
  *   X   [n_rows][n_heads_x][d],  W [Hkv][d][F],  Phi [n_rows][n_heads_x][2F]
  * Row head h uses W[h / (n_heads_x / Hkv)] (queries: h / G; keys: h).
@@ -209,10 +281,7 @@ static int commit_unit(void *p, long unit, double *scratch)
         const double *v = c->V + (((size_t)r * c->T + t) * c->Hkv + g) * d;
         int rc = phi_one(c->phi_kind, k, Wg, d, F, u, phi);
         if (rc) return rc;
-        for (int f = 0; f < P2; ++f) {
-            for (int e = 0; e < d; ++e) S[(size_t)f * d + e] += phi[f] * v[e];
-            z[f] += phi[f];
-        }
+        commit_token(phi, v, P2, d, S, z);
     }
     return 0;
 }
@@ -251,7 +320,7 @@ static int attn_unit(void *p, long unit, double *scratch)
     const attn_ctx *c = (const attn_ctx *)p;
     const int r = (int)(unit / c->Hq), h = (int)(unit % c->Hq);
     const int d = c->d, F = c->F, B = c->B;
-    const int G = c->Hq / c->Hkv, g = h / G;
+    const int g = group_of(h, c->Hq, c->Hkv);
     const int P2 = phi_width(c->phi_kind, d, F);
     const double *Wg = c->W ? c->W + (size_t)g * d * F : NULL;
 
@@ -261,41 +330,28 @@ static int attn_unit(void *p, long unit, double *scratch)
     double *sm_num = phi_k + P2;         /* d      */
     double *lin_num = sm_num + d;        /* d      */
 
-    /* gate w = sigma(alpha) = 1 / (1 + exp(-alpha)); alpha = -inf gives 0, +inf gives 1 */
-    const double w = 1.0 / (1.0 + exp(-c->alpha[h]));
+    const double w = gate(c->alpha[h]);
 
     for (int i = 0; i < B; ++i) {
         const double *q = c->Q + (((size_t)r * B + i) * c->Hq + h) * d;
 
         /* within-block softmax branch: a_j = exp(q . k_j / sqrt(d)) over all j of the block */
         double sm_den = 0.0;
-        for (int e = 0; e < d; ++e) sm_num[e] = 0.0;
-        for (int j = 0; j < B; ++j) {
-            const double *k = c->K + (((size_t)r * B + j) * c->Hkv + g) * d;
-            const double *v = c->V + (((size_t)r * B + j) * c->Hkv + g) * d;
-            double s = 0.0;
-            for (int e = 0; e < d; ++e) s += q[e] * k[e];
-            s /= sqrt((double)d);
-            if (fabs(s) > ORACLE_EXP_LIMIT) return -2;
-            const double a = exp(s);
-            for (int e = 0; e < d; ++e) sm_num[e] += a * v[e];
-            sm_den += a;
-        }
+        const size_t kv0 = ((size_t)r * B * c->Hkv + g) * d;
+        int rc = softmax_branch(q, c->K + kv0, c->V + kv0, (size_t)c->Hkv * d, B, d, sm_num, &sm_den);
+        if (rc) return rc;
 
         /* cross-block linear branch */
-        int rc = phi_one(c->phi_kind, q, Wg, d, F, u, phi_q);
+        rc = phi_one(c->phi_kind, q, Wg, d, F, u, phi_q);
         if (rc) return rc;
         double lin_den = 0.0;
-        for (int e = 0; e < d; ++e) lin_num[e] = 0.0;
         if (c->S) {
             /* route 1: lin_num = phi(q)^T S, lin_den = phi(q)^T z */
             const double *S = c->S + ((size_t)r * c->Hkv + g) * P2 * d;
             const double *z = c->z + ((size_t)r * c->Hkv + g) * P2;
-            for (int f = 0; f < P2; ++f) {
-                for (int e = 0; e < d; ++e) lin_num[e] += phi_q[f] * S[(size_t)f * d + e];
-                lin_den += phi_q[f] * z[f];
-            }
+            linear_branch(phi_q, S, z, P2, d, lin_num, &lin_den);
         } else {
+            for (int e = 0; e < d; ++e) lin_num[e] = 0.0;
             /* route 2: lin_num = sum_t (phi(q) . phi(k_t)) v_t over the prefix tokens (Eq. 1) */
             const int P = c->prefix_len[r];
             for (int t = 0; t < P; ++t) {
@@ -311,9 +367,7 @@ static int attn_unit(void *p, long unit, double *scratch)
         }
 
         /* gated merge through the shared normaliser */
-        double *o = c->O + (((size_t)r * B + i) * c->Hq + h) * d;
-        const double den = w * sm_den + lin_den;
-        for (int e = 0; e < d; ++e) o[e] = (w * sm_num[e] + lin_num[e]) / den;
+        merge(w, sm_num, sm_den, lin_num, lin_den, d, c->O + (((size_t)r * B + i) * c->Hq + h) * d);
     }
     return 0;
 }
@@ -388,55 +442,37 @@ static int train_fwd_unit(void *p, long unit, double *scratch)
     const train_ctx *c = (const train_ctx *)p;
     const int s = (int)(unit / c->Hq), h = (int)(unit % c->Hq);
     const int d = c->d, F = c->F, B = c->B, P2 = 2 * F;
-    const int G = c->Hq / c->Hkv, g = h / G;
+    const int g = group_of(h, c->Hq, c->Hkv);
     const double *Wg = c->W + (size_t)g * d * F;
+    const size_t q_row = (size_t)c->Hq * d, kv_row = (size_t)c->Hkv * d;
     double *S = scratch;                      /* P2 * d */
     double *z = S + (size_t)P2 * d;           /* P2     */
     double *u = z + P2;                       /* F      */
     double *phi = u + F;                      /* P2     */
-    double *num = phi + P2;                   /* d      */
+    double *sm_num = phi + P2;                /* d      */
+    double *lin_num = sm_num + d;             /* d      */
     for (size_t i = 0; i < (size_t)P2 * d + P2; ++i) S[i] = 0.0;
-    const double w = 1.0 / (1.0 + exp(-c->alpha[h]));
+    const double w = gate(c->alpha[h]);
     const int n_blk = c->L / B;
     for (int n = 0; n < n_blk; ++n) {
+        const size_t t0 = (size_t)s * c->L + (size_t)n * B;   /* first token of block n */
+        const double *Kb = c->K + t0 * kv_row + (size_t)g * d;
+        const double *Vb = c->V + t0 * kv_row + (size_t)g * d;
         for (int i = 0; i < B; ++i) {
-            const size_t ti = (size_t)s * c->L + (size_t)n * B + i;
-            const double *q = c->Q + (ti * c->Hq + h) * d;
-            double sm_den = 0.0;
-            for (int e = 0; e < d; ++e) num[e] = 0.0;
-            for (int j = 0; j < B; ++j) {
-                const size_t tj = (size_t)s * c->L + (size_t)n * B + j;
-                const double *k = c->K + (tj * c->Hkv + g) * d;
-                const double *v = c->V + (tj * c->Hkv + g) * d;
-                double sc = 0.0;
-                for (int e = 0; e < d; ++e) sc += q[e] * k[e];
-                sc /= sqrt((double)d);
-                if (fabs(sc) > ORACLE_EXP_LIMIT) return -2;
-                const double a = exp(sc);
-                for (int e = 0; e < d; ++e) num[e] += w * a * v[e];
-                sm_den += a;
-            }
-            int rc = phi_one(PHI_HEDGEHOG, q, Wg, d, F, u, phi);
+            const double *q = c->Q + (t0 + i) * q_row + (size_t)h * d;
+            double sm_den, lin_den;
+            int rc = softmax_branch(q, Kb, Vb, kv_row, B, d, sm_num, &sm_den);
             if (rc) return rc;
-            double lin_den = 0.0;
-            for (int f = 0; f < P2; ++f) {
-                for (int e = 0; e < d; ++e) num[e] += phi[f] * S[(size_t)f * d + e];
-                lin_den += phi[f] * z[f];
-            }
-            double *o = c->O + (ti * c->Hq + h) * d;
-            const double den = w * sm_den + lin_den;
-            for (int e = 0; e < d; ++e) o[e] = num[e] / den;
+            rc = phi_one(PHI_HEDGEHOG, q, Wg, d, F, u, phi);
+            if (rc) return rc;
+            linear_branch(phi, S, z, P2, d, lin_num, &lin_den);
+            merge(w, sm_num, sm_den, lin_num, lin_den, d, c->O + (t0 + i) * q_row + (size_t)h * d);
         }
+        /* block n commits after its own readout */
         for (int t = 0; t < B; ++t) {
-            const size_t tt = (size_t)s * c->L + (size_t)n * B + t;
-            const double *k = c->K + (tt * c->Hkv + g) * d;
-            const double *v = c->V + (tt * c->Hkv + g) * d;
-            int rc = phi_one(PHI_HEDGEHOG, k, Wg, d, F, u, phi);
+            int rc = phi_one(PHI_HEDGEHOG, Kb + (size_t)t * kv_row, Wg, d, F, u, phi);
             if (rc) return rc;
-            for (int f = 0; f < P2; ++f) {
-                for (int e = 0; e < d; ++e) S[(size_t)f * d + e] += phi[f] * v[e];
-                z[f] += phi[f];
-            }
+            commit_token(phi, Vb + (size_t)t * kv_row, P2, d, S, z);
         }
     }
     return 0;
@@ -474,6 +510,7 @@ static int train_bwd_unit(void *p, long unit, double *scratch)
     const int d = c->d, F = c->F, B = c->B, P2 = 2 * F;
     const int G = c->Hq / c->Hkv, n_blk = c->L / B;
     const size_t st = (size_t)P2 * d + P2;    /* one (S, Z) pair */
+    const size_t q_row = (size_t)c->Hq * d, kv_row = (size_t)c->Hkv * d;
     const double *Wg = c->W + (size_t)g * d * F;
     double *Spre = scratch;                   /* n_blk states: S_{n-1}, Z_{n-1} for block n */
     double *dSpre = Spre + (size_t)n_blk * st;/* n_blk gradients of those states */
@@ -481,7 +518,8 @@ static int train_bwd_unit(void *p, long unit, double *scratch)
     double *phi = u + F;                      /* P2 */
     double *gphi = phi + P2;                  /* P2 */
     double *sm_num = gphi + P2;               /* d  */
-    double *o = sm_num + d;                   /* d  */
+    double *lin_num = sm_num + d;             /* d  */
+    double *o = lin_num + d;                  /* d  */
     double *dN = o + d;                       /* d  */
     double *du = dN + d;                      /* F  */
     double *acc = du + F;                     /* st: running sum of dS over later blocks */
@@ -491,62 +529,40 @@ static int train_bwd_unit(void *p, long unit, double *scratch)
 
     /* prefix states: S_{n-1} = S_{n-2} + commit(B_{n-1}) */
     for (int n = 1; n < n_blk; ++n) {
-        double *Sn = Spre + (size_t)n * st, *zn = Sn + (size_t)P2 * d;
-        const double *Sp = Spre + (size_t)(n - 1) * st;
-        for (size_t i = 0; i < st; ++i) Sn[i] = Sp[i];
+        double *Sn = Spre + (size_t)n * st;
+        for (size_t i = 0; i < st; ++i) Sn[i] = Sn[i - st];
+        const size_t t0 = (size_t)s * c->L + (size_t)(n - 1) * B;
         for (int t = 0; t < B; ++t) {
-            const size_t tt = (size_t)s * c->L + (size_t)(n - 1) * B + t;
-            const double *k = c->K + (tt * c->Hkv + g) * d;
-            const double *v = c->V + (tt * c->Hkv + g) * d;
-            int rc = phi_one(PHI_HEDGEHOG, k, Wg, d, F, u, phi);
+            const size_t kv = (t0 + t) * kv_row + (size_t)g * d;
+            int rc = phi_one(PHI_HEDGEHOG, c->K + kv, Wg, d, F, u, phi);
             if (rc) return rc;
-            for (int f = 0; f < P2; ++f) {
-                for (int e = 0; e < d; ++e) Sn[(size_t)f * d + e] += phi[f] * v[e];
-                zn[f] += phi[f];
-            }
+            commit_token(phi, c->V + kv, P2, d, Sn, Sn + (size_t)P2 * d);
         }
     }
 
     /* query side */
     for (int hl = 0; hl < G; ++hl) {
         const int h = g * G + hl;
-        const double w = 1.0 / (1.0 + exp(-c->alpha[h]));
+        const double w = gate(c->alpha[h]);
         double dw = 0.0;
         for (int n = 0; n < n_blk; ++n) {
             const double *S = Spre + (size_t)n * st, *z = S + (size_t)P2 * d;
             double *dS = dSpre + (size_t)n * st, *dz = dS + (size_t)P2 * d;
+            const size_t t0 = (size_t)s * c->L + (size_t)n * B;
+            const double *Kb = c->K + t0 * kv_row + (size_t)g * d;
+            const double *Vb = c->V + t0 * kv_row + (size_t)g * d;
             for (int i = 0; i < B; ++i) {
-                const size_t ti = (size_t)s * c->L + (size_t)n * B + i;
-                const double *q = c->Q + (ti * c->Hq + h) * d;
-                const double *gr = c->dO + (ti * c->Hq + h) * d;
-                double sm_den = 0.0;
-                for (int e = 0; e < d; ++e) sm_num[e] = 0.0;
-                for (int j = 0; j < B; ++j) {
-                    const size_t tj = (size_t)s * c->L + (size_t)n * B + j;
-                    const double *k = c->K + (tj * c->Hkv + g) * d;
-                    const double *v = c->V + (tj * c->Hkv + g) * d;
-                    double sc = 0.0;
-                    for (int e = 0; e < d; ++e) sc += q[e] * k[e];
-                    sc /= sqrt((double)d);
-                    if (fabs(sc) > ORACLE_EXP_LIMIT) return -2;
-                    const double a = exp(sc);
-                    for (int e = 0; e < d; ++e) sm_num[e] += a * v[e];
-                    sm_den += a;
-                }
-                int rc = phi_one(PHI_HEDGEHOG, q, Wg, d, F, u, phi);
+                const double *q = c->Q + (t0 + i) * q_row + (size_t)h * d;
+                const double *gr = c->dO + (t0 + i) * q_row + (size_t)h * d;
+                double sm_den, lin_den;
+                int rc = softmax_branch(q, Kb, Vb, kv_row, B, d, sm_num, &sm_den);
                 if (rc) return rc;
-                double lin_den = 0.0;
-                for (int e = 0; e < d; ++e) o[e] = w * sm_num[e];
-                for (int f = 0; f < P2; ++f) {
-                    for (int e = 0; e < d; ++e) o[e] += phi[f] * S[(size_t)f * d + e];
-                    lin_den += phi[f] * z[f];
-                }
-                const double D = w * sm_den + lin_den;
+                rc = phi_one(PHI_HEDGEHOG, q, Wg, d, F, u, phi);
+                if (rc) return rc;
+                linear_branch(phi, S, z, P2, d, lin_num, &lin_den);
+                const double D = merge(w, sm_num, sm_den, lin_num, lin_den, d, o);
                 double go = 0.0;
-                for (int e = 0; e < d; ++e) {
-                    o[e] /= D;
-                    go += gr[e] * o[e];
-                }
+                for (int e = 0; e < d; ++e) go += gr[e] * o[e];
                 const double dD = -go / D;
                 for (int e = 0; e < d; ++e) dN[e] = gr[e] / D;
                 for (int e = 0; e < d; ++e) dw += dN[e] * sm_num[e];
@@ -572,10 +588,10 @@ static int train_bwd_unit(void *p, long unit, double *scratch)
             for (size_t i = 0; i < st; ++i) acc[i] += dS[i];
         }
         const double *dz = acc + (size_t)P2 * d;
+        const size_t t0 = (size_t)s * c->L + (size_t)m * B;
         for (int t = 0; t < B; ++t) {
-            const size_t tt = (size_t)s * c->L + (size_t)m * B + t;
-            const double *k = c->K + (tt * c->Hkv + g) * d;
-            const double *v = c->V + (tt * c->Hkv + g) * d;
+            const size_t kv = (t0 + t) * kv_row + (size_t)g * d;
+            const double *k = c->K + kv, *v = c->V + kv;
             int rc = phi_one(PHI_HEDGEHOG, k, Wg, d, F, u, phi);
             if (rc) return rc;
             for (int f = 0; f < P2; ++f) {
@@ -607,7 +623,7 @@ int oracle_train_forward(int n_seq, int L, int B, int Hq, int Hkv, int d, int F,
     c.Q = Q; c.K = K; c.V = V; c.W = W; c.alpha = alpha; c.O = O;
     const size_t P2 = 2u * (size_t)F;
     return fanout(train_fwd_unit, &c, (long)n_seq * Hq, n_threads,
-                  P2 * d + 2 * P2 + (size_t)F + (size_t)d);
+                  P2 * d + 2 * P2 + (size_t)F + 2 * (size_t)d);
 }
 
 /* dW [Hkv][d][F] and dalpha [Hq] of sum(dO * O); dalpha_h = dw_h * w_h (1 - w_h). */
@@ -627,7 +643,7 @@ int oracle_train_backward(int n_seq, int L, int B, int Hq, int Hkv, int d, int F
     c.dw_part = (double *)calloc((size_t)n_seq * Hq + 1, sizeof(double));
     if (!c.dW_part || !c.dw_part) { free(c.dW_part); free(c.dw_part); return -1; }
     int rc = fanout(train_bwd_unit, &c, (long)n_seq * Hkv, n_threads,
-                    2 * (size_t)n_blk * st + 3 * P2 + 3 * (size_t)d + 2 * (size_t)F + st);
+                    2 * (size_t)n_blk * st + 2 * P2 + 4 * (size_t)d + 2 * (size_t)F + st);
     if (rc == 0) {
         for (int g = 0; g < Hkv; ++g)
             for (size_t i = 0; i < (size_t)d * F; ++i) {
@@ -636,7 +652,7 @@ int oracle_train_backward(int n_seq, int L, int B, int Hq, int Hkv, int d, int F
                 dW[(size_t)g * d * F + i] = a;
             }
         for (int h = 0; h < Hq; ++h) {
-            const double w = 1.0 / (1.0 + exp(-alpha[h]));
+            const double w = gate(alpha[h]);
             double a = 0.0;
             for (int s = 0; s < n_seq; ++s) a += c.dw_part[(size_t)s * Hq + h];
             dalpha[h] = a * w * (1.0 - w);

@@ -26,7 +26,7 @@ MUTANTS = [
     ("phi W transposed", "acc += x[e] * W[(size_t)e * F + f];", "acc += x[e] * W[((size_t)f * d + e) % ((size_t)d * F)];"),
     ("phi halves swapped", "out[f] = exp(u[f]) / sum_pos;\n        out[F + f] = exp(-u[f]) / sum_neg;",
      "out[F + f] = exp(u[f]) / sum_pos;\n        out[f] = exp(-u[f]) / sum_neg;"),
-    ("gate sign", "const double w = 1.0 / (1.0 + exp(-c->alpha[h]));", "const double w = 1.0 / (1.0 + exp(c->alpha[h]));"),
+    ("gate sign", "return 1.0 / (1.0 + exp(-alpha));", "return 1.0 / (1.0 + exp(alpha));"),
     ("gate dropped in numerator", "o[e] = (w * sm_num[e] + lin_num[e]) / den;", "o[e] = (sm_num[e] + lin_num[e]) / den;"),
     ("gate on the wrong branch", "const double den = w * sm_den + lin_den;", "const double den = sm_den + w * lin_den;"),
     ("separate normalisers", "o[e] = (w * sm_num[e] + lin_num[e]) / den;",
@@ -36,15 +36,19 @@ MUTANTS = [
     ("state read transposed", "lin_num[e] += phi_q[f] * S[(size_t)f * d + e];",
      "lin_num[e] += phi_q[f] * S[((size_t)e * P2 + f) % ((size_t)P2 * d)];"),
     ("commit drops last token", "for (int t = 0; t < c->T; ++t) {", "for (int t = 0; t < c->T - 1; ++t) {"),
-    ("causal mask inside the block", "for (int j = 0; j < B; ++j) {", "for (int j = 0; j <= i; ++j) {"),
-    ("GQA mapping modulo", "const int G = c->Hq / c->Hkv, g = h / G;", "const int G = c->Hq / c->Hkv, g = h % c->Hkv;"),
+    ("causal mask inside the block", "(size_t)c->Hkv * d, B, d, sm_num, &sm_den);",
+     "(size_t)c->Hkv * d, i + 1, d, sm_num, &sm_den);"),
+    ("GQA mapping modulo", "return h / G;", "return h % Hkv;"),
     ("prefix route skips last token", "for (int t = 0; t < P; ++t) {", "for (int t = 0; t + 1 < P; ++t) {"),
     ("value index shifted", "for (int e = 0; e < d; ++e) sm_num[e] += a * v[e];",
      "for (int e = 0; e < d; ++e) sm_num[e] += a * v[(e + 1) % d];"),
     # training form (Stage 1): forward over a sequence and the gradient of W, alpha
-    ("train forward gate dropped", "num[e] += w * a * v[e];", "num[e] += a * v[e];"),
-    ("train forward sees own block", "        for (int t = 0; t < B; ++t) {\n            const size_t tt = (size_t)s * c->L + (size_t)n * B + t;",
-     "        for (int t = 0; t < B && n < 0; ++t) {\n            const size_t tt = (size_t)s * c->L + (size_t)n * B + t;"),
+    ("train forward never commits", "        /* block n commits after its own readout */\n        for (int t = 0; t < B; ++t) {",
+     "        /* block n commits after its own readout */\n        for (int t = 0; t < B && n < 0; ++t) {"),
+    ("train forward commits one block late", "for (int n = 0; n < n_blk; ++n) {\n        const size_t t0 = (size_t)s * c->L + (size_t)n * B;   /* first token of block n */",
+     "for (int n = 0; n < n_blk; ++n) {\n        const size_t t0 = (size_t)s * c->L + (size_t)(n > 0 ? n - 1 : 0) * B;   /* first token of block n */"),
+    ("train prefix states not carried over", "for (size_t i = 0; i < st; ++i) Sn[i] = Sn[i - st];",
+     "for (size_t i = 0; i < st; ++i) Sn[i] = 0.0 * Sn[i - st];"),
     ("train dD sign", "const double dD = -go / D;", "const double dD = go / D;"),
     ("train z gradient dropped", "double acc_f = z[f] * dD;", "double acc_f = 0.0 * dD;"),
     ("train phi backward negative half sign", "- phi[F + f] * (gphi[F + f] - dot_neg);",
