@@ -187,6 +187,53 @@ hybrid_status hybrid_state_pack(const hybrid_cfg *cfg, const float *S_logical,
                                 const float *z_logical, void *const *d_state_ptrs, int n_req,
                                 cudaStream_t stream);
 
+/* ------------------------------------------------------------------------
+ * Training form (Section 3.2, Stage 1 attention transfer).
+ *
+ * A batch of n_seq training sequences of seq_len = n_blk * B tokens, cut into
+ * blocks B_0 .. B_{n_blk-1} of B = cfg->block_size tokens.  Teacher forcing
+ * supplies every block's queries, keys and values; block n attends to itself
+ * with the exact softmax branch and to blocks 0 .. n-1 through
+ * S_{n-1} = sum_{m<n} sum_{t in B_m} phi(k_t) v_t^T and z_{n-1} likewise
+ * (Section 3.1 applied to every block of the sequence; S_{-1} = 0).  Stage 1
+ * trains only psi = {W, alpha} to match a frozen softmax teacher's output
+ * under a squared-error loss; the caller forms dO = dL/dO from its loss.
+ *
+ *   Q, O, dO  [n_seq][seq_len][Hq][d]    bf16
+ *   K, V      [n_seq][seq_len][Hkv][d]   bf16
+ *   W         [Hkv][d][F] bf16;  alpha [Hq] float32
+ *   dW        [Hkv][d][F] float32;  dalpha [Hq] float32  (overwritten)
+ *   workspace device, 1024-byte aligned, >= hybrid_train_workspace_bytes bytes;
+ *             hybrid_train_forward fills it with the states of every block, and
+ *             hybrid_train_backward reads them (and then reuses the space), so
+ *             one forward precedes each backward on the same workspace.
+ * Supported: bf16 I/O, d in {64, 128}, F in {64, 128}, B in {16, 32, 64},
+ * (Hq / Hkv) * B <= 128, seq_len a multiple of B; otherwise
+ * HYBRID_ERR_UNSUPPORTED (seq_len not a multiple of B: HYBRID_ERR_INVALID_ARG).
+ * Both calls are asynchronous on the stream; device-side wait failures are
+ * reported by hybrid_check. */
+
+/* Bytes of workspace for n_seq sequences of seq_len tokens; 0 when the shape is
+ * not supported. */
+size_t hybrid_train_workspace_bytes(const hybrid_cfg *cfg, int n_seq, int seq_len);
+
+/* O = block-hybrid attention of every block against the states of the blocks
+ * before it; leaves those states in the workspace. */
+hybrid_status hybrid_train_forward(const hybrid_cfg *cfg, const void *Q, const void *K, const void *V,
+                                   const void *W, const float *alpha, int n_seq, int seq_len, void *O,
+                                   void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* Gradient of sum(dO * O) with respect to W and alpha, O being the output of
+ * the preceding hybrid_train_forward on this workspace:
+ *   dN = dO / D, dD = -(dO . O) / D (D = the merge's denominator),
+ *   dw_h = sum (dN . sm_num + dD sm_den), dalpha_h = dw_h w_h (1 - w_h),
+ *   dphi(q) = S_{n-1} dN + z_{n-1} dD,  dphi(k_t in B_m) = sum_{n>m} dS_{n-1} v_t + dz_{n-1},
+ *   dW = sum over query and key rows of x du^T through phi's two softmaxes. */
+hybrid_status hybrid_train_backward(const hybrid_cfg *cfg, const void *Q, const void *K, const void *V,
+                                    const void *W, const float *alpha, const void *O, const void *dO,
+                                    int n_seq, int seq_len, void *workspace, size_t workspace_bytes,
+                                    float *dW, float *dalpha, cudaStream_t stream);
+
 /* Synchronise the stream, then read and clear this device's error word.
  * Returns HYBRID_OK, HYBRID_ERR_DEVICE (a state pointer failed its device
  * check), HYBRID_ERR_TIMEOUT (a bounded wait gave up) or HYBRID_ERR_CUDA. */

@@ -6,6 +6,7 @@
 #include "hybrid_common.cuh"
 #include "hybrid_kernels.h"
 #include "hybrid_tc.h"
+#include "hybrid_train.h"
 
 namespace {
 
@@ -242,6 +243,64 @@ hybrid_status hybrid_state_pack(const hybrid_cfg *cfg, const float *S_logical,
     unsigned *err = error_word();
     if (!err) return HYBRID_ERR_CUDA;
     return from_cuda(hyb::launch_state_pack(*cfg, S_logical, z_logical, d_state_ptrs, n_req, err, stream));
+}
+
+size_t hybrid_train_workspace_bytes(const hybrid_cfg *cfg, int n_seq, int seq_len)
+{
+    if (check_cfg(cfg) != HYBRID_OK || n_seq < 1 || !hyb::train_supported(*cfg, seq_len)) return 0;
+    return hyb::train_workspace_bytes(*cfg, n_seq, seq_len);
+}
+
+namespace {
+hybrid_status check_train(const hybrid_cfg *cfg, int n_seq, int seq_len, const void *workspace,
+                          size_t workspace_bytes)
+{
+    hybrid_status s = check_cfg(cfg);
+    if (s != HYBRID_OK) return s;
+    if (n_seq < 1 || seq_len < 1) return HYBRID_ERR_INVALID_ARG;
+    if (seq_len % cfg->block_size != 0) return HYBRID_ERR_INVALID_ARG;
+    if (!hyb::train_supported(*cfg, seq_len)) return HYBRID_ERR_UNSUPPORTED;
+    if (!workspace || !aligned(workspace, 1024)) return HYBRID_ERR_INVALID_ARG;
+    if (workspace_bytes < hyb::train_workspace_bytes(*cfg, n_seq, seq_len)) return HYBRID_ERR_INVALID_ARG;
+    return HYBRID_OK;
+}
+}  // namespace
+
+hybrid_status hybrid_train_forward(const hybrid_cfg *cfg, const void *Q, const void *K, const void *V,
+                                   const void *W, const float *alpha, int n_seq, int seq_len, void *O,
+                                   void *workspace, size_t workspace_bytes, cudaStream_t stream)
+{
+    hybrid_status s = check_train(cfg, n_seq, seq_len, workspace, workspace_bytes);
+    if (s != HYBRID_OK) return s;
+    if (!Q || !K || !V || !W || !alpha || !O) return HYBRID_ERR_INVALID_ARG;
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(W, 16) || !aligned(O, 16) ||
+        !aligned(alpha, 4))
+        return HYBRID_ERR_INVALID_ARG;
+    unsigned *err = error_word();
+    if (!err) return HYBRID_ERR_CUDA;
+    const cudaError_t e = hyb::launch_train_states(*cfg, K, V, W, n_seq, seq_len, workspace, err, stream);
+    if (e != cudaSuccess) return HYBRID_ERR_CUDA;
+    // every block of every sequence is one decode step against the state of its prefix
+    const int n_blk = seq_len / cfg->block_size;
+    return hybrid_block_attn(cfg, Q, K, V, W, alpha, hyb::train_state_ptrs(*cfg, n_seq, seq_len, workspace),
+                             n_seq * n_blk, O, stream);
+}
+
+hybrid_status hybrid_train_backward(const hybrid_cfg *cfg, const void *Q, const void *K, const void *V,
+                                    const void *W, const float *alpha, const void *O, const void *dO,
+                                    int n_seq, int seq_len, void *workspace, size_t workspace_bytes,
+                                    float *dW, float *dalpha, cudaStream_t stream)
+{
+    hybrid_status s = check_train(cfg, n_seq, seq_len, workspace, workspace_bytes);
+    if (s != HYBRID_OK) return s;
+    if (!Q || !K || !V || !W || !alpha || !O || !dO || !dW || !dalpha) return HYBRID_ERR_INVALID_ARG;
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(W, 16) || !aligned(O, 16) ||
+        !aligned(dO, 16) || !aligned(alpha, 4) || !aligned(dW, 16) || !aligned(dalpha, 4))
+        return HYBRID_ERR_INVALID_ARG;
+    unsigned *err = error_word();
+    if (!err) return HYBRID_ERR_CUDA;
+    return from_cuda(hyb::launch_train_backward(*cfg, Q, K, V, W, alpha, O, dO, n_seq, seq_len, workspace, dW,
+                                                dalpha, err, stream));
 }
 
 hybrid_status hybrid_check(cudaStream_t stream)

@@ -1,0 +1,1033 @@
+// hybrid_train.cu -- the training form of block-hybrid attention (Section 3.2,
+// Stage 1 attention transfer): the states seen by every block of a training
+// sequence, and the gradient of sum(dO * O) with respect to W and alpha.
+//
+// A training sequence of L = n_blk * B tokens is cut into blocks of B tokens;
+// block n reads S_{n-1} = sum_{m < n} dS_m, z_{n-1} likewise (Section 3.1 applied
+// to every block, S_{-1} = 0), with dS_m = sum_{t in B_m} phi(k_t) [v_t | 1]^T.
+// Per query row i of block n (N, D = numerator and denominator of the merge,
+// g = dO row, o = O row):
+//     dN = g / D,  dD = -(g . o) / D,  dw_h += dN . sm_num + dD sm_den,
+//     dphi(q) = S_{n-1} dN + z_{n-1} dD,   dR_n += phi(q) [dN | dD]^T,
+// and a key t of block m receives dphi(k_t) = R_m v_t + r_m with
+// [R_m | r_m] = sum_{n > m} dR_n.  Through phi = [softmax(u), softmax(-u)],
+// u = x W:  du = p+ (g+ - <g+, p+>) - p- (g- - <g-, p->),  dW += x du^T.
+//
+// Kernels (one CTA of 128 threads per (sequence, block, state head); thread r
+// owns row r of the tile and Tensor Memory lane r):
+//   k_block_state   U = K W, phi(K), dS_m = phi^T [V | 1] on the tensor cores;
+//                   written into slot m+1 of the decode image P (S^T tiles, read
+//                   by the decode readout kernel) and of the feature-row image
+//                   PT (S tiles: row f holds 32 consecutive e, 128-byte swizzle),
+//                   whose d/32 tiles are K-major tf32 operands for S dN
+//   k_slot_scan     running sums over the slots of a sequence (P and PT
+//                   inclusive; R reverse exclusive)
+//   k_phi_grad<Q>   query side: [U | scores] = Q [W | K^T], dO V^T, the merge
+//                   terms, dN into Tensor Memory, then S dN + z dD streamed over
+//                   the PT tiles, du_q, and dR_n = phi(Q)^T [dN | dD];
+//                   key side: U = K W, V into Tensor Memory, R v + r over the
+//                   R tiles, du_k
+//   k_dw            dW_g = sum over query and key rows of x du^T, split over
+//                   row ranges and added into dW with float atomics
+#include <atomic>
+
+#include "hybrid_common.cuh"
+#include "hybrid_train.h"
+#include "tc_pipeline.cuh"
+
+namespace hyb {
+
+namespace {
+
+using namespace pipe;
+
+constexpr int kThreads = 128;
+constexpr int kSmemLimit = 232448;
+constexpr uint32_t kColS = 0, kColGv = 64, kColU = 256, kColY = 384, kColG = 0, kColDR = 0;
+
+struct TrainArgs {
+    const bf16 *Q, *K, *V, *W, *O, *dO;
+    const float *alpha;
+    float *P, *PT, *R;
+    bf16 *dUq, *dUk;
+    float *dalpha;
+    unsigned *err;
+    int n_seq, L, B, Hq, Hkv, d, F, n_blk;
+};
+
+__host__ __device__ __forceinline__ size_t slot_floats(int Hkv, int d, int F)
+{
+    return (size_t)Hkv * head_floats(d, F);
+}
+
+// Feature-row head block (PT and R): logical S[f][e] at float offset
+//     (e/32)*64F + f*32 + 4*(((e%32)/4) ^ (f%8)) + e%4,
+// i.e. d/32 tiles of 2F rows x 32 consecutive e, each 128-byte row with its
+// 16-byte granules permuted by XOR with (f mod 8); then z[f] at 2F*d + f, as in
+// the decode image.  A tile is a K-major tf32 operand [N = 2F rows, K = 32 e].
+
+// byte offset of 16-byte granule j of row r inside a 128-byte-swizzled panel
+__device__ __forceinline__ uint32_t swz(int r, int j)
+{
+    return (uint32_t)r * 128u + (uint32_t)((j ^ (r & 7)) << 4);
+}
+
+// Rows [0, nalloc) of a bf16 operand image (panels of 64 columns, panel stride
+// nalloc*128 bytes): row r < nrows from rowptr(r), columns [0, ncols); the rest 0.
+template <class RowPtr>
+__device__ __forceinline__ void load_rows_bf16(uint8_t *dst, RowPtr rowptr, int nrows, int nalloc, int ncols,
+                                               int tid)
+{
+    const int gpr = ncols >> 3;
+    for (int i = tid; i < nalloc * gpr; i += kThreads) {
+        const int r = i / gpr, c8 = i - r * gpr;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (r < nrows) v = __ldg(reinterpret_cast<const uint4 *>(rowptr(r)) + c8);
+        *reinterpret_cast<uint4 *>(dst + (uint32_t)(c8 >> 3) * (uint32_t)nalloc * 128u + swz(r, c8 & 7)) = v;
+    }
+}
+
+// Write 32 consecutive columns [c0, c0 + 32) of row r (values x, converted to
+// bf16) into a bf16 operand image with panel stride pstride.
+__device__ __forceinline__ void store_row32_bf16(uint8_t *img, uint32_t pstride, int r, int c0, const float (&x)[32])
+{
+    uint8_t *base = img + (uint32_t)(c0 >> 6) * pstride;
+    const int j0 = (c0 & 63) >> 3;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        uint4 v;
+        v.x = pack_bf16x2(x[8 * q + 0], x[8 * q + 1]);
+        v.y = pack_bf16x2(x[8 * q + 2], x[8 * q + 3]);
+        v.z = pack_bf16x2(x[8 * q + 4], x[8 * q + 5]);
+        v.w = pack_bf16x2(x[8 * q + 6], x[8 * q + 7]);
+        *reinterpret_cast<uint4 *>(base + swz(r, j0 + q)) = v;
+    }
+}
+
+__device__ __forceinline__ void load_row_f32(const bf16 *src, int n, float *out)
+{
+    const uint4 *p = reinterpret_cast<const uint4 *>(src);
+    for (int i = 0; i < n / 8; ++i) {
+        const uint4 v = __ldg(p + i);
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            out[8 * i + 2 * j] = __uint_as_float(w[j] << 16);
+            out[8 * i + 2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
+        }
+    }
+}
+
+// Row statistics of phi = [softmax(u), softmax(-u)] for the F values of u in
+// Tensor Memory columns [col, col + F) of this thread's lane.
+struct PhiStats {
+    float mp, sp, mn, sn;   // max u, sum e^(u - mp), min u, sum e^(mn - u)
+};
+__device__ __forceinline__ PhiStats phi_stats(uint32_t taddr, int F)
+{
+    PhiStats s{-INFINITY, 0.f, INFINITY, 0.f};
+    float x[32];
+    for (int j = 0; j < F / 32; ++j) {
+        ptx::tmem_ld32(taddr + 32 * j, x);
+        ptx::tmem_wait_ld();
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+            s.mp = fmaxf(s.mp, x[k]);
+            s.mn = fminf(s.mn, x[k]);
+        }
+    }
+    for (int j = 0; j < F / 32; ++j) {
+        ptx::tmem_ld32(taddr + 32 * j, x);
+        ptx::tmem_wait_ld();
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+            s.sp += ex2((x[k] - s.mp) * kLog2e);
+            s.sn += ex2((s.mn - x[k]) * kLog2e);
+        }
+    }
+    return s;
+}
+
+// Shared memory of the row kernels (bytes, all 1024-aligned)
+struct RowLayout {
+    uint32_t off_q, off_w, off_k, off_v, off_do, off_phi, off_y, off_z, off_bar, bytes;
+    uint32_t off_ring, ring_slot;
+};
+
+// k_phi_grad: phase-one operands (Q, W, K, V) share their space with the ring of
+// S / R tiles used afterwards; dO shares its space with phi(Q).
+RowLayout make_grad_layout(int d, int F, int B)
+{
+    RowLayout Lr{};
+    const uint32_t rows128 = (uint32_t)(d / 64) * 128 * 128;        // 128 rows x d bf16
+    const uint32_t wbytes = (uint32_t)(F / 64) * d * 128;           // d rows x F bf16
+    const uint32_t kvbytes = (uint32_t)(d / 64) * B * 128;          // B rows x d bf16
+    uint32_t off = 0;
+    Lr.off_q = off;
+    Lr.off_w = Lr.off_q + rows128;
+    Lr.off_k = Lr.off_w + wbytes;
+    Lr.off_v = Lr.off_k + kvbytes;
+    uint32_t phase1 = Lr.off_v + kvbytes;
+    Lr.ring_slot = (uint32_t)2 * F * 128;                            // 2F rows x 32 floats
+    Lr.off_ring = 0;
+    const uint32_t ring = 2 * Lr.ring_slot;
+    off = phase1 > ring ? phase1 : ring;
+    Lr.off_phi = off;                                               // 128 rows x 2F bf16; dO first
+    off += (uint32_t)(2 * F / 64) * 128 * 128;
+    Lr.off_do = Lr.off_phi;
+    Lr.off_y = off;                                                 // 128 rows x (d + 16) bf16
+    off += (uint32_t)((d + 16 + 63) / 64) * 128 * 128;
+    Lr.off_z = off;
+    off += (((uint32_t)2 * F * 4) + 1023) & ~1023u;
+    Lr.off_bar = off;
+    off += 1024;
+    Lr.bytes = off + 1024;
+    return Lr;
+}
+
+// k_block_state: K (128 rows), W, phi(K) (B rows x 2F), [V | 1 | 0] (B rows x (d + 16))
+RowLayout make_state_layout(int d, int F, int B)
+{
+    RowLayout Lr{};
+    uint32_t off = 0;
+    Lr.off_q = off;                                                  // K as the M = 128 operand
+    off += (uint32_t)(d / 64) * 128 * 128;
+    Lr.off_w = off;
+    off += (uint32_t)(F / 64) * d * 128;
+    Lr.off_phi = off;
+    off += (uint32_t)(2 * F / 64) * B * 128;
+    Lr.off_y = off;
+    off += (uint32_t)((d + 16 + 63) / 64) * B * 128;
+    off = (off + 1023) & ~1023u;
+    Lr.off_bar = off;
+    off += 1024;
+    Lr.bytes = off + 1024;
+    return Lr;
+}
+
+__device__ __forceinline__ uint8_t *aligned_smem(uint8_t *raw)
+{
+    return reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
+}
+
+// ---------------------------------------------------------------------------
+// k_block_state: dS_m of one (sequence s, block m, state head g) into slot m+1
+// of P and PT.  The CTA of the last block (whose increment no block reads)
+// clears slot 0 instead.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads, 1) k_block_state(const __grid_constant__ TrainArgs a, RowLayout Lr)
+{
+    using namespace ptx;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = aligned_smem(smem_raw);
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int d = a.d, F = a.F, B = a.B, Hkv = a.Hkv;
+    const int g = blockIdx.x % Hkv, m = (blockIdx.x / Hkv) % a.n_blk, s = blockIdx.x / (Hkv * a.n_blk);
+    const size_t hf = head_floats(d, F);
+    griddep_wait();
+    if (m == a.n_blk - 1) {
+        float4 *p = reinterpret_cast<float4 *>(a.P + ((size_t)s * a.n_blk * Hkv + g) * hf);
+        float4 *pt = reinterpret_cast<float4 *>(a.PT + ((size_t)s * a.n_blk * Hkv + g) * hf);
+        for (size_t i = tid; i < hf / 4; i += kThreads) {
+            p[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+            pt[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        return;
+    }
+    uint64_t *bar = reinterpret_cast<uint64_t *>(smem + Lr.off_bar);
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar + 2);
+    volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
+    if (tid == 0) {
+        mbar_init(&bar[0], 1);
+        *fail = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(tmem_holder, 512);
+        tmem_relinquish();
+    }
+    const size_t t0 = (size_t)s * a.L + (size_t)m * B;
+    const size_t kv_row = (size_t)Hkv * d;
+    // K rows (zero beyond B) as the M = 128 A operand, W, and [V | 1 | 0]
+    load_rows_bf16(smem + Lr.off_q, [&](int r) { return a.K + (t0 + r) * kv_row + (size_t)g * d; }, B, 128, d, tid);
+    load_rows_bf16(smem + Lr.off_w, [&](int r) { return a.W + ((size_t)g * d + r) * F; }, d, d, F, tid);
+    load_rows_bf16(smem + Lr.off_y, [&](int r) { return a.V + (t0 + r) * kv_row + (size_t)g * d; }, B, B, d, tid);
+    {
+        const uint32_t pstride = (uint32_t)B * 128;
+        for (int r = tid; r < B; r += kThreads) {
+            uint8_t *base = smem + Lr.off_y + (uint32_t)(d >> 6) * pstride;
+            *reinterpret_cast<uint4 *>(base + swz(r, 0)) = make_uint4(0x3F80u, 0, 0, 0);   // bf16 1.0 in column d
+            *reinterpret_cast<uint4 *>(base + swz(r, 1)) = make_uint4(0, 0, 0, 0);
+        }
+    }
+    fence_proxy_async_smem();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_holder;
+    const uint32_t lane_off = (uint32_t)(warp & 3) * 32u << 16;
+    bool ok = true;
+    if (tid == 0) {
+        const uint32_t q_u = smem_u32(smem + Lr.off_q), w_u = smem_u32(smem + Lr.off_w);
+        const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
+        for (int k = 0; k < d / 16; ++k)
+            mma_bf16_ss(tmem + kColU, smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B),
+                        smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B), idU, k > 0);
+        mma_commit(&bar[0]);
+    }
+    ok = wait_bar(&bar[0], 0, fail);
+    tc_fence_after();
+    // phi(K) of row tid into the MN-major operand [token][feature]
+    {
+        const PhiStats st = phi_stats(tmem + lane_off + kColU, F);
+        const float ip = 1.f / st.sp, in = 1.f / st.sn;
+        float x[32], yp[32], yn[32];
+        for (int j = 0; j < F / 32; ++j) {
+            tmem_ld32(tmem + lane_off + kColU + 32 * j, x);
+            tmem_wait_ld();
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+                yp[k] = ex2((x[k] - st.mp) * kLog2e) * ip;
+                yn[k] = ex2((st.mn - x[k]) * kLog2e) * in;
+            }
+            if (tid < B) {
+                store_row32_bf16(smem + Lr.off_phi, (uint32_t)B * 128, tid, 32 * j, yp);
+                store_row32_bf16(smem + Lr.off_phi, (uint32_t)B * 128, tid, F + 32 * j, yn);
+            }
+        }
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    if (group_sync_failed(1, kThreads, !ok)) {
+        if (tid == 0) raise_error(a.err, ERR_WAIT_TIMEOUT);
+        __syncthreads();
+        if (warp == 0) tmem_dealloc(tmem, 512);
+        return;
+    }
+    tc_fence_after();
+    // accumulator block i (features 128 i ..) at column i * NYS, NYS = NY rounded up to 32
+    const int NY = d + 16, NYS = (NY + 31) & ~31, NM = 2 * F / 128;
+    if (tid == 0) {
+        const uint32_t p_u = smem_u32(smem + Lr.off_phi), y_u = smem_u32(smem + Lr.off_y);
+        const uint32_t idDS = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, NY);
+        for (int i = 0; i < NM; ++i)
+            for (int ks = 0; ks < B / 16; ++ks)
+                mma_bf16_ss(tmem + kColDR + (uint32_t)(i * NYS),
+                            smem_desc(p_u + (uint32_t)(2 * i) * B * 128 + ks * 2048, B * 128, 1024, SWZ_128B),
+                            smem_desc(y_u + ks * 2048, B * 128, 1024, SWZ_128B), idDS, ks > 0);
+        mma_commit(&bar[0]);
+    }
+    ok = wait_bar(&bar[0], 1, fail);
+    tc_fence_after();
+    if (ok) {
+        // lane tid of M-block i is feature f = 128 i + tid: row f of dS (d values) and dz[f]
+        const size_t slot = ((size_t)s * a.n_blk + m + 1) * Hkv + g;
+        float *P = a.P + slot * hf, *PT = a.PT + slot * hf;
+        for (int i = 0; i < NM; ++i) {
+            const int f = 128 * i + tid;
+            float x[32];
+            for (int c = 0; c < d / 32; ++c) {
+                tmem_ld32(tmem + lane_off + kColDR + (uint32_t)(i * NYS + 32 * c), x);
+                tmem_wait_ld();
+                float4 *row = reinterpret_cast<float4 *>(PT + (size_t)c * 64 * F + (size_t)f * 32);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) row[q ^ (f & 7)] = make_float4(x[4 * q], x[4 * q + 1], x[4 * q + 2], x[4 * q + 3]);
+#pragma unroll
+                for (int k = 0; k < 32; ++k) P[s_offset(f, 32 * c + k, d)] = x[k];
+            }
+            float zz[16];
+            tmem_ld16(tmem + lane_off + kColDR + (uint32_t)(i * NYS + d), zz);
+            tmem_wait_ld();
+            P[z_offset(f, d, F)] = zz[0];
+            PT[z_offset(f, d, F)] = zz[0];
+        }
+    } else if (tid == 0) {
+        raise_error(a.err, ERR_WAIT_TIMEOUT);
+    }
+    tc_fence_before();
+    __syncthreads();
+    griddep_launch_dependents();
+    if (warp == 0) tmem_dealloc(tmem, 512);
+}
+
+// ---------------------------------------------------------------------------
+// k_slot_scan: per sequence, running sums over n_slots slots of nf floats.
+// reverse = false: slot n += slot n-1 (inclusive, slot 0 unchanged);
+// reverse = true : slot m = sum of slots n > m (exclusive, from the end).
+// ---------------------------------------------------------------------------
+__global__ void k_slot_scan(float *buf0, float *buf1, int n_seq, int n_slots, size_t nf, bool reverse)
+{
+    float *buf = blockIdx.y == 0 ? buf0 : buf1;
+    ptx::griddep_wait();
+    if (!buf) return;
+    const size_t n4 = nf / 4;
+    const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n4 * (size_t)n_seq) return;
+    const size_t s = i / n4, j = i % n4;
+    float4 *p = reinterpret_cast<float4 *>(buf) + s * n4 * n_slots + j;
+    if (!reverse) {
+        float4 acc = p[0];
+        float4 nxt = n_slots > 1 ? p[n4] : acc;
+        for (int n = 1; n < n_slots; ++n) {
+            const float4 v = nxt;
+            if (n + 1 < n_slots) nxt = p[(size_t)(n + 1) * n4];
+            acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+            p[(size_t)n * n4] = acc;
+        }
+    } else {
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        float4 nxt = p[(size_t)(n_slots - 1) * n4];
+        for (int n = n_slots - 1; n >= 0; --n) {
+            const float4 v = nxt;
+            if (n > 0) nxt = p[(size_t)(n - 1) * n4];
+            p[(size_t)n * n4] = acc;
+            acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+        }
+    }
+    ptx::griddep_launch_dependents();
+}
+
+// ---------------------------------------------------------------------------
+// k_phi_grad<kQuery>: one (sequence s, block n, state head g).
+// ---------------------------------------------------------------------------
+template <bool kQuery>
+__global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant__ TrainArgs a, RowLayout Lr)
+{
+    using namespace ptx;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = aligned_smem(smem_raw);
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int d = a.d, F = a.F, B = a.B, Hkv = a.Hkv, Hq = a.Hq, G = Hq / Hkv;
+    const int g = blockIdx.x % Hkv, n = (blockIdx.x / Hkv) % a.n_blk, s = blockIdx.x / (Hkv * a.n_blk);
+    const int rows = kQuery ? G * B : B;
+    const size_t hf = head_floats(d, F);
+    const size_t t0 = (size_t)s * a.L + (size_t)n * B;
+    const size_t kv_row = (size_t)Hkv * d, q_row = (size_t)Hq * d;
+    // tile source: PT slot n (query side: S_{n-1}) or R slot n (key side: R_n)
+    const float *src = (kQuery ? a.PT : a.R) + (((size_t)s * a.n_blk + n) * Hkv + g) * hf;
+
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + Lr.off_bar);
+    uint64_t *mbar = bars;          // MMA groups complete
+    uint64_t *full = bars + 1;      // [2] ring slot loaded
+    uint64_t *empty = bars + 3;     // [2] ring slot consumed
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 5);
+    volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
+    float *sDw = reinterpret_cast<float *>(tmem_holder + 2);    // [8] dw per head of the group
+    float *sZ = reinterpret_cast<float *>(smem + Lr.off_z);     // z_{n-1} or r_n
+    if (tid == 0) {
+        for (int i = 0; i < 5; ++i) mbar_init(&bars[i], 1);
+        *fail = 0;
+        fence_mbar_init();
+    }
+    if (tid < 8) sDw[tid] = 0.f;
+    if (warp == 0) {
+        tmem_alloc(tmem_holder, 512);
+        tmem_relinquish();
+    }
+    griddep_wait();
+
+    // phase one: operands of [U | scores] = Q [W | K^T] and dO V^T (query side) or U = K W
+    if (kQuery) {
+        auto qrow = [&](int r) { return a.Q + (t0 + r % B) * q_row + (size_t)(g * G + r / B) * d; };
+        auto orow = [&](int r) { return a.dO + (t0 + r % B) * q_row + (size_t)(g * G + r / B) * d; };
+        load_rows_bf16(smem + Lr.off_q, qrow, rows, 128, d, tid);
+        load_rows_bf16(smem + Lr.off_do, orow, rows, 128, d, tid);
+        load_rows_bf16(smem + Lr.off_k, [&](int r) { return a.K + (t0 + r) * kv_row + (size_t)g * d; }, B, B, d, tid);
+        load_rows_bf16(smem + Lr.off_v, [&](int r) { return a.V + (t0 + r) * kv_row + (size_t)g * d; }, B, B, d, tid);
+    } else {
+        load_rows_bf16(smem + Lr.off_q, [&](int r) { return a.K + (t0 + r) * kv_row + (size_t)g * d; }, B, 128, d, tid);
+    }
+    load_rows_bf16(smem + Lr.off_w, [&](int r) { return a.W + ((size_t)g * d + r) * F; }, d, d, F, tid);
+    for (int f = tid; f < 2 * F; f += kThreads) sZ[f] = src[z_offset(f, d, F)];
+    fence_proxy_async_smem();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_holder;
+    const uint32_t lane_off = (uint32_t)(warp & 3) * 32u << 16;
+    const uint32_t tl = tmem + lane_off;
+    const int NCHUNK = d / 32;
+    const uint32_t ring_u = smem_u32(smem + Lr.off_ring);
+    int loads_issued = 0;
+    if (tid == 0) {
+        const uint32_t q_u = smem_u32(smem + Lr.off_q), w_u = smem_u32(smem + Lr.off_w);
+        const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
+        for (int k = 0; k < d / 16; ++k) {
+            const uint64_t aq = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
+            mma_bf16_ss(tmem + kColU, aq, smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B), idU, k > 0);
+            if (kQuery) {
+                const uint32_t k_u = smem_u32(smem + Lr.off_k), v_u = smem_u32(smem + Lr.off_v),
+                               o_u = smem_u32(smem + Lr.off_do);
+                const uint32_t idS = instr_desc(FMT_BF16, FMT_BF16, false, false, 128, B);
+                const uint32_t kb = (uint32_t)(k >> 2) * B * 128 + (k & 3) * 32;
+                mma_bf16_ss(tmem + kColS, aq, smem_desc(k_u + kb, 16, 1024, SWZ_128B), idS, k > 0);
+                const uint64_t ao = smem_desc(o_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
+                mma_bf16_ss(tmem + kColGv, ao, smem_desc(v_u + kb, 16, 1024, SWZ_128B), idS, k > 0);
+            }
+        }
+        mma_commit(mbar);
+    }
+    bool ok = wait_bar(mbar, 0, fail);
+    tc_fence_after();
+    // the phase-one operands are consumed: the first two tiles go into their space
+    if (tid == 0 && ok) {
+        for (int c = 0; c < 2 && c < NCHUNK; ++c) {
+            mbar_arrive_expect_tx(&full[c], Lr.ring_slot);
+            bulk_g2s(smem + Lr.off_ring + c * Lr.ring_slot, src + (size_t)c * 64 * F, Lr.ring_slot, &full[c]);
+            ++loads_issued;
+        }
+    }
+
+    // ---- row statistics (thread = row) ----
+    const bool valid = tid < rows;
+    const int hl = kQuery ? tid / B : 0;
+    const PhiStats st = phi_stats(tl + kColU, F);
+    const float ip = 1.f / st.sp, in = 1.f / st.sn;
+    float dD = 0.f;   // coefficient of z (query side) / of r (key side) in dphi
+    if (kQuery) {
+        const int h = g * G + hl;
+        const float alpha = valid ? a.alpha[h] : 0.f;
+        const float w = 1.f / (1.f + expf(-alpha));
+        // phi(q) into its operand image; lin_den = phi(q) . z
+        float lin_den = 0.f;
+        {
+            float x[32], yp[32], yn[32];
+            for (int j = 0; j < F / 32; ++j) {
+                tmem_ld32(tl + kColU + 32 * j, x);
+                tmem_wait_ld();
+#pragma unroll
+                for (int k = 0; k < 32; ++k) {
+                    yp[k] = valid ? ex2((x[k] - st.mp) * kLog2e) * ip : 0.f;
+                    yn[k] = valid ? ex2((st.mn - x[k]) * kLog2e) * in : 0.f;
+                    lin_den += yp[k] * sZ[32 * j + k] + yn[k] * sZ[F + 32 * j + k];
+                }
+                store_row32_bf16(smem + Lr.off_phi, 128 * 128, tid, 32 * j, yp);
+                store_row32_bf16(smem + Lr.off_phi, 128 * 128, tid, F + 32 * j, yn);
+            }
+        }
+        // scores, shift c, D' = w sum_j e^(s_j - c) + lin_den e^(-c)  (D = e^c D')
+        const float scale = rsqrtf((float)d);
+        float sc[64];
+        float m = -INFINITY;
+        for (int j = 0; j < B / 16; ++j) {
+            float x[16];
+            tmem_ld16(tl + kColS + 16 * j, x);
+            tmem_wait_ld();
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+                sc[16 * j + k] = x[k] * scale;
+                m = fmaxf(m, sc[16 * j + k]);
+            }
+        }
+        float c = m;
+        if (lin_den > 0.f) c = w > 0.f ? fmaxf(m, logf(lin_den) - logf(w)) : logf(lin_den);
+        float l = 0.f;
+        for (int j = 0; j < B; ++j) {
+            sc[j] = ex2((sc[j] - c) * kLog2e);
+            l += sc[j];
+        }
+        const float ec = ex2(-c * kLog2e);
+        const float Dp = w * l + lin_den * ec;
+        const float inv = valid ? ec / Dp : 0.f;   // 1 / D
+        const float pw = valid ? 1.f / Dp : 0.f;   // e^(s_j - c) / D' = e^(s_j) / D
+        // g . o and dN = g / D (Tensor Memory, fp32; operand image, bf16), dD = -(g . o) / D
+        const bf16 *grow = a.dO + (t0 + tid % B) * q_row + (size_t)(g * G + hl) * d;
+        const bf16 *orow = a.O + (t0 + tid % B) * q_row + (size_t)(g * G + hl) * d;
+        float go = 0.f;
+        if (valid) {
+            float gv[32], ov[32];
+            for (int c0 = 0; c0 < d; c0 += 32) {
+                load_row_f32(grow + c0, 32, gv);
+                load_row_f32(orow + c0, 32, ov);
+#pragma unroll
+                for (int k = 0; k < 32; ++k) go += gv[k] * ov[k];
+            }
+        }
+        dD = -go * inv;
+        {
+            float gv[32];
+            for (int c0 = 0; c0 < d; c0 += 32) {
+                if (valid) {
+                    load_row_f32(grow + c0, 32, gv);
+#pragma unroll
+                    for (int k = 0; k < 32; ++k) gv[k] *= inv;
+                } else {
+#pragma unroll
+                    for (int k = 0; k < 32; ++k) gv[k] = 0.f;
+                }
+                tmem_st32(tl + kColY + c0, gv);
+                store_row32_bf16(smem + Lr.off_y, 128 * 128, tid, c0, gv);
+            }
+            // columns d .. d+15 (the rest of that 32-column group is never read)
+            uint8_t *base = smem + Lr.off_y + (uint32_t)(d >> 6) * (128 * 128);
+            uint4 v0;
+            v0.x = pack_bf16x2(dD, 0.f);
+            v0.y = v0.z = v0.w = 0u;
+            *reinterpret_cast<uint4 *>(base + swz(tid, 0)) = v0;
+            *reinterpret_cast<uint4 *>(base + swz(tid, 1)) = make_uint4(0, 0, 0, 0);
+        }
+        // dw of this row: sum_j (e^(s_j) / D) (g . v_j - g . o)
+        float dw = 0.f;
+        for (int j = 0; j < B / 16; ++j) {
+            float x[16];
+            tmem_ld16(tl + kColGv + 16 * j, x);
+            tmem_wait_ld();
+#pragma unroll
+            for (int k = 0; k < 16; ++k) dw += sc[16 * j + k] * pw * (x[k] - go);
+        }
+        if (valid) atomicAdd(&sDw[hl], dw);
+    } else {
+        // V rows (fp32) as the Tensor Memory A operand of R v; r enters with coefficient 1
+        const bf16 *vrow = a.V + (t0 + tid) * kv_row + (size_t)g * d;
+        float vv[32];
+        for (int c0 = 0; c0 < d; c0 += 32) {
+            if (valid) {
+                load_row_f32(vrow + c0, 32, vv);
+            } else {
+#pragma unroll
+                for (int k = 0; k < 32; ++k) vv[k] = 0.f;
+            }
+            tmem_st32(tl + kColY + c0, vv);
+        }
+        dD = valid ? 1.f : 0.f;
+    }
+    tmem_wait_st();
+    fence_proxy_async_smem();
+    tc_fence_before();
+    const bool failed1 = group_sync_failed(1, kThreads, !ok);
+    tc_fence_after();
+
+    // ---- dphi = [S | z] [dN; dD] (query) or [R | r] [v; 1] (key): tiles of 32 e ----
+    if (!failed1 && tid == 0) {
+        const uint32_t idC = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, 2 * F);
+        for (int c = 0; c < NCHUNK && ok; ++c) {
+            const int slot = c & 1;
+            ok = wait_bar(&full[slot], (uint32_t)(c >> 1) & 1u, fail);
+            if (!ok) break;
+            tc_fence_after();
+            const uint32_t s_u = ring_u + slot * Lr.ring_slot;
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+                mma_tf32_ts(tmem + kColG, tmem + kColY + 32 * c + 8 * kk, smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B),
+                            idC, (c | kk) != 0);
+            mma_commit(&empty[slot]);
+            if (c + 2 < NCHUNK) {
+                ok = wait_bar(&empty[slot], (uint32_t)(c >> 1) & 1u, fail);
+                if (!ok) break;
+                mbar_arrive_expect_tx(&full[slot], Lr.ring_slot);
+                bulk_g2s(smem + Lr.off_ring + slot * Lr.ring_slot, src + (size_t)(c + 2) * 64 * F, Lr.ring_slot,
+                         &full[slot]);
+                ++loads_issued;
+            }
+        }
+        mma_commit(mbar);
+        if (!ok) atomicOr(const_cast<int *>(fail), 1);
+    }
+    if (!failed1) ok = wait_bar(mbar, 1, fail) && ok;
+    tc_fence_after();
+
+    // ---- du = p+ (g+ - <g+, p+>) - p- (g- - <g-, p->) with g = dphi (+ z dD) ----
+    if (!failed1 && !*fail) {
+        float dotp = 0.f, dotn = 0.f;
+        float x[32], gp[32], gn[32];
+        for (int pass = 0; pass < 2; ++pass) {
+            for (int j = 0; j < F / 32; ++j) {
+                tmem_ld32(tl + kColU + 32 * j, x);
+                tmem_ld32(tl + kColG + 32 * j, gp);
+                tmem_ld32(tl + kColG + F + 32 * j, gn);
+                tmem_wait_ld();
+                float du[32];
+#pragma unroll
+                for (int k = 0; k < 32; ++k) {
+                    const float pp = ex2((x[k] - st.mp) * kLog2e) * ip;
+                    const float pn = ex2((st.mn - x[k]) * kLog2e) * in;
+                    const float g1 = gp[k] + sZ[32 * j + k] * dD;
+                    const float g2 = gn[k] + sZ[F + 32 * j + k] * dD;
+                    if (pass == 0) {
+                        dotp += g1 * pp;
+                        dotn += g2 * pn;
+                    } else {
+                        du[k] = pp * (g1 - dotp) - pn * (g2 - dotn);
+                    }
+                }
+                if (pass == 1 && valid) {
+                    bf16 *out = kQuery ? a.dUq + ((t0 + tid % B) * Hq + (size_t)(g * G + hl)) * F
+                                       : a.dUk + ((t0 + tid) * Hkv + (size_t)g) * F;
+                    uint4 *o4 = reinterpret_cast<uint4 *>(out + 32 * j);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        uint4 v;
+                        v.x = pack_bf16x2(du[8 * q + 0], du[8 * q + 1]);
+                        v.y = pack_bf16x2(du[8 * q + 2], du[8 * q + 3]);
+                        v.z = pack_bf16x2(du[8 * q + 4], du[8 * q + 5]);
+                        v.w = pack_bf16x2(du[8 * q + 6], du[8 * q + 7]);
+                        o4[q] = v;
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    const bool failed2 = group_sync_failed(1, kThreads, failed1 || !ok || *fail);
+    tc_fence_after();
+
+    // ---- query side: dR_n = phi(Q)^T [dN | dD], the gate, and the R slot ----
+    if (kQuery && !failed2) {
+        const int NY = d + 16, NYS = (NY + 31) & ~31, NM = 2 * F / 128;
+        if (tid == 0) {
+            const uint32_t p_u = smem_u32(smem + Lr.off_phi), y_u = smem_u32(smem + Lr.off_y);
+            const uint32_t idDR = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, NY);
+            for (int i = 0; i < NM; ++i)
+                for (int ks = 0; ks < rows / 16; ++ks)
+                    mma_bf16_ss(tmem + kColDR + (uint32_t)(i * NYS),
+                                smem_desc(p_u + (uint32_t)(2 * i) * 128 * 128 + ks * 2048, 128 * 128, 1024, SWZ_128B),
+                                smem_desc(y_u + ks * 2048, 128 * 128, 1024, SWZ_128B), idDR, ks > 0);
+            mma_commit(mbar);
+        }
+        if (tid < G) {
+            const float al = a.alpha[g * G + tid];
+            const float w = 1.f / (1.f + expf(-al));
+            atomicAdd(&a.dalpha[g * G + tid], sDw[tid] * w * (1.f - w));
+        }
+        ok = wait_bar(mbar, 0, fail);
+        tc_fence_after();
+        if (ok) {
+            float *R = a.R + (((size_t)s * a.n_blk + n) * Hkv + g) * hf;
+            for (int i = 0; i < NM; ++i) {
+                const int f = 128 * i + tid;
+                float x[32];
+                for (int c = 0; c < d / 32; ++c) {
+                    tmem_ld32(tl + kColDR + (uint32_t)(i * NYS + 32 * c), x);
+                    tmem_wait_ld();
+                    float4 *row = reinterpret_cast<float4 *>(R + (size_t)c * 64 * F + (size_t)f * 32);
+#pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        row[q ^ (f & 7)] = make_float4(x[4 * q], x[4 * q + 1], x[4 * q + 2], x[4 * q + 3]);
+                }
+                float zz[16];
+                tmem_ld16(tl + kColDR + (uint32_t)(i * NYS + d), zz);
+                tmem_wait_ld();
+                R[z_offset(f, d, F)] = zz[0];
+            }
+        }
+    }
+    if (tid == 0 && (failed2 || !ok)) raise_error(a.err, ERR_WAIT_TIMEOUT);
+    // no tile copy may still be landing when the CTA leaves
+    if (tid == 0) {
+        for (int c = 0; c < loads_issued; ++c) {
+            // loads c and c+2 share slot c&1; the later one completes the later phase
+            if (c + 2 >= loads_issued) mbar_wait(&full[c & 1], (uint32_t)(c >> 1) & 1u, kWaitNs);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    griddep_launch_dependents();
+    if (warp == 0) tmem_dealloc(tmem, 512);
+}
+
+// ---------------------------------------------------------------------------
+// k_dw: dW_g += sum over a range of rows of x du^T.  Row rho of group g: token
+// t = rho / (G+1); kinds 0..G-1 are the query heads of the group (Q, dU_q),
+// kind G is the key (K, dU_k).  128 rows per step, two smem stages; the
+// accumulator (d lanes x F columns) stays in Tensor Memory over the range.
+// ---------------------------------------------------------------------------
+struct DwArgs {
+    const bf16 *Q, *K, *dUq, *dUk;
+    float *dW;
+    unsigned *err;
+    long long n_tok;   // n_seq * L
+    int Hq, Hkv, d, F, tiles_per_cta, ctas_per_group;
+};
+
+__global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwArgs a)
+{
+    using namespace ptx;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = aligned_smem(smem_raw);
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int d = a.d, F = a.F, G = a.Hq / a.Hkv, K1 = G + 1;
+    const int g = blockIdx.x / a.ctas_per_group, part = blockIdx.x % a.ctas_per_group;
+    const long long total = a.n_tok * K1;
+    const long long r_begin = (long long)part * a.tiles_per_cta * 128;
+    long long r_end = r_begin + (long long)a.tiles_per_cta * 128;
+    if (r_end > total) r_end = total;
+    const int n_tiles = r_begin < total ? (int)((r_end - r_begin + 127) / 128) : 0;
+    const uint32_t xbytes = 2 * 128 * 128, ubytes = (uint32_t)(F / 64) * 128 * 128, stage = xbytes + ubytes;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + 2 * stage);
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 2);
+    volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
+    if (tid == 0) {
+        mbar_init(&bars[0], 1);
+        mbar_init(&bars[1], 1);
+        *fail = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(tmem_holder, 128);
+        tmem_relinquish();
+    }
+    // for d = 64 the second half of the M = 128 operand X^T stays zero
+    if (d == 64)
+        for (int i = tid; i < 2 * 1024; i += kThreads) {
+            const int st = i / 1024, k = i % 1024;
+            reinterpret_cast<uint4 *>(smem + st * stage + 128 * 128)[k] = make_uint4(0, 0, 0, 0);
+        }
+    griddep_wait();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_holder;
+    const uint32_t idW = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, F);
+    bool ok = true;
+    for (int k = 0; k < n_tiles; ++k) {
+        const int stg = k & 1;
+        if (k >= 2) ok = wait_bar(&bars[stg], (uint32_t)((k - 2) >> 1) & 1u, fail) && ok;
+        if (group_sync_failed(1, kThreads, !ok)) break;
+        uint8_t *sx = smem + stg * stage, *su = sx + xbytes;
+        // row tid of this step
+        const long long rho = r_begin + (long long)k * 128 + tid;
+        const bool valid = rho < r_end;
+        const bf16 *xr = nullptr, *ur = nullptr;
+        if (valid) {
+            const long long t = rho / K1;
+            const int kind = (int)(rho - t * K1);
+            if (kind < G) {
+                const size_t h = (size_t)g * G + kind;
+                xr = a.Q + ((size_t)t * a.Hq + h) * d;
+                ur = a.dUq + ((size_t)t * a.Hq + h) * F;
+            } else {
+                xr = a.K + ((size_t)t * a.Hkv + g) * d;
+                ur = a.dUk + ((size_t)t * a.Hkv + g) * F;
+            }
+        }
+        for (int c8 = 0; c8 < d / 8; ++c8) {
+            const uint4 v = valid ? __ldg(reinterpret_cast<const uint4 *>(xr) + c8) : make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4 *>(sx + (uint32_t)(c8 >> 3) * (128 * 128) + swz(tid, c8 & 7)) = v;
+        }
+        for (int c8 = 0; c8 < F / 8; ++c8) {
+            const uint4 v = valid ? __ldg(reinterpret_cast<const uint4 *>(ur) + c8) : make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4 *>(su + (uint32_t)(c8 >> 3) * (128 * 128) + swz(tid, c8 & 7)) = v;
+        }
+        fence_proxy_async_smem();
+        __syncthreads();
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t x_u = smem_u32(sx), u_u = smem_u32(su);
+            for (int ks = 0; ks < 8; ++ks)
+                mma_bf16_ss(tmem, smem_desc(x_u + ks * 2048, 128 * 128, 1024, SWZ_128B),
+                            smem_desc(u_u + ks * 2048, 128 * 128, 1024, SWZ_128B), idW, (k | ks) != 0);
+            mma_commit(&bars[stg]);
+        }
+    }
+    // the last one or two steps
+    for (int k = n_tiles - 2; k < n_tiles; ++k)
+        if (k >= 0) ok = wait_bar(&bars[k & 1], (uint32_t)(k >> 1) & 1u, fail) && ok;
+    tc_fence_after();
+    if (ok && n_tiles > 0 && tid < d) {
+        float *dst = a.dW + ((size_t)g * d + tid) * F;
+        const uint32_t lane_off = (uint32_t)(warp & 3) * 32u << 16;
+        float x[32];
+        for (int j = 0; j < F / 32; ++j) {
+            tmem_ld32(tmem + lane_off + 32 * j, x);
+            tmem_wait_ld();
+#pragma unroll
+            for (int k = 0; k < 32; ++k) atomicAdd(dst + 32 * j + k, x[k]);
+        }
+    } else if (n_tiles > 0 && !ok && tid == 0) {
+        raise_error(a.err, ERR_WAIT_TIMEOUT);
+    }
+    tc_fence_before();
+    __syncthreads();
+    griddep_launch_dependents();
+    if (warp == 0) tmem_dealloc(tmem, 128);
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+__global__ void k_slot_ptrs(float *P, int n, size_t slot_floats, void **ptrs)
+{
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) ptrs[i] = P + (size_t)i * slot_floats;
+}
+
+template <class Kern, class... Args>
+cudaError_t launch_pdl(Kern k, dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args... args)
+{
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = grid;
+    lc.blockDim = block;
+    lc.dynamicSmemBytes = smem;
+    lc.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 1;
+    return cudaLaunchKernelEx(&lc, k, args...);
+}
+
+template <class Kern>
+cudaError_t opt_in(Kern k, std::atomic<unsigned long long> &opted)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    const unsigned long long bit = 1ull << dev;
+    if (!(opted.load(std::memory_order_acquire) & bit)) {
+        const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
+        if (e != cudaSuccess) return e;
+        opted.fetch_or(bit, std::memory_order_release);
+    }
+    return cudaSuccess;
+}
+
+struct Workspace {
+    float *P, *PT;
+    bf16 *dUq, *dUk;
+    void **ptrs;
+    size_t bytes;
+};
+
+size_t align_up(size_t x) { return (x + 1023) & ~size_t(1023); }
+
+Workspace carve(const hybrid_cfg &c, int n_seq, int L, void *base)
+{
+    const int d = c.head_dim, F = c.feat_dim, B = c.block_size, n_blk = L / B;
+    const size_t slots = (size_t)n_seq * n_blk;
+    const size_t buf = align_up(slots * slot_floats(c.n_kv_heads, d, F) * sizeof(float));
+    const size_t uq = align_up((size_t)n_seq * L * c.n_q_heads * F * sizeof(bf16));
+    const size_t uk = align_up((size_t)n_seq * L * c.n_kv_heads * F * sizeof(bf16));
+    const size_t pt = align_up(slots * sizeof(void *));
+    Workspace w{};
+    uint8_t *p = static_cast<uint8_t *>(base);
+    w.P = reinterpret_cast<float *>(p);
+    w.PT = reinterpret_cast<float *>(p ? p + buf : nullptr);
+    w.dUq = reinterpret_cast<bf16 *>(p ? p + 2 * buf : nullptr);
+    w.dUk = reinterpret_cast<bf16 *>(p ? p + 2 * buf + uq : nullptr);
+    w.ptrs = reinterpret_cast<void **>(p ? p + 2 * buf + uq + uk : nullptr);
+    w.bytes = 2 * buf + uq + uk + pt;
+    return w;
+}
+
+TrainArgs make_args(const hybrid_cfg &c, int n_seq, int L, const Workspace &w)
+{
+    TrainArgs a{};
+    a.n_seq = n_seq;
+    a.L = L;
+    a.B = c.block_size;
+    a.Hq = c.n_q_heads;
+    a.Hkv = c.n_kv_heads;
+    a.d = c.head_dim;
+    a.F = c.feat_dim;
+    a.n_blk = L / c.block_size;
+    a.P = w.P;
+    a.PT = w.PT;
+    a.R = w.P;   // the backward reuses the decode image's space for R
+    a.dUq = w.dUq;
+    a.dUk = w.dUk;
+    return a;
+}
+
+std::atomic<unsigned long long> g_opt_state, g_opt_q, g_opt_k, g_opt_dw;
+
+}  // namespace
+
+bool train_supported(const hybrid_cfg &c, int seq_len)
+{
+    if (c.io_dtype != HYBRID_BF16) return false;
+    if (c.head_dim != 64 && c.head_dim != 128) return false;
+    if (c.feat_dim != 64 && c.feat_dim != 128) return false;
+    const int B = c.block_size;
+    if (B != 16 && B != 32 && B != 64) return false;
+    if (c.n_kv_heads <= 0 || c.n_q_heads % c.n_kv_heads != 0) return false;
+    if ((c.n_q_heads / c.n_kv_heads) * B > 128) return false;
+    if (seq_len <= 0 || seq_len % B != 0) return false;
+    return make_grad_layout(c.head_dim, c.feat_dim, B).bytes <= (uint32_t)kSmemLimit;
+}
+
+size_t train_workspace_bytes(const hybrid_cfg &c, int n_seq, int seq_len)
+{
+    return carve(c, n_seq, seq_len, nullptr).bytes;
+}
+
+void *const *train_state_ptrs(const hybrid_cfg &c, int n_seq, int seq_len, void *workspace)
+{
+    return carve(c, n_seq, seq_len, workspace).ptrs;
+}
+
+cudaError_t launch_train_states(const hybrid_cfg &c, const void *K, const void *V, const void *W, int n_seq,
+                                int seq_len, void *workspace, unsigned *err, cudaStream_t st)
+{
+    const Workspace w = carve(c, n_seq, seq_len, workspace);
+    TrainArgs a = make_args(c, n_seq, seq_len, w);
+    a.K = static_cast<const bf16 *>(K);
+    a.V = static_cast<const bf16 *>(V);
+    a.W = static_cast<const bf16 *>(W);
+    a.err = err;
+    const int slots = n_seq * a.n_blk;
+    const size_t sf = slot_floats(a.Hkv, a.d, a.F);
+    cudaError_t e = cudaSuccess;
+    k_slot_ptrs<<<(slots + 255) / 256, 256, 0, st>>>(w.P, slots, sf, w.ptrs);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    const RowLayout Ls = make_state_layout(a.d, a.F, a.B);
+    if ((e = opt_in(k_block_state, g_opt_state)) != cudaSuccess) return e;
+    e = launch_pdl(k_block_state, dim3((unsigned)(slots * a.Hkv)), dim3(kThreads), Ls.bytes, st, a, Ls);
+    if (e != cudaSuccess) return e;
+    const size_t n4 = sf / 4 * (size_t)n_seq;
+    return launch_pdl(k_slot_scan, dim3((unsigned)((n4 + 255) / 256), 2), dim3(256), 0, st, w.P, w.PT, n_seq,
+                      a.n_blk, sf, false);
+}
+
+cudaError_t launch_train_backward(const hybrid_cfg &c, const void *Q, const void *K, const void *V, const void *W,
+                                  const float *alpha, const void *O, const void *dO, int n_seq, int seq_len,
+                                  void *workspace, float *dW, float *dalpha, unsigned *err, cudaStream_t st)
+{
+    const Workspace w = carve(c, n_seq, seq_len, workspace);
+    TrainArgs a = make_args(c, n_seq, seq_len, w);
+    a.Q = static_cast<const bf16 *>(Q);
+    a.K = static_cast<const bf16 *>(K);
+    a.V = static_cast<const bf16 *>(V);
+    a.W = static_cast<const bf16 *>(W);
+    a.O = static_cast<const bf16 *>(O);
+    a.dO = static_cast<const bf16 *>(dO);
+    a.alpha = alpha;
+    a.dalpha = dalpha;
+    a.err = err;
+    const int units = n_seq * a.n_blk * a.Hkv;
+    const size_t sf = slot_floats(a.Hkv, a.d, a.F);
+    cudaError_t e;
+    if ((e = cudaMemsetAsync(dW, 0, (size_t)a.Hkv * a.d * a.F * sizeof(float), st)) != cudaSuccess) return e;
+    if ((e = cudaMemsetAsync(dalpha, 0, (size_t)a.Hq * sizeof(float), st)) != cudaSuccess) return e;
+    const RowLayout Lg = make_grad_layout(a.d, a.F, a.B);
+    if ((e = opt_in(k_phi_grad<true>, g_opt_q)) != cudaSuccess) return e;
+    if ((e = opt_in(k_phi_grad<false>, g_opt_k)) != cudaSuccess) return e;
+    if ((e = launch_pdl(k_phi_grad<true>, dim3((unsigned)units), dim3(kThreads), Lg.bytes, st, a, Lg)) != cudaSuccess)
+        return e;
+    const size_t n4 = sf / 4 * (size_t)n_seq;
+    if ((e = launch_pdl(k_slot_scan, dim3((unsigned)((n4 + 255) / 256), 1), dim3(256), 0, st, a.R,
+                        static_cast<float *>(nullptr), n_seq, a.n_blk, sf, true)) != cudaSuccess)
+        return e;
+    if ((e = launch_pdl(k_phi_grad<false>, dim3((unsigned)units), dim3(kThreads), Lg.bytes, st, a, Lg)) != cudaSuccess)
+        return e;
+    DwArgs b{};
+    b.Q = a.Q;
+    b.K = a.K;
+    b.dUq = w.dUq;
+    b.dUk = w.dUk;
+    b.dW = dW;
+    b.err = err;
+    b.n_tok = (long long)n_seq * seq_len;
+    b.Hq = a.Hq;
+    b.Hkv = a.Hkv;
+    b.d = a.d;
+    b.F = a.F;
+    const long long rows = b.n_tok * (a.Hq / a.Hkv + 1);
+    const long long tiles = (rows + 127) / 128;
+    int per_group = (2 * sm_count() + a.Hkv - 1) / a.Hkv;
+    if (per_group > tiles) per_group = (int)tiles;
+    if (per_group < 1) per_group = 1;
+    b.tiles_per_cta = (int)((tiles + per_group - 1) / per_group);
+    b.ctas_per_group = per_group;
+    const size_t dw_smem = 2 * ((size_t)2 * 128 * 128 + (size_t)(a.F / 64) * 128 * 128) + 1024 + 1024;
+    if ((e = opt_in(k_dw, g_opt_dw)) != cudaSuccess) return e;
+    return launch_pdl(k_dw, dim3((unsigned)(a.Hkv * per_group)), dim3(kThreads), dw_smem, st, b);
+}
+
+}  // namespace hyb

@@ -25,8 +25,9 @@ HYBRID_BF16 = 1
 
 EXPORTED = (
     "hybrid_state_bytes", "hybrid_state_init", "hybrid_feature_map", "hybrid_block_attn",
-    "hybrid_block_attn_commit", "hybrid_block_attn_commit_logical", "hybrid_commit_block", "hybrid_state_unpack", "hybrid_state_pack", "hybrid_check",
-    "hybrid_status_str",
+    "hybrid_block_attn_commit", "hybrid_block_attn_commit_logical", "hybrid_commit_block", "hybrid_state_unpack",
+    "hybrid_state_pack", "hybrid_train_workspace_bytes", "hybrid_train_forward", "hybrid_train_backward",
+    "hybrid_check", "hybrid_status_str",
 )
 
 
@@ -76,11 +77,16 @@ def lib(path: str | None = None):
     L.hybrid_commit_block.argtypes = [cfgp, P, P, I, P, P, I, P]
     L.hybrid_state_unpack.argtypes = [cfgp, P, I, P, P, P]
     L.hybrid_state_pack.argtypes = [cfgp, P, P, P, I, P]
+    S = ctypes.c_size_t
+    L.hybrid_train_workspace_bytes.argtypes = [cfgp, I, I]
+    L.hybrid_train_workspace_bytes.restype = S
+    L.hybrid_train_forward.argtypes = [cfgp, P, P, P, P, P, I, I, P, P, S, P]
+    L.hybrid_train_backward.argtypes = [cfgp, P, P, P, P, P, P, P, I, I, P, S, P, P, P]
     L.hybrid_check.argtypes = [P]
     L.hybrid_status_str.argtypes = [I]
     L.hybrid_status_str.restype = ctypes.c_char_p
     for name in EXPORTED:
-        if name not in ("hybrid_state_bytes", "hybrid_status_str"):
+        if name not in ("hybrid_state_bytes", "hybrid_status_str", "hybrid_train_workspace_bytes"):
             getattr(L, name).restype = ctypes.c_int
     if path == _build.LIB_PATH:
         _lib = L
@@ -173,6 +179,26 @@ def hybrid_state_pack(cfg, S_logical, z_logical, state_ptrs, n_req, stream=None,
     st = lib().hybrid_state_pack(ctypes.byref(cfg), _ptr(S_logical), _ptr(z_logical), _ptr(state_ptrs),
                                  int(n_req), _stream(stream))
     return _ret(st, "hybrid_state_pack", check)
+
+
+def hybrid_train_workspace_bytes(cfg, n_seq, seq_len) -> int:
+    return int(lib().hybrid_train_workspace_bytes(ctypes.byref(cfg), int(n_seq), int(seq_len)))
+
+
+def hybrid_train_forward(cfg, Q, K, V, W, alpha, n_seq, seq_len, O, workspace, workspace_bytes, stream=None,
+                         check=True):
+    st = lib().hybrid_train_forward(ctypes.byref(cfg), _ptr(Q), _ptr(K), _ptr(V), _ptr(W), _ptr(alpha),
+                                    int(n_seq), int(seq_len), _ptr(O), _ptr(workspace), int(workspace_bytes),
+                                    _stream(stream))
+    return _ret(st, "hybrid_train_forward", check)
+
+
+def hybrid_train_backward(cfg, Q, K, V, W, alpha, O, dO, n_seq, seq_len, workspace, workspace_bytes, dW,
+                          dalpha, stream=None, check=True):
+    st = lib().hybrid_train_backward(ctypes.byref(cfg), _ptr(Q), _ptr(K), _ptr(V), _ptr(W), _ptr(alpha),
+                                     _ptr(O), _ptr(dO), int(n_seq), int(seq_len), _ptr(workspace),
+                                     int(workspace_bytes), _ptr(dW), _ptr(dalpha), _stream(stream))
+    return _ret(st, "hybrid_train_backward", check)
 
 
 def hybrid_check(stream=None, check=True):

@@ -43,6 +43,7 @@ class Workload:
     layers: int = 1
     steps_per_block: int = 1
     blocks: int = 0           # decode loop length (config 4)
+    seq_len: int = 0          # training form: tokens per sequence (n_req sequences)
     description: str = ""
 
     @property
@@ -70,6 +71,13 @@ C5 = Workload("c5_bf16_b256_f256_k8", torch.bfloat16, n_req=256, Hq=16, Hkv=16, 
               seed=4, prefix_min=1024, prefix_max=32768, k_scale=8.0,
               description="bf16, batch 256, 16 heads, d 128, F 256, B 64, ragged 1k-32k, K x8")
 CONFIGS = {w.name: w for w in (C1, C2, C3, C4, C5)}
+
+# Training form (Stage 1 attention transfer): batches of whole sequences with
+# the layer shape of configuration 3; the paper's transfer runs over moderate
+# generation lengths (2048-token sequences here).
+T1 = Workload("t1_bf16_stage1_8x2048_gqa", torch.bfloat16, n_req=8, Hq=16, Hkv=4, d=128, F=128, B=32,
+              seed=5, seq_len=2048,
+              description="bf16, 8 sequences of 2048 tokens (64 blocks of 32), GQA 16:4, d 128, F 128")
 
 
 def sub_seed(base: int, *tags) -> int:
@@ -115,6 +123,18 @@ def block_qkv(wl: Workload, tag, device="cpu", n_req=None):
     K = _randn((n, wl.B, wl.Hkv, wl.d), sub_seed(wl.seed, "K", tag), device, wl.io_dtype, wl.k_scale)
     V = _randn((n, wl.B, wl.Hkv, wl.d), sub_seed(wl.seed, "V", tag), device, wl.io_dtype)
     return Q, K, V
+
+
+def train_batch(wl: Workload, tag=0, device="cpu", n_seq=None, seq_len=None):
+    """Q, dO [n, L, Hq, d] and K, V [n, L, Hkv, d] of a training batch (io dtype).
+    dO stands in for the gradient of the attention-transfer loss."""
+    n = wl.n_req if n_seq is None else n_seq
+    L = wl.seq_len if seq_len is None else seq_len
+    Q = _randn((n, L, wl.Hq, wl.d), sub_seed(wl.seed, "tQ", tag), device, wl.io_dtype)
+    K = _randn((n, L, wl.Hkv, wl.d), sub_seed(wl.seed, "tK", tag), device, wl.io_dtype, wl.k_scale)
+    V = _randn((n, L, wl.Hkv, wl.d), sub_seed(wl.seed, "tV", tag), device, wl.io_dtype)
+    dO = _randn((n, L, wl.Hq, wl.d), sub_seed(wl.seed, "tdO", tag), device, wl.io_dtype)
+    return Q, K, V, dO
 
 
 def prefix_kv(wl: Workload, block: int, device="cpu", n_req=None, n_tok=None, layer: int = 0):

@@ -104,3 +104,44 @@ def test_status_strings(L):
 def test_binding_names_match_abi():
     for name in H.EXPORTED:
         assert callable(getattr(H, name))
+
+
+def _al(x):
+    return (x + 1023) & ~1023
+
+
+def test_train_workspace_bytes(L):
+    # two state buffers of n_seq * n_blk slots, du of the query and key rows (bf16), the slot pointers
+    n, Lq = 8, 2048
+    slots = n * (Lq // 32)
+    want = 2 * _al(slots * 4 * (2 * 128 * 128 + 2 * 128) * 4) + _al(n * Lq * 16 * 128 * 2) \
+        + _al(n * Lq * 4 * 128 * 2) + _al(slots * 8)
+    assert H.hybrid_train_workspace_bytes(cfg(), n, Lq) == want
+    # unsupported shapes give 0
+    assert H.hybrid_train_workspace_bytes(cfg(dt=H.HYBRID_F32), n, Lq) == 0
+    assert H.hybrid_train_workspace_bytes(cfg(F=256, Hq=16, Hkv=16), n, Lq) == 0
+    assert H.hybrid_train_workspace_bytes(cfg(Hq=16, Hkv=2), n, Lq) == 0       # G * B = 256 rows
+    assert H.hybrid_train_workspace_bytes(cfg(), n, 2000) == 0                 # not whole blocks
+    assert H.hybrid_train_workspace_bytes(cfg(), 0, Lq) == 0
+
+
+def test_train_argument_checks(L):
+    """Host-side validation of the training entry points; no device work."""
+    c = cfg()
+    ok = 1 << 20
+    n, Lq = 2, 128
+    nb = H.hybrid_train_workspace_bytes(c, n, Lq)
+    fwd = lambda cc, q=ok, ws=ok, wsb=nb, sl=Lq: L.hybrid_train_forward(  # noqa: E731
+        ctypes.byref(cc), q, ok, ok, ok, ok, n, sl, ok, ws, wsb, None)
+    bwd = lambda cc, do=ok, dw=ok: L.hybrid_train_backward(  # noqa: E731
+        ctypes.byref(cc), ok, ok, ok, ok, ok, ok, do, n, Lq, ok, nb, dw, ok, None)
+    assert fwd(cfg(dt=H.HYBRID_F32)) == H.HYBRID_ERR_UNSUPPORTED
+    assert fwd(cfg(Hq=16, Hkv=2)) == H.HYBRID_ERR_UNSUPPORTED
+    assert fwd(c, sl=100) == H.HYBRID_ERR_INVALID_ARG
+    assert fwd(c, sl=0) == H.HYBRID_ERR_INVALID_ARG
+    assert fwd(c, q=None) == H.HYBRID_ERR_INVALID_ARG
+    assert fwd(c, q=ok + 8) == H.HYBRID_ERR_INVALID_ARG
+    assert fwd(c, ws=ok + 512) == H.HYBRID_ERR_INVALID_ARG
+    assert fwd(c, wsb=nb - 1) == H.HYBRID_ERR_INVALID_ARG
+    assert bwd(c, do=None) == H.HYBRID_ERR_INVALID_ARG
+    assert bwd(c, dw=ok + 4) == H.HYBRID_ERR_INVALID_ARG
