@@ -199,7 +199,7 @@ hybrid_status hybrid_state_pack(const hybrid_cfg *cfg, const float *S_logical,
  * trains only psi = {W, alpha} to match a frozen softmax teacher's output
  * under a squared-error loss; the caller forms dO = dL/dO from its loss.
  *
- *   Q, O, dO  [n_seq][seq_len][Hq][d]    bf16
+ *   Q, O, dO  [n_seq][seq_len][Hq][d]    bf16  (O: output of the forward)
  *   K, V      [n_seq][seq_len][Hkv][d]   bf16
  *   W         [Hkv][d][F] bf16;  alpha [Hq] float32
  *   dW        [Hkv][d][F] float32;  dalpha [Hq] float32  (overwritten)
@@ -224,15 +224,16 @@ hybrid_status hybrid_train_forward(const hybrid_cfg *cfg, const void *Q, const v
                                    void *workspace, size_t workspace_bytes, cudaStream_t stream);
 
 /* Gradient of sum(dO * O) with respect to W and alpha, O being the output of
- * the preceding hybrid_train_forward on this workspace:
+ * the preceding hybrid_train_forward on this workspace (O itself is not read:
+ * dO . O is re-formed in fp32 from the merge's terms):
  *   dN = dO / D, dD = -(dO . O) / D (D = the merge's denominator),
  *   dw_h = sum (dN . sm_num + dD sm_den), dalpha_h = dw_h w_h (1 - w_h),
  *   dphi(q) = S_{n-1} dN + z_{n-1} dD,  dphi(k_t in B_m) = sum_{n>m} dS_{n-1} v_t + dz_{n-1},
  *   dW = sum over query and key rows of x du^T through phi's two softmaxes. */
 hybrid_status hybrid_train_backward(const hybrid_cfg *cfg, const void *Q, const void *K, const void *V,
-                                    const void *W, const float *alpha, const void *O, const void *dO,
-                                    int n_seq, int seq_len, void *workspace, size_t workspace_bytes,
-                                    float *dW, float *dalpha, cudaStream_t stream);
+                                    const void *W, const float *alpha, const void *dO, int n_seq,
+                                    int seq_len, void *workspace, size_t workspace_bytes, float *dW,
+                                    float *dalpha, cudaStream_t stream);
 
 /* Synchronise the stream, then read and clear this device's error word.
  * Returns HYBRID_OK, HYBRID_ERR_DEVICE (a state pointer failed its device

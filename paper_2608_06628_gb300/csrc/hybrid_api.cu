@@ -287,20 +287,20 @@ hybrid_status hybrid_train_forward(const hybrid_cfg *cfg, const void *Q, const v
 }
 
 hybrid_status hybrid_train_backward(const hybrid_cfg *cfg, const void *Q, const void *K, const void *V,
-                                    const void *W, const float *alpha, const void *O, const void *dO,
-                                    int n_seq, int seq_len, void *workspace, size_t workspace_bytes,
-                                    float *dW, float *dalpha, cudaStream_t stream)
+                                    const void *W, const float *alpha, const void *dO, int n_seq,
+                                    int seq_len, void *workspace, size_t workspace_bytes, float *dW,
+                                    float *dalpha, cudaStream_t stream)
 {
     hybrid_status s = check_train(cfg, n_seq, seq_len, workspace, workspace_bytes);
     if (s != HYBRID_OK) return s;
-    if (!Q || !K || !V || !W || !alpha || !O || !dO || !dW || !dalpha) return HYBRID_ERR_INVALID_ARG;
-    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(W, 16) || !aligned(O, 16) ||
-        !aligned(dO, 16) || !aligned(alpha, 4) || !aligned(dW, 16) || !aligned(dalpha, 4))
+    if (!Q || !K || !V || !W || !alpha || !dO || !dW || !dalpha) return HYBRID_ERR_INVALID_ARG;
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(W, 16) || !aligned(dO, 16) ||
+        !aligned(alpha, 4) || !aligned(dW, 16) || !aligned(dalpha, 4))
         return HYBRID_ERR_INVALID_ARG;
     unsigned *err = error_word();
     if (!err) return HYBRID_ERR_CUDA;
-    return from_cuda(hyb::launch_train_backward(*cfg, Q, K, V, W, alpha, O, dO, n_seq, seq_len, workspace, dW,
-                                                dalpha, err, stream));
+    return from_cuda(hyb::launch_train_backward(*cfg, Q, K, V, W, alpha, dO, n_seq, seq_len, workspace, dW, dalpha,
+                                                err, stream));
 }
 
 hybrid_status hybrid_check(cudaStream_t stream)

@@ -6,7 +6,7 @@
 // block n reads S_{n-1} = sum_{m < n} dS_m, z_{n-1} likewise (Section 3.1 applied
 // to every block, S_{-1} = 0), with dS_m = sum_{t in B_m} phi(k_t) [v_t | 1]^T.
 // Per query row i of block n (N, D = numerator and denominator of the merge,
-// g = dO row, o = O row):
+// g = dO row, o = N / D):
 //     dN = g / D,  dD = -(g . o) / D,  dw_h += dN . sm_num + dD sm_den,
 //     dphi(q) = S_{n-1} dN + z_{n-1} dD,   dR_n += phi(q) [dN | dD]^T,
 // and a key t of block m receives dphi(k_t) = R_m v_t + r_m with
@@ -23,8 +23,10 @@
 //   k_slot_scan     running sums over the slots of a sequence (P and PT
 //                   inclusive; R reverse exclusive)
 //   k_phi_grad<Q>   query side: [U | scores] = Q [W | K^T], dO V^T, the merge
-//                   terms, dN into Tensor Memory, then S dN + z dD streamed over
-//                   the PT tiles, du_q, and dR_n = phi(Q)^T [dN | dD];
+//                   terms, dN into Tensor Memory, then S dN streamed over the PT
+//                   tiles; g . o = w g.sm_num/D + phi(q).(S dN) and the gate term
+//                   are formed from these fp32 products (the forward's rounded O is
+//                   not needed), then du_q and dR_n = phi(Q)^T [dN | dD];
 //                   key side: U = K W, V into Tensor Memory, R v + r over the
 //                   R tiles, du_k
 //   k_dw            dW_g = sum over query and key rows of x du^T, split over
@@ -46,7 +48,7 @@ constexpr int kSmemLimit = 232448;
 constexpr uint32_t kColS = 0, kColGv = 64, kColU = 256, kColY = 384, kColG = 0, kColDR = 0;
 
 struct TrainArgs {
-    const bf16 *Q, *K, *V, *W, *O, *dO;
+    const bf16 *Q, *K, *V, *W, *dO;
     const float *alpha;
     float *P, *PT, *R;
     bf16 *dUq, *dUk;
@@ -428,9 +430,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
     // phase one: operands of [U | scores] = Q [W | K^T] and dO V^T (query side) or U = K W
     if (kQuery) {
         auto qrow = [&](int r) { return a.Q + (t0 + r % B) * q_row + (size_t)(g * G + r / B) * d; };
-        auto orow = [&](int r) { return a.dO + (t0 + r % B) * q_row + (size_t)(g * G + r / B) * d; };
+        auto dorow = [&](int r) { return a.dO + (t0 + r % B) * q_row + (size_t)(g * G + r / B) * d; };
         load_rows_bf16(smem + Lr.off_q, qrow, rows, 128, d, tid);
-        load_rows_bf16(smem + Lr.off_do, orow, rows, 128, d, tid);
+        load_rows_bf16(smem + Lr.off_do, dorow, rows, 128, d, tid);
         load_rows_bf16(smem + Lr.off_k, [&](int r) { return a.K + (t0 + r) * kv_row + (size_t)g * d; }, B, B, d, tid);
         load_rows_bf16(smem + Lr.off_v, [&](int r) { return a.V + (t0 + r) * kv_row + (size_t)g * d; }, B, B, d, tid);
     } else {
@@ -481,11 +483,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
     const int hl = kQuery ? tid / B : 0;
     const PhiStats st = phi_stats(tl + kColU, F);
     const float ip = 1.f / st.sp, in = 1.f / st.sn;
-    float dD = 0.f;   // coefficient of z (query side) / of r (key side) in dphi
+    // Query rows: w, 1/D, and the merge terms A = g.sm_num / D, beta = sm_den / D,
+    // lambda = lin_den / D; after S dN, Lambda = g.lin_num / D = phi(q).(S dN)
+    // gives g.o = w A + Lambda and dw = lambda A - beta Lambda (= dN.sm_num + dD sm_den).
+    float w = 0.f, inv = 0.f, A = 0.f, beta = 0.f, lambda = 0.f;
     if (kQuery) {
         const int h = g * G + hl;
         const float alpha = valid ? a.alpha[h] : 0.f;
-        const float w = 1.f / (1.f + expf(-alpha));
+        w = 1.f / (1.f + expf(-alpha));
         // phi(q) into its operand image; lin_den = phi(q) . z
         float lin_den = 0.f;
         {
@@ -526,54 +531,33 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         }
         const float ec = ex2(-c * kLog2e);
         const float Dp = w * l + lin_den * ec;
-        const float inv = valid ? ec / Dp : 0.f;   // 1 / D
-        const float pw = valid ? 1.f / Dp : 0.f;   // e^(s_j - c) / D' = e^(s_j) / D
-        // g . o and dN = g / D (Tensor Memory, fp32; operand image, bf16), dD = -(g . o) / D
-        const bf16 *grow = a.dO + (t0 + tid % B) * q_row + (size_t)(g * G + hl) * d;
-        const bf16 *orow = a.O + (t0 + tid % B) * q_row + (size_t)(g * G + hl) * d;
-        float go = 0.f;
-        if (valid) {
-            float gv[32], ov[32];
-            for (int c0 = 0; c0 < d; c0 += 32) {
-                load_row_f32(grow + c0, 32, gv);
-                load_row_f32(orow + c0, 32, ov);
-#pragma unroll
-                for (int k = 0; k < 32; ++k) go += gv[k] * ov[k];
-            }
-        }
-        dD = -go * inv;
-        {
-            float gv[32];
-            for (int c0 = 0; c0 < d; c0 += 32) {
-                if (valid) {
-                    load_row_f32(grow + c0, 32, gv);
-#pragma unroll
-                    for (int k = 0; k < 32; ++k) gv[k] *= inv;
-                } else {
-#pragma unroll
-                    for (int k = 0; k < 32; ++k) gv[k] = 0.f;
-                }
-                tmem_st32(tl + kColY + c0, gv);
-                store_row32_bf16(smem + Lr.off_y, 128 * 128, tid, c0, gv);
-            }
-            // columns d .. d+15 (the rest of that 32-column group is never read)
-            uint8_t *base = smem + Lr.off_y + (uint32_t)(d >> 6) * (128 * 128);
-            uint4 v0;
-            v0.x = pack_bf16x2(dD, 0.f);
-            v0.y = v0.z = v0.w = 0u;
-            *reinterpret_cast<uint4 *>(base + swz(tid, 0)) = v0;
-            *reinterpret_cast<uint4 *>(base + swz(tid, 1)) = make_uint4(0, 0, 0, 0);
-        }
-        // dw of this row: sum_j (e^(s_j) / D) (g . v_j - g . o)
-        float dw = 0.f;
+        inv = valid ? ec / Dp : 0.f;              // 1 / D
+        const float pw = valid ? 1.f / Dp : 0.f;  // e^(s_j - c) / D' = e^(s_j) / D
+        beta = l * pw;
+        lambda = lin_den * inv;
+        // A = sum_j (e^(s_j) / D) g.v_j
         for (int j = 0; j < B / 16; ++j) {
             float x[16];
             tmem_ld16(tl + kColGv + 16 * j, x);
             tmem_wait_ld();
 #pragma unroll
-            for (int k = 0; k < 16; ++k) dw += sc[16 * j + k] * pw * (x[k] - go);
+            for (int k = 0; k < 16; ++k) A += sc[16 * j + k] * pw * x[k];
         }
-        if (valid) atomicAdd(&sDw[hl], dw);
+        // dN = g / D: Tensor Memory (fp32, A operand of S dN) and the operand image (bf16)
+        const bf16 *grow = a.dO + (t0 + tid % B) * q_row + (size_t)(g * G + hl) * d;
+        float gv[32];
+        for (int c0 = 0; c0 < d; c0 += 32) {
+            if (valid) {
+                load_row_f32(grow + c0, 32, gv);
+#pragma unroll
+                for (int k = 0; k < 32; ++k) gv[k] *= inv;
+            } else {
+#pragma unroll
+                for (int k = 0; k < 32; ++k) gv[k] = 0.f;
+            }
+            tmem_st32(tl + kColY + c0, gv);
+            store_row32_bf16(smem + Lr.off_y, 128 * 128, tid, c0, gv);
+        }
     } else {
         // V rows (fp32) as the Tensor Memory A operand of R v; r enters with coefficient 1
         const bf16 *vrow = a.V + (t0 + tid) * kv_row + (size_t)g * d;
@@ -587,7 +571,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
             }
             tmem_st32(tl + kColY + c0, vv);
         }
-        dD = valid ? 1.f : 0.f;
     }
     tmem_wait_st();
     fence_proxy_async_smem();
@@ -624,47 +607,73 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
     if (!failed1) ok = wait_bar(mbar, 1, fail) && ok;
     tc_fence_after();
 
-    // ---- du = p+ (g+ - <g+, p+>) - p- (g- - <g-, p->) with g = dphi (+ z dD) ----
+    // ---- du = p+ (g+ - <g+, p+>) - p- (g- - <g-, p->) with g = G + zeta dD, where
+    // G = S dN (query) or R v (key) and zeta = z_{n-1} (query) or r_m (key) ----
     if (!failed1 && !*fail) {
-        float dotp = 0.f, dotn = 0.f;
         float x[32], gp[32], gn[32];
-        for (int pass = 0; pass < 2; ++pass) {
-            for (int j = 0; j < F / 32; ++j) {
-                tmem_ld32(tl + kColU + 32 * j, x);
-                tmem_ld32(tl + kColG + 32 * j, gp);
-                tmem_ld32(tl + kColG + F + 32 * j, gn);
-                tmem_wait_ld();
-                float du[32];
+        // pass 0: Lambda+- = <G+-, p+->, Z+- = <zeta+-, p+->
+        float Lp = 0.f, Ln = 0.f, Zp = 0.f, Zn = 0.f;
+        for (int j = 0; j < F / 32; ++j) {
+            tmem_ld32(tl + kColU + 32 * j, x);
+            tmem_ld32(tl + kColG + 32 * j, gp);
+            tmem_ld32(tl + kColG + F + 32 * j, gn);
+            tmem_wait_ld();
 #pragma unroll
-                for (int k = 0; k < 32; ++k) {
-                    const float pp = ex2((x[k] - st.mp) * kLog2e) * ip;
-                    const float pn = ex2((st.mn - x[k]) * kLog2e) * in;
-                    const float g1 = gp[k] + sZ[32 * j + k] * dD;
-                    const float g2 = gn[k] + sZ[F + 32 * j + k] * dD;
-                    if (pass == 0) {
-                        dotp += g1 * pp;
-                        dotn += g2 * pn;
-                    } else {
-                        du[k] = pp * (g1 - dotp) - pn * (g2 - dotn);
-                    }
-                }
-                if (pass == 1 && valid) {
-                    bf16 *out = kQuery ? a.dUq + ((t0 + tid % B) * Hq + (size_t)(g * G + hl)) * F
-                                       : a.dUk + ((t0 + tid) * Hkv + (size_t)g) * F;
-                    uint4 *o4 = reinterpret_cast<uint4 *>(out + 32 * j);
+            for (int k = 0; k < 32; ++k) {
+                const float pp = ex2((x[k] - st.mp) * kLog2e) * ip;
+                const float pn = ex2((st.mn - x[k]) * kLog2e) * in;
+                Lp += gp[k] * pp;
+                Ln += gn[k] * pn;
+                Zp += sZ[32 * j + k] * pp;
+                Zn += sZ[F + 32 * j + k] * pn;
+            }
+        }
+        float dD = valid ? 1.f : 0.f;
+        if (kQuery) {
+            const float Lam = Lp + Ln;
+            dD = -(w * A + Lam) * inv;   // -(g . o) / D
+            if (valid) atomicAdd(&sDw[hl], lambda * A - beta * Lam);
+            // column d of [dN | dD | 0] (the rest of that 32-column group is never read)
+            uint8_t *base = smem + Lr.off_y + (uint32_t)(d >> 6) * (128 * 128);
+            uint4 v0;
+            v0.x = pack_bf16x2(dD, 0.f);
+            v0.y = v0.z = v0.w = 0u;
+            *reinterpret_cast<uint4 *>(base + swz(tid, 0)) = v0;
+            *reinterpret_cast<uint4 *>(base + swz(tid, 1)) = make_uint4(0, 0, 0, 0);
+        }
+        const float dotp = Lp + dD * Zp, dotn = Ln + dD * Zn;
+        // pass 1: du
+        for (int j = 0; j < F / 32; ++j) {
+            tmem_ld32(tl + kColU + 32 * j, x);
+            tmem_ld32(tl + kColG + 32 * j, gp);
+            tmem_ld32(tl + kColG + F + 32 * j, gn);
+            tmem_wait_ld();
+            float du[32];
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        uint4 v;
-                        v.x = pack_bf16x2(du[8 * q + 0], du[8 * q + 1]);
-                        v.y = pack_bf16x2(du[8 * q + 2], du[8 * q + 3]);
-                        v.z = pack_bf16x2(du[8 * q + 4], du[8 * q + 5]);
-                        v.w = pack_bf16x2(du[8 * q + 6], du[8 * q + 7]);
-                        o4[q] = v;
-                    }
+            for (int k = 0; k < 32; ++k) {
+                const float pp = ex2((x[k] - st.mp) * kLog2e) * ip;
+                const float pn = ex2((st.mn - x[k]) * kLog2e) * in;
+                const float g1 = gp[k] + sZ[32 * j + k] * dD;
+                const float g2 = gn[k] + sZ[F + 32 * j + k] * dD;
+                du[k] = pp * (g1 - dotp) - pn * (g2 - dotn);
+            }
+            if (valid) {
+                bf16 *out = kQuery ? a.dUq + ((t0 + tid % B) * Hq + (size_t)(g * G + hl)) * F
+                                   : a.dUk + ((t0 + tid) * Hkv + (size_t)g) * F;
+                uint4 *o4 = reinterpret_cast<uint4 *>(out + 32 * j);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    uint4 v;
+                    v.x = pack_bf16x2(du[8 * q + 0], du[8 * q + 1]);
+                    v.y = pack_bf16x2(du[8 * q + 2], du[8 * q + 3]);
+                    v.z = pack_bf16x2(du[8 * q + 4], du[8 * q + 5]);
+                    v.w = pack_bf16x2(du[8 * q + 6], du[8 * q + 7]);
+                    o4[q] = v;
                 }
             }
         }
     }
+    fence_proxy_async_smem();
     tc_fence_before();
     const bool failed2 = group_sync_failed(1, kThreads, failed1 || !ok || *fail);
     tc_fence_after();
@@ -976,7 +985,7 @@ cudaError_t launch_train_states(const hybrid_cfg &c, const void *K, const void *
 }
 
 cudaError_t launch_train_backward(const hybrid_cfg &c, const void *Q, const void *K, const void *V, const void *W,
-                                  const float *alpha, const void *O, const void *dO, int n_seq, int seq_len,
+                                  const float *alpha, const void *dO, int n_seq, int seq_len,
                                   void *workspace, float *dW, float *dalpha, unsigned *err, cudaStream_t st)
 {
     const Workspace w = carve(c, n_seq, seq_len, workspace);
@@ -985,7 +994,6 @@ cudaError_t launch_train_backward(const hybrid_cfg &c, const void *Q, const void
     a.K = static_cast<const bf16 *>(K);
     a.V = static_cast<const bf16 *>(V);
     a.W = static_cast<const bf16 *>(W);
-    a.O = static_cast<const bf16 *>(O);
     a.dO = static_cast<const bf16 *>(dO);
     a.alpha = alpha;
     a.dalpha = dalpha;

@@ -17,7 +17,7 @@ void *const *train_state_ptrs(const hybrid_cfg &c, int n_seq, int seq_len, void 
 cudaError_t launch_train_states(const hybrid_cfg &c, const void *K, const void *V, const void *W, int n_seq,
                                 int seq_len, void *workspace, unsigned *err, cudaStream_t st);
 cudaError_t launch_train_backward(const hybrid_cfg &c, const void *Q, const void *K, const void *V, const void *W,
-                                  const float *alpha, const void *O, const void *dO, int n_seq, int seq_len,
+                                  const float *alpha, const void *dO, int n_seq, int seq_len,
                                   void *workspace, float *dW, float *dalpha, unsigned *err, cudaStream_t st);
 
 }  // namespace hyb

@@ -81,7 +81,7 @@ def lib(path: str | None = None):
     L.hybrid_train_workspace_bytes.argtypes = [cfgp, I, I]
     L.hybrid_train_workspace_bytes.restype = S
     L.hybrid_train_forward.argtypes = [cfgp, P, P, P, P, P, I, I, P, P, S, P]
-    L.hybrid_train_backward.argtypes = [cfgp, P, P, P, P, P, P, P, I, I, P, S, P, P, P]
+    L.hybrid_train_backward.argtypes = [cfgp, P, P, P, P, P, P, I, I, P, S, P, P, P]
     L.hybrid_check.argtypes = [P]
     L.hybrid_status_str.argtypes = [I]
     L.hybrid_status_str.restype = ctypes.c_char_p
@@ -193,10 +193,10 @@ def hybrid_train_forward(cfg, Q, K, V, W, alpha, n_seq, seq_len, O, workspace, w
     return _ret(st, "hybrid_train_forward", check)
 
 
-def hybrid_train_backward(cfg, Q, K, V, W, alpha, O, dO, n_seq, seq_len, workspace, workspace_bytes, dW,
-                          dalpha, stream=None, check=True):
+def hybrid_train_backward(cfg, Q, K, V, W, alpha, dO, n_seq, seq_len, workspace, workspace_bytes, dW, dalpha,
+                          stream=None, check=True):
     st = lib().hybrid_train_backward(ctypes.byref(cfg), _ptr(Q), _ptr(K), _ptr(V), _ptr(W), _ptr(alpha),
-                                     _ptr(O), _ptr(dO), int(n_seq), int(seq_len), _ptr(workspace),
+                                     _ptr(dO), int(n_seq), int(seq_len), _ptr(workspace),
                                      int(workspace_bytes), _ptr(dW), _ptr(dalpha), _stream(stream))
     return _ret(st, "hybrid_train_backward", check)
 

@@ -134,7 +134,7 @@ def test_train_argument_checks(L):
     fwd = lambda cc, q=ok, ws=ok, wsb=nb, sl=Lq: L.hybrid_train_forward(  # noqa: E731
         ctypes.byref(cc), q, ok, ok, ok, ok, n, sl, ok, ws, wsb, None)
     bwd = lambda cc, do=ok, dw=ok: L.hybrid_train_backward(  # noqa: E731
-        ctypes.byref(cc), ok, ok, ok, ok, ok, ok, do, n, Lq, ok, nb, dw, ok, None)
+        ctypes.byref(cc), ok, ok, ok, ok, ok, do, n, Lq, ok, nb, dw, ok, None)
     assert fwd(cfg(dt=H.HYBRID_F32)) == H.HYBRID_ERR_UNSUPPORTED
     assert fwd(cfg(Hq=16, Hkv=2)) == H.HYBRID_ERR_UNSUPPORTED
     assert fwd(c, sl=100) == H.HYBRID_ERR_INVALID_ARG

@@ -43,7 +43,7 @@ def run_gpu(wl, Q, K, V, W, alpha, dO):
     H.hybrid_train_forward(cfg, Q, K, V, W, alpha, n_seq, L, O, ptr, nbytes)
     dW = torch.empty(W.shape, dtype=torch.float32, device="cuda")
     dalpha = torch.empty(wl.Hq, dtype=torch.float32, device="cuda")
-    H.hybrid_train_backward(cfg, Q, K, V, W, alpha, O, dO, n_seq, L, ptr, nbytes, dW, dalpha)
+    H.hybrid_train_backward(cfg, Q, K, V, W, alpha, dO, n_seq, L, ptr, nbytes, dW, dalpha)
     H.hybrid_check()
     return O, dW, dalpha
 
