@@ -234,15 +234,14 @@ def cpu_baseline(wl, budget_s=12.0):
 def small_config_context(dev, warmup=5, iters=20):
     """Context for the two small configurations (not part of the value): the
     per-call device time of the call the tests make on them, replayed from a CUDA
-    graph and launched directly (median of iters after warmup), and the oracle's
-    one-thread time for the same call.  c1 (fp32, one request) is latency-bound
-    and uses one buffer set; c2 rotates enough sets that each call misses L2."""
+    graph and launched directly (median of iters after warmup); the oracle's
+    one-thread time for the same call is in the CPU-baseline leg.  c1 (fp32, one
+    request) is latency-bound and uses one buffer set; c2 rotates enough sets that
+    each call misses L2."""
     import torch
-    import oracle
     from paper_2608_06628_gb300 import hybrid as H
     from paper_2608_06628_gb300 import workloads as wk
     from paper_2608_06628_gb300.state_pool import StatePool
-    orc = oracle.load()
     out = {}
     for wl, fused in ((wk.C1, False), (wk.C2, True)):
         cfg = H.make_cfg(wl.d, wl.F, wl.Hq, wl.Hkv, wl.B, wl.io_dtype)
@@ -301,7 +300,22 @@ def small_config_context(dev, warmup=5, iters=20):
         status = H.hybrid_check(check=False)
         if status != H.HYBRID_OK:
             raise SystemExit(f"device error in the small-config context: {H.hybrid_status_str(status)}")
-        # the oracle's cost does not depend on the state's values: time it on empty states
+        nbytes = ab["fused"] if fused else ab["attn"]
+        out[wl.name] = {"call": fn.__name__, "graph_us": graph_ms * 1e3, "direct_us_median": direct * 1e3,
+                        "algorithmic_bytes": nbytes, "buffer_sets": n_sets,
+                        "tokens_per_s_graph": wl.n_req * wl.B / (graph_ms * 1e-3)}
+    return out
+
+
+def small_config_oracle():
+    """The oracle's one-thread time for the call small_config_context times on
+    c1 and c2 (its cost does not depend on the state's values: empty states)."""
+    import torch
+    import oracle
+    from paper_2608_06628_gb300 import workloads as wk
+    orc = oracle.load()
+    out = {}
+    for wl, fused in ((wk.C1, False), (wk.C2, True)):
         Wc, alc = wk.params(wl)
         W64, al64 = Wc.double().numpy(), alc.double().numpy()
         Q, K, V = wk.block_qkv(wl, "ctx-oracle", "cpu")
@@ -311,13 +325,96 @@ def small_config_context(dev, warmup=5, iters=20):
         orc.block_attn(Q64, K64, V64, W64, al64, S, z, n_threads=1)
         if fused:
             orc.commit(K64, V64, W64, S, z, n_threads=1)
-        t_orc = time.perf_counter() - t0
-        nbytes = ab["fused"] if fused else ab["attn"]
-        out[wl.name] = {"call": fn.__name__, "graph_us": graph_ms * 1e3, "direct_us_median": direct * 1e3,
-                        "algorithmic_bytes": nbytes, "buffer_sets": n_sets,
-                        "tokens_per_s_graph": wl.n_req * wl.B / (graph_ms * 1e-3),
-                        "oracle_1thread_us": t_orc * 1e6}
+        out[wl.name] = {"oracle_1thread_us": (time.perf_counter() - t0) * 1e6}
     return out
+
+
+def train_flops(wl):
+    """Dense-contraction flops of one training forward and backward (Stage 1) on
+    the workload, per (sequence, state head, block) unit times the units:
+    forward  Q W, Q K^T, P V, phi(Q) [S | z], K W, phi(K)^T [V | 1];
+    backward Q W, Q K^T, dO V^T, S dN, phi(Q)^T [dN | dD], K W, R v, and
+    dW = sum x du^T over the G B query rows and B key rows."""
+    G, B, d, F = wl.Hq // wl.Hkv, wl.B, wl.d, wl.F
+    rq = G * B
+    fwd = rq * 2 * d * F + 2 * rq * B * d * 2 + rq * 2 * F * (d + 1) * 2 + B * 2 * d * F + B * 2 * F * (d + 1) * 2
+    bwd = (rq * 2 * d * F + 2 * rq * B * d * 2 + rq * 2 * F * d * 2 + rq * 2 * F * (d + 1) * 2
+           + B * 2 * d * F + B * 2 * F * d * 2 + (rq + B) * d * F * 2)
+    units = wl.n_req * wl.Hkv * (wl.seq_len // wl.B)
+    return fwd * units, bwd * units
+
+
+def train_context(dev, warmup=2, iters=5):
+    """Context (not part of the value): the training form of Stage 1 attention
+    transfer on the 8 x 2048-token batch (hybrid_train_forward, then
+    hybrid_train_backward), median device time of iters pairs after warmup."""
+    import torch
+    from paper_2608_06628_gb300 import hybrid as H
+    from paper_2608_06628_gb300 import workloads as wk
+    wl = wk.T1
+    Q, K, V, dO = wk.train_batch(wl, device=dev)
+    W, alpha = wk.params(wl, 0, dev)
+    cfg = H.make_cfg(wl.d, wl.F, wl.Hq, wl.Hkv, wl.B, wl.io_dtype)
+    n, L = wl.n_req, wl.seq_len
+    nb = H.hybrid_train_workspace_bytes(cfg, n, L)
+    ws = torch.empty(nb + 1024, dtype=torch.uint8, device=dev)
+    ptr = (ws.data_ptr() + 1023) & ~1023
+    O = torch.empty_like(Q)
+    dW = torch.empty(W.shape, dtype=torch.float32, device=dev)
+    da = torch.empty(wl.Hq, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    st = stream.cuda_stream
+
+    def fwd():
+        H.hybrid_train_forward(cfg, Q, K, V, W, alpha, n, L, O, ptr, nb, st, check=False)
+
+    def bwd():
+        H.hybrid_train_backward(cfg, Q, K, V, W, alpha, dO, n, L, ptr, nb, dW, da, st, check=False)
+
+    for _ in range(warmup):
+        fwd()
+        bwd()
+    H.hybrid_check()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(iters)]
+    for e in ev:
+        e[0].record(stream)
+        fwd()
+        e[1].record(stream)
+        bwd()
+        e[2].record(stream)
+    torch.cuda.synchronize()
+    status = H.hybrid_check(check=False)
+    if status != H.HYBRID_OK:
+        raise SystemExit(f"device error in the training context: {H.hybrid_status_str(status)}")
+    tf = sorted(e[0].elapsed_time(e[1]) for e in ev)[iters // 2] * 1e-3
+    tb = sorted(e[1].elapsed_time(e[2]) for e in ev)[iters // 2] * 1e-3
+    ff, fb = train_flops(wl)
+    peaks, _ = measured_peaks()
+    bf16 = float(peaks.get("bf16_tflops", 1900.0))
+    del ws
+    return {"workload": wl.name, "calls": "hybrid_train_forward + hybrid_train_backward",
+            "tokens": n * L, "fwd_us": tf * 1e6, "bwd_us": tb * 1e6,
+            "tokens_per_s": n * L / (tf + tb), "workspace_bytes": nb,
+            "fwd_TFLOPs": ff / tf / 1e12, "bwd_TFLOPs": fb / tb / 1e12,
+            "frac_bf16_peak": (ff + fb) / (tf + tb) / 1e12 / bf16}
+
+
+def train_oracle_sample(seq_len=1024):
+    """The oracle's training forward and backward on one sequence of seq_len
+    tokens of the training batch's shape (all host threads)."""
+    import oracle
+    from paper_2608_06628_gb300 import workloads as wk
+    orc = oracle.load()
+    wl = wk.T1
+    Q, K, V, dO = wk.train_batch(wl, tag="oracle", n_seq=1, seq_len=seq_len)
+    W, alpha = wk.params(wl)
+    args = [t.double().numpy() for t in (Q, K, V, W, alpha)]
+    t0 = time.perf_counter()
+    orc.train_forward(*args, wl.B)
+    orc.train_backward(*args, dO.double().numpy(), wl.B)
+    t = time.perf_counter() - t0
+    return {"tokens_per_s": seq_len / t, "sample": f"1 sequence x {seq_len} tokens of {wl.name}, "
+            f"forward + backward, {oracle.default_threads()} threads (units: {wl.Hkv} state heads)", "s": t}
 
 
 def prefill_context(dev, wl, T=4096, warmup=2, iters=5):
@@ -669,8 +766,12 @@ def run_hybrid(args, wl):
     if not args.no_small_configs and ws == 1:
         line["small_configs"] = small_config_context(dev)
         line["prefill_context"] = prefill_context(dev, wl)
+        line["train_context"] = train_context(dev)
     if not args.no_cpu_baseline and ws == 1:
         line["cpu_baseline"] = cpu_baseline(wl)
+        if not args.no_small_configs:
+            line["cpu_baseline"]["contexts"] = {"small_configs": small_config_oracle(),
+                                                "train": train_oracle_sample()}
     print(json.dumps(line), flush=True)
     if ws > 1:
         import torch.distributed as dist
