@@ -788,12 +788,24 @@ def main(argv=None):
     ap.add_argument("--config", default="c3_bf16_b64_gqa_ragged")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-small-configs", action="store_true",
-                    help="skip the c1/c2 context timings (graph and direct launches, 1-thread oracle)")
+                    help="skip the context timings (c1/c2, prefill, training form)")
+    ap.add_argument("--context", choices=("train", "prefill", "small"),
+                    help="time only this context on cuda:0 and print its JSON object")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     from paper_2608_06628_gb300 import workloads as wk
     wl = wk.CONFIGS[args.config]
+    if args.context:
+        import torch
+        from paper_2608_06628_gb300 import build
+        build.build()
+        dev = torch.device("cuda", 0)
+        torch.cuda.set_device(dev)
+        fn = {"train": lambda: train_context(dev), "prefill": lambda: prefill_context(dev, wl),
+              "small": lambda: small_config_context(dev)}[args.context]
+        print(json.dumps({"context": args.context, **fn()}), flush=True)
+        return 0
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_hybrid(args, wl)

@@ -13,15 +13,17 @@
 // [R_m | r_m] = sum_{n > m} dR_n.  Through phi = [softmax(u), softmax(-u)],
 // u = x W:  du = p+ (g+ - <g+, p+>) - p- (g- - <g-, p->),  dW += x du^T.
 //
-// Kernels (one CTA of 128 threads per (sequence, block, state head); thread r
-// owns row r of the tile and Tensor Memory lane r):
-//   k_block_state   U = K W, phi(K), dS_m = phi^T [V | 1] on the tensor cores;
-//                   written into slot m+1 of the decode image P (S^T tiles, read
-//                   by the decode readout kernel) and of the feature-row image
-//                   PT (S tiles: row f holds 32 consecutive e, 128-byte swizzle),
-//                   whose d/32 tiles are K-major tf32 operands for S dN
-//   k_slot_scan     running sums over the slots of a sequence (P and PT
-//                   inclusive; R reverse exclusive)
+// Kernels (128 threads; thread r owns row r of a tile and Tensor Memory lane r):
+//   k_prefix_states one CTA per (sequence, state head, 32-feature slice): sweeps
+//                   the blocks in order with the slice of S^T accumulating in
+//                   Tensor Memory (S^T += V^T phi(K), bf16 MMA) and writes
+//                   S_{n-1}, z_{n-1} into slot n of the decode image P (S^T
+//                   tiles, read by the decode readout kernel) and of the
+//                   feature-row image PT (S tiles: row f holds 32 consecutive e,
+//                   128-byte swizzle), whose d/32 tiles are K-major tf32
+//                   operands for S dN
+//   k_slot_scan     reverse exclusive running sums over the R slots of a
+//                   sequence (one CTA per (sequence, block, state head) below)
 //   k_phi_grad<Q>   query side: [U | scores] = Q [W | K^T], dO V^T, the merge
 //                   terms, dN into Tensor Memory, then S dN streamed over the PT
 //                   tiles; g . o = w g.sm_num/D + phi(q).(S dN) and the gate term
@@ -74,8 +76,14 @@ __device__ __forceinline__ uint32_t swz(int r, int j)
     return (uint32_t)r * 128u + (uint32_t)((j ^ (r & 7)) << 4);
 }
 
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
 // Rows [0, nalloc) of a bf16 operand image (panels of 64 columns, panel stride
-// nalloc*128 bytes): row r < nrows from rowptr(r), columns [0, ncols); the rest 0.
+// nalloc*128 bytes): row r < nrows from rowptr(r), columns [0, ncols), by 16-byte
+// cp.async copies that are all in flight at once (the caller commits and waits);
+// rows [nrows, nalloc) are zeroed with plain stores.
 template <class RowPtr>
 __device__ __forceinline__ void load_rows_bf16(uint8_t *dst, RowPtr rowptr, int nrows, int nalloc, int ncols,
                                                int tid)
@@ -83,10 +91,17 @@ __device__ __forceinline__ void load_rows_bf16(uint8_t *dst, RowPtr rowptr, int 
     const int gpr = ncols >> 3;
     for (int i = tid; i < nalloc * gpr; i += kThreads) {
         const int r = i / gpr, c8 = i - r * gpr;
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (r < nrows) v = __ldg(reinterpret_cast<const uint4 *>(rowptr(r)) + c8);
-        *reinterpret_cast<uint4 *>(dst + (uint32_t)(c8 >> 3) * (uint32_t)nalloc * 128u + swz(r, c8 & 7)) = v;
+        uint8_t *d = dst + (uint32_t)(c8 >> 3) * (uint32_t)nalloc * 128u + swz(r, c8 & 7);
+        if (r < nrows)
+            ptx::cp_async16(d, reinterpret_cast<const uint4 *>(rowptr(r)) + c8);
+        else
+            *reinterpret_cast<uint4 *>(d) = make_uint4(0, 0, 0, 0);
     }
+}
+__device__ __forceinline__ void cp_async_all_landed()
+{
+    cp_async_commit();
+    cp_async_wait<0>();
 }
 
 // Write 32 consecutive columns [c0, c0 + 32) of row r (values x, converted to
@@ -103,20 +118,6 @@ __device__ __forceinline__ void store_row32_bf16(uint8_t *img, uint32_t pstride,
         v.z = pack_bf16x2(x[8 * q + 4], x[8 * q + 5]);
         v.w = pack_bf16x2(x[8 * q + 6], x[8 * q + 7]);
         *reinterpret_cast<uint4 *>(base + swz(r, j0 + q)) = v;
-    }
-}
-
-__device__ __forceinline__ void load_row_f32(const bf16 *src, int n, float *out)
-{
-    const uint4 *p = reinterpret_cast<const uint4 *>(src);
-    for (int i = 0; i < n / 8; ++i) {
-        const uint4 v = __ldg(p + i);
-        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            out[8 * i + 2 * j] = __uint_as_float(w[j] << 16);
-            out[8 * i + 2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
-        }
     }
 }
 
@@ -187,168 +188,215 @@ RowLayout make_grad_layout(int d, int F, int B)
     return Lr;
 }
 
-// k_block_state: K (128 rows), W, phi(K) (B rows x 2F), [V | 1 | 0] (B rows x (d + 16))
-RowLayout make_state_layout(int d, int F, int B)
-{
-    RowLayout Lr{};
-    uint32_t off = 0;
-    Lr.off_q = off;                                                  // K as the M = 128 operand
-    off += (uint32_t)(d / 64) * 128 * 128;
-    Lr.off_w = off;
-    off += (uint32_t)(F / 64) * d * 128;
-    Lr.off_phi = off;
-    off += (uint32_t)(2 * F / 64) * B * 128;
-    Lr.off_y = off;
-    off += (uint32_t)((d + 16 + 63) / 64) * B * 128;
-    off = (off + 1023) & ~1023u;
-    Lr.off_bar = off;
-    off += 1024;
-    Lr.bytes = off + 1024;
-    return Lr;
-}
-
 __device__ __forceinline__ uint8_t *aligned_smem(uint8_t *raw)
 {
     return reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
 }
 
 // ---------------------------------------------------------------------------
-// k_block_state: dS_m of one (sequence s, block m, state head g) into slot m+1
-// of P and PT.  The CTA of the last block (whose increment no block reads)
-// clears slot 0 instead.
+// k_prefix_states: S_{n-1}, z_{n-1} of every block n of a sequence for one
+// 32-feature slice of one state head, written into slot n of P and PT.  The CTA
+// sweeps the blocks in order with the running slice S^T (row e per thread):
+//                                S^T += V_n^T phi_slice(K_n)  (bf16 MMA, the
+// slice of phi taken from the full-F softmaxes), z += sum_t phi_slice(k_t)
+// (fp32).  Keys are processed min(4, 128 / B) blocks at a time: U = K W for
+// the rows, phi of the slice into a K-major [feature][token] operand, the
+// increments of the group's blocks into their own Tensor Memory columns (one
+// commit), then per block: store the running state (registers, thread = e)
+// into its slot and add the block's increment.
+// Shared memory: W, K rows, V rows (two panels of 64 e, the second zero for
+// d = 64, so that V^T is an M = 128 operand), phi slice, row scratch (in K's
+// space); 107 KB and 256 Tensor Memory columns, so two CTAs share an SM.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads, 1) k_block_state(const __grid_constant__ TrainArgs a, RowLayout Lr)
+struct PrefixLayout {
+    uint32_t off_w, off_k, off_v, off_p, off_x, off_z, off_bar, bytes;
+};
+
+PrefixLayout make_prefix_layout(int d, int F)
+{
+    PrefixLayout Lp{};
+    uint32_t off = 0;
+    Lp.off_w = off;
+    off += (uint32_t)(F / 64) * d * 128;
+    Lp.off_k = off;
+    off += (uint32_t)(d / 64) * 128 * 128;
+    Lp.off_v = off;
+    off += 2u * 128 * 128;
+    Lp.off_p = off;                    // 32 feature rows x 128 tokens (two 64-token panels)
+    off += 2u * 32 * 128;
+    Lp.off_x = Lp.off_k;               // 128 tokens x 32 fp32 (the slice of phi, for z): K is
+                                       // dead once U = K W is formed
+    Lp.off_z = off;                    // running z of the slice and per-block dz (fp32)
+    off += 1024;
+    Lp.off_bar = off;
+    off += 1024;
+    Lp.bytes = off + 1024;
+    return Lp;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) k_prefix_states(const __grid_constant__ TrainArgs a, PrefixLayout Lp)
 {
     using namespace ptx;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = aligned_smem(smem_raw);
     const int tid = threadIdx.x, warp = tid >> 5;
-    const int d = a.d, F = a.F, B = a.B, Hkv = a.Hkv;
-    const int g = blockIdx.x % Hkv, m = (blockIdx.x / Hkv) % a.n_blk, s = blockIdx.x / (Hkv * a.n_blk);
+    const int d = a.d, F = a.F, B = a.B, Hkv = a.Hkv, n_blk = a.n_blk;
+    const int NSL = 2 * F / 32;
+    const int j = blockIdx.x % NSL, g = (blockIdx.x / NSL) % Hkv, s = blockIdx.x / (NSL * Hkv);
+    const bool neg = j >= F / 32;              // slice of phi- features
+    const int fu = (j % (F / 32)) * 32;        // first column of u the slice reads
     const size_t hf = head_floats(d, F);
-    griddep_wait();
-    if (m == a.n_blk - 1) {
-        float4 *p = reinterpret_cast<float4 *>(a.P + ((size_t)s * a.n_blk * Hkv + g) * hf);
-        float4 *pt = reinterpret_cast<float4 *>(a.PT + ((size_t)s * a.n_blk * Hkv + g) * hf);
-        for (size_t i = tid; i < hf / 4; i += kThreads) {
-            p[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-            pt[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-        return;
-    }
-    uint64_t *bar = reinterpret_cast<uint64_t *>(smem + Lr.off_bar);
+    const size_t kv_row = (size_t)Hkv * d;
+    const int GB = min(4, 128 / B);            // blocks per group (at most 128 key rows)
+    uint64_t *bar = reinterpret_cast<uint64_t *>(smem + Lp.off_bar);
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar + 2);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
+    float *dz = reinterpret_cast<float *>(smem + Lp.off_z);   // [GB][32] dz of the group's blocks
+    float *xs = reinterpret_cast<float *>(smem + Lp.off_x);   // [128][32] phi slice of the rows
     if (tid == 0) {
         mbar_init(&bar[0], 1);
         *fail = 0;
         fence_mbar_init();
     }
     if (warp == 0) {
-        tmem_alloc(tmem_holder, 512);
+        tmem_alloc(tmem_holder, 256);
         tmem_relinquish();
     }
-    const size_t t0 = (size_t)s * a.L + (size_t)m * B;
-    const size_t kv_row = (size_t)Hkv * d;
-    // K rows (zero beyond B) as the M = 128 A operand, W, and [V | 1 | 0]
-    load_rows_bf16(smem + Lr.off_q, [&](int r) { return a.K + (t0 + r) * kv_row + (size_t)g * d; }, B, 128, d, tid);
-    load_rows_bf16(smem + Lr.off_w, [&](int r) { return a.W + ((size_t)g * d + r) * F; }, d, d, F, tid);
-    load_rows_bf16(smem + Lr.off_y, [&](int r) { return a.V + (t0 + r) * kv_row + (size_t)g * d; }, B, B, d, tid);
-    {
-        const uint32_t pstride = (uint32_t)B * 128;
-        for (int r = tid; r < B; r += kThreads) {
-            uint8_t *base = smem + Lr.off_y + (uint32_t)(d >> 6) * pstride;
-            *reinterpret_cast<uint4 *>(base + swz(r, 0)) = make_uint4(0x3F80u, 0, 0, 0);   // bf16 1.0 in column d
-            *reinterpret_cast<uint4 *>(base + swz(r, 1)) = make_uint4(0, 0, 0, 0);
-        }
-    }
-    fence_proxy_async_smem();
+    // the second 64-e panel of V^T stays zero for d = 64
+    if (d == 64)
+        for (int i = tid; i < 1024; i += kThreads)
+            reinterpret_cast<uint4 *>(smem + Lp.off_v + 128 * 128)[i] = make_uint4(0, 0, 0, 0);
+    griddep_wait();
+    load_rows_bf16(smem + Lp.off_w, [&](int r) { return a.W + ((size_t)g * d + r) * F; }, d, d, F, tid);
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
     const uint32_t lane_off = (uint32_t)(warp & 3) * 32u << 16;
+    constexpr uint32_t kAcc = 128;             // the group's dS^T slices: columns [128, 128 + 32 GB)
+    uint32_t phase = 0;
     bool ok = true;
-    if (tid == 0) {
-        const uint32_t q_u = smem_u32(smem + Lr.off_q), w_u = smem_u32(smem + Lr.off_w);
-        const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
-        for (int k = 0; k < d / 16; ++k)
-            mma_bf16_ss(tmem + kColU, smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B),
-                        smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B), idU, k > 0);
-        mma_commit(&bar[0]);
-    }
-    ok = wait_bar(&bar[0], 0, fail);
-    tc_fence_after();
-    // phi(K) of row tid into the MN-major operand [token][feature]
-    {
-        const PhiStats st = phi_stats(tmem + lane_off + kColU, F);
-        const float ip = 1.f / st.sp, in = 1.f / st.sn;
-        float x[32], yp[32], yn[32];
-        for (int j = 0; j < F / 32; ++j) {
-            tmem_ld32(tmem + lane_off + kColU + 32 * j, x);
+    float run[32];                             // S_{n-1}^T slice, row e = tid (e < d)
+#pragma unroll
+    for (int k = 0; k < 32; ++k) run[k] = 0.f;
+    float zc = 0.f;                            // z_{n-1} of feature 32 j + tid (tid < 32)
+    const uint32_t w_u = smem_u32(smem + Lp.off_w), k_u = smem_u32(smem + Lp.off_k),
+                   v_u = smem_u32(smem + Lp.off_v), p_u = smem_u32(smem + Lp.off_p);
+    for (int b0 = 0; b0 < n_blk && ok; b0 += GB) {
+        const int nb = min(GB, n_blk - b0), nt = nb * B;
+        const size_t t0 = (size_t)s * a.L + (size_t)b0 * B;
+        load_rows_bf16(smem + Lp.off_k, [&](int r) { return a.K + (t0 + r) * kv_row + (size_t)g * d; }, nt, 128, d,
+                       tid);
+        load_rows_bf16(smem + Lp.off_v, [&](int r) { return a.V + (t0 + r) * kv_row + (size_t)g * d; }, nt, 128, d,
+                       tid);
+        cp_async_all_landed();
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+        if (tid == 0) {
+            const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
+            for (int k = 0; k < d / 16; ++k)
+                mma_bf16_ss(tmem, smem_desc(k_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B),
+                            smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B), idU, k > 0);
+            mma_commit(&bar[0]);
+        }
+        ok = wait_bar(&bar[0], phase & 1u, fail);
+        ++phase;
+        tc_fence_after();
+        // the slice of phi of row tid (full-F softmax statistics), bf16 into the
+        // [feature][token] operand and fp32 into the row scratch
+        {
+            const PhiStats st = phi_stats(tmem + lane_off, F);
+            const float inv = 1.f / (neg ? st.sn : st.sp);
+            float x[32];
+            tmem_ld32(tmem + lane_off + (uint32_t)fu, x);
             tmem_wait_ld();
+            const bool valid = tid < nt;
 #pragma unroll
             for (int k = 0; k < 32; ++k) {
-                yp[k] = ex2((x[k] - st.mp) * kLog2e) * ip;
-                yn[k] = ex2((st.mn - x[k]) * kLog2e) * in;
-            }
-            if (tid < B) {
-                store_row32_bf16(smem + Lr.off_phi, (uint32_t)B * 128, tid, 32 * j, yp);
-                store_row32_bf16(smem + Lr.off_phi, (uint32_t)B * 128, tid, F + 32 * j, yn);
+                const float ph = valid ? ex2((neg ? (st.mn - x[k]) : (x[k] - st.mp)) * kLog2e) * inv : 0.f;
+                xs[tid * 32 + ((k + tid) & 31)] = ph;   // rotated: conflict-free across the warp
+                const __nv_bfloat16 hb = __float2bfloat16_rn(ph);
+                uint8_t *row = smem + Lp.off_p + (uint32_t)(tid >> 6) * (32 * 128) + (uint32_t)k * 128u;
+                *reinterpret_cast<__nv_bfloat16 *>(row + (((((tid & 63) >> 3) ^ (k & 7))) << 4) + (tid & 7) * 2) = hb;
             }
         }
-    }
-    fence_proxy_async_smem();
-    tc_fence_before();
-    if (group_sync_failed(1, kThreads, !ok)) {
-        if (tid == 0) raise_error(a.err, ERR_WAIT_TIMEOUT);
+        fence_proxy_async_smem();
+        tc_fence_before();
         __syncthreads();
-        if (warp == 0) tmem_dealloc(tmem, 512);
-        return;
-    }
-    tc_fence_after();
-    // accumulator block i (features 128 i ..) at column i * NYS, NYS = NY rounded up to 32
-    const int NY = d + 16, NYS = (NY + 31) & ~31, NM = 2 * F / 128;
-    if (tid == 0) {
-        const uint32_t p_u = smem_u32(smem + Lr.off_phi), y_u = smem_u32(smem + Lr.off_y);
-        const uint32_t idDS = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, NY);
-        for (int i = 0; i < NM; ++i)
-            for (int ks = 0; ks < B / 16; ++ks)
-                mma_bf16_ss(tmem + kColDR + (uint32_t)(i * NYS),
-                            smem_desc(p_u + (uint32_t)(2 * i) * B * 128 + ks * 2048, B * 128, 1024, SWZ_128B),
-                            smem_desc(y_u + ks * 2048, B * 128, 1024, SWZ_128B), idDS, ks > 0);
-        mma_commit(&bar[0]);
-    }
-    ok = wait_bar(&bar[0], 1, fail);
-    tc_fence_after();
-    if (ok) {
-        // lane tid of M-block i is feature f = 128 i + tid: row f of dS (d values) and dz[f]
-        const size_t slot = ((size_t)s * a.n_blk + m + 1) * Hkv + g;
-        float *P = a.P + slot * hf, *PT = a.PT + slot * hf;
-        for (int i = 0; i < NM; ++i) {
-            const int f = 128 * i + tid;
-            float x[32];
-            for (int c = 0; c < d / 32; ++c) {
-                tmem_ld32(tmem + lane_off + kColDR + (uint32_t)(i * NYS + 32 * c), x);
-                tmem_wait_ld();
-                float4 *row = reinterpret_cast<float4 *>(PT + (size_t)c * 64 * F + (size_t)f * 32);
-#pragma unroll
-                for (int q = 0; q < 8; ++q) row[q ^ (f & 7)] = make_float4(x[4 * q], x[4 * q + 1], x[4 * q + 2], x[4 * q + 3]);
-#pragma unroll
-                for (int k = 0; k < 32; ++k) P[s_offset(f, 32 * c + k, d)] = x[k];
-            }
-            float zz[16];
-            tmem_ld16(tmem + lane_off + kColDR + (uint32_t)(i * NYS + d), zz);
-            tmem_wait_ld();
-            P[z_offset(f, d, F)] = zz[0];
-            PT[z_offset(f, d, F)] = zz[0];
+        tc_fence_after();
+        // dz of each block of the group: sum over its B rows, feature tid % 32
+        for (int q = tid; q < nb * 32; q += kThreads) {
+            const int bl = q >> 5, f = q & 31;
+            float acc = 0.f;
+            for (int t = bl * B; t < bl * B + B; ++t) acc += xs[t * 32 + ((f + t) & 31)];
+            dz[bl * 32 + f] = acc;
         }
-    } else if (tid == 0) {
-        raise_error(a.err, ERR_WAIT_TIMEOUT);
+        __syncthreads();
+        // the group's increments dS_n = V_n^T phi_slice(K_n), block bl into columns
+        // [128 + 32 bl, 160 + 32 bl) (not those of the sequence's last block)
+        if (tid == 0) {
+            const uint32_t idS = instr_desc(FMT_BF16, FMT_BF16, true, false, 128, 32);
+            for (int bl = 0; bl < nb; ++bl) {
+                if (b0 + bl == n_blk - 1) break;
+                for (int ks = 0; ks < B / 16; ++ks) {
+                    const int tk = bl * B + 16 * ks;   // first token row of this k-step
+                    mma_bf16_ss(tmem + kAcc + 32u * bl,
+                                smem_desc(v_u + (uint32_t)(tk / 16) * 2048, 128 * 128, 1024, SWZ_128B),
+                                smem_desc(p_u + (uint32_t)(tk >> 6) * (32 * 128) + (uint32_t)(tk & 63) * 2, 16, 1024,
+                                          SWZ_128B),
+                                idS, ks > 0 ? 1u : 0u);
+                }
+            }
+            mma_commit(&bar[0]);
+        }
+        ok = wait_bar(&bar[0], phase & 1u, fail);
+        ++phase;
+        tc_fence_after();
+        if (group_sync_failed(1, kThreads, !ok)) {
+            ok = false;
+            break;
+        }
+        for (int bl = 0; bl < nb; ++bl) {
+            const int n = b0 + bl;
+            // slot n holds S_{n-1} (the running slice, in registers) and z_{n-1}
+            const size_t slot = ((size_t)s * n_blk + n) * Hkv + g;
+            float *P = a.P + slot * hf, *PT = a.PT + slot * hf;
+            const int e = tid;
+            if (e < d) {
+                // decode image: tile j, row e (32 features, granules permuted by e mod 8)
+                float4 *row = reinterpret_cast<float4 *>(P + (size_t)j * 32 * d + (size_t)e * 32);
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    row[q ^ (e & 7)] = make_float4(run[4 * q], run[4 * q + 1], run[4 * q + 2], run[4 * q + 3]);
+                // feature-row image: rows f = 32 j + k, column e of e-tile e / 32
+                float *pt = PT + (size_t)(e >> 5) * 64 * F + (size_t)(32 * j) * 32 + (e & 3);
+#pragma unroll
+                for (int k = 0; k < 32; ++k) pt[(size_t)k * 32 + (size_t)((((e & 31) >> 2) ^ (k & 7)) << 2)] = run[k];
+            }
+            if (tid < 32) {
+                P[z_offset(32 * j + tid, d, F)] = zc;
+                PT[z_offset(32 * j + tid, d, F)] = zc;
+                zc += dz[bl * 32 + tid];
+            }
+            if (n == n_blk - 1) break;
+            if (e < d) {
+                float x[32];
+                tmem_ld32(tmem + lane_off + kAcc + 32u * bl, x);
+                tmem_wait_ld();
+#pragma unroll
+                for (int k = 0; k < 32; ++k) run[k] += x[k];
+            }
+        }
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
     }
+    if (!ok && tid == 0) raise_error(a.err, ERR_WAIT_TIMEOUT);
     tc_fence_before();
     __syncthreads();
     griddep_launch_dependents();
-    if (warp == 0) tmem_dealloc(tmem, 512);
+    if (warp == 0) tmem_dealloc(tmem, 256);
 }
 
 // ---------------------------------------------------------------------------
@@ -440,6 +488,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
     }
     load_rows_bf16(smem + Lr.off_w, [&](int r) { return a.W + ((size_t)g * d + r) * F; }, d, d, F, tid);
     for (int f = tid; f < 2 * F; f += kThreads) sZ[f] = src[z_offset(f, d, F)];
+    cp_async_all_landed();
     fence_proxy_async_smem();
     __syncthreads();
     tc_fence_after();
@@ -510,24 +559,29 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         }
         // scores, shift c, D' = w sum_j e^(s_j - c) + lin_den e^(-c)  (D = e^c D')
         const float scale = rsqrtf((float)d);
-        float sc[64];
         float m = -INFINITY;
         for (int j = 0; j < B / 16; ++j) {
             float x[16];
             tmem_ld16(tl + kColS + 16 * j, x);
             tmem_wait_ld();
 #pragma unroll
-            for (int k = 0; k < 16; ++k) {
-                sc[16 * j + k] = x[k] * scale;
-                m = fmaxf(m, sc[16 * j + k]);
-            }
+            for (int k = 0; k < 16; ++k) m = fmaxf(m, x[k] * scale);
         }
         float c = m;
         if (lin_den > 0.f) c = w > 0.f ? fmaxf(m, logf(lin_den) - logf(w)) : logf(lin_den);
-        float l = 0.f;
-        for (int j = 0; j < B; ++j) {
-            sc[j] = ex2((sc[j] - c) * kLog2e);
-            l += sc[j];
+        // l = sum_j e^(s_j - c), an = sum_j e^(s_j - c) g.v_j
+        float l = 0.f, an = 0.f;
+        for (int j = 0; j < B / 16; ++j) {
+            float x[16], y[16];
+            tmem_ld16(tl + kColS + 16 * j, x);
+            tmem_ld16(tl + kColGv + 16 * j, y);
+            tmem_wait_ld();
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+                const float e = ex2((x[k] * scale - c) * kLog2e);
+                l += e;
+                an += e * y[k];
+            }
         }
         const float ec = ex2(-c * kLog2e);
         const float Dp = w * l + lin_den * ec;
@@ -535,41 +589,51 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         const float pw = valid ? 1.f / Dp : 0.f;  // e^(s_j - c) / D' = e^(s_j) / D
         beta = l * pw;
         lambda = lin_den * inv;
-        // A = sum_j (e^(s_j) / D) g.v_j
-        for (int j = 0; j < B / 16; ++j) {
-            float x[16];
-            tmem_ld16(tl + kColGv + 16 * j, x);
-            tmem_wait_ld();
+        A = an * pw;                              // sum_j (e^(s_j) / D) g.v_j
+        // dN = g / D: Tensor Memory (fp32, A operand of S dN) and the operand image (bf16);
+        // the row's d values are loaded at once (16 x 16 bytes in flight)
+        const uint4 *grow = reinterpret_cast<const uint4 *>(a.dO + (t0 + tid % B) * q_row + (size_t)(g * G + hl) * d);
+        uint4 graw[16];
 #pragma unroll
-            for (int k = 0; k < 16; ++k) A += sc[16 * j + k] * pw * x[k];
-        }
-        // dN = g / D: Tensor Memory (fp32, A operand of S dN) and the operand image (bf16)
-        const bf16 *grow = a.dO + (t0 + tid % B) * q_row + (size_t)(g * G + hl) * d;
-        float gv[32];
-        for (int c0 = 0; c0 < d; c0 += 32) {
-            if (valid) {
-                load_row_f32(grow + c0, 32, gv);
+        for (int i = 0; i < 16; ++i) graw[i] = (valid && i < d / 8) ? __ldg(grow + i) : make_uint4(0, 0, 0, 0);
 #pragma unroll
-                for (int k = 0; k < 32; ++k) gv[k] *= inv;
-            } else {
+        for (int c = 0; c < 4; ++c) {
+            if (c < d / 32) {
+                float gv[32];
 #pragma unroll
-                for (int k = 0; k < 32; ++k) gv[k] = 0.f;
+                for (int i = 0; i < 4; ++i) {
+                    const uint32_t w4[4] = {graw[4 * c + i].x, graw[4 * c + i].y, graw[4 * c + i].z, graw[4 * c + i].w};
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        gv[8 * i + 2 * j] = __uint_as_float(w4[j] << 16) * inv;
+                        gv[8 * i + 2 * j + 1] = __uint_as_float(w4[j] & 0xFFFF0000u) * inv;
+                    }
+                }
+                tmem_st32(tl + kColY + 32 * c, gv);
+                store_row32_bf16(smem + Lr.off_y, 128 * 128, tid, 32 * c, gv);
             }
-            tmem_st32(tl + kColY + c0, gv);
-            store_row32_bf16(smem + Lr.off_y, 128 * 128, tid, c0, gv);
         }
     } else {
         // V rows (fp32) as the Tensor Memory A operand of R v; r enters with coefficient 1
-        const bf16 *vrow = a.V + (t0 + tid) * kv_row + (size_t)g * d;
-        float vv[32];
-        for (int c0 = 0; c0 < d; c0 += 32) {
-            if (valid) {
-                load_row_f32(vrow + c0, 32, vv);
-            } else {
+        const uint4 *vrow = reinterpret_cast<const uint4 *>(a.V + (t0 + tid) * kv_row + (size_t)g * d);
+        uint4 vraw[16];
 #pragma unroll
-                for (int k = 0; k < 32; ++k) vv[k] = 0.f;
+        for (int i = 0; i < 16; ++i) vraw[i] = (valid && i < d / 8) ? __ldg(vrow + i) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            if (c < d / 32) {
+                float vv[32];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const uint32_t w4[4] = {vraw[4 * c + i].x, vraw[4 * c + i].y, vraw[4 * c + i].z, vraw[4 * c + i].w};
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        vv[8 * i + 2 * j] = __uint_as_float(w4[j] << 16);
+                        vv[8 * i + 2 * j + 1] = __uint_as_float(w4[j] & 0xFFFF0000u);
+                    }
+                }
+                tmem_st32(tl + kColY + 32 * c, vv);
             }
-            tmem_st32(tl + kColY + c0, vv);
         }
     }
     tmem_wait_st();
@@ -785,12 +849,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwAr
     const uint32_t tmem = *tmem_holder;
     const uint32_t idW = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, F);
     bool ok = true;
-    for (int k = 0; k < n_tiles; ++k) {
-        const int stg = k & 1;
-        if (k >= 2) ok = wait_bar(&bars[stg], (uint32_t)((k - 2) >> 1) & 1u, fail) && ok;
-        if (group_sync_failed(1, kThreads, !ok)) break;
-        uint8_t *sx = smem + stg * stage, *su = sx + xbytes;
-        // row tid of this step
+    // copies of step k into stage k & 1: row tid of the step (16-byte cp.async, one group per step)
+    auto issue = [&](int k) {
+        uint8_t *sx = smem + (k & 1) * stage, *su = sx + xbytes;
         const long long rho = r_begin + (long long)k * 128 + tid;
         const bool valid = rho < r_end;
         const bf16 *xr = nullptr, *ur = nullptr;
@@ -807,24 +868,43 @@ __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwAr
             }
         }
         for (int c8 = 0; c8 < d / 8; ++c8) {
-            const uint4 v = valid ? __ldg(reinterpret_cast<const uint4 *>(xr) + c8) : make_uint4(0, 0, 0, 0);
-            *reinterpret_cast<uint4 *>(sx + (uint32_t)(c8 >> 3) * (128 * 128) + swz(tid, c8 & 7)) = v;
+            uint8_t *dst = sx + (uint32_t)(c8 >> 3) * (128 * 128) + swz(tid, c8 & 7);
+            if (valid)
+                cp_async16(dst, reinterpret_cast<const uint4 *>(xr) + c8);
+            else
+                *reinterpret_cast<uint4 *>(dst) = make_uint4(0, 0, 0, 0);
         }
         for (int c8 = 0; c8 < F / 8; ++c8) {
-            const uint4 v = valid ? __ldg(reinterpret_cast<const uint4 *>(ur) + c8) : make_uint4(0, 0, 0, 0);
-            *reinterpret_cast<uint4 *>(su + (uint32_t)(c8 >> 3) * (128 * 128) + swz(tid, c8 & 7)) = v;
+            uint8_t *dst = su + (uint32_t)(c8 >> 3) * (128 * 128) + swz(tid, c8 & 7);
+            if (valid)
+                cp_async16(dst, reinterpret_cast<const uint4 *>(ur) + c8);
+            else
+                *reinterpret_cast<uint4 *>(dst) = make_uint4(0, 0, 0, 0);
+        }
+        cp_async_commit();
+    };
+    if (n_tiles > 0) issue(0);
+    for (int k = 0; k < n_tiles; ++k) {
+        if (k + 1 < n_tiles) {
+            // stage (k + 1) & 1 was last read by the MMAs of step k - 1
+            if (k >= 1) ok = wait_bar(&bars[(k + 1) & 1], (uint32_t)((k - 1) >> 1) & 1u, fail) && ok;
+            issue(k + 1);
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
         }
         fence_proxy_async_smem();
-        __syncthreads();
+        if (group_sync_failed(1, kThreads, !ok)) break;
         if (tid == 0) {
             tc_fence_after();
-            const uint32_t x_u = smem_u32(sx), u_u = smem_u32(su);
+            const uint32_t x_u = smem_u32(smem + (k & 1) * stage), u_u = x_u + xbytes;
             for (int ks = 0; ks < 8; ++ks)
                 mma_bf16_ss(tmem, smem_desc(x_u + ks * 2048, 128 * 128, 1024, SWZ_128B),
                             smem_desc(u_u + ks * 2048, 128 * 128, 1024, SWZ_128B), idW, (k | ks) != 0);
-            mma_commit(&bars[stg]);
+            mma_commit(&bars[k & 1]);
         }
     }
+    cp_async_wait<0>();
     // the last one or two steps
     for (int k = n_tiles - 2; k < n_tiles; ++k)
         if (k >= 0) ok = wait_bar(&bars[k & 1], (uint32_t)(k >> 1) & 1u, fail) && ok;
@@ -975,13 +1055,10 @@ cudaError_t launch_train_states(const hybrid_cfg &c, const void *K, const void *
     cudaError_t e = cudaSuccess;
     k_slot_ptrs<<<(slots + 255) / 256, 256, 0, st>>>(w.P, slots, sf, w.ptrs);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    const RowLayout Ls = make_state_layout(a.d, a.F, a.B);
-    if ((e = opt_in(k_block_state, g_opt_state)) != cudaSuccess) return e;
-    e = launch_pdl(k_block_state, dim3((unsigned)(slots * a.Hkv)), dim3(kThreads), Ls.bytes, st, a, Ls);
-    if (e != cudaSuccess) return e;
-    const size_t n4 = sf / 4 * (size_t)n_seq;
-    return launch_pdl(k_slot_scan, dim3((unsigned)((n4 + 255) / 256), 2), dim3(256), 0, st, w.P, w.PT, n_seq,
-                      a.n_blk, sf, false);
+    const PrefixLayout Lp = make_prefix_layout(a.d, a.F);
+    if ((e = opt_in(k_prefix_states, g_opt_state)) != cudaSuccess) return e;
+    return launch_pdl(k_prefix_states, dim3((unsigned)(n_seq * a.Hkv * (2 * a.F / 32))), dim3(kThreads), Lp.bytes,
+                      st, a, Lp);
 }
 
 cudaError_t launch_train_backward(const hybrid_cfg &c, const void *Q, const void *K, const void *V, const void *W,
