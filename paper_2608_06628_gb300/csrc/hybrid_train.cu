@@ -81,19 +81,19 @@ template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 // Rows [0, nalloc) of a bf16 operand image (panels of 64 columns, panel stride
-// nalloc*128 bytes): row r < nrows from rowptr(r), columns [0, ncols), by 16-byte
+// nalloc*128 bytes): row r from rowptr(r), columns [0, ncols), by 16-byte
 // cp.async copies that are all in flight at once (the caller commits and waits);
-// rows [nrows, nalloc) are zeroed with plain stores.
+// rows whose rowptr is null are zeroed with plain stores.
 template <class RowPtr>
-__device__ __forceinline__ void load_rows_bf16(uint8_t *dst, RowPtr rowptr, int nrows, int nalloc, int ncols,
-                                               int tid)
+__device__ __forceinline__ void load_rows_bf16(uint8_t *dst, RowPtr rowptr, int nalloc, int ncols, int tid)
 {
     const int gpr = ncols >> 3;
     for (int i = tid; i < nalloc * gpr; i += kThreads) {
         const int r = i / gpr, c8 = i - r * gpr;
         uint8_t *d = dst + (uint32_t)(c8 >> 3) * (uint32_t)nalloc * 128u + swz(r, c8 & 7);
-        if (r < nrows)
-            ptx::cp_async16(d, reinterpret_cast<const uint4 *>(rowptr(r)) + c8);
+        const bf16 *src = rowptr(r);
+        if (src)
+            ptx::cp_async16(d, reinterpret_cast<const uint4 *>(src) + c8);
         else
             *reinterpret_cast<uint4 *>(d) = make_uint4(0, 0, 0, 0);
     }
@@ -267,7 +267,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefix_states(const __grid_cons
         for (int i = tid; i < 1024; i += kThreads)
             reinterpret_cast<uint4 *>(smem + Lp.off_v + 128 * 128)[i] = make_uint4(0, 0, 0, 0);
     griddep_wait();
-    load_rows_bf16(smem + Lp.off_w, [&](int r) { return a.W + ((size_t)g * d + r) * F; }, d, d, F, tid);
+    load_rows_bf16(smem + Lp.off_w, [&](int r) { return a.W + ((size_t)g * d + r) * F; }, d, F, tid);
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
@@ -284,10 +284,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefix_states(const __grid_cons
     for (int b0 = 0; b0 < n_blk && ok; b0 += GB) {
         const int nb = min(GB, n_blk - b0), nt = nb * B;
         const size_t t0 = (size_t)s * a.L + (size_t)b0 * B;
-        load_rows_bf16(smem + Lp.off_k, [&](int r) { return a.K + (t0 + r) * kv_row + (size_t)g * d; }, nt, 128, d,
-                       tid);
-        load_rows_bf16(smem + Lp.off_v, [&](int r) { return a.V + (t0 + r) * kv_row + (size_t)g * d; }, nt, 128, d,
-                       tid);
+        auto krow = [&](int r) -> const bf16 * { return r < nt ? a.K + (t0 + r) * kv_row + (size_t)g * d : nullptr; };
+        auto vrow = [&](int r) -> const bf16 * { return r < nt ? a.V + (t0 + r) * kv_row + (size_t)g * d : nullptr; };
+        load_rows_bf16(smem + Lp.off_k, krow, 128, d, tid);
+        load_rows_bf16(smem + Lp.off_v, vrow, 128, d, tid);
         cp_async_all_landed();
         fence_proxy_async_smem();
         tc_fence_before();
@@ -448,7 +448,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
     const int tid = threadIdx.x, warp = tid >> 5;
     const int d = a.d, F = a.F, B = a.B, Hkv = a.Hkv, Hq = a.Hq, G = Hq / Hkv;
     const int g = blockIdx.x % Hkv, n = (blockIdx.x / Hkv) % a.n_blk, s = blockIdx.x / (Hkv * a.n_blk);
+    // The tile's rows (G*B query rows or B key rows) are spread evenly over the four
+    // 32-lane quadrants of Tensor Memory, so that all four warps share the per-row
+    // math: lane r = 32 q + i holds row q * rpq + i if i < rpq (rpq = rows / 4).
     const int rows = kQuery ? G * B : B;
+    const int rpq = rows / 4;
+    auto row_of = [&](int r) -> int { return (r & 31) < rpq ? (r >> 5) * rpq + (r & 31) : -1; };
     const size_t hf = head_floats(d, F);
     const size_t t0 = (size_t)s * a.L + (size_t)n * B;
     const size_t kv_row = (size_t)Hkv * d, q_row = (size_t)Hq * d;
@@ -477,16 +482,28 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
 
     // phase one: operands of [U | scores] = Q [W | K^T] and dO V^T (query side) or U = K W
     if (kQuery) {
-        auto qrow = [&](int r) { return a.Q + (t0 + r % B) * q_row + (size_t)(g * G + r / B) * d; };
-        auto dorow = [&](int r) { return a.dO + (t0 + r % B) * q_row + (size_t)(g * G + r / B) * d; };
-        load_rows_bf16(smem + Lr.off_q, qrow, rows, 128, d, tid);
-        load_rows_bf16(smem + Lr.off_do, dorow, rows, 128, d, tid);
-        load_rows_bf16(smem + Lr.off_k, [&](int r) { return a.K + (t0 + r) * kv_row + (size_t)g * d; }, B, B, d, tid);
-        load_rows_bf16(smem + Lr.off_v, [&](int r) { return a.V + (t0 + r) * kv_row + (size_t)g * d; }, B, B, d, tid);
+        auto qrow = [&](int r) -> const bf16 * {
+            const int q = row_of(r);
+            return q < 0 ? nullptr : a.Q + (t0 + q % B) * q_row + (size_t)(g * G + q / B) * d;
+        };
+        auto dorow = [&](int r) -> const bf16 * {
+            const int q = row_of(r);
+            return q < 0 ? nullptr : a.dO + (t0 + q % B) * q_row + (size_t)(g * G + q / B) * d;
+        };
+        load_rows_bf16(smem + Lr.off_q, qrow, 128, d, tid);
+        load_rows_bf16(smem + Lr.off_do, dorow, 128, d, tid);
+        load_rows_bf16(smem + Lr.off_k, [&](int r) -> const bf16 * { return a.K + (t0 + r) * kv_row + (size_t)g * d; },
+                       B, d, tid);
+        load_rows_bf16(smem + Lr.off_v, [&](int r) -> const bf16 * { return a.V + (t0 + r) * kv_row + (size_t)g * d; },
+                       B, d, tid);
     } else {
-        load_rows_bf16(smem + Lr.off_q, [&](int r) { return a.K + (t0 + r) * kv_row + (size_t)g * d; }, B, 128, d, tid);
+        auto krow = [&](int r) -> const bf16 * {
+            const int q = row_of(r);
+            return q < 0 ? nullptr : a.K + (t0 + q) * kv_row + (size_t)g * d;
+        };
+        load_rows_bf16(smem + Lr.off_q, krow, 128, d, tid);
     }
-    load_rows_bf16(smem + Lr.off_w, [&](int r) { return a.W + ((size_t)g * d + r) * F; }, d, d, F, tid);
+    load_rows_bf16(smem + Lr.off_w, [&](int r) -> const bf16 * { return a.W + ((size_t)g * d + r) * F; }, d, F, tid);
     for (int f = tid; f < 2 * F; f += kThreads) sZ[f] = src[z_offset(f, d, F)];
     cp_async_all_landed();
     fence_proxy_async_smem();
@@ -528,8 +545,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
     }
 
     // ---- row statistics (thread = row) ----
-    const bool valid = tid < rows;
-    const int hl = kQuery ? tid / B : 0;
+    const int myrow = row_of(tid);
+    const bool valid = myrow >= 0;
+    const int hl = (kQuery && valid) ? myrow / B : 0;              // query head within the group
+    const int tok = valid ? (kQuery ? myrow % B : myrow) : 0;      // token within the block
     const PhiStats st = phi_stats(tl + kColU, F);
     const float ip = 1.f / st.sp, in = 1.f / st.sn;
     // Query rows: w, 1/D, and the merge terms A = g.sm_num / D, beta = sm_den / D,
@@ -592,7 +611,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         A = an * pw;                              // sum_j (e^(s_j) / D) g.v_j
         // dN = g / D: Tensor Memory (fp32, A operand of S dN) and the operand image (bf16);
         // the row's d values are loaded at once (16 x 16 bytes in flight)
-        const uint4 *grow = reinterpret_cast<const uint4 *>(a.dO + (t0 + tid % B) * q_row + (size_t)(g * G + hl) * d);
+        const uint4 *grow = reinterpret_cast<const uint4 *>(a.dO + (t0 + tok) * q_row + (size_t)(g * G + hl) * d);
         uint4 graw[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) graw[i] = (valid && i < d / 8) ? __ldg(grow + i) : make_uint4(0, 0, 0, 0);
@@ -615,7 +634,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         }
     } else {
         // V rows (fp32) as the Tensor Memory A operand of R v; r enters with coefficient 1
-        const uint4 *vrow = reinterpret_cast<const uint4 *>(a.V + (t0 + tid) * kv_row + (size_t)g * d);
+        const uint4 *vrow = reinterpret_cast<const uint4 *>(a.V + (t0 + tok) * kv_row + (size_t)g * d);
         uint4 vraw[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) vraw[i] = (valid && i < d / 8) ? __ldg(vrow + i) : make_uint4(0, 0, 0, 0);
@@ -722,8 +741,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
                 du[k] = pp * (g1 - dotp) - pn * (g2 - dotn);
             }
             if (valid) {
-                bf16 *out = kQuery ? a.dUq + ((t0 + tid % B) * Hq + (size_t)(g * G + hl)) * F
-                                   : a.dUk + ((t0 + tid) * Hkv + (size_t)g) * F;
+                bf16 *out = kQuery ? a.dUq + ((t0 + tok) * Hq + (size_t)(g * G + hl)) * F
+                                   : a.dUk + ((t0 + tok) * Hkv + (size_t)g) * F;
                 uint4 *o4 = reinterpret_cast<uint4 *>(out + 32 * j);
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
@@ -749,7 +768,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
             const uint32_t p_u = smem_u32(smem + Lr.off_phi), y_u = smem_u32(smem + Lr.off_y);
             const uint32_t idDR = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, NY);
             for (int i = 0; i < NM; ++i)
-                for (int ks = 0; ks < rows / 16; ++ks)
+                for (int ks = 0; ks < 8; ++ks)   // all 128 lanes (rows of unused lanes are zero)
                     mma_bf16_ss(tmem + kColDR + (uint32_t)(i * NYS),
                                 smem_desc(p_u + (uint32_t)(2 * i) * 128 * 128 + ks * 2048, 128 * 128, 1024, SWZ_128B),
                                 smem_desc(y_u + ks * 2048, 128 * 128, 1024, SWZ_128B), idDR, ks > 0);
