@@ -17,8 +17,9 @@
 //   warp 1     MMA issuer (one thread); owns the Tensor Memory allocation.
 //   warp 2     producer: TMA of Q and W, the transposed key tile K^T (built by
 //              the warp from global memory) and V, one unit ahead.
-//   warp 3     storer: TMA stores of the output tile and, with the commit, bulk
-//              reduce-adds of the dS^T tiles into the state, and the store of z.
+//   warp 3     storer (commit): bulk reduce-adds of the dS^T tiles into the state,
+//              the store of z, and TMA stores of the output tile (the step's math
+//              warps store the output from registers).
 //   warps 4-11 math: two threads per query row (one per TMEM lane and "part");
 //              a part owns every other 32-feature chunk of each half of phi.
 //
@@ -87,6 +88,7 @@ constexpr uint32_t kCmEK = 320;
 struct FusedArgs {
     CUtensorMap tmQ, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
     const bf16 *K;
+    bf16 *O;                          // step: the output is stored from registers
     const float *alpha;
     void *const *states;
     unsigned *err;
@@ -162,13 +164,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     const int d = a.d, F = a.F, B = a.B, G = a.G, NS = a.NS;
     const int NCH = F / 32;          // 32-feature chunks (state tiles) per half of phi
     const int NC = 2 * NCH;          // state tiles per unit
-    // the output tile is staged in the slots of tiles ocm, ocm + 1 of its unit:
-    // with the commit, the first two second-half tiles (their increments are
+    // with the commit the output tile is staged in the slots of tiles ocm, ocm + 1
+    // of its unit: the first two second-half tiles (their increments are
     // reduce-added before the epilogue), so the next unit's first-half tiles,
     // needed first, can enter the ring early; if a unit has more tiles than the
-    // ring, first-half tiles that no later tile of the unit reuses; without the
-    // commit, the last two
-    const int ocm = kCommit ? (NC > NS ? NC - NS : NCH) : NC - 2;
+    // ring, first-half tiles that no later tile of the unit reuses
+    const int ocm = NC > NS ? NC - NS : NCH;
     const uint32_t chunk_bytes = (uint32_t)d * 128;
     const int per = a.n_units / (int)gridDim.x, rem = a.n_units % (int)gridDim.x;
     const int u_begin = (int)blockIdx.x * per + min((int)blockIdx.x, rem);
@@ -345,7 +346,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     for (int c = NCH; c < NC; ++c) {
                         const int slot = readout(T + 128, T + 32 * (c - NCH), iq + c);
                         if (slot < 0) return false;
-                        if (c < ocm) mma_commit(&empty[slot]);
+                        mma_commit(&empty[slot]);
                     }
                     mma_commit(&dready[ik & 1]);
                     return true;
@@ -481,7 +482,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         }
     } else if (warp == 3) {
         // --------------------------------------------------------------- storer
-        if (lane == 0) {
+        // (commit only: the step's math warps store the output themselves)
+        if (kCommit && lane == 0) {
             uint32_t q = 0, kp = 0;
             for (int u = u_begin; u < u_end; ++u) {
                 float *Sg = unit_state(a, u);
@@ -560,14 +562,39 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                            : group_sync_failed(pair_bar, 64, local_fail);
         };
 
-        // out = D / den, staged as the TMA box image in the unit's held-back ring
-        // slots (row i = t*G + hh, 128-byte swizzle)
-        auto epilogue = [&](uint32_t ek, uint32_t eq, float inv) -> bool {
+        // out = D / den.  Commit: staged as the TMA box image in the unit's held-back
+        // ring slots (row i = t*G + hh, 128-byte swizzle) for the storer.  Step: stored
+        // from registers (each thread 16-byte runs of its row's d/2 columns), so every
+        // ring slot is free as soon as its readout has run and the next unit's last
+        // tiles do not wait for this unit's output.
+        auto epilogue = [&](uint32_t ek, uint32_t eq, float inv, int eu) -> bool {
             const uint32_t dcol = kCommit ? kCmD : (ek & 1) * 256 + 128;
             bool ok = wait_bar(&dready[ek & 1], (ek >> 1) & 1u, fail);
             if (kCommit && ok) ok = wait_bar(ofree, ek & 1u, fail);
             tc_fence_after();
             const int dh = d / 2;
+            if (!kCommit) {
+                const int r = eu / a.Hkv, gg = eu % a.Hkv;
+                const int t = row / G, hh = row % G;
+                bf16 *orow = a.O + (((size_t)r * B + t) * a.Hq + (size_t)gg * G + hh) * d + part * dh;
+                for (int hc = 0; hc < dh / 32; ++hc) {
+                    float v[32];
+                    tmem_ld32(tmem + dcol + lane_off + part * dh + 32 * hc, v);
+                    tmem_wait_ld();
+                    if (ok && valid) {
+                        uint32_t pk[16];
+#pragma unroll
+                        for (int i = 0; i < 32; i += 2) pk[i / 2] = pack_bf16x2(v[i] * inv, v[i + 1] * inv);
+                        uint4 *dst = reinterpret_cast<uint4 *>(orow + 32 * hc);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0 && ok) mbar_arrive(&dfree[ek & 1]);
+                return ok;
+            }
             // d = 128: column half -> slot; d = 64: token half -> slot (one 64-column atom)
             const int rows_half = G * B / 2;
             const int sidx = d == 128 ? part : (row >= rows_half ? 1 : 0);
@@ -601,6 +628,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
 
         uint32_t q = 0, kp = 0, prev_q = 0;
         float prev_inv = 0.f;   // 1 / den of the unit whose output is still pending (step)
+        int prev_u = 0;         // and that unit
         bool ok = true;
         for (int u = u_begin; u < u_end; ++u) {
             float *Sg = unit_state(a, u);
@@ -904,7 +932,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             if (lane == 0) mbar_arrive(pready);
 
             // previous unit's output, while R+ of this one runs (step)
-            if (!kCommit && kp >= 1) bad = !epilogue(kp - 1, prev_q, prev_inv);
+            if (!kCommit && kp >= 1) bad = !epilogue(kp - 1, prev_q, prev_inv, prev_u);
             // ---- phase D: phi- scaled by cneg in the phi columns (step: once R+ has
             // consumed phi+ there)
             if (kCommit) {
@@ -971,14 +999,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                         if (h == 0) mbar_arrive(efree);
                     }
                 }
-                epilogue(kp, q, inv_den);
+                epilogue(kp, q, inv_den, u);
             }
             prev_q = q;
             prev_inv = inv_den;
+            prev_u = u;
             q += NC;
             ++kp;
         }
-        if (!kCommit && ok && kp >= 1) epilogue(kp - 1, prev_q, prev_inv);
+        if (!kCommit && ok && kp >= 1) epilogue(kp - 1, prev_q, prev_inv, prev_u);
         if (mt == 0 && *fail) raise_error(a.err, ERR_WAIT_TIMEOUT);
     }
 
@@ -1035,6 +1064,7 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
             return cudaErrorInvalidValue;
     }
     a.K = static_cast<const bf16 *>(K);
+    a.O = static_cast<bf16 *>(O);
     a.alpha = alpha;
     a.states = states;
     a.err = err;
