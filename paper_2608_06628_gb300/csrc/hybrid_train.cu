@@ -48,6 +48,7 @@ using namespace pipe;
 constexpr int kThreads = 128;
 constexpr int kSmemLimit = 232448;
 constexpr uint32_t kColS = 0, kColGv = 64, kColU = 256, kColY = 384, kColG = 0, kColDR = 0;
+constexpr int kDwStages = 3;   // shared-memory stages of k_dw
 
 struct TrainArgs {
     const bf16 *Q, *K, *V, *W, *dO;
@@ -402,7 +403,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefix_states(const __grid_cons
 // ---------------------------------------------------------------------------
 // k_slot_scan: per sequence, running sums over n_slots slots of nf floats.
 // reverse = false: slot n += slot n-1 (inclusive, slot 0 unchanged);
-// reverse = true : slot m = sum of slots n > m (exclusive, from the end).
+// reverse = true : slot m = sum of slots n > m (exclusive, from the end; the
+// backward's R_m = sum_{n > m} dR_n, the only use at present).
 // ---------------------------------------------------------------------------
 __global__ void k_slot_scan(float *buf0, float *buf1, int n_seq, int n_slots, size_t nf, bool reverse)
 {
@@ -818,8 +820,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
 // ---------------------------------------------------------------------------
 // k_dw: dW_g += sum over a range of rows of x du^T.  Row rho of group g: token
 // t = rho / (G+1); kinds 0..G-1 are the query heads of the group (Q, dU_q),
-// kind G is the key (K, dU_k).  128 rows per step, two smem stages; the
-// accumulator (d lanes x F columns) stays in Tensor Memory over the range.
+// kind G is the key (K, dU_k).  128 rows per step, three shared-memory stages
+// (copies two steps ahead); the accumulator (d lanes x F columns) stays in
+// Tensor Memory over the range.
 // ---------------------------------------------------------------------------
 struct DwArgs {
     const bf16 *Q, *K, *dUq, *dUk;
@@ -843,12 +846,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwAr
     if (r_end > total) r_end = total;
     const int n_tiles = r_begin < total ? (int)((r_end - r_begin + 127) / 128) : 0;
     const uint32_t xbytes = 2 * 128 * 128, ubytes = (uint32_t)(F / 64) * 128 * 128, stage = xbytes + ubytes;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + 2 * stage);
-    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 2);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kDwStages * stage);   // [kDwStages] MMAs of a stage done
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + kDwStages);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
     if (tid == 0) {
-        mbar_init(&bars[0], 1);
-        mbar_init(&bars[1], 1);
+        for (int i = 0; i < kDwStages; ++i) mbar_init(&bars[i], 1);
         *fail = 0;
         fence_mbar_init();
     }
@@ -858,7 +860,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwAr
     }
     // for d = 64 the second half of the M = 128 operand X^T stays zero
     if (d == 64)
-        for (int i = tid; i < 2 * 1024; i += kThreads) {
+        for (int i = tid; i < kDwStages * 1024; i += kThreads) {
             const int st = i / 1024, k = i % 1024;
             reinterpret_cast<uint4 *>(smem + st * stage + 128 * 128)[k] = make_uint4(0, 0, 0, 0);
         }
@@ -868,9 +870,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwAr
     const uint32_t tmem = *tmem_holder;
     const uint32_t idW = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, F);
     bool ok = true;
-    // copies of step k into stage k & 1: row tid of the step (16-byte cp.async, one group per step)
+    // copies of step k into stage k % kDwStages: row tid of the step (16-byte
+    // cp.async, one group per step), issued two steps ahead of the MMAs
     auto issue = [&](int k) {
-        uint8_t *sx = smem + (k & 1) * stage, *su = sx + xbytes;
+        uint8_t *sx = smem + (k % kDwStages) * stage, *su = sx + xbytes;
         const long long rho = r_begin + (long long)k * 128 + tid;
         const bool valid = rho < r_end;
         const bf16 *xr = nullptr, *ur = nullptr;
@@ -902,12 +905,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwAr
         }
         cp_async_commit();
     };
+    // the MMAs of step k commit to bars[k % kDwStages]: its (k / kDwStages)-th phase
     if (n_tiles > 0) issue(0);
+    if (n_tiles > 1) issue(1);
     for (int k = 0; k < n_tiles; ++k) {
-        if (k + 1 < n_tiles) {
-            // stage (k + 1) & 1 was last read by the MMAs of step k - 1
-            if (k >= 1) ok = wait_bar(&bars[(k + 1) & 1], (uint32_t)((k - 1) >> 1) & 1u, fail) && ok;
-            issue(k + 1);
+        if (k + 2 < n_tiles) {
+            // stage (k + 2) % kDwStages was last read by the MMAs of step k - 1
+            if (k >= 1)
+                ok = wait_bar(&bars[(k - 1) % kDwStages], (uint32_t)((k - 1) / kDwStages) & 1u, fail) && ok;
+            issue(k + 2);
+            cp_async_wait<2>();
+        } else if (k + 1 < n_tiles) {
             cp_async_wait<1>();
         } else {
             cp_async_wait<0>();
@@ -916,17 +924,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwAr
         if (group_sync_failed(1, kThreads, !ok)) break;
         if (tid == 0) {
             tc_fence_after();
-            const uint32_t x_u = smem_u32(smem + (k & 1) * stage), u_u = x_u + xbytes;
+            const uint32_t x_u = smem_u32(smem + (k % kDwStages) * stage), u_u = x_u + xbytes;
             for (int ks = 0; ks < 8; ++ks)
                 mma_bf16_ss(tmem, smem_desc(x_u + ks * 2048, 128 * 128, 1024, SWZ_128B),
                             smem_desc(u_u + ks * 2048, 128 * 128, 1024, SWZ_128B), idW, (k | ks) != 0);
-            mma_commit(&bars[k & 1]);
+            mma_commit(&bars[k % kDwStages]);
         }
     }
     cp_async_wait<0>();
-    // the last one or two steps
-    for (int k = n_tiles - 2; k < n_tiles; ++k)
-        if (k >= 0) ok = wait_bar(&bars[k & 1], (uint32_t)(k >> 1) & 1u, fail) && ok;
+    // the last steps (those not waited for in the loop)
+    for (int k = n_tiles - kDwStages; k < n_tiles; ++k)
+        if (k >= 0) ok = wait_bar(&bars[k % kDwStages], (uint32_t)(k / kDwStages) & 1u, fail) && ok;
     tc_fence_after();
     if (ok && n_tiles > 0 && tid < d) {
         float *dst = a.dW + ((size_t)g * d + tid) * F;
@@ -1124,12 +1132,13 @@ cudaError_t launch_train_backward(const hybrid_cfg &c, const void *Q, const void
     b.F = a.F;
     const long long rows = b.n_tok * (a.Hq / a.Hkv + 1);
     const long long tiles = (rows + 127) / 128;
-    int per_group = (2 * sm_count() + a.Hkv - 1) / a.Hkv;
+    // one CTA per SM (three 64 KB stages each), row ranges split evenly within a group
+    int per_group = sm_count() / a.Hkv;
     if (per_group > tiles) per_group = (int)tiles;
     if (per_group < 1) per_group = 1;
     b.tiles_per_cta = (int)((tiles + per_group - 1) / per_group);
     b.ctas_per_group = per_group;
-    const size_t dw_smem = 2 * ((size_t)2 * 128 * 128 + (size_t)(a.F / 64) * 128 * 128) + 1024 + 1024;
+    const size_t dw_smem = kDwStages * ((size_t)2 * 128 * 128 + (size_t)(a.F / 64) * 128 * 128) + 1024 + 1024;
     if ((e = opt_in(k_dw, g_opt_dw)) != cudaSuccess) return e;
     return launch_pdl(k_dw, dim3((unsigned)(a.Hkv * per_group)), dim3(kThreads), dw_smem, st, b);
 }

@@ -78,6 +78,23 @@ def test_train_parity(wl):
         assert r <= TOL, f"{wl.name} {what}: rel-L2 {r:.3e}"
 
 
+def test_train_stress_keys_and_saturated_gate():
+    """Keys x 8 (scores up to ~30, the stress setting of the decoding configs) and
+    one gate saturated at alpha = +inf (w = 1, so its dalpha is 0)."""
+    wl = TW("k8_sat", 2, 128, 8, 2, 128, 128, 32, 47).with_(k_scale=8.0)
+    Q, K, V, W, alpha, dO = inputs(wl)
+    alpha[3] = float("inf")
+    O, dW, dalpha = run_gpu(wl, Q, K, V, W, alpha, dO)
+    orc = oracle.load()
+    args = (h64(Q), h64(K), h64(V), h64(W), h64(alpha))
+    O_ref = orc.train_forward(*args, wl.B)
+    dW_ref, da_ref = orc.train_backward(*args, h64(dO), wl.B)
+    assert rel_l2(h64(O), O_ref) <= TOL
+    assert rel_l2(h64(dW), dW_ref) <= TOL
+    assert rel_l2(h64(dalpha), da_ref) <= TOL
+    assert float(dalpha[3]) == 0.0
+
+
 def test_train_single_block_has_no_gradient():
     """One block per sequence: no prefix anywhere, so O is the in-block softmax
     and dW is exactly zero; dalpha is zero up to rounding."""
