@@ -146,3 +146,33 @@ def test_train_gradient_linear_in_dO():
     _, dW3, da3 = run_gpu(wl, Q, K, V, W, alpha, (dO.float() + dO2.float()).to(dO.dtype))
     assert rel_l2(h64(dW3), h64(dW1) + h64(dW2)) <= TOL
     assert rel_l2(h64(da3), h64(da1) + h64(da2)) <= TOL
+
+
+def test_train_calls_allocate_nothing():
+    """After a first call (kernel attributes set), forward and backward allocate no
+    device memory: free device memory is unchanged across further calls, and the
+    results are bitwise repeatable on the same workspace."""
+    wl = TW("no_alloc", 2, 128, 8, 2, 128, 128, 32, 48)
+    Q, K, V, W, alpha, dO = inputs(wl)
+    cfg = H.make_cfg(wl.d, wl.F, wl.Hq, wl.Hkv, wl.B, wl.io_dtype)
+    n, L = Q.shape[0], Q.shape[1]
+    nbytes = H.hybrid_train_workspace_bytes(cfg, n, L)
+    ws = torch.empty(nbytes + 1024, dtype=torch.uint8, device="cuda")
+    ptr = (ws.data_ptr() + 1023) & ~1023
+    outs = []
+    for call in range(3):
+        O = torch.empty_like(Q)
+        dW = torch.empty(W.shape, dtype=torch.float32, device="cuda")
+        da = torch.empty(wl.Hq, dtype=torch.float32, device="cuda")
+        torch.cuda.synchronize()
+        free_before = torch.cuda.mem_get_info()[0]
+        H.hybrid_train_forward(cfg, Q, K, V, W, alpha, n, L, O, ptr, nbytes)
+        H.hybrid_train_backward(cfg, Q, K, V, W, alpha, dO, n, L, ptr, nbytes, dW, da)
+        H.hybrid_check()
+        if call > 0:
+            assert torch.cuda.mem_get_info()[0] == free_before, f"call {call} allocated device memory"
+        outs.append((O, dW, da))
+    assert torch.equal(outs[1][0], outs[2][0])
+    # dW and dalpha sum partial results with float atomics: equal up to the order of the adds
+    assert rel_l2(h64(outs[1][1]), h64(outs[2][1])) < 1e-6
+    assert rel_l2(h64(outs[1][2]), h64(outs[2][2])) < 1e-6
