@@ -78,6 +78,7 @@ __device__ __forceinline__ uint32_t swz(int r, int j)
 }
 
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
@@ -360,25 +361,43 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefix_states(const __grid_cons
         }
         for (int bl = 0; bl < nb; ++bl) {
             const int n = b0 + bl;
-            // slot n holds S_{n-1} (the running slice, in registers) and z_{n-1}
+            // slot n holds S_{n-1} (the running slice, in registers) and z_{n-1}.  The
+            // slice's bytes are contiguous runs of both images: decode-image tile j (d
+            // rows x 128 bytes) and, per e-tile c, feature rows 32 j .. 32 j + 31 (4 KB).
+            // They are laid out in shared memory exactly as in global memory and stored
+            // by bulk copies; K's space stages even blocks and V's space odd ones (both
+            // idle until the next group), so a block's staging waits only for the bulk
+            // stores of the block two before it.
             const size_t slot = ((size_t)s * n_blk + n) * Hkv + g;
             float *P = a.P + slot * hf, *PT = a.PT + slot * hf;
+            uint8_t *stg = smem + ((bl & 1) ? Lp.off_v : Lp.off_k);
+            if (tid == 0 && bl >= 2) bulk_wait_read_1();
+            __syncthreads();
             const int e = tid;
             if (e < d) {
-                // decode image: tile j, row e (32 features, granules permuted by e mod 8)
-                float4 *row = reinterpret_cast<float4 *>(P + (size_t)j * 32 * d + (size_t)e * 32);
+                // decode-image tile j: row e at e * 128 bytes, granules permuted by e mod 8
+                float4 *row = reinterpret_cast<float4 *>(stg + (size_t)e * 128);
 #pragma unroll
                 for (int q = 0; q < 8; ++q)
                     row[q ^ (e & 7)] = make_float4(run[4 * q], run[4 * q + 1], run[4 * q + 2], run[4 * q + 3]);
-                // feature-row image: rows f = 32 j + k, column e of e-tile e / 32
-                float *pt = PT + (size_t)(e >> 5) * 64 * F + (size_t)(32 * j) * 32 + (e & 3);
+                // feature-row piece of e-tile e / 32: row k (f = 32 j + k), column e mod 32
+                float *pt = reinterpret_cast<float *>(stg + (size_t)d * 128 + (size_t)(e >> 5) * 4096) + (e & 3);
 #pragma unroll
-                for (int k = 0; k < 32; ++k) pt[(size_t)k * 32 + (size_t)((((e & 31) >> 2) ^ (k & 7)) << 2)] = run[k];
+                for (int k = 0; k < 32; ++k) pt[k * 32 + ((((e & 31) >> 2) ^ (k & 7)) << 2)] = run[k];
             }
             if (tid < 32) {
                 P[z_offset(32 * j + tid, d, F)] = zc;
                 PT[z_offset(32 * j + tid, d, F)] = zc;
                 zc += dz[bl * 32 + tid];
+            }
+            fence_proxy_async_smem();
+            __syncthreads();
+            if (tid == 0) {
+                bulk_s2g(P + (size_t)j * 32 * d, stg, (uint32_t)d * 128);
+                for (int c = 0; c < d / 32; ++c)
+                    bulk_s2g(PT + (size_t)c * 64 * F + (size_t)(32 * j) * 32, stg + (size_t)d * 128 + (size_t)c * 4096,
+                             4096);
+                bulk_commit();
             }
             if (n == n_blk - 1) break;
             if (e < d) {
@@ -389,10 +408,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefix_states(const __grid_cons
                 for (int k = 0; k < 32; ++k) run[k] += x[k];
             }
         }
+        // the next group's copies reuse K's and V's space
+        if (tid == 0) bulk_wait_read_all();
         tc_fence_before();
         __syncthreads();
         tc_fence_after();
     }
+    if (tid == 0) bulk_wait_all();
     if (!ok && tid == 0) raise_error(a.err, ERR_WAIT_TIMEOUT);
     tc_fence_before();
     __syncthreads();
