@@ -33,6 +33,7 @@
 //                   R tiles, du_k
 //   k_dw            dW_g = sum over query and key rows of x du^T, split over
 //                   row ranges and added into dW with float atomics
+#include <algorithm>
 #include <atomic>
 
 #include "hybrid_common.cuh"
@@ -51,6 +52,10 @@ constexpr uint32_t kColS = 0, kColGv = 64, kColU = 256, kColY = 384, kColG = 0, 
 constexpr int kDwStages = 3;   // shared-memory stages of k_dw
 
 struct TrainArgs {
+    // 128-byte-swizzled tensor maps: Q and dO [n*L][Hq][d] with box {64, G, B} (rows t*G + h),
+    // K and V [n*L][Hkv][d] with box {64, 1, B} (a block) and {64, 1, GR} (a group of the prefix
+    // sweep), W [Hkv*d][F] with box {64, d}
+    CUtensorMap tmQ, tmdO, tmK, tmV, tmKg, tmVg, tmW;
     const bf16 *Q, *K, *V, *W, *dO;
     const float *alpha;
     float *P, *PT, *R;
@@ -81,30 +86,6 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 __device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
-
-// Rows [0, nalloc) of a bf16 operand image (panels of 64 columns, panel stride
-// nalloc*128 bytes): row r from rowptr(r), columns [0, ncols), by 16-byte
-// cp.async copies that are all in flight at once (the caller commits and waits);
-// rows whose rowptr is null are zeroed with plain stores.
-template <class RowPtr>
-__device__ __forceinline__ void load_rows_bf16(uint8_t *dst, RowPtr rowptr, int nalloc, int ncols, int tid)
-{
-    const int gpr = ncols >> 3;
-    for (int i = tid; i < nalloc * gpr; i += kThreads) {
-        const int r = i / gpr, c8 = i - r * gpr;
-        uint8_t *d = dst + (uint32_t)(c8 >> 3) * (uint32_t)nalloc * 128u + swz(r, c8 & 7);
-        const bf16 *src = rowptr(r);
-        if (src)
-            ptx::cp_async16(d, reinterpret_cast<const uint4 *>(src) + c8);
-        else
-            *reinterpret_cast<uint4 *>(d) = make_uint4(0, 0, 0, 0);
-    }
-}
-__device__ __forceinline__ void cp_async_all_landed()
-{
-    cp_async_commit();
-    cp_async_wait<0>();
-}
 
 // Write 32 consecutive columns [c0, c0 + 32) of row r (values x, converted to
 // bf16) into a bf16 operand image with panel stride pstride.
@@ -248,17 +229,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefix_states(const __grid_cons
     const bool neg = j >= F / 32;              // slice of phi- features
     const int fu = (j % (F / 32)) * 32;        // first column of u the slice reads
     const size_t hf = head_floats(d, F);
-    const size_t kv_row = (size_t)Hkv * d;
     const int GB = min(4, 128 / B);            // blocks per group (at most 128 key rows)
     uint64_t *bar = reinterpret_cast<uint64_t *>(smem + Lp.off_bar);
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar + 2);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
     float *dz = reinterpret_cast<float *>(smem + Lp.off_z);   // [GB][32] dz of the group's blocks
     float *xs = reinterpret_cast<float *>(smem + Lp.off_x);   // [128][32] phi slice of the rows
+    uint64_t *tbar = &bar[1];   // a group's K and V rows (and, with the first, W) have landed
     if (tid == 0) {
         mbar_init(&bar[0], 1);
+        mbar_init(tbar, 1);
         *fail = 0;
         fence_mbar_init();
+        prefetch_tensormap(&a.tmKg);
+        prefetch_tensormap(&a.tmVg);
+        prefetch_tensormap(&a.tmW);
     }
     if (warp == 0) {
         tmem_alloc(tmem_holder, 256);
@@ -268,9 +253,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefix_states(const __grid_cons
     if (d == 64)
         for (int i = tid; i < 1024; i += kThreads)
             reinterpret_cast<uint4 *>(smem + Lp.off_v + 128 * 128)[i] = make_uint4(0, 0, 0, 0);
-    griddep_wait();
-    load_rows_bf16(smem + Lp.off_w, [&](int r) { return a.W + ((size_t)g * d + r) * F; }, d, F, tid);
+    fence_proxy_async_smem();
     __syncthreads();
+    griddep_wait();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
     const uint32_t lane_off = (uint32_t)(warp & 3) * 32u << 16;
@@ -286,12 +271,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefix_states(const __grid_cons
     for (int b0 = 0; b0 < n_blk && ok; b0 += GB) {
         const int nb = min(GB, n_blk - b0), nt = nb * B;
         const size_t t0 = (size_t)s * a.L + (size_t)b0 * B;
-        auto krow = [&](int r) -> const bf16 * { return r < nt ? a.K + (t0 + r) * kv_row + (size_t)g * d : nullptr; };
-        auto vrow = [&](int r) -> const bf16 * { return r < nt ? a.V + (t0 + r) * kv_row + (size_t)g * d : nullptr; };
-        load_rows_bf16(smem + Lp.off_k, krow, 128, d, tid);
-        load_rows_bf16(smem + Lp.off_v, vrow, 128, d, tid);
-        cp_async_all_landed();
-        fence_proxy_async_smem();
+        // the group's K and V rows by TMA (boxes of GB*B rows; rows past the sequence or past
+        // the tensor are not used: their phi is zeroed and no MMA reads them)
+        if (tid == 0) {
+            const uint32_t box = (uint32_t)(d / 64) * (uint32_t)(GB * B) * 128;
+            mbar_arrive_expect_tx(tbar, 2 * box + (b0 == 0 ? (uint32_t)(F / 64) * d * 128 : 0u));
+            for (int p = 0; p < d / 64; ++p) {
+                tma_load_3d(smem + Lp.off_k + p * 128 * 128, &a.tmKg, 64 * p, g, (int)t0, tbar);
+                tma_load_3d(smem + Lp.off_v + p * 128 * 128, &a.tmVg, 64 * p, g, (int)t0, tbar);
+            }
+            if (b0 == 0)
+                for (int p = 0; p < F / 64; ++p)
+                    tma_load_2d(smem + Lp.off_w + p * d * 128, &a.tmW, 64 * p, g * d, tbar);
+        }
+        ok = wait_bar(tbar, (uint32_t)(b0 / GB) & 1u, fail) && ok;
         tc_fence_before();
         __syncthreads();
         tc_fence_after();
@@ -472,15 +465,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
     const int tid = threadIdx.x, warp = tid >> 5;
     const int d = a.d, F = a.F, B = a.B, Hkv = a.Hkv, Hq = a.Hq, G = Hq / Hkv;
     const int g = blockIdx.x % Hkv, n = (blockIdx.x / Hkv) % a.n_blk, s = blockIdx.x / (Hkv * a.n_blk);
-    // The tile's rows (G*B query rows or B key rows) are spread evenly over the four
-    // 32-lane quadrants of Tensor Memory, so that all four warps share the per-row
-    // math: lane r = 32 q + i holds row q * rpq + i if i < rpq (rpq = rows / 4).
+    // Rows of the tile on Tensor Memory lanes: query side, lane r < G*B is token r / G,
+    // head r % G of the group (the order the TMA box lands in); key side, lane r < B is
+    // token r.  Lanes beyond are zero rows.
     const int rows = kQuery ? G * B : B;
-    const int rpq = rows / 4;
-    auto row_of = [&](int r) -> int { return (r & 31) < rpq ? (r >> 5) * rpq + (r & 31) : -1; };
     const size_t hf = head_floats(d, F);
     const size_t t0 = (size_t)s * a.L + (size_t)n * B;
-    const size_t kv_row = (size_t)Hkv * d, q_row = (size_t)Hq * d;
+    const size_t kv_row = (size_t)Hkv * d;
     // tile source: PT slot n (query side: S_{n-1}) or R slot n (key side: R_n)
     const float *src = (kQuery ? a.PT : a.R) + (((size_t)s * a.n_blk + n) * Hkv + g) * hf;
 
@@ -488,48 +479,57 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
     uint64_t *mbar = bars;          // MMA groups complete
     uint64_t *full = bars + 1;      // [2] ring slot loaded
     uint64_t *empty = bars + 3;     // [2] ring slot consumed
-    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 5);
+    uint64_t *tbar = bars + 5;      // the phase-one operands have landed
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 6);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
     float *sDw = reinterpret_cast<float *>(tmem_holder + 2);    // [8] dw per head of the group
     float *sZ = reinterpret_cast<float *>(smem + Lr.off_z);     // z_{n-1} or r_n
     if (tid == 0) {
-        for (int i = 0; i < 5; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 6; ++i) mbar_init(&bars[i], 1);
         *fail = 0;
         fence_mbar_init();
+        prefetch_tensormap(&a.tmW);
+        prefetch_tensormap(&a.tmK);
+        if (kQuery) {
+            prefetch_tensormap(&a.tmQ);
+            prefetch_tensormap(&a.tmdO);
+            prefetch_tensormap(&a.tmV);
+        }
     }
     if (tid < 8) sDw[tid] = 0.f;
     if (warp == 0) {
         tmem_alloc(tmem_holder, 512);
         tmem_relinquish();
     }
+    // rows of the M = 128 operands beyond the tile stay zero (the TMA boxes fill rows < rows)
+    for (int i = tid; i < (128 - rows) * (d / 8); i += kThreads) {
+        const int r = rows + i / (d / 8), c8 = i % (d / 8);
+        const uint32_t off = (uint32_t)(c8 >> 3) * (128 * 128) + swz(r, c8 & 7);
+        *reinterpret_cast<uint4 *>(smem + Lr.off_q + off) = make_uint4(0, 0, 0, 0);
+        if (kQuery) *reinterpret_cast<uint4 *>(smem + Lr.off_do + off) = make_uint4(0, 0, 0, 0);
+    }
+    __syncthreads();
     griddep_wait();
 
-    // phase one: operands of [U | scores] = Q [W | K^T] and dO V^T (query side) or U = K W
-    if (kQuery) {
-        auto qrow = [&](int r) -> const bf16 * {
-            const int q = row_of(r);
-            return q < 0 ? nullptr : a.Q + (t0 + q % B) * q_row + (size_t)(g * G + q / B) * d;
-        };
-        auto dorow = [&](int r) -> const bf16 * {
-            const int q = row_of(r);
-            return q < 0 ? nullptr : a.dO + (t0 + q % B) * q_row + (size_t)(g * G + q / B) * d;
-        };
-        load_rows_bf16(smem + Lr.off_q, qrow, 128, d, tid);
-        load_rows_bf16(smem + Lr.off_do, dorow, 128, d, tid);
-        load_rows_bf16(smem + Lr.off_k, [&](int r) -> const bf16 * { return a.K + (t0 + r) * kv_row + (size_t)g * d; },
-                       B, d, tid);
-        load_rows_bf16(smem + Lr.off_v, [&](int r) -> const bf16 * { return a.V + (t0 + r) * kv_row + (size_t)g * d; },
-                       B, d, tid);
-    } else {
-        auto krow = [&](int r) -> const bf16 * {
-            const int q = row_of(r);
-            return q < 0 ? nullptr : a.K + (t0 + q) * kv_row + (size_t)g * d;
-        };
-        load_rows_bf16(smem + Lr.off_q, krow, 128, d, tid);
+    // phase one by TMA: [U | scores] = Q [W | K^T] and dO V^T (query side) or U = K W
+    if (tid == 0) {
+        const uint32_t qbytes = (uint32_t)(d / 64) * rows * 128, kvbytes = (uint32_t)(d / 64) * B * 128;
+        const uint32_t wbytes = (uint32_t)(F / 64) * d * 128;
+        mbar_arrive_expect_tx(tbar, kQuery ? 2 * qbytes + 2 * kvbytes + wbytes : kvbytes + wbytes);
+        for (int p = 0; p < d / 64; ++p) {
+            if (kQuery) {
+                tma_load_3d(smem + Lr.off_q + p * 128 * 128, &a.tmQ, 64 * p, g * G, (int)t0, tbar);
+                tma_load_3d(smem + Lr.off_do + p * 128 * 128, &a.tmdO, 64 * p, g * G, (int)t0, tbar);
+                tma_load_3d(smem + Lr.off_k + p * B * 128, &a.tmK, 64 * p, g, (int)t0, tbar);
+                tma_load_3d(smem + Lr.off_v + p * B * 128, &a.tmV, 64 * p, g, (int)t0, tbar);
+            } else {
+                tma_load_3d(smem + Lr.off_q + p * 128 * 128, &a.tmK, 64 * p, g, (int)t0, tbar);
+            }
+        }
+        for (int p = 0; p < F / 64; ++p) tma_load_2d(smem + Lr.off_w + p * d * 128, &a.tmW, 64 * p, g * d, tbar);
     }
-    load_rows_bf16(smem + Lr.off_w, [&](int r) -> const bf16 * { return a.W + ((size_t)g * d + r) * F; }, d, F, tid);
     for (int f = tid; f < 2 * F; f += kThreads) sZ[f] = src[z_offset(f, d, F)];
-    cp_async_all_landed();
+    bool ok = wait_bar(tbar, 0, fail);
     fence_proxy_async_smem();
     __syncthreads();
     tc_fence_after();
@@ -557,7 +557,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         }
         mma_commit(mbar);
     }
-    bool ok = wait_bar(mbar, 0, fail);
+    ok = wait_bar(mbar, 0, fail) && ok;
     tc_fence_after();
     // the phase-one operands are consumed: the first two tiles go into their space
     if (tid == 0 && ok) {
@@ -569,10 +569,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
     }
 
     // ---- row statistics (thread = row) ----
-    const int myrow = row_of(tid);
-    const bool valid = myrow >= 0;
-    const int hl = (kQuery && valid) ? myrow / B : 0;              // query head within the group
-    const int tok = valid ? (kQuery ? myrow % B : myrow) : 0;      // token within the block
+    const bool valid = tid < rows;
+    const int hl = (kQuery && valid) ? tid % G : 0;                // query head within the group
+    const int tok = valid ? (kQuery ? tid / G : tid) : 0;          // token within the block
+    const size_t q_row = (size_t)Hq * d;
     const PhiStats st = phi_stats(tl + kColU, F);
     const float ip = 1.f / st.sp, in = 1.f / st.sn;
     // Query rows: w, 1/D, and the merge terms A = g.sm_num / D, beta = sm_den / D,
@@ -805,24 +805,45 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         }
         ok = wait_bar(mbar, 0, fail);
         tc_fence_after();
-        if (ok) {
+        // R's slot: per e-tile c the 2F feature rows (2F x 128 bytes, contiguous in global
+        // memory) are staged in the space of phi(Q) and [dN | dD], which the dR MMAs have
+        // consumed, laid out as in global memory, and written by bulk copies
+        if (!group_sync_failed(1, kThreads, !ok)) {
             float *R = a.R + (((size_t)s * a.n_blk + n) * Hkv + g) * hf;
-            for (int i = 0; i < NM; ++i) {
-                const int f = 128 * i + tid;
-                float x[32];
-                for (int c = 0; c < d / 32; ++c) {
+            const uint32_t tile_bytes = (uint32_t)2 * F * 128;
+            for (int c = 0; c < d / 32; ++c) {
+                // buffers: phi's space (two tiles), then [dN | dD]'s; tile 3 reuses the first
+                uint8_t *buf = (c % 3 == 2) ? smem + Lr.off_y : smem + Lr.off_phi + (uint32_t)(c % 3) * tile_bytes;
+                if (c == 3) {
+                    if (tid == 0) bulk_wait_read_all();
+                    __syncthreads();
+                }
+                for (int i = 0; i < NM; ++i) {
+                    const int f = 128 * i + tid;
+                    float x[32];
                     tmem_ld32(tl + kColDR + (uint32_t)(i * NYS + 32 * c), x);
                     tmem_wait_ld();
-                    float4 *row = reinterpret_cast<float4 *>(R + (size_t)c * 64 * F + (size_t)f * 32);
+                    float4 *row = reinterpret_cast<float4 *>(buf + (size_t)f * 128);
 #pragma unroll
                     for (int q = 0; q < 8; ++q)
                         row[q ^ (f & 7)] = make_float4(x[4 * q], x[4 * q + 1], x[4 * q + 2], x[4 * q + 3]);
                 }
+                fence_proxy_async_smem();
+                __syncthreads();
+                if (tid == 0) {
+                    bulk_s2g(R + (size_t)c * 64 * F, buf, tile_bytes);
+                    bulk_commit();
+                }
+            }
+            for (int i = 0; i < NM; ++i) {
                 float zz[16];
                 tmem_ld16(tl + kColDR + (uint32_t)(i * NYS + d), zz);
                 tmem_wait_ld();
-                R[z_offset(f, d, F)] = zz[0];
+                R[z_offset(128 * i + tid, d, F)] = zz[0];
             }
+            if (tid == 0) bulk_wait_all();
+        } else {
+            ok = false;
         }
     }
     if (tid == 0 && (failed2 || !ok)) raise_error(a.err, ERR_WAIT_TIMEOUT);
@@ -1065,6 +1086,22 @@ TrainArgs make_args(const hybrid_cfg &c, int n_seq, int L, const Workspace &w)
 
 std::atomic<unsigned long long> g_opt_state, g_opt_q, g_opt_k, g_opt_dw;
 
+// Tensor maps of [n*L][H][d] (box {64, bh, bt}) and of W [Hkv*d][F] (box {64, d}).
+bool encode_rows(CUtensorMap *m, const void *base, long long n_tok, int H, int d, int bh, int bt)
+{
+    const cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)H, (cuuint64_t)n_tok};
+    const cuuint64_t strides[2] = {(cuuint64_t)d * 2, (cuuint64_t)H * d * 2};
+    const cuuint32_t box[3] = {64, (cuuint32_t)bh, (cuuint32_t)bt};
+    return encode_bf16(m, base, 3, dims, strides, box);
+}
+bool encode_w(CUtensorMap *m, const void *W, int Hkv, int d, int F)
+{
+    const cuuint64_t dims[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
+    const cuuint64_t strides[1] = {(cuuint64_t)F * 2};
+    const cuuint32_t box[2] = {64, (cuuint32_t)d};
+    return encode_bf16(m, W, 2, dims, strides, box);
+}
+
 }  // namespace
 
 bool train_supported(const hybrid_cfg &c, int seq_len)
@@ -1099,6 +1136,13 @@ cudaError_t launch_train_states(const hybrid_cfg &c, const void *K, const void *
     a.V = static_cast<const bf16 *>(V);
     a.W = static_cast<const bf16 *>(W);
     a.err = err;
+    {
+        const long long n_tok = (long long)n_seq * seq_len;
+        const int GR = std::min(4, 128 / a.B) * a.B;   // rows of a prefix-sweep group (k_prefix_states' GB * B)
+        if (!encode_rows(&a.tmKg, K, n_tok, a.Hkv, a.d, 1, GR) || !encode_rows(&a.tmVg, V, n_tok, a.Hkv, a.d, 1, GR) ||
+            !encode_w(&a.tmW, W, a.Hkv, a.d, a.F))
+            return cudaErrorInvalidValue;
+    }
     const int slots = n_seq * a.n_blk;
     const size_t sf = slot_floats(a.Hkv, a.d, a.F);
     cudaError_t e = cudaSuccess;
@@ -1124,6 +1168,14 @@ cudaError_t launch_train_backward(const hybrid_cfg &c, const void *Q, const void
     a.alpha = alpha;
     a.dalpha = dalpha;
     a.err = err;
+    {
+        const long long n_tok = (long long)n_seq * seq_len;
+        const int G = a.Hq / a.Hkv;
+        if (!encode_rows(&a.tmQ, Q, n_tok, a.Hq, a.d, G, a.B) || !encode_rows(&a.tmdO, dO, n_tok, a.Hq, a.d, G, a.B) ||
+            !encode_rows(&a.tmK, K, n_tok, a.Hkv, a.d, 1, a.B) || !encode_rows(&a.tmV, V, n_tok, a.Hkv, a.d, 1, a.B) ||
+            !encode_w(&a.tmW, W, a.Hkv, a.d, a.F))
+            return cudaErrorInvalidValue;
+    }
     const int units = n_seq * a.n_blk * a.Hkv;
     const size_t sf = slot_floats(a.Hkv, a.d, a.F);
     cudaError_t e;
