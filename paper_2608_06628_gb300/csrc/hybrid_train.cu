@@ -50,6 +50,8 @@ constexpr int kThreads = 128;
 constexpr int kSmemLimit = 232448;
 constexpr uint32_t kColS = 0, kColGv = 64, kColU = 256, kColY = 384, kColG = 0, kColDR = 0;
 constexpr int kDwStages = 3;   // shared-memory stages of k_dw
+constexpr int kGradThreads = 256;   // k_phi_grad: two threads (parts) per Tensor Memory lane
+constexpr uint32_t kXchBytes = 14 * 1024;   // k_phi_grad: the parts' exchange of row partials
 
 struct TrainArgs {
     // 128-byte-swizzled tensor maps: Q and dO [n*L][Hq][d] with box {64, G, B} (rows t*G + h),
@@ -134,9 +136,47 @@ __device__ __forceinline__ PhiStats phi_stats(uint32_t taddr, int F)
     return s;
 }
 
+// Partial statistics of the same over the 32-column chunks [j0, j1) only, to be
+// combined with the other chunks' by combine_stats.
+__device__ __forceinline__ PhiStats phi_stats_chunks(uint32_t taddr, int j0, int j1)
+{
+    PhiStats s{-INFINITY, 0.f, INFINITY, 0.f};
+    float x[32];
+    for (int j = j0; j < j1; ++j) {
+        ptx::tmem_ld32(taddr + 32 * j, x);
+        ptx::tmem_wait_ld();
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+            s.mp = fmaxf(s.mp, x[k]);
+            s.mn = fminf(s.mn, x[k]);
+        }
+    }
+    for (int j = j0; j < j1; ++j) {
+        ptx::tmem_ld32(taddr + 32 * j, x);
+        ptx::tmem_wait_ld();
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+            s.sp += ex2((x[k] - s.mp) * kLog2e);
+            s.sn += ex2((s.mn - x[k]) * kLog2e);
+        }
+    }
+    return s;
+}
+// Statistics of the whole row from the two halves' (a first, then b: both threads
+// of a row combine in the same order and get the same bits).
+__device__ __forceinline__ PhiStats combine_stats(const PhiStats &a, const PhiStats &b)
+{
+    PhiStats s;
+    s.mp = fmaxf(a.mp, b.mp);
+    s.mn = fminf(a.mn, b.mn);
+    s.sp = a.sp * ex2((a.mp - s.mp) * kLog2e) + b.sp * ex2((b.mp - s.mp) * kLog2e);
+    s.sn = a.sn * ex2((s.mn - a.mn) * kLog2e) + b.sn * ex2((s.mn - b.mn) * kLog2e);
+    return s;
+}
+
 // Shared memory of the row kernels (bytes, all 1024-aligned)
 struct RowLayout {
-    uint32_t off_q, off_w, off_k, off_v, off_do, off_phi, off_y, off_z, off_bar, bytes;
+    uint32_t off_q, off_w, off_k, off_v, off_do, off_phi, off_y, off_z, off_x, off_bar, bytes;
     uint32_t off_ring, ring_slot;
 };
 
@@ -165,6 +205,8 @@ RowLayout make_grad_layout(int d, int F, int B)
     off += (uint32_t)((d + 16 + 63) / 64) * 128 * 128;
     Lr.off_z = off;
     off += (((uint32_t)2 * F * 4) + 1023) & ~1023u;
+    Lr.off_x = off;
+    off += kXchBytes;
     Lr.off_bar = off;
     off += 1024;
     Lr.bytes = off + 1024;
@@ -457,12 +499,15 @@ __global__ void k_slot_scan(float *buf0, float *buf1, int n_seq, int n_slots, si
 // k_phi_grad<kQuery>: one (sequence s, block n, state head g).
 // ---------------------------------------------------------------------------
 template <bool kQuery>
-__global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant__ TrainArgs a, RowLayout Lr)
+__global__ void __launch_bounds__(kGradThreads, 1) k_phi_grad(const __grid_constant__ TrainArgs a, RowLayout Lr)
 {
     using namespace ptx;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = aligned_smem(smem_raw);
     const int tid = threadIdx.x, warp = tid >> 5;
+    // two threads per Tensor Memory lane (row): lr = the lane, part = which half of each
+    // row's columns the thread takes; warps w and w + 4 share lanes 32 (w & 3) ..
+    const int lr = tid & 127, part = tid >> 7;
     const int d = a.d, F = a.F, B = a.B, Hkv = a.Hkv, Hq = a.Hq, G = Hq / Hkv;
     const int g = blockIdx.x % Hkv, n = (blockIdx.x / Hkv) % a.n_blk, s = blockIdx.x / (Hkv * a.n_blk);
     // Rows of the tile on Tensor Memory lanes: query side, lane r < G*B is token r / G,
@@ -502,7 +547,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         tmem_relinquish();
     }
     // rows of the M = 128 operands beyond the tile stay zero (the TMA boxes fill rows < rows)
-    for (int i = tid; i < (128 - rows) * (d / 8); i += kThreads) {
+    for (int i = tid; i < (128 - rows) * (d / 8); i += kGradThreads) {
         const int r = rows + i / (d / 8), c8 = i % (d / 8);
         const uint32_t off = (uint32_t)(c8 >> 3) * (128 * 128) + swz(r, c8 & 7);
         *reinterpret_cast<uint4 *>(smem + Lr.off_q + off) = make_uint4(0, 0, 0, 0);
@@ -528,7 +573,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         }
         for (int p = 0; p < F / 64; ++p) tma_load_2d(smem + Lr.off_w + p * d * 128, &a.tmW, 64 * p, g * d, tbar);
     }
-    for (int f = tid; f < 2 * F; f += kThreads) sZ[f] = src[z_offset(f, d, F)];
+    for (int f = tid; f < 2 * F; f += kGradThreads) sZ[f] = src[z_offset(f, d, F)];
     bool ok = wait_bar(tbar, 0, fail);
     fence_proxy_async_smem();
     __syncthreads();
@@ -568,64 +613,89 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         }
     }
 
-    // ---- row statistics (thread = row) ----
-    const bool valid = tid < rows;
-    const int hl = (kQuery && valid) ? tid % G : 0;                // query head within the group
-    const int tok = valid ? (kQuery ? tid / G : tid) : 0;          // token within the block
+    // ---- row statistics: the two parts of a row each take half of its columns and
+    // exchange partial sums through shared memory (pair barrier of warps w, w + 4) ----
+    const bool valid = lr < rows;
+    const int hl = (kQuery && valid) ? lr % G : 0;                 // query head within the group
+    const int tok = valid ? (kQuery ? lr / G : lr) : 0;            // token within the block
     const size_t q_row = (size_t)Hq * d;
-    const PhiStats st = phi_stats(tl + kColU, F);
+    const uint32_t pair_bar = 2 + (uint32_t)(warp & 3);
+    float *x1 = reinterpret_cast<float *>(smem + Lr.off_x);        // [2][128][8] statistics
+    float *x2 = x1 + 2 * 128 * 8;                                  // [2][128]    lin_den
+    float *x3 = x2 + 2 * 128;                                      // [2][128][4] pass-0 dots
+    const int uj0 = part * (F / 64), uj1 = uj0 + F / 64;           // this part's 32-column chunks of U
+    const float scale = rsqrtf((float)d);
+    float w = 0.f;
+    if (kQuery) {
+        const float alpha = valid ? a.alpha[g * G + hl] : 0.f;
+        w = 1.f / (1.f + expf(-alpha));
+    }
+    PhiStats st;
+    {
+        const PhiStats mine = phi_stats_chunks(tl + kColU, uj0, uj1);
+        float *o = x1 + (part * 128 + lr) * 8;
+        o[0] = mine.mp; o[1] = mine.sp; o[2] = mine.mn; o[3] = mine.sn;
+        if (kQuery) {
+            // scores: this part's 16-column chunks j = part, part + 2, ..: m, sum e^(s - m), sum e^(s - m) g.v
+            float m = -INFINITY, l = 0.f, an = 0.f;
+            for (int j = part; j < B / 16; j += 2) {
+                float x[16];
+                tmem_ld16(tl + kColS + 16 * j, x);
+                tmem_wait_ld();
+#pragma unroll
+                for (int k = 0; k < 16; ++k) m = fmaxf(m, x[k] * scale);
+            }
+            for (int j = part; j < B / 16; j += 2) {
+                float x[16], y[16];
+                tmem_ld16(tl + kColS + 16 * j, x);
+                tmem_ld16(tl + kColGv + 16 * j, y);
+                tmem_wait_ld();
+#pragma unroll
+                for (int k = 0; k < 16; ++k) {
+                    const float e = ex2((x[k] * scale - m) * kLog2e);
+                    l += e;
+                    an += e * y[k];
+                }
+            }
+            o[4] = m; o[5] = l; o[6] = an;
+        }
+        named_bar(pair_bar, 64);
+        const float *o0 = x1 + lr * 8, *o1 = x1 + (128 + lr) * 8;
+        st = combine_stats(PhiStats{o0[0], o0[1], o0[2], o0[3]}, PhiStats{o1[0], o1[1], o1[2], o1[3]});
+    }
     const float ip = 1.f / st.sp, in = 1.f / st.sn;
-    // Query rows: w, 1/D, and the merge terms A = g.sm_num / D, beta = sm_den / D,
+    // Query rows: 1/D and the merge terms A = g.sm_num / D, beta = sm_den / D,
     // lambda = lin_den / D; after S dN, Lambda = g.lin_num / D = phi(q).(S dN)
     // gives g.o = w A + Lambda and dw = lambda A - beta Lambda (= dN.sm_num + dD sm_den).
-    float w = 0.f, inv = 0.f, A = 0.f, beta = 0.f, lambda = 0.f;
+    float inv = 0.f, A = 0.f, beta = 0.f, lambda = 0.f;
     if (kQuery) {
-        const int h = g * G + hl;
-        const float alpha = valid ? a.alpha[h] : 0.f;
-        w = 1.f / (1.f + expf(-alpha));
-        // phi(q) into its operand image; lin_den = phi(q) . z
-        float lin_den = 0.f;
+        // phi(q) of this part's columns into its operand image; partial lin_den = phi(q) . z
+        float ld = 0.f;
         {
             float x[32], yp[32], yn[32];
-            for (int j = 0; j < F / 32; ++j) {
+            for (int j = uj0; j < uj1; ++j) {
                 tmem_ld32(tl + kColU + 32 * j, x);
                 tmem_wait_ld();
 #pragma unroll
                 for (int k = 0; k < 32; ++k) {
                     yp[k] = valid ? ex2((x[k] - st.mp) * kLog2e) * ip : 0.f;
                     yn[k] = valid ? ex2((st.mn - x[k]) * kLog2e) * in : 0.f;
-                    lin_den += yp[k] * sZ[32 * j + k] + yn[k] * sZ[F + 32 * j + k];
+                    ld += yp[k] * sZ[32 * j + k] + yn[k] * sZ[F + 32 * j + k];
                 }
-                store_row32_bf16(smem + Lr.off_phi, 128 * 128, tid, 32 * j, yp);
-                store_row32_bf16(smem + Lr.off_phi, 128 * 128, tid, F + 32 * j, yn);
+                store_row32_bf16(smem + Lr.off_phi, 128 * 128, lr, 32 * j, yp);
+                store_row32_bf16(smem + Lr.off_phi, 128 * 128, lr, F + 32 * j, yn);
             }
         }
-        // scores, shift c, D' = w sum_j e^(s_j - c) + lin_den e^(-c)  (D = e^c D')
-        const float scale = rsqrtf((float)d);
-        float m = -INFINITY;
-        for (int j = 0; j < B / 16; ++j) {
-            float x[16];
-            tmem_ld16(tl + kColS + 16 * j, x);
-            tmem_wait_ld();
-#pragma unroll
-            for (int k = 0; k < 16; ++k) m = fmaxf(m, x[k] * scale);
-        }
+        x2[part * 128 + lr] = ld;
+        named_bar(pair_bar, 64);
+        const float lin_den = x2[lr] + x2[128 + lr];
+        // scores of the whole row: shift c, D' = w sum_j e^(s_j - c) + lin_den e^(-c) (D = e^c D')
+        const float *o0 = x1 + lr * 8, *o1 = x1 + (128 + lr) * 8;
+        const float m = fmaxf(o0[4], o1[4]);
         float c = m;
         if (lin_den > 0.f) c = w > 0.f ? fmaxf(m, logf(lin_den) - logf(w)) : logf(lin_den);
-        // l = sum_j e^(s_j - c), an = sum_j e^(s_j - c) g.v_j
-        float l = 0.f, an = 0.f;
-        for (int j = 0; j < B / 16; ++j) {
-            float x[16], y[16];
-            tmem_ld16(tl + kColS + 16 * j, x);
-            tmem_ld16(tl + kColGv + 16 * j, y);
-            tmem_wait_ld();
-#pragma unroll
-            for (int k = 0; k < 16; ++k) {
-                const float e = ex2((x[k] * scale - c) * kLog2e);
-                l += e;
-                an += e * y[k];
-            }
-        }
+        const float e0 = ex2((o0[4] - c) * kLog2e), e1 = o1[4] == -INFINITY ? 0.f : ex2((o1[4] - c) * kLog2e);
+        const float l = o0[5] * e0 + o1[5] * e1, an = o0[6] * e0 + o1[6] * e1;
         const float ec = ex2(-c * kLog2e);
         const float Dp = w * l + lin_den * ec;
         inv = valid ? ec / Dp : 0.f;              // 1 / D
@@ -633,56 +703,61 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         beta = l * pw;
         lambda = lin_den * inv;
         A = an * pw;                              // sum_j (e^(s_j) / D) g.v_j
-        // dN = g / D: Tensor Memory (fp32, A operand of S dN) and the operand image (bf16);
-        // the row's d values are loaded at once (16 x 16 bytes in flight)
-        const uint4 *grow = reinterpret_cast<const uint4 *>(a.dO + (t0 + tok) * q_row + (size_t)(g * G + hl) * d);
-        uint4 graw[16];
+        // dN = g / D of this part's half of the columns: Tensor Memory (fp32, A operand
+        // of S dN) and the operand image (bf16); its d/2 values are loaded at once
+        const uint4 *grow = reinterpret_cast<const uint4 *>(a.dO + (t0 + tok) * q_row + (size_t)(g * G + hl) * d) +
+                            part * (d / 16);
+        uint4 graw[8];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) graw[i] = (valid && i < d / 8) ? __ldg(grow + i) : make_uint4(0, 0, 0, 0);
+        for (int i = 0; i < 8; ++i) graw[i] = (valid && i < d / 16) ? __ldg(grow + i) : make_uint4(0, 0, 0, 0);
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            if (c < d / 32) {
+        for (int cc = 0; cc < 2; ++cc) {
+            if (cc < d / 64) {
                 float gv[32];
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
-                    const uint32_t w4[4] = {graw[4 * c + i].x, graw[4 * c + i].y, graw[4 * c + i].z, graw[4 * c + i].w};
+                    const uint4 q4 = graw[4 * cc + i];
+                    const uint32_t w4[4] = {q4.x, q4.y, q4.z, q4.w};
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        gv[8 * i + 2 * j] = __uint_as_float(w4[j] << 16) * inv;
-                        gv[8 * i + 2 * j + 1] = __uint_as_float(w4[j] & 0xFFFF0000u) * inv;
+                    for (int jj = 0; jj < 4; ++jj) {
+                        gv[8 * i + 2 * jj] = __uint_as_float(w4[jj] << 16) * inv;
+                        gv[8 * i + 2 * jj + 1] = __uint_as_float(w4[jj] & 0xFFFF0000u) * inv;
                     }
                 }
-                tmem_st32(tl + kColY + 32 * c, gv);
-                store_row32_bf16(smem + Lr.off_y, 128 * 128, tid, 32 * c, gv);
+                const int col = part * (d / 2) + 32 * cc;
+                tmem_st32(tl + kColY + col, gv);
+                store_row32_bf16(smem + Lr.off_y, 128 * 128, lr, col, gv);
             }
         }
     } else {
-        // V rows (fp32) as the Tensor Memory A operand of R v; r enters with coefficient 1
-        const uint4 *vrow = reinterpret_cast<const uint4 *>(a.V + (t0 + tok) * kv_row + (size_t)g * d);
-        uint4 vraw[16];
+        // V rows (fp32, this part's half of the columns) as the Tensor Memory A operand of
+        // R v; r enters with coefficient 1
+        const uint4 *vrow = reinterpret_cast<const uint4 *>(a.V + (t0 + tok) * kv_row + (size_t)g * d) + part * (d / 16);
+        uint4 vraw[8];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) vraw[i] = (valid && i < d / 8) ? __ldg(vrow + i) : make_uint4(0, 0, 0, 0);
+        for (int i = 0; i < 8; ++i) vraw[i] = (valid && i < d / 16) ? __ldg(vrow + i) : make_uint4(0, 0, 0, 0);
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            if (c < d / 32) {
+        for (int cc = 0; cc < 2; ++cc) {
+            if (cc < d / 64) {
                 float vv[32];
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
-                    const uint32_t w4[4] = {vraw[4 * c + i].x, vraw[4 * c + i].y, vraw[4 * c + i].z, vraw[4 * c + i].w};
+                    const uint4 q4 = vraw[4 * cc + i];
+                    const uint32_t w4[4] = {q4.x, q4.y, q4.z, q4.w};
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        vv[8 * i + 2 * j] = __uint_as_float(w4[j] << 16);
-                        vv[8 * i + 2 * j + 1] = __uint_as_float(w4[j] & 0xFFFF0000u);
+                    for (int jj = 0; jj < 4; ++jj) {
+                        vv[8 * i + 2 * jj] = __uint_as_float(w4[jj] << 16);
+                        vv[8 * i + 2 * jj + 1] = __uint_as_float(w4[jj] & 0xFFFF0000u);
                     }
                 }
-                tmem_st32(tl + kColY + 32 * c, vv);
+                tmem_st32(tl + kColY + part * (d / 2) + 32 * cc, vv);
             }
         }
     }
     tmem_wait_st();
     fence_proxy_async_smem();
     tc_fence_before();
-    const bool failed1 = group_sync_failed(1, kThreads, !ok);
+    const bool failed1 = group_sync_failed(1, kGradThreads, !ok);
     tc_fence_after();
 
     // ---- dphi = [S | z] [dN; dD] (query) or [R | r] [v; 1] (key): tiles of 32 e ----
@@ -712,15 +787,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         if (!ok) atomicOr(const_cast<int *>(fail), 1);
     }
     if (!failed1) ok = wait_bar(mbar, 1, fail) && ok;
+    tc_fence_before();
+    // one decision for the whole CTA: the pair barriers below need both parts of a row
+    const bool failedC = group_sync_failed(1, kGradThreads, failed1 || !ok || *fail);
     tc_fence_after();
 
     // ---- du = p+ (g+ - <g+, p+>) - p- (g- - <g-, p->) with g = G + zeta dD, where
-    // G = S dN (query) or R v (key) and zeta = z_{n-1} (query) or r_m (key) ----
-    if (!failed1 && !*fail) {
+    // G = S dN (query) or R v (key) and zeta = z_{n-1} (query) or r_m (key); each part
+    // takes its half of the features ----
+    if (!failedC) {
         float x[32], gp[32], gn[32];
-        // pass 0: Lambda+- = <G+-, p+->, Z+- = <zeta+-, p+->
+        // pass 0: Lambda+- = <G+-, p+->, Z+- = <zeta+-, p+-> over this part's features
         float Lp = 0.f, Ln = 0.f, Zp = 0.f, Zn = 0.f;
-        for (int j = 0; j < F / 32; ++j) {
+        for (int j = uj0; j < uj1; ++j) {
             tmem_ld32(tl + kColU + 32 * j, x);
             tmem_ld32(tl + kColG + 32 * j, gp);
             tmem_ld32(tl + kColG + F + 32 * j, gn);
@@ -735,22 +814,34 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
                 Zn += sZ[F + 32 * j + k] * pn;
             }
         }
+        {
+            float *o = x3 + (part * 128 + lr) * 4;
+            o[0] = Lp; o[1] = Ln; o[2] = Zp; o[3] = Zn;
+            named_bar(pair_bar, 64);
+            const float *o0 = x3 + lr * 4, *o1 = x3 + (128 + lr) * 4;
+            Lp = o0[0] + o1[0];
+            Ln = o0[1] + o1[1];
+            Zp = o0[2] + o1[2];
+            Zn = o0[3] + o1[3];
+        }
         float dD = valid ? 1.f : 0.f;
         if (kQuery) {
             const float Lam = Lp + Ln;
             dD = -(w * A + Lam) * inv;   // -(g . o) / D
-            if (valid) atomicAdd(&sDw[hl], lambda * A - beta * Lam);
-            // column d of [dN | dD | 0] (the rest of that 32-column group is never read)
-            uint8_t *base = smem + Lr.off_y + (uint32_t)(d >> 6) * (128 * 128);
-            uint4 v0;
-            v0.x = pack_bf16x2(dD, 0.f);
-            v0.y = v0.z = v0.w = 0u;
-            *reinterpret_cast<uint4 *>(base + swz(tid, 0)) = v0;
-            *reinterpret_cast<uint4 *>(base + swz(tid, 1)) = make_uint4(0, 0, 0, 0);
+            if (part == 0) {
+                if (valid) atomicAdd(&sDw[hl], lambda * A - beta * Lam);
+                // column d of [dN | dD | 0] (the rest of that 32-column group is never read)
+                uint8_t *base = smem + Lr.off_y + (uint32_t)(d >> 6) * (128 * 128);
+                uint4 v0;
+                v0.x = pack_bf16x2(dD, 0.f);
+                v0.y = v0.z = v0.w = 0u;
+                *reinterpret_cast<uint4 *>(base + swz(lr, 0)) = v0;
+                *reinterpret_cast<uint4 *>(base + swz(lr, 1)) = make_uint4(0, 0, 0, 0);
+            }
         }
         const float dotp = Lp + dD * Zp, dotn = Ln + dD * Zn;
-        // pass 1: du
-        for (int j = 0; j < F / 32; ++j) {
+        // pass 1: du of this part's features
+        for (int j = uj0; j < uj1; ++j) {
             tmem_ld32(tl + kColU + 32 * j, x);
             tmem_ld32(tl + kColG + 32 * j, gp);
             tmem_ld32(tl + kColG + F + 32 * j, gn);
@@ -782,7 +873,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
     }
     fence_proxy_async_smem();
     tc_fence_before();
-    const bool failed2 = group_sync_failed(1, kThreads, failed1 || !ok || *fail);
+    const bool failed2 = group_sync_failed(1, kGradThreads, failedC || !ok || *fail);
     tc_fence_after();
 
     // ---- query side: dR_n = phi(Q)^T [dN | dD], the gate, and the R slot ----
@@ -808,7 +899,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
         // R's slot: per e-tile c the 2F feature rows (2F x 128 bytes, contiguous in global
         // memory) are staged in the space of phi(Q) and [dN | dD], which the dR MMAs have
         // consumed, laid out as in global memory, and written by bulk copies
-        if (!group_sync_failed(1, kThreads, !ok)) {
+        if (!group_sync_failed(1, kGradThreads, !ok)) {
             float *R = a.R + (((size_t)s * a.n_blk + n) * Hkv + g) * hf;
             const uint32_t tile_bytes = (uint32_t)2 * F * 128;
             for (int c = 0; c < d / 32; ++c) {
@@ -818,8 +909,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
                     if (tid == 0) bulk_wait_read_all();
                     __syncthreads();
                 }
-                for (int i = 0; i < NM; ++i) {
-                    const int f = 128 * i + tid;
+                // part p stages the features of M-block p (with one block, part 0 alone)
+                for (int i = part; i < NM; i += 2) {
+                    const int f = 128 * i + lr;
                     float x[32];
                     tmem_ld32(tl + kColDR + (uint32_t)(i * NYS + 32 * c), x);
                     tmem_wait_ld();
@@ -835,11 +927,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_phi_grad(const __grid_constant_
                     bulk_commit();
                 }
             }
-            for (int i = 0; i < NM; ++i) {
+            for (int i = part; i < NM; i += 2) {
                 float zz[16];
                 tmem_ld16(tl + kColDR + (uint32_t)(i * NYS + d), zz);
                 tmem_wait_ld();
-                R[z_offset(128 * i + tid, d, F)] = zz[0];
+                R[z_offset(128 * i + lr, d, F)] = zz[0];
             }
             if (tid == 0) bulk_wait_all();
         } else {
@@ -1184,13 +1276,15 @@ cudaError_t launch_train_backward(const hybrid_cfg &c, const void *Q, const void
     const RowLayout Lg = make_grad_layout(a.d, a.F, a.B);
     if ((e = opt_in(k_phi_grad<true>, g_opt_q)) != cudaSuccess) return e;
     if ((e = opt_in(k_phi_grad<false>, g_opt_k)) != cudaSuccess) return e;
-    if ((e = launch_pdl(k_phi_grad<true>, dim3((unsigned)units), dim3(kThreads), Lg.bytes, st, a, Lg)) != cudaSuccess)
+    if ((e = launch_pdl(k_phi_grad<true>, dim3((unsigned)units), dim3(kGradThreads), Lg.bytes, st, a, Lg)) !=
+        cudaSuccess)
         return e;
     const size_t n4 = sf / 4 * (size_t)n_seq;
     if ((e = launch_pdl(k_slot_scan, dim3((unsigned)((n4 + 255) / 256), 1), dim3(256), 0, st, a.R,
                         static_cast<float *>(nullptr), n_seq, a.n_blk, sf, true)) != cudaSuccess)
         return e;
-    if ((e = launch_pdl(k_phi_grad<false>, dim3((unsigned)units), dim3(kThreads), Lg.bytes, st, a, Lg)) != cudaSuccess)
+    if ((e = launch_pdl(k_phi_grad<false>, dim3((unsigned)units), dim3(kGradThreads), Lg.bytes, st, a, Lg)) !=
+        cudaSuccess)
         return e;
     DwArgs b{};
     b.Q = a.Q;
