@@ -556,6 +556,11 @@ __global__ void __launch_bounds__(kGradThreads, 1) k_phi_grad(const __grid_const
     __syncthreads();
     griddep_wait();
 
+    // ring of S / R tiles: in the phase-one operands' space on the query side (free once
+    // the first MMAs have run); the key side has phi's space to itself, so its first two
+    // tiles are loaded right away, next to the operands
+    const uint32_t ring_off = kQuery ? Lr.off_ring : Lr.off_phi;
+    int loads_issued = 0;
     // phase one by TMA: [U | scores] = Q [W | K^T] and dO V^T (query side) or U = K W
     if (tid == 0) {
         const uint32_t qbytes = (uint32_t)(d / 64) * rows * 128, kvbytes = (uint32_t)(d / 64) * B * 128;
@@ -572,6 +577,12 @@ __global__ void __launch_bounds__(kGradThreads, 1) k_phi_grad(const __grid_const
             }
         }
         for (int p = 0; p < F / 64; ++p) tma_load_2d(smem + Lr.off_w + p * d * 128, &a.tmW, 64 * p, g * d, tbar);
+        if (!kQuery)
+            for (int c = 0; c < 2 && c < d / 32; ++c) {
+                mbar_arrive_expect_tx(&full[c], Lr.ring_slot);
+                bulk_g2s(smem + ring_off + c * Lr.ring_slot, src + (size_t)c * 64 * F, Lr.ring_slot, &full[c]);
+                ++loads_issued;
+            }
     }
     for (int f = tid; f < 2 * F; f += kGradThreads) sZ[f] = src[z_offset(f, d, F)];
     bool ok = wait_bar(tbar, 0, fail);
@@ -582,8 +593,7 @@ __global__ void __launch_bounds__(kGradThreads, 1) k_phi_grad(const __grid_const
     const uint32_t lane_off = (uint32_t)(warp & 3) * 32u << 16;
     const uint32_t tl = tmem + lane_off;
     const int NCHUNK = d / 32;
-    const uint32_t ring_u = smem_u32(smem + Lr.off_ring);
-    int loads_issued = 0;
+    const uint32_t ring_u = smem_u32(smem + ring_off);
     if (tid == 0) {
         const uint32_t q_u = smem_u32(smem + Lr.off_q), w_u = smem_u32(smem + Lr.off_w);
         const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
@@ -604,11 +614,11 @@ __global__ void __launch_bounds__(kGradThreads, 1) k_phi_grad(const __grid_const
     }
     ok = wait_bar(mbar, 0, fail) && ok;
     tc_fence_after();
-    // the phase-one operands are consumed: the first two tiles go into their space
-    if (tid == 0 && ok) {
+    // query side: the phase-one operands are consumed, the first two tiles go into their space
+    if (kQuery && tid == 0 && ok) {
         for (int c = 0; c < 2 && c < NCHUNK; ++c) {
             mbar_arrive_expect_tx(&full[c], Lr.ring_slot);
-            bulk_g2s(smem + Lr.off_ring + c * Lr.ring_slot, src + (size_t)c * 64 * F, Lr.ring_slot, &full[c]);
+            bulk_g2s(smem + ring_off + c * Lr.ring_slot, src + (size_t)c * 64 * F, Lr.ring_slot, &full[c]);
             ++loads_issued;
         }
     }
@@ -778,7 +788,7 @@ __global__ void __launch_bounds__(kGradThreads, 1) k_phi_grad(const __grid_const
                 ok = wait_bar(&empty[slot], (uint32_t)(c >> 1) & 1u, fail);
                 if (!ok) break;
                 mbar_arrive_expect_tx(&full[slot], Lr.ring_slot);
-                bulk_g2s(smem + Lr.off_ring + slot * Lr.ring_slot, src + (size_t)(c + 2) * 64 * F, Lr.ring_slot,
+                bulk_g2s(smem + ring_off + slot * Lr.ring_slot, src + (size_t)(c + 2) * 64 * F, Lr.ring_slot,
                          &full[slot]);
                 ++loads_issued;
             }
