@@ -84,10 +84,7 @@ __device__ __forceinline__ uint32_t swz(int r, int j)
     return (uint32_t)r * 128u + (uint32_t)((j ^ (r & 7)) << 4);
 }
 
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 // Write 32 consecutive columns [c0, c0 + 32) of row r (values x, converted to
 // bf16) into a bf16 operand image with panel stride pstride.
@@ -963,18 +960,22 @@ __global__ void __launch_bounds__(kGradThreads, 1) k_phi_grad(const __grid_const
 }
 
 // ---------------------------------------------------------------------------
-// k_dw: dW_g += sum over a range of rows of x du^T.  Row rho of group g: token
-// t = rho / (G+1); kinds 0..G-1 are the query heads of the group (Q, dU_q),
-// kind G is the key (K, dU_k).  128 rows per step, three shared-memory stages
-// (copies two steps ahead); the accumulator (d lanes x F columns) stays in
-// Tensor Memory over the range.
+// k_dw: dW_g += sum over a range of rows of x du^T.  The rows of group g come in
+// 128-token chunks: G query tiles of 128 / G tokens x G heads (Q, dU_q) and one key
+// tile of 128 tokens (K, dU_k), each a TMA box of 128 rows in (token, head) order
+// for both operands (rows past the batch read zeros).  One thread runs a ring of
+// three shared-memory stages (boxes in flight two steps ahead, each stage freed by
+// the commit of its MMAs); the accumulator (d lanes x F columns) stays in Tensor
+// Memory over the CTA's range of tiles.
 // ---------------------------------------------------------------------------
 struct DwArgs {
-    const bf16 *Q, *K, *dUq, *dUk;
+    // X and dU boxes of 128 rows in the same (token, head) order: Q / dU_q with box
+    // {64, G, 128 / G}, K / dU_k with box {64, 1, 128}
+    CUtensorMap tmXq, tmUq, tmXk, tmUk;
     float *dW;
     unsigned *err;
-    long long n_tok;   // n_seq * L
-    int Hq, Hkv, d, F, tiles_per_cta, ctas_per_group;
+    int n_chunks;      // 128-token chunks of the batch
+    int G, d, F, tiles_per_cta, ctas_per_group;
 };
 
 __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwArgs a)
@@ -983,21 +984,27 @@ __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwAr
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = aligned_smem(smem_raw);
     const int tid = threadIdx.x, warp = tid >> 5;
-    const int d = a.d, F = a.F, G = a.Hq / a.Hkv, K1 = G + 1;
+    const int d = a.d, F = a.F, G = a.G, K1 = G + 1;
     const int g = blockIdx.x / a.ctas_per_group, part = blockIdx.x % a.ctas_per_group;
-    const long long total = a.n_tok * K1;
-    const long long r_begin = (long long)part * a.tiles_per_cta * 128;
-    long long r_end = r_begin + (long long)a.tiles_per_cta * 128;
-    if (r_end > total) r_end = total;
-    const int n_tiles = r_begin < total ? (int)((r_end - r_begin + 127) / 128) : 0;
+    // tiles of group g: chunk c has G query tiles (kind < G) then the key tile (kind G)
+    const int total = a.n_chunks * K1;
+    const int t_begin = part * a.tiles_per_cta;
+    const int n_tiles = max(0, min(a.tiles_per_cta, total - t_begin));
     const uint32_t xbytes = 2 * 128 * 128, ubytes = (uint32_t)(F / 64) * 128 * 128, stage = xbytes + ubytes;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kDwStages * stage);   // [kDwStages] MMAs of a stage done
-    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + kDwStages);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kDwStages * stage);
+    uint64_t *full = bars;                   // [kDwStages] a stage's boxes have landed
+    uint64_t *empty = bars + kDwStages;      // [kDwStages] the MMAs of a stage are done
+    uint64_t *done = bars + 2 * kDwStages;   // every MMA of the CTA is done
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 2 * kDwStages + 1);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
     if (tid == 0) {
-        for (int i = 0; i < kDwStages; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 2 * kDwStages + 1; ++i) mbar_init(&bars[i], 1);
         *fail = 0;
         fence_mbar_init();
+        prefetch_tensormap(&a.tmXq);
+        prefetch_tensormap(&a.tmUq);
+        prefetch_tensormap(&a.tmXk);
+        prefetch_tensormap(&a.tmUk);
     }
     if (warp == 0) {
         tmem_alloc(tmem_holder, 128);
@@ -1009,79 +1016,53 @@ __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwAr
             const int st = i / 1024, k = i % 1024;
             reinterpret_cast<uint4 *>(smem + st * stage + 128 * 128)[k] = make_uint4(0, 0, 0, 0);
         }
-    griddep_wait();
+    fence_proxy_async_smem();
     __syncthreads();
+    griddep_wait();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
-    const uint32_t idW = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, F);
     bool ok = true;
-    // copies of step k into stage k % kDwStages: row tid of the step (16-byte
-    // cp.async, one group per step), issued two steps ahead of the MMAs
-    auto issue = [&](int k) {
-        uint8_t *sx = smem + (k % kDwStages) * stage, *su = sx + xbytes;
-        const long long rho = r_begin + (long long)k * 128 + tid;
-        const bool valid = rho < r_end;
-        const bf16 *xr = nullptr, *ur = nullptr;
-        if (valid) {
-            const long long t = rho / K1;
-            const int kind = (int)(rho - t * K1);
-            if (kind < G) {
-                const size_t h = (size_t)g * G + kind;
-                xr = a.Q + ((size_t)t * a.Hq + h) * d;
-                ur = a.dUq + ((size_t)t * a.Hq + h) * F;
-            } else {
-                xr = a.K + ((size_t)t * a.Hkv + g) * d;
-                ur = a.dUk + ((size_t)t * a.Hkv + g) * F;
-            }
-        }
-        for (int c8 = 0; c8 < d / 8; ++c8) {
-            uint8_t *dst = sx + (uint32_t)(c8 >> 3) * (128 * 128) + swz(tid, c8 & 7);
-            if (valid)
-                cp_async16(dst, reinterpret_cast<const uint4 *>(xr) + c8);
-            else
-                *reinterpret_cast<uint4 *>(dst) = make_uint4(0, 0, 0, 0);
-        }
-        for (int c8 = 0; c8 < F / 8; ++c8) {
-            uint8_t *dst = su + (uint32_t)(c8 >> 3) * (128 * 128) + swz(tid, c8 & 7);
-            if (valid)
-                cp_async16(dst, reinterpret_cast<const uint4 *>(ur) + c8);
-            else
-                *reinterpret_cast<uint4 *>(dst) = make_uint4(0, 0, 0, 0);
-        }
-        cp_async_commit();
-    };
-    // the MMAs of step k commit to bars[k % kDwStages]: its (k / kDwStages)-th phase
-    if (n_tiles > 0) issue(0);
-    if (n_tiles > 1) issue(1);
-    for (int k = 0; k < n_tiles; ++k) {
-        if (k + 2 < n_tiles) {
-            // stage (k + 2) % kDwStages was last read by the MMAs of step k - 1
-            if (k >= 1)
-                ok = wait_bar(&bars[(k - 1) % kDwStages], (uint32_t)((k - 1) / kDwStages) & 1u, fail) && ok;
-            issue(k + 2);
-            cp_async_wait<2>();
-        } else if (k + 1 < n_tiles) {
-            cp_async_wait<1>();
-        } else {
-            cp_async_wait<0>();
-        }
-        fence_proxy_async_smem();
-        if (group_sync_failed(1, kThreads, !ok)) break;
-        if (tid == 0) {
+    int issued = 0;
+    if (tid == 0 && n_tiles > 0) {
+        const uint32_t idW = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, F);
+        // step k (tile t_begin + k) into stage k % kDwStages
+        auto issue = [&](int k) {
+            const int t = t_begin + k, c = t / K1, kind = t % K1;
+            uint8_t *sx = smem + (k % kDwStages) * stage, *su = sx + xbytes;
+            uint64_t *bar = &full[k % kDwStages];
+            mbar_arrive_expect_tx(bar, (uint32_t)(d / 64) * 128 * 128 + ubytes);
+            const bool q = kind < G;
+            const int tok = c * 128 + (q ? kind * (128 / G) : 0);
+            for (int p = 0; p < d / 64; ++p)
+                tma_load_3d(sx + p * 128 * 128, q ? &a.tmXq : &a.tmXk, 64 * p, q ? g * G : g, tok, bar);
+            for (int p = 0; p < F / 64; ++p)
+                tma_load_3d(su + p * 128 * 128, q ? &a.tmUq : &a.tmUk, 64 * p, q ? g * G : g, tok, bar);
+            ++issued;
+        };
+        for (int k = 0; k < kDwStages && k < n_tiles; ++k) issue(k);
+        for (int k = 0; k < n_tiles && ok; ++k) {
+            ok = wait_bar(&full[k % kDwStages], (uint32_t)(k / kDwStages) & 1u, fail);
+            if (!ok) break;
             tc_fence_after();
             const uint32_t x_u = smem_u32(smem + (k % kDwStages) * stage), u_u = x_u + xbytes;
             for (int ks = 0; ks < 8; ++ks)
                 mma_bf16_ss(tmem, smem_desc(x_u + ks * 2048, 128 * 128, 1024, SWZ_128B),
                             smem_desc(u_u + ks * 2048, 128 * 128, 1024, SWZ_128B), idW, (k | ks) != 0);
-            mma_commit(&bars[k % kDwStages]);
+            mma_commit(&empty[k % kDwStages]);
+            // refill the previous step's stage once its MMAs are done
+            const int kn = k - 1 + kDwStages;
+            if (k >= 1 && kn < n_tiles) {
+                ok = wait_bar(&empty[(k - 1) % kDwStages], (uint32_t)((k - 1) / kDwStages) & 1u, fail);
+                if (ok) issue(kn);
+            }
         }
+        mma_commit(done);
+        if (!ok) atomicOr(const_cast<int *>(fail), 1);
     }
-    cp_async_wait<0>();
-    // the last steps (those not waited for in the loop)
-    for (int k = n_tiles - kDwStages; k < n_tiles; ++k)
-        if (k >= 0) ok = wait_bar(&bars[k % kDwStages], (uint32_t)(k / kDwStages) & 1u, fail) && ok;
+    if (n_tiles > 0) ok = wait_bar(done, 0, fail) && ok;
     tc_fence_after();
-    if (ok && n_tiles > 0 && tid < d) {
+    const bool failed = group_sync_failed(1, kThreads, !ok);
+    if (!failed && n_tiles > 0 && tid < d) {
         float *dst = a.dW + ((size_t)g * d + tid) * F;
         const uint32_t lane_off = (uint32_t)(warp & 3) * 32u << 16;
         float x[32];
@@ -1091,8 +1072,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwAr
 #pragma unroll
             for (int k = 0; k < 32; ++k) atomicAdd(dst + 32 * j + k, x[k]);
         }
-    } else if (n_tiles > 0 && !ok && tid == 0) {
-        raise_error(a.err, ERR_WAIT_TIMEOUT);
+    }
+    if (tid == 0) {
+        if (failed) raise_error(a.err, ERR_WAIT_TIMEOUT);
+        // no box may still be landing when the CTA leaves
+        for (int k = max(0, issued - kDwStages); k < issued; ++k)
+            mbar_wait(&full[k % kDwStages], (uint32_t)(k / kDwStages) & 1u, kWaitNs);
     }
     tc_fence_before();
     __syncthreads();
@@ -1297,20 +1282,22 @@ cudaError_t launch_train_backward(const hybrid_cfg &c, const void *Q, const void
         cudaSuccess)
         return e;
     DwArgs b{};
-    b.Q = a.Q;
-    b.K = a.K;
-    b.dUq = w.dUq;
-    b.dUk = w.dUk;
+    {
+        const long long n_tok = (long long)n_seq * seq_len;
+        const int G = a.Hq / a.Hkv;
+        if (!encode_rows(&b.tmXq, Q, n_tok, a.Hq, a.d, G, 128 / G) ||
+            !encode_rows(&b.tmUq, w.dUq, n_tok, a.Hq, a.F, G, 128 / G) ||
+            !encode_rows(&b.tmXk, K, n_tok, a.Hkv, a.d, 1, 128) || !encode_rows(&b.tmUk, w.dUk, n_tok, a.Hkv, a.F, 1, 128))
+            return cudaErrorInvalidValue;
+        b.G = G;
+        b.n_chunks = (int)((n_tok + 127) / 128);
+    }
     b.dW = dW;
     b.err = err;
-    b.n_tok = (long long)n_seq * seq_len;
-    b.Hq = a.Hq;
-    b.Hkv = a.Hkv;
     b.d = a.d;
     b.F = a.F;
-    const long long rows = b.n_tok * (a.Hq / a.Hkv + 1);
-    const long long tiles = (rows + 127) / 128;
-    // one CTA per SM (three 64 KB stages each), row ranges split evenly within a group
+    const long long tiles = (long long)b.n_chunks * (b.G + 1);
+    // one CTA per SM (three 64 KB stages each), the group's tiles split evenly
     int per_group = sm_count() / a.Hkv;
     if (per_group > tiles) per_group = (int)tiles;
     if (per_group < 1) per_group = 1;
