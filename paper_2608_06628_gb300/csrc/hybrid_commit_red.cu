@@ -19,6 +19,11 @@
 // accumulates over the unit's chunks in Tensor Memory:
 //   [0,32) and [32,64)   U_k^T of the two chunk buffers
 //   [256,256+F)          dS^T of phi+ features,  [384,384+F) of phi- features
+// With F = 256 the two halves of dS^T (512 columns) do not fit: the unit is then
+// taken in two passes, one per sign of the feature map, each re-forming U_k^T as
+// two 128-feature tiles ([0,32) and [64,96) for buffer 0, +32 for buffer 1), with
+// the math warps' two parts on the two feature tiles instead of the two signs,
+// and dS^T of the pass's sign in [256,512).
 #include <atomic>
 
 #include "hybrid_common.cuh"
@@ -47,6 +52,7 @@ struct CommitArgs {
     void *const *states;
     unsigned *err;
     int n_units, T, Hkv, d, F;
+    int n_pass;             // passes per (request, head): 1, or 2 for F = 256 (one per sign)
     uint32_t off_w, off_c, off_s, off_dz, off_tk, off_bar, chunk_stride;
 };
 
@@ -62,25 +68,28 @@ CLayout make_clayout(int d, int F)
     CLayout L{};
     const uint32_t atom = (uint32_t)d * 128;
     const uint32_t v = (uint32_t)(d / 64) * kChunk * 128;
-    const uint32_t pk = (uint32_t)(2 * F / 64) * kChunk * 128;
+    const int nf = F > 128 ? F : 2 * F;   // phi(K) features of one pass
+    const uint32_t pk = (uint32_t)(nf / 64) * kChunk * 128;
     uint32_t off = 0;
-    L.off_w = off; off += 2 * atom;
+    L.off_w = off; off += (uint32_t)(F / 64 > 2 ? F / 64 : 2) * atom;
     L.chunk = atom + v + pk;
     L.off_c = off; off += 2 * L.chunk;
     L.off_s = off; off += kStage * atom;
     L.off_dz = off; off += (((uint32_t)2 * F * 4) + 1023) & ~1023u;
-    L.off_tk = off; off += 4 * 32 * 4 * 4;
+    L.off_tk = off; off += 512 * 4;
     L.off_bar = off; off += 1024;
     L.bytes = off + 1024;
     if ((int)L.bytes < kOneCtaPerSm) L.bytes = kOneCtaPerSm;
     return L;
 }
 
+// unit u = pass (u % n_pass) of state head g of request r, (r, g) = (u / n_pass) / Hkv, % Hkv
 __device__ __forceinline__ float *unit_head(const CommitArgs &a, int u)
 {
-    float *st = reinterpret_cast<float *>(a.states[u / a.Hkv]);
+    const int hu = u / a.n_pass;
+    float *st = reinterpret_cast<float *>(a.states[hu / a.Hkv]);
     if (!state_ptr_ok(st)) return nullptr;
-    return st + (size_t)(u % a.Hkv) * head_floats(a.d, a.F);
+    return st + (size_t)(hu % a.Hkv) * head_floats(a.d, a.F);
 }
 
 __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constant__ CommitArgs a)
@@ -90,7 +99,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int d = a.d, F = a.F, T = a.T;
-    const int NCH = F / 32, NC = 2 * NCH;
+    const bool wide = a.n_pass > 1;       // F = 256: one sign per pass
+    const int NH = F / 32;                 // dS^T tiles per half
+    const int NCP = wide ? NH : 2 * NH;    // dS^T tiles per pass
     const int n_chunks = (T + kChunk - 1) / kChunk;
     const uint32_t atom = (uint32_t)d * 128;
     const uint32_t vbytes = (uint32_t)(d / 64) * kChunk * 128;
@@ -152,7 +163,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
         bool ok = true;
         for (int u = u_begin; u < u_end && ok; ++u) {
             if (!unit_head(a, u)) continue;
-            const int r = u / a.Hkv, g = u % a.Hkv;
+            const int r = (u / a.n_pass) / a.Hkv, g = (u / a.n_pass) % a.Hkv;
             if (kp > 0) ok = wait_bar(wfree, (kp - 1) & 1u, fail);
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
@@ -194,21 +205,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
             const uint32_t idDS = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, F);
             uint32_t kp = 0, cc = 0;
             bool ok = true;
-            // U_k^T of chunk cc into buffer cc & 1
+            // U_k^T of chunk cc into buffer cc & 1 (F = 256: two 128-feature tiles)
             auto ukt = [&](uint32_t ci) {
                 const uint32_t kt_u = c_u + (ci & 1) * a.chunk_stride;
-                for (int k = 0; k < d / 16; ++k) {
-                    const uint64_t aw = smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
-                    const uint64_t bk = smem_desc(kt_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
-                    mma_bf16_ss(tmem + 32 * (ci & 1), aw, bk, idKT, k > 0);
-                }
+                for (int t = 0; t < (wide ? 2 : 1); ++t)
+                    for (int k = 0; k < d / 16; ++k) {
+                        const uint64_t aw = smem_desc(w_u + 2 * t * atom + 2 * k * 1024, d * 128, 1024, SWZ_128B);
+                        const uint64_t bk = smem_desc(kt_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
+                        mma_bf16_ss(tmem + 32 * (ci & 1) + 64 * t, aw, bk, idKT, k > 0);
+                    }
                 mma_commit(&ukready[ci & 1]);
             };
             // dS^T (+)= V^T phi(K)^T of chunk ci for both halves
             auto dst = [&](uint32_t ci, bool first) {
                 const uint32_t cb = c_u + (ci & 1) * a.chunk_stride;
                 const uint32_t v_u = cb + atom, pk_u = cb + atom + vbytes;
-                for (int h = 0; h < 2; ++h)
+                for (int h = 0; h < (wide ? 1 : 2); ++h)
                     for (int ks = 0; ks < kChunk / 16; ++ks) {
                         const uint64_t av = smem_desc(v_u + ks * 2048, kChunk * 128, 1024, SWZ_128B);
                         const uint64_t bp = smem_desc(pk_u + (uint32_t)h * (F / 64) * (kChunk * 128) + ks * 2048,
@@ -254,15 +266,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
             for (int u = u_begin; u < u_end && ok; ++u) {
                 float *Sg = unit_head(a, u);
                 if (!Sg) continue;
+                const int pass = u % a.n_pass;
                 if (!wait_bar(dzready, kp & 1u, fail)) break;
-                bulk_reduce_add_f32(Sg + (size_t)2 * F * d, dzs, 2 * F * 4);
+                bulk_reduce_add_f32(Sg + (size_t)2 * F * d + (size_t)pass * F, dzs, (uint32_t)NCP * 32 * 4);
                 bulk_commit();
                 bulk_wait_read_all();
                 mbar_arrive(dzfree);
-                for (int c = 0; c < NC; ++c, ++sg) {
+                for (int c = 0; c < NCP; ++c, ++sg) {
                     const int slot = sg % kStage;
                     if (!wait_bar(&sfull[slot], (sg / kStage) & 1u, fail)) { ok = false; break; }
-                    bulk_reduce_add_f32(Sg + (size_t)c * 32 * d, stage + (size_t)slot * atom, atom);
+                    bulk_reduce_add_f32(Sg + (size_t)(pass * NCP + c) * 32 * d, stage + (size_t)slot * atom, atom);
                     bulk_commit();
                     bulk_wait_read_all();
                     mbar_arrive(&sempty[slot]);
@@ -278,8 +291,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
         const int row = 32 * q4 + lane;
         const uint32_t lane_off = (uint32_t)(32 * q4) << 16;
         const bool fval = row < F;
-        float *tk = reinterpret_cast<float *>(smem + a.off_tk);   // [s][token][quarter]
-        const float sgn = part == 0 ? kLog2e : -kLog2e;
+        // the thread's feature within the pass: one per part (the sign) for F <= 128;
+        // for F = 256 the parts are the two 128-feature tiles of the pass's sign
+        const int fp = wide ? 128 * part + row : part * F + row;
+        // per-token partial extrema and sums: [token][quarter] per part, or, for
+        // F = 256, [token][part][quarter] shared by both parts
+        float *tk = reinterpret_cast<float *>(smem + a.off_tk);
+        const int tk_m = wide ? 8 * lane : (part * 32 + lane) * 4;
+        const int tk_w = wide ? 4 * part + q4 : q4;
         uint32_t kp = 0, cc = 0, sg = 0;
         bool ok = true;
         for (int u = u_begin; u < u_end && ok; ++u) {
@@ -287,6 +306,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
                 if (mt == 0) raise_error(a.err, ERR_BAD_STATE_PTR);
                 continue;
             }
+            const float sgn = (wide ? u % a.n_pass : part) == 0 ? kLog2e : -kLog2e;
+            const bool neg = sgn < 0.f;
             float dz = 0.f;
             for (int j = 0; j < n_chunks; ++j, ++cc) {
                 const int b = cc & 1;
@@ -296,16 +317,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
                 tc_fence_after();
                 // per-token maximum of +-U_k over this warp's 32 features
                 float uk[32], ek[32];
-                tmem_ld32(tmem + 32 * b + lane_off, uk);
+                tmem_ld32(tmem + 32 * b + (wide ? 64 * part : 0) + lane_off, uk);
                 tmem_wait_ld();
 #pragma unroll
-                for (int t = 0; t < 32; ++t) ek[t] = (fval && t < nt) ? (part == 0 ? uk[t] : -uk[t]) : -INFINITY;
-                tk[(part * 32 + lane) * 4 + q4] = warp_reduce32<1>(ek, lane);
+                for (int t = 0; t < 32; ++t) ek[t] = (fval && t < nt) ? (neg ? -uk[t] : uk[t]) : -INFINITY;
+                tk[tk_m + tk_w] = warp_reduce32<1>(ek, lane);
                 if (group_sync_failed(kBarMath, kMathThreads, bad)) { ok = false; break; }
                 float m_l;
                 {
-                    const float4 x = *reinterpret_cast<const float4 *>(&tk[(part * 32 + lane) * 4]);
-                    m_l = fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w)) * kLog2e;
+                    const float4 x = *reinterpret_cast<const float4 *>(&tk[tk_m]);
+                    m_l = fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w));
+                    if (wide) {
+                        const float4 y = *reinterpret_cast<const float4 *>(&tk[tk_m + 4]);
+                        m_l = fmaxf(m_l, fmaxf(fmaxf(y.x, y.y), fmaxf(y.z, y.w)));
+                    }
+                    m_l *= kLog2e;
                 }
 #pragma unroll
                 for (int t = 0; t < 32; ++t) {
@@ -313,17 +339,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
                     ek[t] = (fval && t < nt) ? ex2(fmaf(uk[t], sgn, -m)) : 0.f;
                     uk[t] = ek[t];
                 }
-                tk[((2 + part) * 32 + lane) * 4 + q4] = warp_reduce32<0>(uk, lane);
+                tk[256 + tk_m + tk_w] = warp_reduce32<0>(uk, lane);
                 if (group_sync_failed(kBarMath, kMathThreads, false)) { ok = false; break; }
                 // phi(K) normalised into the bf16 MN-major operand [token][feature];
                 // lane t holds token t's normaliser (0 for an empty slot)
                 float inv_l;
                 {
-                    const float4 v = *reinterpret_cast<const float4 *>(&tk[((2 + part) * 32 + lane) * 4]);
-                    const float sum = (v.x + v.y) + (v.z + v.w);
+                    const float4 v = *reinterpret_cast<const float4 *>(&tk[256 + tk_m]);
+                    float sum = (v.x + v.y) + (v.z + v.w);
+                    if (wide) {
+                        const float4 y = *reinterpret_cast<const float4 *>(&tk[256 + tk_m + 4]);
+                        sum += (y.x + y.y) + (y.z + y.w);
+                    }
                     inv_l = sum > 0.f ? 1.f / sum : 0.f;
                 }
-                const int f = part * F + row;
+                const int f = fp;
                 uint8_t *bf = pkb + (f >> 6) * (kChunk * 128) + ((f & 7) << 1);
                 const int gf = (f & 63) >> 3;
 #pragma unroll
@@ -339,7 +369,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
             if (!ok) break;
             // dz of this thread's feature, then the dS^T tiles into the staging ring
             bool bad = !wait_bar(dzfree, (kp & 1u) ^ 1u, fail);
-            if (fval && !bad) dzs[part * F + row] = dz;
+            if (fval && !bad) dzs[fp] = dz;
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0 && !bad) mbar_arrive(dzready);
@@ -347,12 +377,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
             tc_fence_after();
             const int e = row;
 #pragma unroll 1
-            for (int i = 0; i < NCH; ++i) {
-                // tiles of this part: chunks part, part + 2 of each half, in storer order
-                const int h = i / (NCH / 2 > 0 ? NCH / 2 : 1);
-                const int k = part + 2 * (i % (NCH / 2 > 0 ? NCH / 2 : 1));
-                if (k >= NCH) continue;
-                const int c = h * NCH + k;
+            for (int i = 0; i < NCP / 2; ++i) {
+                // tiles of this part: chunks part, part + 2, ... of each half, in storer order
+                const int hp = NH / 2 > 0 ? NH / 2 : 1;   // tiles per half and part
+                const int h = i / hp;
+                const int k = part + 2 * (i % hp);
+                if (k >= NH) continue;
+                const int c = h * NH + k;
                 const uint32_t sgc = sg + c;
                 const int slot = sgc % kStage;
                 bool okc = wait_bar(&sempty[slot], ((sgc / kStage) & 1u) ^ 1u, fail) && !bad;
@@ -374,7 +405,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
             tc_fence_before();
             __syncwarp();
             if (lane == 0 && !bad) mbar_arrive(dsfree);
-            sg += NC;
+            sg += NCP;
             ++kp;
         }
         if (mt == 0 && *fail) raise_error(a.err, ERR_WAIT_TIMEOUT);
@@ -393,7 +424,7 @@ bool commit_red_supported(const hybrid_cfg &c)
 {
     if (c.io_dtype != HYBRID_BF16) return false;
     if (c.head_dim != 64 && c.head_dim != 128) return false;
-    if (c.feat_dim != 64 && c.feat_dim != 128) return false;
+    if (c.feat_dim != 64 && c.feat_dim != 128 && c.feat_dim != 256) return false;
     return (int)make_clayout(c.head_dim, c.feat_dim).bytes <= kSmemLimit;
 }
 
@@ -417,7 +448,8 @@ cudaError_t launch_commit_red(const hybrid_cfg &c, const void *K, const void *V,
     a.K = static_cast<const bf16 *>(K);
     a.states = states;
     a.err = err;
-    a.n_units = n_req * Hkv;
+    a.n_pass = F > 128 ? 2 : 1;
+    a.n_units = n_req * Hkv * a.n_pass;
     a.T = n_tok;
     a.Hkv = Hkv;
     a.d = d;

@@ -12,6 +12,9 @@
 // Per-row work (one thread per TMEM lane/row, two threads per row splitting
 // the columns): phi = [softmax(U), softmax(-U)], lin_den = phi . z_g, the
 // in-block softmax statistics, and the gated shared-normaliser merge.
+// With F = 256, phi = [phi+, phi-] (512 columns) does not fit beside D_lin and D_s
+// in Tensor Memory: phi+ is written over U and read out first, then U = Q W is
+// formed again and phi- takes its place for the second half of the readout.
 //
 // The state arrives by 1-D bulk copies: its HBM layout (hybrid.h) is already
 // the 128-byte-swizzled K-major operand image, so each 32-feature tile is one
@@ -26,7 +29,7 @@ namespace hyb {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr uint32_t kColA = 0;     // U, then phi = [phi+, phi-]  (2F <= 256 columns)
+constexpr uint32_t kColA = 0;     // U, then phi = [phi+, phi-] (F <= 128); F = 256: phi+, then phi-
 constexpr uint32_t kColD = 256;   // D_lin (d columns)
 constexpr uint32_t kColS = 384;   // scores (B columns), then D_s (d columns)
 constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s per bounded wait
@@ -44,11 +47,11 @@ struct TcAttnArgs {
     int n_slots;
     float scale_log2;   // log2(e) / sqrt(d)
     float inv_sqrt_d;
-    uint32_t off_q, off_w, off_k, off_v, off_p, off_z, off_bar;
+    uint32_t off_q, off_w, off_k, off_v, off_p, off_z, off_st, off_bar;
 };
 
 struct Layout {
-    uint32_t off_q, off_w, off_k, off_v, off_p, off_z, off_bar, bytes;
+    uint32_t off_q, off_w, off_k, off_v, off_p, off_z, off_st, off_bar, bytes;
     int n_slots;
 };
 
@@ -59,7 +62,9 @@ Layout make_layout(int d, int F, int B)
     const int NC = 2 * F / 32;
     const uint32_t q = (uint32_t)d * 256, w = (uint32_t)d * F * 2, k = (uint32_t)B * d * 2,
                    v = (uint32_t)B * d * 2, p = 128u * B * 2, z = ((uint32_t)2 * F * 4 + 1023) & ~1023u;
-    const uint32_t fixed = q + w + k + v + p + z + 1024 /*barriers*/ + 1024 /*alignment slack*/;
+    // F = 256 keeps Q for a second U = Q W, so the row statistics get their own space
+    const uint32_t stb = F > 128 ? 10u * 1024 : 0u;
+    const uint32_t fixed = q + w + k + v + p + z + stb + 1024 /*barriers*/ + 1024 /*alignment slack*/;
     int slots = (int)((kSmemLimit - (int)fixed) / (int)chunk);
     if (slots > NC) slots = NC;
     L.n_slots = slots;
@@ -70,6 +75,8 @@ Layout make_layout(int d, int F, int B)
     L.off_v = off; off += v;
     L.off_p = off; off += p;
     L.off_z = off; off += z;
+    L.off_st = F > 128 ? off : L.off_q;
+    off += stb;
     L.off_bar = off; off += 1024;
     L.bytes = off + 1024;
     if ((int)L.bytes < kOneCtaPerSm) L.bytes = kOneCtaPerSm;
@@ -115,12 +122,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     uint64_t *bar_z = bars + 2 * a.n_slots;
     uint64_t *bar_u = bar_z + 1;
     uint64_t *bar_d = bar_z + 2;
-    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_z + 3);
+    uint64_t *bar_p = bar_z + 3;    // F = 256: the phi+ readout is done
+    uint64_t *bar_u2 = bar_z + 4;   // F = 256: U = Q W formed again, for phi-
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_z + 5);
     int *fail = reinterpret_cast<int *>(tmem_holder + 1);
     int *issued = fail + 1;   // S chunks issued so far (for draining after a failure)
 
     if (tid == 0) {
-        for (int i = 0; i < 2 * a.n_slots + 3; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 2 * a.n_slots + 5; ++i) mbar_init(&bars[i], 1);
         *fail = 0;
         fence_mbar_init();
     }
@@ -191,8 +200,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     if (!mbar_wait(bar_u, 0, kWaitNs)) atomicOr(fail, 1);
     tc_fence_after();
 
-    // Q is no longer read by the tensor cores: its buffer holds the row statistics.
-    float *stat = reinterpret_cast<float *>(smem + a.off_q);   // [3][128] m, l, lin_den
+    // row statistics: in Q's buffer once Q is no longer read (F <= 128), else their own
+    const bool wide = F > 128;   // phi+ and phi- take turns in U's columns
+    float *stat = reinterpret_cast<float *>(smem + a.off_st);  // [3][128] m, l, lin_den
     float *ex = stat + 3 * 128;                                 // [8][2][128] exchange
     const int q4 = warp & 3, half = warp >> 2;
     const int row = 32 * q4 + lane;
@@ -265,7 +275,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
                 ln = fmaf(en[i], zs[F + 32 * k + i], ln);
             }
             tmem_st32(tmem + lane_off + kColA + 32 * k, ep);
-            tmem_st32(tmem + lane_off + kColA + F + 32 * k, en);
+            if (!wide) tmem_st32(tmem + lane_off + kColA + F + 32 * k, en);   // F = 256: formed later
         }
         ex[3 * 256 + half * 128 + row] = l;
         ex[4 * 256 + half * 128 + row] = sp;
@@ -289,6 +299,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = tf32_round(v[i] * isp);
             tmem_st32(tmem + lane_off + kColA + 32 * k, v);
+            if (wide) continue;
             tmem_ld32(tmem + lane_off + kColA + F + 32 * k, v);
             tmem_wait_ld();
 #pragma unroll
@@ -307,31 +318,86 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     tc_fence_before();
     __syncthreads();
 
-    // ---- readout D_lin = phi(Q) S_g over the 2F/32 state tiles, then D_s = P V
+    // ---- readout D_lin = phi(Q) S_g over the 2F/32 state tiles, then D_s = P V.
+    // Tile c of phi sits at column kColA + 32 (c - c0) of the phase [c0, c1) that reads
+    // it: one phase for F <= 128; for F = 256 the phi+ tiles, then the phi- tiles.
+    const int NC1 = wide ? NC / 2 : NC;
+    bool ok = true;   // thread 0 only
+    auto issue_tiles = [&](int c0, int c1) {
+        const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
+        for (int c = c0; c < c1 && ok; ++c) {
+            const int slot = c % a.n_slots;
+            const uint32_t ph = (uint32_t)(c / a.n_slots) & 1u;
+            if (!mbar_wait(&full[slot], ph, kWaitNs)) { ok = false; break; }
+            const uint32_t s_u = smem_u32(smem + (size_t)slot * chunk_bytes);
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+                mma_tf32_ts(tmem + kColD, tmem + kColA + 32 * (c - c0) + 8 * kk,
+                            smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B), idR, (c | kk) != 0);
+            if (c + a.n_slots < NC) {
+                // refill this slot once the tensor cores have read it
+                mma_commit(&empty[slot]);
+                if (!mbar_wait(&empty[slot], ph, kWaitNs)) { ok = false; break; }
+                mbar_arrive_expect_tx(&full[slot], chunk_bytes);
+                bulk_g2s(smem + (size_t)slot * chunk_bytes, Sg + (size_t)(c + a.n_slots) * 32 * d, chunk_bytes,
+                         &full[slot]);
+                *issued = c + a.n_slots + 1;
+            }
+        }
+    };
     if (tid == 0) {
-        bool ok = *fail == 0;
+        ok = *fail == 0;
         if (ok) {
             tc_fence_after();
-            const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
-            for (int c = 0; c < NC && ok; ++c) {
-                const int slot = c % a.n_slots;
-                const uint32_t ph = (uint32_t)(c / a.n_slots) & 1u;
-                if (!mbar_wait(&full[slot], ph, kWaitNs)) { ok = false; break; }
-                const uint32_t s_u = smem_u32(smem + (size_t)slot * chunk_bytes);
-#pragma unroll
-                for (int kk = 0; kk < 4; ++kk)
-                    mma_tf32_ts(tmem + kColD, tmem + kColA + 32 * c + 8 * kk,
-                                smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B), idR, (c | kk) != 0);
-                if (c + a.n_slots < NC) {
-                    // refill this slot once the tensor cores have read it
-                    mma_commit(&empty[slot]);
-                    if (!mbar_wait(&empty[slot], ph, kWaitNs)) { ok = false; break; }
-                    mbar_arrive_expect_tx(&full[slot], chunk_bytes);
-                    bulk_g2s(smem + (size_t)slot * chunk_bytes, Sg + (size_t)(c + a.n_slots) * 32 * d,
-                             chunk_bytes, &full[slot]);
-                    *issued = c + a.n_slots + 1;
-                }
+            issue_tiles(0, NC1);
+        }
+        if (wide) {
+            if (ok) mma_commit(bar_p);
+            else mbar_arrive(bar_p);
+        }
+    }
+    if (wide) {
+        // the tensor cores are done with phi+: form U = Q W_g again in its columns
+        if (!mbar_wait(bar_p, 0, kWaitNs)) atomicOr(fail, 1);
+        if (tid == 0) {
+            ok = ok && *fail == 0;
+            if (ok) {
+                tc_fence_after();
+                const uint32_t q_u = smem_u32(smem + a.off_q), w_u = smem_u32(smem + a.off_w);
+                const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
+                for (int k = 0; k < d / 16; ++k)
+                    mma_bf16_ss(tmem + kColA, smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B),
+                                smem_desc(w_u + 2 * k * ((F / 64) * 1024), 1024, (F / 64) * 1024, SWZ_128B), idU,
+                                k > 0);
+                mma_commit(bar_u2);
+            } else {
+                mbar_arrive(bar_u2);
             }
+        }
+        if (!mbar_wait(bar_u2, 0, kWaitNs)) atomicOr(fail, 1);
+        tc_fence_after();
+        // phi- = softmax(-U), from the same extremum and sum as round 2, rounded to tf32
+        {
+            const float mnl = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]) * kLog2e;
+            const float isn = 1.f / (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
+            for (int k = half; k < nfc; k += 2) {
+                float v[32];
+                tmem_ld32(tmem + lane_off + kColA + 32 * k, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) v[i] = tf32_round(exp2f(fmaf(-v[i], kLog2e, mnl)) * isn);
+                tmem_st32(tmem + lane_off + kColA + 32 * k, v);
+            }
+            tmem_wait_st();
+        }
+        tc_fence_before();
+        __syncthreads();
+    }
+    if (tid == 0) {
+        ok = ok && *fail == 0;
+        if (ok) {
+            tc_fence_after();
+            if (NC1 < NC) issue_tiles(NC1, NC);
             if (ok) {
                 const uint32_t p_u = smem_u32(smem + a.off_p), v_u = smem_u32(smem + a.off_v);
                 const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
@@ -400,7 +466,7 @@ bool tc_attn_supported(const hybrid_cfg &c)
 {
     if (c.io_dtype != HYBRID_BF16) return false;
     if (c.head_dim != 64 && c.head_dim != 128) return false;
-    if (c.feat_dim != 64 && c.feat_dim != 128) return false;
+    if (c.feat_dim != 64 && c.feat_dim != 128 && c.feat_dim != 256) return false;
     if (c.block_size % 16 != 0) return false;
     const int G = c.n_q_heads / c.n_kv_heads;
     if (G * c.block_size > 128) return false;
@@ -437,6 +503,7 @@ cudaError_t launch_attn_tc(const hybrid_cfg &c, const void *Q, const void *K, co
     a.off_v = L.off_v;
     a.off_p = L.off_p;
     a.off_z = L.off_z;
+    a.off_st = L.off_st;
     a.off_bar = L.off_bar;
     cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.bytes);
     if (e != cudaSuccess) return e;

@@ -48,6 +48,11 @@ SMALL = [
     (W_("bf16_b16_g2", BF16, 3, 4, 2, 128, 128, 16, 19), [16, 0, 80]),
     (W_("bf16_b64_g2", BF16, 2, 4, 2, 64, 128, 64, 20), [128, 64]),
     (W_("f32_mha_f128", F32, 2, 2, 2, 128, 128, 32, 21), [64, 32]),
+    # F = 256 on the tensor cores: phi+ and phi- read out in turn; commits in one
+    # pass per sign.  GQA with d = 64; 320 commit passes over 152 CTAs; G = 4, B = 16
+    (W_("f256_gqa2_d64_b32", BF16, 4, 4, 2, 64, 256, 32, 22), [32, 0, 96, 160]),
+    (W_("f256_many_units", BF16, 40, 8, 4, 128, 256, 32, 23), list((np.arange(40) % 4) * 32)),
+    (W_("f256_g4_b16", BF16, 3, 8, 2, 128, 256, 16, 24), [16, 48, 0]),
 ]
 
 
@@ -270,6 +275,8 @@ PREFILL = [
     (W_("prefill_cross_units", BF16, 20, 8, 4, 128, 128, 32, 47), 300, 0),
     # d = F = 64, a one-token last chunk
     (W_("prefill_d64_f64", BF16, 4, 4, 4, 64, 64, 32, 48), 257, 32),
+    # F = 256: six chunks per sign pass, a one-token tail
+    (W_("prefill_f256", BF16, 3, 2, 2, 128, 256, 32, 49), 161, 64),
 ]
 
 
@@ -313,6 +320,8 @@ FUSED = [
     (W_("fused_d128_f64", BF16, 4, 8, 4, 128, 64, 32, 57), [0, 64, 32, 96]),
     # d = 64, F = 128: a ring longer than a unit; 192 units, two or more per CTA
     (W_("fused_d64_f128_many", BF16, 48, 16, 4, 64, 128, 32, 58), None),
+    # F = 256: the step, then the commit, from one call
+    (W_("fused_f256_step_then_commit", BF16, 3, 4, 2, 128, 256, 32, 59), [32, 0, 64]),
 ]
 
 
