@@ -307,6 +307,66 @@ def small_config_context(dev, warmup=5, iters=20):
     return out
 
 
+def large_config_context(dev, warmup=3, iters=15):
+    """Context for the two other large configurations (not part of the value):
+    the per-call device time of the step (hybrid_block_attn) and of the block
+    commit (hybrid_commit_block, B tokens), each launched directly, median of
+    iters after warmup.  c4 is one layer of the decode loop (32 requests, MHA);
+    its state fits in L2, so it rotates enough buffer sets that each call misses
+    L2.  c5 (256 requests, F = 256) holds a 1.08 GB state and uses one set.  The
+    kernels' cost does not depend on the state's values: states start empty."""
+    import torch
+    from paper_2608_06628_gb300 import hybrid as H
+    from paper_2608_06628_gb300 import workloads as wk
+    from paper_2608_06628_gb300.state_pool import StatePool
+    peaks, _ = measured_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    out = {}
+    for wl in (wk.C4, wk.C5):
+        cfg = H.make_cfg(wl.d, wl.F, wl.Hq, wl.Hkv, wl.B, wl.io_dtype)
+        W, alpha = wk.params(wl, device=dev)
+        ab = algorithmic_bytes(wl, 2 if wl.io_dtype == torch.bfloat16 else 4)
+        l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+        per_set = ab["q"] * 2 + ab["kv"] * 2 + ab["state"]
+        n_sets = 1 if per_set > 4 * l2 else math.ceil(4 * l2 / per_set) + 1
+        sets = []
+        for i in range(n_sets):
+            pool = StatePool(cfg, wl.n_req, dev)
+            ptrs = pool.all_ptrs()
+            H.hybrid_state_init(cfg, ptrs, wl.n_req)
+            Q, K, V = wk.block_qkv(wl, ("large", i), dev)
+            sets.append(dict(pool=pool, ptrs=ptrs, Q=Q, K=K, V=V, O=torch.empty_like(Q)))
+        stream = torch.cuda.current_stream(dev)
+        calls = {
+            "step": lambda s: H.hybrid_block_attn(cfg, s["Q"], s["K"], s["V"], W, alpha, s["ptrs"], wl.n_req,
+                                                  s["O"], stream.cuda_stream, check=False),
+            "commit": lambda s: H.hybrid_commit_block(cfg, s["K"], s["V"], wl.B, W, s["ptrs"], wl.n_req,
+                                                      stream.cuda_stream, check=False),
+        }
+        res = {"buffer_sets": n_sets}
+        for name, fn in calls.items():
+            for i in range(warmup):
+                fn(sets[i % n_sets])
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(iters)]
+            for i, (a_, b_) in enumerate(evs):
+                a_.record(stream)
+                fn(sets[i % n_sets])
+                b_.record(stream)
+            torch.cuda.synchronize()
+            us = sorted(a_.elapsed_time(b_) for a_, b_ in evs)[iters // 2] * 1e3
+            nbytes = ab["attn"] if name == "step" else ab["commit"]
+            res[name] = {"us_median": us, "algorithmic_bytes": nbytes, "GBps": nbytes / us / 1e3,
+                         "frac_of_measured_hbm": nbytes / us / 1e3 / hbm}
+        status = H.hybrid_check(check=False)
+        if status != H.HYBRID_OK:
+            raise SystemExit(f"device error in the large-config context: {H.hybrid_status_str(status)}")
+        out[wl.name] = res
+        del sets
+        torch.cuda.empty_cache()
+    return out
+
+
 def small_config_oracle():
     """The oracle's one-thread time for the call small_config_context times on
     c1 and c2 (its cost does not depend on the state's values: empty states)."""
@@ -765,6 +825,7 @@ def run_hybrid(args, wl):
     }
     if not args.no_small_configs and ws == 1:
         line["small_configs"] = small_config_context(dev)
+        line["large_configs"] = large_config_context(dev)
         line["prefill_context"] = prefill_context(dev, wl)
         line["train_context"] = train_context(dev)
     if not args.no_cpu_baseline and ws == 1:
@@ -788,8 +849,8 @@ def main(argv=None):
     ap.add_argument("--config", default="c3_bf16_b64_gqa_ragged")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-small-configs", action="store_true",
-                    help="skip the context timings (c1/c2, prefill, training form)")
-    ap.add_argument("--context", choices=("train", "prefill", "small"),
+                    help="skip the context timings (c1/c2, c4/c5, prefill, training form)")
+    ap.add_argument("--context", choices=("train", "prefill", "small", "large"),
                     help="time only this context on cuda:0 and print its JSON object")
     args = ap.parse_args(argv)
     if args.warmup < 3:
@@ -803,7 +864,7 @@ def main(argv=None):
         dev = torch.device("cuda", 0)
         torch.cuda.set_device(dev)
         fn = {"train": lambda: train_context(dev), "prefill": lambda: prefill_context(dev, wl),
-              "small": lambda: small_config_context(dev)}[args.context]
+              "small": lambda: small_config_context(dev), "large": lambda: large_config_context(dev)}[args.context]
         print(json.dumps({"context": args.context, **fn()}), flush=True)
         return 0
     if args.impl == "reference":

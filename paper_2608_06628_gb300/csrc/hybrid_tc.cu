@@ -18,10 +18,13 @@
 //
 // The state arrives by 1-D bulk copies: its HBM layout (hybrid.h) is already
 // the 128-byte-swizzled K-major operand image, so each 32-feature tile is one
-// copy straight into an MMA-ready buffer.  Q, K, V and W are gathered with
-// 16-byte cp.async into their swizzled operand layouts.
+// copy straight into an MMA-ready buffer.  Q, K, V and W arrive by TMA as
+// 128-byte-swizzled boxes, each 64-element panel of a row one 128-byte line:
+// Q as the G x B rows of the group's heads over the block's tokens (row t G + hh),
+// K and V as B token rows, W as its d rows.
 #include "hybrid_common.cuh"
 #include "hybrid_tc.h"
+#include "tc_pipeline.cuh"
 #include "tc_ptx.cuh"
 
 namespace hyb {
@@ -38,7 +41,7 @@ constexpr int kSmemLimit = 232448;            // 227 KB opt-in per CTA
 constexpr int kOneCtaPerSm = 118 * 1024;      // request at least this much: 1 CTA / SM (TMEM 512 cols)
 
 struct TcAttnArgs {
-    const __nv_bfloat16 *Q, *K, *V, *W;
+    CUtensorMap tmQ, tmK, tmV, tmW;   // Q [n B][Hq][d] box {64, G, B}; K, V box {64, 1, B}; W box {64, d}
     const float *alpha;
     void *const *states;
     __nv_bfloat16 *O;
@@ -124,12 +127,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     uint64_t *bar_d = bar_z + 2;
     uint64_t *bar_p = bar_z + 3;    // F = 256: the phi+ readout is done
     uint64_t *bar_u2 = bar_z + 4;   // F = 256: U = Q W formed again, for phi-
-    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_z + 5);
+    uint64_t *bar_ld = bar_z + 5;   // Q, K, V and W have landed
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_z + 6);
     int *fail = reinterpret_cast<int *>(tmem_holder + 1);
     int *issued = fail + 1;   // S chunks issued so far (for draining after a failure)
 
     if (tid == 0) {
-        for (int i = 0; i < 2 * a.n_slots + 5; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 2 * a.n_slots + 6; ++i) mbar_init(&bars[i], 1);
         *fail = 0;
         fence_mbar_init();
     }
@@ -141,8 +145,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
 
-    // ---- producer: z and the first S tiles (bulk copies of the state image)
+    // ---- producer: Q, K, V, W (TMA), z and the first S tiles (bulk copies of the state image)
     if (tid == 0) {
+        mbar_arrive_expect_tx(bar_ld, (uint32_t)(Mv + 2 * B + F) * d * 2);
+        for (int c = 0; c < d / 64; ++c) {
+            tma_load_3d(smem + a.off_q + c * (128 * 128), &a.tmQ, 64 * c, g * G, r * B, bar_ld);
+            tma_load_3d(smem + a.off_k + c * (B * 128), &a.tmK, 64 * c, g, r * B, bar_ld);
+            tma_load_3d(smem + a.off_v + c * (B * 128), &a.tmV, 64 * c, g, r * B, bar_ld);
+        }
+        for (int f = 0; f < F / 64; ++f) tma_load_2d(smem + a.off_w + f * (d * 128), &a.tmW, 64 * f, g * d, bar_ld);
         mbar_arrive_expect_tx(bar_z, 2 * F * 4);
         bulk_g2s(smem + a.off_z, zg, 2 * F * 4, bar_z);
         const int pre = NC < a.n_slots ? NC : a.n_slots;
@@ -152,50 +163,28 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         }
         *issued = pre;
     }
-    // ---- Q, K, V, W into their operand layouts (16-byte cp.async)
-    {
-        const int gpr = d / 8;
-        for (int idx = tid; idx < Mv * gpr; idx += kThreads) {
-            const int i = idx / gpr, c = idx % gpr;
-            const int t = i / G, hh = i % G;
-            const __nv_bfloat16 *src = a.Q + (((size_t)r * B + t) * a.Hq + g * G + hh) * d + 8 * c;
-            cp_async16(smem + a.off_q + (c >> 3) * (128 * 128) + i * 128 + (((c & 7) ^ (i & 7)) << 4), src);
-        }
-        for (int idx = tid; idx < B * gpr; idx += kThreads) {
-            const int j = idx / gpr, c = idx % gpr;
-            const size_t so = (((size_t)r * B + j) * a.Hkv + g) * d + 8 * c;
-            cp_async16(smem + a.off_k + (c >> 3) * (B * 128) + j * 128 + (((c & 7) ^ (j & 7)) << 4), a.K + so);
-            cp_async16(smem + a.off_v + (j >> 3) * ((d / 64) * 1024) + (c >> 3) * 1024 + (j & 7) * 128 +
-                           (((c & 7) ^ (j & 7)) << 4),
-                       a.V + so);
-        }
-        const int gw = F / 8;
-        for (int idx = tid; idx < d * gw; idx += kThreads) {
-            const int e = idx / gw, c = idx % gw;
-            cp_async16(smem + a.off_w + (e >> 3) * ((F / 64) * 1024) + (c >> 3) * 1024 + (e & 7) * 128 +
-                           (((c & 7) ^ (e & 7)) << 4),
-                       a.W + ((size_t)g * d + e) * F + 8 * c);
-        }
-    }
-    cp_async_wait_all();
-    fence_proxy_async_smem();
-    __syncthreads();
 
-    // ---- U = Q W_g and scores = Q K^T
+    // ---- U = Q W_g and scores = Q K^T.  W and V are MN-major: 64-wide panels of
+    // d (W) or B (V) rows, 8-row groups 1024 bytes apart.
     if (tid == 0) {
-        tc_fence_after();
-        const uint32_t q_u = smem_u32(smem + a.off_q), w_u = smem_u32(smem + a.off_w),
-                       k_u = smem_u32(smem + a.off_k);
-        const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
-        const uint32_t idS = instr_desc(FMT_BF16, FMT_BF16, false, false, 128, B);
-        for (int k = 0; k < d / 16; ++k) {
-            const uint64_t ad = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
-            const uint64_t bw = smem_desc(w_u + 2 * k * ((F / 64) * 1024), 1024, (F / 64) * 1024, SWZ_128B);
-            const uint64_t bk = smem_desc(k_u + (k >> 2) * (B * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
-            mma_bf16_ss(tmem + kColA, ad, bw, idU, k > 0);
-            mma_bf16_ss(tmem + kColS, ad, bk, idS, k > 0);
+        if (mbar_wait(bar_ld, 0, kWaitNs)) {
+            tc_fence_after();
+            const uint32_t q_u = smem_u32(smem + a.off_q), w_u = smem_u32(smem + a.off_w),
+                           k_u = smem_u32(smem + a.off_k);
+            const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
+            const uint32_t idS = instr_desc(FMT_BF16, FMT_BF16, false, false, 128, B);
+            for (int k = 0; k < d / 16; ++k) {
+                const uint64_t ad = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
+                const uint64_t bw = smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
+                const uint64_t bk = smem_desc(k_u + (k >> 2) * (B * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
+                mma_bf16_ss(tmem + kColA, ad, bw, idU, k > 0);
+                mma_bf16_ss(tmem + kColS, ad, bk, idS, k > 0);
+            }
+            mma_commit(bar_u);
+        } else {
+            atomicOr(fail, 1);
+            mbar_arrive(bar_u);
         }
-        mma_commit(bar_u);
     }
     if (!mbar_wait(bar_u, 0, kWaitNs)) atomicOr(fail, 1);
     tc_fence_after();
@@ -367,8 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
                 const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
                 for (int k = 0; k < d / 16; ++k)
                     mma_bf16_ss(tmem + kColA, smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B),
-                                smem_desc(w_u + 2 * k * ((F / 64) * 1024), 1024, (F / 64) * 1024, SWZ_128B), idU,
-                                k > 0);
+                                smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B), idU, k > 0);
                 mma_commit(bar_u2);
             } else {
                 mbar_arrive(bar_u2);
@@ -403,7 +391,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
                 const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
                 for (int k = 0; k < B / 16; ++k) {
                     const uint64_t ad = smem_desc(p_u + k * 256, 128, (B / 8) * 128, SWZ_NONE);
-                    const uint64_t bd = smem_desc(v_u + 2 * k * ((d / 64) * 1024), 1024, (d / 64) * 1024, SWZ_128B);
+                    const uint64_t bd = smem_desc(v_u + 2 * k * 1024, B * 128, 1024, SWZ_128B);
                     mma_bf16_ss(tmem + kColS, ad, bd, idP, k > 0);
                 }
                 mma_commit(bar_d);
@@ -448,6 +436,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     } else if (tid == 0) {
         raise_error(a.err, ERR_WAIT_TIMEOUT);
         // drain bulk copies that may still be landing in this CTA's shared memory
+        mbar_wait(bar_ld, 0, kWaitNs);
         mbar_wait(bar_z, 0, kWaitNs);
         for (int c = 0; c < *issued; ++c)
             mbar_wait(&full[c % a.n_slots], (uint32_t)(c / a.n_slots) & 1u, kWaitNs);
@@ -480,10 +469,22 @@ cudaError_t launch_attn_tc(const hybrid_cfg &c, const void *Q, const void *K, co
 {
     const Layout L = make_layout(c.head_dim, c.feat_dim, c.block_size);
     TcAttnArgs a;
-    a.Q = static_cast<const __nv_bfloat16 *>(Q);
-    a.K = static_cast<const __nv_bfloat16 *>(K);
-    a.V = static_cast<const __nv_bfloat16 *>(V);
-    a.W = static_cast<const __nv_bfloat16 *>(W);
+    {
+        const int d = c.head_dim, F = c.feat_dim, B = c.block_size, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
+        const cuuint64_t rows = (cuuint64_t)n_req * B;
+        const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)Hq, rows};
+        const cuuint64_t sq[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hq * d * 2};
+        const cuuint32_t bq[3] = {64, (cuuint32_t)(Hq / Hkv), (cuuint32_t)B};
+        const cuuint64_t dk[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, rows};
+        const cuuint64_t sk[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
+        const cuuint32_t bk[3] = {64, 1, (cuuint32_t)B};
+        const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
+        const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
+        const cuuint32_t bw[2] = {64, (cuuint32_t)d};
+        if (!pipe::encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !pipe::encode_bf16(&a.tmK, K, 3, dk, sk, bk) ||
+            !pipe::encode_bf16(&a.tmV, V, 3, dk, sk, bk) || !pipe::encode_bf16(&a.tmW, W, 2, dw, sw, bw))
+            return cudaErrorInvalidValue;
+    }
     a.alpha = alpha;
     a.states = states;
     a.O = static_cast<__nv_bfloat16 *>(O);

@@ -123,7 +123,9 @@ def test_c5_full_sampled():
     """c5: 256 requests, 16 heads, F = 256, B = 64, ragged prefixes 1k-32k with
     keys x8 (normaliser and softmax range).  The GPU builds every prefix; the
     oracle rebuilds the shortest, the longest and one other, then checks a step
-    and the following commit on them."""
+    and the following commit on them.  The step is also checked for every
+    request, the oracle reading the GPU's prefix states (a full oracle rebuild of
+    all 256 prefixes is out of reach)."""
     wl = wk.C5
     plen = wk.prefix_lengths(wl)
     pair = Pair(wl, tracked=_sample(plen, 1, 105))
@@ -132,8 +134,14 @@ def test_c5_full_sampled():
     assert_parity(S, pair.S, wl.io_dtype, "c5 prefix state S")
     assert_parity(z, pair.z, wl.io_dtype, "c5 prefix state z")
     Q, K, V = wk.block_qkv(wl, "c5_step", pair.dev)
-    got, want, _ = pair.step(Q, K, V)
+    got, want, O = pair.step(Q, K, V)
     assert_parity(got, want, wl.io_dtype, "c5 output")
+    for r0 in range(0, wl.n_req, 32):
+        reqs = np.arange(r0, min(r0 + 32, wl.n_req))
+        Sg, zg = pair.gpu_state(reqs)
+        t = torch.as_tensor(reqs, device=pair.dev)
+        want = pair.orc.block_attn(h64(Q[t]), h64(K[t]), h64(V[t]), pair.W64, pair.alpha64, Sg, zg)
+        assert_parity(h64(O[t]), want, wl.io_dtype, f"c5 output, requests {r0}..{reqs[-1]}")
     pair.commit(K, V)
     S, z = pair.gpu_state()
     assert_parity(S, pair.S, wl.io_dtype, "c5 committed state S")
