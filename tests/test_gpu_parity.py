@@ -142,7 +142,10 @@ def test_state_init_zeroes():
 # ---------------------------------------------------------------------------
 EDGE_WL = [W_("edge_gqa_bf16", BF16, 3, 8, 2, 128, 128, 32, 31),
            W_("edge_gqa_k24_bf16", BF16, 3, 8, 2, 128, 128, 32, 33, k_scale=24.0),
-           W_("edge_f32", F32, 2, 2, 2, 64, 64, 16, 32)]
+           W_("edge_f32", F32, 2, 2, 2, 64, 64, 16, 32),
+           # the one-CTA-per-unit tensor-core step: F = 256 (phi+ then phi-), and G B = 128
+           W_("edge_f256_k8_bf16", BF16, 3, 2, 2, 128, 256, 64, 34, k_scale=8.0),
+           W_("edge_b64_g2_bf16", BF16, 3, 4, 2, 64, 128, 64, 35)]
 
 
 @pytest.mark.parametrize("wl", EDGE_WL, ids=[w.name for w in EDGE_WL])
@@ -246,10 +249,14 @@ def test_state_copy_out_and_back_resumes():
     assert torch.equal(O1, O2)
 
 
-def test_bad_state_pointer_is_reported_not_faulted():
+BADPTR_WL = [W_("badptr_bf16", BF16, 3, 4, 4, 128, 128, 32, 44),
+             W_("badptr_f256", BF16, 3, 2, 2, 128, 256, 64, 45)]
+
+
+@pytest.mark.parametrize("wl", BADPTR_WL, ids=[w.name for w in BADPTR_WL])
+def test_bad_state_pointer_is_reported_not_faulted(wl):
     """A null or misaligned entry in d_state_ptrs is skipped on the device and
     reported by hybrid_check; the context stays usable."""
-    wl = W_("badptr_bf16", BF16, 3, 4, 4, 128, 128, 32, 44)
     pair = Pair(wl)
     Q, K, V = wk.block_qkv(wl, "bad", pair.dev)
     good = pair.pool.ptr_array([0, 1, 2])
