@@ -13,8 +13,11 @@
 // the columns): phi = [softmax(U), softmax(-U)], lin_den = phi . z_g, the
 // in-block softmax statistics, and the gated shared-normaliser merge.
 // With F = 256, phi = [phi+, phi-] (512 columns) does not fit beside D_lin and D_s
-// in Tensor Memory: phi+ is written over U and read out first, then U = Q W is
-// formed again and phi- takes its place for the second half of the readout.
+// in Tensor Memory: phi+ is written over U and read out first, then phi- takes its
+// place for the second half of the readout.  phi- comes from phi+ by the identity
+// e^(mn - u) = e^(mn - mx) / e^(u - mx) when every row's range of U is moderate (then
+// W and Q are dead after U = Q W and their space holds six more state tiles, loaded
+// while the feature map is computed); otherwise U = Q W is formed again.
 //
 // The state arrives by 1-D bulk copies: its HBM layout (hybrid.h) is already
 // the 128-byte-swizzled K-major operand image, so each 32-feature tile is one
@@ -39,6 +42,8 @@ constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s per bounded wait
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kSmemLimit = 232448;            // 227 KB opt-in per CTA
 constexpr int kOneCtaPerSm = 118 * 1024;      // request at least this much: 1 CTA / SM (TMEM 512 cols)
+constexpr int kExtraSlots = 6;                // F = 256: W (4 tiles) and Q (2 tiles) as ring slots
+constexpr float kRecipRange = 64.f;           // largest row range of U for phi- from phi+
 
 struct TcAttnArgs {
     CUtensorMap tmQ, tmK, tmV, tmW;   // Q [n B][Hq][d] box {64, G, B}; K, V box {64, 1, B}; W box {64, d}
@@ -110,6 +115,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     const int NC = (2 * F) / 32;
     const int Mv = G * B;
     const uint32_t chunk_bytes = (uint32_t)d * 128;
+    const bool wide = F > 128;   // phi+ and phi- take turns in U's columns
+    const int RM = a.n_slots + (wide ? kExtraSlots : 0);   // ring slots at most
 
     const float *state = reinterpret_cast<const float *>(a.states[r]);
     if (!state_ptr_ok(state)) {
@@ -121,8 +128,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
 
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + a.off_bar);
     uint64_t *full = bars;
-    uint64_t *empty = bars + a.n_slots;
-    uint64_t *bar_z = bars + 2 * a.n_slots;
+    uint64_t *empty = bars + RM;
+    uint64_t *bar_z = bars + 2 * RM;
     uint64_t *bar_u = bar_z + 1;
     uint64_t *bar_d = bar_z + 2;
     uint64_t *bar_p = bar_z + 3;    // F = 256: the phi+ readout is done
@@ -133,7 +140,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     int *issued = fail + 1;   // S chunks issued so far (for draining after a failure)
 
     if (tid == 0) {
-        for (int i = 0; i < 2 * a.n_slots + 6; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 2 * RM + 6; ++i) mbar_init(&bars[i], 1);
         *fail = 0;
         fence_mbar_init();
     }
@@ -189,8 +196,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     if (!mbar_wait(bar_u, 0, kWaitNs)) atomicOr(fail, 1);
     tc_fence_after();
 
+    // ring slot s: the dedicated slots, then (F = 256, phi- from phi+) W's and Q's space
+    auto slot_ptr = [&](int sl) -> uint8_t * {
+        if (sl < a.n_slots) return smem + (size_t)sl * chunk_bytes;
+        sl -= a.n_slots;
+        return sl < 4 ? smem + a.off_w + (size_t)sl * chunk_bytes : smem + a.off_q + (size_t)(sl - 4) * chunk_bytes;
+    };
+
     // row statistics: in Q's buffer once Q is no longer read (F <= 128), else their own
-    const bool wide = F > 128;   // phi+ and phi- take turns in U's columns
     float *stat = reinterpret_cast<float *>(smem + a.off_st);  // [3][128] m, l, lin_den
     float *ex = stat + 3 * 128;                                 // [8][2][128] exchange
     const int q4 = warp & 3, half = warp >> 2;
@@ -222,6 +235,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         ex[2 * 256 + half * 128 + row] = mn;
     }
     __syncthreads();
+    // F = 256: while every valid row's range of U stays within kRecipRange, phi- follows
+    // from phi+ (phi-_j = e^(mn - mx) / (sp sn phi+_j), both sides far from underflow), so
+    // U = Q W is not formed again and W's and Q's space takes six more state tiles now
+    bool recip = false;
+    if (wide) {
+        const float rng = fmaxf(ex[1 * 256 + row], ex[1 * 256 + 128 + row]) -
+                          fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]);
+        recip = __syncthreads_and(!valid || rng <= kRecipRange) != 0;
+    }
+    const int R = recip ? min(NC, RM) : a.n_slots;   // ring slots in use
+    if (tid == 0 && R > a.n_slots && *fail == 0) {
+        for (int c = a.n_slots; c < R; ++c) {
+            mbar_arrive_expect_tx(&full[c], chunk_bytes);
+            bulk_g2s(slot_ptr(c), Sg + (size_t)c * 32 * d, chunk_bytes, &full[c]);
+        }
+        *issued = R;
+    }
     if (!mbar_wait(bar_z, 0, kWaitNs)) atomicOr(fail, 1);
 
     // ---- round 2: exponentials, P, unnormalised phi halves, partial sums
@@ -312,28 +342,44 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     // it: one phase for F <= 128; for F = 256 the phi+ tiles, then the phi- tiles.
     const int NC1 = wide ? NC / 2 : NC;
     bool ok = true;   // thread 0 only
+    // Thread 0 issues the MMAs; a slot whose tile c is read out in the first phase is
+    // refilled (tile c + R) by thread 32 as soon as the tensor cores release it, so the
+    // issue loop never waits for a tile to finish.  A second-phase tile's slot (F = 256
+    // with the 4-slot ring) is refilled by thread 0 itself, after the tile's MMAs.
     auto issue_tiles = [&](int c0, int c1) {
         const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
         for (int c = c0; c < c1 && ok; ++c) {
-            const int slot = c % a.n_slots;
-            const uint32_t ph = (uint32_t)(c / a.n_slots) & 1u;
+            const int slot = c % R;
+            const uint32_t ph = (uint32_t)(c / R) & 1u;
             if (!mbar_wait(&full[slot], ph, kWaitNs)) { ok = false; break; }
-            const uint32_t s_u = smem_u32(smem + (size_t)slot * chunk_bytes);
+            const uint32_t s_u = smem_u32(slot_ptr(slot));
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
                 mma_tf32_ts(tmem + kColD, tmem + kColA + 32 * (c - c0) + 8 * kk,
                             smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B), idR, (c | kk) != 0);
-            if (c + a.n_slots < NC) {
-                // refill this slot once the tensor cores have read it
+            if (c + R < NC) {
                 mma_commit(&empty[slot]);
-                if (!mbar_wait(&empty[slot], ph, kWaitNs)) { ok = false; break; }
-                mbar_arrive_expect_tx(&full[slot], chunk_bytes);
-                bulk_g2s(smem + (size_t)slot * chunk_bytes, Sg + (size_t)(c + a.n_slots) * 32 * d, chunk_bytes,
-                         &full[slot]);
-                *issued = c + a.n_slots + 1;
+                if (c >= NC1) {
+                    if (!mbar_wait(&empty[slot], ph, kWaitNs)) { ok = false; break; }
+                    mbar_arrive_expect_tx(&full[slot], chunk_bytes);
+                    bulk_g2s(slot_ptr(slot), Sg + (size_t)(c + R) * 32 * d, chunk_bytes, &full[slot]);
+                    *issued = c + R + 1;
+                }
             }
         }
     };
+    if (tid == 32 && *fail == 0) {
+        for (int c = R; c < NC && c - R < NC1; ++c) {
+            const int slot = c % R;
+            if (!mbar_wait(&empty[slot], (uint32_t)((c - R) / R) & 1u, kWaitNs)) {
+                atomicOr(fail, 1);
+                break;
+            }
+            mbar_arrive_expect_tx(&full[slot], chunk_bytes);
+            bulk_g2s(slot_ptr(slot), Sg + (size_t)c * 32 * d, chunk_bytes, &full[slot]);
+            *issued = c + 1;
+        }
+    }
     if (tid == 0) {
         ok = *fail == 0;
         if (ok) {
@@ -346,26 +392,45 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         }
     }
     if (wide) {
-        // the tensor cores are done with phi+: form U = Q W_g again in its columns
+        // the tensor cores are done with phi+; phi- takes its columns
         if (!mbar_wait(bar_p, 0, kWaitNs)) atomicOr(fail, 1);
-        if (tid == 0) {
-            ok = ok && *fail == 0;
-            if (ok) {
-                tc_fence_after();
-                const uint32_t q_u = smem_u32(smem + a.off_q), w_u = smem_u32(smem + a.off_w);
-                const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
-                for (int k = 0; k < d / 16; ++k)
-                    mma_bf16_ss(tmem + kColA, smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B),
-                                smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B), idU, k > 0);
-                mma_commit(bar_u2);
-            } else {
-                mbar_arrive(bar_u2);
+        if (recip) {
+            // phi-_j = e^(mn - mx) isp isn / phi+_j, rounded to tf32
+            tc_fence_after();
+            const float mx = fmaxf(ex[1 * 256 + row], ex[1 * 256 + 128 + row]);
+            const float mn = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]);
+            const float isp = 1.f / (ex[4 * 256 + row] + ex[4 * 256 + 128 + row]);
+            const float isn = 1.f / (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
+            const float kr = exp2f((mn - mx) * kLog2e) * isp * isn;
+            for (int k = half; k < nfc; k += 2) {
+                float v[32];
+                tmem_ld32(tmem + lane_off + kColA + 32 * k, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) v[i] = tf32_round(__fdividef(kr, v[i]));
+                tmem_st32(tmem + lane_off + kColA + 32 * k, v);
             }
-        }
-        if (!mbar_wait(bar_u2, 0, kWaitNs)) atomicOr(fail, 1);
-        tc_fence_after();
-        // phi- = softmax(-U), from the same extremum and sum as round 2, rounded to tf32
-        {
+            tmem_wait_st();
+        } else {
+            // form U = Q W_g again in phi+'s columns
+            if (tid == 0) {
+                ok = ok && *fail == 0;
+                if (ok) {
+                    tc_fence_after();
+                    const uint32_t q_u = smem_u32(smem + a.off_q), w_u = smem_u32(smem + a.off_w);
+                    const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
+                    for (int k = 0; k < d / 16; ++k)
+                        mma_bf16_ss(tmem + kColA,
+                                    smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B),
+                                    smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B), idU, k > 0);
+                    mma_commit(bar_u2);
+                } else {
+                    mbar_arrive(bar_u2);
+                }
+            }
+            if (!mbar_wait(bar_u2, 0, kWaitNs)) atomicOr(fail, 1);
+            tc_fence_after();
+            // phi- = softmax(-U), from the same extremum and sum as round 2, rounded to tf32
             const float mnl = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]) * kLog2e;
             const float isn = 1.f / (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
             for (int k = half; k < nfc; k += 2) {
@@ -438,8 +503,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         // drain bulk copies that may still be landing in this CTA's shared memory
         mbar_wait(bar_ld, 0, kWaitNs);
         mbar_wait(bar_z, 0, kWaitNs);
-        for (int c = 0; c < *issued; ++c)
-            mbar_wait(&full[c % a.n_slots], (uint32_t)(c / a.n_slots) & 1u, kWaitNs);
+        for (int c = 0; c < *issued; ++c) mbar_wait(&full[c % R], (uint32_t)(c / R) & 1u, kWaitNs);
     }
     tc_fence_before();
     __syncthreads();

@@ -249,6 +249,42 @@ def test_state_copy_out_and_back_resumes():
     assert torch.equal(O1, O2)
 
 
+def _u_ranges(wl, W, Q):
+    """Per state head, the largest row range max_f u - min_f u of U = Q W_g."""
+    G = wl.Hq // wl.Hkv
+    q = Q.float().reshape(wl.n_req, wl.B, wl.Hkv, G, wl.d)
+    U = torch.einsum("nbhgd,hdf->nbhgf", q, W.float().reshape(wl.Hkv, wl.d, wl.F))
+    return (U.amax(-1) - U.amin(-1)).amax(dim=(0, 1, 3)).cpu().numpy()
+
+
+@pytest.mark.parametrize("scaled_heads", [(), (0, 1), (1,)], ids=["from_phi_plus", "u_again", "mixed"])
+def test_f256_phi_minus_paths(scaled_heads):
+    """F = 256 step: phi- is derived from phi+ while every row of a unit has a range of
+    U = Q W within 64, and U is formed again otherwise (W x 20 on the listed state
+    heads); "mixed" runs both kinds of unit in one launch.  Both against the oracle."""
+    wl = W_("f256_phi_minus", BF16, 4, 4, 2, 128, 256, 32, 37)
+    pair = Pair(wl)
+    if scaled_heads:
+        W = pair.W.float()
+        for g in scaled_heads:
+            W[g] *= 20.0
+        pair.W = W.to(pair.W.dtype)
+        pair.W64 = h64(pair.W)
+    pair.build_prefixes(np.array([32, 0, 96, 64]))
+    Q, K, V = wk.block_qkv(wl, "phim", pair.dev)
+    rng = _u_ranges(wl, pair.W, Q)
+    for g in range(wl.Hkv):
+        assert (rng[g] > 64.0) if g in scaled_heads else (rng[g] < 32.0), (g, rng)
+    got, want, _ = pair.step(Q, K, V)
+    assert_parity(got, want, wl.io_dtype, f"W x 20 on heads {scaled_heads}")
+    pair.commit(K, V)
+    S, z = pair.gpu_state()
+    assert_parity(S, pair.S, wl.io_dtype, "state after the commit")
+    Q2, K2, V2 = wk.block_qkv(wl, "phim2", pair.dev)
+    got, want, _ = pair.step(Q2, K2, V2)
+    assert_parity(got, want, wl.io_dtype, "second step")
+
+
 BADPTR_WL = [W_("badptr_bf16", BF16, 3, 4, 4, 128, 128, 32, 44),
              W_("badptr_f256", BF16, 3, 2, 2, 128, 256, 64, 45)]
 
