@@ -104,6 +104,57 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b)
     return *reinterpret_cast<const uint32_t *>(&v);
 }
 
+// Tensor Memory accesses of 16 lanes by a whole warp (shape 16x32bx2): threads 0-15
+// read lanes base + t at columns c .. c + n - 1, threads 16-31 the same lanes at
+// columns c + n .. c + 2n - 1 (the split offset equals the width n here).
+__device__ __forceinline__ void tmem_ld16x2_32(uint32_t taddr, float (&v)[32])
+{
+    uint32_t r[32];
+    asm volatile("tcgen05.ld.sync.aligned.16x32bx2.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32], 32;"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+                 : "r"(taddr));
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tmem_ld16x2_16(uint32_t taddr, float (&v)[16])
+{
+    uint32_t r[16];
+    asm volatile("tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16], 16;"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+                 : "r"(taddr));
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tmem_st16x2_32(uint32_t taddr, const float (&v)[32])
+{
+    asm volatile("tcgen05.st.sync.aligned.16x32bx2.x32.b32 [%0], 32, {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+                 "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])), "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])), "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])), "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])), "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])), "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])), "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])), "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+                 : "memory");
+}
+
+// This thread's column chunk at taddr (lane quarter and column included): in the
+// spread layout the warp addresses its low half's chunk, n columns before a high
+// thread's own.
+template <bool kSpread>
+__device__ __forceinline__ void ld_chunk32(uint32_t taddr, int hi, float (&v)[32])
+{
+    if (kSpread) tmem_ld16x2_32(taddr - 32u * hi, v);
+    else ptx::tmem_ld32(taddr, v);
+}
+template <bool kSpread>
+__device__ __forceinline__ void ld_chunk16(uint32_t taddr, int hi, float (&v)[16])
+{
+    if (kSpread) tmem_ld16x2_16(taddr - 16u * hi, v);
+    else ptx::tmem_ld16(taddr, v);
+}
+template <bool kSpread>
+__device__ __forceinline__ void st_chunk32(uint32_t taddr, int hi, const float (&v)[32])
+{
+    if (kSpread) tmem_st16x2_32(taddr - 32u * hi, v);
+    else ptx::tmem_st32(taddr, v);
+}
+
+template <bool kSpread>
 __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__ TcAttnArgs a)
 {
     using namespace ptx;
@@ -156,7 +207,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     if (tid == 0) {
         mbar_arrive_expect_tx(bar_ld, (uint32_t)(Mv + 2 * B + F) * d * 2);
         for (int c = 0; c < d / 64; ++c) {
-            tma_load_3d(smem + a.off_q + c * (128 * 128), &a.tmQ, 64 * c, g * G, r * B, bar_ld);
+            if (kSpread) {
+                // query rows 16 q .. 16 q + 15 onto lanes 32 q .. 32 q + 15 (G = 1)
+                for (int q = 0; q < Mv / 16; ++q)
+                    tma_load_3d(smem + a.off_q + c * (128 * 128) + q * (32 * 128), &a.tmQ, 64 * c, g, r * B + 16 * q,
+                                bar_ld);
+            } else {
+                tma_load_3d(smem + a.off_q + c * (128 * 128), &a.tmQ, 64 * c, g * G, r * B, bar_ld);
+            }
             tma_load_3d(smem + a.off_k + c * (B * 128), &a.tmK, 64 * c, g, r * B, bar_ld);
             tma_load_3d(smem + a.off_v + c * (B * 128), &a.tmV, 64 * c, g, r * B, bar_ld);
         }
@@ -206,33 +264,46 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     // row statistics: in Q's buffer once Q is no longer read (F <= 128), else their own
     float *stat = reinterpret_cast<float *>(smem + a.off_st);  // [3][128] m, l, lin_den
     float *ex = stat + 3 * 128;                                 // [8][2][128] exchange
+    // Thread -> (TMEM lane, column subset).  Default: lane 32 q4 + lane and the warp's
+    // half as subset, two threads per row.  Spread (G = 1, B = 64): query row i sits on
+    // lane 32 (i / 16) + i % 16, so the rows occupy all four lane quarters (and SM
+    // sub-partitions), and a warp's two 16-thread halves take the same 16 lanes at
+    // different columns: four threads per row.
     const int q4 = warp & 3, half = warp >> 2;
-    const int row = 32 * q4 + lane;
+    const int hi = kSpread ? lane >> 4 : 0;
+    const int row = kSpread ? 32 * q4 + (lane & 15) : 32 * q4 + lane;   // TMEM lane of the query row
+    const int qrow = kSpread ? 16 * q4 + (lane & 15) : row;              // query row t G + hh
     const uint32_t lane_off = (uint32_t)(32 * q4) << 16;
-    const bool valid = row < Mv;
-    const int nsc = B / 16;       // 16-column chunks of scores; chunk k -> half k % 2
-    const int nfc = F / 32;       // 32-column chunks of U;      chunk k -> half k % 2
+    const bool valid = qrow < Mv;
+    constexpr int NS = kSpread ? 4 : 2;               // column subsets per row
+    const int sub = kSpread ? 2 * half + hi : half;   // owns the chunks k with k % NS == sub
+    const int nsc = B / 16;       // 16-column chunks of scores
+    const int nfc = F / 32;       // 32-column chunks of U
+    // in the spread layout a row's partial results meet across lanes l and l ^ 16 first
+    auto comb_max = [&](float x) { return kSpread ? fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 16)) : x; };
+    auto comb_min = [&](float x) { return kSpread ? fminf(x, __shfl_xor_sync(0xffffffffu, x, 16)) : x; };
+    auto comb_add = [&](float x) { return kSpread ? x + __shfl_xor_sync(0xffffffffu, x, 16) : x; };
 
     // ---- round 1: local extrema
     {
         float ms = -INFINITY, mx = -INFINITY, mn = INFINITY;
-        for (int k = half; k < nsc; k += 2) {
+        for (int k = sub; k < nsc; k += NS) {
             float v[16];
-            tmem_ld16(tmem + lane_off + kColS + 16 * k, v);
+            ld_chunk16<kSpread>(tmem + lane_off + kColS + 16 * k, hi, v);
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 16; ++i) ms = fmaxf(ms, v[i]);
         }
-        for (int k = half; k < nfc; k += 2) {
+        for (int k = sub; k < nfc; k += NS) {
             float v[32];
-            tmem_ld32(tmem + lane_off + kColA + 32 * k, v);
+            ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, v[i]); mn = fminf(mn, v[i]); }
         }
-        ex[0 * 256 + half * 128 + row] = ms;
-        ex[1 * 256 + half * 128 + row] = mx;
-        ex[2 * 256 + half * 128 + row] = mn;
+        ex[0 * 256 + half * 128 + row] = comb_max(ms);
+        ex[1 * 256 + half * 128 + row] = comb_max(mx);
+        ex[2 * 256 + half * 128 + row] = comb_min(mn);
     }
     __syncthreads();
     // F = 256: while every valid row's range of U stays within kRecipRange, phi- follows
@@ -260,9 +331,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         const float mx = fmaxf(ex[1 * 256 + row], ex[1 * 256 + 128 + row]);
         const float mn = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]);
         float l = 0.f, sp = 0.f, sn = 0.f, lp = 0.f, ln = 0.f;
-        for (int k = half; k < nsc; k += 2) {
+        for (int k = sub; k < nsc; k += NS) {
             float v[16];
-            tmem_ld16(tmem + lane_off + kColS + 16 * k, v);
+            ld_chunk16<kSpread>(tmem + lane_off + kColS + 16 * k, hi, v);
             tmem_wait_ld();
             uint32_t pk[8];
 #pragma unroll
@@ -280,9 +351,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         }
         const float *zs = reinterpret_cast<const float *>(smem + a.off_z);
         const float mxl = mx * kLog2e, mnl = mn * kLog2e;
-        for (int k = half; k < nfc; k += 2) {
+        for (int k = sub; k < nfc; k += NS) {
             float u[32], ep[32], en[32];
-            tmem_ld32(tmem + lane_off + kColA + 32 * k, u);
+            ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, u);
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
@@ -293,14 +364,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
                 lp = fmaf(ep[i], zs[32 * k + i], lp);
                 ln = fmaf(en[i], zs[F + 32 * k + i], ln);
             }
-            tmem_st32(tmem + lane_off + kColA + 32 * k, ep);
-            if (!wide) tmem_st32(tmem + lane_off + kColA + F + 32 * k, en);   // F = 256: formed later
+            st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, ep);
+            if (!wide) st_chunk32<kSpread>(tmem + lane_off + kColA + F + 32 * k, hi, en);   // F = 256: formed later
         }
-        ex[3 * 256 + half * 128 + row] = l;
-        ex[4 * 256 + half * 128 + row] = sp;
-        ex[5 * 256 + half * 128 + row] = sn;
-        ex[6 * 256 + half * 128 + row] = lp;
-        ex[7 * 256 + half * 128 + row] = ln;
+        ex[3 * 256 + half * 128 + row] = comb_add(l);
+        ex[4 * 256 + half * 128 + row] = comb_add(sp);
+        ex[5 * 256 + half * 128 + row] = comb_add(sn);
+        ex[6 * 256 + half * 128 + row] = comb_add(lp);
+        ex[7 * 256 + half * 128 + row] = comb_add(ln);
         if (half == 0) stat[row] = m_raw * a.inv_sqrt_d;
         tmem_wait_st();
     }
@@ -311,19 +382,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         const float sp = ex[4 * 256 + row] + ex[4 * 256 + 128 + row];
         const float sn = ex[5 * 256 + row] + ex[5 * 256 + 128 + row];
         const float isp = 1.f / sp, isn = 1.f / sn;
-        for (int k = half; k < nfc; k += 2) {
+        for (int k = sub; k < nfc; k += NS) {
             float v[32];
-            tmem_ld32(tmem + lane_off + kColA + 32 * k, v);
+            ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = tf32_round(v[i] * isp);
-            tmem_st32(tmem + lane_off + kColA + 32 * k, v);
+            st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
             if (wide) continue;
-            tmem_ld32(tmem + lane_off + kColA + F + 32 * k, v);
+            ld_chunk32<kSpread>(tmem + lane_off + kColA + F + 32 * k, hi, v);
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = tf32_round(v[i] * isn);
-            tmem_st32(tmem + lane_off + kColA + F + 32 * k, v);
+            st_chunk32<kSpread>(tmem + lane_off + kColA + F + 32 * k, hi, v);
         }
         if (half == 0) {
             stat[128 + row] = ex[3 * 256 + row] + ex[3 * 256 + 128 + row];
@@ -402,13 +473,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
             const float isp = 1.f / (ex[4 * 256 + row] + ex[4 * 256 + 128 + row]);
             const float isn = 1.f / (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
             const float kr = exp2f((mn - mx) * kLog2e) * isp * isn;
-            for (int k = half; k < nfc; k += 2) {
+            for (int k = sub; k < nfc; k += NS) {
                 float v[32];
-                tmem_ld32(tmem + lane_off + kColA + 32 * k, v);
+                ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
                 tmem_wait_ld();
 #pragma unroll
                 for (int i = 0; i < 32; ++i) v[i] = tf32_round(__fdividef(kr, v[i]));
-                tmem_st32(tmem + lane_off + kColA + 32 * k, v);
+                st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
             }
             tmem_wait_st();
         } else {
@@ -433,13 +504,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
             // phi- = softmax(-U), from the same extremum and sum as round 2, rounded to tf32
             const float mnl = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]) * kLog2e;
             const float isn = 1.f / (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
-            for (int k = half; k < nfc; k += 2) {
+            for (int k = sub; k < nfc; k += NS) {
                 float v[32];
-                tmem_ld32(tmem + lane_off + kColA + 32 * k, v);
+                ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
                 tmem_wait_ld();
 #pragma unroll
                 for (int i = 0; i < 32; ++i) v[i] = tf32_round(exp2f(fmaf(-v[i], kLog2e, mnl)) * isn);
-                tmem_st32(tmem + lane_off + kColA + 32 * k, v);
+                st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
             }
             tmem_wait_st();
         }
@@ -474,16 +545,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
 
     // ---- epilogue: out = ws * D_s + wl * D_lin, stored as bf16
     if (!failed) {
-        const int dh = d / 2;
         const float m = stat[row], l = stat[128 + row], ld = stat[256 + row];
-        const int t = row / G, hh = row % G;
+        const int t = qrow / G, hh = qrow % G;
         MergeWeights mw{0.f, 0.f};
         if (valid) mw = merge_weights(log_sigmoid(a.alpha[g * G + hh]), m, l, ld);
-        __nv_bfloat16 *orow = a.O + (((size_t)r * B + t) * a.Hq + g * G + hh) * d + half * dh;
-        for (int c0 = 0; c0 < dh; c0 += 32) {
+        __nv_bfloat16 *orow0 = a.O + (((size_t)r * B + t) * a.Hq + g * G + hh) * d;
+        for (int kd = sub; kd < d / 32; kd += NS) {
+            const int c0 = 32 * kd;
             float dl[32], ds[32];
-            tmem_ld32(tmem + lane_off + kColD + half * dh + c0, dl);
-            tmem_ld32(tmem + lane_off + kColS + half * dh + c0, ds);
+            ld_chunk32<kSpread>(tmem + lane_off + kColD + c0, hi, dl);
+            ld_chunk32<kSpread>(tmem + lane_off + kColS + c0, hi, ds);
             tmem_wait_ld();
             if (valid) {
                 uint32_t pk[16];
@@ -493,7 +564,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
                     const float o1 = mw.ws * ds[i + 1] + (mw.wl == 0.f ? 0.f : mw.wl * dl[i + 1]);
                     pk[i / 2] = pack_bf16x2(o0, o1);
                 }
-                uint4 *dst = reinterpret_cast<uint4 *>(orow + c0);
+                uint4 *dst = reinterpret_cast<uint4 *>(orow0 + c0);
 #pragma unroll
                 for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
             }
@@ -533,12 +604,14 @@ cudaError_t launch_attn_tc(const hybrid_cfg &c, const void *Q, const void *K, co
 {
     const Layout L = make_layout(c.head_dim, c.feat_dim, c.block_size);
     TcAttnArgs a;
+    // G = 1 with B = 64: 64 query rows spread over the four TMEM lane quarters
+    const bool spread = c.n_q_heads == c.n_kv_heads && c.block_size == 64;
     {
         const int d = c.head_dim, F = c.feat_dim, B = c.block_size, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
         const cuuint64_t rows = (cuuint64_t)n_req * B;
         const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)Hq, rows};
         const cuuint64_t sq[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hq * d * 2};
-        const cuuint32_t bq[3] = {64, (cuuint32_t)(Hq / Hkv), (cuuint32_t)B};
+        const cuuint32_t bq[3] = {64, (cuuint32_t)(Hq / Hkv), (cuuint32_t)(spread ? 16 : B)};
         const cuuint64_t dk[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, rows};
         const cuuint64_t sk[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
         const cuuint32_t bk[3] = {64, 1, (cuuint32_t)B};
@@ -570,10 +643,11 @@ cudaError_t launch_attn_tc(const hybrid_cfg &c, const void *Q, const void *K, co
     a.off_z = L.off_z;
     a.off_st = L.off_st;
     a.off_bar = L.off_bar;
-    cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.bytes);
+    auto kern = spread ? k_attn_tc<true> : k_attn_tc<false>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.bytes);
     if (e != cudaSuccess) return e;
     const long long blocks = (long long)n_req * c.n_kv_heads;
-    k_attn_tc<<<(unsigned)blocks, kThreads, L.bytes, st>>>(a);
+    kern<<<(unsigned)blocks, kThreads, L.bytes, st>>>(a);
     return cudaGetLastError();
 }
 

@@ -53,6 +53,9 @@ SMALL = [
     (W_("f256_gqa2_d64_b32", BF16, 4, 4, 2, 64, 256, 32, 22), [32, 0, 96, 160]),
     (W_("f256_many_units", BF16, 40, 8, 4, 128, 256, 32, 23), list((np.arange(40) % 4) * 32)),
     (W_("f256_g4_b16", BF16, 3, 8, 2, 128, 256, 16, 24), [16, 48, 0]),
+    # G = 1, B = 64: the step spreads its 64 rows over all four TMEM lane quarters
+    (W_("spread_f128_b64", BF16, 3, 4, 4, 128, 128, 64, 25), [64, 0, 128]),
+    (W_("spread_d64_f64_b64", BF16, 3, 2, 2, 64, 64, 64, 26), [128, 64, 0]),
 ]
 
 
