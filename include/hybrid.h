@@ -60,8 +60,10 @@
  * Supported sizes: head_dim d in {64, 128}; feat_dim F in {16, 32, 64, 128,
  * 256}; 1 <= B <= 128; 1 <= Hkv <= Hq <= 256 with Hq % Hkv == 0; io_dtype
  * float32 or bfloat16.  The state is always float32.  Arithmetic is float32
- * throughout; with bfloat16 inputs the block-attention contractions run on
- * the tensor cores (bf16 and tf32 operands, float32 accumulation).
+ * throughout.  With bfloat16 inputs and F >= 64 the contractions of the
+ * step (B a multiple of 16, G * B <= 128) and of the commit run on the
+ * tensor cores (bf16 and tf32 operands, float32 accumulation); other shapes
+ * and float32 inputs run float32 FMA kernels.
  *
  * Errors: argument checks run synchronously on the host and return
  * HYBRID_ERR_INVALID_ARG (null or misaligned pointer, inconsistent sizes) or
