@@ -180,6 +180,22 @@ hybrid_status hybrid_commit_block(const hybrid_cfg *cfg, const void *K, const vo
                                   const void *W, void *const *d_state_ptrs, int n_req,
                                   cudaStream_t stream);
 
+/* Prompt prefill with a different length per request (the state update of
+ * Section 3.1, folding a prompt's tokens): request r folds tokens
+ * [tok_offsets[r], tok_offsets[r + 1]) of the packed K, V
+ * [tok_offsets[n_req]][Hkv][d] (io_dtype) into its state d_state_ptrs[r].
+ *   tok_offsets  HOST array of n_req + 1 ints, tok_offsets[0] = 0, non-decreasing
+ *                (a request with no tokens is left unchanged); read during the
+ *                call, so the caller may reuse it on return
+ *   K, V         device, 16-byte aligned, packed token-major as above
+ * Equivalent to one hybrid_commit_block per request with n_tok = its length,
+ * in one launch per 2048 requests (the offsets travel in the kernel
+ * parameters, so the call can be captured in a CUDA graph).  Errors:
+ * HYBRID_ERR_INVALID_ARG for null or misaligned pointers or offsets that do not
+ * start at 0 or decrease; otherwise as hybrid_commit_block. */
+hybrid_status hybrid_commit_ragged(const hybrid_cfg *cfg, const void *K, const void *V, const int *tok_offsets,
+                                   int n_req, const void *W, void *const *d_state_ptrs, cudaStream_t stream);
+
 /* Convert states to / from the logical layout (device buffers):
  *   S_logical [n][Hkv][2F][d] float32 (S[f][e] as in Section 3.1)
  *   z_logical [n][Hkv][2F]    float32 */

@@ -214,6 +214,58 @@ hybrid_status hybrid_commit_block(const hybrid_cfg *cfg, const void *K, const vo
     return from_cuda(hyb::launch_commit_generic(*cfg, K, V, n_tok, W, d_state_ptrs, n_req, err, stream));
 }
 
+hybrid_status hybrid_commit_ragged(const hybrid_cfg *cfg, const void *K, const void *V, const int *tok_offsets,
+                                   int n_req, const void *W, void *const *d_state_ptrs, cudaStream_t stream)
+{
+    hybrid_status s = check_cfg(cfg);
+    if (s != HYBRID_OK) return s;
+    if (n_req < 0) return HYBRID_ERR_INVALID_ARG;
+    if (n_req == 0) return HYBRID_OK;
+    if (!tok_offsets || tok_offsets[0] != 0) return HYBRID_ERR_INVALID_ARG;
+    for (int r = 0; r < n_req; ++r)
+        if (tok_offsets[r + 1] < tok_offsets[r]) return HYBRID_ERR_INVALID_ARG;
+    if (tok_offsets[n_req] == 0) return HYBRID_OK;
+    if (!K || !V || !W || !d_state_ptrs) return HYBRID_ERR_INVALID_ARG;
+    if (!aligned(K, 16) || !aligned(V, 16) || !aligned(W, 16) || !aligned(d_state_ptrs, 8))
+        return HYBRID_ERR_INVALID_ARG;
+    unsigned *err = error_word();
+    if (!err) return HYBRID_ERR_CUDA;
+    const size_t row_bytes = (size_t)cfg->n_kv_heads * cfg->head_dim * (cfg->io_dtype == HYBRID_BF16 ? 2 : 4);
+    const unsigned char *Kb = static_cast<const unsigned char *>(K);
+    const unsigned char *Vb = static_cast<const unsigned char *>(V);
+    const bool red = hyb::commit_red_supported(*cfg), pre = hyb::prefill_supported(*cfg);
+    if (!red && !pre) {
+        // FMA kernels: one launch per request that has tokens
+        for (int r = 0; r < n_req; ++r) {
+            const int T = tok_offsets[r + 1] - tok_offsets[r];
+            if (T == 0) continue;
+            const size_t off = (size_t)tok_offsets[r] * row_bytes;
+            const cudaError_t e =
+                hyb::launch_commit_generic(*cfg, Kb + off, Vb + off, T, W, d_state_ptrs + r, 1, err, stream);
+            if (e != cudaSuccess) return from_cuda(e);
+        }
+        return HYBRID_OK;
+    }
+    // tensor-core kernels, up to kMaxRaggedRequests requests per launch (offsets rebased)
+    static thread_local int tok[hyb::kMaxRaggedRequests + 1];
+    for (int r0 = 0; r0 < n_req; r0 += hyb::kMaxRaggedRequests) {
+        const int nb = n_req - r0 < hyb::kMaxRaggedRequests ? n_req - r0 : hyb::kMaxRaggedRequests;
+        int longest = 0;
+        for (int i = 0; i <= nb; ++i) tok[i] = tok_offsets[r0 + i] - tok_offsets[r0];
+        for (int i = 0; i < nb; ++i) longest = tok[i + 1] - tok[i] > longest ? tok[i + 1] - tok[i] : longest;
+        if (tok[nb] == 0) continue;
+        const size_t off = (size_t)tok_offsets[r0] * row_bytes;
+        // as for uniform prompts: the token-major kernel once a prompt is longer than a
+        // block commit (it balances chunks across SMs), else the per-unit reduction kernel
+        const cudaError_t e =
+            pre && (longest > kPrefillMinTokens || !red)
+                ? hyb::launch_prefill_ragged(*cfg, Kb + off, Vb + off, tok, W, d_state_ptrs + r0, nb, err, stream)
+                : hyb::launch_commit_red_ragged(*cfg, Kb + off, Vb + off, tok, W, d_state_ptrs + r0, nb, err, stream);
+        if (e != cudaSuccess) return from_cuda(e);
+    }
+    return HYBRID_OK;
+}
+
 hybrid_status hybrid_state_unpack(const hybrid_cfg *cfg, void *const *d_state_ptrs, int n_req,
                                   float *S_logical, float *z_logical, cudaStream_t stream)
 {

@@ -84,6 +84,25 @@ CLayout make_clayout(int d, int F)
 }
 
 // unit u = pass (u % n_pass) of state head g of request r, (r, g) = (u / n_pass) / Hkv, % Hkv
+// Ragged prompts: request r owns tokens [tok[r], tok[r + 1]) of the packed K and V;
+// carried in the parameters.
+struct CommitRaggedArgs : CommitArgs {
+    int n_req;
+    int tok[kMaxRaggedRequests + 1];
+};
+// tokens of unit u and the K/V row of its first token, uniform or ragged
+__device__ __forceinline__ int unit_len(const CommitArgs &a, int) { return a.T; }
+__device__ __forceinline__ long long unit_tok0(const CommitArgs &a, int u)
+{
+    return (long long)((u / a.n_pass) / a.Hkv) * a.T;
+}
+__device__ __forceinline__ int unit_len(const CommitRaggedArgs &a, int u)
+{
+    const int r = (u / a.n_pass) / a.Hkv;
+    return a.tok[r + 1] - a.tok[r];
+}
+__device__ __forceinline__ long long unit_tok0(const CommitRaggedArgs &a, int u) { return a.tok[(u / a.n_pass) / a.Hkv]; }
+
 __device__ __forceinline__ float *unit_head(const CommitArgs &a, int u)
 {
     const int hu = u / a.n_pass;
@@ -92,17 +111,17 @@ __device__ __forceinline__ float *unit_head(const CommitArgs &a, int u)
     return st + (size_t)(hu % a.Hkv) * head_floats(a.d, a.F);
 }
 
-__global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constant__ CommitArgs a)
+template <class A>
+__global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constant__ A a)
 {
     using namespace ptx;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int d = a.d, F = a.F, T = a.T;
+    const int d = a.d, F = a.F;
     const bool wide = a.n_pass > 1;       // F = 256: one sign per pass
     const int NH = F / 32;                 // dS^T tiles per half
     const int NCP = wide ? NH : 2 * NH;    // dS^T tiles per pass
-    const int n_chunks = (T + kChunk - 1) / kChunk;
     const uint32_t atom = (uint32_t)d * 128;
     const uint32_t vbytes = (uint32_t)(d / 64) * kChunk * 128;
     const int per = a.n_units / (int)gridDim.x, rem = a.n_units % (int)gridDim.x;
@@ -162,8 +181,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
         int nw = 0, nv = 0;
         bool ok = true;
         for (int u = u_begin; u < u_end && ok; ++u) {
-            if (!unit_head(a, u)) continue;
-            const int r = (u / a.n_pass) / a.Hkv, g = (u / a.n_pass) % a.Hkv;
+            const int Tu = unit_len(a, u);   // a request without tokens has no work
+            if (Tu == 0 || !unit_head(a, u)) continue;
+            const int n_chunks = (Tu + kChunk - 1) / kChunk;
+            const long long tok0 = unit_tok0(a, u);
+            const int g = (u / a.n_pass) % a.Hkv;
             if (kp > 0) ok = wait_bar(wfree, (kp - 1) & 1u, fail);
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
@@ -175,13 +197,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
                 const int b = cc & 1;
                 uint8_t *cb = smem + a.off_c + b * a.chunk_stride;
                 KtRegs kr;
-                kt_load(a.K, (size_t)r * T + (size_t)j * kChunk, min(kChunk, T - j * kChunk), a.Hkv, g, d, kr, lane);
+                kt_load(a.K, (size_t)tok0 + (size_t)j * kChunk, min(kChunk, Tu - j * kChunk), a.Hkv, g, d, kr, lane);
                 ok = wait_bar(&cfree[b], ((cc >> 1) & 1u) ^ 1u, fail);
                 if (__any_sync(0xffffffffu, !ok)) break;
                 if (lane == 0) {
                     mbar_arrive_expect_tx(&cfull[b], vbytes);
                     for (int e = 0; e < d / 64; ++e)
-                        tma_load_3d(cb + atom + e * (kChunk * 128), &a.tmV, 64 * e, g, r * T + j * kChunk, &cfull[b]);
+                        tma_load_3d(cb + atom + e * (kChunk * 128), &a.tmV, 64 * e, g, (int)tok0 + j * kChunk,
+                                    &cfull[b]);
                 }
                 ++nv;
                 kt_store(kr, d, cb, lane);
@@ -230,7 +253,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
                 mma_commit(&cfree[ci & 1]);
             };
             for (int u = u_begin; u < u_end && ok; ++u) {
-                if (!unit_head(a, u)) continue;
+                const int Tu = unit_len(a, u);
+                if (Tu == 0 || !unit_head(a, u)) continue;
+                const int n_chunks = (Tu + kChunk - 1) / kChunk;
                 if (!wait_bar(wfull, kp & 1u, fail)) { ok = false; break; }
                 for (int j = 0; j <= n_chunks && ok; ++j) {
                     // U_k^T of chunk j ahead of dS^T of chunk j - 1 (its phi(K) is on the math warps)
@@ -264,6 +289,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
             uint32_t kp = 0, sg = 0;
             bool ok = true;
             for (int u = u_begin; u < u_end && ok; ++u) {
+                if (unit_len(a, u) == 0) continue;
                 float *Sg = unit_head(a, u);
                 if (!Sg) continue;
                 const int pass = u % a.n_pass;
@@ -302,16 +328,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
         uint32_t kp = 0, cc = 0, sg = 0;
         bool ok = true;
         for (int u = u_begin; u < u_end && ok; ++u) {
+            const int Tu = unit_len(a, u);
+            if (Tu == 0) continue;
             if (!unit_head(a, u)) {
                 if (mt == 0) raise_error(a.err, ERR_BAD_STATE_PTR);
                 continue;
             }
+            const int n_chunks = (Tu + kChunk - 1) / kChunk;
             const float sgn = (wide ? u % a.n_pass : part) == 0 ? kLog2e : -kLog2e;
             const bool neg = sgn < 0.f;
             float dz = 0.f;
             for (int j = 0; j < n_chunks; ++j, ++cc) {
                 const int b = cc & 1;
-                const int nt = min(kChunk, T - j * kChunk);
+                const int nt = min(kChunk, Tu - j * kChunk);
                 uint8_t *pkb = smem + a.off_c + b * a.chunk_stride + atom + vbytes;
                 bool bad = !wait_bar(&ukready[b], (cc >> 1) & 1u, fail);
                 tc_fence_after();
@@ -428,29 +457,26 @@ bool commit_red_supported(const hybrid_cfg &c)
     return (int)make_clayout(c.head_dim, c.feat_dim).bytes <= kSmemLimit;
 }
 
-cudaError_t launch_commit_red(const hybrid_cfg &c, const void *K, const void *V, int n_tok, const void *W,
-                              void *const *states, int n_req, unsigned *err, cudaStream_t st)
+namespace {
+
+// Tensor maps and sizes shared by the uniform and the ragged launch; rows = tokens of K and V.
+bool fill_commit_args(const hybrid_cfg &c, const void *K, const void *V, long long rows, const void *W,
+                      void *const *states, int n_req, unsigned *err, CommitArgs &a)
 {
     const CLayout L = make_clayout(c.head_dim, c.feat_dim);
-    CommitArgs a;
     const int d = c.head_dim, F = c.feat_dim, Hkv = c.n_kv_heads;
-    {
-        const cuuint64_t rows = (cuuint64_t)n_req * n_tok;
-        const cuuint64_t dv[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, rows};
-        const cuuint64_t sv[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
-        const cuuint32_t bv[3] = {64, 1, (cuuint32_t)kChunk};
-        const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
-        const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
-        const cuuint32_t bw[2] = {64, (cuuint32_t)d};
-        if (!encode_bf16(&a.tmV, V, 3, dv, sv, bv) || !encode_bf16(&a.tmW, W, 2, dw, sw, bw))
-            return cudaErrorInvalidValue;
-    }
+    const cuuint64_t dv[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, (cuuint64_t)rows};
+    const cuuint64_t sv[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
+    const cuuint32_t bv[3] = {64, 1, (cuuint32_t)kChunk};
+    const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
+    const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
+    const cuuint32_t bw[2] = {64, (cuuint32_t)d};
+    if (!encode_bf16(&a.tmV, V, 3, dv, sv, bv) || !encode_bf16(&a.tmW, W, 2, dw, sw, bw)) return false;
     a.K = static_cast<const bf16 *>(K);
     a.states = states;
     a.err = err;
     a.n_pass = F > 128 ? 2 : 1;
     a.n_units = n_req * Hkv * a.n_pass;
-    a.T = n_tok;
     a.Hkv = Hkv;
     a.d = d;
     a.F = F;
@@ -461,13 +487,21 @@ cudaError_t launch_commit_red(const hybrid_cfg &c, const void *K, const void *V,
     a.off_tk = L.off_tk;
     a.off_bar = L.off_bar;
     a.chunk_stride = L.chunk;
+    return true;
+}
+
+template <class A>
+cudaError_t run_commit_red(const hybrid_cfg &c, const A &a, cudaStream_t st)
+{
+    const CLayout L = make_clayout(c.head_dim, c.feat_dim);
     const int grid = a.n_units < sm_count() ? a.n_units : sm_count();
     static std::atomic<unsigned long long> opted;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     const unsigned long long bit = 1ull << dev;
     if (!(opted.load(std::memory_order_acquire) & bit)) {
-        const cudaError_t e = cudaFuncSetAttribute(k_commit_red, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
+        const cudaError_t e =
+            cudaFuncSetAttribute(k_commit_red<A>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
         if (e != cudaSuccess) return e;
         opted.fetch_or(bit, std::memory_order_release);
     }
@@ -481,7 +515,31 @@ cudaError_t launch_commit_red(const hybrid_cfg &c, const void *K, const void *V,
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = attr;
     lc.numAttrs = 1;
-    return cudaLaunchKernelEx(&lc, k_commit_red, a);
+    return cudaLaunchKernelEx(&lc, k_commit_red<A>, a);
+}
+
+}  // namespace
+
+cudaError_t launch_commit_red(const hybrid_cfg &c, const void *K, const void *V, int n_tok, const void *W,
+                              void *const *states, int n_req, unsigned *err, cudaStream_t st)
+{
+    CommitArgs a;
+    if (!fill_commit_args(c, K, V, (long long)n_req * n_tok, W, states, n_req, err, a)) return cudaErrorInvalidValue;
+    a.T = n_tok;
+    return run_commit_red(c, a, st);
+}
+
+cudaError_t launch_commit_red_ragged(const hybrid_cfg &c, const void *K, const void *V, const int *tok,
+                                     const void *W, void *const *states, int n_req, unsigned *err, cudaStream_t st)
+{
+    if (n_req < 1 || n_req > kMaxRaggedRequests) return cudaErrorInvalidValue;
+    static thread_local CommitRaggedArgs a;   // 8 KB of offsets: kept off the stack
+    if (!fill_commit_args(c, K, V, tok[n_req] > 0 ? tok[n_req] : 1, W, states, n_req, err, a))
+        return cudaErrorInvalidValue;
+    a.T = 0;
+    a.n_req = n_req;
+    for (int r = 0; r <= n_req; ++r) a.tok[r] = tok[r];
+    return run_commit_red(c, a, st);
 }
 
 }  // namespace hyb

@@ -44,14 +44,49 @@ constexpr int kSmemLimit = 232448;
 constexpr int kOneCtaPerSm = 118 * 1024;
 constexpr uint32_t kColDS = 256;      // dS^T: phi+ features at [256, 256 + F), phi- at [256 + F, 256 + 2F)
 constexpr uint32_t kAtom = kCT * 128;   // one 64-column atom of a 128-row operand
+constexpr int kMaxRaggedReq = kMaxRaggedRequests;
 
 struct PrefillArgs {
-    CUtensorMap tmK, tmV, tmW;   // K, V [n*T][Hkv][d] (box 64 x 1 x 128), W [Hkv*d][F] (box 64 x d); 128-byte swizzle
+    CUtensorMap tmK, tmV, tmW;   // K, V [tokens][Hkv][d] (box 64 x 1 x 128), W [Hkv*d][F] (box 64 x d); 128-byte swizzle
     void *const *states;
     unsigned *err;
     int n_units, T, Hkv, d, F, n_chunks;
     uint32_t off_w, off_k, off_v, off_p, off_s, off_dz, off_bar;
 };
+// Ragged prompts: request r owns tokens [tok[r], tok[r + 1]) of the packed K and V
+// and chunks [ch[r], ch[r + 1]) of each of its heads; carried in the parameters.
+struct PrefillRaggedArgs : PrefillArgs {
+    int n_req;
+    int tok[kMaxRaggedReq + 1];
+    int ch[kMaxRaggedReq + 1];
+};
+
+// Per-request token ranges and chunk counts, uniform or ragged.
+__device__ __forceinline__ int req_tok0(const PrefillArgs &a, int r) { return r * a.T; }
+__device__ __forceinline__ int req_len(const PrefillArgs &a, int) { return a.T; }
+__device__ __forceinline__ int req_nch(const PrefillArgs &a, int) { return a.n_chunks; }
+__device__ __forceinline__ long long total_chunks(const PrefillArgs &a) { return (long long)a.n_units * a.n_chunks; }
+__device__ __forceinline__ int req_tok0(const PrefillRaggedArgs &a, int r) { return a.tok[r]; }
+__device__ __forceinline__ int req_len(const PrefillRaggedArgs &a, int r) { return a.tok[r + 1] - a.tok[r]; }
+__device__ __forceinline__ int req_nch(const PrefillRaggedArgs &a, int r) { return a.ch[r + 1] - a.ch[r]; }
+__device__ __forceinline__ long long total_chunks(const PrefillRaggedArgs &a) { return (long long)a.Hkv * a.ch[a.n_req]; }
+// request of global chunk c: request r holds chunks [Hkv ch[r], Hkv ch[r + 1])
+__device__ __forceinline__ int chunk_req(const PrefillArgs &a, long long c)
+{
+    return (int)(c / ((long long)a.Hkv * a.n_chunks));
+}
+__device__ __forceinline__ long long req_chunk0(const PrefillArgs &a, int r) { return (long long)r * a.Hkv * a.n_chunks; }
+__device__ __forceinline__ int chunk_req(const PrefillRaggedArgs &a, long long c)
+{
+    int lo = 0, hi = a.n_req;   // the last r with Hkv ch[r] <= c (empty requests precede it)
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if ((long long)a.Hkv * a.ch[mid] <= c) lo = mid;
+        else hi = mid;
+    }
+    return lo;
+}
+__device__ __forceinline__ long long req_chunk0(const PrefillRaggedArgs &a, int r) { return (long long)a.Hkv * a.ch[r]; }
 
 // Shared memory: [W: F/64 atoms of d rows][K: 2 atoms of 128 rows][V x 2: 2 atoms each]
 // [phi(K): 2F/64 atoms of 128 rows][dz: 4 x 2F][barriers].  K and V always have
@@ -103,49 +138,64 @@ struct UnitCache {
 };
 
 // Position of a chunk within its unit and run.  A role walks its CTA's chunk
-// range in order: one division at the start, then the unit and the chunk index
-// advance incrementally.
+// range in order: the request is located once at the start, then the head and
+// the chunk index advance incrementally (skipping requests without tokens).
 struct ChunkPos {
     int u, j;
+    int row0, nt;       // first token row in K and V, valid tokens
     bool first, last;   // first / last chunk of its run in this CTA's range
 };
+template <class A>
 struct ChunkWalk {
     long long c, lo, hi;
-    int u, j;
-    __device__ __forceinline__ ChunkWalk(const PrefillArgs &a, long long lo_, long long hi_)
-        : c(lo_), lo(lo_), hi(hi_), u((int)(lo_ / a.n_chunks)), j((int)(lo_ % a.n_chunks)) {}
+    int r, g, j, nch;
+    __device__ __forceinline__ ChunkWalk(const A &a, long long lo_, long long hi_) : c(lo_), lo(lo_), hi(hi_)
+    {
+        r = lo_ < hi_ ? chunk_req(a, lo_) : 0;
+        nch = lo_ < hi_ ? req_nch(a, r) : 1;
+        const long long rem = lo_ - req_chunk0(a, r);
+        g = (int)(rem / nch);
+        j = (int)(rem % nch);
+    }
     __device__ __forceinline__ bool more() const { return c < hi; }
-    __device__ __forceinline__ ChunkPos pos(const PrefillArgs &a) const
+    __device__ __forceinline__ ChunkPos pos(const A &a) const
     {
         ChunkPos p;
-        p.u = u;
+        p.u = r * a.Hkv + g;
         p.j = j;
+        p.row0 = req_tok0(a, r) + j * kCT;
+        p.nt = min(kCT, req_len(a, r) - j * kCT);
         p.first = c == lo || j == 0;
-        p.last = c == hi - 1 || j == a.n_chunks - 1;
+        p.last = c == hi - 1 || j == nch - 1;
         return p;
     }
-    __device__ __forceinline__ void next(const PrefillArgs &a)
+    __device__ __forceinline__ void next(const A &a)
     {
-        ++c;
-        if (++j == a.n_chunks) {
-            j = 0;
-            ++u;
-        }
+        if (++c >= hi) return;
+        if (++j < nch) return;
+        j = 0;
+        if (++g < a.Hkv) return;
+        g = 0;
+        do {
+            ++r;
+        } while (req_nch(a, r) == 0);
+        nch = req_nch(a, r);
     }
 };
 
-__global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__ PrefillArgs a)
+template <class A>
+__global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__ A a)
 {
     using namespace ptx;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int d = a.d, F = a.F, T = a.T;
+    const int d = a.d, F = a.F;
     const int NCH = F / 32, NC = 2 * NCH;
     const uint32_t tile = (uint32_t)d * 128;
     // staging slots that fit in the phi(K) buffer (2 for d = 128, F = 64)
     const int NSS = min(kStage, (int)(((uint32_t)(2 * F / 64) * kAtom) / tile));
-    const long long total = (long long)a.n_units * a.n_chunks;
+    const long long total = total_chunks(a);
     const long long lo = total * (long long)blockIdx.x / (long long)gridDim.x;
     const long long hi = total * (long long)(blockIdx.x + 1) / (long long)gridDim.x;
 
@@ -207,11 +257,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
             int nw = 0, nk = 0, nv = 0;
             bool ok = true;
             UnitCache uc;
-            for (ChunkWalk w(a, lo, hi); w.more() && ok; w.next(a)) {
+            for (ChunkWalk<A> w(a, lo, hi); w.more() && ok; w.next(a)) {
                 const ChunkPos p = w.pos(a);
                 if (!uc.get(a, p.u)) continue;
-                const int r = p.u / a.Hkv, g = p.u % a.Hkv;
-                const int row0 = r * T + p.j * kCT;
+                const int g = p.u % a.Hkv;
+                const int row0 = p.row0;
                 if (p.first) {
                     if (s > 0 && !wait_bar(wfree, (s - 1) & 1u, fail)) break;
                     mbar_arrive_expect_tx(wfull, (uint32_t)(F / 64) * tile);
@@ -279,13 +329,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
                 if (pp.first && sd > 0 && !wait_bar(dsfree, (sd - 1) & 1u, fail)) return false;
                 if (pp.first) ++sd;
                 tc_fence_after();
-                dst(pi, min(kCT, T - pp.j * kCT), pp.first);
+                dst(pi, pp.nt, pp.first);
                 mma_commit(dsdone);
                 mma_commit(&vfree[pi & 1]);
                 if (pp.last) mma_commit(segdone);
                 return true;
             };
-            for (ChunkWalk w(a, lo, hi); w.more() && ok; w.next(a)) {
+            for (ChunkWalk<A> w(a, lo, hi); w.more() && ok; w.next(a)) {
                 const ChunkPos p = w.pos(a);
                 if (!uc.get(a, p.u)) continue;
                 if (p.first) {
@@ -315,7 +365,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
             uint32_t s = 0, sg = 0;
             bool ok = true;
             UnitCache uc;
-            for (ChunkWalk w(a, lo, hi); w.more() && ok; w.next(a)) {
+            for (ChunkWalk<A> w(a, lo, hi); w.more() && ok; w.next(a)) {
                 const ChunkPos p = w.pos(a);
                 float *Sg = uc.get(a, p.u);
                 if (!Sg || !p.last) continue;
@@ -353,13 +403,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
         float dzacc[4] = {0.f, 0.f, 0.f, 0.f};   // token sums of features part*F + 32*jj + lane
         bool ok = true;
         UnitCache uc;
-        for (ChunkWalk w(a, lo, hi); w.more() && ok; w.next(a)) {
+        for (ChunkWalk<A> w(a, lo, hi); w.more() && ok; w.next(a)) {
             const ChunkPos p = w.pos(a);
             if (!uc.get(a, p.u)) {
                 if (mt == 0) raise_error(a.err, ERR_BAD_STATE_PTR);
                 continue;
             }
-            const int nt = min(kCT, T - p.j * kCT);
+            const int nt = p.nt;
             const bool active = 32 * q4 < nt;      // warp-uniform: the warp holds a valid token
             const bool valid = tok < nt;
             const uint32_t ub = tmem + (i & 1) * F + lane_off;
@@ -522,32 +572,29 @@ bool prefill_supported(const hybrid_cfg &c)
     return (int)make_playout(c.head_dim, c.feat_dim).bytes <= kSmemLimit;
 }
 
-cudaError_t launch_prefill(const hybrid_cfg &c, const void *K, const void *V, int n_tok, const void *W,
-                           void *const *states, int n_req, unsigned *err, cudaStream_t st)
+namespace {
+
+// Tensor maps and sizes shared by the uniform and the ragged launch; rows = tokens of K and V.
+bool fill_prefill_args(const hybrid_cfg &c, const void *K, const void *V, long long rows, const void *W,
+                       void *const *states, int n_req, unsigned *err, PrefillArgs &a)
 {
     const PLayout L = make_playout(c.head_dim, c.feat_dim);
-    PrefillArgs a;
     const int d = c.head_dim, F = c.feat_dim, Hkv = c.n_kv_heads;
-    {
-        const cuuint64_t rows = (cuuint64_t)n_req * n_tok;
-        const cuuint64_t dk[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, rows};
-        const cuuint64_t sk[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
-        const cuuint32_t bk[3] = {64, 1, (cuuint32_t)kCT};
-        const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
-        const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
-        const cuuint32_t bw[2] = {64, (cuuint32_t)d};
-        if (!encode_bf16(&a.tmK, K, 3, dk, sk, bk) || !encode_bf16(&a.tmV, V, 3, dk, sk, bk) ||
-            !encode_bf16(&a.tmW, W, 2, dw, sw, bw))
-            return cudaErrorInvalidValue;
-    }
+    const cuuint64_t dk[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, (cuuint64_t)rows};
+    const cuuint64_t sk[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
+    const cuuint32_t bk[3] = {64, 1, (cuuint32_t)kCT};
+    const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
+    const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
+    const cuuint32_t bw[2] = {64, (cuuint32_t)d};
+    if (!encode_bf16(&a.tmK, K, 3, dk, sk, bk) || !encode_bf16(&a.tmV, V, 3, dk, sk, bk) ||
+        !encode_bf16(&a.tmW, W, 2, dw, sw, bw))
+        return false;
     a.states = states;
     a.err = err;
     a.n_units = n_req * Hkv;
-    a.T = n_tok;
     a.Hkv = Hkv;
     a.d = d;
     a.F = F;
-    a.n_chunks = (n_tok + kCT - 1) / kCT;
     a.off_w = L.off_w;
     a.off_k = L.off_k;
     a.off_v = L.off_v;
@@ -555,15 +602,22 @@ cudaError_t launch_prefill(const hybrid_cfg &c, const void *K, const void *V, in
     a.off_s = L.off_s;
     a.off_dz = L.off_dz;
     a.off_bar = L.off_bar;
-    const long long total = (long long)a.n_units * a.n_chunks;
+    return true;
+}
+
+template <class A>
+cudaError_t run_prefill(const hybrid_cfg &c, const A &a, long long total, cudaStream_t st)
+{
     if (total <= 0) return cudaSuccess;
+    const PLayout L = make_playout(c.head_dim, c.feat_dim);
     const int grid = total < sm_count() ? (int)total : sm_count();
     static std::atomic<unsigned long long> opted;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     const unsigned long long bit = 1ull << dev;
     if (!(opted.load(std::memory_order_acquire) & bit)) {
-        const cudaError_t e = cudaFuncSetAttribute(k_prefill, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
+        const cudaError_t e =
+            cudaFuncSetAttribute(k_prefill<A>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
         if (e != cudaSuccess) return e;
         opted.fetch_or(bit, std::memory_order_acq_rel);
     }
@@ -577,7 +631,35 @@ cudaError_t launch_prefill(const hybrid_cfg &c, const void *K, const void *V, in
     at[0].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = at;
     lc.numAttrs = 1;
-    return cudaLaunchKernelEx(&lc, k_prefill, a);
+    return cudaLaunchKernelEx(&lc, k_prefill<A>, a);
+}
+
+}  // namespace
+
+cudaError_t launch_prefill(const hybrid_cfg &c, const void *K, const void *V, int n_tok, const void *W,
+                           void *const *states, int n_req, unsigned *err, cudaStream_t st)
+{
+    PrefillArgs a;
+    if (!fill_prefill_args(c, K, V, (long long)n_req * n_tok, W, states, n_req, err, a)) return cudaErrorInvalidValue;
+    a.T = n_tok;
+    a.n_chunks = (n_tok + kCT - 1) / kCT;
+    return run_prefill(c, a, (long long)a.n_units * a.n_chunks, st);
+}
+
+cudaError_t launch_prefill_ragged(const hybrid_cfg &c, const void *K, const void *V, const int *tok, const void *W,
+                                  void *const *states, int n_req, unsigned *err, cudaStream_t st)
+{
+    if (n_req < 1 || n_req > kMaxRaggedReq) return cudaErrorInvalidValue;
+    static thread_local PrefillRaggedArgs a;   // 16 KB of offsets: kept off the stack
+    if (!fill_prefill_args(c, K, V, tok[n_req] > 0 ? tok[n_req] : 1, W, states, n_req, err, a))
+        return cudaErrorInvalidValue;
+    a.T = 0;
+    a.n_chunks = 0;
+    a.n_req = n_req;
+    a.ch[0] = 0;
+    for (int r = 0; r <= n_req; ++r) a.tok[r] = tok[r];
+    for (int r = 0; r < n_req; ++r) a.ch[r + 1] = a.ch[r] + (tok[r + 1] - tok[r] + kCT - 1) / kCT;
+    return run_prefill(c, a, (long long)c.n_kv_heads * a.ch[n_req], st);
 }
 
 }  // namespace hyb

@@ -32,4 +32,13 @@ cudaError_t launch_prefill(const hybrid_cfg &c, const void *K, const void *V, in
 cudaError_t launch_commit_red(const hybrid_cfg &c, const void *K, const void *V, int n_tok, const void *W,
                               void *const *states, int n_req, unsigned *err, cudaStream_t st);
 
+// Ragged prompts: request r folds tokens [tok[r], tok[r + 1]) of the packed K, V
+// [tok[n_req]][Hkv][d]; tok is a host array read at launch (its values travel in
+// the kernel parameters), so at most kMaxRaggedRequests requests per launch.
+constexpr int kMaxRaggedRequests = 2048;
+cudaError_t launch_prefill_ragged(const hybrid_cfg &c, const void *K, const void *V, const int *tok, const void *W,
+                                  void *const *states, int n_req, unsigned *err, cudaStream_t st);
+cudaError_t launch_commit_red_ragged(const hybrid_cfg &c, const void *K, const void *V, const int *tok,
+                                     const void *W, void *const *states, int n_req, unsigned *err, cudaStream_t st);
+
 }  // namespace hyb

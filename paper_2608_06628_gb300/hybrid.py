@@ -25,7 +25,8 @@ HYBRID_BF16 = 1
 
 EXPORTED = (
     "hybrid_state_bytes", "hybrid_state_init", "hybrid_feature_map", "hybrid_block_attn",
-    "hybrid_block_attn_commit", "hybrid_block_attn_commit_logical", "hybrid_commit_block", "hybrid_state_unpack",
+    "hybrid_block_attn_commit", "hybrid_block_attn_commit_logical", "hybrid_commit_block", "hybrid_commit_ragged",
+    "hybrid_state_unpack",
     "hybrid_state_pack", "hybrid_train_workspace_bytes", "hybrid_train_forward", "hybrid_train_backward",
     "hybrid_check", "hybrid_status_str",
 )
@@ -75,6 +76,7 @@ def lib(path: str | None = None):
     L.hybrid_block_attn_commit.argtypes = [cfgp, P, P, P, P, P, P, I, P, P]
     L.hybrid_block_attn_commit_logical.argtypes = [cfgp, P, P, P, P, P, P, P, I, P, P]
     L.hybrid_commit_block.argtypes = [cfgp, P, P, I, P, P, I, P]
+    L.hybrid_commit_ragged.argtypes = [cfgp, P, P, ctypes.POINTER(ctypes.c_int), I, P, P, P]
     L.hybrid_state_unpack.argtypes = [cfgp, P, I, P, P, P]
     L.hybrid_state_pack.argtypes = [cfgp, P, P, P, I, P]
     S = ctypes.c_size_t
@@ -167,6 +169,18 @@ def hybrid_commit_block(cfg, K, V, n_tok, W, state_ptrs, n_req, stream=None, che
     st = lib().hybrid_commit_block(ctypes.byref(cfg), _ptr(K), _ptr(V), int(n_tok), _ptr(W),
                                    _ptr(state_ptrs), int(n_req), _stream(stream))
     return _ret(st, "hybrid_commit_block", check)
+
+
+def hybrid_commit_ragged(cfg, K, V, tok_offsets, W, state_ptrs, n_req, stream=None, check=True):
+    """Prompt prefill with per-request lengths: request r folds rows
+    tok_offsets[r]:tok_offsets[r + 1] of the packed K, V [total, Hkv, d]."""
+    offs = [int(x) for x in tok_offsets]
+    if len(offs) != int(n_req) + 1:
+        raise ValueError(f"tok_offsets needs n_req + 1 = {int(n_req) + 1} entries, got {len(offs)}")
+    arr = (ctypes.c_int * len(offs))(*offs)
+    st = lib().hybrid_commit_ragged(ctypes.byref(cfg), _ptr(K), _ptr(V), arr, int(n_req), _ptr(W),
+                                    _ptr(state_ptrs), _stream(stream))
+    return _ret(st, "hybrid_commit_ragged", check)
 
 
 def hybrid_state_unpack(cfg, state_ptrs, n_req, S_logical, z_logical, stream=None, check=True):

@@ -87,6 +87,26 @@ def test_null_and_misaligned_pointers_rejected_on_host(L):
     assert L.hybrid_block_attn(None, ok, ok, ok, ok, ok, ok, 1, ok, None) == H.HYBRID_ERR_INVALID_ARG
 
 
+def test_ragged_commit_argument_checks(L):
+    """hybrid_commit_ragged validates its host offsets before touching the device."""
+    c = cfg()
+    ok = 1 << 20
+
+    def offs(*v):
+        return (ctypes.c_int * len(v))(*v)
+
+    rag = L.hybrid_commit_ragged
+    assert rag(ctypes.byref(c), ok, ok, offs(1, 5), 1, ok, ok, None) == H.HYBRID_ERR_INVALID_ARG    # not from 0
+    assert rag(ctypes.byref(c), ok, ok, offs(0, 5, 3), 2, ok, ok, None) == H.HYBRID_ERR_INVALID_ARG  # decreasing
+    assert rag(ctypes.byref(c), ok, ok, None, 2, ok, ok, None) == H.HYBRID_ERR_INVALID_ARG
+    assert rag(ctypes.byref(c), ok, None, offs(0, 3), 1, ok, ok, None) == H.HYBRID_ERR_INVALID_ARG
+    assert rag(ctypes.byref(c), ok + 8, ok, offs(0, 3), 1, ok, ok, None) == H.HYBRID_ERR_INVALID_ARG
+    assert rag(ctypes.byref(c), ok, ok, offs(0, 3), -1, ok, ok, None) == H.HYBRID_ERR_INVALID_ARG
+    # nothing to fold: no requests, or requests without tokens
+    assert rag(ctypes.byref(c), None, None, None, 0, None, None, None) == H.HYBRID_OK
+    assert rag(ctypes.byref(c), None, None, offs(0, 0, 0), 2, None, None, None) == H.HYBRID_OK
+
+
 def test_empty_batches_are_no_ops(L):
     c = cfg()
     assert L.hybrid_block_attn(ctypes.byref(c), None, None, None, None, None, None, 0, None, None) == H.HYBRID_OK

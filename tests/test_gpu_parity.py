@@ -340,6 +340,62 @@ def test_prefill_split_across_ctas(wl, T, prefix):
     assert_parity(z, pair.z, BF16, f"prefill {T} z")
 
 
+RAGGED = [
+    # token-major prefill kernel: long and empty prompts, tails of 1 and 1 + 128 tokens
+    (W_("ragged_prefill", BF16, 7, 4, 2, 128, 128, 32, 61), [300, 0, 129, 1, 1000, 64, 257], 64),
+    # per-unit reduction kernel: every prompt at most 64 tokens
+    (W_("ragged_short", BF16, 5, 4, 4, 128, 64, 32, 62), [32, 0, 17, 64, 1], 0),
+    # F = 256: one pass per sign, a prompt longer than a block
+    (W_("ragged_f256", BF16, 3, 2, 2, 128, 256, 64, 63), [100, 0, 33], 64),
+    # float32: the FMA kernel once per request
+    (W_("ragged_f32", F32, 3, 2, 1, 64, 32, 16, 64), [20, 0, 7], 16),
+]
+
+
+def _ragged_commit(pair, lens, tag):
+    """hybrid_commit_ragged on packed K, V; the oracle folds each tracked request's
+    own tokens alone."""
+    wl = pair.wl
+    lens = np.asarray(lens, dtype=np.int64)
+    offs = np.concatenate([[0], np.cumsum(lens)])
+    K, V = wk.prefix_kv(wl, tag, pair.dev, n_req=1, n_tok=int(offs[-1]))
+    Kp, Vp = K[0].contiguous(), V[0].contiguous()
+    H.hybrid_commit_ragged(pair.cfg, Kp, Vp, offs.tolist(), pair.W, pair.ptrs, wl.n_req)
+    H.hybrid_check()
+    for i, r in enumerate(pair.tracked):
+        if lens[r] == 0:
+            continue
+        a, b = int(offs[r]), int(offs[r + 1])
+        Sx, zx = pair.S[i:i + 1].copy(), pair.z[i:i + 1].copy()
+        pair.orc.commit(h64(Kp[a:b][None]), h64(Vp[a:b][None]), pair.W64, Sx, zx)
+        pair.S[i:i + 1], pair.z[i:i + 1] = Sx, zx
+
+
+@pytest.mark.parametrize("wl,lens,prefix", RAGGED, ids=[w.name for w, _, _ in RAGGED])
+def test_ragged_prefill(wl, lens, prefix):
+    """Prompts of different lengths in one hybrid_commit_ragged call, on top of a
+    prefix already in the state; an empty prompt leaves its state unchanged."""
+    pair = Pair(wl)
+    if prefix:
+        pair.build_prefixes(np.full(wl.n_req, prefix, dtype=np.int64))
+    _ragged_commit(pair, lens, 71)
+    S, z = pair.gpu_state()
+    assert_parity(S, pair.S, wl.io_dtype, "ragged prefill S")
+    assert_parity(z, pair.z, wl.io_dtype, "ragged prefill z")
+
+
+def test_ragged_prefill_more_requests_than_one_launch():
+    """2100 requests of 0-3 tokens: two launches of at most 2048 requests, offsets
+    rebased for the second; the requests on both sides of the split are checked."""
+    wl = W_("ragged_many", BF16, 2100, 2, 1, 64, 64, 32, 65)
+    pair = Pair(wl, tracked=[0, 1, 3, 2046, 2047, 2048, 2049, 2099])
+    lens = np.arange(wl.n_req) % 4
+    _ragged_commit(pair, lens, 72)
+    S, z = pair.gpu_state()
+    assert_parity(S, pair.S, wl.io_dtype, "ragged S")
+    assert_parity(z, pair.z, wl.io_dtype, "ragged z")
+
+
 def test_prefill_commit_long_ragged():
     """Prompt prefill: commits of many tokens (T not a multiple of 32) in one call
     equal the same tokens committed in B-sized pieces."""
