@@ -518,11 +518,36 @@ def prefill_context(dev, wl, T=4096, warmup=2, iters=5):
     hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     bf16 = float(peaks.get("bf16_tflops", 1900.0))
     del K, V
-    return {"call": "hybrid_commit_block", "tokens_per_request": T, "us": ms * 1e3,
-            "algorithmic_bytes": nbytes, "GBps": nbytes / (ms * 1e-3) / 1e9,
-            "frac_hbm": nbytes / (ms * 1e-3) / 1e9 / hbm,
-            "TFLOPs": flops / (ms * 1e-3) / 1e12, "frac_bf16_peak": flops / (ms * 1e-3) / 1e12 / bf16,
-            "prompt_tokens_per_s": wl.n_req * T / (ms * 1e-3)}
+    out = {"call": "hybrid_commit_block", "tokens_per_request": T, "us": ms * 1e3,
+           "algorithmic_bytes": nbytes, "GBps": nbytes / (ms * 1e-3) / 1e9,
+           "frac_hbm": nbytes / (ms * 1e-3) / 1e9 / hbm,
+           "TFLOPs": flops / (ms * 1e-3) / 1e12, "frac_bf16_peak": flops / (ms * 1e-3) / 1e12 / bf16,
+           "prompt_tokens_per_s": wl.n_req * T / (ms * 1e-3)}
+    # the same requests with ragged prompt lengths, seeded U{1, ..., 2T - 1}, packed
+    # token-major (hybrid_commit_ragged); same bytes per token and per state
+    lens = np.random.default_rng(4097).integers(1, 2 * T, size=wl.n_req)
+    offs = np.concatenate([[0], np.cumsum(lens)]).tolist()
+    total = int(offs[-1])
+    Kr = torch.randn((total, wl.Hkv, wl.d), generator=g, device=dev, dtype=torch.float32).to(wl.io_dtype)
+    Vr = torch.randn((total, wl.Hkv, wl.d), generator=g, device=dev, dtype=torch.float32).to(wl.io_dtype)
+    for _ in range(warmup):
+        H.hybrid_commit_ragged(cfg, Kr, Vr, offs, W, ptrs, wl.n_req, stream.cuda_stream, check=False)
+    for a_, b_ in evs:
+        a_.record(stream)
+        H.hybrid_commit_ragged(cfg, Kr, Vr, offs, W, ptrs, wl.n_req, stream.cuda_stream, check=False)
+        b_.record(stream)
+    torch.cuda.synchronize()
+    status = H.hybrid_check(check=False)
+    if status != H.HYBRID_OK:
+        raise SystemExit(f"device error in the ragged prefill context: {H.hybrid_status_str(status)}")
+    ms_r = sorted(a_.elapsed_time(b_) for a_, b_ in evs)[iters // 2]
+    nbytes_r = 2 * Kr.numel() * io + 2 * units * (2 * wl.F * wl.d + 2 * wl.F) * 4 + wl.Hkv * wl.d * wl.F * io
+    out["ragged"] = {"call": "hybrid_commit_ragged", "tokens_per_request": f"U{{1..{2 * T - 1}}} (seeded)",
+                     "tokens": total, "us": ms_r * 1e3, "algorithmic_bytes": nbytes_r,
+                     "GBps": nbytes_r / (ms_r * 1e-3) / 1e9, "frac_hbm": nbytes_r / (ms_r * 1e-3) / 1e9 / hbm,
+                     "prompt_tokens_per_s": total / (ms_r * 1e-3)}
+    del Kr, Vr
+    return out
 
 
 # ---------------------------------------------------------------------------
