@@ -284,7 +284,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     auto comb_min = [&](float x) { return kSpread ? fminf(x, __shfl_xor_sync(0xffffffffu, x, 16)) : x; };
     auto comb_add = [&](float x) { return kSpread ? x + __shfl_xor_sync(0xffffffffu, x, 16) : x; };
 
-    // ---- round 1: local extrema
+    // ---- pass 1: local extrema
     {
         float ms = -INFINITY, mx = -INFINITY, mn = INFINITY;
         for (int k = sub; k < nsc; k += NS) {
@@ -325,7 +325,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     }
     if (!mbar_wait(bar_z, 0, kWaitNs)) atomicOr(fail, 1);
 
-    // ---- round 2: exponentials, P, unnormalised phi halves, partial sums
+    // ---- pass 2: exponentials, P, unnormalised phi halves, partial sums
     {
         const float m_raw = fmaxf(ex[0 * 256 + row], ex[0 * 256 + 128 + row]);
         const float mx = fmaxf(ex[1 * 256 + row], ex[1 * 256 + 128 + row]);
@@ -377,7 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     }
     __syncthreads();
 
-    // ---- round 3: normalise phi in place (rounded to tf32), row statistics
+    // ---- pass 3: normalise phi in place (rounded to tf32), row statistics
     {
         const float sp = ex[4 * 256 + row] + ex[4 * 256 + 128 + row];
         const float sn = ex[5 * 256 + row] + ex[5 * 256 + 128 + row];
@@ -501,7 +501,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
             }
             if (!mbar_wait(bar_u2, 0, kWaitNs)) atomicOr(fail, 1);
             tc_fence_after();
-            // phi- = softmax(-U), from the same extremum and sum as round 2, rounded to tf32
+            // phi- = softmax(-U), from the same extremum and sum as pass 2, rounded to tf32
             const float mnl = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]) * kLog2e;
             const float isn = 1.f / (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
             for (int k = sub; k < nfc; k += NS) {
