@@ -23,6 +23,7 @@ sample per step), printing the same JSON line with "impl": "reference".
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import math
@@ -307,14 +308,16 @@ def small_config_context(dev, warmup=5, iters=20):
     return out
 
 
-def large_config_context(dev, warmup=3, iters=15):
+def large_config_context(dev, warmup=3, iters=15, n_req=None):
     """Context for the two other large configurations (not part of the value):
     the per-call device time of the step (hybrid_block_attn) and of the block
     commit (hybrid_commit_block, B tokens), each launched directly, median of
     iters after warmup.  c4 is one layer of the decode loop (32 requests, MHA);
     its state fits in L2, so it rotates enough buffer sets that each call misses
     L2.  c5 (256 requests, F = 256) holds a 1.08 GB state and uses one set.  The
-    kernels' cost does not depend on the state's values: states start empty."""
+    kernels' cost does not depend on the state's values: states start empty.
+    n_req, if given, replaces both configurations' request count (a smaller case
+    of the same kernels, e.g. for a profiler capture)."""
     import torch
     from paper_2608_06628_gb300 import hybrid as H
     from paper_2608_06628_gb300 import workloads as wk
@@ -323,6 +326,8 @@ def large_config_context(dev, warmup=3, iters=15):
     hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     out = {}
     for wl in (wk.C4, wk.C5):
+        if n_req is not None:
+            wl = dataclasses.replace(wl, n_req=n_req)
         cfg = H.make_cfg(wl.d, wl.F, wl.Hq, wl.Hkv, wl.B, wl.io_dtype)
         W, alpha = wk.params(wl, device=dev)
         ab = algorithmic_bytes(wl, 2 if wl.io_dtype == torch.bfloat16 else 4)
@@ -875,6 +880,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-small-configs", action="store_true",
                     help="skip the context timings (c1/c2, c4/c5, prefill, training form)")
+    ap.add_argument("--n-req", type=int, default=None,
+                    help="with --context large: requests per configuration (default: the configs' own)")
     ap.add_argument("--context", choices=("train", "prefill", "small", "large"),
                     help="time only this context on cuda:0 and print its JSON object")
     args = ap.parse_args(argv)
@@ -889,7 +896,7 @@ def main(argv=None):
         dev = torch.device("cuda", 0)
         torch.cuda.set_device(dev)
         fn = {"train": lambda: train_context(dev), "prefill": lambda: prefill_context(dev, wl),
-              "small": lambda: small_config_context(dev), "large": lambda: large_config_context(dev)}[args.context]
+              "small": lambda: small_config_context(dev), "large": lambda: large_config_context(dev, n_req=args.n_req)}[args.context]
         print(json.dumps({"context": args.context, **fn()}), flush=True)
         return 0
     if args.impl == "reference":
