@@ -122,13 +122,14 @@ def test_c4_decode_loop_drift():
 def test_c5_full_sampled():
     """c5: 256 requests, 16 heads, F = 256, B = 64, ragged prefixes 1k-32k with
     keys x8 (normaliser and softmax range).  The GPU builds every prefix; the
-    oracle rebuilds the shortest, the longest and one other, then checks a step
-    and the following commit on them.  The step is also checked for every
+    oracle rebuilds 8 seeded requests (the shortest, the longest and six others),
+    then checks a step and the following commit on them.  The step is also checked for every
     request, the oracle reading the GPU's prefix states (a full oracle rebuild of
     all 256 prefixes is out of reach)."""
     wl = wk.C5
     plen = wk.prefix_lengths(wl)
-    pair = Pair(wl, tracked=_sample(plen, 1, 105))
+    pair = Pair(wl, tracked=_sample(plen, 6, 105))
+    assert len(pair.tracked) == 8
     pair.build_prefixes(plen)
     S, z = pair.gpu_state()
     assert_parity(S, pair.S, wl.io_dtype, "c5 prefix state S")
