@@ -150,23 +150,35 @@ hybrid_status hybrid_block_attn_commit(const hybrid_cfg *cfg, const void *Q, con
  * (64 MiB, part of the library's device image on every device it runs on). */
 #define HYBRID_LOGICAL_SCRATCH_BYTES (64u << 20)
 
-/* hybrid_block_attn_commit on states held in the LOGICAL layout (the paper has
- * no counterpart: this is an interface convenience for callers that keep
- * S [n][Hkv][2F][d] and z [n][Hkv][2F] float32 themselves, e.g. states moved in
- * from another framework).  One call packs the n_req states into the library's
- * static scratch (operand-image layout, plus the state-pointer array), runs the
- * fused step and commit there, and unpacks the updated states back in place:
+/* hybrid_block_attn_commit on states held in the LOGICAL layout, for callers
+ * that cannot allocate device memory.  The paper has no counterpart.  Some
+ * callers keep S [n][Hkv][2F][d] and z [n][Hkv][2F] float32 in their own
+ * buffers and cannot call cudaMalloc: a host application that owns all device
+ * memory through its own pool or budget, so that a library may not take any;
+ * a latency-critical decode loop, where an allocation can stall the loop
+ * (cudaFree synchronises the device).  Such callers cannot provide the pointer
+ * array and the operand-image states that hybrid_block_attn_commit reads.
+ * This entry point brings its own device memory instead: one file-scope array
+ * of HYBRID_LOGICAL_SCRATCH_BYTES per device, part of the library's device
+ * image and held by every GPU that loads the library until the process exits.
+ * One call packs the n_req states into that scratch (with the state-pointer
+ * array), runs the fused step and commit there, and unpacks the updated states
+ * back in place:
  *   Q, K, V, W, alpha, O  as in hybrid_block_attn (device pointers)
  *   S_logical, z_logical  device, read and overwritten with the committed state
- * It allocates nothing.  Errors: HYBRID_ERR_UNSUPPORTED when
- * ceil256(8 n_req) + n_req * hybrid_state_bytes(cfg) exceeds
- * HYBRID_LOGICAL_SCRATCH_BYTES (c3: 64 requests x 528 KB fit); otherwise as
- * hybrid_block_attn_commit.
- * Races: the scratch is one per device and shared by every caller, so two calls
- * must not overlap on a device (issue them on one stream, or synchronise).
- * Set-up: the first call on a device looks the scratch address up with the CUDA
- * runtime; make that call (n_req = 0 is enough) before capturing this entry
- * point in a CUDA graph. */
+ * It allocates nothing: no cudaMalloc, cudaFree or allocating library call.
+ * Errors (the size and pointer checks run on the host before anything is
+ * queued on the stream):
+ * HYBRID_ERR_UNSUPPORTED when n_req * (hybrid_state_bytes(cfg) + 8) + 255
+ * exceeds HYBRID_LOGICAL_SCRATCH_BYTES (up to 127 requests of 528 KB at c3's
+ * shape, 15 of 4.2 MB at c5's); HYBRID_ERR_INVALID_ARG for a null or misaligned
+ * pointer (S_logical, z_logical: 4-byte); otherwise as hybrid_block_attn_commit.
+ * Races: the scratch is one per device, shared by every call, and keeps the
+ * last call's contents (each call overwrites every byte it reads).  Calls that
+ * overlap on the GPU race on it: issue them on one stream, or synchronise.
+ * Set-up: the first call on a device, with that device current, looks the
+ * scratch address up with cudaGetSymbolAddress (n_req = 0 does only that).
+ * Make that first call before any stream capture begins. */
 hybrid_status hybrid_block_attn_commit_logical(const hybrid_cfg *cfg, const void *Q, const void *K,
                                                const void *V, const void *W, const float *alpha,
                                                float *S_logical, float *z_logical, int n_req, void *O,
@@ -252,6 +264,22 @@ hybrid_status hybrid_train_backward(const hybrid_cfg *cfg, const void *Q, const 
                                     const void *W, const float *alpha, const void *dO, int n_seq,
                                     int seq_len, void *workspace, size_t workspace_bytes, float *dW,
                                     float *dalpha, cudaStream_t stream);
+
+/* Testing hook for the device-side failure path; the paper has no counterpart.
+ * Every wait inside the tensor-core kernels is bounded (1 s of the device's
+ * global timer); when a bound runs out the kernel sets a bit in the device
+ * error word, leaves its remaining work, waits (bounded) for its own copies in
+ * flight, frees its Tensor Memory and returns, and hybrid_check() then reports
+ * HYBRID_ERR_TIMEOUT.  Arming makes the NEXT launch of the persistent step
+ * kernel (hybrid_block_attn on bf16 shapes with d, F in {64, 128}, B in
+ * {16, 32}, G*B <= 128) exercise that path without faulting anything: its
+ * waits give up after wait_ns nanoseconds instead of 1 s, and its math warps
+ * never signal the barrier that releases the readout of the first feature
+ * half (a barrier that no asynchronous copy targets), so the tensor-core
+ * issuer's wait on it runs out.  The launch consumes the setting; later
+ * launches run normally.  wait_ns = 0 disarms.  Errors: HYBRID_ERR_INVALID_ARG
+ * for wait_ns above 10 s.  Host-only; touches no device. */
+hybrid_status hybrid_debug_arm_wait_timeout(unsigned long long wait_ns);
 
 /* Synchronise the stream, then read and clear this device's error word.
  * Returns HYBRID_OK, HYBRID_ERR_DEVICE (a state pointer failed its device

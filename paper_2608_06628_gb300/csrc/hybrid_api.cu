@@ -86,6 +86,10 @@ hybrid_status from_cuda(cudaError_t e) { return e == cudaSuccess ? HYBRID_OK : H
 
 }  // namespace
 
+namespace hyb {
+std::atomic<unsigned long long> g_armed_wait_ns{0};
+}
+
 extern "C" {
 
 size_t hybrid_state_bytes(const hybrid_cfg *cfg)
@@ -169,18 +173,35 @@ hybrid_status hybrid_block_attn_commit_logical(const hybrid_cfg *cfg, const void
     hybrid_status s = check_cfg(cfg);
     if (s != HYBRID_OK) return s;
     if (n_req < 0) return HYBRID_ERR_INVALID_ARG;
+    // Size first, on the host, in a form that cannot wrap: the pointer array takes
+    // at most 8 n_req + 255 bytes once rounded up to 256, so
+    //   n_req (8 + sb) + 255 <= kScratchBytes  implies  ceil256(8 n_req) + n_req sb <= kScratchBytes.
+    const size_t sb = hybrid_state_bytes(cfg);   // a multiple of 16 bytes
+    if (sb == 0) return HYBRID_ERR_UNSUPPORTED;
+    if ((size_t)n_req > (kScratchBytes - 255) / (sb + sizeof(void *))) return HYBRID_ERR_UNSUPPORTED;
+    // every pointer is checked before any work is queued on the stream
+    if (n_req > 0) {
+        if (!Q || !K || !V || !W || !alpha || !O || !S_logical || !z_logical) return HYBRID_ERR_INVALID_ARG;
+        if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(W, 16) || !aligned(O, 16) ||
+            !aligned(alpha, 4) || !aligned(S_logical, 4) || !aligned(z_logical, 4))
+            return HYBRID_ERR_INVALID_ARG;
+    }
     // the scratch address is looked up here, also for n_req = 0 (set-up call)
     unsigned char *base = scratch();
     if (!base) return HYBRID_ERR_CUDA;
     if (n_req == 0) return HYBRID_OK;
-    if (!S_logical || !z_logical || !aligned(S_logical, 4) || !aligned(z_logical, 4)) return HYBRID_ERR_INVALID_ARG;
-    const size_t sb = hybrid_state_bytes(cfg);   // a multiple of 16 bytes
     const size_t ptr_bytes = ((size_t)n_req * sizeof(void *) + 255) & ~(size_t)255;
-    if (sb == 0 || (size_t)n_req > (kScratchBytes - ptr_bytes) / sb) return HYBRID_ERR_UNSUPPORTED;
     void **d_ptrs = reinterpret_cast<void **>(base);
     unsigned char *states = base + ptr_bytes;
-    k_fill_ptrs<<<(n_req + 127) / 128, 128, 0, stream>>>(d_ptrs, states, sb, n_req);
-    if (cudaGetLastError() != cudaSuccess) return HYBRID_ERR_CUDA;
+    {
+        // the launch's own status (not an error left over from earlier work)
+        size_t stride = sb;
+        int n = n_req;
+        void *args[] = {&d_ptrs, &states, &stride, &n};
+        const cudaError_t e = cudaLaunchKernel(reinterpret_cast<const void *>(&k_fill_ptrs),
+                                               dim3((unsigned)((n_req + 127) / 128)), dim3(128), args, 0, stream);
+        if (e != cudaSuccess) return HYBRID_ERR_CUDA;
+    }
     s = hybrid_state_pack(cfg, S_logical, z_logical, d_ptrs, n_req, stream);
     if (s != HYBRID_OK) return s;
     s = hybrid_block_attn_commit(cfg, Q, K, V, W, alpha, d_ptrs, n_req, O, stream);
@@ -353,6 +374,13 @@ hybrid_status hybrid_train_backward(const hybrid_cfg *cfg, const void *Q, const 
     if (!err) return HYBRID_ERR_CUDA;
     return from_cuda(hyb::launch_train_backward(*cfg, Q, K, V, W, alpha, dO, n_seq, seq_len, workspace, dW, dalpha,
                                                 err, stream));
+}
+
+hybrid_status hybrid_debug_arm_wait_timeout(unsigned long long wait_ns)
+{
+    if (wait_ns > 10000000000ull) return HYBRID_ERR_INVALID_ARG;
+    hyb::g_armed_wait_ns.store(wait_ns);
+    return HYBRID_OK;
 }
 
 hybrid_status hybrid_check(cudaStream_t stream)

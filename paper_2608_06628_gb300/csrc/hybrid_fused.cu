@@ -94,6 +94,8 @@ struct FusedArgs {
     unsigned *err;
     int n_units, B, Hq, Hkv, G, d, F, NS;
     float scale;
+    unsigned long long wait_ns;       // limit of every bounded wait (1 s unless a test armed less)
+    int withhold;                     // test hook: the math warps never signal phip
     uint32_t off_q, off_wk, off_vb, off_p, off_pk, off_z, off_st, off_bar;
 };
 
@@ -162,6 +164,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int d = a.d, F = a.F, B = a.B, G = a.G, NS = a.NS;
+    const uint64_t wlim = a.wait_ns;
     const int NCH = F / 32;          // 32-feature chunks (state tiles) per half of phi
     const int NC = 2 * NCH;          // state tiles per unit
     // with the commit the output tile is staged in the slots of tiles ocm, ocm + 1
@@ -259,16 +262,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 float *Sg = unit_state(a, u);
                 if (!Sg) continue;
                 const int zb = kp & 1;
-                if (!wait_bar(&zempty[zb], ((kp >> 1) & 1u) ^ 1u, fail)) break;
+                if (!wait_bar(&zempty[zb], ((kp >> 1) & 1u) ^ 1u, fail, wlim)) break;
                 mbar_arrive_expect_tx(&zfull[zb], 2 * F * 4);
                 bulk_g2s(zbuf0 + zb * zstride, Sg + (size_t)2 * F * d, 2 * F * 4, &zfull[zb]);
                 ++issued_z[zb];
                 // at start-up every SM asks for its first unit at once: let Q, W and K
                 // (needed first) arrive before the state tiles (needed after g1 and phi)
-                if (kp == 0 && !wait_bar(xfull, 0, fail)) break;
+                if (kp == 0 && !wait_bar(xfull, 0, fail, wlim)) break;
                 for (int c = 0; c < NC; ++c, ++q) {
                     const int slot = q % NS;
-                    if (!wait_bar(&empty[slot], ((q / NS) & 1u) ^ 1u, fail)) { ok = false; break; }
+                    if (!wait_bar(&empty[slot], ((q / NS) & 1u) ^ 1u, fail, wlim)) { ok = false; break; }
                     mbar_arrive_expect_tx(&full[slot], chunk_bytes);
                     bulk_g2s(ring + (size_t)slot * chunk_bytes, Sg + (size_t)c * 32 * d, chunk_bytes, &full[slot]);
                     ++issued_slot[slot];
@@ -318,7 +321,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             // (first: the tile's first MMA initialises the accumulator)
             auto readout = [&](uint32_t dcol, uint32_t acol, uint32_t qc, bool first = false) -> int {
                 const int slot = qc % NS;
-                if (!wait_bar(&full[slot], (qc / NS) & 1u, fail)) return -1;
+                if (!wait_bar(&full[slot], (qc / NS) & 1u, fail, wlim)) return -1;
                 tc_fence_after();
                 const uint32_t s_u = ring_u + slot * chunk_bytes;
 #pragma unroll
@@ -341,7 +344,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 // R- of the previous unit: its phi- sits in the phi columns R+ has consumed
                 auto tail = [&](uint32_t ik, uint32_t iq) -> bool {
                     const uint32_t T = (ik & 1) * 256;
-                    if (!wait_bar(phim, ik & 1u, fail)) return false;
+                    if (!wait_bar(phim, ik & 1u, fail, wlim)) return false;
                     tc_fence_after();
                     for (int c = NCH; c < NC; ++c) {
                         const int slot = readout(T + 128, T + 32 * (c - NCH), iq + c);
@@ -353,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 };
                 // P'V and R- of the previous unit: its P' and phi- come last
                 auto finish = [&](uint32_t ik, uint32_t iq) -> bool {
-                    if (!wait_bar(pready, ik & 1u, fail) || !wait_bar(vfull, ik & 1u, fail)) return false;
+                    if (!wait_bar(pready, ik & 1u, fail, wlim) || !wait_bar(vfull, ik & 1u, fail, wlim)) return false;
                     tc_fence_after();
                     pv((ik & 1) * 256 + 128);
                     mma_commit(vfree);
@@ -362,14 +365,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 for (int u = u_begin; u < u_end; ++u) {
                     if (!unit_state(a, u)) continue;
                     const uint32_t T = (kp & 1) * 256;
-                    if (!wait_bar(xfull, kp & 1u, fail)) { ok = false; break; }
-                    if (kp >= 2 && !wait_bar(&dfree[kp & 1], ((kp - 2) >> 1) & 1u, fail)) { ok = false; break; }
+                    if (!wait_bar(xfull, kp & 1u, fail, wlim)) { ok = false; break; }
+                    if (kp >= 2 && !wait_bar(&dfree[kp & 1], ((kp - 2) >> 1) & 1u, fail, wlim)) { ok = false; break; }
                     tc_fence_after();
                     g1(T, 0);
                     mma_commit(uready);
                     mma_commit(xfree);
                     if (kp >= 1 && !finish(kp - 1, prev_qt)) { ok = false; break; }
-                    if (!wait_bar(phip, kp & 1u, fail)) { ok = false; break; }
+                    if (!wait_bar(phip, kp & 1u, fail, wlim)) { ok = false; break; }
                     tc_fence_after();
                     for (int c = 0; c < NCH; ++c) {
                         const int slot = readout(T + 128, T + 32 * c, qt + c, c == 0);
@@ -390,29 +393,29 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 // free for their increments as soon as dS^T is in Tensor Memory.
                 for (int u = u_begin; u < u_end; ++u) {
                     if (!unit_state(a, u)) continue;
-                    if (!wait_bar(xfull, kp & 1u, fail)) { ok = false; break; }
+                    if (!wait_bar(xfull, kp & 1u, fail, wlim)) { ok = false; break; }
                     // U_k^T and the scores land in the dS+ columns: the previous unit's
                     // first-half update must have read them (its R- precedes in issue order)
-                    if (kp >= 1 && !wait_bar(efree, (kp - 1) & 1u, fail)) { ok = false; break; }
+                    if (kp >= 1 && !wait_bar(efree, (kp - 1) & 1u, fail, wlim)) { ok = false; break; }
                     tc_fence_after();
                     g1(kCmP, kCmK);
                     mma_commit(uready);
                     mma_commit(xfree);
                     // phip also covers the previous unit's output epilogue and second-half update
-                    if (!wait_bar(phip, kp & 1u, fail)) { ok = false; break; }
+                    if (!wait_bar(phip, kp & 1u, fail, wlim)) { ok = false; break; }
                     tc_fence_after();
                     for (int c = 0; c < NCH && ok; ++c) ok = readout(kCmD, kCmDSm + 32 * c, qt + c, c == 0) >= 0;
                     if (!ok) break;
-                    if (!wait_bar(kready, kp & 1u, fail) || !wait_bar(vfull, kp & 1u, fail)) { ok = false; break; }
+                    if (!wait_bar(kready, kp & 1u, fail, wlim) || !wait_bar(vfull, kp & 1u, fail, wlim)) { ok = false; break; }
                     tc_fence_after();
                     ds(kCmDSp, 0);
                     ds(kCmDSm, 1);
                     mma_commit(dsdone);
-                    if (!wait_bar(pready, kp & 1u, fail)) { ok = false; break; }
+                    if (!wait_bar(pready, kp & 1u, fail, wlim)) { ok = false; break; }
                     tc_fence_after();
                     pv(kCmD);
                     mma_commit(pvdone);
-                    if (!wait_bar(phim, kp & 1u, fail)) { ok = false; break; }
+                    if (!wait_bar(phim, kp & 1u, fail, wlim)) { ok = false; break; }
                     tc_fence_after();
                     for (int c = NCH; c < NC && ok; ++c) ok = readout(kCmD, kCmP + 32 * (c - NCH), qt + c) >= 0;
                     if (!ok) break;
@@ -437,7 +440,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             KtRegs kr;
             kt_load(a.K, (size_t)r * B, B, a.Hkv, g, d, kr, lane);   // in flight while the region drains
             bool ok = true;
-            if (kp > 0) ok = wait_bar(xfree, (kp - 1) & 1u, fail);
+            if (kp > 0) ok = wait_bar(xfree, (kp - 1) & 1u, fail, wlim);
             if (__any_sync(0xffffffffu, !ok)) break;
             // with the commit the Q region holds the previous unit's V, P' and phi(K)
             // until its dS^T and P V have run (Q then follows K^T, which measured
@@ -454,7 +457,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             kt_store(kr, d, kt, lane);
             fence_proxy_async_smem();
             __syncwarp();
-            if (!q_early && kp > 0) ok = wait_bar(pvdone, (kp - 1) & 1u, fail);
+            if (!q_early && kp > 0) ok = wait_bar(pvdone, (kp - 1) & 1u, fail, wlim);
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
                 if (!q_early)
@@ -465,7 +468,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             ++nx;
             // V: after the previous unit's P V (step), after this unit's g1 has read
             // Q (commit: V shares the Q region)
-            ok = kCommit ? wait_bar(xfree, kp & 1u, fail) : (kp == 0 || wait_bar(vfree, (kp - 1) & 1u, fail));
+            ok = kCommit ? wait_bar(xfree, kp & 1u, fail, wlim) : (kp == 0 || wait_bar(vfree, (kp - 1) & 1u, fail, wlim));
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
                 mbar_arrive_expect_tx(vfull, (uint32_t)(d / 64) * (B * 128));
@@ -492,13 +495,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 bool ok = true;
                 if (kCommit) {
                     const int zb = kp & 1;
-                    if (!wait_bar(zdone, kp & 1u, fail)) break;
+                    if (!wait_bar(zdone, kp & 1u, fail, wlim)) break;
                     bulk_s2g(Sg + (size_t)2 * F * d, zbuf0 + zb * zstride, 2 * F * 4);
                     bulk_commit();
                     bulk_wait_read_all();
                     mbar_arrive(&zempty[zb]);
                     for (int h = 0; h < 2 && ok; ++h) {
-                        if (!wait_bar(&tready[h], kp & 1u, fail)) { ok = false; break; }
+                        if (!wait_bar(&tready[h], kp & 1u, fail, wlim)) { ok = false; break; }
                         // one bulk group per tile; the two output slots are freed as
                         // soon as their reductions have read them
                         for (int c = h * NCH; c < (h + 1) * NCH; ++c) {
@@ -519,7 +522,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     if (!ok) break;
                 }
                 // output tile: two TMA boxes from the two held-back slots
-                if (!wait_bar(ostaged, kp & 1u, fail)) break;
+                if (!wait_bar(ostaged, kp & 1u, fail, wlim)) break;
                 uint8_t *s0 = ring + (size_t)((q + ocm) % NS) * chunk_bytes;
                 uint8_t *s1 = ring + (size_t)((q + ocm + 1) % NS) * chunk_bytes;
                 if (d == 128) {
@@ -569,8 +572,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         // tiles do not wait for this unit's output.
         auto epilogue = [&](uint32_t ek, uint32_t eq, float inv, int eu) -> bool {
             const uint32_t dcol = kCommit ? kCmD : (ek & 1) * 256 + 128;
-            bool ok = wait_bar(&dready[ek & 1], (ek >> 1) & 1u, fail);
-            if (kCommit && ok) ok = wait_bar(ofree, ek & 1u, fail);
+            bool ok = wait_bar(&dready[ek & 1], (ek >> 1) & 1u, fail, wlim);
+            if (kCommit && ok) ok = wait_bar(ofree, ek & 1u, fail, wlim);
             tc_fence_after();
             const int dh = d / 2;
             if (!kCommit) {
@@ -652,7 +655,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
 
             // ---- phase A: row extrema of U and of the scores (U kept in registers);
             // commit: per-token extrema of U_k^T over this warp's 32 features
-            bool bad = !wait_bar(uready, kp & 1u, fail);
+            bool bad = !wait_bar(uready, kp & 1u, fail, wlim);
             tc_fence_after();
             float sc[16], u0[32], u1[32];
             if (kCommit) {
@@ -708,7 +711,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
 
             // ---- phase B1: phi+ (unnormalised) into Tensor Memory; once the row sums are
             // exchanged, R+ may start on it (unless the warp needs the exact rescale)
-            bad = !wait_bar(&zfull[zb], (kp >> 1) & 1u, fail);
+            bad = !wait_bar(&zfull[zb], (kp >> 1) & 1u, fail, wlim);
             const float mxl = mx * kLog2e, mnl = mn * kLog2e, ml = ms * scale_l2;
             const float lw = valid ? log_sigmoid(alpha_row) : 0.f;
             float lp = 0.f;
@@ -758,7 +761,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(phip);
+                if (lane == 0 && !a.withhold) mbar_arrive(phip);
             }
 
             // ---- phase B2: phi- (kept in registers until R+ has consumed phi+), the
@@ -910,10 +913,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     tmem_wait_st();
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(phip);
+                    if (lane == 0 && !a.withhold) mbar_arrive(phip);
                 }
                 // step: the previous unit's P'V (issued after this unit's g1) has read P'
-                if (!kCommit && kp >= 1) bad = !wait_bar(vfree, (kp - 1) & 1u, fail) || bad;
+                if (!kCommit && kp >= 1) bad = !wait_bar(vfree, (kp - 1) & 1u, fail, wlim) || bad;
                 if (has_sc) {
                     // P' (w e^(s - sigma), or w sp e^s on the fast path): K-major, no swizzle
                     // (8-row x 16-byte core matrices)
@@ -947,7 +950,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     tmem_st32(pcol + 32 * k, x);
                 }
             } else {
-                bad = !wait_bar(pread, kp & 1u, fail) || bad;
+                bad = !wait_bar(pread, kp & 1u, fail, wlim) || bad;
                 tc_fence_after();
 #pragma unroll
                 for (int i = 0; i < 32; ++i) u0[i] *= cneg;
@@ -971,8 +974,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 const int e = row;
 #pragma unroll 1
                 for (int h = 0; h < 2; ++h) {
-                    const bool bad2 = h == 0 ? !wait_bar(dsdone, kp & 1u, fail) || bad
-                                             : !wait_bar(&dready[kp & 1], (kp >> 1) & 1u, fail);
+                    const bool bad2 = h == 0 ? !wait_bar(dsdone, kp & 1u, fail, wlim) || bad
+                                             : !wait_bar(&dready[kp & 1], (kp >> 1) & 1u, fail, wlim);
                     tc_fence_after();
                     const uint32_t src = tmem + (h == 0 ? kCmDSp : kCmDSm) + lane_off;
                     auto upd = [&](int k) {
@@ -1077,6 +1080,12 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
     a.F = c.feat_dim;
     a.NS = L.NS;
     a.scale = 1.f / sqrtf((float)c.head_dim);
+    {
+        // a test may arm one step launch with a short wait limit and a withheld arrival
+        const unsigned long long armed = commit ? 0ull : g_armed_wait_ns.exchange(0ull);
+        a.wait_ns = armed ? armed : (unsigned long long)kWaitNs;
+        a.withhold = armed ? 1 : 0;
+    }
     a.off_q = L.off_q;
     a.off_wk = L.off_wk;
     a.off_vb = L.off_vb;

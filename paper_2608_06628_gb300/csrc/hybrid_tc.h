@@ -3,9 +3,16 @@
 
 #include <cuda_runtime.h>
 
+#include <atomic>
+
 #include "hybrid.h"
 
 namespace hyb {
+
+// Test hook (hybrid_debug_arm_wait_timeout): when nonzero, the next launch of the
+// persistent step kernel takes it as its wait limit in nanoseconds and withholds
+// one barrier arrival; the launch consumes it.
+extern std::atomic<unsigned long long> g_armed_wait_ns;
 
 // True when hybrid_block_attn for this cfg runs on the tcgen05 kernel.
 bool tc_attn_supported(const hybrid_cfg &c);

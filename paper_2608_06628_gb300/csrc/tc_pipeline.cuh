@@ -34,15 +34,17 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b)
     return *reinterpret_cast<const uint32_t *>(&v);
 }
 
-// Bounded wait that also gives up as soon as another role has failed.
-__device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, volatile int *fail)
+// Bounded wait that also gives up as soon as another role has failed (limit in
+// nanoseconds of %globaltimer; kernels may take it from their arguments).
+__device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, volatile int *fail,
+                                         uint64_t limit_ns = kWaitNs)
 {
     if (ptx::mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = ptx::global_timer_ns();
     while (true) {
         if (ptx::mbar_try_wait_sleep(bar, parity, 200000u)) return true;
         if (*fail) return false;
-        if (ptx::global_timer_ns() - t0 > kWaitNs) {
+        if (ptx::global_timer_ns() - t0 > limit_ns) {
             atomicOr(const_cast<int *>(fail), 1);
             return false;
         }

@@ -28,7 +28,7 @@ EXPORTED = (
     "hybrid_block_attn_commit", "hybrid_block_attn_commit_logical", "hybrid_commit_block", "hybrid_commit_ragged",
     "hybrid_state_unpack",
     "hybrid_state_pack", "hybrid_train_workspace_bytes", "hybrid_train_forward", "hybrid_train_backward",
-    "hybrid_check", "hybrid_status_str",
+    "hybrid_debug_arm_wait_timeout", "hybrid_check", "hybrid_status_str",
 )
 
 
@@ -84,6 +84,7 @@ def lib(path: str | None = None):
     L.hybrid_train_workspace_bytes.restype = S
     L.hybrid_train_forward.argtypes = [cfgp, P, P, P, P, P, I, I, P, P, S, P]
     L.hybrid_train_backward.argtypes = [cfgp, P, P, P, P, P, P, I, I, P, S, P, P, P]
+    L.hybrid_debug_arm_wait_timeout.argtypes = [ctypes.c_ulonglong]
     L.hybrid_check.argtypes = [P]
     L.hybrid_status_str.argtypes = [I]
     L.hybrid_status_str.restype = ctypes.c_char_p
@@ -213,6 +214,13 @@ def hybrid_train_backward(cfg, Q, K, V, W, alpha, dO, n_seq, seq_len, workspace,
                                      _ptr(dO), int(n_seq), int(seq_len), _ptr(workspace),
                                      int(workspace_bytes), _ptr(dW), _ptr(dalpha), _stream(stream))
     return _ret(st, "hybrid_train_backward", check)
+
+
+def hybrid_debug_arm_wait_timeout(wait_ns, check=True):
+    """Test hook: the next persistent step launch gives up its waits after
+    wait_ns nanoseconds and withholds one barrier arrival (see hybrid.h)."""
+    st = lib().hybrid_debug_arm_wait_timeout(int(wait_ns))
+    return _ret(st, "hybrid_debug_arm_wait_timeout", check)
 
 
 def hybrid_check(stream=None, check=True):

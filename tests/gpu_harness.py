@@ -29,7 +29,30 @@ def rel_l2(got, want):
     return float(np.linalg.norm(got - want) / (den if den > 0 else 1.0))
 
 
-def assert_parity(got, want, dtype, what=""):
+# Axes that index one unit of work in each kind of compared array:
+#   "out"   [n, B, Hq, d]     one (request, query head)
+#   "state" [n, Hkv, 2F, d] and z [n, Hkv, 2F]: one (request, state head)
+UNIT_AXES = {"out": (0, 2), "state": (0, 1)}
+
+
+def unit_rel_l2(got, want, axes):
+    """rel-L2 of every unit (the indices along `axes`), as an array over units."""
+    got = np.asarray(got, dtype=np.float64)
+    want = np.asarray(want, dtype=np.float64)
+    rest = tuple(i for i in range(got.ndim) if i not in axes)
+    g = np.transpose(got, axes + rest).reshape(int(np.prod([got.shape[i] for i in axes])), -1)
+    w = np.transpose(want, axes + rest).reshape(g.shape)
+    num = np.linalg.norm(g - w, axis=1)
+    den = np.linalg.norm(w, axis=1)
+    return num / np.where(den > 0, den, 1.0)
+
+
+def assert_parity(got, want, dtype, what="", units=None):
+    """Element-wise parity of a GPU result with the oracle's.
+
+    The bound of the dtype applies to the whole tensor and, for bf16, also to
+    every unit on its own (units = "out" or "state", see UNIT_AXES), so that an
+    error confined to one (request, head) cannot hide in the batch's norm."""
     got = np.asarray(got, dtype=np.float64)
     want = np.asarray(want, dtype=np.float64)
     assert got.shape == want.shape, f"{what}: shapes {got.shape} vs {want.shape}"
@@ -37,9 +60,16 @@ def assert_parity(got, want, dtype, what=""):
     tol = TOL[dtype]
     r = rel_l2(got, want)
     assert r <= tol["rel"], f"{what}: rel-L2 {r:.3e} > {tol['rel']}"
+    worst = None
+    if units is not None and dtype == torch.bfloat16 and got.size:
+        per = unit_rel_l2(got, want, UNIT_AXES[units])
+        k = int(np.argmax(per))
+        worst = float(per[k])
+        assert worst <= tol["rel"], f"{what}: unit {k} rel-L2 {worst:.3e} > {tol['rel']}"
     if tol["abs"] is not None:
         m = float(np.max(np.abs(got - want))) if got.size else 0.0
         assert m <= tol["abs"], f"{what}: max-abs {m:.3e} > {tol['abs']}"
+    print(f"parity {what}: rel-L2 {r:.2e}" + (f", worst unit {worst:.2e}" if worst is not None else ""))
     return r
 
 

@@ -165,3 +165,31 @@ def test_train_argument_checks(L):
     assert fwd(c, wsb=nb - 1) == H.HYBRID_ERR_INVALID_ARG
     assert bwd(c, do=None) == H.HYBRID_ERR_INVALID_ARG
     assert bwd(c, dw=ok + 4) == H.HYBRID_ERR_INVALID_ARG
+
+
+def test_logical_entry_checks_size_and_pointers_before_the_device(L):
+    """hybrid_block_attn_commit_logical rejects a batch larger than its static
+    scratch, and null or misaligned pointers, on the host: no device is needed
+    and nothing is queued."""
+    c = cfg()
+    ok = 1 << 20
+    f = L.hybrid_block_attn_commit_logical
+    per_req = H.hybrid_state_bytes(c)
+    most = ((64 << 20) - 255) // (per_req + 8)
+    for n in (1 << 30, 2 ** 31 - 1, most + 1):
+        assert f(ctypes.byref(c), ok, ok, ok, ok, ok, ok, ok, n, ok, None) == H.HYBRID_ERR_UNSUPPORTED
+    assert f(ctypes.byref(c), ok, ok, ok, ok, ok, ok, ok, -1, ok, None) == H.HYBRID_ERR_INVALID_ARG
+    assert f(ctypes.byref(c), ok, ok, ok, ok, ok, None, ok, 1, ok, None) == H.HYBRID_ERR_INVALID_ARG
+    assert f(ctypes.byref(c), ok, ok, ok, ok, ok, ok, None, most, ok, None) == H.HYBRID_ERR_INVALID_ARG
+    assert f(ctypes.byref(c), None, ok, ok, ok, ok, ok, ok, 1, ok, None) == H.HYBRID_ERR_INVALID_ARG
+    assert f(ctypes.byref(c), ok + 8, ok, ok, ok, ok, ok, ok, 1, ok, None) == H.HYBRID_ERR_INVALID_ARG
+    assert f(ctypes.byref(c), ok, ok, ok, ok, ok + 2, ok, ok, 1, ok, None) == H.HYBRID_ERR_INVALID_ARG
+    assert f(ctypes.byref(c), ok, ok, ok, ok, ok, ok + 2, ok, 1, ok, None) == H.HYBRID_ERR_INVALID_ARG
+    assert f(ctypes.byref(cfg(d=96)), ok, ok, ok, ok, ok, ok, ok, 1, ok, None) == H.HYBRID_ERR_UNSUPPORTED
+
+
+def test_debug_arm_wait_timeout_host_checks(L):
+    """The failure-path test hook validates its limit on the host and can be disarmed."""
+    assert L.hybrid_debug_arm_wait_timeout(10_000_000_001) == H.HYBRID_ERR_INVALID_ARG
+    assert L.hybrid_debug_arm_wait_timeout(1_000_000) == H.HYBRID_OK
+    assert L.hybrid_debug_arm_wait_timeout(0) == H.HYBRID_OK

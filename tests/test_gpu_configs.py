@@ -56,12 +56,12 @@ def test_c2_full_step_plus_commit():
     pair = Pair(wl, tracked=[0, 3, 7])
     pair.build_prefixes(wk.prefix_lengths(wl))
     S, z = pair.gpu_state()
-    assert_parity(S, pair.S, wl.io_dtype, "c2 prefix state S")
+    assert_parity(S, pair.S, wl.io_dtype, "c2 prefix state S", units="state")
     got, want = _fused_call(pair, "c2_step")
-    assert_parity(got, want, wl.io_dtype, "c2 output")
+    assert_parity(got, want, wl.io_dtype, "c2 output", units="out")
     S, z = pair.gpu_state()
-    assert_parity(S, pair.S, wl.io_dtype, "c2 committed state S")
-    assert_parity(z, pair.z, wl.io_dtype, "c2 committed state z")
+    assert_parity(S, pair.S, wl.io_dtype, "c2 committed state S", units="state")
+    assert_parity(z, pair.z, wl.io_dtype, "c2 committed state z", units="state")
 
 
 def test_c3_full_bench_launch():
@@ -73,14 +73,14 @@ def test_c3_full_bench_launch():
     pair.build_prefixes(plen)
     for step in range(2):
         got, want = _fused_call(pair, ("c3_step", step))
-        assert_parity(got, want, wl.io_dtype, f"c3 output, step {step}")
+        assert_parity(got, want, wl.io_dtype, f"c3 output, step {step}", units="out")
         S, z = pair.gpu_state()
-        assert_parity(S, pair.S, wl.io_dtype, f"c3 committed state S, step {step}")
-        assert_parity(z, pair.z, wl.io_dtype, f"c3 committed state z, step {step}")
+        assert_parity(S, pair.S, wl.io_dtype, f"c3 committed state S, step {step}", units="state")
+        assert_parity(z, pair.z, wl.io_dtype, f"c3 committed state z, step {step}", units="state")
     # the attention-only step against the grown state as well
     Q, K, V = wk.block_qkv(wl, "c3_attn", pair.dev)
     got, want, _ = pair.step(Q, K, V)
-    assert_parity(got, want, wl.io_dtype, "c3 attention-only output")
+    assert_parity(got, want, wl.io_dtype, "c3 attention-only output", units="out")
 
 
 def test_c4_decode_loop_drift():
@@ -107,7 +107,7 @@ def test_c4_decode_loop_drift():
                     H.hybrid_check()
                     want = pair.orc.block_attn(h64(Q[t]), h64(K[t]), h64(V[t]), pair.W64, pair.alpha64,
                                                pair.S, pair.z)
-                    assert_parity(h64(O[t]), want, wl.io_dtype, f"c4 layer {L} block {blk} step {step}")
+                    assert_parity(h64(O[t]), want, wl.io_dtype, f"c4 layer {L} block {blk} step {step}", units="out")
                     checked += 1
                 if last:
                     pair.orc.commit(h64(K[t]), h64(V[t]), pair.W64, pair.S, pair.z)
@@ -115,8 +115,8 @@ def test_c4_decode_loop_drift():
     assert checked == 6 * wl.layers
     for L, pair in enumerate(pairs):
         S, z = pair.gpu_state()
-        assert_parity(S, pair.S, wl.io_dtype, f"c4 final state S, layer {L}")
-        assert_parity(z, pair.z, wl.io_dtype, f"c4 final state z, layer {L}")
+        assert_parity(S, pair.S, wl.io_dtype, f"c4 final state S, layer {L}", units="state")
+        assert_parity(z, pair.z, wl.io_dtype, f"c4 final state z, layer {L}", units="state")
 
 
 def test_c5_full_sampled():
@@ -132,18 +132,18 @@ def test_c5_full_sampled():
     assert len(pair.tracked) == 8
     pair.build_prefixes(plen)
     S, z = pair.gpu_state()
-    assert_parity(S, pair.S, wl.io_dtype, "c5 prefix state S")
-    assert_parity(z, pair.z, wl.io_dtype, "c5 prefix state z")
+    assert_parity(S, pair.S, wl.io_dtype, "c5 prefix state S", units="state")
+    assert_parity(z, pair.z, wl.io_dtype, "c5 prefix state z", units="state")
     Q, K, V = wk.block_qkv(wl, "c5_step", pair.dev)
     got, want, O = pair.step(Q, K, V)
-    assert_parity(got, want, wl.io_dtype, "c5 output")
+    assert_parity(got, want, wl.io_dtype, "c5 output", units="out")
     for r0 in range(0, wl.n_req, 32):
         reqs = np.arange(r0, min(r0 + 32, wl.n_req))
         Sg, zg = pair.gpu_state(reqs)
         t = torch.as_tensor(reqs, device=pair.dev)
         want = pair.orc.block_attn(h64(Q[t]), h64(K[t]), h64(V[t]), pair.W64, pair.alpha64, Sg, zg)
-        assert_parity(h64(O[t]), want, wl.io_dtype, f"c5 output, requests {r0}..{reqs[-1]}")
+        assert_parity(h64(O[t]), want, wl.io_dtype, f"c5 output, requests {r0}..{reqs[-1]}", units="out")
     pair.commit(K, V)
     S, z = pair.gpu_state()
-    assert_parity(S, pair.S, wl.io_dtype, "c5 committed state S")
-    assert_parity(z, pair.z, wl.io_dtype, "c5 committed state z")
+    assert_parity(S, pair.S, wl.io_dtype, "c5 committed state S", units="state")
+    assert_parity(z, pair.z, wl.io_dtype, "c5 committed state z", units="state")

@@ -69,20 +69,20 @@ def test_commit_then_step_parity(wl, plen):
     plen = _plen(wl, plen)
     pair.build_prefixes(plen)
     S, z = pair.gpu_state()
-    assert_parity(S, pair.S, wl.io_dtype, "prefix state S")
-    assert_parity(z, pair.z, wl.io_dtype, "prefix state z")
+    assert_parity(S, pair.S, wl.io_dtype, "prefix state S", units="state")
+    assert_parity(z, pair.z, wl.io_dtype, "prefix state z", units="state")
     Q, K, V = wk.block_qkv(wl, "step", pair.dev)
     got, want, _ = pair.step(Q, K, V)
-    assert_parity(got, want, wl.io_dtype, "block attention output")
+    assert_parity(got, want, wl.io_dtype, "block attention output", units="out")
     # fold the active block in (the final denoising step's K/V) and compare the state
     pair.commit(K, V)
     S, z = pair.gpu_state()
-    assert_parity(S, pair.S, wl.io_dtype, "post-commit state S")
-    assert_parity(z, pair.z, wl.io_dtype, "post-commit state z")
+    assert_parity(S, pair.S, wl.io_dtype, "post-commit state S", units="state")
+    assert_parity(z, pair.z, wl.io_dtype, "post-commit state z", units="state")
     # a second step against the grown state
     Q2, K2, V2 = wk.block_qkv(wl, "step2", pair.dev)
     got, want, _ = pair.step(Q2, K2, V2)
-    assert_parity(got, want, wl.io_dtype, "second step output")
+    assert_parity(got, want, wl.io_dtype, "second step output", units="out")
 
 
 @pytest.mark.parametrize("dt", [F32, BF16])
@@ -159,7 +159,7 @@ def test_gate_limits(wl):
     for a in (math.inf, -math.inf, 30.0, -30.0, 0.0):
         alpha = torch.full((wl.Hq,), a, dtype=torch.float32, device=pair.dev)
         got, want, _ = pair.step(Q, K, V, alpha)
-        assert_parity(got, want, wl.io_dtype, f"alpha={a}")
+        assert_parity(got, want, wl.io_dtype, f"alpha={a}", units="out")
 
 
 @pytest.mark.parametrize("wl", EDGE_WL, ids=[w.name for w in EDGE_WL])
@@ -167,7 +167,7 @@ def test_empty_prefix_is_block_softmax(wl):
     pair = Pair(wl)
     Q, K, V = wk.block_qkv(wl, "empty", pair.dev)
     got, want, O = pair.step(Q, K, V)
-    assert_parity(got, want, wl.io_dtype, "empty prefix")
+    assert_parity(got, want, wl.io_dtype, "empty prefix", units="out")
     G = wl.Hq // wl.Hkv
     q = Q.float().permute(0, 2, 1, 3)
     k = K.float().repeat_interleave(G, dim=2).permute(0, 2, 1, 3)
@@ -196,7 +196,7 @@ def test_tied_keys(wl):
     Q, K, V = wk.block_qkv(wl, "ties", pair.dev)
     K = K[:, :1].expand_as(K).contiguous()
     got, want, _ = pair.step(Q, K, V)
-    assert_parity(got, want, wl.io_dtype, "tied keys")
+    assert_parity(got, want, wl.io_dtype, "tied keys", units="out")
 
 
 def test_permuted_and_subset_pointer_arrays():
@@ -279,13 +279,13 @@ def test_f256_phi_minus_paths(scaled_heads):
     for g in range(wl.Hkv):
         assert (rng[g] > 64.0) if g in scaled_heads else (rng[g] < 32.0), (g, rng)
     got, want, _ = pair.step(Q, K, V)
-    assert_parity(got, want, wl.io_dtype, f"W x 20 on heads {scaled_heads}")
+    assert_parity(got, want, wl.io_dtype, f"W x 20 on heads {scaled_heads}", units="out")
     pair.commit(K, V)
     S, z = pair.gpu_state()
-    assert_parity(S, pair.S, wl.io_dtype, "state after the commit")
+    assert_parity(S, pair.S, wl.io_dtype, "state after the commit", units="state")
     Q2, K2, V2 = wk.block_qkv(wl, "phim2", pair.dev)
     got, want, _ = pair.step(Q2, K2, V2)
-    assert_parity(got, want, wl.io_dtype, "second step")
+    assert_parity(got, want, wl.io_dtype, "second step", units="out")
 
 
 BADPTR_WL = [W_("badptr_bf16", BF16, 3, 4, 4, 128, 128, 32, 44),
@@ -313,6 +313,32 @@ def test_bad_state_pointer_is_reported_not_faulted(wl):
     assert H.hybrid_check(check=False) == H.HYBRID_OK
 
 
+def test_bounded_wait_timeout_is_reported_not_hung():
+    """A bounded device wait that runs out comes back as HYBRID_ERR_TIMEOUT from
+    hybrid_check, with the context usable.  The hook arms one step launch with a
+    1 ms limit and makes its math warps withhold one arrival on a barrier that no
+    asynchronous copy targets; every role then leaves through the failure path.
+    Two units per CTA on some CTAs (160 units on at most 152 CTAs) and one on the
+    rest, so both a unit's own wait and the next unit's start meet the flag."""
+    wl = W_("timeout_c3_shape", BF16, 40, 16, 4, 128, 128, 32, 50)
+    pair = Pair(wl)
+    pair.build_prefixes(np.full(wl.n_req, 64))
+    Q, K, V = wk.block_qkv(wl, "timeout", pair.dev)
+    O = torch.zeros_like(Q)
+    H.hybrid_debug_arm_wait_timeout(1_000_000)
+    H.hybrid_block_attn(pair.cfg, Q, K, V, pair.W, pair.alpha, pair.ptrs, wl.n_req, O)
+    assert H.hybrid_check(check=False) == H.HYBRID_ERR_TIMEOUT
+    # the launch consumed the setting: the next one runs normally and is correct
+    got, want, _ = pair.step(Q, K, V)
+    assert H.hybrid_check(check=False) == H.HYBRID_OK
+    assert_parity(got, want, wl.io_dtype, "after a timed-out launch", units="out")
+    # disarming leaves later launches alone
+    H.hybrid_debug_arm_wait_timeout(1_000_000)
+    H.hybrid_debug_arm_wait_timeout(0)
+    got, want, _ = pair.step(Q, K, V)
+    assert_parity(got, want, wl.io_dtype, "after disarming", units="out")
+
+
 PREFILL = [
     # 6 units x 8 chunks: every unit's chunks are spread over 8 CTAs and combined
     # by the reduce-adds, on top of a prefix already in the state
@@ -336,8 +362,8 @@ def test_prefill_split_across_ctas(wl, T, prefix):
     K, V = wk.prefix_kv(wl, 1, pair.dev, n_tok=T)
     pair.commit(K, V)
     S, z = pair.gpu_state()
-    assert_parity(S, pair.S, BF16, f"prefill {T} S")
-    assert_parity(z, pair.z, BF16, f"prefill {T} z")
+    assert_parity(S, pair.S, BF16, f"prefill {T} S", units="state")
+    assert_parity(z, pair.z, BF16, f"prefill {T} z", units="state")
 
 
 RAGGED = [
@@ -380,8 +406,8 @@ def test_ragged_prefill(wl, lens, prefix):
         pair.build_prefixes(np.full(wl.n_req, prefix, dtype=np.int64))
     _ragged_commit(pair, lens, 71)
     S, z = pair.gpu_state()
-    assert_parity(S, pair.S, wl.io_dtype, "ragged prefill S")
-    assert_parity(z, pair.z, wl.io_dtype, "ragged prefill z")
+    assert_parity(S, pair.S, wl.io_dtype, "ragged prefill S", units="state")
+    assert_parity(z, pair.z, wl.io_dtype, "ragged prefill z", units="state")
 
 
 def test_ragged_prefill_more_requests_than_one_launch():
@@ -392,8 +418,8 @@ def test_ragged_prefill_more_requests_than_one_launch():
     lens = np.arange(wl.n_req) % 4
     _ragged_commit(pair, lens, 72)
     S, z = pair.gpu_state()
-    assert_parity(S, pair.S, wl.io_dtype, "ragged S")
-    assert_parity(z, pair.z, wl.io_dtype, "ragged z")
+    assert_parity(S, pair.S, wl.io_dtype, "ragged S", units="state")
+    assert_parity(z, pair.z, wl.io_dtype, "ragged z", units="state")
 
 
 def test_prefill_commit_long_ragged():
@@ -404,8 +430,8 @@ def test_prefill_commit_long_ragged():
     K, V = wk.prefix_kv(wl, 0, pair.dev, n_tok=161)
     pair.commit(K, V)
     S, z = pair.gpu_state()
-    assert_parity(S, pair.S, BF16, "prefill S")
-    assert_parity(z, pair.z, BF16, "prefill z")
+    assert_parity(S, pair.S, BF16, "prefill S", units="state")
+    assert_parity(z, pair.z, BF16, "prefill z", units="state")
 
 
 # ---------------------------------------------------------------------------
@@ -440,11 +466,11 @@ def test_fused_step_commit_parity(wl, plen):
         t = torch.as_tensor(pair.tracked, device=Q.device)
         want = pair.orc.block_attn(h64(Q[t]), h64(K[t]), h64(V[t]), pair.W64, pair.alpha64,
                                    pair.S, pair.z)
-        assert_parity(h64(O[t]), want, wl.io_dtype, f"fused output, step {step}")
+        assert_parity(h64(O[t]), want, wl.io_dtype, f"fused output, step {step}", units="out")
         pair.orc.commit(h64(K[t]), h64(V[t]), pair.W64, pair.S, pair.z)
         S, z = pair.gpu_state()
-        assert_parity(S, pair.S, wl.io_dtype, f"fused state S, step {step}")
-        assert_parity(z, pair.z, wl.io_dtype, f"fused state z, step {step}")
+        assert_parity(S, pair.S, wl.io_dtype, f"fused state S, step {step}", units="state")
+        assert_parity(z, pair.z, wl.io_dtype, f"fused state z, step {step}", units="state")
 
 
 def test_fused_matches_separate_calls():
