@@ -136,8 +136,8 @@ hybrid_status hybrid_block_attn(const hybrid_cfg *cfg, const void *Q, const void
         return HYBRID_ERR_INVALID_ARG;
     unsigned *err = error_word();
     if (!err) return HYBRID_ERR_CUDA;
-    if (hyb::fused_supported(*cfg, false))
-        return from_cuda(hyb::launch_fused(*cfg, false, Q, K, V, W, alpha, d_state_ptrs, n_req, O, err, stream));
+    if (hyb::step_supported(*cfg))
+        return from_cuda(hyb::launch_step(*cfg, Q, K, V, W, alpha, d_state_ptrs, n_req, O, err, stream));
     if (hyb::tc_attn_supported(*cfg))
         return from_cuda(hyb::launch_attn_tc(*cfg, Q, K, V, W, alpha, d_state_ptrs, n_req, O, err, stream));
     return from_cuda(hyb::launch_attn_generic(*cfg, Q, K, V, W, alpha, d_state_ptrs, n_req, O, err, stream));

@@ -148,12 +148,18 @@ FLayout make_flayout(int d, int F, int B, bool commit)
     return L;
 }
 
-__device__ __forceinline__ float *unit_state(const FusedArgs &a, int u)
+// Every role walks the same units and skips those whose state pointer fails its
+// check.  The pointer of the next unit is loaded one unit ahead (state_raw), so
+// its latency hides behind the current unit; state_at checks it when it is used.
+__device__ __forceinline__ void *state_raw(const FusedArgs &a, int u, int u_end)
 {
-    const int r = u / a.Hkv, g = u % a.Hkv;
-    float *st = reinterpret_cast<float *>(a.states[r]);
+    return u < u_end ? a.states[u / a.Hkv] : nullptr;
+}
+__device__ __forceinline__ float *state_at(const FusedArgs &a, void *raw, int u)
+{
+    float *st = reinterpret_cast<float *>(raw);
     if (!state_ptr_ok(st)) return nullptr;
-    return st + (size_t)g * head_floats(a.d, a.F);
+    return st + (size_t)(u % a.Hkv) * head_floats(a.d, a.F);
 }
 
 template <bool kCommit>
@@ -186,24 +192,30 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint64_t *dready = zempty + 2;    // [2] MMA -> math: the unit's output accumulator is complete
     uint64_t *dfree = dready + 2;     // [2] math -> MMA: the output accumulator has been read
     uint64_t *tready = dfree + 2;     // [2] math -> storer: a feature half of the tiles is updated
-    uint64_t *xfull = tready + 2;     // Q, W (TMA) and K^T (producer warp) are in place
-    uint64_t *xfree = xfull + 1;
+    // Barriers of one unit's stages.  The step issues the MMAs of even and odd units
+    // from two threads (one per Tensor Memory slot), so it keeps these per slot:
+    // entry k & 1 with parity (k >> 1) & 1 for the unit of index k; the commit uses
+    // entry 0 with parity k & 1 (see SB, SP).
+    uint64_t *xfull = tready + 2;     // [2] Q, W (TMA) and K^T (producer warp) are in place
+    uint64_t *uready = xfull + 2;     // [2] MMA -> math: g1 done
+    uint64_t *phip = uready + 2;      // [2] math -> MMA: phi+ is in the phi columns
+    uint64_t *phim = phip + 2;        // [2] math -> MMA: phi- in the phi columns
+    uint64_t *pread = phim + 2;       // [2] MMA -> math: R+ has consumed phi+
+    uint64_t *pready = pread + 2;     // [2] math -> MMA: P' is written
+    uint64_t *mmadone = pready + 2;   // [2] per issuing thread: all of its MMAs have completed
+    uint64_t *xfree = mmadone + 2;
     uint64_t *vfull = xfree + 1;
     uint64_t *vfree = vfull + 1;
-    uint64_t *uready = vfree + 1;     // MMA -> math: g1 done
-    uint64_t *phip = uready + 1;      // math -> MMA: phi+ is in the phi columns
-    uint64_t *phim = phip + 1;        // math -> MMA: phi- in the phi columns
-    uint64_t *pread = phim + 1;       // MMA -> math: R+ has consumed phi+
-    uint64_t *pready = pread + 1;     // math -> MMA: P' is written
-    uint64_t *kready = pready + 1;    // math -> MMA: phi(K) is written (commit)
+    uint64_t *kready = vfree + 1;     // math -> MMA: phi(K) is written (commit)
     uint64_t *dsdone = kready + 1;    // MMA -> math: dS^T is formed (commit)
     uint64_t *pvdone = dsdone + 1;    // MMA -> producer: P V has read V and P' (commit)
     uint64_t *efree = pvdone + 1;     // math -> MMA: the first-half update has read dS+ (commit)
     uint64_t *zdone = efree + 1;      // math -> storer: z is updated (commit)
     uint64_t *ofree = zdone + 1;      // storer -> math: the output slots may be written (commit)
     uint64_t *ostaged = ofree + 1;    // math -> storer: the output tile is in its slots
-    uint64_t *mmadone = ostaged + 1;
-    const int n_bars = 2 * NS + 10 + 17;
+    const int n_bars = 2 * NS + 10 + 14 + 10;
+    auto SB = [&](uint64_t *b, uint32_t k) -> uint64_t * { return kCommit ? b : b + (k & 1u); };
+    auto SP = [&](uint32_t k) -> uint32_t { return kCommit ? (k & 1u) : ((k >> 1) & 1u); };
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + n_bars);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
@@ -215,18 +227,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     if (warp == 3 && lane == 0) prefetch_tensormap(&a.tmO);
     if (tid == 0) {
         for (int i = 0; i < n_bars; ++i) mbar_init(&bars[i], 1);
-        mbar_init(xfull, 2);
-        mbar_init(phip, 8);
-        mbar_init(phim, 8);
-        mbar_init(pready, 8);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&xfull[i], 2);
+            mbar_init(&phip[i], 8);
+            mbar_init(&phim[i], 8);
+            mbar_init(&pready[i], 8);
+            mbar_init(&dfree[i], 8);
+            mbar_init(&tready[i], 8);
+        }
         mbar_init(kready, 8);
         mbar_init(efree, 8);
         mbar_init(zdone, 8);
         mbar_init(ostaged, 8);
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(&dfree[i], 8);
-            mbar_init(&tready[i], 8);
-        }
         if (!kCommit) {
             mbar_init(&zempty[0], 8);
             mbar_init(&zempty[1], 8);
@@ -258,16 +270,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             int issued_z[2] = {0, 0};
             for (int i = 0; i < kMaxSlots; ++i) issued_slot[i] = 0;
             bool ok = true;
+            void *nraw = state_raw(a, u_begin, u_end);
             for (int u = u_begin; u < u_end && ok; ++u) {
-                float *Sg = unit_state(a, u);
+                void *raw = nraw;
+                nraw = state_raw(a, u + 1, u_end);
+                float *Sg = state_at(a, raw, u);
                 if (!Sg) continue;
                 const int zb = kp & 1;
                 if (!wait_bar(&zempty[zb], ((kp >> 1) & 1u) ^ 1u, fail, wlim)) break;
                 mbar_arrive_expect_tx(&zfull[zb], 2 * F * 4);
                 bulk_g2s(zbuf0 + zb * zstride, Sg + (size_t)2 * F * d, 2 * F * 4, &zfull[zb]);
                 ++issued_z[zb];
-                // at start-up every SM asks for its first unit at once: let Q, W and K
-                // (needed first) arrive before the state tiles (needed after g1 and phi)
                 if (kp == 0 && !wait_bar(xfull, 0, fail, wlim)) break;
                 for (int c = 0; c < NC; ++c, ++q) {
                     const int slot = q % NS;
@@ -285,9 +298,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     if (issued_z[s]) mbar_wait(&zfull[s], (uint32_t)(issued_z[s] - 1) & 1u, kWaitNs);
             }
         }
-    } else if (warp == 1) {
-        // ------------------------------------------------------- MMA issuer
+    } else if (warp == 1 || (!kCommit && warp == 3)) {
+        // ------------------------------------------------------- MMA issuers
+        // commit: warp 1 issues every MMA.  Step: warp 1 issues the MMAs of the even
+        // units (Tensor Memory slot 0) and warp 3 those of the odd units (slot 1), so
+        // one unit's phi- readout runs beside the next unit's phi+ readout (an M = 128
+        // tf32 MMA keeps its issuing thread ~140 cycles, twice the tensor pipe's time).
         if (lane == 0) {
+            const uint32_t iss = warp == 1 ? 0u : 1u;
             const uint32_t q_u = smem_u32(smem + a.off_q), wk_u = smem_u32(smem + a.off_wk),
                            vb_u = smem_u32(smem + a.off_vb), p_u = smem_u32(smem + a.off_p),
                            pk_u = smem_u32(smem + a.off_pk), ring_u = smem_u32(ring);
@@ -338,61 +356,64 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     mma_bf16_ss(tmem + dcol, av, bp, idDS, ks > 0);
                 }
             };
-            uint32_t kp = 0, qt = 0, prev_qt = 0;
+            uint32_t kp = 0, qt = 0;
             bool ok = true;
             if (!kCommit) {
-                // R- of the previous unit: its phi- sits in the phi columns R+ has consumed
-                auto tail = [&](uint32_t ik, uint32_t iq) -> bool {
-                    const uint32_t T = (ik & 1) * 256;
-                    if (!wait_bar(phim, ik & 1u, fail, wlim)) return false;
-                    tc_fence_after();
-                    for (int c = NCH; c < NC; ++c) {
-                        const int slot = readout(T + 128, T + 32 * (c - NCH), iq + c);
-                        if (slot < 0) return false;
-                        mma_commit(&empty[slot]);
-                    }
-                    mma_commit(&dready[ik & 1]);
-                    return true;
-                };
-                // P'V and R- of the previous unit: its P' and phi- come last
-                auto finish = [&](uint32_t ik, uint32_t iq) -> bool {
-                    if (!wait_bar(pready, ik & 1u, fail, wlim) || !wait_bar(vfull, ik & 1u, fail, wlim)) return false;
-                    tc_fence_after();
-                    pv((ik & 1) * 256 + 128);
-                    mma_commit(vfree);
-                    return tail(ik, iq);
-                };
+                // this thread's units: g1, R+ once phi+ is written, P'V, R- once phi- is
+                // written, all into its slot's [phi | D] columns
+                const uint32_t T = iss * 256;
+                void *nraw = state_raw(a, u_begin, u_end);
                 for (int u = u_begin; u < u_end; ++u) {
-                    if (!unit_state(a, u)) continue;
-                    const uint32_t T = (kp & 1) * 256;
-                    if (!wait_bar(xfull, kp & 1u, fail, wlim)) { ok = false; break; }
-                    if (kp >= 2 && !wait_bar(&dfree[kp & 1], ((kp - 2) >> 1) & 1u, fail, wlim)) { ok = false; break; }
-                    tc_fence_after();
-                    g1(T, 0);
-                    mma_commit(uready);
-                    mma_commit(xfree);
-                    if (kp >= 1 && !finish(kp - 1, prev_qt)) { ok = false; break; }
-                    if (!wait_bar(phip, kp & 1u, fail, wlim)) { ok = false; break; }
-                    tc_fence_after();
-                    for (int c = 0; c < NCH; ++c) {
-                        const int slot = readout(T + 128, T + 32 * c, qt + c, c == 0);
-                        if (slot < 0) { ok = false; break; }
-                        mma_commit(&empty[slot]);
+                    void *raw = nraw;
+                    nraw = state_raw(a, u + 1, u_end);
+                    if (!state_at(a, raw, u)) continue;
+                    if ((kp & 1u) == iss) {
+                        if (!wait_bar(SB(xfull, kp), SP(kp), fail, wlim)) { ok = false; break; }
+                        if (kp >= 2 && !wait_bar(&dfree[iss], ((kp - 2) >> 1) & 1u, fail, wlim)) { ok = false; break; }
+                        tc_fence_after();
+                        g1(T, 0);
+                        mma_commit(SB(uready, kp));
+                        mma_commit(xfree);
+                        if (!wait_bar(SB(phip, kp), SP(kp), fail, wlim)) { ok = false; break; }
+                        tc_fence_after();
+                        for (int c = 0; c < NCH && ok; ++c) {
+                            const int slot = readout(T + 128, T + 32 * c, qt + c, c == 0);
+                            if (slot < 0) ok = false;
+                            else mma_commit(&empty[slot]);
+                        }
+                        if (!ok) break;
+                        mma_commit(SB(pread, kp));
+                        // P'V: V and P' are single buffers, released in unit order
+                        if (!wait_bar(SB(pready, kp), SP(kp), fail, wlim) || !wait_bar(vfull, kp & 1u, fail, wlim)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        pv(T + 128);
+                        mma_commit(vfree);
+                        if (!wait_bar(SB(phim, kp), SP(kp), fail, wlim)) { ok = false; break; }
+                        tc_fence_after();
+                        for (int c = NCH; c < NC && ok; ++c) {
+                            const int slot = readout(T + 128, T + 32 * (c - NCH), qt + c);
+                            if (slot < 0) ok = false;
+                            else mma_commit(&empty[slot]);
+                        }
+                        if (!ok) break;
+                        mma_commit(&dready[iss]);
                     }
-                    if (!ok) break;
-                    mma_commit(pread);
-                    prev_qt = qt;
                     qt += NC;
                     ++kp;
                 }
-                if (ok && kp >= 1) finish(kp - 1, prev_qt);
             } else {
                 // Tensor Memory: [0,128) D, [128,128+F) phi (U, then phi+, then phi-),
                 // scores after U, [256,256+F) dS+ (U_k^T at 288 until then),
                 // [384,384+F) dS-.  dS^T follows R+, so the first half's tiles are
                 // free for their increments as soon as dS^T is in Tensor Memory.
+                void *nraw = state_raw(a, u_begin, u_end);
                 for (int u = u_begin; u < u_end; ++u) {
-                    if (!unit_state(a, u)) continue;
+                    void *raw = nraw;
+                    nraw = state_raw(a, u + 1, u_end);
+                    if (!state_at(a, raw, u)) continue;
                     if (!wait_bar(xfull, kp & 1u, fail, wlim)) { ok = false; break; }
                     // U_k^T and the scores land in the dS+ columns: the previous unit's
                     // first-half update must have read them (its R- precedes in issue order)
@@ -425,8 +446,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     ++kp;
                 }
             }
-            mma_commit(mmadone);
-            mbar_wait(mmadone, 0, kWaitNs);
+            mma_commit(&mmadone[iss]);
+            mbar_wait(&mmadone[iss], 0, kWaitNs);
         }
     } else if (warp == 2) {
         // ------------------------------------------------------------- producer
@@ -434,8 +455,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         int nx = 0, nv = 0;
         const uint32_t xbytes = (uint32_t)(d / 64) * (G * B * 128) + (uint32_t)(F / 64) * (d * 128);
         uint8_t *kt = smem + a.off_wk + (F / 64) * d * 128;
+        void *nraw = state_raw(a, u_begin, u_end);
         for (int u = u_begin; u < u_end; ++u) {
-            if (!unit_state(a, u)) continue;
+            void *raw = nraw;
+            nraw = state_raw(a, u + 1, u_end);
+            if (!state_at(a, raw, u)) continue;
             const int r = u / a.Hkv, g = u % a.Hkv;
             KtRegs kr;
             kt_load(a.K, (size_t)r * B, B, a.Hkv, g, d, kr, lane);   // in flight while the region drains
@@ -445,14 +469,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             // with the commit the Q region holds the previous unit's V, P' and phi(K)
             // until its dS^T and P V have run (Q then follows K^T, which measured
             // faster at start-up too); otherwise Q goes with W, before K^T
-            const bool q_early = !kCommit;
+            const bool q_early = !kCommit || kp == 0;
+            uint64_t *xf = SB(xfull, kp);
             if (lane == 0) {
-                mbar_arrive_expect_tx(xfull, xbytes);
+                mbar_arrive_expect_tx(xf, xbytes);
                 if (q_early)
                     for (int e = 0; e < d / 64; ++e)
-                        tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xfull);
+                        tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xf);
                 for (int f = 0; f < F / 64; ++f)
-                    tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xfull);
+                    tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xf);
             }
             kt_store(kr, d, kt, lane);
             fence_proxy_async_smem();
@@ -462,8 +487,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             if (lane == 0) {
                 if (!q_early)
                     for (int e = 0; e < d / 64; ++e)
-                        tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xfull);
-                mbar_arrive(xfull);
+                        tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xf);
+                mbar_arrive(xf);
             }
             ++nx;
             // V: after the previous unit's P V (step), after this unit's g1 has read
@@ -480,7 +505,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         }
         if (lane == 0 && *fail) {
             // let copies in flight land before the CTA exits
-            if (nx) mbar_wait(xfull, (uint32_t)(nx - 1) & 1u, kWaitNs);
+            // the last loads of each xfull entry (one entry with the commit, two in the step)
+            for (int k = nx - 1; k >= 0 && k >= nx - (kCommit ? 1 : 2); --k)
+                mbar_wait(SB(xfull, (uint32_t)k), SP((uint32_t)k), kWaitNs);
             if (nv) mbar_wait(vfull, (uint32_t)(nv - 1) & 1u, kWaitNs);
         }
     } else if (warp == 3) {
@@ -488,8 +515,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         // (commit only: the step's math warps store the output themselves)
         if (kCommit && lane == 0) {
             uint32_t q = 0, kp = 0;
+            void *nraw = state_raw(a, u_begin, u_end);
             for (int u = u_begin; u < u_end; ++u) {
-                float *Sg = unit_state(a, u);
+                void *raw = nraw;
+                nraw = state_raw(a, u + 1, u_end);
+                float *Sg = state_at(a, raw, u);
                 if (!Sg) continue;
                 const int r = u / a.Hkv, g = u % a.Hkv;
                 bool ok = true;
@@ -633,16 +663,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         float prev_inv = 0.f;   // 1 / den of the unit whose output is still pending (step)
         int prev_u = 0;         // and that unit
         bool ok = true;
+        void *nraw = state_raw(a, u_begin, u_end);
+        float nalpha = valid && u_begin < u_end ? a.alpha[(u_begin % a.Hkv) * G + row % G] : 0.f;
         for (int u = u_begin; u < u_end; ++u) {
-            float *Sg = unit_state(a, u);
+            void *raw = nraw;
+            nraw = state_raw(a, u + 1, u_end);
+            // gate of this row's query head, loaded one unit ahead
+            const float alpha_row = nalpha;
+            nalpha = valid && u + 1 < u_end ? a.alpha[((u + 1) % a.Hkv) * G + row % G] : 0.f;
+            float *Sg = state_at(a, raw, u);
             if (!Sg) {
                 if (mt == 0) raise_error(a.err, ERR_BAD_STATE_PTR);
                 continue;
             }
-            const int g = u % a.Hkv;
             const int zb = kp & 1;
-            // gate of this row's query head, loaded now so the latency overlaps the first phase
-            const float alpha_row = valid ? a.alpha[g * G + row % G] : 0.f;
             float *zs = zbuf0 + zb * zstride;
             const uint32_t T = (kp & 1) * 256;
             const uint32_t pcol = tmem + (kCommit ? kCmP : T) + lane_off;       // U, phi+, phi-
@@ -655,7 +689,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
 
             // ---- phase A: row extrema of U and of the scores (U kept in registers);
             // commit: per-token extrema of U_k^T over this warp's 32 features
-            bool bad = !wait_bar(uready, kp & 1u, fail, wlim);
+            bool bad = !wait_bar(SB(uready, kp), SP(kp), fail, wlim);
             tc_fence_after();
             float sc[16], u0[32], u1[32];
             if (kCommit) {
@@ -761,7 +795,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0 && !a.withhold) mbar_arrive(phip);
+                if (lane == 0 && !a.withhold) mbar_arrive(SB(phip, kp));
             }
 
             // ---- phase B2: phi- (kept in registers until R+ has consumed phi+), the
@@ -913,7 +947,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     tmem_wait_st();
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0 && !a.withhold) mbar_arrive(phip);
+                    if (lane == 0 && !a.withhold) mbar_arrive(SB(phip, kp));
                 }
                 // step: the previous unit's P'V (issued after this unit's g1) has read P'
                 if (!kCommit && kp >= 1) bad = !wait_bar(vfree, (kp - 1) & 1u, fail, wlim) || bad;
@@ -932,7 +966,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             }
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(pready);
+            if (lane == 0) mbar_arrive(SB(pready, kp));
 
             // previous unit's output, while R+ of this one runs (step)
             if (!kCommit && kp >= 1) bad = !epilogue(kp - 1, prev_q, prev_inv, prev_u);
@@ -950,7 +984,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     tmem_st32(pcol + 32 * k, x);
                 }
             } else {
-                bad = !wait_bar(pread, kp & 1u, fail, wlim) || bad;
+                bad = !wait_bar(SB(pread, kp), SP(kp), fail, wlim) || bad;
                 tc_fence_after();
 #pragma unroll
                 for (int i = 0; i < 32; ++i) u0[i] *= cneg;
@@ -964,7 +998,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             tmem_wait_st();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0 && !bad) mbar_arrive(phim);
+            if (lane == 0 && !bad) mbar_arrive(SB(phim, kp));
 
             if (kCommit) {
                 // ---- state update: S^T += dS^T for a feature half as soon as the readout
@@ -1046,6 +1080,8 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
                          const void *W, const float *alpha, void *const *states, int n_req, void *O,
                          unsigned *err, cudaStream_t st)
 {
+    // the step alone runs in hybrid_step.cu
+    if (!commit) return cudaErrorNotSupported;
     const FLayout L = make_flayout(c.head_dim, c.feat_dim, c.block_size, commit);
     FusedArgs a;
     {
@@ -1097,15 +1133,14 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
     const int grid = a.n_units < sm_count() ? a.n_units : sm_count();
     // opt in to the full shared memory once per device and kernel (the attribute
     // is set to the maximum, so every layout fits)
-    static std::atomic<unsigned long long> opted[2];
+    static std::atomic<unsigned long long> opted{0};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     const unsigned long long bit = 1ull << dev;
-    if (!(opted[commit].load(std::memory_order_acquire) & bit)) {
-        const cudaError_t e = commit ? cudaFuncSetAttribute(k_fused<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit)
-                                     : cudaFuncSetAttribute(k_fused<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
+    if (!(opted.load(std::memory_order_acquire) & bit)) {
+        const cudaError_t e = cudaFuncSetAttribute(k_fused<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
         if (e != cudaSuccess) return e;
-        opted[commit].fetch_or(bit, std::memory_order_release);
+        opted.fetch_or(bit, std::memory_order_release);
     }
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(grid);
@@ -1117,7 +1152,7 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = attr;
     lc.numAttrs = 1;
-    return commit ? cudaLaunchKernelEx(&lc, k_fused<true>, a) : cudaLaunchKernelEx(&lc, k_fused<false>, a);
+    return cudaLaunchKernelEx(&lc, k_fused<true>, a);
 }
 
 }  // namespace hyb

@@ -1,0 +1,733 @@
+// hybrid_step.cu -- the block-hybrid step of Section 3.1 (in-block softmax,
+// linear readout from the committed state, gated shared-normaliser merge) on the
+// tcgen05 tensor cores: one persistent CTA per SM walks a contiguous range of
+// work units, one unit at a time, with both feature halves of the readout on
+// the tensor cores at once.
+//
+// Work unit = (request r, state head g): the G*B query rows of the unit share one
+// state.  Warp roles (12 warps):
+//   warp 0     state producer: z and the 2F/32 state tiles of each unit, by 1-D
+//              bulk copies into an NS-slot ring, phi+ and phi- tiles interleaved
+//              (the state layout is the MMA operand image, see hybrid.h)
+//   warp 1     MMA issuer A; owns the Tensor Memory allocation:
+//              g1 = [U | scores] = Q [W | K^T], the phi+ readout, P'V
+//   warp 2     producer: TMA of Q and W, K^T (transposed by the warp), V by TMA
+//   warp 3     MMA issuer B: the phi- readout
+//   warps 4-11 math: two threads per query row (one per TMEM lane and "part";
+//              a part owns every other 32-feature chunk of each half of phi)
+//
+// Tensor Memory (512 columns):
+//   [0, F)          U, then phi+ = e^(u - max u), written in place
+//   [F, F + B)      scores (read before phi- lands there)
+//   [F, 2F)         phi- = e^(min u - u)
+//   [2F, 2F + d)    D+ = phi+ S+ (+ P'V)
+//   [2F + d, 2F+2d) D- = phi- S-
+// A tcgen05.mma with M = 128 keeps its issuing thread ~140 cycles whatever N is,
+// twice the time the tensor pipe needs for a tf32 product with N = 128, so the
+// two halves of the readout go out from two threads into two accumulators.
+// Per unit: g1; the math warps take the row extrema, write phi+ and then phi-
+// (released to issuers A and B as each lands), take the exponential sums and
+// P'; the epilogue combines out = a+ D+ + a- D- from registers.  The next
+// unit's g1 follows as soon as its phi- readout has read the phi- columns, so
+// its feature map runs while this unit's epilogue drains.
+//
+// Merge (Section 3.1, out = (w sm_num + lin_num) / (w sm_den + lin_den)): phi+
+// and phi- stay unnormalised, P' = w sp e^s rides in D+, so
+//   out = (D+ / sp + D- / sn) e^-sigma / den_sigma,
+// den_sigma = e^(log lin_den - sigma) + e^(log(w sm_den) - sigma) in [1, 2],
+// sigma the log of the larger branch mass.  This needs w sp e^(s) (sp <= F) in
+// float range; a warp with a row whose bound w F e^(max s) passes e^60 scales
+// phi+ and phi- by e^-sigma / sp and e^-sigma / sn in Tensor Memory before it
+// releases them, and uses P' = w e^(s - sigma).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <atomic>
+
+#include "hybrid_common.cuh"
+#include "hybrid_tc.h"
+#include "tc_pipeline.cuh"
+
+namespace hyb {
+
+namespace {
+
+using namespace pipe;
+
+constexpr int kWarps = 12;
+constexpr int kThreads = kWarps * 32;
+constexpr int kMaxSlots = 16;
+constexpr int kSmemLimit = 232448;
+constexpr int kOneCtaPerSm = 118 * 1024;
+constexpr uint32_t kBarPair = 2;      // 2..5: the two math warps of one TMEM lane quarter
+constexpr uint32_t kStatBytes = 8 * 1024;
+
+struct StepArgs {
+    CUtensorMap tmQ, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
+    const bf16 *K;
+    bf16 *O;
+    const float *alpha;
+    void *const *states;
+    unsigned *err;
+    int n_units, B, Hq, Hkv, G, d, F, NS;
+    float scale;
+    unsigned long long wait_ns;       // limit of every bounded wait (1 s unless a test armed less)
+    int withhold;                     // test hook: the math warps never release phi+
+    uint32_t off_q, off_wk, off_vb, off_p, off_z, off_st, off_bar;
+};
+
+// Shared memory: [ring NS x d*128][Q][W | K^T][X][z x2][stats][barriers], where X
+// holds V and P' until the unit's P'V has read them and then the output tile,
+// staged as the image of d/64 TMA boxes of 64 columns x G*B rows (row t*G + h,
+// 128-byte swizzle) that the producer warp stores.
+// Q, V and W land by TMA with the 128-byte swizzle: Q as d/64 atoms of 128 rows
+// (16 KB apart; rows t*G + h), V as d/64 atoms of B rows (MN-major operand), W as
+// F/64 atoms of d rows (MN-major) followed by the K^T atom (row e holds
+// K[0..B)[e]), so that [W | K^T] is one MN-major B operand.  The ring has an even
+// number of slots, so a slot always holds tiles of the same half and is read by
+// the same issuer, in order.
+struct SLayout {
+    uint32_t off_q, off_wk, off_vb, off_p, off_z, off_st, off_bar, bytes;
+    int NS;
+};
+
+SLayout make_slayout(int d, int F, int B, int G)
+{
+    SLayout L{};
+    const uint32_t chunk = (uint32_t)d * 128;
+    const uint32_t zb = (((uint32_t)2 * F * 4) + 1023) & ~1023u;
+    const uint32_t q = (uint32_t)d * 256;
+    const uint32_t wk = (uint32_t)(F / 64 + 1) * d * 128;
+    const uint32_t vb = (((uint32_t)B * d * 2) + 1023) & ~1023u;
+    const uint32_t p = (((uint32_t)128 * B * 2) + 1023) & ~1023u;
+    const uint32_t oimg = (uint32_t)(d / 64) * G * B * 128;
+    const uint32_t x = ((vb + p > oimg ? vb + p : oimg) + 1023) & ~1023u;
+    const uint32_t bar = 1024;
+    const uint32_t fixed = q + wk + x + 2 * zb + kStatBytes + bar + 1024;
+    int ns = ((int)kSmemLimit - (int)fixed) / (int)chunk;
+    if (ns > kMaxSlots) ns = kMaxSlots;
+    ns &= ~1;
+    L.NS = ns;
+    uint32_t off = (uint32_t)(ns > 0 ? ns : 0) * chunk;
+    L.off_q = off; off += q;
+    L.off_wk = off; off += wk;
+    L.off_vb = off;
+    L.off_p = off + vb;
+    off += x;
+    L.off_z = off; off += 2 * zb;
+    L.off_st = off; off += kStatBytes;
+    L.off_bar = off; off += bar;
+    L.bytes = off + 1024;
+    if ((int)L.bytes < kOneCtaPerSm) L.bytes = kOneCtaPerSm;
+    return L;
+}
+
+// Every role walks the same units and skips those whose state pointer fails its
+// check.  The pointer of the next unit is loaded one unit ahead (state_raw), so
+// its latency hides behind the current unit; state_at checks it when it is used.
+__device__ __forceinline__ void *state_raw(const StepArgs &a, int u, int u_end)
+{
+    return u < u_end ? a.states[u / a.Hkv] : nullptr;
+}
+__device__ __forceinline__ float *state_at(const StepArgs &a, void *raw, int u)
+{
+    float *st = reinterpret_cast<float *>(raw);
+    if (!state_ptr_ok(st)) return nullptr;
+    return st + (size_t)(u % a.Hkv) * head_floats(a.d, a.F);
+}
+
+// ring position p of a unit (0 .. 2F/32 - 1) -> state tile: phi+ and phi- tiles
+// alternate, so issuer A reads the even positions and issuer B the odd ones
+__device__ __forceinline__ int tile_of_pos(int p, int NCH) { return (p & 1) ? NCH + (p >> 1) : (p >> 1); }
+
+__global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ StepArgs a)
+{
+    using namespace ptx;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int d = a.d, F = a.F, B = a.B, G = a.G, NS = a.NS;
+    const uint64_t wlim = a.wait_ns;
+    const int NCH = F / 32;          // 32-feature chunks (state tiles) per half of phi
+    const int NC = 2 * NCH;          // state tiles per unit
+    const uint32_t chunk_bytes = (uint32_t)d * 128;
+    const int per = a.n_units / (int)gridDim.x, rem = a.n_units % (int)gridDim.x;
+    const int u_begin = (int)blockIdx.x * per + min((int)blockIdx.x, rem);
+    const int u_end = u_begin + per + ((int)blockIdx.x < rem ? 1 : 0);
+    // Tensor Memory columns
+    const uint32_t cU = 0, cM = (uint32_t)F, cDp = 2u * F, cDm = 2u * F + d;
+
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + a.off_bar);
+    uint64_t *full = bars;            // [NS] a state tile has landed in the slot
+    uint64_t *empty = full + NS;      // [NS] the slot's tile has been read by its MMAs
+    uint64_t *zfull = empty + NS;     // [2]
+    uint64_t *zempty = zfull + 2;     // [2]
+    uint64_t *mmadone = zempty + 2;   // [2] per issuer: all of its MMAs have completed
+    uint64_t *xfull = mmadone + 2;    // Q, W (TMA) and K^T (producer warp) are in place
+    uint64_t *xfree = xfull + 1;      // g1 has read Q, W, K^T
+    uint64_t *vfull = xfree + 1;
+    uint64_t *uready = vfull + 1;     // A -> math: g1 done
+    uint64_t *phip = uready + 1;      // math -> A: phi+ is written
+    uint64_t *phim = phip + 1;        // math -> B: phi- is written
+    uint64_t *pready = phim + 1;      // math -> A: P' is written
+    uint64_t *dpdone = pready + 1;    // A -> math: D+ (phi+ readout and P'V) is complete
+    uint64_t *dmdone = dpdone + 1;    // B -> math, A: D- is complete (phi- has been read)
+    uint64_t *dfree = dmdone + 1;     // math -> A, B: the epilogue has read D+ and D-
+    uint64_t *ostaged = dfree + 1;    // math -> producer: the output tile is staged in X
+    uint64_t *ofree = ostaged + 1;    // producer -> math: the output stores have read X
+    const int n_bars = 2 * NS + 6 + 12;
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + n_bars);
+    volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
+
+    if (warp == 2 && lane == 0) {
+        prefetch_tensormap(&a.tmQ);
+        prefetch_tensormap(&a.tmW);
+        prefetch_tensormap(&a.tmV);
+        prefetch_tensormap(&a.tmO);
+    }
+    if (tid == 0) {
+        for (int i = 0; i < n_bars; ++i) mbar_init(&bars[i], 1);
+        mbar_init(xfull, 2);
+        mbar_init(phip, 8);
+        mbar_init(phim, 8);
+        mbar_init(pready, 8);
+        mbar_init(dfree, 8);
+        mbar_init(ostaged, 8);
+        mbar_init(&zempty[0], 8);
+        mbar_init(&zempty[1], 8);
+        *fail = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_holder, 512);
+        tmem_relinquish();
+    }
+    __syncthreads();
+    tc_fence_after();
+    // launched with programmatic stream serialisation: the set-up above may run
+    // while the previous kernel of the stream drains; nothing below touches
+    // global memory before that kernel has completed
+    if (tid == 0) griddep_launch_dependents();
+    griddep_wait();
+    const uint32_t tmem = *tmem_holder;
+    uint8_t *ring = smem;
+    float *zbuf0 = reinterpret_cast<float *>(smem + a.off_z);
+    const int zstride = ((2 * F * 4 + 1023) & ~1023) / 4;
+
+    if (warp == 0) {
+        // ------------------------------------------------------- state producer
+        if (lane == 0) {
+            uint32_t q = 0, kp = 0;
+            int issued_slot[kMaxSlots];
+            int issued_z[2] = {0, 0};
+            for (int i = 0; i < kMaxSlots; ++i) issued_slot[i] = 0;
+            bool ok = true;
+            void *nraw = state_raw(a, u_begin, u_end);
+            for (int u = u_begin; u < u_end && ok; ++u) {
+                void *raw = nraw;
+                nraw = state_raw(a, u + 1, u_end);
+                float *Sg = state_at(a, raw, u);
+                if (!Sg) continue;
+                const int zb = kp & 1;
+                if (!wait_bar(&zempty[zb], ((kp >> 1) & 1u) ^ 1u, fail, wlim)) break;
+                mbar_arrive_expect_tx(&zfull[zb], 2 * F * 4);
+                bulk_g2s(zbuf0 + zb * zstride, Sg + (size_t)2 * F * d, 2 * F * 4, &zfull[zb]);
+                ++issued_z[zb];
+                for (int p = 0; p < NC; ++p, ++q) {
+                    const int slot = q % NS;
+                    if (!wait_bar(&empty[slot], ((q / NS) & 1u) ^ 1u, fail, wlim)) break;
+                    mbar_arrive_expect_tx(&full[slot], chunk_bytes);
+                    bulk_g2s(ring + (size_t)slot * chunk_bytes, Sg + (size_t)tile_of_pos(p, NCH) * 32 * d,
+                             chunk_bytes, &full[slot]);
+                    ++issued_slot[slot];
+                }
+                ++kp;
+            }
+            if (*fail) {
+                for (int s = 0; s < NS; ++s)
+                    if (issued_slot[s]) mbar_wait(&full[s], (uint32_t)(issued_slot[s] - 1) & 1u, kWaitNs);
+                for (int s = 0; s < 2; ++s)
+                    if (issued_z[s]) mbar_wait(&zfull[s], (uint32_t)(issued_z[s] - 1) & 1u, kWaitNs);
+            }
+        }
+    } else if (warp == 1 || warp == 3) {
+        // ------------------------------------------------------------- MMA issuers
+        if (lane == 0) {
+            const uint32_t iss = warp == 1 ? 0u : 1u;
+            const uint32_t ring_u = smem_u32(ring);
+            const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
+            // tiles of this issuer: ring positions iss, iss + 2, ... of each unit, into D+ or D-
+            const uint32_t acol0 = iss ? cM : cU, dcol = iss ? cDm : cDp;
+            auto readout_half = [&](uint32_t qt) -> bool {
+                for (int c = 0; c < NCH; ++c) {
+                    const uint32_t qc = qt + 2 * c + iss;
+                    const int slot = (int)(qc % (uint32_t)NS);
+                    if (!wait_bar(&full[slot], (qc / NS) & 1u, fail, wlim)) return false;
+                    tc_fence_after();
+                    const uint64_t b0 = smem_desc(ring_u + (uint32_t)slot * chunk_bytes, 16, 1024, SWZ_128B);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        mma_tf32_ts(tmem + dcol, tmem + acol0 + 32 * c + 8 * kk, b0 + 2 * kk, idR, (c | kk) != 0);
+                    mma_commit(&empty[slot]);
+                }
+                return true;
+            };
+            uint32_t kp = 0, qt = 0;
+            if (iss == 0) {
+                const uint32_t q_u = smem_u32(smem + a.off_q), wk_u = smem_u32(smem + a.off_wk),
+                               vb_u = smem_u32(smem + a.off_vb), p_u = smem_u32(smem + a.off_p);
+                const uint32_t idUS = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F + B);
+                const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
+                void *nraw = state_raw(a, u_begin, u_end);
+                for (int u = u_begin; u < u_end; ++u) {
+                    void *raw = nraw;
+                    nraw = state_raw(a, u + 1, u_end);
+                    if (!state_at(a, raw, u)) continue;
+                    if (!wait_bar(xfull, kp & 1u, fail, wlim)) break;
+                    // g1 writes [U | scores] over the previous unit's phi+ (read by this
+                    // thread's own earlier MMAs, in issue order) and phi- (read by issuer B)
+                    if (kp >= 1 && !wait_bar(dmdone, (kp - 1) & 1u, fail, wlim)) break;
+                    tc_fence_after();
+                    for (int k = 0; k < d / 16; ++k) {
+                        const uint64_t aq = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
+                        const uint64_t bwk = smem_desc(wk_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
+                        mma_bf16_ss(tmem + cU, aq, bwk, idUS, k > 0);
+                    }
+                    mma_commit(uready);
+                    mma_commit(xfree);
+                    if (!wait_bar(phip, kp & 1u, fail, wlim)) break;
+                    // D+ is written from the first phi+ MMA on: the previous epilogue has read it
+                    if (kp >= 1 && !wait_bar(dfree, (kp - 1) & 1u, fail, wlim)) break;
+                    if (!readout_half(qt)) break;
+                    if (!wait_bar(pready, kp & 1u, fail, wlim) || !wait_bar(vfull, kp & 1u, fail, wlim)) break;
+                    tc_fence_after();
+                    for (int k = 0; k < B / 16; ++k) {
+                        const uint64_t ap = smem_desc(p_u + k * 256, 128, (B / 8) * 128, SWZ_NONE);
+                        const uint64_t bv = smem_desc(vb_u + 2 * k * 1024, B * 128, 1024, SWZ_128B);
+                        mma_bf16_ss(tmem + cDp, ap, bv, idP, 1);
+                    }
+                    mma_commit(dpdone);
+                    qt += NC;
+                    ++kp;
+                }
+            } else {
+                void *nraw = state_raw(a, u_begin, u_end);
+                for (int u = u_begin; u < u_end; ++u) {
+                    void *raw = nraw;
+                    nraw = state_raw(a, u + 1, u_end);
+                    if (!state_at(a, raw, u)) continue;
+                    if (!wait_bar(phim, kp & 1u, fail, wlim)) break;
+                    if (kp >= 1 && !wait_bar(dfree, (kp - 1) & 1u, fail, wlim)) break;
+                    if (!readout_half(qt)) break;
+                    mma_commit(dmdone);
+                    qt += NC;
+                    ++kp;
+                }
+            }
+            mma_commit(&mmadone[iss]);
+            mbar_wait(&mmadone[iss], 0, kWaitNs);
+        }
+    } else if (warp == 2) {
+        // ------------------------------------------------------------- producer
+        uint32_t kp = 0;
+        int nx = 0, nv = 0;
+        const uint32_t xbytes = (uint32_t)(d / 64) * (G * B * 128) + (uint32_t)(F / 64) * (d * 128);
+        uint8_t *kt = smem + a.off_wk + (F / 64) * d * 128;
+        int pr = 0, pg = 0;             // request and head of the previous unit
+        void *nraw = state_raw(a, u_begin, u_end);
+        for (int u = u_begin; u < u_end; ++u) {
+            void *raw = nraw;
+            nraw = state_raw(a, u + 1, u_end);
+            if (!state_at(a, raw, u)) continue;
+            const int r = u / a.Hkv, g = u % a.Hkv;
+            KtRegs kr;
+            kt_load(a.K, (size_t)r * B, B, a.Hkv, g, d, kr, lane);   // in flight while the region drains
+            bool ok = true;
+            if (kp > 0) ok = wait_bar(xfree, (kp - 1) & 1u, fail, wlim);
+            if (__any_sync(0xffffffffu, !ok)) break;
+            if (lane == 0) {
+                mbar_arrive_expect_tx(xfull, xbytes);
+                for (int e = 0; e < d / 64; ++e)
+                    tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xfull);
+                for (int f = 0; f < F / 64; ++f)
+                    tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xfull);
+            }
+            kt_store(kr, d, kt, lane);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(xfull);
+            ++nx;
+            // the previous unit's output tile (staged in X over its V and P') goes out
+            // by TMA stores; once they have read X, this unit's V may land there
+            if (kp > 0) {
+                ok = wait_bar(ostaged, (kp - 1) & 1u, fail, wlim);
+                if (__any_sync(0xffffffffu, !ok)) break;
+                if (lane == 0) {
+                    for (int j = 0; j < d / 64; ++j)
+                        tma_store_3d(&a.tmO, 64 * j, pg * G, pr * B, smem + a.off_vb + j * (G * B * 128));
+                    bulk_commit();
+                    bulk_wait_read_all();
+                    mbar_arrive(ofree);
+                }
+                __syncwarp();
+            }
+            if (lane == 0) {
+                mbar_arrive_expect_tx(vfull, (uint32_t)(d / 64) * (B * 128));
+                for (int e = 0; e < d / 64; ++e)
+                    tma_load_3d(smem + a.off_vb + e * (B * 128), &a.tmV, 64 * e, g, r * B, vfull);
+            }
+            ++nv;
+            ++kp;
+            pr = r;
+            pg = g;
+        }
+        // the last unit's output tile
+        if (kp > 0 && !*fail && wait_bar(ostaged, (kp - 1) & 1u, fail, wlim) && lane == 0) {
+            for (int j = 0; j < d / 64; ++j)
+                tma_store_3d(&a.tmO, 64 * j, pg * G, pr * B, smem + a.off_vb + j * (G * B * 128));
+            bulk_commit();
+        }
+        if (lane == 0) {
+            bulk_wait_all();
+            if (*fail) {
+                // let copies in flight land before the CTA exits
+                if (nx) mbar_wait(xfull, (uint32_t)(nx - 1) & 1u, kWaitNs);
+                if (nv) mbar_wait(vfull, (uint32_t)(nv - 1) & 1u, kWaitNs);
+            }
+        }
+    } else if (warp >= 4) {
+        // ------------------------------------------------------------- math
+        const int mt = tid - 128;
+        const int q4 = warp & 3, part = (warp - 4) >> 2;
+        const int row = 32 * q4 + lane;
+        const uint32_t lane_off = (uint32_t)(32 * q4) << 16;
+        const bool two = NCH >= 4;          // a part owns chunks part and part + 2 of each half
+        const bool has_sc = part < B / 16;  // score columns [16 part, 16 part + 16)
+        const int Mv = G * B;
+        const bool valid = row < Mv;
+        float *xa = reinterpret_cast<float *>(smem + a.off_st);   // [part][ms, mx, mn][128]
+        float *xb = xa + 6 * 128;                                  // [part][sp, lp, sn, ln, l][128]
+        const float scale_l2 = a.scale * kLog2e;
+        const uint32_t pair_bar = kBarPair + q4;
+        const float log_f = logf((float)F);
+        auto pair_failed = [&](bool local_fail) -> bool { return group_sync_failed(pair_bar, 64, local_fail); };
+
+        uint32_t kp = 0;
+        void *nraw = state_raw(a, u_begin, u_end);
+        float nalpha = valid && u_begin < u_end ? a.alpha[(u_begin % a.Hkv) * G + row % G] : 0.f;
+        for (int u = u_begin; u < u_end; ++u) {
+            void *raw = nraw;
+            nraw = state_raw(a, u + 1, u_end);
+            // gate of this row's query head, loaded one unit ahead
+            const float alpha_row = nalpha;
+            nalpha = valid && u + 1 < u_end ? a.alpha[((u + 1) % a.Hkv) * G + row % G] : 0.f;
+            if (!state_at(a, raw, u)) {
+                if (mt == 0) raise_error(a.err, ERR_BAD_STATE_PTR);
+                continue;
+            }
+            const int r = u / a.Hkv, g = u % a.Hkv;
+            const int zb = kp & 1;
+            const float *zs = zbuf0 + zb * zstride;
+            const uint32_t ucol = tmem + cU + lane_off, mcol = tmem + cM + lane_off;
+
+            // ---- phase A: row extrema of U and of the scores (U kept in registers)
+            bool bad = !wait_bar(uready, kp & 1u, fail, wlim);
+            tc_fence_after();
+            float sc[16], u0[32], u1[32];
+            if (has_sc) tmem_ld16(mcol + 16 * part, sc);
+            tmem_ld32(ucol + 32 * part, u0);
+            if (two) tmem_ld32(ucol + 32 * (part + 2), u1);
+            tmem_wait_ld();
+            {
+                float ms = -INFINITY, mx = -INFINITY, mn = INFINITY;
+                if (has_sc) {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) ms = fmaxf(ms, sc[i]);
+                }
+#pragma unroll
+                for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, u0[i]); mn = fminf(mn, u0[i]); }
+                if (two) {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, u1[i]); mn = fminf(mn, u1[i]); }
+                }
+                xa[(part * 3 + 0) * 128 + row] = ms;
+                xa[(part * 3 + 1) * 128 + row] = mx;
+                xa[(part * 3 + 2) * 128 + row] = mn;
+            }
+            // both parts have read their scores: phi- may overwrite the score columns
+            if (pair_failed(bad)) break;
+            const float ms = fmaxf(xa[0 * 128 + row], xa[3 * 128 + row]);
+            const float mx = fmaxf(xa[1 * 128 + row], xa[4 * 128 + row]);
+            const float mn = fminf(xa[2 * 128 + row], xa[5 * 128 + row]);
+            const float lw = valid ? log_sigmoid(alpha_row) : 0.f;
+            // fast: w sp e^(max s) <= w F e^(max s) stays below e^60 for every row of the
+            // warp, so phi+ and phi- are released unnormalised as soon as they are written
+            const bool fast = __all_sync(0xffffffffu, !(lw + ms * a.scale + log_f > 60.f));
+
+            // ---- phase B: phi+ then phi- into Tensor Memory, with their sums and
+            // their dot products with z
+            bad = !wait_bar(&zfull[zb], (kp >> 1) & 1u, fail, wlim) || bad;
+            const float mxl = mx * kLog2e, mnl = mn * kLog2e, ml = ms * scale_l2;
+            float sp = 0.f, lp = 0.f, sn = 0.f, ln = 0.f, l = 0.f;
+            auto expp = [&](const float (&uu)[32], int k) {
+                float ep[32];
+                const float4 *zp = reinterpret_cast<const float4 *>(zs + 32 * k);
+#pragma unroll
+                for (int i4 = 0; i4 < 8; ++i4) {
+                    const float4 z4 = zp[i4];
+                    const float za[4] = {z4.x, z4.y, z4.z, z4.w};
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const int i = 4 * i4 + j;
+                        const float e = ex2(fmaf(uu[i], kLog2e, -mxl));
+                        ep[i] = e;
+                        sp += e;
+                        lp = fmaf(e, za[j], lp);
+                    }
+                }
+                tmem_st32(ucol + 32 * k, ep);
+            };
+            auto expm = [&](float (&uu)[32], int k) {
+                const float4 *zn = reinterpret_cast<const float4 *>(zs + F + 32 * k);
+#pragma unroll
+                for (int i4 = 0; i4 < 8; ++i4) {
+                    const float4 z4 = zn[i4];
+                    const float za[4] = {z4.x, z4.y, z4.z, z4.w};
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const int i = 4 * i4 + j;
+                        const float e = ex2(fmaf(-uu[i], kLog2e, mnl));
+                        uu[i] = e;
+                        sn += e;
+                        ln = fmaf(e, za[j], ln);
+                    }
+                }
+                tmem_st32(mcol + 32 * k, uu);
+            };
+            auto release = [&](uint64_t *bar) {
+                tmem_wait_st();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0 && !bad && !(a.withhold && bar == phip)) mbar_arrive(bar);
+            };
+            expp(u0, part);
+            if (two) expp(u1, part + 2);
+            if (fast) release(phip);
+            expm(u0, part);
+            if (two) expm(u1, part + 2);
+            if (fast) release(phim);
+            if (has_sc) {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) l += ex2(fmaf(sc[i], scale_l2, -ml));
+            }
+            xb[(part * 5 + 0) * 128 + row] = sp;
+            xb[(part * 5 + 1) * 128 + row] = lp;
+            xb[(part * 5 + 2) * 128 + row] = sn;
+            xb[(part * 5 + 3) * 128 + row] = ln;
+            xb[(part * 5 + 4) * 128 + row] = l;
+            // z has been read
+            __syncwarp();
+            if (lane == 0 && !bad) mbar_arrive(&zempty[zb]);
+            if (pair_failed(bad)) break;
+
+            // ---- phase C: sigma, den, P' (and off the fast path the rescale of phi)
+            sp = xb[0 * 128 + row] + xb[5 * 128 + row];
+            lp = xb[1 * 128 + row] + xb[6 * 128 + row];
+            sn = xb[2 * 128 + row] + xb[7 * 128 + row];
+            ln = xb[3 * 128 + row] + xb[8 * 128 + row];
+            l = xb[4 * 128 + row] + xb[9 * 128 + row];
+            const float lin_den = lp / sp + ln / sn;
+            const float log_s = lw + ms * a.scale + logf(l);   // log(w sm_den)
+            const float log_l = logf(lin_den);                   // log(lin_den), -inf if empty
+            const float sig = fmaxf(fmaxf(log_s, log_l), -60.f);
+            const float esig = expf(-sig);
+            const float inv_den = 1.f / (expf(log_l - sig) + expf(log_s - sig));
+            float ap, am, pofs;
+            if (fast) {
+                ap = esig / sp * inv_den;
+                am = esig / sn * inv_den;
+                pofs = (lw + logf(sp)) * kLog2e;
+            } else {
+                const float cpos = lin_den > 0.f ? esig / sp : 0.f;
+                const float cneg = lin_den > 0.f ? esig / sn : 0.f;
+                auto scale_chunk = [&](uint32_t col, float c) {
+                    float v[32];
+                    tmem_ld32(col, v);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] *= c;
+                    tmem_st32(col, v);
+                };
+                scale_chunk(ucol + 32 * part, cpos);
+                if (two) scale_chunk(ucol + 32 * (part + 2), cpos);
+                release(phip);
+                scale_chunk(mcol + 32 * part, cneg);
+                if (two) scale_chunk(mcol + 32 * (part + 2), cneg);
+                release(phim);
+                ap = inv_den;
+                am = inv_den;
+                pofs = (lw - sig) * kLog2e;
+            }
+            // P' lands in X: the previous unit's output stores must have read it
+            if (kp >= 1) bad = !wait_bar(ofree, (kp - 1) & 1u, fail, wlim) || bad;
+            if (has_sc) {
+                // P' (w sp e^s on the fast path, w e^(s - sigma) off it): K-major, no
+                // swizzle (8-row x 16-byte core matrices).
+                uint32_t pk[8];
+#pragma unroll
+                for (int i = 0; i < 16; i += 2)
+                    pk[i / 2] = pack_bf16x2(ex2(fmaf(sc[i], scale_l2, pofs)), ex2(fmaf(sc[i + 1], scale_l2, pofs)));
+                uint8_t *prow = smem + a.off_p + (row >> 3) * (B / 8) * 128 + (row & 7) * 16;
+                *reinterpret_cast<uint4 *>(prow + (2 * part) * 128) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                *reinterpret_cast<uint4 *>(prow + (2 * part + 1) * 128) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0 && !bad) mbar_arrive(pready);
+
+            // ---- phase E: out = a+ D+ + a- D-, staged in X as the TMA box image (row
+            // t*G + h, 16-byte granule k of a 64-column box at k ^ (row mod 8)); the
+            // producer warp stores it
+            bad = !wait_bar(dpdone, kp & 1u, fail, wlim) || bad;
+            bad = !wait_bar(dmdone, kp & 1u, fail, wlim) || bad;
+            tc_fence_after();
+            {
+                const int dh = d / 2;
+#pragma unroll 1
+                for (int hc = 0; hc < dh / 32; ++hc) {
+                    float vp[32], vm[32];
+                    tmem_ld32(tmem + cDp + lane_off + part * dh + 32 * hc, vp);
+                    tmem_ld32(tmem + cDm + lane_off + part * dh + 32 * hc, vm);
+                    tmem_wait_ld();
+                    if (hc == dh / 32 - 1) {
+                        // D+ and D- are read: the next unit's readout may start
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0 && !bad) mbar_arrive(dfree);
+                    }
+                    if (valid) {
+                        const int c0 = part * dh + 32 * hc;
+                        uint8_t *box = smem + a.off_vb + (c0 >> 6) * (Mv * 128) + row * 128;
+                        const int kb = (c0 & 63) >> 3;
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            uint32_t w4[4];
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const int c = 8 * j + 2 * i;
+                                w4[i] = pack_bf16x2(fmaf(vp[c], ap, vm[c] * am), fmaf(vp[c + 1], ap, vm[c + 1] * am));
+                            }
+                            *reinterpret_cast<uint4 *>(box + (((kb + j) ^ (row & 7)) << 4)) =
+                                make_uint4(w4[0], w4[1], w4[2], w4[3]);
+                        }
+                    }
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0 && !bad) mbar_arrive(ostaged);
+            }
+            if (bad) break;
+            ++kp;
+        }
+        if (mt == 0 && *fail) raise_error(a.err, ERR_WAIT_TIMEOUT);
+    }
+
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+}  // namespace
+
+bool step_supported(const hybrid_cfg &c)
+{
+    if (c.io_dtype != HYBRID_BF16) return false;
+    if (c.head_dim != 64 && c.head_dim != 128) return false;
+    if (c.feat_dim != 64 && c.feat_dim != 128) return false;
+    // scores ride in one 16-column chunk per part and fit under phi-; the K^T
+    // atom holds B <= 64 tokens
+    if (c.block_size != 16 && c.block_size != 32) return false;
+    const int G = c.n_q_heads / c.n_kv_heads;
+    if (G * c.block_size > 128) return false;
+    const SLayout L = make_slayout(c.head_dim, c.feat_dim, c.block_size, c.n_q_heads / c.n_kv_heads);
+    if (L.NS < 4) return false;
+    return (int)L.bytes <= kSmemLimit;
+}
+
+cudaError_t launch_step(const hybrid_cfg &c, const void *Q, const void *K, const void *V, const void *W,
+                        const float *alpha, void *const *states, int n_req, void *O, unsigned *err,
+                        cudaStream_t st)
+{
+    const SLayout L = make_slayout(c.head_dim, c.feat_dim, c.block_size, c.n_q_heads / c.n_kv_heads);
+    StepArgs a;
+    {
+        const int d = c.head_dim, F = c.feat_dim, B = c.block_size, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
+        const int G = Hq / Hkv;
+        const cuuint64_t rows = (cuuint64_t)n_req * B;
+        const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)Hq, rows};
+        const cuuint64_t sq[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hq * d * 2};
+        const cuuint32_t bq[3] = {64, (cuuint32_t)G, (cuuint32_t)B};
+        const cuuint64_t dv[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, rows};
+        const cuuint64_t sv[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
+        const cuuint32_t bv[3] = {64, 1, (cuuint32_t)B};
+        const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
+        const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
+        const cuuint32_t bw[2] = {64, (cuuint32_t)d};
+        if (!encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !encode_bf16(&a.tmV, V, 3, dv, sv, bv) ||
+            !encode_bf16(&a.tmW, W, 2, dw, sw, bw) || !encode_bf16(&a.tmO, O, 3, dq, sq, bq))
+            return cudaErrorInvalidValue;
+    }
+    a.K = static_cast<const bf16 *>(K);
+    a.O = static_cast<bf16 *>(O);
+    a.alpha = alpha;
+    a.states = states;
+    a.err = err;
+    a.n_units = n_req * c.n_kv_heads;
+    a.B = c.block_size;
+    a.Hq = c.n_q_heads;
+    a.Hkv = c.n_kv_heads;
+    a.G = c.n_q_heads / c.n_kv_heads;
+    a.d = c.head_dim;
+    a.F = c.feat_dim;
+    a.NS = L.NS;
+    a.scale = 1.f / sqrtf((float)c.head_dim);
+    {
+        // a test may arm one step launch with a short wait limit and a withheld arrival
+        const unsigned long long armed = g_armed_wait_ns.exchange(0ull);
+        a.wait_ns = armed ? armed : (unsigned long long)kWaitNs;
+        a.withhold = armed ? 1 : 0;
+    }
+    a.off_q = L.off_q;
+    a.off_wk = L.off_wk;
+    a.off_vb = L.off_vb;
+    a.off_p = L.off_p;
+    a.off_z = L.off_z;
+    a.off_st = L.off_st;
+    a.off_bar = L.off_bar;
+    const int grid = a.n_units < sm_count() ? a.n_units : sm_count();
+    // opt in to the full shared memory once per device
+    static std::atomic<unsigned long long> opted{0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    const unsigned long long bit = 1ull << dev;
+    if (!(opted.load(std::memory_order_acquire) & bit)) {
+        const cudaError_t e = cudaFuncSetAttribute(k_step, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
+        if (e != cudaSuccess) return e;
+        opted.fetch_or(bit, std::memory_order_release);
+    }
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid);
+    lc.blockDim = dim3(kThreads);
+    lc.dynamicSmemBytes = L.bytes;
+    lc.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 1;
+    return cudaLaunchKernelEx(&lc, k_step, a);
+}
+
+}  // namespace hyb

@@ -20,6 +20,13 @@ cudaError_t launch_attn_tc(const hybrid_cfg &c, const void *Q, const void *K, co
                            const void *W, const float *alpha, void *const *states, int n_req,
                            void *O, unsigned *err, cudaStream_t st);
 
+// Persistent step kernel, one unit at a time with both feature halves read out
+// at once (hybrid_step.cu).
+bool step_supported(const hybrid_cfg &c);
+cudaError_t launch_step(const hybrid_cfg &c, const void *Q, const void *K, const void *V, const void *W,
+                        const float *alpha, void *const *states, int n_req, void *O, unsigned *err,
+                        cudaStream_t st);
+
 // Persistent warp-specialised step kernel (hybrid_fused.cu); commit = true also
 // folds the block's K/V into the state in the same pass.
 bool fused_supported(const hybrid_cfg &c, bool commit);
