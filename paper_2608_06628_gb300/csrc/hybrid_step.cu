@@ -6,12 +6,14 @@
 //
 // Work unit = (request r, state head g): the G*B query rows of the unit share one
 // state.  Warp roles (12 warps):
-//   warp 0     state producer: z and the 2F/32 state tiles of each unit, by 1-D
-//              bulk copies into an NS-slot ring, phi+ and phi- tiles interleaved
-//              (the state layout is the MMA operand image, see hybrid.h)
+//   warp 0     ring producer: per unit Q (TMA) and then the F/32 pairs of state
+//              tiles (phi+ tile c with phi- tile c, 1-D bulk copies) into an
+//              NS-slot ring of 2 d x 128-byte slots (the state layout is the MMA
+//              operand image, see hybrid.h); z beside the ring
 //   warp 1     MMA issuer A; owns the Tensor Memory allocation:
 //              g1 = [U | scores] = Q [W | K^T], the phi+ readout, P'V
-//   warp 2     producer: TMA of Q and W, K^T (transposed by the warp), V by TMA
+//   warp 2     producer: TMA of W, K^T (transposed by the warp), V by TMA, and the
+//              TMA stores of the output tile
 //   warp 3     MMA issuer B: the phi- readout
 //   warps 4-11 math: two threads per query row (one per TMEM lane and "part";
 //              a part owns every other 32-feature chunk of each half of phi)
@@ -73,43 +75,42 @@ struct StepArgs {
     float scale;
     unsigned long long wait_ns;       // limit of every bounded wait (1 s unless a test armed less)
     int withhold;                     // test hook: the math warps never release phi+
-    uint32_t off_q, off_wk, off_vb, off_p, off_z, off_st, off_bar;
+    uint32_t off_wk, off_vb, off_p, off_z, off_st, off_bar;
 };
 
-// Shared memory: [ring NS x d*128][Q][W | K^T][X][z x2][stats][barriers], where X
+// Shared memory: [ring NS x 2*d*128][W | K^T][X][z x2][stats][barriers], where X
 // holds V and P' until the unit's P'V has read them and then the output tile,
 // staged as the image of d/64 TMA boxes of 64 columns x G*B rows (row t*G + h,
 // 128-byte swizzle) that the producer warp stores.
 // Q, V and W land by TMA with the 128-byte swizzle: Q as d/64 atoms of 128 rows
 // (16 KB apart; rows t*G + h), V as d/64 atoms of B rows (MN-major operand), W as
 // F/64 atoms of d rows (MN-major) followed by the K^T atom (row e holds
-// K[0..B)[e]), so that [W | K^T] is one MN-major B operand.  The ring has an even
-// number of slots, so a slot always holds tiles of the same half and is read by
-// the same issuer, in order.
+// K[0..B)[e]), so that [W | K^T] is one MN-major B operand.  A ring slot holds
+// either a unit's Q (d/64 atoms of 128 rows, as big as two state tiles) or a pair
+// of state tiles that the two issuers read at once; Q passing through the ring
+// frees its space for tiles as soon as g1 has read it, so a whole unit's tiles
+// can be in flight.
 struct SLayout {
-    uint32_t off_q, off_wk, off_vb, off_p, off_z, off_st, off_bar, bytes;
+    uint32_t off_wk, off_vb, off_p, off_z, off_st, off_bar, bytes;
     int NS;
 };
 
 SLayout make_slayout(int d, int F, int B, int G)
 {
     SLayout L{};
-    const uint32_t chunk = (uint32_t)d * 128;
+    const uint32_t slot = (uint32_t)d * 256;
     const uint32_t zb = (((uint32_t)2 * F * 4) + 1023) & ~1023u;
-    const uint32_t q = (uint32_t)d * 256;
     const uint32_t wk = (uint32_t)(F / 64 + 1) * d * 128;
     const uint32_t vb = (((uint32_t)B * d * 2) + 1023) & ~1023u;
     const uint32_t p = (((uint32_t)128 * B * 2) + 1023) & ~1023u;
     const uint32_t oimg = (uint32_t)(d / 64) * G * B * 128;
     const uint32_t x = ((vb + p > oimg ? vb + p : oimg) + 1023) & ~1023u;
     const uint32_t bar = 1024;
-    const uint32_t fixed = q + wk + x + 2 * zb + kStatBytes + bar + 1024;
-    int ns = ((int)kSmemLimit - (int)fixed) / (int)chunk;
+    const uint32_t fixed = wk + x + 2 * zb + kStatBytes + bar + 1024;
+    int ns = ((int)kSmemLimit - (int)fixed) / (int)slot;
     if (ns > kMaxSlots) ns = kMaxSlots;
-    ns &= ~1;
     L.NS = ns;
-    uint32_t off = (uint32_t)(ns > 0 ? ns : 0) * chunk;
-    L.off_q = off; off += q;
+    uint32_t off = (uint32_t)(ns > 0 ? ns : 0) * slot;
     L.off_wk = off; off += wk;
     L.off_vb = off;
     L.off_p = off + vb;
@@ -136,9 +137,6 @@ __device__ __forceinline__ float *state_at(const StepArgs &a, void *raw, int u)
     return st + (size_t)(u % a.Hkv) * head_floats(a.d, a.F);
 }
 
-// ring position p of a unit (0 .. 2F/32 - 1) -> state tile: phi+ and phi- tiles
-// alternate, so issuer A reads the even positions and issuer B the odd ones
-__device__ __forceinline__ int tile_of_pos(int p, int NCH) { return (p & 1) ? NCH + (p >> 1) : (p >> 1); }
 
 __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ StepArgs a)
 {
@@ -149,8 +147,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
     const int d = a.d, F = a.F, B = a.B, G = a.G, NS = a.NS;
     const uint64_t wlim = a.wait_ns;
     const int NCH = F / 32;          // 32-feature chunks (state tiles) per half of phi
-    const int NC = 2 * NCH;          // state tiles per unit
-    const uint32_t chunk_bytes = (uint32_t)d * 128;
+    const uint32_t chunk_bytes = (uint32_t)d * 128;   // one state tile
+    const uint32_t slot_bytes = 2 * chunk_bytes;      // a ring slot: Q, or a phi+ / phi- tile pair
+    const int NI = 1 + NCH;                           // ring items per unit
     const int per = a.n_units / (int)gridDim.x, rem = a.n_units % (int)gridDim.x;
     const int u_begin = (int)blockIdx.x * per + min((int)blockIdx.x, rem);
     const int u_end = u_begin + per + ((int)blockIdx.x < rem ? 1 : 0);
@@ -158,8 +157,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
     const uint32_t cU = 0, cM = (uint32_t)F, cDp = 2u * F, cDm = 2u * F + d;
 
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + a.off_bar);
-    uint64_t *full = bars;            // [NS] a state tile has landed in the slot
-    uint64_t *empty = full + NS;      // [NS] the slot's tile has been read by its MMAs
+    uint64_t *full = bars;            // [NS] the slot's item (Q or a tile pair) has landed
+    uint64_t *empty = full + NS;      // [NS] both issuers are done with the slot's item
     uint64_t *zfull = empty + NS;     // [2]
     uint64_t *zempty = zfull + 2;     // [2]
     uint64_t *mmadone = zempty + 2;   // [2] per issuer: all of its MMAs have completed
@@ -179,14 +178,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + n_bars);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
+    if (warp == 0 && lane == 0) prefetch_tensormap(&a.tmQ);
     if (warp == 2 && lane == 0) {
-        prefetch_tensormap(&a.tmQ);
         prefetch_tensormap(&a.tmW);
         prefetch_tensormap(&a.tmV);
         prefetch_tensormap(&a.tmO);
     }
     if (tid == 0) {
         for (int i = 0; i < n_bars; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < NS; ++i) mbar_init(&empty[i], 2);
         mbar_init(xfull, 2);
         mbar_init(phip, 8);
         mbar_init(phim, 8);
@@ -228,17 +228,31 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                 nraw = state_raw(a, u + 1, u_end);
                 float *Sg = state_at(a, raw, u);
                 if (!Sg) continue;
+                const int r = u / a.Hkv, g = u % a.Hkv;
+                // item 0: Q of the unit (the first thing g1 needs)
+                {
+                    const int slot = q % NS;
+                    if (!wait_bar(&empty[slot], ((q / NS) & 1u) ^ 1u, fail, wlim)) break;
+                    mbar_arrive_expect_tx(&full[slot], (uint32_t)(d / 64) * (G * B * 128));
+                    for (int e = 0; e < d / 64; ++e)
+                        tma_load_3d(ring + (size_t)slot * slot_bytes + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B,
+                                    &full[slot]);
+                    ++issued_slot[slot];
+                    ++q;
+                }
                 const int zb = kp & 1;
                 if (!wait_bar(&zempty[zb], ((kp >> 1) & 1u) ^ 1u, fail, wlim)) break;
                 mbar_arrive_expect_tx(&zfull[zb], 2 * F * 4);
                 bulk_g2s(zbuf0 + zb * zstride, Sg + (size_t)2 * F * d, 2 * F * 4, &zfull[zb]);
                 ++issued_z[zb];
-                for (int p = 0; p < NC; ++p, ++q) {
+                // items 1 .. F/32: phi+ tile c with phi- tile c
+                for (int c = 0; c < NCH; ++c, ++q) {
                     const int slot = q % NS;
-                    if (!wait_bar(&empty[slot], ((q / NS) & 1u) ^ 1u, fail, wlim)) break;
-                    mbar_arrive_expect_tx(&full[slot], chunk_bytes);
-                    bulk_g2s(ring + (size_t)slot * chunk_bytes, Sg + (size_t)tile_of_pos(p, NCH) * 32 * d,
-                             chunk_bytes, &full[slot]);
+                    if (!wait_bar(&empty[slot], ((q / NS) & 1u) ^ 1u, fail, wlim)) { ok = false; break; }
+                    uint8_t *dst = ring + (size_t)slot * slot_bytes;
+                    mbar_arrive_expect_tx(&full[slot], slot_bytes);
+                    bulk_g2s(dst, Sg + (size_t)c * 32 * d, chunk_bytes, &full[slot]);
+                    bulk_g2s(dst + chunk_bytes, Sg + (size_t)(NCH + c) * 32 * d, chunk_bytes, &full[slot]);
                     ++issued_slot[slot];
                 }
                 ++kp;
@@ -258,13 +272,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
             // tiles of this issuer: ring positions iss, iss + 2, ... of each unit, into D+ or D-
             const uint32_t acol0 = iss ? cM : cU, dcol = iss ? cDm : cDp;
-            auto readout_half = [&](uint32_t qt) -> bool {
+            // this issuer's tile of each pair item of the unit whose items start at qb
+            auto readout_half = [&](uint32_t qb) -> bool {
                 for (int c = 0; c < NCH; ++c) {
-                    const uint32_t qc = qt + 2 * c + iss;
+                    const uint32_t qc = qb + 1 + c;
                     const int slot = (int)(qc % (uint32_t)NS);
                     if (!wait_bar(&full[slot], (qc / NS) & 1u, fail, wlim)) return false;
                     tc_fence_after();
-                    const uint64_t b0 = smem_desc(ring_u + (uint32_t)slot * chunk_bytes, 16, 1024, SWZ_128B);
+                    const uint64_t b0 =
+                        smem_desc(ring_u + (uint32_t)slot * slot_bytes + iss * chunk_bytes, 16, 1024, SWZ_128B);
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
                         mma_tf32_ts(tmem + dcol, tmem + acol0 + 32 * c + 8 * kk, b0 + 2 * kk, idR, (c | kk) != 0);
@@ -274,7 +290,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             };
             uint32_t kp = 0, qt = 0;
             if (iss == 0) {
-                const uint32_t q_u = smem_u32(smem + a.off_q), wk_u = smem_u32(smem + a.off_wk),
+                const uint32_t wk_u = smem_u32(smem + a.off_wk),
                                vb_u = smem_u32(smem + a.off_vb), p_u = smem_u32(smem + a.off_p);
                 const uint32_t idUS = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F + B);
                 const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
@@ -287,6 +303,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                     // g1 writes [U | scores] over the previous unit's phi+ (read by this
                     // thread's own earlier MMAs, in issue order) and phi- (read by issuer B)
                     if (kp >= 1 && !wait_bar(dmdone, (kp - 1) & 1u, fail, wlim)) break;
+                    const int qs = (int)(qt % (uint32_t)NS);
+                    if (!wait_bar(&full[qs], (qt / NS) & 1u, fail, wlim)) break;
+                    const uint32_t q_u = ring_u + (uint32_t)qs * slot_bytes;
                     tc_fence_after();
                     for (int k = 0; k < d / 16; ++k) {
                         const uint64_t aq = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
@@ -295,6 +314,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                     }
                     mma_commit(uready);
                     mma_commit(xfree);
+                    mma_commit(&empty[qs]);
                     if (!wait_bar(phip, kp & 1u, fail, wlim)) break;
                     // D+ is written from the first phi+ MMA on: the previous epilogue has read it
                     if (kp >= 1 && !wait_bar(dfree, (kp - 1) & 1u, fail, wlim)) break;
@@ -307,7 +327,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                         mma_bf16_ss(tmem + cDp, ap, bv, idP, 1);
                     }
                     mma_commit(dpdone);
-                    qt += NC;
+                    qt += NI;
                     ++kp;
                 }
             } else {
@@ -316,11 +336,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                     void *raw = nraw;
                     nraw = state_raw(a, u + 1, u_end);
                     if (!state_at(a, raw, u)) continue;
+                    // the unit's Q item is read by issuer A alone: this thread's share of
+                    // its release, once it has landed
+                    const int qs = (int)(qt % (uint32_t)NS);
+                    if (!wait_bar(&full[qs], (qt / NS) & 1u, fail, wlim)) break;
+                    mbar_arrive(&empty[qs]);
                     if (!wait_bar(phim, kp & 1u, fail, wlim)) break;
                     if (kp >= 1 && !wait_bar(dfree, (kp - 1) & 1u, fail, wlim)) break;
                     if (!readout_half(qt)) break;
                     mma_commit(dmdone);
-                    qt += NC;
+                    qt += NI;
                     ++kp;
                 }
             }
@@ -331,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
         // ------------------------------------------------------------- producer
         uint32_t kp = 0;
         int nx = 0, nv = 0;
-        const uint32_t xbytes = (uint32_t)(d / 64) * (G * B * 128) + (uint32_t)(F / 64) * (d * 128);
+        const uint32_t xbytes = (uint32_t)(F / 64) * (d * 128);
         uint8_t *kt = smem + a.off_wk + (F / 64) * d * 128;
         int pr = 0, pg = 0;             // request and head of the previous unit
         void *nraw = state_raw(a, u_begin, u_end);
@@ -347,8 +372,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
                 mbar_arrive_expect_tx(xfull, xbytes);
-                for (int e = 0; e < d / 64; ++e)
-                    tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xfull);
                 for (int f = 0; f < F / 64; ++f)
                     tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xfull);
             }
@@ -425,7 +448,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                 if (mt == 0) raise_error(a.err, ERR_BAD_STATE_PTR);
                 continue;
             }
-            const int r = u / a.Hkv, g = u % a.Hkv;
             const int zb = kp & 1;
             const float *zs = zbuf0 + zb * zstride;
             const uint32_t ucol = tmem + cU + lane_off, mcol = tmem + cM + lane_off;
@@ -652,7 +674,7 @@ bool step_supported(const hybrid_cfg &c)
     const int G = c.n_q_heads / c.n_kv_heads;
     if (G * c.block_size > 128) return false;
     const SLayout L = make_slayout(c.head_dim, c.feat_dim, c.block_size, c.n_q_heads / c.n_kv_heads);
-    if (L.NS < 4) return false;
+    if (L.NS < 2) return false;
     return (int)L.bytes <= kSmemLimit;
 }
 
@@ -699,7 +721,6 @@ cudaError_t launch_step(const hybrid_cfg &c, const void *Q, const void *K, const
         a.wait_ns = armed ? armed : (unsigned long long)kWaitNs;
         a.withhold = armed ? 1 : 0;
     }
-    a.off_q = L.off_q;
     a.off_wk = L.off_wk;
     a.off_vb = L.off_vb;
     a.off_p = L.off_p;
