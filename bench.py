@@ -839,6 +839,13 @@ def run_hybrid(args, wl):
                      else "fallback 6.8 TB/s", "unit": "GB/s", "frac": achieved / hbm,
                      "traffic": recorded_traffic(kname, wl.name),
                      "algorithmic_bytes_per_launch": ab["fused"]},
+        # the step alone (the attention-only launches of the denoising steps that do
+        # not commit), timed the same way in its own graph of the rotating sets
+        "roofline_step": {"bound": "hbm", "kernel": "hybrid_block_attn",
+                          "achieved": ab["attn"] / (attn_ms * 1e-3) / 1e9, "peak": hbm,
+                          "unit": "GB/s", "frac": ab["attn"] / (attn_ms * 1e-3) / 1e9 / hbm,
+                          "traffic": recorded_traffic("hybrid_block_attn", wl.name),
+                          "algorithmic_bytes_per_launch": ab["attn"], "us_per_launch": attn_ms * 1e3},
         "timing": "K steps replayed from CUDA graphs (one launch per step); "
                   f"direct Python launches: {direct_ms * 1e3:.1f} us/step",
         "kernels": {
