@@ -177,8 +177,7 @@ hybrid_status hybrid_block_attn_commit(const hybrid_cfg *cfg, const void *Q, con
  * last call's contents (each call overwrites every byte it reads).  Calls that
  * overlap on the GPU race on it: issue them on one stream, or synchronise.
  * Set-up: the first call on a device, with that device current, looks the
- * scratch address up with cudaGetSymbolAddress (n_req = 0 does only that).
- * Make that first call before any stream capture begins. */
+ * scratch address up with cudaGetSymbolAddress (n_req = 0 does only that). */
 hybrid_status hybrid_block_attn_commit_logical(const hybrid_cfg *cfg, const void *Q, const void *K,
                                                const void *V, const void *W, const float *alpha,
                                                float *S_logical, float *z_logical, int n_req, void *O,

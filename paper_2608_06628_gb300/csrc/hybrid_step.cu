@@ -29,7 +29,8 @@
 // two halves of the readout go out from two threads into two accumulators.
 // Per unit: g1; the math warps take the row extrema, write phi+ and then phi-
 // (released to issuers A and B as each lands), take the exponential sums and
-// P'; the epilogue combines out = a+ D+ + a- D- from registers.  The next
+// P'; the epilogue combines out = a+ D+ + a- D- and writes it into a staged
+// TMA box image that warp 2 stores.  The next
 // unit's g1 follows as soon as its phi- readout has read the phi- columns, so
 // its feature map runs while this unit's epilogue drains.
 //
