@@ -11,12 +11,13 @@
 //              NS-slot ring of 2 d x 128-byte slots (the state layout is the MMA
 //              operand image, see hybrid.h); z beside the ring
 //   warp 1     MMA issuer A; owns the Tensor Memory allocation:
-//              g1 = [U | scores] = Q [W | K^T], the phi+ readout, P'V
-//   warp 2     producer: TMA of W, K^T (transposed by the warp), V by TMA, and the
-//              TMA stores of the output tile
-//   warp 3     MMA issuer B: the phi- readout
-//   warps 4-11 math: two threads per query row (one per TMEM lane and "part";
-//              a part owns every other 32-feature chunk of each half of phi)
+//              U = Q W, the phi+ readout, P'V
+//   warp 2     producer: TMA of W, K and V, and the TMA stores of the output tile
+//   warp 3     MMA issuer B: the scores Q K^T (K, as loaded, is the K-major
+//              operand), the phi- readout
+//   warps 4-11 math: two threads per query row (one warp per TMEM lane quarter
+//              and "part"; part p owns the 32-feature chunks p, p + 2, ... of each
+//              half of phi, d / 2 output columns and 16 score columns)
 //
 // Tensor Memory (512 columns):
 //   [0, F)          U, then phi+ = e^(u - max u), written in place
@@ -27,12 +28,13 @@
 // A tcgen05.mma with M = 128 keeps its issuing thread ~140 cycles whatever N is,
 // twice the time the tensor pipe needs for a tf32 product with N = 128, so the
 // two halves of the readout go out from two threads into two accumulators.
-// Per unit: g1; the math warps take the row extrema, write phi+ and then phi-
-// (released to issuers A and B as each lands), take the exponential sums and
-// P'; the epilogue combines out = a+ D+ + a- D- and writes it into a staged
-// TMA box image that warp 2 stores.  The next
-// unit's g1 follows as soon as its phi- readout has read the phi- columns, so
-// its feature map runs while this unit's epilogue drains.
+// Per unit: g1 (U on issuer A, the scores on issuer B); the math warps take the
+// row extrema, write phi+ and then phi- (released to issuers A and B as each
+// lands), take the exponential sums and P'; the epilogue combines
+// out = a+ D+ + a- D- and writes it into a staged TMA box image that warp 2
+// stores.  Each issuer starts the next unit's half of g1 right after its own
+// readout of this unit, so the next feature map can start while this unit's
+// epilogue drains.
 //
 // Merge (Section 3.1, out = (w sm_num + lin_num) / (w sm_den + lin_den)): phi+
 // and phi- stay unnormalised, P' = w sp e^s rides in D+, so
@@ -57,17 +59,20 @@ namespace {
 
 using namespace pipe;
 
-constexpr int kWarps = 12;
-constexpr int kThreads = kWarps * 32;
 constexpr int kMaxSlots = 16;
 constexpr int kSmemLimit = 232448;
 constexpr int kOneCtaPerSm = 118 * 1024;
 constexpr uint32_t kBarPair = 2;      // 2..5: the two math warps of one TMEM lane quarter
-constexpr uint32_t kStatBytes = 8 * 1024;
+constexpr int P = 2;                  // math threads ("parts") per query row
+constexpr int kThreads = (4 + 4 * P) * 32;
+constexpr int kMath = 4 * P;          // math warps
+// row statistics exchanged between the parts of a row, per part: the score maximum
+// and exponential sum, the extrema of U, and the sums and z products of phi+ and phi-
+constexpr uint32_t kStatBytes = 8 * 128 * 4 * P;
+constexpr int SC = 16;                // score columns per part (parts 0 .. B/16 - 1)
 
 struct StepArgs {
-    CUtensorMap tmQ, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
-    const bf16 *K;
+    CUtensorMap tmQ, tmK, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], K, V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
     bf16 *O;
     const float *alpha;
     void *const *states;
@@ -101,12 +106,12 @@ SLayout make_slayout(int d, int F, int B, int G)
     SLayout L{};
     const uint32_t slot = (uint32_t)d * 256;
     const uint32_t zb = (((uint32_t)2 * F * 4) + 1023) & ~1023u;
-    const uint32_t wk = (uint32_t)(F / 64 + 1) * d * 128;
+    const uint32_t wk = (uint32_t)(F / 64) * d * 128 + ((((uint32_t)B * d * 2) + 1023) & ~1023u);
     const uint32_t vb = (((uint32_t)B * d * 2) + 1023) & ~1023u;
     const uint32_t p = (((uint32_t)128 * B * 2) + 1023) & ~1023u;
     const uint32_t oimg = (uint32_t)(d / 64) * G * B * 128;
     const uint32_t x = ((vb + p > oimg ? vb + p : oimg) + 1023) & ~1023u;
-    const uint32_t bar = 1024;
+    const uint32_t bar = 512;   // up to 2 * kMaxSlots + 18 barriers, the TMEM address, the failure flag
     const uint32_t fixed = wk + x + 2 * zb + kStatBytes + bar + 1024;
     int ns = ((int)kSmemLimit - (int)fixed) / (int)slot;
     if (ns > kMaxSlots) ns = kMaxSlots;
@@ -150,7 +155,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
     const int NCH = F / 32;          // 32-feature chunks (state tiles) per half of phi
     const uint32_t chunk_bytes = (uint32_t)d * 128;   // one state tile
     const uint32_t slot_bytes = 2 * chunk_bytes;      // a ring slot: Q, or a phi+ / phi- tile pair
-    const int NI = 1 + NCH;                           // ring items per unit
     const int per = a.n_units / (int)gridDim.x, rem = a.n_units % (int)gridDim.x;
     const int u_begin = (int)blockIdx.x * per + min((int)blockIdx.x, rem);
     const int u_end = u_begin + per + ((int)blockIdx.x < rem ? 1 : 0);
@@ -163,39 +167,43 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
     uint64_t *zfull = empty + NS;     // [2]
     uint64_t *zempty = zfull + 2;     // [2]
     uint64_t *mmadone = zempty + 2;   // [2] per issuer: all of its MMAs have completed
-    uint64_t *xfull = mmadone + 2;    // Q, W (TMA) and K^T (producer warp) are in place
-    uint64_t *xfree = xfull + 1;      // g1 has read Q, W, K^T
+    uint64_t *xfull = mmadone + 2;    // W and K (TMA) are in place
+    uint64_t *xfree = xfull + 1;      // A, B -> producer: U and the scores have read W and K
     uint64_t *vfull = xfree + 1;
-    uint64_t *uready = vfull + 1;     // A -> math: g1 done
-    uint64_t *phip = uready + 1;      // math -> A: phi+ is written
-    uint64_t *phim = phip + 1;        // math -> B: phi- is written
-    uint64_t *pready = phim + 1;      // math -> A: P' is written
+    uint64_t *uready = vfull + 1;     // A, B -> math: U and the scores are in Tensor Memory
+    uint64_t *phip = uready + 1;      // [2] math -> A: phi+ chunks 0, 1 / 2, 3 are written
+    uint64_t *phim = phip + 2;        // [2] math -> B: the same for phi-
+    uint64_t *pready = phim + 2;      // math -> A: P' is written
     uint64_t *dpdone = pready + 1;    // A -> math: D+ (phi+ readout and P'V) is complete
     uint64_t *dmdone = dpdone + 1;    // B -> math, A: D- is complete (phi- has been read)
     uint64_t *dfree = dmdone + 1;     // math -> A, B: the epilogue has read D+ and D-
     uint64_t *ostaged = dfree + 1;    // math -> producer: the output tile is staged in X
     uint64_t *ofree = ostaged + 1;    // producer -> math: the output stores have read X
-    const int n_bars = 2 * NS + 6 + 12;
+    const int n_bars = 2 * NS + 6 + 14;
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + n_bars);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
     if (warp == 0 && lane == 0) prefetch_tensormap(&a.tmQ);
     if (warp == 2 && lane == 0) {
         prefetch_tensormap(&a.tmW);
+        prefetch_tensormap(&a.tmK);
         prefetch_tensormap(&a.tmV);
         prefetch_tensormap(&a.tmO);
     }
     if (tid == 0) {
         for (int i = 0; i < n_bars; ++i) mbar_init(&bars[i], 1);
         for (int i = 0; i < NS; ++i) mbar_init(&empty[i], 2);
-        mbar_init(xfull, 2);
-        mbar_init(phip, 8);
-        mbar_init(phim, 8);
-        mbar_init(pready, 8);
-        mbar_init(dfree, 8);
-        mbar_init(ostaged, 8);
-        mbar_init(&zempty[0], 8);
-        mbar_init(&zempty[1], 8);
+        mbar_init(xfree, 2);
+        mbar_init(uready, 2);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&phip[i], kMath);
+            mbar_init(&phim[i], kMath);
+        }
+        mbar_init(pready, kMath);
+        mbar_init(dfree, kMath);
+        mbar_init(ostaged, kMath);
+        mbar_init(&zempty[0], kMath);
+        mbar_init(&zempty[1], kMath);
         *fail = 0;
         fence_mbar_init();
     }
@@ -218,19 +226,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
     if (warp == 0) {
         // ------------------------------------------------------- state producer
         if (lane == 0) {
-            uint32_t q = 0, kp = 0;
-            int issued_slot[kMaxSlots];
-            int issued_z[2] = {0, 0};
-            for (int i = 0; i < kMaxSlots; ++i) issued_slot[i] = 0;
+            // q counts the ring items issued (slot q % NS, round robin) and nz the z
+            // loads (buffer nz % 2), so the copies in flight follow from the two counts
+            uint32_t q = 0, kp = 0, nz = 0;
             bool ok = true;
             void *nraw = state_raw(a, u_begin, u_end);
             for (int u = u_begin; u < u_end && ok; ++u) {
                 void *raw = nraw;
                 nraw = state_raw(a, u + 1, u_end);
-                float *Sg = state_at(a, raw, u);
-                if (!Sg) continue;
                 const int r = u / a.Hkv, g = u % a.Hkv;
-                // item 0: Q of the unit (the first thing g1 needs)
+                // item 0: Q of the unit (the first thing g1 needs), issued before the
+                // state pointer has arrived and been checked; a unit whose pointer
+                // fails the check passes its Q item through the ring unused
                 {
                     const int slot = q % NS;
                     if (!wait_bar(&empty[slot], ((q / NS) & 1u) ^ 1u, fail, wlim)) break;
@@ -238,14 +245,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                     for (int e = 0; e < d / 64; ++e)
                         tma_load_3d(ring + (size_t)slot * slot_bytes + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B,
                                     &full[slot]);
-                    ++issued_slot[slot];
                     ++q;
                 }
+                float *Sg = state_at(a, raw, u);
+                if (!Sg) continue;
                 const int zb = kp & 1;
                 if (!wait_bar(&zempty[zb], ((kp >> 1) & 1u) ^ 1u, fail, wlim)) break;
                 mbar_arrive_expect_tx(&zfull[zb], 2 * F * 4);
                 bulk_g2s(zbuf0 + zb * zstride, Sg + (size_t)2 * F * d, 2 * F * 4, &zfull[zb]);
-                ++issued_z[zb];
+                ++nz;
                 // items 1 .. F/32: phi+ tile c with phi- tile c
                 for (int c = 0; c < NCH; ++c, ++q) {
                     const int slot = q % NS;
@@ -254,15 +262,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                     mbar_arrive_expect_tx(&full[slot], slot_bytes);
                     bulk_g2s(dst, Sg + (size_t)c * 32 * d, chunk_bytes, &full[slot]);
                     bulk_g2s(dst + chunk_bytes, Sg + (size_t)(NCH + c) * 32 * d, chunk_bytes, &full[slot]);
-                    ++issued_slot[slot];
                 }
                 ++kp;
             }
             if (*fail) {
-                for (int s = 0; s < NS; ++s)
-                    if (issued_slot[s]) mbar_wait(&full[s], (uint32_t)(issued_slot[s] - 1) & 1u, kWaitNs);
-                for (int s = 0; s < 2; ++s)
-                    if (issued_z[s]) mbar_wait(&zfull[s], (uint32_t)(issued_z[s] - 1) & 1u, kWaitNs);
+                for (int s = 0; s < NS; ++s) {
+                    const uint32_t n = q / NS + ((uint32_t)s < q % NS ? 1u : 0u);
+                    if (n) mbar_wait(&full[s], (n - 1) & 1u, kWaitNs);
+                }
+                for (int s = 0; s < 2; ++s) {
+                    const uint32_t n = nz / 2 + ((uint32_t)s < nz % 2 ? 1u : 0u);
+                    if (n) mbar_wait(&zfull[s], (n - 1) & 1u, kWaitNs);
+                }
             }
         }
     } else if (warp == 1 || warp == 3) {
@@ -271,14 +282,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             const uint32_t iss = warp == 1 ? 0u : 1u;
             const uint32_t ring_u = smem_u32(ring);
             const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
-            // tiles of this issuer: ring positions iss, iss + 2, ... of each unit, into D+ or D-
+            // issuer A reads the phi+ tile of each pair slot (its first half) into D+,
+            // issuer B the phi- tile (second half) into D-
             const uint32_t acol0 = iss ? cM : cU, dcol = iss ? cDm : cDp;
-            // this issuer's tile of each pair item of the unit whose items start at qb
-            auto readout_half = [&](uint32_t qb) -> bool {
+            // both issuers read every ring item in order (Q for g1, then the pairs)
+            uint32_t rs = 0, rph = 0;   // ring slot and phase of the next item this issuer reads
+            auto next_item = [&]() { if (++rs == (uint32_t)NS) { rs = 0; rph ^= 1u; } };
+            auto readout_half = [&](uint64_t *phi_rel, uint32_t par) -> bool {
                 for (int c = 0; c < NCH; ++c) {
-                    const uint32_t qc = qb + 1 + c;
-                    const int slot = (int)(qc % (uint32_t)NS);
-                    if (!wait_bar(&full[slot], (qc / NS) & 1u, fail, wlim)) return false;
+                    // chunks 2 and 3 are written in the math warps' second pass
+                    if (c == 2 && !wait_bar(&phi_rel[1], par, fail, wlim)) return false;
+                    const int slot = (int)rs;
+                    if (!wait_bar(&full[slot], rph, fail, wlim)) return false;
+                    next_item();
                     tc_fence_after();
                     const uint64_t b0 =
                         smem_desc(ring_u + (uint32_t)slot * slot_bytes + iss * chunk_bytes, 16, 1024, SWZ_128B);
@@ -289,37 +305,54 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                 }
                 return true;
             };
-            uint32_t kp = 0, qt = 0;
-            if (iss == 0) {
-                const uint32_t wk_u = smem_u32(smem + a.off_wk),
-                               vb_u = smem_u32(smem + a.off_vb), p_u = smem_u32(smem + a.off_p);
-                const uint32_t idUS = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F + B);
-                const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
-                void *nraw = state_raw(a, u_begin, u_end);
-                for (int u = u_begin; u < u_end; ++u) {
-                    void *raw = nraw;
-                    nraw = state_raw(a, u + 1, u_end);
-                    if (!state_at(a, raw, u)) continue;
-                    if (!wait_bar(xfull, kp & 1u, fail, wlim)) break;
-                    // g1 writes [U | scores] over the previous unit's phi+ (read by this
-                    // thread's own earlier MMAs, in issue order) and phi- (read by issuer B)
-                    if (kp >= 1 && !wait_bar(dmdone, (kp - 1) & 1u, fail, wlim)) break;
-                    const int qs = (int)(qt % (uint32_t)NS);
-                    if (!wait_bar(&full[qs], (qt / NS) & 1u, fail, wlim)) break;
-                    const uint32_t q_u = ring_u + (uint32_t)qs * slot_bytes;
-                    tc_fence_after();
-                    for (int k = 0; k < d / 16; ++k) {
-                        const uint64_t aq = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
-                        const uint64_t bwk = smem_desc(wk_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
-                        mma_bf16_ss(tmem + cU, aq, bwk, idUS, k > 0);
-                    }
-                    mma_commit(uready);
-                    mma_commit(xfree);
-                    mma_commit(&empty[qs]);
-                    if (!wait_bar(phip, kp & 1u, fail, wlim)) break;
-                    // D+ is written from the first phi+ MMA on: the previous epilogue has read it
-                    if (kp >= 1 && !wait_bar(dfree, (kp - 1) & 1u, fail, wlim)) break;
-                    if (!readout_half(qt)) break;
+            uint32_t kp = 0, kx = 0;   // processed units, all units
+            const uint32_t wk_u = smem_u32(smem + a.off_wk);
+            const uint32_t k_u = wk_u + (uint32_t)(F / 64) * d * 128;   // K: d/64 atoms of B rows
+            // g1 of a unit: U = Q W (issuer A, W as the MN-major operand) and the
+            // scores Q K^T (issuer B) at once.  Each overwrites only columns that its
+            // own issuer's earlier readout MMAs read (phi+ under U, phi- under the
+            // scores), which run in issue order.
+            const uint32_t idG = iss ? instr_desc(FMT_BF16, FMT_BF16, false, false, 128, B)
+                                     : instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
+            const uint32_t gcol = iss ? cM : cU;
+            auto g1 = [&](uint32_t q_u) {
+                for (int k = 0; k < d / 16; ++k) {
+                    const uint64_t aq = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
+                    const uint64_t bo = iss ? smem_desc(k_u + (k >> 2) * (B * 128) + (k & 3) * 32, 16, 1024, SWZ_128B)
+                                            : smem_desc(wk_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
+                    mma_bf16_ss(tmem + gcol, aq, bo, idG, k > 0);
+                }
+            };
+            const uint32_t vb_u = smem_u32(smem + a.off_vb), p_u = smem_u32(smem + a.off_p);
+            const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
+            void *nraw = state_raw(a, u_begin, u_end);
+            for (int u = u_begin; u < u_end; ++u) {
+                void *raw = nraw;
+                nraw = state_raw(a, u + 1, u_end);
+                // W, K and Q of every unit are loaded before its state pointer is checked
+                if (!wait_bar(xfull, kx & 1u, fail, wlim)) break;
+                ++kx;
+                const int qs = (int)rs;
+                if (!wait_bar(&full[qs], rph, fail, wlim)) break;
+                next_item();
+                if (!state_at(a, raw, u)) {
+                    // skipped unit: release its W, K and Q unread
+                    mbar_arrive(xfree);
+                    mbar_arrive(&empty[qs]);
+                    continue;
+                }
+                tc_fence_after();
+                g1(ring_u + (uint32_t)qs * slot_bytes);
+                mma_commit(uready);
+                mma_commit(xfree);
+                mma_commit(&empty[qs]);
+                uint64_t *phi_rel = iss ? phim : phip;   // this issuer's half of phi, [2]
+                if (!wait_bar(&phi_rel[0], kp & 1u, fail, wlim)) break;
+                // D+ and D- are written from the first readout MMA on: the previous
+                // epilogue has read them
+                if (kp >= 1 && !wait_bar(dfree, (kp - 1) & 1u, fail, wlim)) break;
+                if (!readout_half(phi_rel, kp & 1u)) break;
+                if (iss == 0) {
                     if (!wait_bar(pready, kp & 1u, fail, wlim) || !wait_bar(vfull, kp & 1u, fail, wlim)) break;
                     tc_fence_after();
                     for (int k = 0; k < B / 16; ++k) {
@@ -328,27 +361,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                         mma_bf16_ss(tmem + cDp, ap, bv, idP, 1);
                     }
                     mma_commit(dpdone);
-                    qt += NI;
-                    ++kp;
-                }
-            } else {
-                void *nraw = state_raw(a, u_begin, u_end);
-                for (int u = u_begin; u < u_end; ++u) {
-                    void *raw = nraw;
-                    nraw = state_raw(a, u + 1, u_end);
-                    if (!state_at(a, raw, u)) continue;
-                    // the unit's Q item is read by issuer A alone: this thread's share of
-                    // its release, once it has landed
-                    const int qs = (int)(qt % (uint32_t)NS);
-                    if (!wait_bar(&full[qs], (qt / NS) & 1u, fail, wlim)) break;
-                    mbar_arrive(&empty[qs]);
-                    if (!wait_bar(phim, kp & 1u, fail, wlim)) break;
-                    if (kp >= 1 && !wait_bar(dfree, (kp - 1) & 1u, fail, wlim)) break;
-                    if (!readout_half(qt)) break;
+                } else {
                     mma_commit(dmdone);
-                    qt += NI;
-                    ++kp;
                 }
+                ++kp;
             }
             mma_commit(&mmadone[iss]);
             mbar_wait(&mmadone[iss], 0, kWaitNs);
@@ -357,30 +373,27 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
         // ------------------------------------------------------------- producer
         uint32_t kp = 0;
         int nx = 0, nv = 0;
-        const uint32_t xbytes = (uint32_t)(F / 64) * (d * 128);
-        uint8_t *kt = smem + a.off_wk + (F / 64) * d * 128;
+        const uint32_t xbytes = (uint32_t)(F / 64) * (d * 128) + (uint32_t)(d / 64) * (B * 128);
+        uint8_t *kb = smem + a.off_wk + (F / 64) * d * 128;
         int pr = 0, pg = 0;             // request and head of the previous unit
         void *nraw = state_raw(a, u_begin, u_end);
         for (int u = u_begin; u < u_end; ++u) {
             void *raw = nraw;
             nraw = state_raw(a, u + 1, u_end);
-            if (!state_at(a, raw, u)) continue;
             const int r = u / a.Hkv, g = u % a.Hkv;
-            KtRegs kr;
-            kt_load(a.K, (size_t)r * B, B, a.Hkv, g, d, kr, lane);   // in flight while the region drains
+            // W and K of every unit go out before its state pointer is checked
             bool ok = true;
-            if (kp > 0) ok = wait_bar(xfree, (kp - 1) & 1u, fail, wlim);
+            if (nx > 0) ok = wait_bar(xfree, (nx - 1) & 1u, fail, wlim);
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
                 mbar_arrive_expect_tx(xfull, xbytes);
                 for (int f = 0; f < F / 64; ++f)
                     tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xfull);
+                for (int e = 0; e < d / 64; ++e)
+                    tma_load_3d(kb + e * (B * 128), &a.tmK, 64 * e, g, r * B, xfull);
             }
-            kt_store(kr, d, kt, lane);
-            fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(xfull);
             ++nx;
+            if (!state_at(a, raw, u)) continue;
             // the previous unit's output tile (staged in X over its V and P') goes out
             // by TMA stores; once they have read X, this unit's V may land there
             if (kp > 0) {
@@ -426,15 +439,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
         const int row = 32 * q4 + lane;
         const uint32_t lane_off = (uint32_t)(32 * q4) << 16;
         const bool two = NCH >= 4;          // a part owns chunks part and part + 2 of each half
-        const bool has_sc = part < B / 16;  // score columns [16 part, 16 part + 16)
+        const int nsc = B / SC;             // parts holding scores
+        const bool has_sc = part < nsc;     // score columns [SC part, SC part + SC)
         const int Mv = G * B;
         const bool valid = row < Mv;
-        float *xa = reinterpret_cast<float *>(smem + a.off_st);   // [part][ms, mx, mn][128]
-        float *xb = xa + 6 * 128;                                  // [part][sp, lp, sn, ln, l][128]
+        // row statistics: X(k, p) is statistic k of this row from part p, one
+        // [P][128] array per statistic
+        enum { kMs, kL, kMx, kMn, kSp, kLp, kSn, kLn };
+        float *xrow = reinterpret_cast<float *>(smem + a.off_st) + row;
+        auto X = [&](int k, int p) -> float & { return xrow[(k * P + p) * 128]; };
         const float scale_l2 = a.scale * kLog2e;
         const uint32_t pair_bar = kBarPair + q4;
         const float log_f = logf((float)F);
-        auto pair_failed = [&](bool local_fail) -> bool { return group_sync_failed(pair_bar, 64, local_fail); };
+        auto pair_failed = [&](bool local_fail) -> bool { return group_sync_failed(pair_bar, 32 * P, local_fail); };
 
         uint32_t kp = 0;
         void *nraw = state_raw(a, u_begin, u_end);
@@ -456,16 +473,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             // ---- phase A: row extrema of U and of the scores (U kept in registers)
             bool bad = !wait_bar(uready, kp & 1u, fail, wlim);
             tc_fence_after();
-            float sc[16], u0[32], u1[32];
+            float sc[SC], u0[32], u1[32];
             if (has_sc) tmem_ld16(mcol + 16 * part, sc);
             tmem_ld32(ucol + 32 * part, u0);
-            if (two) tmem_ld32(ucol + 32 * (part + 2), u1);
+            if (two) tmem_ld32(ucol + 32 * (part + P), u1);
             tmem_wait_ld();
             {
                 float ms = -INFINITY, mx = -INFINITY, mn = INFINITY;
                 if (has_sc) {
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) ms = fmaxf(ms, sc[i]);
+                    for (int i = 0; i < SC; ++i) ms = fmaxf(ms, sc[i]);
                 }
 #pragma unroll
                 for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, u0[i]); mn = fminf(mn, u0[i]); }
@@ -473,15 +490,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
 #pragma unroll
                     for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, u1[i]); mn = fminf(mn, u1[i]); }
                 }
-                xa[(part * 3 + 0) * 128 + row] = ms;
-                xa[(part * 3 + 1) * 128 + row] = mx;
-                xa[(part * 3 + 2) * 128 + row] = mn;
+                if (has_sc) X(kMs, part) = ms;
+                X(kMx, part) = mx;
+                X(kMn, part) = mn;
             }
-            // both parts have read their scores: phi- may overwrite the score columns
+            // every part has read its scores: phi- may overwrite the score columns
             if (pair_failed(bad)) break;
-            const float ms = fmaxf(xa[0 * 128 + row], xa[3 * 128 + row]);
-            const float mx = fmaxf(xa[1 * 128 + row], xa[4 * 128 + row]);
-            const float mn = fminf(xa[2 * 128 + row], xa[5 * 128 + row]);
+            float ms = X(kMs, 0), mx = X(kMx, 0), mn = X(kMn, 0);
+            for (int p = 1; p < nsc; ++p) ms = fmaxf(ms, X(kMs, p));
+#pragma unroll
+            for (int p = 1; p < P; ++p) {
+                mx = fmaxf(mx, X(kMx, p));
+                mn = fminf(mn, X(kMn, p));
+            }
             const float lw = valid ? log_sigmoid(alpha_row) : 0.f;
             // fast: w sp e^(max s) <= w F e^(max s) stays below e^60 for every row of the
             // warp, so phi+ and phi- are released unnormalised as soon as they are written
@@ -493,22 +514,25 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             const float mxl = mx * kLog2e, mnl = mn * kLog2e, ml = ms * scale_l2;
             float sp = 0.f, lp = 0.f, sn = 0.f, ln = 0.f, l = 0.f;
             auto expp = [&](const float (&uu)[32], int k) {
-                float ep[32];
                 const float4 *zp = reinterpret_cast<const float4 *>(zs + 32 * k);
 #pragma unroll
-                for (int i4 = 0; i4 < 8; ++i4) {
-                    const float4 z4 = zp[i4];
-                    const float za[4] = {z4.x, z4.y, z4.z, z4.w};
+                for (int h = 0; h < 2; ++h) {
+                    float ep[16];
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const int i = 4 * i4 + j;
-                        const float e = ex2(fmaf(uu[i], kLog2e, -mxl));
-                        ep[i] = e;
-                        sp += e;
-                        lp = fmaf(e, za[j], lp);
+                    for (int i4 = 0; i4 < 4; ++i4) {
+                        const float4 z4 = zp[4 * h + i4];
+                        const float za[4] = {z4.x, z4.y, z4.z, z4.w};
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const int i = 4 * i4 + j;
+                            const float e = ex2(fmaf(uu[16 * h + i], kLog2e, -mxl));
+                            ep[i] = e;
+                            sp += e;
+                            lp = fmaf(e, za[j], lp);
+                        }
                     }
+                    tmem_st16(ucol + 32 * k + 16 * h, ep);
                 }
-                tmem_st32(ucol + 32 * k, ep);
             };
             auto expm = [&](float (&uu)[32], int k) {
                 const float4 *zn = reinterpret_cast<const float4 *>(zs + F + 32 * k);
@@ -531,48 +555,64 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                 tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0 && !bad && !(a.withhold && bar == phip)) mbar_arrive(bar);
+                if (lane == 0 && !bad && !(a.withhold && (bar == &phip[0] || bar == &phip[1]))) mbar_arrive(bar);
             };
+            // chunk part of phi+ and of phi-, then chunk part + 2 of each, each
+            // released as soon as it is written
             expp(u0, part);
-            if (two) expp(u1, part + 2);
-            if (fast) release(phip);
+            if (fast) release(&phip[0]);
             expm(u0, part);
-            if (two) expm(u1, part + 2);
-            if (fast) release(phim);
+            if (fast) release(&phim[0]);
+            if (two) {
+                expp(u1, part + P);
+                if (fast) release(&phip[1]);
+                expm(u1, part + P);
+                if (fast) release(&phim[1]);
+            }
             if (has_sc) {
 #pragma unroll
-                for (int i = 0; i < 16; ++i) l += ex2(fmaf(sc[i], scale_l2, -ml));
+                for (int i = 0; i < SC; ++i) l += ex2(fmaf(sc[i], scale_l2, -ml));
             }
-            xb[(part * 5 + 0) * 128 + row] = sp;
-            xb[(part * 5 + 1) * 128 + row] = lp;
-            xb[(part * 5 + 2) * 128 + row] = sn;
-            xb[(part * 5 + 3) * 128 + row] = ln;
-            xb[(part * 5 + 4) * 128 + row] = l;
+            X(kSp, part) = sp;
+            X(kLp, part) = lp;
+            X(kSn, part) = sn;
+            X(kLn, part) = ln;
+            if (has_sc) X(kL, part) = l;
             // z has been read
             __syncwarp();
             if (lane == 0 && !bad) mbar_arrive(&zempty[zb]);
             if (pair_failed(bad)) break;
 
             // ---- phase C: sigma, den, P' (and off the fast path the rescale of phi)
-            sp = xb[0 * 128 + row] + xb[5 * 128 + row];
-            lp = xb[1 * 128 + row] + xb[6 * 128 + row];
-            sn = xb[2 * 128 + row] + xb[7 * 128 + row];
-            ln = xb[3 * 128 + row] + xb[8 * 128 + row];
-            l = xb[4 * 128 + row] + xb[9 * 128 + row];
-            const float lin_den = lp / sp + ln / sn;
-            const float log_s = lw + ms * a.scale + logf(l);   // log(w sm_den)
-            const float log_l = logf(lin_den);                   // log(lin_den), -inf if empty
+            sp = X(kSp, 0);
+            lp = X(kLp, 0);
+            sn = X(kSn, 0);
+            ln = X(kLn, 0);
+#pragma unroll
+            for (int p = 1; p < P; ++p) {
+                sp += X(kSp, p);
+                lp += X(kLp, p);
+                sn += X(kSn, p);
+                ln += X(kLn, p);
+            }
+            l = X(kL, 0);
+            for (int p = 1; p < nsc; ++p) l += X(kL, p);
+            // (approximate intrinsics: the result is rounded to bf16)
+            const float rsp = __fdividef(1.f, sp), rsn = __fdividef(1.f, sn);
+            const float lin_den = lp * rsp + ln * rsn;
+            const float log_s = lw + ms * a.scale + __logf(l);   // log(w sm_den)
+            const float log_l = __logf(lin_den);                   // log(lin_den), -inf if empty
             const float sig = fmaxf(fmaxf(log_s, log_l), -60.f);
-            const float esig = expf(-sig);
-            const float inv_den = 1.f / (expf(log_l - sig) + expf(log_s - sig));
+            const float esig = __expf(-sig);
+            const float inv_den = __fdividef(1.f, __expf(log_l - sig) + __expf(log_s - sig));
             float ap, am, pofs;
             if (fast) {
-                ap = esig / sp * inv_den;
-                am = esig / sn * inv_den;
-                pofs = (lw + logf(sp)) * kLog2e;
+                ap = esig * rsp * inv_den;
+                am = esig * rsn * inv_den;
+                pofs = lw * kLog2e + __log2f(sp);
             } else {
-                const float cpos = lin_den > 0.f ? esig / sp : 0.f;
-                const float cneg = lin_den > 0.f ? esig / sn : 0.f;
+                const float cpos = lin_den > 0.f ? esig * rsp : 0.f;
+                const float cneg = lin_den > 0.f ? esig * rsn : 0.f;
                 auto scale_chunk = [&](uint32_t col, float c) {
                     float v[32];
                     tmem_ld32(col, v);
@@ -582,11 +622,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                     tmem_st32(col, v);
                 };
                 scale_chunk(ucol + 32 * part, cpos);
-                if (two) scale_chunk(ucol + 32 * (part + 2), cpos);
-                release(phip);
+                if (two) scale_chunk(ucol + 32 * (part + P), cpos);
+                release(&phip[0]);
+                if (two) release(&phip[1]);
                 scale_chunk(mcol + 32 * part, cneg);
-                if (two) scale_chunk(mcol + 32 * (part + 2), cneg);
-                release(phim);
+                if (two) scale_chunk(mcol + 32 * (part + P), cneg);
+                release(&phim[0]);
+                if (two) release(&phim[1]);
                 ap = inv_den;
                 am = inv_den;
                 pofs = (lw - sig) * kLog2e;
@@ -596,13 +638,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             if (has_sc) {
                 // P' (w sp e^s on the fast path, w e^(s - sigma) off it): K-major, no
                 // swizzle (8-row x 16-byte core matrices).
-                uint32_t pk[8];
+                uint32_t pk[SC / 2];
 #pragma unroll
-                for (int i = 0; i < 16; i += 2)
+                for (int i = 0; i < SC; i += 2)
                     pk[i / 2] = pack_bf16x2(ex2(fmaf(sc[i], scale_l2, pofs)), ex2(fmaf(sc[i + 1], scale_l2, pofs)));
-                uint8_t *prow = smem + a.off_p + (row >> 3) * (B / 8) * 128 + (row & 7) * 16;
-                *reinterpret_cast<uint4 *>(prow + (2 * part) * 128) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-                *reinterpret_cast<uint4 *>(prow + (2 * part + 1) * 128) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+                // core matrix j holds the columns [8j, 8j + 8) of the row's 8-row group
+                uint8_t *prow = smem + a.off_p + (row >> 3) * (B / 8) * 128 + (row & 7) * 16 + (SC / 8) * part * 128;
+#pragma unroll
+                for (int j = 0; j < SC / 8; ++j)
+                    *reinterpret_cast<uint4 *>(prow + j * 128) =
+                        make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
             }
             fence_proxy_async_smem();
             __syncwarp();
@@ -615,7 +660,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             bad = !wait_bar(dmdone, kp & 1u, fail, wlim) || bad;
             tc_fence_after();
             {
-                const int dh = d / 2;
+                const int dh = d / P;   // output columns of this part
 #pragma unroll 1
                 for (int hc = 0; hc < dh / 32; ++hc) {
                     float vp[32], vm[32];
@@ -698,11 +743,11 @@ cudaError_t launch_step(const hybrid_cfg &c, const void *Q, const void *K, const
         const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
         const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
         const cuuint32_t bw[2] = {64, (cuuint32_t)d};
-        if (!encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !encode_bf16(&a.tmV, V, 3, dv, sv, bv) ||
-            !encode_bf16(&a.tmW, W, 2, dw, sw, bw) || !encode_bf16(&a.tmO, O, 3, dq, sq, bq))
+        if (!encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !encode_bf16(&a.tmK, K, 3, dv, sv, bv) ||
+            !encode_bf16(&a.tmV, V, 3, dv, sv, bv) || !encode_bf16(&a.tmW, W, 2, dw, sw, bw) ||
+            !encode_bf16(&a.tmO, O, 3, dq, sq, bq))
             return cudaErrorInvalidValue;
     }
-    a.K = static_cast<const bf16 *>(K);
     a.O = static_cast<bf16 *>(O);
     a.alpha = alpha;
     a.states = states;
