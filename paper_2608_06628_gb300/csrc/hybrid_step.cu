@@ -470,6 +470,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             const float *zs = zbuf0 + zb * zstride;
             const uint32_t ucol = tmem + cU + lane_off, mcol = tmem + cM + lane_off;
 
+            // log w of the row's gate, formed while g1 runs
+            const float lw = valid ? log_sigmoid(alpha_row) : 0.f;
             // ---- phase A: row extrema of U and of the scores (U kept in registers)
             bool bad = !wait_bar(uready, kp & 1u, fail, wlim);
             tc_fence_after();
@@ -503,7 +505,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                 mx = fmaxf(mx, X(kMx, p));
                 mn = fminf(mn, X(kMn, p));
             }
-            const float lw = valid ? log_sigmoid(alpha_row) : 0.f;
             // fast: w sp e^(max s) <= w F e^(max s) stays below e^60 for every row of the
             // warp, so phi+ and phi- are released unnormalised as soon as they are written
             const bool fast = __all_sync(0xffffffffu, !(lw + ms * a.scale + log_f > 60.f));
@@ -571,7 +572,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             }
             if (has_sc) {
 #pragma unroll
-                for (int i = 0; i < SC; ++i) l += ex2(fmaf(sc[i], scale_l2, -ml));
+                for (int i = 0; i < SC; ++i) {
+                    sc[i] = ex2(fmaf(sc[i], scale_l2, -ml));   // e^(s - max s), kept for P'
+                    l += sc[i];
+                }
             }
             X(kSp, part) = sp;
             X(kLp, part) = lp;
@@ -638,10 +642,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             if (has_sc) {
                 // P' (w sp e^s on the fast path, w e^(s - sigma) off it): K-major, no
                 // swizzle (8-row x 16-byte core matrices).
+                const float pf = ex2(pofs + ml);   // P' = e^(s - max s) 2^(pofs + max s log2 e)
                 uint32_t pk[SC / 2];
 #pragma unroll
-                for (int i = 0; i < SC; i += 2)
-                    pk[i / 2] = pack_bf16x2(ex2(fmaf(sc[i], scale_l2, pofs)), ex2(fmaf(sc[i + 1], scale_l2, pofs)));
+                for (int i = 0; i < SC; i += 2) pk[i / 2] = pack_bf16x2(sc[i] * pf, sc[i + 1] * pf);
                 // core matrix j holds the columns [8j, 8j + 8) of the row's 8-row group
                 uint8_t *prow = smem + a.off_p + (row >> 3) * (B / 8) * 128 + (row & 7) * 16 + (SC / 8) * part * 128;
 #pragma unroll
