@@ -157,8 +157,8 @@ hybrid_status hybrid_block_attn_commit(const hybrid_cfg *cfg, const void *Q, con
         return HYBRID_ERR_INVALID_ARG;
     unsigned *err = error_word();
     if (!err) return HYBRID_ERR_CUDA;
-    if (hyb::fused_supported(*cfg, true))
-        return from_cuda(hyb::launch_fused(*cfg, true, Q, K, V, W, alpha, d_state_ptrs, n_req, O, err, stream));
+    if (hyb::fused_supported(*cfg))
+        return from_cuda(hyb::launch_fused(*cfg, Q, K, V, W, alpha, d_state_ptrs, n_req, O, err, stream));
     // other shapes: the step, then the commit, on the same stream
     s = hybrid_block_attn(cfg, Q, K, V, W, alpha, d_state_ptrs, n_req, O, stream);
     if (s != HYBRID_OK) return s;

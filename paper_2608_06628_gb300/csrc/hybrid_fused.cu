@@ -1,12 +1,12 @@
-// hybrid_fused.cu -- persistent, warp-specialised block-hybrid step on the
-// tcgen05 tensor cores, optionally fused with the block commit.
+// hybrid_fused.cu -- persistent, warp-specialised block-hybrid step fused with
+// the block commit, on the tcgen05 tensor cores.
 //
 // Section 3.1 of "Retrofitting Linear Attention into Diffusion Language
 // Models" defines the step (in-block softmax, linear readout from the committed
 // state, gated shared-normaliser merge) and the state update; its serving
-// section computes both in one kernel launch, which kCommit = true does here:
-// every state tile is read once, used for the readout with the pre-commit
-// state, updated with this block's phi(k) v^T and written back.
+// section computes both in one kernel launch, as this kernel does: every state
+// tile is read once, used for the readout with the pre-commit state, and
+// updated with this block's phi(k) v^T.
 //
 // Work unit = (request r, state head g): the G*B query rows of the unit share
 // one state.  One CTA per SM loops over a contiguous range of units.  Warp
@@ -16,18 +16,17 @@
 //              operand image, see hybrid.h).
 //   warp 1     MMA issuer (one thread); owns the Tensor Memory allocation.
 //   warp 2     producer: TMA of Q and W, the transposed key tile K^T (built by
-//              the warp from global memory) and V, one unit ahead.
-//   warp 3     storer (commit): bulk reduce-adds of the dS^T tiles into the state,
-//              the store of z, and TMA stores of the output tile (the step's math
-//              warps store the output from registers).
+//              the warp from global memory) and V.
+//   warp 3     storer: bulk reduce-adds of the dS^T tiles into the state, the
+//              store of z, and TMA stores of the output tile.
 //   warps 4-11 math: two threads per query row (one per TMEM lane and "part");
 //              a part owns every other 32-feature chunk of each half of phi.
 //
 // Per unit the tensor cores run, in this order,
 //   g1   [U | scores] = Q [W | K^T]  (one N = F + B product; U = Q W)
-//        and, with the commit, U_k^T = W^T K^T (phi of the block's keys)
+//        and U_k^T = W^T K^T (phi of the block's keys)
 //   R+   D  = phi+'(Q) S+             (tf32, A operand in Tensor Memory)
-//   dS   dS^T = V^T phi(K)^T per feature half (commit; bf16 from the TMA'd V)
+//   dS   dS^T = V^T phi(K)^T per feature half (bf16 from the TMA'd V)
 //   PV   D += P' V                    (P' = w e^(s - sigma), bf16)
 //   R-   D += phi-'(Q) S-
 // The math warps publish phi+ as soon as its exponentials are in Tensor
@@ -41,15 +40,13 @@
 // kernel accumulates D / kappa (kappa = e^-sigma / sp) instead, so phi+ needs
 // no rescaling in Tensor Memory; kappa is folded into 1 / den.
 //
-// A unit's phi+ and phi- share its F phi columns: phi- waits in registers until
-// R+ has consumed phi+.  Step: Tensor Memory holds two unit slots of 256
-// columns, [phi | D] each, so the next unit's g1 runs between this unit's R+
-// and R- and its feature map overlaps R-.  Commit: [D | phi | dS+ | dS-]; once
-// a half's tiles have been read out, their ring slots take that half's dS^T
-// rows and the storer adds them into the state in global memory by bulk
-// reduce-adds (the float32 add happens at L2), so the SM never writes a state
-// tile back.  V, P' and phi(K) share the Q region once g1 has consumed Q, so
-// all 2F/32 state tiles of a unit fit in the ring.
+// Tensor Memory: [D | phi | dS+ | dS-].  phi+ is parked in the dS- columns
+// while R+ reads it; phi- replaces U in the phi columns.  Once a half's tiles
+// have been read out, their ring slots take that half's dS^T rows and the
+// storer adds them into the state in global memory by bulk reduce-adds (the
+// float32 add happens at L2), so the SM never writes a state tile back.  V, P'
+// and phi(K) share the Q region once g1 has consumed Q, so all 2F/32 state
+// tiles of a unit fit in the ring.
 //
 // MMA cost note: on this part a tcgen05.mma with M = 128 costs about the same
 // time for any N up to 128-256, so contractions are shaped for few, wide
@@ -77,7 +74,6 @@ constexpr int kMaxSlots = 16;
 constexpr int kSmemLimit = 232448;
 constexpr int kOneCtaPerSm = 118 * 1024;
 constexpr uint32_t kBarMath = 1;      // named barrier over the 256 math threads
-constexpr uint32_t kBarPair = 2;      // 2..5: the two math warps of one TMEM lane quarter
 constexpr uint32_t kStatBytes = 14 * 1024;
 // Tensor Memory columns with the commit (F <= 128, d <= 128)
 constexpr uint32_t kCmD = 0, kCmP = 128, kCmDSp = 256, kCmK = 288, kCmDSm = 384;
@@ -88,14 +84,11 @@ constexpr uint32_t kCmEK = 320;
 struct FusedArgs {
     CUtensorMap tmQ, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
     const bf16 *K;
-    bf16 *O;                          // step: the output is stored from registers
     const float *alpha;
     void *const *states;
     unsigned *err;
     int n_units, B, Hq, Hkv, G, d, F, NS;
     float scale;
-    unsigned long long wait_ns;       // limit of every bounded wait (1 s unless a test armed less)
-    int withhold;                     // test hook: the math warps never signal phip
     uint32_t off_q, off_wk, off_vb, off_p, off_pk, off_z, off_st, off_bar;
 };
 
@@ -110,7 +103,7 @@ struct FLayout {
     int NS;
 };
 
-FLayout make_flayout(int d, int F, int B, bool commit)
+FLayout make_flayout(int d, int F, int B)
 {
     FLayout L{};
     const uint32_t chunk = (uint32_t)d * 128;
@@ -119,11 +112,11 @@ FLayout make_flayout(int d, int F, int B, bool commit)
     const uint32_t wk = (uint32_t)(F / 64 + 1) * d * 128;
     const uint32_t vb = (((uint32_t)B * d * 2) + 1023) & ~1023u;
     const uint32_t p = (((uint32_t)128 * B * 2) + 1023) & ~1023u;
-    const uint32_t pk = commit ? ((((uint32_t)(2 * F / 64) * B * 128) + 1023) & ~1023u) : 0u;
+    const uint32_t pk = (((uint32_t)(2 * F / 64) * B * 128) + 1023) & ~1023u;
     const uint32_t bar = 1024;
-    // with the commit, V, P' and phi(K) live in the Q region once g1 has read Q
-    // (the next unit's Q is loaded after the unit's dS^T and P V are done)
-    const bool overlay = commit && vb + p + pk <= q;
+    // V, P' and phi(K) live in the Q region once g1 has read Q (the next unit's
+    // Q is loaded after the unit's dS^T and P V are done)
+    const bool overlay = vb + p + pk <= q;
     const uint32_t fixed = q + wk + (overlay ? 0u : vb + p + pk) + 2 * zb + kStatBytes + bar + 1024;
     int ns = ((int)kSmemLimit - (int)fixed) / (int)chunk;
     if (ns > kMaxSlots) ns = kMaxSlots;
@@ -162,7 +155,6 @@ __device__ __forceinline__ float *state_at(const FusedArgs &a, void *raw, int u)
     return st + (size_t)(u % a.Hkv) * head_floats(a.d, a.F);
 }
 
-template <bool kCommit>
 __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ FusedArgs a)
 {
     using namespace ptx;
@@ -170,14 +162,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int d = a.d, F = a.F, B = a.B, G = a.G, NS = a.NS;
-    const uint64_t wlim = a.wait_ns;
+    const uint64_t wlim = kWaitNs;
     const int NCH = F / 32;          // 32-feature chunks (state tiles) per half of phi
     const int NC = 2 * NCH;          // state tiles per unit
-    // with the commit the output tile is staged in the slots of tiles ocm, ocm + 1
-    // of its unit: the first two second-half tiles (their increments are
-    // reduce-added before the epilogue), so the next unit's first-half tiles,
-    // needed first, can enter the ring early; if a unit has more tiles than the
-    // ring, first-half tiles that no later tile of the unit reuses
+    // the output tile is staged in the slots of tiles ocm, ocm + 1 of its unit:
+    // the first two second-half tiles (their increments are reduce-added before
+    // the epilogue), so the next unit's first-half tiles, needed first, can enter
+    // the ring early; if a unit has more tiles than the ring, first-half tiles
+    // that no later tile of the unit reuses
     const int ocm = NC > NS ? NC - NS : NCH;
     const uint32_t chunk_bytes = (uint32_t)d * 128;
     const int per = a.n_units / (int)gridDim.x, rem = a.n_units % (int)gridDim.x;
@@ -190,32 +182,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint64_t *zfull = empty + NS;     // [2]
     uint64_t *zempty = zfull + 2;     // [2]
     uint64_t *dready = zempty + 2;    // [2] MMA -> math: the unit's output accumulator is complete
-    uint64_t *dfree = dready + 2;     // [2] math -> MMA: the output accumulator has been read
-    uint64_t *tready = dfree + 2;     // [2] math -> storer: a feature half of the tiles is updated
-    // Barriers of one unit's stages.  The step issues the MMAs of even and odd units
-    // from two threads (one per Tensor Memory slot), so it keeps these per slot:
-    // entry k & 1 with parity (k >> 1) & 1 for the unit of index k; the commit uses
-    // entry 0 with parity k & 1 (see SB, SP).
-    uint64_t *xfull = tready + 2;     // [2] Q, W (TMA) and K^T (producer warp) are in place
-    uint64_t *uready = xfull + 2;     // [2] MMA -> math: g1 done
-    uint64_t *phip = uready + 2;      // [2] math -> MMA: phi+ is in the phi columns
-    uint64_t *phim = phip + 2;        // [2] math -> MMA: phi- in the phi columns
-    uint64_t *pread = phim + 2;       // [2] MMA -> math: R+ has consumed phi+
-    uint64_t *pready = pread + 2;     // [2] math -> MMA: P' is written
-    uint64_t *mmadone = pready + 2;   // [2] per issuing thread: all of its MMAs have completed
-    uint64_t *xfree = mmadone + 2;
+    uint64_t *tready = dready + 2;    // [2] math -> storer: a feature half of the tiles is updated
+    uint64_t *xfull = tready + 2;     // Q, W (TMA) and K^T (producer warp) are in place
+    uint64_t *uready = xfull + 1;     // MMA -> math: g1 done
+    uint64_t *phip = uready + 1;      // math -> MMA: phi+ is in the dS- columns
+    uint64_t *phim = phip + 1;        // math -> MMA: phi- in the phi columns
+    uint64_t *pready = phim + 1;      // math -> MMA: P' is written
+    uint64_t *mmadone = pready + 1;   // the issuing thread's MMAs have completed
+    uint64_t *xfree = mmadone + 1;
     uint64_t *vfull = xfree + 1;
-    uint64_t *vfree = vfull + 1;
-    uint64_t *kready = vfree + 1;     // math -> MMA: phi(K) is written (commit)
-    uint64_t *dsdone = kready + 1;    // MMA -> math: dS^T is formed (commit)
-    uint64_t *pvdone = dsdone + 1;    // MMA -> producer: P V has read V and P' (commit)
-    uint64_t *efree = pvdone + 1;     // math -> MMA: the first-half update has read dS+ (commit)
-    uint64_t *zdone = efree + 1;      // math -> storer: z is updated (commit)
-    uint64_t *ofree = zdone + 1;      // storer -> math: the output slots may be written (commit)
+    uint64_t *kready = vfull + 1;     // math -> MMA: phi(K) is written
+    uint64_t *dsdone = kready + 1;    // MMA -> math: dS^T is formed
+    uint64_t *pvdone = dsdone + 1;    // MMA -> producer: P V has read V and P'
+    uint64_t *efree = pvdone + 1;     // math -> MMA: the first-half update has read dS+
+    uint64_t *zdone = efree + 1;      // math -> storer: z is updated
+    uint64_t *ofree = zdone + 1;      // storer -> math: the output slots may be written
     uint64_t *ostaged = ofree + 1;    // math -> storer: the output tile is in its slots
-    const int n_bars = 2 * NS + 10 + 14 + 10;
-    auto SB = [&](uint64_t *b, uint32_t k) -> uint64_t * { return kCommit ? b : b + (k & 1u); };
-    auto SP = [&](uint32_t k) -> uint32_t { return kCommit ? (k & 1u) : ((k >> 1) & 1u); };
+    const int n_bars = 2 * NS + 8 + 15;
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + n_bars);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
@@ -227,22 +210,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     if (warp == 3 && lane == 0) prefetch_tensormap(&a.tmO);
     if (tid == 0) {
         for (int i = 0; i < n_bars; ++i) mbar_init(&bars[i], 1);
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(&xfull[i], 2);
-            mbar_init(&phip[i], 8);
-            mbar_init(&phim[i], 8);
-            mbar_init(&pready[i], 8);
-            mbar_init(&dfree[i], 8);
-            mbar_init(&tready[i], 8);
-        }
+        mbar_init(xfull, 2);
+        mbar_init(phip, 8);
+        mbar_init(phim, 8);
+        mbar_init(pready, 8);
+        for (int i = 0; i < 2; ++i) mbar_init(&tready[i], 8);
         mbar_init(kready, 8);
         mbar_init(efree, 8);
         mbar_init(zdone, 8);
         mbar_init(ostaged, 8);
-        if (!kCommit) {
-            mbar_init(&zempty[0], 8);
-            mbar_init(&zempty[1], 8);
-        }
         *fail = 0;
         fence_mbar_init();
     }
@@ -298,14 +274,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     if (issued_z[s]) mbar_wait(&zfull[s], (uint32_t)(issued_z[s] - 1) & 1u, kWaitNs);
             }
         }
-    } else if (warp == 1 || (!kCommit && warp == 3)) {
-        // ------------------------------------------------------- MMA issuers
-        // commit: warp 1 issues every MMA.  Step: warp 1 issues the MMAs of the even
-        // units (Tensor Memory slot 0) and warp 3 those of the odd units (slot 1), so
-        // one unit's phi- readout runs beside the next unit's phi+ readout (an M = 128
-        // tf32 MMA keeps its issuing thread ~140 cycles, twice the tensor pipe's time).
+    } else if (warp == 1) {
+        // ------------------------------------------------------- MMA issuer
         if (lane == 0) {
-            const uint32_t iss = warp == 1 ? 0u : 1u;
             const uint32_t q_u = smem_u32(smem + a.off_q), wk_u = smem_u32(smem + a.off_wk),
                            vb_u = smem_u32(smem + a.off_vb), p_u = smem_u32(smem + a.off_p),
                            pk_u = smem_u32(smem + a.off_pk), ring_u = smem_u32(ring);
@@ -315,16 +286,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
             const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
             const uint32_t idDS = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, F);
-            // g1: [U | scores] at column ucol, and (commit) U_k^T at column kcol
+            // g1: [U | scores] at column ucol, and U_k^T at column kcol
             auto g1 = [&](uint32_t ucol, uint32_t kcol) {
                 for (int k = 0; k < d / 16; ++k) {
                     const uint64_t aq = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
                     const uint64_t bwk = smem_desc(wk_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
                     mma_bf16_ss(tmem + ucol, aq, bwk, idUS, k > 0);
-                    if (kCommit) {
-                        const uint64_t bkt = smem_desc(kt_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
-                        mma_bf16_ss(tmem + kcol, bwk, bkt, idKT, k > 0);
-                    }
+                    const uint64_t bkt = smem_desc(kt_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
+                    mma_bf16_ss(tmem + kcol, bwk, bkt, idKT, k > 0);
                 }
             };
             // P'V accumulates onto the phi+ readout
@@ -335,11 +304,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     mma_bf16_ss(tmem + dcol, ap, bv, idP, 1);
                 }
             };
-            // readout of state tile c (global tile counter qt + c) with phi columns acol
+            // readout of the next state tile in the ring with phi columns acol
             // (first: the tile's first MMA initialises the accumulator)
-            auto readout = [&](uint32_t dcol, uint32_t acol, uint32_t qc, bool first = false) -> int {
-                const int slot = qc % NS;
-                if (!wait_bar(&full[slot], (qc / NS) & 1u, fail, wlim)) return -1;
+            uint32_t rs = 0, rph = 0;   // ring slot and phase of the next tile, read in ring order
+            auto readout = [&](uint32_t dcol, uint32_t acol, bool first = false) -> int {
+                const int slot = (int)rs;
+                if (!wait_bar(&full[slot], rph, fail, wlim)) return -1;
+                if (++rs == (uint32_t)NS) { rs = 0; rph ^= 1u; }
                 tc_fence_after();
                 const uint32_t s_u = ring_u + slot * chunk_bytes;
 #pragma unroll
@@ -356,98 +327,44 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     mma_bf16_ss(tmem + dcol, av, bp, idDS, ks > 0);
                 }
             };
-            uint32_t kp = 0, qt = 0;
+            uint32_t kp = 0;
             bool ok = true;
-            if (!kCommit) {
-                // this thread's units: g1, R+ once phi+ is written, P'V, R- once phi- is
-                // written, all into its slot's [phi | D] columns
-                const uint32_t T = iss * 256;
-                void *nraw = state_raw(a, u_begin, u_end);
-                for (int u = u_begin; u < u_end; ++u) {
-                    void *raw = nraw;
-                    nraw = state_raw(a, u + 1, u_end);
-                    if (!state_at(a, raw, u)) continue;
-                    if ((kp & 1u) == iss) {
-                        if (!wait_bar(SB(xfull, kp), SP(kp), fail, wlim)) { ok = false; break; }
-                        if (kp >= 2 && !wait_bar(&dfree[iss], ((kp - 2) >> 1) & 1u, fail, wlim)) { ok = false; break; }
-                        tc_fence_after();
-                        g1(T, 0);
-                        mma_commit(SB(uready, kp));
-                        mma_commit(xfree);
-                        if (!wait_bar(SB(phip, kp), SP(kp), fail, wlim)) { ok = false; break; }
-                        tc_fence_after();
-                        for (int c = 0; c < NCH && ok; ++c) {
-                            const int slot = readout(T + 128, T + 32 * c, qt + c, c == 0);
-                            if (slot < 0) ok = false;
-                            else mma_commit(&empty[slot]);
-                        }
-                        if (!ok) break;
-                        mma_commit(SB(pread, kp));
-                        // P'V: V and P' are single buffers, released in unit order
-                        if (!wait_bar(SB(pready, kp), SP(kp), fail, wlim) || !wait_bar(vfull, kp & 1u, fail, wlim)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                        pv(T + 128);
-                        mma_commit(vfree);
-                        if (!wait_bar(SB(phim, kp), SP(kp), fail, wlim)) { ok = false; break; }
-                        tc_fence_after();
-                        for (int c = NCH; c < NC && ok; ++c) {
-                            const int slot = readout(T + 128, T + 32 * (c - NCH), qt + c);
-                            if (slot < 0) ok = false;
-                            else mma_commit(&empty[slot]);
-                        }
-                        if (!ok) break;
-                        mma_commit(&dready[iss]);
-                    }
-                    qt += NC;
-                    ++kp;
-                }
-            } else {
-                // Tensor Memory: [0,128) D, [128,128+F) phi (U, then phi+, then phi-),
-                // scores after U, [256,256+F) dS+ (U_k^T at 288 until then),
-                // [384,384+F) dS-.  dS^T follows R+, so the first half's tiles are
-                // free for their increments as soon as dS^T is in Tensor Memory.
-                void *nraw = state_raw(a, u_begin, u_end);
-                for (int u = u_begin; u < u_end; ++u) {
-                    void *raw = nraw;
-                    nraw = state_raw(a, u + 1, u_end);
-                    if (!state_at(a, raw, u)) continue;
-                    if (!wait_bar(xfull, kp & 1u, fail, wlim)) { ok = false; break; }
-                    // U_k^T and the scores land in the dS+ columns: the previous unit's
-                    // first-half update must have read them (its R- precedes in issue order)
-                    if (kp >= 1 && !wait_bar(efree, (kp - 1) & 1u, fail, wlim)) { ok = false; break; }
-                    tc_fence_after();
-                    g1(kCmP, kCmK);
-                    mma_commit(uready);
-                    mma_commit(xfree);
-                    // phip also covers the previous unit's output epilogue and second-half update
-                    if (!wait_bar(phip, kp & 1u, fail, wlim)) { ok = false; break; }
-                    tc_fence_after();
-                    for (int c = 0; c < NCH && ok; ++c) ok = readout(kCmD, kCmDSm + 32 * c, qt + c, c == 0) >= 0;
-                    if (!ok) break;
-                    if (!wait_bar(kready, kp & 1u, fail, wlim) || !wait_bar(vfull, kp & 1u, fail, wlim)) { ok = false; break; }
-                    tc_fence_after();
-                    ds(kCmDSp, 0);
-                    ds(kCmDSm, 1);
-                    mma_commit(dsdone);
-                    if (!wait_bar(pready, kp & 1u, fail, wlim)) { ok = false; break; }
-                    tc_fence_after();
-                    pv(kCmD);
-                    mma_commit(pvdone);
-                    if (!wait_bar(phim, kp & 1u, fail, wlim)) { ok = false; break; }
-                    tc_fence_after();
-                    for (int c = NCH; c < NC && ok; ++c) ok = readout(kCmD, kCmP + 32 * (c - NCH), qt + c) >= 0;
-                    if (!ok) break;
-                    mma_commit(&dready[kp & 1]);
-                    mma_commit(vfree);
-                    qt += NC;
-                    ++kp;
-                }
+            void *nraw = state_raw(a, u_begin, u_end);
+            for (int u = u_begin; u < u_end; ++u) {
+                void *raw = nraw;
+                nraw = state_raw(a, u + 1, u_end);
+                if (!state_at(a, raw, u)) continue;
+                if (!wait_bar(xfull, kp & 1u, fail, wlim)) { ok = false; break; }
+                // U_k^T and the scores land in the dS+ columns: the previous unit's
+                // first-half update must have read them (its R- precedes in issue order)
+                if (kp >= 1 && !wait_bar(efree, (kp - 1) & 1u, fail, wlim)) { ok = false; break; }
+                tc_fence_after();
+                g1(kCmP, kCmK);
+                mma_commit(uready);
+                mma_commit(xfree);
+                // phip also covers the previous unit's output epilogue and second-half update
+                if (!wait_bar(phip, kp & 1u, fail, wlim)) { ok = false; break; }
+                tc_fence_after();
+                for (int c = 0; c < NCH && ok; ++c) ok = readout(kCmD, kCmDSm + 32 * c, c == 0) >= 0;
+                if (!ok) break;
+                if (!wait_bar(kready, kp & 1u, fail, wlim) || !wait_bar(vfull, kp & 1u, fail, wlim)) { ok = false; break; }
+                tc_fence_after();
+                ds(kCmDSp, 0);
+                ds(kCmDSm, 1);
+                mma_commit(dsdone);
+                if (!wait_bar(pready, kp & 1u, fail, wlim)) { ok = false; break; }
+                tc_fence_after();
+                pv(kCmD);
+                mma_commit(pvdone);
+                if (!wait_bar(phim, kp & 1u, fail, wlim)) { ok = false; break; }
+                tc_fence_after();
+                for (int c = NCH; c < NC && ok; ++c) ok = readout(kCmD, kCmP + 32 * (c - NCH)) >= 0;
+                if (!ok) break;
+                mma_commit(&dready[kp & 1]);
+                ++kp;
             }
-            mma_commit(&mmadone[iss]);
-            mbar_wait(&mmadone[iss], 0, kWaitNs);
+            mma_commit(mmadone);
+            mbar_wait(mmadone, 0, kWaitNs);
         }
     } else if (warp == 2) {
         // ------------------------------------------------------------- producer
@@ -466,11 +383,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             bool ok = true;
             if (kp > 0) ok = wait_bar(xfree, (kp - 1) & 1u, fail, wlim);
             if (__any_sync(0xffffffffu, !ok)) break;
-            // with the commit the Q region holds the previous unit's V, P' and phi(K)
-            // until its dS^T and P V have run (Q then follows K^T, which measured
-            // faster at start-up too); otherwise Q goes with W, before K^T
-            const bool q_early = !kCommit || kp == 0;
-            uint64_t *xf = SB(xfull, kp);
+            // the Q region holds the previous unit's V, P' and phi(K) until its dS^T
+            // and P V have run, so Q follows K^T (except for the first unit)
+            const bool q_early = kp == 0;
+            uint64_t *xf = xfull;
             if (lane == 0) {
                 mbar_arrive_expect_tx(xf, xbytes);
                 if (q_early)
@@ -491,9 +407,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 mbar_arrive(xf);
             }
             ++nx;
-            // V: after the previous unit's P V (step), after this unit's g1 has read
-            // Q (commit: V shares the Q region)
-            ok = kCommit ? wait_bar(xfree, kp & 1u, fail, wlim) : (kp == 0 || wait_bar(vfree, (kp - 1) & 1u, fail, wlim));
+            // V shares the Q region: after this unit's g1 has read Q
+            ok = wait_bar(xfree, kp & 1u, fail, wlim);
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
                 mbar_arrive_expect_tx(vfull, (uint32_t)(d / 64) * (B * 128));
@@ -505,15 +420,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         }
         if (lane == 0 && *fail) {
             // let copies in flight land before the CTA exits
-            // the last loads of each xfull entry (one entry with the commit, two in the step)
-            for (int k = nx - 1; k >= 0 && k >= nx - (kCommit ? 1 : 2); --k)
-                mbar_wait(SB(xfull, (uint32_t)k), SP((uint32_t)k), kWaitNs);
+            if (nx) mbar_wait(xfull, (uint32_t)(nx - 1) & 1u, kWaitNs);
             if (nv) mbar_wait(vfull, (uint32_t)(nv - 1) & 1u, kWaitNs);
         }
     } else if (warp == 3) {
         // --------------------------------------------------------------- storer
-        // (commit only: the step's math warps store the output themselves)
-        if (kCommit && lane == 0) {
+        if (lane == 0) {
             uint32_t q = 0, kp = 0;
             void *nraw = state_raw(a, u_begin, u_end);
             for (int u = u_begin; u < u_end; ++u) {
@@ -523,34 +435,32 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 if (!Sg) continue;
                 const int r = u / a.Hkv, g = u % a.Hkv;
                 bool ok = true;
-                if (kCommit) {
-                    const int zb = kp & 1;
-                    if (!wait_bar(zdone, kp & 1u, fail, wlim)) break;
-                    bulk_s2g(Sg + (size_t)2 * F * d, zbuf0 + zb * zstride, 2 * F * 4);
-                    bulk_commit();
-                    bulk_wait_read_all();
-                    mbar_arrive(&zempty[zb]);
-                    for (int h = 0; h < 2 && ok; ++h) {
-                        if (!wait_bar(&tready[h], kp & 1u, fail, wlim)) { ok = false; break; }
-                        // one bulk group per tile; the two output slots are freed as
-                        // soon as their reductions have read them
-                        for (int c = h * NCH; c < (h + 1) * NCH; ++c) {
-                            bulk_reduce_add_f32(Sg + (size_t)c * 32 * d, ring + (size_t)((q + c) % NS) * chunk_bytes,
-                                                chunk_bytes);
-                            bulk_commit();
-                        }
-                        if (h == ocm / NCH) {
-                            // the output slots may be written once their reductions have read them
-                            if ((h + 1) * NCH - (ocm + 2) >= 2) bulk_wait_read_2();
-                            else bulk_wait_read_all();
-                            mbar_arrive(ofree);
-                        }
-                        bulk_wait_read_all();
-                        for (int c = h * NCH; c < (h + 1) * NCH; ++c)
-                            if (c < ocm || c > ocm + 1) mbar_arrive(&empty[(q + c) % NS]);
+                const int zb = kp & 1;
+                if (!wait_bar(zdone, kp & 1u, fail, wlim)) break;
+                bulk_s2g(Sg + (size_t)2 * F * d, zbuf0 + zb * zstride, 2 * F * 4);
+                bulk_commit();
+                bulk_wait_read_all();
+                mbar_arrive(&zempty[zb]);
+                for (int h = 0; h < 2 && ok; ++h) {
+                    if (!wait_bar(&tready[h], kp & 1u, fail, wlim)) { ok = false; break; }
+                    // one bulk group per tile; the two output slots are freed as
+                    // soon as their reductions have read them
+                    for (int c = h * NCH; c < (h + 1) * NCH; ++c) {
+                        bulk_reduce_add_f32(Sg + (size_t)c * 32 * d, ring + (size_t)((q + c) % NS) * chunk_bytes,
+                                            chunk_bytes);
+                        bulk_commit();
                     }
-                    if (!ok) break;
+                    if (h == ocm / NCH) {
+                        // the output slots may be written once their reductions have read them
+                        if ((h + 1) * NCH - (ocm + 2) >= 2) bulk_wait_read_2();
+                        else bulk_wait_read_all();
+                        mbar_arrive(ofree);
+                    }
+                    bulk_wait_read_all();
+                    for (int c = h * NCH; c < (h + 1) * NCH; ++c)
+                        if (c < ocm || c > ocm + 1) mbar_arrive(&empty[(q + c) % NS]);
                 }
+                if (!ok) break;
                 // output tile: two TMA boxes from the two held-back slots
                 if (!wait_bar(ostaged, kp & 1u, fail, wlim)) break;
                 uint8_t *s0 = ring + (size_t)((q + ocm) % NS) * chunk_bytes;
@@ -588,46 +498,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         float *tk = xb + 8 * 128;                                  // token statistics (commit)
         uint8_t *pkb = smem + a.off_pk;
         const float scale_l2 = a.scale * kLog2e;
-        const uint32_t pair_bar = kBarPair + q4;
-        // one exchange point: pair barrier for the step, all math warps with the commit
-        auto sync_failed = [&](bool local_fail) -> bool {
-            return kCommit ? group_sync_failed(kBarMath, kMathThreads, local_fail)
-                           : group_sync_failed(pair_bar, 64, local_fail);
-        };
+        // exchange point of all math warps
+        auto sync_failed = [&](bool local_fail) -> bool { return group_sync_failed(kBarMath, kMathThreads, local_fail); };
 
-        // out = D / den.  Commit: staged as the TMA box image in the unit's held-back
-        // ring slots (row i = t*G + hh, 128-byte swizzle) for the storer.  Step: stored
-        // from registers (each thread 16-byte runs of its row's d/2 columns), so every
-        // ring slot is free as soon as its readout has run and the next unit's last
-        // tiles do not wait for this unit's output.
-        auto epilogue = [&](uint32_t ek, uint32_t eq, float inv, int eu) -> bool {
-            const uint32_t dcol = kCommit ? kCmD : (ek & 1) * 256 + 128;
+        // out = D / den, staged as the TMA box image in the unit's held-back ring
+        // slots (row i = t*G + hh, 128-byte swizzle) for the storer
+        auto epilogue = [&](uint32_t ek, uint32_t eq, float inv) -> bool {
             bool ok = wait_bar(&dready[ek & 1], (ek >> 1) & 1u, fail, wlim);
-            if (kCommit && ok) ok = wait_bar(ofree, ek & 1u, fail, wlim);
+            if (ok) ok = wait_bar(ofree, ek & 1u, fail, wlim);
             tc_fence_after();
             const int dh = d / 2;
-            if (!kCommit) {
-                const int r = eu / a.Hkv, gg = eu % a.Hkv;
-                const int t = row / G, hh = row % G;
-                bf16 *orow = a.O + (((size_t)r * B + t) * a.Hq + (size_t)gg * G + hh) * d + part * dh;
-                for (int hc = 0; hc < dh / 32; ++hc) {
-                    float v[32];
-                    tmem_ld32(tmem + dcol + lane_off + part * dh + 32 * hc, v);
-                    tmem_wait_ld();
-                    if (ok && valid) {
-                        uint32_t pk[16];
-#pragma unroll
-                        for (int i = 0; i < 32; i += 2) pk[i / 2] = pack_bf16x2(v[i] * inv, v[i + 1] * inv);
-                        uint4 *dst = reinterpret_cast<uint4 *>(orow + 32 * hc);
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-                    }
-                }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0 && ok) mbar_arrive(&dfree[ek & 1]);
-                return ok;
-            }
             // d = 128: column half -> slot; d = 64: token half -> slot (one 64-column atom)
             const int rows_half = G * B / 2;
             const int sidx = d == 128 ? part : (row >= rows_half ? 1 : 0);
@@ -635,7 +515,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             uint8_t *base = ring + (size_t)((eq + ocm + sidx) % NS) * chunk_bytes + srow * 128;
             for (int hc = 0; hc < dh / 32; ++hc) {
                 float v[32];
-                tmem_ld32(tmem + dcol + lane_off + part * dh + 32 * hc, v);
+                tmem_ld32(tmem + kCmD + lane_off + part * dh + 32 * hc, v);
                 tmem_wait_ld();
                 if (ok && valid) {
                     uint32_t pk[16];
@@ -652,17 +532,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             fence_proxy_async_smem();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0 && ok) {
-                mbar_arrive(ostaged);
-                mbar_arrive(&dfree[ek & 1]);
-            }
+            if (lane == 0 && ok) mbar_arrive(ostaged);
             return ok;
         };
 
-        uint32_t q = 0, kp = 0, prev_q = 0;
-        float prev_inv = 0.f;   // 1 / den of the unit whose output is still pending (step)
-        int prev_u = 0;         // and that unit
-        bool ok = true;
+        uint32_t q = 0, kp = 0;
         void *nraw = state_raw(a, u_begin, u_end);
         float nalpha = valid && u_begin < u_end ? a.alpha[(u_begin % a.Hkv) * G + row % G] : 0.f;
         for (int u = u_begin; u < u_end; ++u) {
@@ -678,21 +552,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             }
             const int zb = kp & 1;
             float *zs = zbuf0 + zb * zstride;
-            const uint32_t T = (kp & 1) * 256;
-            const uint32_t pcol = tmem + (kCommit ? kCmP : T) + lane_off;       // U, phi+, phi-
-            const uint32_t scol = pcol + F;                                    // scores
-            const uint32_t kcol = tmem + kCmK + lane_off;                      // U_k^T (commit)
-            // phi+: with the commit in the dS- columns (free until dS^T is formed), so U
-            // stays in place for phi- and no thread holds U in registers; the step keeps
-            // U in registers and writes phi+ over it
-            const uint32_t ppcol = kCommit ? tmem + kCmDSm + lane_off : pcol;
+            const uint32_t pcol = tmem + kCmP + lane_off;    // U, then phi-
+            const uint32_t scol = pcol + F;                  // scores
+            const uint32_t kcol = tmem + kCmK + lane_off;    // U_k^T
+            // phi+ in the dS- columns (free until dS^T is formed), so U stays in place
+            // for phi- and no thread holds U in registers
+            const uint32_t ppcol = tmem + kCmDSm + lane_off;
 
-            // ---- phase A: row extrema of U and of the scores (U kept in registers);
-            // commit: per-token extrema of U_k^T over this warp's 32 features
-            bool bad = !wait_bar(SB(uready, kp), SP(kp), fail, wlim);
+            // ---- phase A: row extrema of U and of the scores, and the per-token
+            // extrema of U_k^T over this warp's 32 features
+            bool bad = !wait_bar(uready, kp & 1u, fail, wlim);
             tc_fence_after();
-            float sc[16], u0[32], u1[32];
-            if (kCommit) {
+            float sc[16];
+            {
                 // phi(K): thread (feature row, part) owns feature part*F + row of every
                 // token; part 0 needs the per-token max of U_k over features, part 1
                 // the min (features on lanes: reduce over the warp, then the quarters)
@@ -705,10 +577,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 tk[(part * 32 + lane) * 4 + q4] = ext;   // max of +-U_k for token lane
             }
             if (has_sc) tmem_ld16(scol + 16 * part, sc);
-            if (!kCommit) {
-                tmem_ld32(pcol + 32 * part, u0);
-                if (two) tmem_ld32(pcol + 32 * (part + 2), u1);
-            }
             tmem_wait_ld();
             {
                 float ms = -INFINITY, mx = -INFINITY, mn = INFINITY;
@@ -716,29 +584,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
 #pragma unroll
                     for (int i = 0; i < 16; ++i) ms = fmaxf(ms, sc[i]);
                 }
-                if (kCommit) {
-                    // this thread's 32-feature chunks of U, one at a time
+                // this thread's 32-feature chunks of U, one at a time
 #pragma unroll 1
-                    for (int k = part; k < NCH; k += 2) {
-                        float x[32];
-                        tmem_ld32(pcol + 32 * k, x);
-                        tmem_wait_ld();
+                for (int k = part; k < NCH; k += 2) {
+                    float x[32];
+                    tmem_ld32(pcol + 32 * k, x);
+                    tmem_wait_ld();
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, x[i]); mn = fminf(mn, x[i]); }
-                    }
-                } else {
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, u0[i]); mn = fminf(mn, u0[i]); }
-                    if (two) {
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, u1[i]); mn = fminf(mn, u1[i]); }
-                    }
+                    for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, x[i]); mn = fminf(mn, x[i]); }
                 }
                 xa[(part * 3 + 0) * 128 + row] = ms;
                 xa[(part * 3 + 1) * 128 + row] = mx;
                 xa[(part * 3 + 2) * 128 + row] = mn;
             }
-            if (sync_failed(bad)) { ok = false; break; }
+            if (sync_failed(bad)) break;
             const float ms = fmaxf(xa[0 * 128 + row], xa[3 * 128 + row]);
             const float mx = fmaxf(xa[1 * 128 + row], xa[4 * 128 + row]);
             const float mn = fminf(xa[2 * 128 + row], xa[5 * 128 + row]);
@@ -769,44 +628,36 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     }
                     tmem_st32(ppcol + 32 * k, ep);
                 };
-                if (kCommit) {
 #pragma unroll 1
-                    for (int k = part; k < NCH; k += 2) {
-                        float x[32];
-                        tmem_ld32(pcol + 32 * k, x);
-                        tmem_wait_ld();
-                        expp(x, k);
-                    }
-                } else {
-                    expp(u0, part);
-                    if (two) expp(u1, part + 2);
+                for (int k = part; k < NCH; k += 2) {
+                    float x[32];
+                    tmem_ld32(pcol + 32 * k, x);
+                    tmem_wait_ld();
+                    expp(x, k);
                 }
                 xs[part * 128 + row] = sp;
             }
-            if (sync_failed(bad)) { ok = false; break; }
+            if (sync_failed(bad)) break;
             const float sp = xs[row] + xs[128 + row];
             // Accumulate D / kappa with kappa = e^-sigma / sp: phi+ then stays
             // unnormalised in Tensor Memory (no rescale pass) and phi- (in registers)
             // and P' absorb the factor (phi- x sp/sn, P' = w sp e^s).  This needs the
             // unshifted softmax mass w sp e^(s) inside float range; a warp with any row
             // beyond e^60 rescales phi+ exactly once sigma is known (phase C).
-            const bool fast = __all_sync(0xffffffffu, !(lw + ms * a.scale + logf(sp) > 60.f));
+            const bool fast = __all_sync(0xffffffffu, !(lw + ms * a.scale + __logf(sp) > 60.f));
             if (fast) {
                 tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0 && !a.withhold) mbar_arrive(SB(phip, kp));
+                if (lane == 0) mbar_arrive(phip);
             }
 
-            // ---- phase B2: phi- (kept in registers until R+ has consumed phi+), the
-            // score sums; commit: unnormalised phi(K)
+            // ---- phase B2: phi- over U (unscaled), the score sums, unnormalised phi(K)
             {
                 float l = 0.f, sn = 0.f, ln = 0.f;
                 if (has_sc) {
-                    if (kCommit) {
-                        tmem_ld16(scol + 16 * part, sc);
-                        tmem_wait_ld();
-                    }
+                    tmem_ld16(scol + 16 * part, sc);
+                    tmem_wait_ld();
 #pragma unroll
                     for (int i = 0; i < 16; ++i) l += ex2(fmaf(sc[i], scale_l2, -ml));
                 }
@@ -826,21 +677,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                         }
                     }
                 };
-                if (kCommit) {
-                    // phi- (unscaled) over U in its columns; scaled by cneg in phase D
+                // phi- (unscaled) over U in its columns; scaled by cneg in phase D
 #pragma unroll 1
-                    for (int k = part; k < NCH; k += 2) {
-                        float x[32];
-                        tmem_ld32(pcol + 32 * k, x);
-                        tmem_wait_ld();
-                        expm(x, k);
-                        tmem_st32(pcol + 32 * k, x);
-                    }
-                } else {
-                    expm(u0, part);
-                    if (two) expm(u1, part + 2);
+                for (int k = part; k < NCH; k += 2) {
+                    float x[32];
+                    tmem_ld32(pcol + 32 * k, x);
+                    tmem_wait_ld();
+                    expm(x, k);
+                    tmem_st32(pcol + 32 * k, x);
                 }
-                if (kCommit) {
+                {
                     // unnormalised phi(K) of this thread's feature for every token
                     float uk[32];
                     tmem_ld32(kcol, uk);
@@ -867,28 +713,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 xb[(part * 4 + 2) * 128 + row] = sn;
                 xb[(part * 4 + 3) * 128 + row] = ln;
             }
-            if (!kCommit) {
-                // z has been read
-                __syncwarp();
-                if (lane == 0 && !bad) mbar_arrive(&zempty[zb]);
-            }
-            if (sync_failed(bad)) { ok = false; break; }
+            if (sync_failed(bad)) break;
 
-            // ---- phase C: sigma, P', den (and, off the fast path, phi+ rescaled);
-            // commit: phi(K), z
+            // ---- phase C: phi(K), z, sigma, P', den (and, off the fast path, phi+
+            // rescaled)
             float cneg, inv_den;
             {
-                // with the commit the scores share the dS+ columns, which dS^T may
-                // overwrite once phi(K) is signalled: P' takes them from registers
-                if (kCommit && has_sc) tmem_ld16(scol + 16 * part, sc);
-                if (kCommit) {
+                // the scores share the dS+ columns, which dS^T may overwrite once
+                // phi(K) is signalled: P' takes them from registers
+                if (has_sc) tmem_ld16(scol + 16 * part, sc);
+                {
                     // phi(K) normalised, as the bf16 MN-major operand [token][feature]
                     // (64-feature atoms of B rows), and z[part*F + row] += sum_t phi(k_t)
                     // (this thread is the only writer); lane t holds token t's normaliser
                     float inv_l;
                     {
                         const float4 v = *reinterpret_cast<const float4 *>(&tk[((2 + part) * 32 + lane) * 4]);
-                        inv_l = 1.f / ((v.x + v.y) + (v.z + v.w));
+                        inv_l = __fdividef(1.f, (v.x + v.y) + (v.z + v.w));
                     }
                     float ek[32];   // unnormalised phi(K) of feature part*F + row, per token
                     tmem_wait_st();
@@ -919,19 +760,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 const float lpf = xb[1 * 128 + row] + xb[5 * 128 + row];
                 const float sn = xb[2 * 128 + row] + xb[6 * 128 + row];
                 const float ln = xb[3 * 128 + row] + xb[7 * 128 + row];
-                const float lin_den = lpf / sp + ln / sn;
-                const float log_s = lw + ms * a.scale + logf(l);   // log(w sm_den)
-                const float log_l = logf(lin_den);                   // log(lin_den), -inf if empty
+                // (approximate intrinsics: the result is rounded to bf16)
+                const float rsp = __fdividef(1.f, sp), rsn = __fdividef(1.f, sn);
+                const float lin_den = lpf * rsp + ln * rsn;
+                const float log_s = lw + ms * a.scale + __logf(l);   // log(w sm_den)
+                const float log_l = __logf(lin_den);                   // log(lin_den), -inf if empty
                 const float sig = fmaxf(fmaxf(log_s, log_l), -60.f);
-                const float esig = expf(-sig);
+                const float esig = __expf(-sig);
                 float kappa, pofs;
                 if (fast) {
-                    kappa = esig / sp;
-                    cneg = lin_den > 0.f ? sp / sn : 0.f;
-                    pofs = (lw + logf(sp)) * kLog2e;
+                    kappa = esig * rsp;
+                    cneg = lin_den > 0.f ? sp * rsn : 0.f;
+                    pofs = lw * kLog2e + __log2f(sp);
                 } else {
-                    const float cpos = lin_den > 0.f ? esig / sp : 0.f;
-                    cneg = lin_den > 0.f ? esig / sn : 0.f;
+                    const float cpos = lin_den > 0.f ? esig * rsp : 0.f;
+                    cneg = lin_den > 0.f ? esig * rsn : 0.f;
                     kappa = 1.f;
                     pofs = (lw - sig) * kLog2e;
                     auto scale_chunk = [&](uint32_t col) {
@@ -947,10 +790,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     tmem_wait_st();
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0 && !a.withhold) mbar_arrive(SB(phip, kp));
+                    if (lane == 0) mbar_arrive(phip);
                 }
-                // step: the previous unit's P'V (issued after this unit's g1) has read P'
-                if (!kCommit && kp >= 1) bad = !wait_bar(vfree, (kp - 1) & 1u, fail, wlim) || bad;
                 if (has_sc) {
                     // P' (w e^(s - sigma), or w sp e^s on the fast path): K-major, no swizzle
                     // (8-row x 16-byte core matrices)
@@ -962,17 +803,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     *reinterpret_cast<uint4 *>(prow + (2 * part) * 128) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
                     *reinterpret_cast<uint4 *>(prow + (2 * part + 1) * 128) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                 }
-                inv_den = kappa / (expf(log_l - sig) + expf(log_s - sig));
+                inv_den = __fdividef(kappa, __expf(log_l - sig) + __expf(log_s - sig));
             }
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(SB(pready, kp));
+            if (lane == 0) mbar_arrive(pready);
 
-            // previous unit's output, while R+ of this one runs (step)
-            if (!kCommit && kp >= 1) bad = !epilogue(kp - 1, prev_q, prev_inv, prev_u);
-            // ---- phase D: phi- scaled by cneg in the phi columns (step: once R+ has
-            // consumed phi+ there)
-            if (kCommit) {
+            // ---- phase D: phi- scaled by cneg in the phi columns
+            {
                 tmem_wait_st();
 #pragma unroll 1
                 for (int k = part; k < NCH; k += 2) {
@@ -983,24 +821,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     for (int i = 0; i < 32; ++i) x[i] *= cneg;
                     tmem_st32(pcol + 32 * k, x);
                 }
-            } else {
-                bad = !wait_bar(SB(pread, kp), SP(kp), fail, wlim) || bad;
-                tc_fence_after();
-#pragma unroll
-                for (int i = 0; i < 32; ++i) u0[i] *= cneg;
-                tmem_st32(pcol + 32 * part, u0);
-                if (two) {
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) u1[i] *= cneg;
-                    tmem_st32(pcol + 32 * (part + 2), u1);
-                }
             }
             tmem_wait_st();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0 && !bad) mbar_arrive(SB(phim, kp));
+            if (lane == 0 && !bad) mbar_arrive(phim);
 
-            if (kCommit) {
+            {
                 // ---- state update: S^T += dS^T for a feature half as soon as the readout
                 // has consumed its tiles (first half now, second after R-): dS^T rows go
                 // into the tiles' slots and the storer adds them into the state by
@@ -1036,15 +863,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                         if (h == 0) mbar_arrive(efree);
                     }
                 }
-                epilogue(kp, q, inv_den, u);
+                epilogue(kp, q, inv_den);
             }
-            prev_q = q;
-            prev_inv = inv_den;
-            prev_u = u;
             q += NC;
             ++kp;
         }
-        if (!kCommit && ok && kp >= 1) epilogue(kp - 1, prev_q, prev_inv, prev_u);
         if (mt == 0 && *fail) raise_error(a.err, ERR_WAIT_TIMEOUT);
     }
 
@@ -1057,32 +880,29 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
 
 }  // namespace
 
-bool fused_supported(const hybrid_cfg &c, bool commit)
+bool fused_supported(const hybrid_cfg &c)
 {
     if (c.io_dtype != HYBRID_BF16) return false;
     if (c.head_dim != 64 && c.head_dim != 128) return false;
     if (c.feat_dim != 64 && c.feat_dim != 128) return false;
-    // scores ride in one 16-column chunk per part; the K^T atom holds B <= 64 tokens
-    if (c.block_size != 16 && c.block_size != 32) return false;
+    // phi(K) is formed for 32 tokens on the 32 lanes of a warp; the scores ride in
+    // one 16-column chunk per part
+    if (c.block_size != 32) return false;
     const int G = c.n_q_heads / c.n_kv_heads;
     if (G * c.block_size > 128) return false;
-    if (commit && c.block_size != 32) return false;
-    const FLayout L = make_flayout(c.head_dim, c.feat_dim, c.block_size, commit);
+    const FLayout L = make_flayout(c.head_dim, c.feat_dim, c.block_size);
     const int NCH = c.feat_dim / 32;
-    // step: the last two tiles of a unit are held for the output; commit: a ring
-    // shorter than a unit stages the output in first-half slots that no later tile
-    // of the unit reuses, which needs NCH + 2 slots
-    if (L.NS < (commit ? NCH + 2 : 4)) return false;
+    // a ring shorter than a unit stages the output in first-half slots that no
+    // later tile of the unit reuses, which needs NCH + 2 slots
+    if (L.NS < NCH + 2) return false;
     return (int)L.bytes <= kSmemLimit;
 }
 
-cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const void *K, const void *V,
-                         const void *W, const float *alpha, void *const *states, int n_req, void *O,
-                         unsigned *err, cudaStream_t st)
+cudaError_t launch_fused(const hybrid_cfg &c, const void *Q, const void *K, const void *V, const void *W,
+                         const float *alpha, void *const *states, int n_req, void *O, unsigned *err,
+                         cudaStream_t st)
 {
-    // the step alone runs in hybrid_step.cu
-    if (!commit) return cudaErrorNotSupported;
-    const FLayout L = make_flayout(c.head_dim, c.feat_dim, c.block_size, commit);
+    const FLayout L = make_flayout(c.head_dim, c.feat_dim, c.block_size);
     FusedArgs a;
     {
         const int d = c.head_dim, F = c.feat_dim, B = c.block_size, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
@@ -1103,7 +923,6 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
             return cudaErrorInvalidValue;
     }
     a.K = static_cast<const bf16 *>(K);
-    a.O = static_cast<bf16 *>(O);
     a.alpha = alpha;
     a.states = states;
     a.err = err;
@@ -1116,12 +935,6 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
     a.F = c.feat_dim;
     a.NS = L.NS;
     a.scale = 1.f / sqrtf((float)c.head_dim);
-    {
-        // a test may arm one step launch with a short wait limit and a withheld arrival
-        const unsigned long long armed = commit ? 0ull : g_armed_wait_ns.exchange(0ull);
-        a.wait_ns = armed ? armed : (unsigned long long)kWaitNs;
-        a.withhold = armed ? 1 : 0;
-    }
     a.off_q = L.off_q;
     a.off_wk = L.off_wk;
     a.off_vb = L.off_vb;
@@ -1138,7 +951,7 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     const unsigned long long bit = 1ull << dev;
     if (!(opted.load(std::memory_order_acquire) & bit)) {
-        const cudaError_t e = cudaFuncSetAttribute(k_fused<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
+        const cudaError_t e = cudaFuncSetAttribute(k_fused, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
         if (e != cudaSuccess) return e;
         opted.fetch_or(bit, std::memory_order_release);
     }
@@ -1152,7 +965,7 @@ cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const 
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = attr;
     lc.numAttrs = 1;
-    return cudaLaunchKernelEx(&lc, k_fused<true>, a);
+    return cudaLaunchKernelEx(&lc, k_fused, a);
 }
 
 }  // namespace hyb

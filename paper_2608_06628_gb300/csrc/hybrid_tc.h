@@ -27,12 +27,13 @@ cudaError_t launch_step(const hybrid_cfg &c, const void *Q, const void *K, const
                         const float *alpha, void *const *states, int n_req, void *O, unsigned *err,
                         cudaStream_t st);
 
-// Persistent warp-specialised step kernel (hybrid_fused.cu); commit = true also
-// folds the block's K/V into the state in the same pass.
-bool fused_supported(const hybrid_cfg &c, bool commit);
-cudaError_t launch_fused(const hybrid_cfg &c, bool commit, const void *Q, const void *K, const void *V,
-                         const void *W, const float *alpha, void *const *states, int n_req, void *O,
-                         unsigned *err, cudaStream_t st);
+// Persistent warp-specialised step fused with the block commit (hybrid_fused.cu):
+// the readout uses the pre-commit state and the block's K/V are folded into the
+// state in the same pass.
+bool fused_supported(const hybrid_cfg &c);
+cudaError_t launch_fused(const hybrid_cfg &c, const void *Q, const void *K, const void *V, const void *W,
+                         const float *alpha, void *const *states, int n_req, void *O, unsigned *err,
+                         cudaStream_t st);
 
 // Commit / prefill as a reduction (hybrid_commit_red.cu): S += dS and z += dz are
 // added into the state in global memory by bulk reduce-adds; any n_tok >= 1.
