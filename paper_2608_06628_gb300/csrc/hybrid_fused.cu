@@ -15,16 +15,15 @@
 //              copies, through an NS-slot ring (the state layout is the MMA
 //              operand image, see hybrid.h).
 //   warp 1     MMA issuer (one thread); owns the Tensor Memory allocation.
-//   warp 2     producer: TMA of Q and W, the transposed key tile K^T (built by
-//              the warp from global memory) and V.
+//   warp 2     producer: TMA of Q, W, K and V.
 //   warp 3     storer: bulk reduce-adds of the dS^T tiles into the state, the
 //              store of z, and TMA stores of the output tile.
 //   warps 4-11 math: two threads per query row (one per TMEM lane and "part");
 //              a part owns every other 32-feature chunk of each half of phi.
 //
 // Per unit the tensor cores run, in this order,
-//   g1   [U | scores] = Q [W | K^T]  (one N = F + B product; U = Q W)
-//        and U_k^T = W^T K^T (phi of the block's keys)
+//   g1   U = Q W, scores = Q K^T and U_k^T = W^T K^T (phi of the block's keys);
+//        K, as loaded, is the K-major operand of the last two
 //   R+   D  = phi+'(Q) S+             (tf32, A operand in Tensor Memory)
 //   dS   dS^T = V^T phi(K)^T per feature half (bf16 from the TMA'd V)
 //   PV   D += P' V                    (P' = w e^(s - sigma), bf16)
@@ -48,9 +47,9 @@
 // and phi(K) share the Q region once g1 has consumed Q, so all 2F/32 state
 // tiles of a unit fit in the ring.
 //
-// MMA cost note: on this part a tcgen05.mma with M = 128 costs about the same
-// time for any N up to 128-256, so contractions are shaped for few, wide
-// instructions (the scores ride along with U; dS^T is two N = F products).
+// MMA cost note: on this part a tcgen05.mma with M = 128 costs its issuing thread
+// about the same time for any N up to 128-256, so contractions are shaped for few,
+// wide instructions (dS^T is two N = F products).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -82,8 +81,7 @@ constexpr uint32_t kCmD = 0, kCmP = 128, kCmDSp = 256, kCmK = 288, kCmDSm = 384;
 constexpr uint32_t kCmEK = 320;
 
 struct FusedArgs {
-    CUtensorMap tmQ, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
-    const bf16 *K;
+    CUtensorMap tmQ, tmK, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], K, V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
     const float *alpha;
     void *const *states;
     unsigned *err;
@@ -92,12 +90,12 @@ struct FusedArgs {
     uint32_t off_q, off_wk, off_vb, off_p, off_pk, off_z, off_st, off_bar;
 };
 
-// Shared memory: [ring NS x d*128][Q][W | K^T][V][P'][phi(K) (commit)][z x2][stats][barriers].
-// Q, V and W land by TMA with the 128-byte swizzle: Q as d/64 atoms of 128 rows
-// (16 KB apart; rows t*G + h), V as d/64 atoms of B rows (MN-major operand:
-// 8-row groups 1 KB apart, atoms B*128 apart), W as F/64 atoms of d rows
-// (MN-major: e-groups 1 KB apart, atoms d*128 apart) followed by the K^T atom
-// (row e holds K[0..B)[e]), so that [W | K^T] is one MN-major B operand.
+// Shared memory: [ring NS x d*128][Q][W][K][V][P'][phi(K)][z x2][stats][barriers]
+// (V, P' and phi(K) overlay the Q region once g1 has read Q).  Q, K, V and W land
+// by TMA with the 128-byte swizzle: Q as d/64 atoms of 128 rows (16 KB apart;
+// rows t*G + h), K and V as d/64 atoms of B rows (K the K-major operand, V the
+// MN-major one: 8-row groups 1 KB apart, atoms B*128 apart), W as F/64 atoms of
+// d rows (MN-major: e-groups 1 KB apart, atoms d*128 apart).
 struct FLayout {
     uint32_t off_q, off_wk, off_vb, off_p, off_pk, off_z, off_st, off_bar, bytes;
     int NS;
@@ -109,7 +107,7 @@ FLayout make_flayout(int d, int F, int B)
     const uint32_t chunk = (uint32_t)d * 128;
     const uint32_t zb = (((uint32_t)2 * F * 4) + 1023) & ~1023u;
     const uint32_t q = (uint32_t)d * 256;
-    const uint32_t wk = (uint32_t)(F / 64 + 1) * d * 128;
+    const uint32_t wk = (uint32_t)(F / 64) * d * 128 + ((((uint32_t)B * d * 2) + 1023) & ~1023u);
     const uint32_t vb = (((uint32_t)B * d * 2) + 1023) & ~1023u;
     const uint32_t p = (((uint32_t)128 * B * 2) + 1023) & ~1023u;
     const uint32_t pk = (((uint32_t)(2 * F / 64) * B * 128) + 1023) & ~1023u;
@@ -183,7 +181,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     uint64_t *zempty = zfull + 2;     // [2]
     uint64_t *dready = zempty + 2;    // [2] MMA -> math: the unit's output accumulator is complete
     uint64_t *tready = dready + 2;    // [2] math -> storer: a feature half of the tiles is updated
-    uint64_t *xfull = tready + 2;     // Q, W (TMA) and K^T (producer warp) are in place
+    uint64_t *xfull = tready + 2;     // Q, W and K have landed
     uint64_t *uready = xfull + 1;     // MMA -> math: g1 done
     uint64_t *phip = uready + 1;      // math -> MMA: phi+ is in the dS- columns
     uint64_t *phim = phip + 1;        // math -> MMA: phi- in the phi columns
@@ -205,6 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     if (warp == 2 && lane == 0) {
         prefetch_tensormap(&a.tmQ);
         prefetch_tensormap(&a.tmW);
+        prefetch_tensormap(&a.tmK);
         prefetch_tensormap(&a.tmV);
     }
     if (warp == 3 && lane == 0) prefetch_tensormap(&a.tmO);
@@ -280,20 +279,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             const uint32_t q_u = smem_u32(smem + a.off_q), wk_u = smem_u32(smem + a.off_wk),
                            vb_u = smem_u32(smem + a.off_vb), p_u = smem_u32(smem + a.off_p),
                            pk_u = smem_u32(smem + a.off_pk), ring_u = smem_u32(ring);
-            const uint32_t kt_u = wk_u + (uint32_t)(F / 64) * d * 128;
-            const uint32_t idUS = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F + B);
-            const uint32_t idKT = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, B);
+            const uint32_t k_u = wk_u + (uint32_t)(F / 64) * d * 128;   // K: d/64 atoms of B rows
+            const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
+            const uint32_t idS = instr_desc(FMT_BF16, FMT_BF16, false, false, 128, B);
+            const uint32_t idKT = instr_desc(FMT_BF16, FMT_BF16, true, false, 128, B);
             const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
             const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
             const uint32_t idDS = instr_desc(FMT_BF16, FMT_BF16, true, true, 128, F);
-            // g1: [U | scores] at column ucol, and U_k^T at column kcol
+            // g1: U = Q W at column ucol and the scores Q K^T after it, U_k^T = W^T K^T at
+            // column kcol; K as loaded is the K-major operand of both
             auto g1 = [&](uint32_t ucol, uint32_t kcol) {
                 for (int k = 0; k < d / 16; ++k) {
                     const uint64_t aq = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
-                    const uint64_t bwk = smem_desc(wk_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
-                    mma_bf16_ss(tmem + ucol, aq, bwk, idUS, k > 0);
-                    const uint64_t bkt = smem_desc(kt_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
-                    mma_bf16_ss(tmem + kcol, bwk, bkt, idKT, k > 0);
+                    const uint64_t bw = smem_desc(wk_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
+                    const uint64_t bk = smem_desc(k_u + (k >> 2) * (B * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
+                    mma_bf16_ss(tmem + ucol, aq, bw, idU, k > 0);
+                    mma_bf16_ss(tmem + ucol + F, aq, bk, idS, k > 0);
+                    mma_bf16_ss(tmem + kcol, bw, bk, idKT, k > 0);
                 }
             };
             // P'V accumulates onto the phi+ readout
@@ -370,21 +372,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         // ------------------------------------------------------------- producer
         uint32_t kp = 0;
         int nx = 0, nv = 0;
-        const uint32_t xbytes = (uint32_t)(d / 64) * (G * B * 128) + (uint32_t)(F / 64) * (d * 128);
-        uint8_t *kt = smem + a.off_wk + (F / 64) * d * 128;
+        const uint32_t xbytes =
+            (uint32_t)(d / 64) * (G * B * 128) + (uint32_t)(F / 64) * (d * 128) + (uint32_t)(d / 64) * (B * 128);
+        uint8_t *kb = smem + a.off_wk + (F / 64) * d * 128;
         void *nraw = state_raw(a, u_begin, u_end);
         for (int u = u_begin; u < u_end; ++u) {
             void *raw = nraw;
             nraw = state_raw(a, u + 1, u_end);
             if (!state_at(a, raw, u)) continue;
             const int r = u / a.Hkv, g = u % a.Hkv;
-            KtRegs kr;
-            kt_load(a.K, (size_t)r * B, B, a.Hkv, g, d, kr, lane);   // in flight while the region drains
             bool ok = true;
             if (kp > 0) ok = wait_bar(xfree, (kp - 1) & 1u, fail, wlim);
             if (__any_sync(0xffffffffu, !ok)) break;
             // the Q region holds the previous unit's V, P' and phi(K) until its dS^T
-            // and P V have run, so Q follows K^T (except for the first unit)
+            // and P V have run, so Q follows W and K (except for the first unit)
             const bool q_early = kp == 0;
             uint64_t *xf = xfull;
             if (lane == 0) {
@@ -394,9 +395,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                         tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xf);
                 for (int f = 0; f < F / 64; ++f)
                     tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xf);
+                for (int e = 0; e < d / 64; ++e)
+                    tma_load_3d(kb + e * (B * 128), &a.tmK, 64 * e, g, r * B, xf);
             }
-            kt_store(kr, d, kt, lane);
-            fence_proxy_async_smem();
             __syncwarp();
             if (!q_early && kp > 0) ok = wait_bar(pvdone, (kp - 1) & 1u, fail, wlim);
             if (__any_sync(0xffffffffu, !ok)) break;
@@ -918,11 +919,11 @@ cudaError_t launch_fused(const hybrid_cfg &c, const void *Q, const void *K, cons
         const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
         const cuuint32_t bw[2] = {64, (cuuint32_t)d};
         const cuuint32_t bo[3] = {64, (cuuint32_t)G, (cuuint32_t)(d == 128 ? B : B / 2)};
-        if (!encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !encode_bf16(&a.tmV, V, 3, dv, sv, bv) ||
+        if (!encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !encode_bf16(&a.tmK, K, 3, dv, sv, bv) ||
+            !encode_bf16(&a.tmV, V, 3, dv, sv, bv) ||
             !encode_bf16(&a.tmW, W, 2, dw, sw, bw) || !encode_bf16(&a.tmO, O, 3, dq, sq, bo))
             return cudaErrorInvalidValue;
     }
-    a.K = static_cast<const bf16 *>(K);
     a.alpha = alpha;
     a.states = states;
     a.err = err;
