@@ -35,9 +35,10 @@ namespace hyb {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr uint32_t kColA = 0;     // U, then phi = [phi+, phi-] (F <= 128); F = 256: phi+, then phi-
-constexpr uint32_t kColD = 256;   // D_lin (d columns)
-constexpr uint32_t kColS = 384;   // scores (B columns), then D_s (d columns)
+constexpr uint32_t kColA = 0;     // U, then phi = [phi+, phi-] (F <= 128); F = 256: phi+, then phi-;
+                                  // then D_s = P V (d columns)
+constexpr uint32_t kColD = 256;   // D_lin of issuer A's tiles (d columns)
+constexpr uint32_t kColS = 384;   // scores (B columns), then D_lin of issuer B's tiles
 constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s per bounded wait
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kSmemLimit = 232448;            // 227 KB opt-in per CTA
@@ -182,16 +183,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     uint64_t *empty = bars + RM;
     uint64_t *bar_z = bars + 2 * RM;
     uint64_t *bar_u = bar_z + 1;
-    uint64_t *bar_d = bar_z + 2;
-    uint64_t *bar_p = bar_z + 3;    // F = 256: the phi+ readout is done
+    uint64_t *bar_d = bar_z + 2;    // both issuers: D_lin halves and D_s are complete
+    uint64_t *bar_p = bar_z + 3;    // F = 256, both issuers: the phi+ readout is done
     uint64_t *bar_u2 = bar_z + 4;   // F = 256: U = Q W formed again, for phi-
     uint64_t *bar_ld = bar_z + 5;   // Q, K, V and W have landed
-    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_z + 6);
+    uint64_t *bar_b = bar_z + 6;    // issuer B's readout is complete
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_z + 7);
     int *fail = reinterpret_cast<int *>(tmem_holder + 1);
     int *issued = fail + 1;   // S chunks issued so far (for draining after a failure)
 
     if (tid == 0) {
-        for (int i = 0; i < 2 * RM + 6; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 2 * RM + 7; ++i) mbar_init(&bars[i], 1);
+        mbar_init(bar_d, 2);
+        mbar_init(bar_p, 2);
         *fail = 0;
         fence_mbar_init();
     }
@@ -411,30 +415,39 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     // ---- readout D_lin = phi(Q) S_g over the 2F/32 state tiles, then D_s = P V.
     // Tile c of phi sits at column kColA + 32 (c - c0) of the phase [c0, c1) that reads
     // it: one phase for F <= 128; for F = 256 the phi+ tiles, then the phi- tiles.
+    // Two threads issue the readout: a tcgen05.mma with M = 128 keeps its issuing thread
+    // about as long as two tf32 products take on the tensor pipe.  Thread 0 (issuer A)
+    // reads the first half of each phase's tiles into D_lin at kColD, thread 64 (issuer
+    // B) the second half into kColS (the scores' columns, free once P is written); the
+    // epilogue adds the two.  Each accumulator has a fixed issue order.
     const int NC1 = wide ? NC / 2 : NC;
-    bool ok = true;   // thread 0 only
-    // Thread 0 issues the MMAs; a slot whose tile c is read out in the first phase is
-    // refilled (tile c + R) by thread 32 as soon as the tensor cores release it, so the
-    // issue loop never waits for a tile to finish.  A second-phase tile's slot (F = 256
-    // with the 4-slot ring) is refilled by thread 0 itself, after the tile's MMAs.
+    bool ok = true;   // issuers only
+    const int iss = tid == 64 ? 1 : 0;
+    // A slot whose tile c is read out in the first phase is refilled (tile c + R) by
+    // thread 32 as soon as the tensor cores release it, so the issue loops never wait for
+    // a tile to finish.  A second-phase tile's slot (F = 256 with the 4-slot ring) is
+    // refilled by the thread that read it, after the tile's MMAs.
     auto issue_tiles = [&](int c0, int c1) {
         const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
-        for (int c = c0; c < c1 && ok; ++c) {
+        const int hn = (c1 - c0) / 2;
+        const int cb = c0 + iss * hn, ce = cb + hn;
+        const uint32_t dcol = iss ? kColS : kColD;
+        for (int c = cb; c < ce && ok; ++c) {
             const int slot = c % R;
             const uint32_t ph = (uint32_t)(c / R) & 1u;
             if (!mbar_wait(&full[slot], ph, kWaitNs)) { ok = false; break; }
             const uint32_t s_u = smem_u32(slot_ptr(slot));
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
-                mma_tf32_ts(tmem + kColD, tmem + kColA + 32 * (c - c0) + 8 * kk,
-                            smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B), idR, (c | kk) != 0);
+                mma_tf32_ts(tmem + dcol, tmem + kColA + 32 * (c - c0) + 8 * kk,
+                            smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B), idR, (c0 != 0 || c != cb || kk != 0));
             if (c + R < NC) {
                 mma_commit(&empty[slot]);
                 if (c >= NC1) {
                     if (!mbar_wait(&empty[slot], ph, kWaitNs)) { ok = false; break; }
                     mbar_arrive_expect_tx(&full[slot], chunk_bytes);
                     bulk_g2s(slot_ptr(slot), Sg + (size_t)(c + R) * 32 * d, chunk_bytes, &full[slot]);
-                    *issued = c + R + 1;
+                    atomicMax(issued, c + R + 1);
                 }
             }
         }
@@ -448,10 +461,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
             }
             mbar_arrive_expect_tx(&full[slot], chunk_bytes);
             bulk_g2s(slot_ptr(slot), Sg + (size_t)c * 32 * d, chunk_bytes, &full[slot]);
-            *issued = c + 1;
+            atomicMax(issued, c + 1);
         }
     }
-    if (tid == 0) {
+    if (tid == 0 || tid == 64) {
         ok = *fail == 0;
         if (ok) {
             tc_fence_after();
@@ -517,24 +530,31 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         tc_fence_before();
         __syncthreads();
     }
-    if (tid == 0) {
+    if (tid == 0 || tid == 64) {
         ok = ok && *fail == 0;
         if (ok) {
             tc_fence_after();
             if (NC1 < NC) issue_tiles(NC1, NC);
-            if (ok) {
+            // D_s = P V over phi's first d columns.  Issuer B's tiles of the last phase sit
+            // from column 32 (NC - NC1) / 2 on (F with F <= 128, 128 with F = 256); if d
+            // reaches there, A waits for B's readout, else only A's own earlier (in-order)
+            // MMAs read those columns
+            if (iss == 1 && ok) mma_commit(bar_b);
+            if (ok && iss == 0 && d > 16 * (wide ? NC - NC1 : NC) && !mbar_wait(bar_b, 0, kWaitNs)) ok = false;
+            if (ok && iss == 0) {
                 const uint32_t p_u = smem_u32(smem + a.off_p), v_u = smem_u32(smem + a.off_v);
                 const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
                 for (int k = 0; k < B / 16; ++k) {
                     const uint64_t ad = smem_desc(p_u + k * 256, 128, (B / 8) * 128, SWZ_NONE);
                     const uint64_t bd = smem_desc(v_u + 2 * k * 1024, B * 128, 1024, SWZ_128B);
-                    mma_bf16_ss(tmem + kColS, ad, bd, idP, k > 0);
+                    mma_bf16_ss(tmem + kColA, ad, bd, idP, k > 0);
                 }
-                mma_commit(bar_d);
             }
+            if (ok) mma_commit(bar_d);
         }
         if (!ok) {
             atomicOr(fail, 1);
+            if (iss == 1) mbar_arrive(bar_b);
             mbar_arrive(bar_d);   // release the waiting threads
         }
     }
@@ -552,10 +572,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         __nv_bfloat16 *orow0 = a.O + (((size_t)r * B + t) * a.Hq + g * G + hh) * d;
         for (int kd = sub; kd < d / 32; kd += NS) {
             const int c0 = 32 * kd;
-            float dl[32], ds[32];
+            float dl[32], d2[32], ds[32];
             ld_chunk32<kSpread>(tmem + lane_off + kColD + c0, hi, dl);
-            ld_chunk32<kSpread>(tmem + lane_off + kColS + c0, hi, ds);
+            ld_chunk32<kSpread>(tmem + lane_off + kColS + c0, hi, d2);
+            ld_chunk32<kSpread>(tmem + lane_off + kColA + c0, hi, ds);
             tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) dl[i] += d2[i];
             if (valid) {
                 uint32_t pk[16];
 #pragma unroll

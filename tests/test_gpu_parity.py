@@ -47,6 +47,8 @@ SMALL = [
     (W_("bf16_g8_b32_generic", BF16, 2, 8, 1, 128, 64, 32, 18), [64, 32]),
     (W_("bf16_b16_g2", BF16, 3, 4, 2, 128, 128, 16, 19), [16, 0, 80]),
     (W_("bf16_b64_g2", BF16, 2, 4, 2, 64, 128, 64, 20), [128, 64]),
+    # d > F on the two-issuer readout: P'V waits for the second issuer's tiles
+    (W_("bf16_d128_f64_b64", BF16, 2, 4, 2, 128, 64, 64, 27), [64, 0]),
     (W_("f32_mha_f128", F32, 2, 2, 2, 128, 128, 32, 21), [64, 32]),
     # F = 256 on the tensor cores: phi+ and phi- read out in turn; commits in one
     # pass per sign.  GQA with d = 64; 320 commit passes over 152 CTAs; G = 4, B = 16
