@@ -243,7 +243,10 @@ hybrid_status hybrid_state_pack(const hybrid_cfg *cfg, const float *S_logical,
  * reported by hybrid_check. */
 
 /* Bytes of workspace for n_seq sequences of seq_len tokens; 0 when the shape is
- * not supported. */
+ * not supported.  It holds the state of every block in two layouts, du of every
+ * query and key row, the block-state pointers, and the partial sums of dW (at
+ * most 256 slices of d x F) and of dalpha (one per block and query head) that
+ * the backward adds in a fixed order. */
 size_t hybrid_train_workspace_bytes(const hybrid_cfg *cfg, int n_seq, int seq_len);
 
 /* O = block-hybrid attention of every block against the states of the blocks
@@ -258,7 +261,9 @@ hybrid_status hybrid_train_forward(const hybrid_cfg *cfg, const void *Q, const v
  *   dN = dO / D, dD = -(dO . O) / D (D = the merge's denominator),
  *   dw_h = sum (dN . sm_num + dD sm_den), dalpha_h = dw_h w_h (1 - w_h),
  *   dphi(q) = S_{n-1} dN + z_{n-1} dD,  dphi(k_t in B_m) = sum_{n>m} dS_{n-1} v_t + dz_{n-1},
- *   dW = sum over query and key rows of x du^T through phi's two softmaxes. */
+ *   dW = sum over query and key rows of x du^T through phi's two softmaxes.
+ * Partial sums are added in a fixed order (no floating-point atomics), so the
+ * same inputs give the same dW and dalpha bits on every call. */
 hybrid_status hybrid_train_backward(const hybrid_cfg *cfg, const void *Q, const void *K, const void *V,
                                     const void *W, const float *alpha, const void *dO, int n_seq,
                                     int seq_len, void *workspace, size_t workspace_bytes, float *dW,

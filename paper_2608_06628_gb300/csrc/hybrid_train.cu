@@ -32,7 +32,10 @@
 //                   key side: U = K W, V into Tensor Memory, R v + r over the
 //                   R tiles, du_k
 //   k_dw            dW_g = sum over query and key rows of x du^T, split over
-//                   row ranges and added into dW with float atomics
+//                   row ranges; each CTA writes its partial sum
+//   k_grad_reduce   dW and d alpha from the per-CTA and per-block partial sums,
+//                   added in a fixed order, so the gradients are the same bits
+//                   from run to run
 #include <algorithm>
 #include <atomic>
 
@@ -63,9 +66,14 @@ struct TrainArgs {
     float *P, *PT, *R;
     bf16 *dUq, *dUk;
     float *dalpha;
+    float *dap;   // per (sequence, block, state head): the G gate terms, summed by k_grad_reduce
     unsigned *err;
     int n_seq, L, B, Hq, Hkv, d, F, n_blk;
 };
+
+// Partial sums of dW kept for the ordered reduction: at most this many CTAs of
+// k_dw in all, kMaxDwParts / Hkv per state head.
+constexpr int kMaxDwParts = 256;
 
 __host__ __device__ __forceinline__ size_t slot_floats(int Hkv, int d, int F)
 {
@@ -524,7 +532,7 @@ __global__ void __launch_bounds__(kGradThreads, 1) k_phi_grad(const __grid_const
     uint64_t *tbar = bars + 5;      // the phase-one operands have landed
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 6);
     volatile int *fail = reinterpret_cast<volatile int *>(tmem_holder + 1);
-    float *sDw = reinterpret_cast<float *>(tmem_holder + 2);    // [8] dw per head of the group
+    float *sRowDw = reinterpret_cast<float *>(tmem_holder + 2);  // [128] each query row's gate term
     float *sZ = reinterpret_cast<float *>(smem + Lr.off_z);     // z_{n-1} or r_n
     if (tid == 0) {
         for (int i = 0; i < 6; ++i) mbar_init(&bars[i], 1);
@@ -538,7 +546,6 @@ __global__ void __launch_bounds__(kGradThreads, 1) k_phi_grad(const __grid_const
             prefetch_tensormap(&a.tmV);
         }
     }
-    if (tid < 8) sDw[tid] = 0.f;
     if (warp == 0) {
         tmem_alloc(tmem_holder, 512);
         tmem_relinquish();
@@ -836,7 +843,7 @@ __global__ void __launch_bounds__(kGradThreads, 1) k_phi_grad(const __grid_const
             const float Lam = Lp + Ln;
             dD = -(w * A + Lam) * inv;   // -(g . o) / D
             if (part == 0) {
-                if (valid) atomicAdd(&sDw[hl], lambda * A - beta * Lam);
+                sRowDw[lr] = valid ? lambda * A - beta * Lam : 0.f;
                 // column d of [dN | dD | 0] (the rest of that 32-column group is never read)
                 uint8_t *base = smem + Lr.off_y + (uint32_t)(d >> 6) * (128 * 128);
                 uint4 v0;
@@ -897,9 +904,12 @@ __global__ void __launch_bounds__(kGradThreads, 1) k_phi_grad(const __grid_const
             mma_commit(mbar);
         }
         if (tid < G) {
+            // rows t*G + h of head h, added in row order
+            float sum = 0.f;
+            for (int r = tid; r < 128; r += G) sum += sRowDw[r];
             const float al = a.alpha[g * G + tid];
             const float w = 1.f / (1.f + expf(-al));
-            atomicAdd(&a.dalpha[g * G + tid], sDw[tid] * w * (1.f - w));
+            a.dap[(((size_t)s * a.n_blk + n) * Hkv + g) * G + tid] = sum * w * (1.f - w);
         }
         ok = wait_bar(mbar, 0, fail);
         tc_fence_after();
@@ -972,7 +982,7 @@ struct DwArgs {
     // X and dU boxes of 128 rows in the same (token, head) order: Q / dU_q with box
     // {64, G, 128 / G}, K / dU_k with box {64, 1, 128}
     CUtensorMap tmXq, tmUq, tmXk, tmUk;
-    float *dW;
+    float *dWp;   // [Hkv][ctas_per_group][d][F] partial sums, one per CTA
     unsigned *err;
     int n_chunks;      // 128-token chunks of the batch
     int G, d, F, tiles_per_cta, ctas_per_group;
@@ -1062,15 +1072,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwAr
     if (n_tiles > 0) ok = wait_bar(done, 0, fail) && ok;
     tc_fence_after();
     const bool failed = group_sync_failed(1, kThreads, !ok);
-    if (!failed && n_tiles > 0 && tid < d) {
-        float *dst = a.dW + ((size_t)g * d + tid) * F;
+    if (!failed && tid < d) {
+        // this CTA's partial sum (zero without tiles); k_grad_reduce adds the parts in order
+        float4 *dst = reinterpret_cast<float4 *>(a.dWp + (((size_t)g * a.ctas_per_group + part) * d + tid) * F);
         const uint32_t lane_off = (uint32_t)(warp & 3) * 32u << 16;
         float x[32];
         for (int j = 0; j < F / 32; ++j) {
-            tmem_ld32(tmem + lane_off + 32 * j, x);
-            tmem_wait_ld();
+            if (n_tiles > 0) {
+                tmem_ld32(tmem + lane_off + 32 * j, x);
+                tmem_wait_ld();
+            } else {
 #pragma unroll
-            for (int k = 0; k < 32; ++k) atomicAdd(dst + 32 * j + k, x[k]);
+                for (int k = 0; k < 32; ++k) x[k] = 0.f;
+            }
+#pragma unroll
+            for (int k = 0; k < 8; ++k) dst[8 * j + k] = make_float4(x[4 * k], x[4 * k + 1], x[4 * k + 2], x[4 * k + 3]);
         }
     }
     if (tid == 0) {
@@ -1083,6 +1099,38 @@ __global__ void __launch_bounds__(kThreads, 1) k_dw(const __grid_constant__ DwAr
     __syncthreads();
     griddep_launch_dependents();
     if (warp == 0) tmem_dealloc(tmem, 128);
+}
+
+// ---------------------------------------------------------------------------
+// k_grad_reduce: dW[g] = sum over parts p = 0, 1, ... of dWp[g][p] and
+// d alpha[g G + h] = sum over blocks u = 0, 1, ... of dap[u][g][h], each in that order.
+// ---------------------------------------------------------------------------
+struct ReduceArgs {
+    const float *dWp, *dap;
+    float *dW, *dalpha;
+    int Hkv, G, dF, parts, blocks;   // dF = d * F; blocks = n_seq * n_blk
+};
+
+__global__ void k_grad_reduce(const ReduceArgs a)
+{
+    using namespace ptx;
+    griddep_wait();
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    const long long nw = (long long)a.Hkv * a.dF;
+    if (i < nw) {
+        const int g = (int)(i / a.dF);
+        const long long e = i % a.dF;
+        const float *p = a.dWp + (long long)g * a.parts * a.dF + e;
+        float sum = 0.f;
+        for (int k = 0; k < a.parts; ++k) sum += p[(long long)k * a.dF];
+        a.dW[i] = sum;
+    } else if (i < nw + (long long)a.Hkv * a.G) {
+        const int j = (int)(i - nw);   // g G + h
+        float sum = 0.f;
+        for (int u = 0; u < a.blocks; ++u) sum += a.dap[(long long)u * a.Hkv * a.G + j];
+        a.dalpha[j] = sum;
+    }
+    griddep_launch_dependents();
 }
 
 // ---------------------------------------------------------------------------
@@ -1128,6 +1176,7 @@ struct Workspace {
     float *P, *PT;
     bf16 *dUq, *dUk;
     void **ptrs;
+    float *dWp, *dap;
     size_t bytes;
 };
 
@@ -1141,6 +1190,8 @@ Workspace carve(const hybrid_cfg &c, int n_seq, int L, void *base)
     const size_t uq = align_up((size_t)n_seq * L * c.n_q_heads * F * sizeof(bf16));
     const size_t uk = align_up((size_t)n_seq * L * c.n_kv_heads * F * sizeof(bf16));
     const size_t pt = align_up(slots * sizeof(void *));
+    const size_t dwp = align_up((size_t)kMaxDwParts * d * F * sizeof(float));
+    const size_t dap = align_up(slots * c.n_q_heads * sizeof(float));
     Workspace w{};
     uint8_t *p = static_cast<uint8_t *>(base);
     w.P = reinterpret_cast<float *>(p);
@@ -1148,7 +1199,9 @@ Workspace carve(const hybrid_cfg &c, int n_seq, int L, void *base)
     w.dUq = reinterpret_cast<bf16 *>(p ? p + 2 * buf : nullptr);
     w.dUk = reinterpret_cast<bf16 *>(p ? p + 2 * buf + uq : nullptr);
     w.ptrs = reinterpret_cast<void **>(p ? p + 2 * buf + uq + uk : nullptr);
-    w.bytes = 2 * buf + uq + uk + pt;
+    w.dWp = reinterpret_cast<float *>(p ? p + 2 * buf + uq + uk + pt : nullptr);
+    w.dap = reinterpret_cast<float *>(p ? p + 2 * buf + uq + uk + pt + dwp : nullptr);
+    w.bytes = 2 * buf + uq + uk + pt + dwp + dap;
     return w;
 }
 
@@ -1168,6 +1221,7 @@ TrainArgs make_args(const hybrid_cfg &c, int n_seq, int L, const Workspace &w)
     a.R = w.P;   // the backward reuses the decode image's space for R
     a.dUq = w.dUq;
     a.dUk = w.dUk;
+    a.dap = w.dap;
     return a;
 }
 
@@ -1266,8 +1320,6 @@ cudaError_t launch_train_backward(const hybrid_cfg &c, const void *Q, const void
     const int units = n_seq * a.n_blk * a.Hkv;
     const size_t sf = slot_floats(a.Hkv, a.d, a.F);
     cudaError_t e;
-    if ((e = cudaMemsetAsync(dW, 0, (size_t)a.Hkv * a.d * a.F * sizeof(float), st)) != cudaSuccess) return e;
-    if ((e = cudaMemsetAsync(dalpha, 0, (size_t)a.Hq * sizeof(float), st)) != cudaSuccess) return e;
     const RowLayout Lg = make_grad_layout(a.d, a.F, a.B);
     if ((e = opt_in(k_phi_grad<true>, g_opt_q)) != cudaSuccess) return e;
     if ((e = opt_in(k_phi_grad<false>, g_opt_k)) != cudaSuccess) return e;
@@ -1292,20 +1344,34 @@ cudaError_t launch_train_backward(const hybrid_cfg &c, const void *Q, const void
         b.G = G;
         b.n_chunks = (int)((n_tok + 127) / 128);
     }
-    b.dW = dW;
+    b.dWp = w.dWp;
     b.err = err;
     b.d = a.d;
     b.F = a.F;
     const long long tiles = (long long)b.n_chunks * (b.G + 1);
     // one CTA per SM (three 64 KB stages each), the group's tiles split evenly
     int per_group = sm_count() / a.Hkv;
+    if (per_group > kMaxDwParts / a.Hkv) per_group = kMaxDwParts / a.Hkv;
     if (per_group > tiles) per_group = (int)tiles;
     if (per_group < 1) per_group = 1;
     b.tiles_per_cta = (int)((tiles + per_group - 1) / per_group);
     b.ctas_per_group = per_group;
     const size_t dw_smem = kDwStages * ((size_t)2 * 128 * 128 + (size_t)(a.F / 64) * 128 * 128) + 1024 + 1024;
     if ((e = opt_in(k_dw, g_opt_dw)) != cudaSuccess) return e;
-    return launch_pdl(k_dw, dim3((unsigned)(a.Hkv * per_group)), dim3(kThreads), dw_smem, st, b);
+    if ((e = launch_pdl(k_dw, dim3((unsigned)(a.Hkv * per_group)), dim3(kThreads), dw_smem, st, b)) != cudaSuccess)
+        return e;
+    ReduceArgs rd{};
+    rd.dWp = w.dWp;
+    rd.dap = w.dap;
+    rd.dW = dW;
+    rd.dalpha = dalpha;
+    rd.Hkv = a.Hkv;
+    rd.G = a.Hq / a.Hkv;
+    rd.dF = a.d * a.F;
+    rd.parts = per_group;
+    rd.blocks = a.n_seq * a.n_blk;
+    const long long n_out = (long long)a.Hkv * rd.dF + a.Hq;
+    return launch_pdl(k_grad_reduce, dim3((unsigned)((n_out + 255) / 256)), dim3(256), 0, st, rd);
 }
 
 }  // namespace hyb

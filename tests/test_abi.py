@@ -131,11 +131,12 @@ def _al(x):
 
 
 def test_train_workspace_bytes(L):
-    # two state buffers of n_seq * n_blk slots, du of the query and key rows (bf16), the slot pointers
+    # two state buffers of n_seq * n_blk slots, du of the query and key rows (bf16), the slot
+    # pointers, 256 partial d x F sums of dW and one partial dalpha per block and query head
     n, Lq = 8, 2048
     slots = n * (Lq // 32)
     want = 2 * _al(slots * 4 * (2 * 128 * 128 + 2 * 128) * 4) + _al(n * Lq * 16 * 128 * 2) \
-        + _al(n * Lq * 4 * 128 * 2) + _al(slots * 8)
+        + _al(n * Lq * 4 * 128 * 2) + _al(slots * 8) + _al(256 * 128 * 128 * 4) + _al(slots * 16 * 4)
     assert H.hybrid_train_workspace_bytes(cfg(), n, Lq) == want
     # unsupported shapes give 0
     assert H.hybrid_train_workspace_bytes(cfg(dt=H.HYBRID_F32), n, Lq) == 0
