@@ -218,6 +218,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
     // global memory before that kernel has completed
     if (tid == 0) griddep_launch_dependents();
     griddep_wait();
+    // the first unit's Q (ring slot 0), W and K go out from here, before the roles
+    // branch off, so their latency starts as early as possible
+    if (u_begin < u_end && (tid == 0 || tid == 64)) {
+        const int r = u_begin / a.Hkv, g = u_begin % a.Hkv;
+        if (tid == 0) {
+            mbar_arrive_expect_tx(&full[0], (uint32_t)(d / 64) * (G * B * 128));
+            for (int e = 0; e < d / 64; ++e)
+                tma_load_3d(smem + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, &full[0]);
+        } else {
+            uint8_t *kb = smem + a.off_wk + (F / 64) * d * 128;
+            mbar_arrive_expect_tx(xfull, (uint32_t)(F / 64) * (d * 128) + (uint32_t)(d / 64) * (B * 128));
+            for (int f = 0; f < F / 64; ++f)
+                tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xfull);
+            for (int e = 0; e < d / 64; ++e)
+                tma_load_3d(kb + e * (B * 128), &a.tmK, 64 * e, g, r * B, xfull);
+        }
+    }
     const uint32_t tmem = *tmem_holder;
     uint8_t *ring = smem;
     float *zbuf0 = reinterpret_cast<float *>(smem + a.off_z);
@@ -238,7 +255,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                 // item 0: Q of the unit (the first thing g1 needs), issued before the
                 // state pointer has arrived and been checked; a unit whose pointer
                 // fails the check passes its Q item through the ring unused
-                {
+                if (q > 0) {
                     const int slot = q % NS;
                     if (!wait_bar(&empty[slot], ((q / NS) & 1u) ^ 1u, fail, wlim)) break;
                     mbar_arrive_expect_tx(&full[slot], (uint32_t)(d / 64) * (G * B * 128));
@@ -246,6 +263,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                         tma_load_3d(ring + (size_t)slot * slot_bytes + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B,
                                     &full[slot]);
                     ++q;
+                } else {
+                    ++q;   // issued in the prologue
                 }
                 float *Sg = state_at(a, raw, u);
                 if (!Sg) continue;
@@ -385,7 +404,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             bool ok = true;
             if (nx > 0) ok = wait_bar(xfree, (nx - 1) & 1u, fail, wlim);
             if (__any_sync(0xffffffffu, !ok)) break;
-            if (lane == 0) {
+            if (lane == 0 && nx > 0) {   // the first unit's W and K went out in the prologue
                 mbar_arrive_expect_tx(xfull, xbytes);
                 for (int f = 0; f < F / 64; ++f)
                     tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xfull);
