@@ -318,8 +318,11 @@ def small_config_context(dev, warmup=5, iters=20):
 def large_config_context(dev, warmup=3, iters=15, n_req=None):
     """Context for the two other large configurations (not part of the value):
     the per-call device time of the step (hybrid_block_attn) and of the block
-    commit (hybrid_commit_block, B tokens), each launched directly, median of
-    iters after warmup.  c4 is one layer of the decode loop (32 requests, MHA);
+    commit (hybrid_commit_block, B tokens), replayed from a CUDA graph of iters
+    calls over the rotating buffer sets (graph_us, the figure the fraction of HBM
+    is taken from) and launched directly (direct_us_median, which for a call of a
+    few tens of microseconds also holds the host's launch latency).  c4 is one
+    layer of the decode loop (32 requests, MHA);
     its state fits in L2, so it rotates enough buffer sets that each call misses
     L2.  c5 (256 requests, F = 256) holds a 1.08 GB state and uses one set.  The
     kernels' cost does not depend on the state's values: states start empty.
@@ -350,26 +353,42 @@ def large_config_context(dev, warmup=3, iters=15, n_req=None):
             sets.append(dict(pool=pool, ptrs=ptrs, Q=Q, K=K, V=V, O=torch.empty_like(Q)))
         stream = torch.cuda.current_stream(dev)
         calls = {
-            "step": lambda s: H.hybrid_block_attn(cfg, s["Q"], s["K"], s["V"], W, alpha, s["ptrs"], wl.n_req,
-                                                  s["O"], stream.cuda_stream, check=False),
-            "commit": lambda s: H.hybrid_commit_block(cfg, s["K"], s["V"], wl.B, W, s["ptrs"], wl.n_req,
-                                                      stream.cuda_stream, check=False),
+            "step": lambda s, st: H.hybrid_block_attn(cfg, s["Q"], s["K"], s["V"], W, alpha, s["ptrs"], wl.n_req,
+                                                      s["O"], st.cuda_stream, check=False),
+            "commit": lambda s, st: H.hybrid_commit_block(cfg, s["K"], s["V"], wl.B, W, s["ptrs"], wl.n_req,
+                                                          st.cuda_stream, check=False),
         }
         res = {"buffer_sets": n_sets}
+        side = torch.cuda.Stream(dev)
         for name, fn in calls.items():
             for i in range(warmup):
-                fn(sets[i % n_sets])
+                fn(sets[i % n_sets], stream)
             evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                    for _ in range(iters)]
             for i, (a_, b_) in enumerate(evs):
                 a_.record(stream)
-                fn(sets[i % n_sets])
+                fn(sets[i % n_sets], stream)
                 b_.record(stream)
             torch.cuda.synchronize()
-            us = sorted(a_.elapsed_time(b_) for a_, b_ in evs)[iters // 2] * 1e3
+            direct = sorted(a_.elapsed_time(b_) for a_, b_ in evs)[iters // 2] * 1e3
+            side.wait_stream(stream)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=side):
+                for i in range(iters):
+                    fn(sets[i % n_sets], side)
+            torch.cuda.synchronize()
+            g.replay()
+            torch.cuda.synchronize()
+            a_, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a_.record(stream)
+            g.replay()
+            b_.record(stream)
+            torch.cuda.synchronize()
+            us = a_.elapsed_time(b_) * 1e3 / iters
+            del g
             nbytes = ab["attn"] if name == "step" else ab["commit"]
-            res[name] = {"us_median": us, "algorithmic_bytes": nbytes, "GBps": nbytes / us / 1e3,
-                         "frac_of_measured_hbm": nbytes / us / 1e3 / hbm}
+            res[name] = {"graph_us": us, "direct_us_median": direct, "algorithmic_bytes": nbytes,
+                         "GBps": nbytes / us / 1e3, "frac_of_measured_hbm": nbytes / us / 1e3 / hbm}
         status = H.hybrid_check(check=False)
         if status != H.HYBRID_OK:
             raise SystemExit(f"device error in the large-config context: {H.hybrid_status_str(status)}")
