@@ -53,6 +53,7 @@ struct TcAttnArgs {
     __nv_bfloat16 *O;
     unsigned *err;
     int B, Hq, Hkv, G, d, F;
+    int n_units;        // n_req Hkv (request, state head) units, u = r Hkv + g
     int n_slots;
     float scale_log2;   // log2(e) / sqrt(d)
     float inv_sqrt_d;
@@ -162,35 +163,31 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int r = blockIdx.x / a.Hkv, g = blockIdx.x % a.Hkv;
     const int d = a.d, F = a.F, B = a.B, G = a.G;
     const int NC = (2 * F) / 32;
     const int Mv = G * B;
     const uint32_t chunk_bytes = (uint32_t)d * 128;
     const bool wide = F > 128;   // phi+ and phi- take turns in U's columns
     const int RM = a.n_slots + (wide ? kExtraSlots : 0);   // ring slots at most
-
-    const float *state = reinterpret_cast<const float *>(a.states[r]);
-    if (!state_ptr_ok(state)) {
-        if (tid == 0) raise_error(a.err, ERR_BAD_STATE_PTR);
-        return;
-    }
-    const float *Sg = state + (size_t)g * head_floats(d, F);
-    const float *zg = Sg + (size_t)2 * F * d;
+    // the CTA's contiguous range of units
+    const int per = a.n_units / (int)gridDim.x, rem = a.n_units % (int)gridDim.x;
+    const int u_begin = (int)blockIdx.x * per + min((int)blockIdx.x, rem);
+    const int u_end = u_begin + per + ((int)blockIdx.x < rem ? 1 : 0);
 
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + a.off_bar);
     uint64_t *full = bars;
     uint64_t *empty = bars + RM;
     uint64_t *bar_z = bars + 2 * RM;
     uint64_t *bar_u = bar_z + 1;
-    uint64_t *bar_d = bar_z + 2;    // both issuers: D_lin halves and D_s are complete
+    uint64_t *bar_d = bar_z + 2;    // both issuers: D_lin halves and D_s are complete (every
+                                    // shared-memory operand of the unit has been read)
     uint64_t *bar_p = bar_z + 3;    // F = 256, both issuers: the phi+ readout is done
     uint64_t *bar_u2 = bar_z + 4;   // F = 256: U = Q W formed again, for phi-
     uint64_t *bar_ld = bar_z + 5;   // Q, K, V and W have landed
     uint64_t *bar_b = bar_z + 6;    // issuer B's readout is complete
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_z + 7);
     int *fail = reinterpret_cast<int *>(tmem_holder + 1);
-    int *issued = fail + 1;   // S chunks issued so far (for draining after a failure)
+    int *issued = fail + 1;   // S chunks of the unit issued so far (for draining after a failure)
 
     if (tid == 0) {
         for (int i = 0; i < 2 * RM + 7; ++i) mbar_init(&bars[i], 1);
@@ -207,8 +204,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
 
-    // ---- producer: Q, K, V, W (TMA), z and the first S tiles (bulk copies of the state image)
-    if (tid == 0) {
+    // the first unit from u on whose state pointer is usable (u_end if none); each
+    // unusable pointer is reported once and its unit skipped
+    auto next_unit = [&](int u) -> int {
+        for (; u < u_end; ++u) {
+            if (state_ptr_ok(a.states[u / a.Hkv])) break;
+            if (tid == 0) raise_error(a.err, ERR_BAD_STATE_PTR);
+        }
+        return u;
+    };
+    auto head_state = [&](int u) -> const float * {
+        return reinterpret_cast<const float *>(a.states[u / a.Hkv]) + (size_t)(u % a.Hkv) * head_floats(d, F);
+    };
+    // ---- loads of unit u (one thread): Q, K, V, W (TMA), z and the first S tiles
+    // (bulk copies of the state image)
+    auto issue_loads = [&](int u) {
+        const int r = u / a.Hkv, g = u % a.Hkv;
+        const float *Sg = head_state(u);
         mbar_arrive_expect_tx(bar_ld, (uint32_t)(Mv + 2 * B + F) * d * 2);
         for (int c = 0; c < d / 64; ++c) {
             if (kSpread) {
@@ -224,383 +236,418 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         }
         for (int f = 0; f < F / 64; ++f) tma_load_2d(smem + a.off_w + f * (d * 128), &a.tmW, 64 * f, g * d, bar_ld);
         mbar_arrive_expect_tx(bar_z, 2 * F * 4);
-        bulk_g2s(smem + a.off_z, zg, 2 * F * 4, bar_z);
+        bulk_g2s(smem + a.off_z, Sg + (size_t)2 * F * d, 2 * F * 4, bar_z);
         const int pre = NC < a.n_slots ? NC : a.n_slots;
         for (int c = 0; c < pre; ++c) {
             mbar_arrive_expect_tx(&full[c], chunk_bytes);
             bulk_g2s(smem + (size_t)c * chunk_bytes, Sg + (size_t)c * 32 * d, chunk_bytes, &full[c]);
         }
         *issued = pre;
-    }
-
-    // ---- U = Q W_g and scores = Q K^T.  W and V are MN-major: 64-wide panels of
-    // d (W) or B (V) rows, 8-row groups 1024 bytes apart.
-    if (tid == 0) {
-        if (mbar_wait(bar_ld, 0, kWaitNs)) {
-            tc_fence_after();
-            const uint32_t q_u = smem_u32(smem + a.off_q), w_u = smem_u32(smem + a.off_w),
-                           k_u = smem_u32(smem + a.off_k);
-            const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
-            const uint32_t idS = instr_desc(FMT_BF16, FMT_BF16, false, false, 128, B);
-            for (int k = 0; k < d / 16; ++k) {
-                const uint64_t ad = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
-                const uint64_t bw = smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
-                const uint64_t bk = smem_desc(k_u + (k >> 2) * (B * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
-                mma_bf16_ss(tmem + kColA, ad, bw, idU, k > 0);
-                mma_bf16_ss(tmem + kColS, ad, bk, idS, k > 0);
-            }
-            mma_commit(bar_u);
-        } else {
-            atomicOr(fail, 1);
-            mbar_arrive(bar_u);
-        }
-    }
-    if (!mbar_wait(bar_u, 0, kWaitNs)) atomicOr(fail, 1);
-    tc_fence_after();
-
-    // ring slot s: the dedicated slots, then (F = 256, phi- from phi+) W's and Q's space
-    auto slot_ptr = [&](int sl) -> uint8_t * {
-        if (sl < a.n_slots) return smem + (size_t)sl * chunk_bytes;
-        sl -= a.n_slots;
-        return sl < 4 ? smem + a.off_w + (size_t)sl * chunk_bytes : smem + a.off_q + (size_t)(sl - 4) * chunk_bytes;
     };
 
-    // row statistics: in Q's buffer once Q is no longer read (F <= 128), else their own
-    float *stat = reinterpret_cast<float *>(smem + a.off_st);  // [3][128] m, l, lin_den
-    float *ex = stat + 3 * 128;                                 // [8][2][128] exchange
-    // Thread -> (TMEM lane, column subset).  Default: lane 32 q4 + lane and the warp's
-    // half as subset, two threads per row.  Spread (G = 1, B = 64): query row i sits on
-    // lane 32 (i / 16) + i % 16, so the rows occupy all four lane quarters (and SM
-    // sub-partitions), and a warp's two 16-thread halves take the same 16 lanes at
-    // different columns: four threads per row.
-    const int q4 = warp & 3, half = warp >> 2;
-    const int hi = kSpread ? lane >> 4 : 0;
-    const int row = kSpread ? 32 * q4 + (lane & 15) : 32 * q4 + lane;   // TMEM lane of the query row
-    const int qrow = kSpread ? 16 * q4 + (lane & 15) : row;              // query row t G + hh
-    const uint32_t lane_off = (uint32_t)(32 * q4) << 16;
-    const bool valid = qrow < Mv;
-    constexpr int NS = kSpread ? 4 : 2;               // column subsets per row
-    const int sub = kSpread ? 2 * half + hi : half;   // owns the chunks k with k % NS == sub
-    const int nsc = B / 16;       // 16-column chunks of scores
-    const int nfc = F / 32;       // 32-column chunks of U
-    // in the spread layout a row's partial results meet across lanes l and l ^ 16 first
-    auto comb_max = [&](float x) { return kSpread ? fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 16)) : x; };
-    auto comb_min = [&](float x) { return kSpread ? fminf(x, __shfl_xor_sync(0xffffffffu, x, 16)) : x; };
-    auto comb_add = [&](float x) { return kSpread ? x + __shfl_xor_sync(0xffffffffu, x, 16) : x; };
+    // Units run one after another; the barriers used once per unit complete with
+    // the parity of the unit's index it in this CTA.  Ring slot s has had fills and
+    // releases of earlier units; fmask / emask bit s hold the parity of their counts.
+    uint32_t fmask = 0, emask = 0, it = 0, n_u2 = 0;
+    int u = next_unit(u_begin);
+    if (tid == 0 && u < u_end) issue_loads(u);
+    while (u < u_end) {
+        const uint32_t up = it & 1u;
+        const int r = u / a.Hkv, g = u % a.Hkv;
+        const float *Sg = head_state(u);
+        // phase parity of fill j (or release j) of ring slot s in this unit
+        auto fph = [&](int s, int j) -> uint32_t { return ((fmask >> s) & 1u) ^ ((uint32_t)j & 1u); };
+        auto eph = [&](int s, int j) -> uint32_t { return ((emask >> s) & 1u) ^ ((uint32_t)j & 1u); };
 
-    // ---- pass 1: local extrema
-    {
-        float ms = -INFINITY, mx = -INFINITY, mn = INFINITY;
-        for (int k = sub; k < nsc; k += NS) {
-            float v[16];
-            ld_chunk16<kSpread>(tmem + lane_off + kColS + 16 * k, hi, v);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 16; ++i) ms = fmaxf(ms, v[i]);
-        }
-        for (int k = sub; k < nfc; k += NS) {
-            float v[32];
-            ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, v[i]); mn = fminf(mn, v[i]); }
-        }
-        ex[0 * 256 + half * 128 + row] = comb_max(ms);
-        ex[1 * 256 + half * 128 + row] = comb_max(mx);
-        ex[2 * 256 + half * 128 + row] = comb_min(mn);
-    }
-    __syncthreads();
-    // F = 256: while every valid row's range of U stays within kRecipRange, phi- follows
-    // from phi+ (phi-_j = e^(mn - mx) / (sp sn phi+_j), both sides far from underflow), so
-    // U = Q W is not formed again and W's and Q's space takes six more state tiles now
-    bool recip = false;
-    if (wide) {
-        const float rng = fmaxf(ex[1 * 256 + row], ex[1 * 256 + 128 + row]) -
-                          fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]);
-        recip = __syncthreads_and(!valid || rng <= kRecipRange) != 0;
-    }
-    const int R = recip ? min(NC, RM) : a.n_slots;   // ring slots in use
-    if (tid == 0 && R > a.n_slots && *fail == 0) {
-        for (int c = a.n_slots; c < R; ++c) {
-            mbar_arrive_expect_tx(&full[c], chunk_bytes);
-            bulk_g2s(slot_ptr(c), Sg + (size_t)c * 32 * d, chunk_bytes, &full[c]);
-        }
-        *issued = R;
-    }
-    if (!mbar_wait(bar_z, 0, kWaitNs)) atomicOr(fail, 1);
-
-    // ---- pass 2: exponentials, P, unnormalised phi halves, partial sums
-    {
-        const float m_raw = fmaxf(ex[0 * 256 + row], ex[0 * 256 + 128 + row]);
-        const float mx = fmaxf(ex[1 * 256 + row], ex[1 * 256 + 128 + row]);
-        const float mn = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]);
-        float l = 0.f, sp = 0.f, sn = 0.f, lp = 0.f, ln = 0.f;
-        for (int k = sub; k < nsc; k += NS) {
-            float v[16];
-            ld_chunk16<kSpread>(tmem + lane_off + kColS + 16 * k, hi, v);
-            tmem_wait_ld();
-            uint32_t pk[8];
-#pragma unroll
-            for (int i = 0; i < 16; i += 2) {
-                const float p0 = exp2f((v[i] - m_raw) * a.scale_log2);
-                const float p1 = exp2f((v[i + 1] - m_raw) * a.scale_log2);
-                pk[i / 2] = pack_bf16x2(p0, p1);
-                const __nv_bfloat162 b2 = *reinterpret_cast<const __nv_bfloat162 *>(&pk[i / 2]);
-                l += __low2float(b2) + __high2float(b2);   // sum what the MMA will use
-            }
-            // P is K-major without swizzle: core matrices of 8 rows x 16 bytes
-            uint8_t *prow = smem + a.off_p + (row >> 3) * (B / 8) * 128 + (row & 7) * 16;
-            *reinterpret_cast<uint4 *>(prow + (2 * k) * 128) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            *reinterpret_cast<uint4 *>(prow + (2 * k + 1) * 128) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-        }
-        const float *zs = reinterpret_cast<const float *>(smem + a.off_z);
-        const float mxl = mx * kLog2e, mnl = mn * kLog2e;
-        for (int k = sub; k < nfc; k += NS) {
-            float u[32], ep[32], en[32];
-            ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, u);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-                ep[i] = exp2f(fmaf(u[i], kLog2e, -mxl));
-                en[i] = exp2f(fmaf(-u[i], kLog2e, mnl));
-                sp += ep[i];
-                sn += en[i];
-                lp = fmaf(ep[i], zs[32 * k + i], lp);
-                ln = fmaf(en[i], zs[F + 32 * k + i], ln);
-            }
-            st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, ep);
-            if (!wide) st_chunk32<kSpread>(tmem + lane_off + kColA + F + 32 * k, hi, en);   // F = 256: formed later
-        }
-        ex[3 * 256 + half * 128 + row] = comb_add(l);
-        ex[4 * 256 + half * 128 + row] = comb_add(sp);
-        ex[5 * 256 + half * 128 + row] = comb_add(sn);
-        ex[6 * 256 + half * 128 + row] = comb_add(lp);
-        ex[7 * 256 + half * 128 + row] = comb_add(ln);
-        if (half == 0) stat[row] = m_raw * a.inv_sqrt_d;
-        tmem_wait_st();
-    }
-    __syncthreads();
-
-    // ---- pass 3: normalise phi in place (rounded to tf32), row statistics
-    {
-        const float sp = ex[4 * 256 + row] + ex[4 * 256 + 128 + row];
-        const float sn = ex[5 * 256 + row] + ex[5 * 256 + 128 + row];
-        const float isp = 1.f / sp, isn = 1.f / sn;
-        for (int k = sub; k < nfc; k += NS) {
-            float v[32];
-            ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = tf32_round(v[i] * isp);
-            st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
-            if (wide) continue;
-            ld_chunk32<kSpread>(tmem + lane_off + kColA + F + 32 * k, hi, v);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = tf32_round(v[i] * isn);
-            st_chunk32<kSpread>(tmem + lane_off + kColA + F + 32 * k, hi, v);
-        }
-        if (half == 0) {
-            stat[128 + row] = ex[3 * 256 + row] + ex[3 * 256 + 128 + row];
-            const float lp = ex[6 * 256 + row] + ex[6 * 256 + 128 + row];
-            const float ln = ex[7 * 256 + row] + ex[7 * 256 + 128 + row];
-            stat[256 + row] = lp * isp + ln * isn;
-        }
-        tmem_wait_st();
-    }
-    fence_proxy_async_smem();
-    tc_fence_before();
-    __syncthreads();
-
-    // ---- readout D_lin = phi(Q) S_g over the 2F/32 state tiles, then D_s = P V.
-    // Tile c of phi sits at column kColA + 32 (c - c0) of the phase [c0, c1) that reads
-    // it: one phase for F <= 128; for F = 256 the phi+ tiles, then the phi- tiles.
-    // Two threads issue the readout: a tcgen05.mma with M = 128 keeps its issuing thread
-    // about as long as two tf32 products take on the tensor pipe.  Thread 0 (issuer A)
-    // reads the first half of each phase's tiles into D_lin at kColD, thread 64 (issuer
-    // B) the second half into kColS (the scores' columns, free once P is written); the
-    // epilogue adds the two.  Each accumulator has a fixed issue order.
-    const int NC1 = wide ? NC / 2 : NC;
-    bool ok = true;   // issuers only
-    const int iss = tid == 64 ? 1 : 0;
-    // A slot whose tile c is read out in the first phase is refilled (tile c + R) by
-    // thread 32 as soon as the tensor cores release it, so the issue loops never wait for
-    // a tile to finish.  A second-phase tile's slot (F = 256 with the 4-slot ring) is
-    // refilled by the thread that read it, after the tile's MMAs.
-    auto issue_tiles = [&](int c0, int c1) {
-        const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
-        const int hn = (c1 - c0) / 2;
-        const int cb = c0 + iss * hn, ce = cb + hn;
-        const uint32_t dcol = iss ? kColS : kColD;
-        for (int c = cb; c < ce && ok; ++c) {
-            const int slot = c % R;
-            const uint32_t ph = (uint32_t)(c / R) & 1u;
-            if (!mbar_wait(&full[slot], ph, kWaitNs)) { ok = false; break; }
-            const uint32_t s_u = smem_u32(slot_ptr(slot));
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-                mma_tf32_ts(tmem + dcol, tmem + kColA + 32 * (c - c0) + 8 * kk,
-                            smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B), idR, (c0 != 0 || c != cb || kk != 0));
-            if (c + R < NC) {
-                mma_commit(&empty[slot]);
-                if (c >= NC1) {
-                    if (!mbar_wait(&empty[slot], ph, kWaitNs)) { ok = false; break; }
-                    mbar_arrive_expect_tx(&full[slot], chunk_bytes);
-                    bulk_g2s(slot_ptr(slot), Sg + (size_t)(c + R) * 32 * d, chunk_bytes, &full[slot]);
-                    atomicMax(issued, c + R + 1);
+        // ---- U = Q W_g and scores = Q K^T.  W and V are MN-major: 64-wide panels of
+        // d (W) or B (V) rows, 8-row groups 1024 bytes apart.
+        if (tid == 0) {
+            if (mbar_wait(bar_ld, up, kWaitNs)) {
+                tc_fence_after();
+                const uint32_t q_u = smem_u32(smem + a.off_q), w_u = smem_u32(smem + a.off_w),
+                               k_u = smem_u32(smem + a.off_k);
+                const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
+                const uint32_t idS = instr_desc(FMT_BF16, FMT_BF16, false, false, 128, B);
+                for (int k = 0; k < d / 16; ++k) {
+                    const uint64_t ad = smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
+                    const uint64_t bw = smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B);
+                    const uint64_t bk = smem_desc(k_u + (k >> 2) * (B * 128) + (k & 3) * 32, 16, 1024, SWZ_128B);
+                    mma_bf16_ss(tmem + kColA, ad, bw, idU, k > 0);
+                    mma_bf16_ss(tmem + kColS, ad, bk, idS, k > 0);
                 }
-            }
-        }
-    };
-    if (tid == 32 && *fail == 0) {
-        for (int c = R; c < NC && c - R < NC1; ++c) {
-            const int slot = c % R;
-            if (!mbar_wait(&empty[slot], (uint32_t)((c - R) / R) & 1u, kWaitNs)) {
+                mma_commit(bar_u);
+            } else {
                 atomicOr(fail, 1);
-                break;
+                mbar_arrive(bar_u);
             }
-            mbar_arrive_expect_tx(&full[slot], chunk_bytes);
-            bulk_g2s(slot_ptr(slot), Sg + (size_t)c * 32 * d, chunk_bytes, &full[slot]);
-            atomicMax(issued, c + 1);
         }
-    }
-    if (tid == 0 || tid == 64) {
-        ok = *fail == 0;
-        if (ok) {
-            tc_fence_after();
-            issue_tiles(0, NC1);
+        if (!mbar_wait(bar_u, up, kWaitNs)) atomicOr(fail, 1);
+        tc_fence_after();
+
+        // ring slot s: the dedicated slots, then (F = 256, phi- from phi+) W's and Q's space
+        auto slot_ptr = [&](int sl) -> uint8_t * {
+            if (sl < a.n_slots) return smem + (size_t)sl * chunk_bytes;
+            sl -= a.n_slots;
+            return sl < 4 ? smem + a.off_w + (size_t)sl * chunk_bytes : smem + a.off_q + (size_t)(sl - 4) * chunk_bytes;
+        };
+
+        // row statistics: in Q's buffer once Q is no longer read (F <= 128), else their own
+        float *stat = reinterpret_cast<float *>(smem + a.off_st);  // [3][128] m, l, lin_den
+        float *ex = stat + 3 * 128;                                 // [8][2][128] exchange
+        // Thread -> (TMEM lane, column subset).  Default: lane 32 q4 + lane and the warp's
+        // half as subset, two threads per row.  Spread (G = 1, B = 64): query row i sits on
+        // lane 32 (i / 16) + i % 16, so the rows occupy all four lane quarters (and SM
+        // sub-partitions), and a warp's two 16-thread halves take the same 16 lanes at
+        // different columns: four threads per row.
+        const int q4 = warp & 3, half = warp >> 2;
+        const int hi = kSpread ? lane >> 4 : 0;
+        const int row = kSpread ? 32 * q4 + (lane & 15) : 32 * q4 + lane;   // TMEM lane of the query row
+        const int qrow = kSpread ? 16 * q4 + (lane & 15) : row;              // query row t G + hh
+        const uint32_t lane_off = (uint32_t)(32 * q4) << 16;
+        const bool valid = qrow < Mv;
+        constexpr int NS = kSpread ? 4 : 2;               // column subsets per row
+        const int sub = kSpread ? 2 * half + hi : half;   // owns the chunks k with k % NS == sub
+        const int nsc = B / 16;       // 16-column chunks of scores
+        const int nfc = F / 32;       // 32-column chunks of U
+        // in the spread layout a row's partial results meet across lanes l and l ^ 16 first
+        auto comb_max = [&](float x) { return kSpread ? fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 16)) : x; };
+        auto comb_min = [&](float x) { return kSpread ? fminf(x, __shfl_xor_sync(0xffffffffu, x, 16)) : x; };
+        auto comb_add = [&](float x) { return kSpread ? x + __shfl_xor_sync(0xffffffffu, x, 16) : x; };
+
+        // ---- pass 1: local extrema
+        {
+            float ms = -INFINITY, mx = -INFINITY, mn = INFINITY;
+            for (int k = sub; k < nsc; k += NS) {
+                float v[16];
+                ld_chunk16<kSpread>(tmem + lane_off + kColS + 16 * k, hi, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 16; ++i) ms = fmaxf(ms, v[i]);
+            }
+            for (int k = sub; k < nfc; k += NS) {
+                float v[32];
+                ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) { mx = fmaxf(mx, v[i]); mn = fminf(mn, v[i]); }
+            }
+            ex[0 * 256 + half * 128 + row] = comb_max(ms);
+            ex[1 * 256 + half * 128 + row] = comb_max(mx);
+            ex[2 * 256 + half * 128 + row] = comb_min(mn);
         }
+        __syncthreads();
+        // F = 256: while every valid row's range of U stays within kRecipRange, phi- follows
+        // from phi+ (phi-_j = e^(mn - mx) / (sp sn phi+_j), both sides far from underflow), so
+        // U = Q W is not formed again and W's and Q's space takes six more state tiles now
+        bool recip = false;
         if (wide) {
-            if (ok) mma_commit(bar_p);
-            else mbar_arrive(bar_p);
+            const float rng = fmaxf(ex[1 * 256 + row], ex[1 * 256 + 128 + row]) -
+                              fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]);
+            recip = __syncthreads_and(!valid || rng <= kRecipRange) != 0;
         }
-    }
-    if (wide) {
-        // the tensor cores are done with phi+; phi- takes its columns
-        if (!mbar_wait(bar_p, 0, kWaitNs)) atomicOr(fail, 1);
-        if (recip) {
-            // phi-_j = e^(mn - mx) isp isn / phi+_j, rounded to tf32
-            tc_fence_after();
+        const int R = recip ? min(NC, RM) : a.n_slots;   // ring slots in use
+        if (tid == 0 && R > a.n_slots && *fail == 0) {
+            for (int c = a.n_slots; c < R; ++c) {
+                mbar_arrive_expect_tx(&full[c], chunk_bytes);
+                bulk_g2s(slot_ptr(c), Sg + (size_t)c * 32 * d, chunk_bytes, &full[c]);
+            }
+            *issued = R;
+        }
+        if (!mbar_wait(bar_z, up, kWaitNs)) atomicOr(fail, 1);
+
+        // ---- pass 2: exponentials, P, unnormalised phi halves, partial sums
+        {
+            const float m_raw = fmaxf(ex[0 * 256 + row], ex[0 * 256 + 128 + row]);
             const float mx = fmaxf(ex[1 * 256 + row], ex[1 * 256 + 128 + row]);
             const float mn = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]);
-            const float isp = 1.f / (ex[4 * 256 + row] + ex[4 * 256 + 128 + row]);
-            const float isn = 1.f / (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
-            const float kr = exp2f((mn - mx) * kLog2e) * isp * isn;
-            for (int k = sub; k < nfc; k += NS) {
-                float v[32];
-                ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
+            float l = 0.f, sp = 0.f, sn = 0.f, lp = 0.f, ln = 0.f;
+            for (int k = sub; k < nsc; k += NS) {
+                float v[16];
+                ld_chunk16<kSpread>(tmem + lane_off + kColS + 16 * k, hi, v);
                 tmem_wait_ld();
+                uint32_t pk[8];
 #pragma unroll
-                for (int i = 0; i < 32; ++i) v[i] = tf32_round(__fdividef(kr, v[i]));
-                st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
-            }
-            tmem_wait_st();
-        } else {
-            // form U = Q W_g again in phi+'s columns
-            if (tid == 0) {
-                ok = ok && *fail == 0;
-                if (ok) {
-                    tc_fence_after();
-                    const uint32_t q_u = smem_u32(smem + a.off_q), w_u = smem_u32(smem + a.off_w);
-                    const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
-                    for (int k = 0; k < d / 16; ++k)
-                        mma_bf16_ss(tmem + kColA,
-                                    smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B),
-                                    smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B), idU, k > 0);
-                    mma_commit(bar_u2);
-                } else {
-                    mbar_arrive(bar_u2);
+                for (int i = 0; i < 16; i += 2) {
+                    const float p0 = exp2f((v[i] - m_raw) * a.scale_log2);
+                    const float p1 = exp2f((v[i + 1] - m_raw) * a.scale_log2);
+                    pk[i / 2] = pack_bf16x2(p0, p1);
+                    const __nv_bfloat162 b2 = *reinterpret_cast<const __nv_bfloat162 *>(&pk[i / 2]);
+                    l += __low2float(b2) + __high2float(b2);   // sum what the MMA will use
                 }
+                // P is K-major without swizzle: core matrices of 8 rows x 16 bytes
+                uint8_t *prow = smem + a.off_p + (row >> 3) * (B / 8) * 128 + (row & 7) * 16;
+                *reinterpret_cast<uint4 *>(prow + (2 * k) * 128) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                *reinterpret_cast<uint4 *>(prow + (2 * k + 1) * 128) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
             }
-            if (!mbar_wait(bar_u2, 0, kWaitNs)) atomicOr(fail, 1);
-            tc_fence_after();
-            // phi- = softmax(-U), from the same extremum and sum as pass 2, rounded to tf32
-            const float mnl = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]) * kLog2e;
-            const float isn = 1.f / (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
+            const float *zs = reinterpret_cast<const float *>(smem + a.off_z);
+            const float mxl = mx * kLog2e, mnl = mn * kLog2e;
+            for (int k = sub; k < nfc; k += NS) {
+                float u[32], ep[32], en[32];
+                ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, u);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    ep[i] = exp2f(fmaf(u[i], kLog2e, -mxl));
+                    en[i] = exp2f(fmaf(-u[i], kLog2e, mnl));
+                    sp += ep[i];
+                    sn += en[i];
+                    lp = fmaf(ep[i], zs[32 * k + i], lp);
+                    ln = fmaf(en[i], zs[F + 32 * k + i], ln);
+                }
+                st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, ep);
+                if (!wide) st_chunk32<kSpread>(tmem + lane_off + kColA + F + 32 * k, hi, en);   // F = 256: formed later
+            }
+            ex[3 * 256 + half * 128 + row] = comb_add(l);
+            ex[4 * 256 + half * 128 + row] = comb_add(sp);
+            ex[5 * 256 + half * 128 + row] = comb_add(sn);
+            ex[6 * 256 + half * 128 + row] = comb_add(lp);
+            ex[7 * 256 + half * 128 + row] = comb_add(ln);
+            if (half == 0) stat[row] = m_raw * a.inv_sqrt_d;
+            tmem_wait_st();
+        }
+        __syncthreads();
+
+        // ---- pass 3: normalise phi in place (rounded to tf32), row statistics
+        {
+            const float sp = ex[4 * 256 + row] + ex[4 * 256 + 128 + row];
+            const float sn = ex[5 * 256 + row] + ex[5 * 256 + 128 + row];
+            const float isp = 1.f / sp, isn = 1.f / sn;
             for (int k = sub; k < nfc; k += NS) {
                 float v[32];
                 ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
                 tmem_wait_ld();
 #pragma unroll
-                for (int i = 0; i < 32; ++i) v[i] = tf32_round(exp2f(fmaf(-v[i], kLog2e, mnl)) * isn);
+                for (int i = 0; i < 32; ++i) v[i] = tf32_round(v[i] * isp);
                 st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
+                if (wide) continue;
+                ld_chunk32<kSpread>(tmem + lane_off + kColA + F + 32 * k, hi, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) v[i] = tf32_round(v[i] * isn);
+                st_chunk32<kSpread>(tmem + lane_off + kColA + F + 32 * k, hi, v);
+            }
+            if (half == 0) {
+                stat[128 + row] = ex[3 * 256 + row] + ex[3 * 256 + 128 + row];
+                const float lp = ex[6 * 256 + row] + ex[6 * 256 + 128 + row];
+                const float ln = ex[7 * 256 + row] + ex[7 * 256 + 128 + row];
+                stat[256 + row] = lp * isp + ln * isn;
             }
             tmem_wait_st();
         }
+        fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
-    }
-    if (tid == 0 || tid == 64) {
-        ok = ok && *fail == 0;
-        if (ok) {
-            tc_fence_after();
-            if (NC1 < NC) issue_tiles(NC1, NC);
-            // D_s = P V over phi's first d columns.  Issuer B's tiles of the last phase sit
-            // from column 32 (NC - NC1) / 2 on (F with F <= 128, 128 with F = 256); if d
-            // reaches there, A waits for B's readout, else only A's own earlier (in-order)
-            // MMAs read those columns
-            if (iss == 1 && ok) mma_commit(bar_b);
-            if (ok && iss == 0 && d > 16 * (wide ? NC - NC1 : NC) && !mbar_wait(bar_b, 0, kWaitNs)) ok = false;
-            if (ok && iss == 0) {
-                const uint32_t p_u = smem_u32(smem + a.off_p), v_u = smem_u32(smem + a.off_v);
-                const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
-                for (int k = 0; k < B / 16; ++k) {
-                    const uint64_t ad = smem_desc(p_u + k * 256, 128, (B / 8) * 128, SWZ_NONE);
-                    const uint64_t bd = smem_desc(v_u + 2 * k * 1024, B * 128, 1024, SWZ_128B);
-                    mma_bf16_ss(tmem + kColA, ad, bd, idP, k > 0);
-                }
-            }
-            if (ok) mma_commit(bar_d);
-        }
-        if (!ok) {
-            atomicOr(fail, 1);
-            if (iss == 1) mbar_arrive(bar_b);
-            mbar_arrive(bar_d);   // release the waiting threads
-        }
-    }
-    if (!mbar_wait(bar_d, 0, kWaitNs)) atomicOr(fail, 1);
-    tc_fence_after();
-    __syncthreads();
-    const bool failed = *fail != 0;
 
-    // ---- epilogue: out = ws * D_s + wl * D_lin, stored as bf16
-    if (!failed) {
-        const float m = stat[row], l = stat[128 + row], ld = stat[256 + row];
-        const int t = qrow / G, hh = qrow % G;
-        MergeWeights mw{0.f, 0.f};
-        if (valid) mw = merge_weights(log_sigmoid(a.alpha[g * G + hh]), m, l, ld);
-        __nv_bfloat16 *orow0 = a.O + (((size_t)r * B + t) * a.Hq + g * G + hh) * d;
-        for (int kd = sub; kd < d / 32; kd += NS) {
-            const int c0 = 32 * kd;
-            float dl[32], d2[32], ds[32];
-            ld_chunk32<kSpread>(tmem + lane_off + kColD + c0, hi, dl);
-            ld_chunk32<kSpread>(tmem + lane_off + kColS + c0, hi, d2);
-            ld_chunk32<kSpread>(tmem + lane_off + kColA + c0, hi, ds);
-            tmem_wait_ld();
+        // ---- readout D_lin = phi(Q) S_g over the 2F/32 state tiles, then D_s = P V.
+        // Tile c of phi sits at column kColA + 32 (c - c0) of the phase [c0, c1) that reads
+        // it: one phase for F <= 128; for F = 256 the phi+ tiles, then the phi- tiles.
+        // Two threads issue the readout: a tcgen05.mma with M = 128 keeps its issuing thread
+        // about as long as two tf32 products take on the tensor pipe.  Thread 0 (issuer A)
+        // reads the first half of each phase's tiles into D_lin at kColD, thread 64 (issuer
+        // B) the second half into kColS (the scores' columns, free once P is written); the
+        // epilogue adds the two.  Each accumulator has a fixed issue order.
+        const int NC1 = wide ? NC / 2 : NC;
+        bool ok = true;   // issuers only
+        const int iss = tid == 64 ? 1 : 0;
+        // A slot whose tile c is read out in the first phase is refilled (tile c + R) by
+        // thread 32 as soon as the tensor cores release it, so the issue loops never wait for
+        // a tile to finish.  A second-phase tile's slot (F = 256 with the 4-slot ring) is
+        // refilled by the thread that read it, after the tile's MMAs.
+        auto issue_tiles = [&](int c0, int c1) {
+            const uint32_t idR = instr_desc(FMT_TF32, FMT_TF32, false, false, 128, d);
+            const int hn = (c1 - c0) / 2;
+            const int cb = c0 + iss * hn, ce = cb + hn;
+            const uint32_t dcol = iss ? kColS : kColD;
+            for (int c = cb; c < ce && ok; ++c) {
+                const int slot = c % R;
+                if (!mbar_wait(&full[slot], fph(slot, c / R), kWaitNs)) { ok = false; break; }
+                const uint32_t s_u = smem_u32(slot_ptr(slot));
 #pragma unroll
-            for (int i = 0; i < 32; ++i) dl[i] += d2[i];
-            if (valid) {
-                uint32_t pk[16];
-#pragma unroll
-                for (int i = 0; i < 32; i += 2) {
-                    const float o0 = mw.ws * ds[i] + (mw.wl == 0.f ? 0.f : mw.wl * dl[i]);
-                    const float o1 = mw.ws * ds[i + 1] + (mw.wl == 0.f ? 0.f : mw.wl * dl[i + 1]);
-                    pk[i / 2] = pack_bf16x2(o0, o1);
+                for (int kk = 0; kk < 4; ++kk)
+                    mma_tf32_ts(tmem + dcol, tmem + kColA + 32 * (c - c0) + 8 * kk,
+                                smem_desc(s_u + 32 * kk, 16, 1024, SWZ_128B), idR, (c0 != 0 || c != cb || kk != 0));
+                if (c + R < NC) {
+                    mma_commit(&empty[slot]);
+                    if (c >= NC1) {
+                        if (!mbar_wait(&empty[slot], eph(slot, c / R), kWaitNs)) { ok = false; break; }
+                        mbar_arrive_expect_tx(&full[slot], chunk_bytes);
+                        bulk_g2s(slot_ptr(slot), Sg + (size_t)(c + R) * 32 * d, chunk_bytes, &full[slot]);
+                        atomicMax(issued, c + R + 1);
+                    }
                 }
-                uint4 *dst = reinterpret_cast<uint4 *>(orow0 + c0);
-#pragma unroll
-                for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+            }
+        };
+        if (tid == 32 && *fail == 0) {
+            for (int c = R; c < NC && c - R < NC1; ++c) {
+                const int slot = c % R;
+                if (!mbar_wait(&empty[slot], eph(slot, (c - R) / R), kWaitNs)) {
+                    atomicOr(fail, 1);
+                    break;
+                }
+                mbar_arrive_expect_tx(&full[slot], chunk_bytes);
+                bulk_g2s(slot_ptr(slot), Sg + (size_t)c * 32 * d, chunk_bytes, &full[slot]);
+                atomicMax(issued, c + 1);
             }
         }
-    } else if (tid == 0) {
-        raise_error(a.err, ERR_WAIT_TIMEOUT);
-        // drain bulk copies that may still be landing in this CTA's shared memory
-        mbar_wait(bar_ld, 0, kWaitNs);
-        mbar_wait(bar_z, 0, kWaitNs);
-        for (int c = 0; c < *issued; ++c) mbar_wait(&full[c % R], (uint32_t)(c / R) & 1u, kWaitNs);
+        if (tid == 0 || tid == 64) {
+            ok = *fail == 0;
+            if (ok) {
+                tc_fence_after();
+                issue_tiles(0, NC1);
+            }
+            if (wide) {
+                if (ok) mma_commit(bar_p);
+                else mbar_arrive(bar_p);
+            }
+        }
+        if (wide) {
+            // the tensor cores are done with phi+; phi- takes its columns
+            if (!mbar_wait(bar_p, up, kWaitNs)) atomicOr(fail, 1);
+            if (recip) {
+                // phi-_j = e^(mn - mx) isp isn / phi+_j, rounded to tf32
+                tc_fence_after();
+                const float mx = fmaxf(ex[1 * 256 + row], ex[1 * 256 + 128 + row]);
+                const float mn = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]);
+                const float isp = 1.f / (ex[4 * 256 + row] + ex[4 * 256 + 128 + row]);
+                const float isn = 1.f / (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
+                const float kr = exp2f((mn - mx) * kLog2e) * isp * isn;
+                for (int k = sub; k < nfc; k += NS) {
+                    float v[32];
+                    ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = tf32_round(__fdividef(kr, v[i]));
+                    st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
+                }
+                tmem_wait_st();
+            } else {
+                // form U = Q W_g again in phi+'s columns
+                if (tid == 0) {
+                    ok = ok && *fail == 0;
+                    if (ok) {
+                        tc_fence_after();
+                        const uint32_t q_u = smem_u32(smem + a.off_q), w_u = smem_u32(smem + a.off_w);
+                        const uint32_t idU = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, F);
+                        for (int k = 0; k < d / 16; ++k)
+                            mma_bf16_ss(tmem + kColA,
+                                        smem_desc(q_u + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024, SWZ_128B),
+                                        smem_desc(w_u + 2 * k * 1024, d * 128, 1024, SWZ_128B), idU, k > 0);
+                        mma_commit(bar_u2);
+                    } else {
+                        mbar_arrive(bar_u2);
+                    }
+                }
+                if (!mbar_wait(bar_u2, n_u2 & 1u, kWaitNs)) atomicOr(fail, 1);
+                ++n_u2;
+                tc_fence_after();
+                // phi- = softmax(-U), from the same extremum and sum as pass 2, rounded to tf32
+                const float mnl = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]) * kLog2e;
+                const float isn = 1.f / (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
+                for (int k = sub; k < nfc; k += NS) {
+                    float v[32];
+                    ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = tf32_round(exp2f(fmaf(-v[i], kLog2e, mnl)) * isn);
+                    st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
+                }
+                tmem_wait_st();
+            }
+            tc_fence_before();
+            __syncthreads();
+        }
+        if (tid == 0 || tid == 64) {
+            ok = ok && *fail == 0;
+            if (ok) {
+                tc_fence_after();
+                if (NC1 < NC) issue_tiles(NC1, NC);
+                // D_s = P V over phi's first d columns.  Issuer B's tiles of the last phase sit
+                // from column 32 (NC - NC1) / 2 on (F with F <= 128, 128 with F = 256); if d
+                // reaches there, A waits for B's readout, else only A's own earlier (in-order)
+                // MMAs read those columns
+                if (iss == 1 && ok) mma_commit(bar_b);
+                if (ok && iss == 0 && d > 16 * (wide ? NC - NC1 : NC) && !mbar_wait(bar_b, up, kWaitNs)) ok = false;
+                if (ok && iss == 0) {
+                    const uint32_t p_u = smem_u32(smem + a.off_p), v_u = smem_u32(smem + a.off_v);
+                    const uint32_t idP = instr_desc(FMT_BF16, FMT_BF16, false, true, 128, d);
+                    for (int k = 0; k < B / 16; ++k) {
+                        const uint64_t ad = smem_desc(p_u + k * 256, 128, (B / 8) * 128, SWZ_NONE);
+                        const uint64_t bd = smem_desc(v_u + 2 * k * 1024, B * 128, 1024, SWZ_128B);
+                        mma_bf16_ss(tmem + kColA, ad, bd, idP, k > 0);
+                    }
+                }
+                if (ok) mma_commit(bar_d);
+            }
+            if (!ok) {
+                atomicOr(fail, 1);
+                if (iss == 1) mbar_arrive(bar_b);
+                mbar_arrive(bar_d);   // release the waiting threads
+            }
+        }
+        if (!mbar_wait(bar_d, up, kWaitNs)) atomicOr(fail, 1);
+        tc_fence_after();
+        // the row's statistics (with F <= 128 in Q's buffer, which the next unit's Q overwrites)
+        const float m = stat[row], l = stat[128 + row], ld = stat[256 + row];
+        __syncthreads();
+        const bool failed = *fail != 0;
+        // every operand in shared memory has been read: the next unit's loads go out now and
+        // land while this unit's epilogue runs.  Ring slot s held ceil((NC - s) / R) tiles of
+        // this unit, each released but the last.
+        uint32_t fmask_n = fmask, emask_n = emask;
+        for (int sl = 0; sl < R; ++sl) {
+            const int cnt = (NC - sl + R - 1) / R;
+            fmask_n ^= (uint32_t)(cnt & 1) << sl;
+            emask_n ^= (uint32_t)((cnt - 1) & 1) << sl;
+        }
+        const int un = failed ? u_end : next_unit(u + 1);
+        if (tid == 32 && un < u_end) {
+            fence_proxy_async_smem();
+            issue_loads(un);
+        }
+
+        // ---- epilogue: out = ws * D_s + wl * D_lin, stored as bf16
+        if (!failed) {
+            const int t = qrow / G, hh = qrow % G;
+            MergeWeights mw{0.f, 0.f};
+            if (valid) mw = merge_weights(log_sigmoid(a.alpha[g * G + hh]), m, l, ld);
+            __nv_bfloat16 *orow0 = a.O + (((size_t)r * B + t) * a.Hq + g * G + hh) * d;
+            for (int kd = sub; kd < d / 32; kd += NS) {
+                const int c0 = 32 * kd;
+                float dl[32], d2[32], ds[32];
+                ld_chunk32<kSpread>(tmem + lane_off + kColD + c0, hi, dl);
+                ld_chunk32<kSpread>(tmem + lane_off + kColS + c0, hi, d2);
+                ld_chunk32<kSpread>(tmem + lane_off + kColA + c0, hi, ds);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) dl[i] += d2[i];
+                if (valid) {
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int i = 0; i < 32; i += 2) {
+                        const float o0 = mw.ws * ds[i] + (mw.wl == 0.f ? 0.f : mw.wl * dl[i]);
+                        const float o1 = mw.ws * ds[i + 1] + (mw.wl == 0.f ? 0.f : mw.wl * dl[i + 1]);
+                        pk[i / 2] = pack_bf16x2(o0, o1);
+                    }
+                    uint4 *dst = reinterpret_cast<uint4 *>(orow0 + c0);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                }
+            }
+        } else if (tid == 0) {
+            raise_error(a.err, ERR_WAIT_TIMEOUT);
+            // drain bulk copies that may still be landing in this CTA's shared memory
+            mbar_wait(bar_ld, up, kWaitNs);
+            mbar_wait(bar_z, up, kWaitNs);
+            for (int c = 0; c < *issued; ++c) mbar_wait(&full[c % R], fph(c % R, c / R), kWaitNs);
+        }
+        fmask = fmask_n;
+        emask = emask_n;
+        ++it;
+        tc_fence_before();
+        __syncthreads();
+        if (failed) break;
+        u = un;
     }
-    tc_fence_before();
-    __syncthreads();
     if (warp == 0) {
         tc_fence_after();
         tmem_dealloc(tmem, 512);
@@ -669,8 +716,9 @@ cudaError_t launch_attn_tc(const hybrid_cfg &c, const void *Q, const void *K, co
     auto kern = spread ? k_attn_tc<true> : k_attn_tc<false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.bytes);
     if (e != cudaSuccess) return e;
-    const long long blocks = (long long)n_req * c.n_kv_heads;
-    kern<<<(unsigned)blocks, kThreads, L.bytes, st>>>(a);
+    a.n_units = n_req * c.n_kv_heads;
+    const int grid = a.n_units < pipe::sm_count() ? a.n_units : pipe::sm_count();
+    kern<<<grid, kThreads, L.bytes, st>>>(a);
     return cudaGetLastError();
 }
 
