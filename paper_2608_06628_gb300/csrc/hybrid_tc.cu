@@ -1,10 +1,12 @@
 // hybrid_tc.cu -- block-hybrid attention on the 5th-generation tensor cores.
 //
-// One CTA per (request r, state head g).  Its M = G*B query rows (the G query
+// A unit is one (request r, state head g).  Its M = G*B query rows (the G query
 // heads of the group times the B tokens of the active block, padded to 128)
 // share the state (S_g, z_g) of Section 3.1 of "Retrofitting Linear Attention
 // into Diffusion Language Models", so the state is streamed from HBM once per
-// group.  Contractions (tcgen05.mma, accumulators in Tensor Memory):
+// group.  One CTA per SM takes a contiguous range of units one after another; a
+// unit's loads go out as soon as the previous unit's MMAs are complete and land
+// during its epilogue.  Contractions (tcgen05.mma, accumulators in Tensor Memory):
 //   U      = Q W_g              bf16 x bf16 -> f32   (feature-map projection)
 //   scores = Q K^T              bf16 x bf16 -> f32   (in-block softmax logits)
 //   D_lin  = phi(Q) S_g         tf32 x tf32 -> f32   (linear readout; phi(Q) in TMEM)
@@ -14,7 +16,9 @@
 // in-block softmax statistics, and the gated shared-normaliser merge.
 // With F = 256, phi = [phi+, phi-] (512 columns) does not fit beside D_lin and D_s
 // in Tensor Memory: phi+ is written over U and read out first, then phi- takes its
-// place for the second half of the readout.  phi- comes from phi+ by the identity
+// place for the second half of the readout.  Both are held scaled by the row's sum sp
+// of e^(u - max u) (phi+ unnormalised, no pass over it), and the epilogue divides the
+// readout by sp.  phi- comes from phi+ by the identity
 // e^(mn - u) = e^(mn - mx) / e^(u - mx) when every row's range of U is moderate (then
 // W and Q are dead after U = Q W and their space holds six more state tiles, loaded
 // while the feature map is computed); otherwise U = Q W is formed again.
@@ -245,6 +249,29 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         *issued = pre;
     };
 
+    // row statistics: in Q's buffer once Q is no longer read (F <= 128), else their own
+    float *stat = reinterpret_cast<float *>(smem + a.off_st);  // [3][128] m, l, lin_den
+    float *ex = stat + 3 * 128;                                 // [8][2][128] exchange
+    // Thread -> (TMEM lane, column subset).  Default: lane 32 q4 + lane and the warp's
+    // half as subset, two threads per row.  Spread (G = 1, B = 64): query row i sits on
+    // lane 32 (i / 16) + i % 16, so the rows occupy all four lane quarters (and SM
+    // sub-partitions), and a warp's two 16-thread halves take the same 16 lanes at
+    // different columns: four threads per row.
+    const int q4 = warp & 3, half = warp >> 2;
+    const int hi = kSpread ? lane >> 4 : 0;
+    const int row = kSpread ? 32 * q4 + (lane & 15) : 32 * q4 + lane;   // TMEM lane of the query row
+    const int qrow = kSpread ? 16 * q4 + (lane & 15) : row;              // query row t G + hh
+    const uint32_t lane_off = (uint32_t)(32 * q4) << 16;
+    const bool valid = qrow < Mv;
+    constexpr int NS = kSpread ? 4 : 2;               // column subsets per row
+    const int sub = kSpread ? 2 * half + hi : half;   // owns the chunks k with k % NS == sub
+    const int nsc = B / 16;       // 16-column chunks of scores
+    const int nfc = F / 32;       // 32-column chunks of U
+    // in the spread layout a row's partial results meet across lanes l and l ^ 16 first
+    auto comb_max = [&](float x) { return kSpread ? fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 16)) : x; };
+    auto comb_min = [&](float x) { return kSpread ? fminf(x, __shfl_xor_sync(0xffffffffu, x, 16)) : x; };
+    auto comb_add = [&](float x) { return kSpread ? x + __shfl_xor_sync(0xffffffffu, x, 16) : x; };
+
     // Units run one after another; the barriers used once per unit complete with
     // the parity of the unit's index it in this CTA.  Ring slot s has had fills and
     // releases of earlier units; fmask / emask bit s hold the parity of their counts.
@@ -255,6 +282,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         const uint32_t up = it & 1u;
         const int r = u / a.Hkv, g = u % a.Hkv;
         const float *Sg = head_state(u);
+        // the next unit's state pointer and this row's gate, loaded now (used after the readout)
+        const void *nstate = u + 1 < u_end ? a.states[(u + 1) / a.Hkv] : nullptr;
+        const float alpha_row = valid ? a.alpha[g * G + qrow % G] : 0.f;
         // phase parity of fill j (or release j) of ring slot s in this unit
         auto fph = [&](int s, int j) -> uint32_t { return ((fmask >> s) & 1u) ^ ((uint32_t)j & 1u); };
         auto eph = [&](int s, int j) -> uint32_t { return ((emask >> s) & 1u) ^ ((uint32_t)j & 1u); };
@@ -290,29 +320,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
             sl -= a.n_slots;
             return sl < 4 ? smem + a.off_w + (size_t)sl * chunk_bytes : smem + a.off_q + (size_t)(sl - 4) * chunk_bytes;
         };
-
-        // row statistics: in Q's buffer once Q is no longer read (F <= 128), else their own
-        float *stat = reinterpret_cast<float *>(smem + a.off_st);  // [3][128] m, l, lin_den
-        float *ex = stat + 3 * 128;                                 // [8][2][128] exchange
-        // Thread -> (TMEM lane, column subset).  Default: lane 32 q4 + lane and the warp's
-        // half as subset, two threads per row.  Spread (G = 1, B = 64): query row i sits on
-        // lane 32 (i / 16) + i % 16, so the rows occupy all four lane quarters (and SM
-        // sub-partitions), and a warp's two 16-thread halves take the same 16 lanes at
-        // different columns: four threads per row.
-        const int q4 = warp & 3, half = warp >> 2;
-        const int hi = kSpread ? lane >> 4 : 0;
-        const int row = kSpread ? 32 * q4 + (lane & 15) : 32 * q4 + lane;   // TMEM lane of the query row
-        const int qrow = kSpread ? 16 * q4 + (lane & 15) : row;              // query row t G + hh
-        const uint32_t lane_off = (uint32_t)(32 * q4) << 16;
-        const bool valid = qrow < Mv;
-        constexpr int NS = kSpread ? 4 : 2;               // column subsets per row
-        const int sub = kSpread ? 2 * half + hi : half;   // owns the chunks k with k % NS == sub
-        const int nsc = B / 16;       // 16-column chunks of scores
-        const int nfc = F / 32;       // 32-column chunks of U
-        // in the spread layout a row's partial results meet across lanes l and l ^ 16 first
-        auto comb_max = [&](float x) { return kSpread ? fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 16)) : x; };
-        auto comb_min = [&](float x) { return kSpread ? fminf(x, __shfl_xor_sync(0xffffffffu, x, 16)) : x; };
-        auto comb_add = [&](float x) { return kSpread ? x + __shfl_xor_sync(0xffffffffu, x, 16) : x; };
 
         // ---- pass 1: local extrema
         {
@@ -394,6 +401,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
                     lp = fmaf(ep[i], zs[32 * k + i], lp);
                     ln = fmaf(en[i], zs[F + 32 * k + i], ln);
                 }
+                if (wide) {
+                    // F = 256: phi+ stays unnormalised (the readout is scaled by 1 / sp)
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) ep[i] = tf32_round(ep[i]);
+                }
                 st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, ep);
                 if (!wide) st_chunk32<kSpread>(tmem + lane_off + kColA + F + 32 * k, hi, en);   // F = 256: formed later
             }
@@ -407,19 +419,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         }
         __syncthreads();
 
-        // ---- pass 3: normalise phi in place (rounded to tf32), row statistics
+        // ---- pass 3: normalise phi in place (rounded to tf32; F <= 128), row statistics.
+        // With F = 256 the readout accumulates sp phi+ and sp phi-, and lin_scale = 1 / sp
+        // scales it back in the epilogue.
+        float lin_scale = 1.f;
         {
             const float sp = ex[4 * 256 + row] + ex[4 * 256 + 128 + row];
             const float sn = ex[5 * 256 + row] + ex[5 * 256 + 128 + row];
             const float isp = 1.f / sp, isn = 1.f / sn;
-            for (int k = sub; k < nfc; k += NS) {
+            if (wide) lin_scale = isp;
+            for (int k = sub; !wide && k < nfc; k += NS) {
                 float v[32];
                 ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
                 tmem_wait_ld();
 #pragma unroll
                 for (int i = 0; i < 32; ++i) v[i] = tf32_round(v[i] * isp);
                 st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
-                if (wide) continue;
                 ld_chunk32<kSpread>(tmem + lane_off + kColA + F + 32 * k, hi, v);
                 tmem_wait_ld();
 #pragma unroll
@@ -504,13 +519,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
             // the tensor cores are done with phi+; phi- takes its columns
             if (!mbar_wait(bar_p, up, kWaitNs)) atomicOr(fail, 1);
             if (recip) {
-                // phi-_j = e^(mn - mx) isp isn / phi+_j, rounded to tf32
+                // sp phi-_j = e^(mn - mx) sp isn / e^(u_j - mx), rounded to tf32 (the
+                // unnormalised phi+ in Tensor Memory is e^(u_j - mx))
                 tc_fence_after();
                 const float mx = fmaxf(ex[1 * 256 + row], ex[1 * 256 + 128 + row]);
                 const float mn = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]);
-                const float isp = 1.f / (ex[4 * 256 + row] + ex[4 * 256 + 128 + row]);
+                const float sp = ex[4 * 256 + row] + ex[4 * 256 + 128 + row];
                 const float isn = 1.f / (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
-                const float kr = exp2f((mn - mx) * kLog2e) * isp * isn;
+                const float kr = exp2f((mn - mx) * kLog2e) * sp * isn;
                 for (int k = sub; k < nfc; k += NS) {
                     float v[32];
                     ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
@@ -540,15 +556,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
                 if (!mbar_wait(bar_u2, n_u2 & 1u, kWaitNs)) atomicOr(fail, 1);
                 ++n_u2;
                 tc_fence_after();
-                // phi- = softmax(-U), from the same extremum and sum as pass 2, rounded to tf32
+                // sp phi- = sp softmax(-U), from the same extremum and sums as pass 2, rounded to tf32
                 const float mnl = fminf(ex[2 * 256 + row], ex[2 * 256 + 128 + row]) * kLog2e;
-                const float isn = 1.f / (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
+                const float spn = (ex[4 * 256 + row] + ex[4 * 256 + 128 + row]) /
+                                  (ex[5 * 256 + row] + ex[5 * 256 + 128 + row]);
                 for (int k = sub; k < nfc; k += NS) {
                     float v[32];
                     ld_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
                     tmem_wait_ld();
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] = tf32_round(exp2f(fmaf(-v[i], kLog2e, mnl)) * isn);
+                    for (int i = 0; i < 32; ++i) v[i] = tf32_round(exp2f(fmaf(-v[i], kLog2e, mnl)) * spn);
                     st_chunk32<kSpread>(tmem + lane_off + kColA + 32 * k, hi, v);
                 }
                 tmem_wait_st();
@@ -599,7 +616,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
             fmask_n ^= (uint32_t)(cnt & 1) << sl;
             emask_n ^= (uint32_t)((cnt - 1) & 1) << sl;
         }
-        const int un = failed ? u_end : next_unit(u + 1);
+        const int un = failed ? u_end : u + 1 < u_end && state_ptr_ok(nstate) ? u + 1 : next_unit(u + 1);
         if (tid == 32 && un < u_end) {
             fence_proxy_async_smem();
             issue_loads(un);
@@ -609,7 +626,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         if (!failed) {
             const int t = qrow / G, hh = qrow % G;
             MergeWeights mw{0.f, 0.f};
-            if (valid) mw = merge_weights(log_sigmoid(a.alpha[g * G + hh]), m, l, ld);
+            if (valid) mw = merge_weights(log_sigmoid(alpha_row), m, l, ld);
+            mw.wl *= lin_scale;
             __nv_bfloat16 *orow0 = a.O + (((size_t)r * B + t) * a.Hq + g * G + hh) * d;
             for (int kd = sub; kd < d / 32; kd += NS) {
                 const int c0 = 32 * kd;
