@@ -51,7 +51,8 @@ constexpr int kExtraSlots = 6;                // F = 256: W (4 tiles) and Q (2 t
 constexpr float kRecipRange = 64.f;           // largest row range of U for phi- from phi+
 
 struct TcAttnArgs {
-    CUtensorMap tmQ, tmK, tmV, tmW;   // Q [n B][Hq][d] box {64, G, B}; K, V box {64, 1, B}; W box {64, d}
+    CUtensorMap tmQ, tmK, tmV, tmW;   // Q [n B][Hq][d] box {64, G, B}; K, V box {64, 1, B, d / 64};
+                                      // W box {64, d, F / 64} (panels outermost)
     const float *alpha;
     void *const *states;
     __nv_bfloat16 *O;
@@ -222,9 +223,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     };
     // ---- loads of unit u (one thread): Q, K, V, W (TMA), z and the first S tiles
     // (bulk copies of the state image)
-    auto issue_loads = [&](int u) {
+    auto issue_loads = [&](int u, const void *st) {
         const int r = u / a.Hkv, g = u % a.Hkv;
-        const float *Sg = head_state(u);
+        const float *Sg = reinterpret_cast<const float *>(st) + (size_t)g * head_floats(d, F);
         mbar_arrive_expect_tx(bar_ld, (uint32_t)(Mv + 2 * B + F) * d * 2);
         for (int c = 0; c < d / 64; ++c) {
             if (kSpread) {
@@ -235,10 +236,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
             } else {
                 tma_load_3d(smem + a.off_q + c * (128 * 128), &a.tmQ, 64 * c, g * G, r * B, bar_ld);
             }
-            tma_load_3d(smem + a.off_k + c * (B * 128), &a.tmK, 64 * c, g, r * B, bar_ld);
-            tma_load_3d(smem + a.off_v + c * (B * 128), &a.tmV, 64 * c, g, r * B, bar_ld);
         }
-        for (int f = 0; f < F / 64; ++f) tma_load_2d(smem + a.off_w + f * (d * 128), &a.tmW, 64 * f, g * d, bar_ld);
+        // K and V: all d / 64 panels in one box; W: all F / 64 panels in one box
+        tma_load_4d(smem + a.off_k, &a.tmK, 0, g, r * B, 0, bar_ld);
+        tma_load_4d(smem + a.off_v, &a.tmV, 0, g, r * B, 0, bar_ld);
+        tma_load_3d(smem + a.off_w, &a.tmW, 0, g * d, 0, bar_ld);
         mbar_arrive_expect_tx(bar_z, 2 * F * 4);
         bulk_g2s(smem + a.off_z, Sg + (size_t)2 * F * d, 2 * F * 4, bar_z);
         const int pre = NC < a.n_slots ? NC : a.n_slots;
@@ -276,8 +278,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     // the parity of the unit's index it in this CTA.  Ring slot s has had fills and
     // releases of earlier units; fmask / emask bit s hold the parity of their counts.
     uint32_t fmask = 0, emask = 0, it = 0, n_u2 = 0;
+    // what one unit adds to them, for the two ring sizes (n_slots, and min(NC, RM) slots
+    // when phi- comes from phi+): slot s holds ceil((NC - s) / R) tiles, each released
+    // but the last
+    auto ring_x = [&](int Rv, bool rel) -> uint32_t {
+        uint32_t x = 0;
+        for (int sl = 0; sl < Rv; ++sl) {
+            const int cnt = (NC - sl + Rv - 1) / Rv;
+            x ^= (uint32_t)((rel ? cnt - 1 : cnt) & 1) << sl;
+        }
+        return x;
+    };
+    const uint32_t xf0 = ring_x(a.n_slots, false), xe0 = ring_x(a.n_slots, true);
+    const uint32_t xf1 = ring_x(min(NC, RM), false), xe1 = ring_x(min(NC, RM), true);
     int u = next_unit(u_begin);
-    if (tid == 0 && u < u_end) issue_loads(u);
+    if (tid == 0 && u < u_end) issue_loads(u, a.states[u / a.Hkv]);
     while (u < u_end) {
         const uint32_t up = it & 1u;
         const int r = u / a.Hkv, g = u % a.Hkv;
@@ -608,18 +623,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         __syncthreads();
         const bool failed = *fail != 0;
         // every operand in shared memory has been read: the next unit's loads go out now and
-        // land while this unit's epilogue runs.  Ring slot s held ceil((NC - s) / R) tiles of
-        // this unit, each released but the last.
-        uint32_t fmask_n = fmask, emask_n = emask;
-        for (int sl = 0; sl < R; ++sl) {
-            const int cnt = (NC - sl + R - 1) / R;
-            fmask_n ^= (uint32_t)(cnt & 1) << sl;
-            emask_n ^= (uint32_t)((cnt - 1) & 1) << sl;
-        }
+        // land while this unit's epilogue runs
+        const uint32_t fmask_n = fmask ^ (recip ? xf1 : xf0), emask_n = emask ^ (recip ? xe1 : xe0);
         const int un = failed ? u_end : u + 1 < u_end && state_ptr_ok(nstate) ? u + 1 : next_unit(u + 1);
         if (tid == 32 && un < u_end) {
             fence_proxy_async_smem();
-            issue_loads(un);
+            issue_loads(un, un == u + 1 ? nstate : a.states[un / a.Hkv]);
         }
 
         // ---- epilogue: out = ws * D_s + wl * D_lin, stored as bf16
@@ -700,14 +709,16 @@ cudaError_t launch_attn_tc(const hybrid_cfg &c, const void *Q, const void *K, co
         const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)Hq, rows};
         const cuuint64_t sq[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hq * d * 2};
         const cuuint32_t bq[3] = {64, (cuuint32_t)(Hq / Hkv), (cuuint32_t)(spread ? 16 : B)};
-        const cuuint64_t dk[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, rows};
-        const cuuint64_t sk[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
-        const cuuint32_t bk[3] = {64, 1, (cuuint32_t)B};
-        const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
-        const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
-        const cuuint32_t bw[2] = {64, (cuuint32_t)d};
-        if (!pipe::encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !pipe::encode_bf16(&a.tmK, K, 3, dk, sk, bk) ||
-            !pipe::encode_bf16(&a.tmV, V, 3, dk, sk, bk) || !pipe::encode_bf16(&a.tmW, W, 2, dw, sw, bw))
+        // K, V [rows][Hkv][d] and W [Hkv d][F] with their 64-element panels as the
+        // outermost box dimension (stride 128 bytes), so one copy brings every panel
+        const cuuint64_t dk[4] = {64, (cuuint64_t)Hkv, rows, (cuuint64_t)d / 64};
+        const cuuint64_t sk[3] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2, 128};
+        const cuuint32_t bk[4] = {64, 1, (cuuint32_t)B, (cuuint32_t)d / 64};
+        const cuuint64_t dw[3] = {64, (cuuint64_t)Hkv * d, (cuuint64_t)F / 64};
+        const cuuint64_t sw[2] = {(cuuint64_t)F * 2, 128};
+        const cuuint32_t bw[3] = {64, (cuuint32_t)d, (cuuint32_t)F / 64};
+        if (!pipe::encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !pipe::encode_bf16(&a.tmK, K, 4, dk, sk, bk) ||
+            !pipe::encode_bf16(&a.tmV, V, 4, dk, sk, bk) || !pipe::encode_bf16(&a.tmW, W, 3, dw, sw, bw))
             return cudaErrorInvalidValue;
     }
     a.alpha = alpha;
