@@ -315,6 +315,55 @@ def test_bad_state_pointer_is_reported_not_faulted(wl):
     assert H.hybrid_check(check=False) == H.HYBRID_OK
 
 
+# More units than SMs, so the persistent kernels take two or three units per CTA:
+# request 0's units end one CTA's range and request 1's start it (bad-then-good and
+# good-then-bad inside one CTA's run)
+BADRUN_WL = [W_("badrun_c3_shape", BF16, 80, 8, 4, 128, 128, 32, 51),
+             W_("badrun_f256_g1", BF16, 60, 3, 3, 128, 256, 64, 52)]
+
+
+@pytest.mark.parametrize("wl", BADRUN_WL, ids=[w.name for w in BADRUN_WL])
+def test_bad_state_pointer_inside_a_run_of_units(wl):
+    """A request whose state pointer is unusable is skipped inside a CTA's run of
+    units: the error is reported, its output rows are left as they were, and every
+    other request's output (and, for the fused step + commit, its committed state)
+    is the oracle's."""
+    tracked = [0, 1, 2, 3, wl.n_req - 1]
+    pair = Pair(wl, tracked=tracked)
+    pair.build_prefixes(np.full(wl.n_req, 2 * wl.B))
+    Q, K, V = wk.block_qkv(wl, "badrun", pair.dev)
+    t = torch.as_tensor(tracked, device=pair.dev)
+    want = pair.orc.block_attn(h64(Q[t]), h64(K[t]), h64(V[t]), pair.W64, pair.alpha64, pair.S, pair.z)
+    for bad in (0, 1):
+        keep = [i for i, r in enumerate(tracked) if r != bad]
+        ptrs = pair.ptrs.clone()
+        ptrs[bad] = 0
+        O = torch.full_like(Q, 7.0)
+        H.hybrid_block_attn(pair.cfg, Q, K, V, pair.W, pair.alpha, ptrs, wl.n_req, O)
+        assert H.hybrid_check(check=False) == H.HYBRID_ERR_DEVICE
+        assert torch.all(O[bad] == 7.0), "the skipped request's output was written"
+        assert_parity(h64(O[t])[keep], want[keep], wl.io_dtype, f"step, request {bad} skipped", units="out")
+    if wl.B != 32:
+        return
+    # step + commit on the same batch with request 1 skipped (the fused kernel)
+    bad = 1
+    keep = [i for i, r in enumerate(tracked) if r != bad]
+    ptrs = pair.ptrs.clone()
+    ptrs[bad] = 0
+    O = torch.full_like(Q, 7.0)
+    H.hybrid_block_attn_commit(pair.cfg, Q, K, V, pair.W, pair.alpha, ptrs, wl.n_req, O)
+    assert H.hybrid_check(check=False) == H.HYBRID_ERR_DEVICE
+    assert torch.all(O[bad] == 7.0), "the skipped request's output was written"
+    assert_parity(h64(O[t])[keep], want[keep], wl.io_dtype, "step + commit, request 1 skipped", units="out")
+    tk = torch.as_tensor([tracked[i] for i in keep], device=pair.dev)
+    S_want, z_want = pair.S[keep].copy(), pair.z[keep].copy()
+    pair.orc.commit(h64(K[tk]), h64(V[tk]), pair.W64, S_want, z_want)
+    S_got, z_got = pair.gpu_state([tracked[i] for i in keep])
+    assert_parity(S_got, S_want, wl.io_dtype, "state after step + commit", units="state")
+    S_bad, _ = pair.gpu_state([bad])
+    assert_parity(S_bad, pair.S[[tracked.index(bad)]], wl.io_dtype, "skipped request's state", units="state")
+
+
 def test_bounded_wait_timeout_is_reported_not_hung():
     """A bounded device wait that runs out comes back as HYBRID_ERR_TIMEOUT from
     hybrid_check, with the context usable.  The hook arms one step launch with a
