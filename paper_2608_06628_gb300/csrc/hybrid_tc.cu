@@ -223,26 +223,32 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     };
     // ---- loads of unit u (one thread): Q, K, V, W (TMA), z and the first S tiles
     // (bulk copies of the state image)
-    auto issue_loads = [&](int u, const void *st) {
+    // part 1: K and z (their space is free once the unit's phi- has been formed); part 2:
+    // Q, V, W and the first state tiles (free once the unit's MMAs are complete: W's space
+    // holds state tiles of the phi- readout when phi- comes from phi+)
+    auto issue_loads = [&](int u, const void *st, int part) {
         const int r = u / a.Hkv, g = u % a.Hkv;
         const float *Sg = reinterpret_cast<const float *>(st) + (size_t)g * head_floats(d, F);
-        mbar_arrive_expect_tx(bar_ld, (uint32_t)(Mv + 2 * B + F) * d * 2);
-        for (int c = 0; c < d / 64; ++c) {
-            if (kSpread) {
-                // query rows 16 q .. 16 q + 15 onto lanes 32 q .. 32 q + 15 (G = 1)
-                for (int q = 0; q < Mv / 16; ++q)
-                    tma_load_3d(smem + a.off_q + c * (128 * 128) + q * (32 * 128), &a.tmQ, 64 * c, g, r * B + 16 * q,
-                                bar_ld);
-            } else {
-                tma_load_3d(smem + a.off_q + c * (128 * 128), &a.tmQ, 64 * c, g * G, r * B, bar_ld);
-            }
+        if (part != 2) {
+            // the spread Q box brings 128 rows, its padding rows zero-filled
+            mbar_arrive_expect_tx(bar_ld, (uint32_t)((kSpread ? 128 : Mv) + 2 * B + F) * d * 2);
+            // K: all d / 64 panels in one box
+            tma_load_4d(smem + a.off_k, &a.tmK, 0, g, r * B, 0, bar_ld);
+            mbar_arrive_expect_tx(bar_z, 2 * F * 4);
+            bulk_g2s(smem + a.off_z, Sg + (size_t)2 * F * d, 2 * F * 4, bar_z);
         }
-        // K and V: all d / 64 panels in one box; W: all F / 64 panels in one box
-        tma_load_4d(smem + a.off_k, &a.tmK, 0, g, r * B, 0, bar_ld);
+        if (part == 1) return;
+        if (kSpread) {
+            // query rows 16 q .. 16 q + 15 onto lanes 32 q .. 32 q + 15 (G = 1), rows
+            // 16 q + 16 .. 16 q + 31 zero: one box of 2 panels x 4 groups x 32 rows
+            tma_load_5d(smem + a.off_q, &a.tmQ, 0, g, 0, r * (B / 16), 0, bar_ld);
+        } else {
+            for (int c = 0; c < d / 64; ++c)
+                tma_load_3d(smem + a.off_q + c * (128 * 128), &a.tmQ, 64 * c, g * G, r * B, bar_ld);
+        }
+        // V: all d / 64 panels in one box; W: all F / 64 panels in one box
         tma_load_4d(smem + a.off_v, &a.tmV, 0, g, r * B, 0, bar_ld);
         tma_load_3d(smem + a.off_w, &a.tmW, 0, g * d, 0, bar_ld);
-        mbar_arrive_expect_tx(bar_z, 2 * F * 4);
-        bulk_g2s(smem + a.off_z, Sg + (size_t)2 * F * d, 2 * F * 4, bar_z);
         const int pre = NC < a.n_slots ? NC : a.n_slots;
         for (int c = 0; c < pre; ++c) {
             mbar_arrive_expect_tx(&full[c], chunk_bytes);
@@ -292,7 +298,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     const uint32_t xf0 = ring_x(a.n_slots, false), xe0 = ring_x(a.n_slots, true);
     const uint32_t xf1 = ring_x(min(NC, RM), false), xe1 = ring_x(min(NC, RM), true);
     int u = next_unit(u_begin);
-    if (tid == 0 && u < u_end) issue_loads(u, a.states[u / a.Hkv]);
+    if (tid == 0 && u < u_end) issue_loads(u, a.states[u / a.Hkv], 0);
     while (u < u_end) {
         const uint32_t up = it & 1u;
         const int r = u / a.Hkv, g = u % a.Hkv;
@@ -303,6 +309,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         // phase parity of fill j (or release j) of ring slot s in this unit
         auto fph = [&](int s, int j) -> uint32_t { return ((fmask >> s) & 1u) ^ ((uint32_t)j & 1u); };
         auto eph = [&](int s, int j) -> uint32_t { return ((emask >> s) & 1u) ^ ((uint32_t)j & 1u); };
+        bool early = false;   // thread 32: the next unit's first loads went out during this unit
 
         // ---- U = Q W_g and scores = Q K^T.  W and V are MN-major: 64-wide panels of
         // d (W) or B (V) rows, 8-row groups 1024 bytes apart.
@@ -587,6 +594,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
             }
             tc_fence_before();
             __syncthreads();
+            // the next unit's K and z: K was read by the scores, z by pass 2
+            if (tid == 32 && *fail == 0 && u + 1 < u_end && state_ptr_ok(nstate)) {
+                early = true;
+                fence_proxy_async_smem();
+                issue_loads(u + 1, nstate, 1);
+            }
         }
         if (tid == 0 || tid == 64) {
             ok = ok && *fail == 0;
@@ -620,15 +633,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
         tc_fence_after();
         // the row's statistics (with F <= 128 in Q's buffer, which the next unit's Q overwrites)
         const float m = stat[row], l = stat[128 + row], ld = stat[256 + row];
-        __syncthreads();
+        const int issued_now = *issued;   // the next unit's copies reset the count
+        // (a unit whose first part of loads went out is completed even after a failure,
+        // so that every barrier the drain waits on completes)
+        const bool early_any = __syncthreads_or(early) != 0;
         const bool failed = *fail != 0;
         // every operand in shared memory has been read: the next unit's loads go out now and
         // land while this unit's epilogue runs
         const uint32_t fmask_n = fmask ^ (recip ? xf1 : xf0), emask_n = emask ^ (recip ? xe1 : xe0);
-        const int un = failed ? u_end : u + 1 < u_end && state_ptr_ok(nstate) ? u + 1 : next_unit(u + 1);
+        const int un = early_any ? u + 1 : failed ? u_end : u + 1 < u_end && state_ptr_ok(nstate) ? u + 1
+                                                                                      : next_unit(u + 1);
         if (tid == 32 && un < u_end) {
             fence_proxy_async_smem();
-            issue_loads(un, un == u + 1 ? nstate : a.states[un / a.Hkv]);
+            issue_loads(un, un == u + 1 ? nstate : a.states[un / a.Hkv], early ? 2 : 0);
         }
 
         // ---- epilogue: out = ws * D_s + wl * D_lin, stored as bf16
@@ -665,7 +682,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
             // drain bulk copies that may still be landing in this CTA's shared memory
             mbar_wait(bar_ld, up, kWaitNs);
             mbar_wait(bar_z, up, kWaitNs);
-            for (int c = 0; c < *issued; ++c) mbar_wait(&full[c % R], fph(c % R, c / R), kWaitNs);
+            for (int c = 0; c < issued_now; ++c) mbar_wait(&full[c % R], fph(c % R, c / R), kWaitNs);
+            if (un < u_end) {
+                // the next unit's loads, issued before the failure was seen
+                mbar_wait(bar_ld, up ^ 1u, kWaitNs);
+                mbar_wait(bar_z, up ^ 1u, kWaitNs);
+                for (int c = 0; c < NC && c < a.n_slots; ++c) mbar_wait(&full[c], (fmask_n >> c) & 1u, kWaitNs);
+            }
         }
         fmask = fmask_n;
         emask = emask_n;
@@ -708,7 +731,13 @@ cudaError_t launch_attn_tc(const hybrid_cfg &c, const void *Q, const void *K, co
         const cuuint64_t rows = (cuuint64_t)n_req * B;
         const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)Hq, rows};
         const cuuint64_t sq[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hq * d * 2};
-        const cuuint32_t bq[3] = {64, (cuuint32_t)(Hq / Hkv), (cuuint32_t)(spread ? 16 : B)};
+        const cuuint32_t bq[3] = {64, (cuuint32_t)(Hq / Hkv), (cuuint32_t)B};
+        // spread (G = 1, B = 64): Q as [panel][16-token group][token in group][head][64],
+        // the box 32 tokens deep over a dimension of 16, so that each group's 16 rows are
+        // followed by 16 zero-filled ones (lanes 32 q .. 32 q + 31 of quarter q)
+        const cuuint64_t dqs[5] = {64, (cuuint64_t)Hq, 16, rows / 16, (cuuint64_t)d / 64};
+        const cuuint64_t sqs[4] = {(cuuint64_t)d * 2, (cuuint64_t)Hq * d * 2, (cuuint64_t)16 * Hq * d * 2, 128};
+        const cuuint32_t bqs[5] = {64, 1, 32, (cuuint32_t)B / 16, (cuuint32_t)d / 64};
         // K, V [rows][Hkv][d] and W [Hkv d][F] with their 64-element panels as the
         // outermost box dimension (stride 128 bytes), so one copy brings every panel
         const cuuint64_t dk[4] = {64, (cuuint64_t)Hkv, rows, (cuuint64_t)d / 64};
@@ -717,7 +746,7 @@ cudaError_t launch_attn_tc(const hybrid_cfg &c, const void *Q, const void *K, co
         const cuuint64_t dw[3] = {64, (cuuint64_t)Hkv * d, (cuuint64_t)F / 64};
         const cuuint64_t sw[2] = {(cuuint64_t)F * 2, 128};
         const cuuint32_t bw[3] = {64, (cuuint32_t)d, (cuuint32_t)F / 64};
-        if (!pipe::encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !pipe::encode_bf16(&a.tmK, K, 4, dk, sk, bk) ||
+        if (!(spread ? pipe::encode_bf16(&a.tmQ, Q, 5, dqs, sqs, bqs) : pipe::encode_bf16(&a.tmQ, Q, 3, dq, sq, bq)) || !pipe::encode_bf16(&a.tmK, K, 4, dk, sk, bk) ||
             !pipe::encode_bf16(&a.tmV, V, 4, dk, sk, bk) || !pipe::encode_bf16(&a.tmW, W, 3, dw, sw, bw))
             return cudaErrorInvalidValue;
     }
