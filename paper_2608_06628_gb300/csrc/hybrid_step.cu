@@ -72,7 +72,11 @@ constexpr uint32_t kStatBytes = 8 * 128 * 4 * P;
 constexpr int SC = 16;                // score columns per part (parts 0 .. B/16 - 1)
 
 struct StepArgs {
-    CUtensorMap tmQ, tmK, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], K, V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
+    // Q, O [n*B][Hq][d], K, V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle, the
+    // 64-element panels as the outermost box dimension so that one copy brings all of
+    // them.  Q's box is 128 / G tokens deep over a dimension of B, so the rows of a
+    // unit's 128-row tile beyond G B are zero-filled.
+    CUtensorMap tmQ, tmK, tmV, tmW, tmO;
     bf16 *O;
     const float *alpha;
     void *const *states;
@@ -218,21 +222,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
     // global memory before that kernel has completed
     if (tid == 0) griddep_launch_dependents();
     griddep_wait();
+    // a unit's Q into a ring slot: one box of all panels x 128 rows (rows beyond G B
+    // zero-filled)
+    auto load_q = [&](uint8_t *dst, int r, int g, uint64_t *bar) {
+        mbar_arrive_expect_tx(bar, (uint32_t)(d / 64) * (128 * 128));
+        tma_load_5d(dst, &a.tmQ, 0, g * G, 0, r, 0, bar);
+    };
     // the first unit's Q (ring slot 0), W and K go out from here, before the roles
     // branch off, so their latency starts as early as possible
     if (u_begin < u_end && (tid == 0 || tid == 64)) {
         const int r = u_begin / a.Hkv, g = u_begin % a.Hkv;
         if (tid == 0) {
-            mbar_arrive_expect_tx(&full[0], (uint32_t)(d / 64) * (G * B * 128));
-            for (int e = 0; e < d / 64; ++e)
-                tma_load_3d(smem + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, &full[0]);
+            load_q(smem, r, g, &full[0]);
         } else {
             uint8_t *kb = smem + a.off_wk + (F / 64) * d * 128;
             mbar_arrive_expect_tx(xfull, (uint32_t)(F / 64) * (d * 128) + (uint32_t)(d / 64) * (B * 128));
-            for (int f = 0; f < F / 64; ++f)
-                tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xfull);
-            for (int e = 0; e < d / 64; ++e)
-                tma_load_3d(kb + e * (B * 128), &a.tmK, 64 * e, g, r * B, xfull);
+            tma_load_3d(smem + a.off_wk, &a.tmW, 0, g * d, 0, xfull);
+            tma_load_4d(kb, &a.tmK, 0, g, r * B, 0, xfull);
         }
     }
     const uint32_t tmem = *tmem_holder;
@@ -258,10 +264,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                 if (q > 0) {
                     const int slot = q % NS;
                     if (!wait_bar(&empty[slot], ((q / NS) & 1u) ^ 1u, fail, wlim)) break;
-                    mbar_arrive_expect_tx(&full[slot], (uint32_t)(d / 64) * (G * B * 128));
-                    for (int e = 0; e < d / 64; ++e)
-                        tma_load_3d(ring + (size_t)slot * slot_bytes + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B,
-                                    &full[slot]);
+                    load_q(ring + (size_t)slot * slot_bytes, r, g, &full[slot]);
                     ++q;
                 } else {
                     ++q;   // issued in the prologue
@@ -406,10 +409,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0 && nx > 0) {   // the first unit's W and K went out in the prologue
                 mbar_arrive_expect_tx(xfull, xbytes);
-                for (int f = 0; f < F / 64; ++f)
-                    tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xfull);
-                for (int e = 0; e < d / 64; ++e)
-                    tma_load_3d(kb + e * (B * 128), &a.tmK, 64 * e, g, r * B, xfull);
+                tma_load_3d(smem + a.off_wk, &a.tmW, 0, g * d, 0, xfull);
+                tma_load_4d(kb, &a.tmK, 0, g, r * B, 0, xfull);
             }
             ++nx;
             if (!state_at(a, raw, u)) continue;
@@ -419,8 +420,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
                 ok = wait_bar(ostaged, (kp - 1) & 1u, fail, wlim);
                 if (__any_sync(0xffffffffu, !ok)) break;
                 if (lane == 0) {
-                    for (int j = 0; j < d / 64; ++j)
-                        tma_store_3d(&a.tmO, 64 * j, pg * G, pr * B, smem + a.off_vb + j * (G * B * 128));
+                    tma_store_4d(&a.tmO, 0, pg * G, pr * B, 0, smem + a.off_vb);
                     bulk_commit();
                     bulk_wait_read_all();
                     mbar_arrive(ofree);
@@ -429,8 +429,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             }
             if (lane == 0) {
                 mbar_arrive_expect_tx(vfull, (uint32_t)(d / 64) * (B * 128));
-                for (int e = 0; e < d / 64; ++e)
-                    tma_load_3d(smem + a.off_vb + e * (B * 128), &a.tmV, 64 * e, g, r * B, vfull);
+                tma_load_4d(smem + a.off_vb, &a.tmV, 0, g, r * B, 0, vfull);
             }
             ++nv;
             ++kp;
@@ -439,8 +438,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
         }
         // the last unit's output tile
         if (kp > 0 && !*fail && wait_bar(ostaged, (kp - 1) & 1u, fail, wlim) && lane == 0) {
-            for (int j = 0; j < d / 64; ++j)
-                tma_store_3d(&a.tmO, 64 * j, pg * G, pr * B, smem + a.off_vb + j * (G * B * 128));
+            tma_store_4d(&a.tmO, 0, pg * G, pr * B, 0, smem + a.off_vb);
             bulk_commit();
         }
         if (lane == 0) {
@@ -743,6 +741,8 @@ bool step_supported(const hybrid_cfg &c)
     if (c.block_size != 16 && c.block_size != 32) return false;
     const int G = c.n_q_heads / c.n_kv_heads;
     if (G * c.block_size > 128) return false;
+    // a unit's Q arrives as one box of 128 / G tokens x G heads
+    if (128 % G != 0) return false;
     const SLayout L = make_slayout(c.head_dim, c.feat_dim, c.block_size, c.n_q_heads / c.n_kv_heads);
     if (L.NS < 2) return false;
     return (int)L.bytes <= kSmemLimit;
@@ -758,18 +758,26 @@ cudaError_t launch_step(const hybrid_cfg &c, const void *Q, const void *K, const
         const int d = c.head_dim, F = c.feat_dim, B = c.block_size, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
         const int G = Hq / Hkv;
         const cuuint64_t rows = (cuuint64_t)n_req * B;
-        const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)Hq, rows};
-        const cuuint64_t sq[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hq * d * 2};
-        const cuuint32_t bq[3] = {64, (cuuint32_t)G, (cuuint32_t)B};
-        const cuuint64_t dv[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, rows};
-        const cuuint64_t sv[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
-        const cuuint32_t bv[3] = {64, 1, (cuuint32_t)B};
-        const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
-        const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
-        const cuuint32_t bw[2] = {64, (cuuint32_t)d};
-        if (!encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !encode_bf16(&a.tmK, K, 3, dv, sv, bv) ||
-            !encode_bf16(&a.tmV, V, 3, dv, sv, bv) || !encode_bf16(&a.tmW, W, 2, dw, sw, bw) ||
-            !encode_bf16(&a.tmO, O, 3, dq, sq, bq))
+        const cuuint64_t P = (cuuint64_t)d / 64;
+        // Q: [panel][request][token][head][64]; a box of G heads x 128 / G tokens
+        const cuuint64_t dq5[5] = {64, (cuuint64_t)Hq, (cuuint64_t)B, (cuuint64_t)n_req, P};
+        const cuuint64_t sq5[4] = {(cuuint64_t)d * 2, (cuuint64_t)Hq * d * 2, (cuuint64_t)B * Hq * d * 2, 128};
+        const cuuint32_t bq5[5] = {64, (cuuint32_t)G, (cuuint32_t)(128 / G), 1, (cuuint32_t)P};
+        // O: [panel][row][head][64], a box of B rows x G heads
+        const cuuint64_t dq4[4] = {64, (cuuint64_t)Hq, rows, P};
+        const cuuint64_t sq4[3] = {(cuuint64_t)d * 2, (cuuint64_t)Hq * d * 2, 128};
+        const cuuint32_t bq4[4] = {64, (cuuint32_t)G, (cuuint32_t)B, (cuuint32_t)P};
+        // K, V: [panel][row][head][64], a box of B rows of one head
+        const cuuint64_t dv[4] = {64, (cuuint64_t)Hkv, rows, P};
+        const cuuint64_t sv[3] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2, 128};
+        const cuuint32_t bv[4] = {64, 1, (cuuint32_t)B, (cuuint32_t)P};
+        // W: [panel][row][64], a box of d rows
+        const cuuint64_t dw[3] = {64, (cuuint64_t)Hkv * d, (cuuint64_t)F / 64};
+        const cuuint64_t sw[2] = {(cuuint64_t)F * 2, 128};
+        const cuuint32_t bw[3] = {64, (cuuint32_t)d, (cuuint32_t)F / 64};
+        if (!encode_bf16(&a.tmQ, Q, 5, dq5, sq5, bq5) ||
+            !encode_bf16(&a.tmK, K, 4, dv, sv, bv) || !encode_bf16(&a.tmV, V, 4, dv, sv, bv) ||
+            !encode_bf16(&a.tmW, W, 3, dw, sw, bw) || !encode_bf16(&a.tmO, O, 4, dq4, sq4, bq4))
             return cudaErrorInvalidValue;
     }
     a.O = static_cast<bf16 *>(O);
