@@ -81,7 +81,11 @@ constexpr uint32_t kCmD = 0, kCmP = 128, kCmDSp = 256, kCmK = 288, kCmDSm = 384;
 constexpr uint32_t kCmEK = 320;
 
 struct FusedArgs {
-    CUtensorMap tmQ, tmK, tmV, tmW, tmO;   // Q, O [n*B][Hq][d], K, V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
+    // Q, O [n*B][Hq][d], K, V [n*B][Hkv][d], W [Hkv*d][F]; 128-byte swizzle.  Q, K, V
+    // and W with the 64-element panels as the outermost box dimension (one copy each);
+    // Q's box is 128 / G tokens deep over a dimension of B, so the rows of a unit's
+    // 128-row tile beyond G B are zero-filled.
+    CUtensorMap tmQ, tmK, tmV, tmW, tmO;
     const float *alpha;
     void *const *states;
     unsigned *err;
@@ -373,7 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
         uint32_t kp = 0;
         int nx = 0, nv = 0;
         const uint32_t xbytes =
-            (uint32_t)(d / 64) * (G * B * 128) + (uint32_t)(F / 64) * (d * 128) + (uint32_t)(d / 64) * (B * 128);
+            (uint32_t)(d / 64) * (128 * 128) + (uint32_t)(F / 64) * (d * 128) + (uint32_t)(d / 64) * (B * 128);
         uint8_t *kb = smem + a.off_wk + (F / 64) * d * 128;
         void *nraw = state_raw(a, u_begin, u_end);
         for (int u = u_begin; u < u_end; ++u) {
@@ -390,21 +394,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             uint64_t *xf = xfull;
             if (lane == 0) {
                 mbar_arrive_expect_tx(xf, xbytes);
-                if (q_early)
-                    for (int e = 0; e < d / 64; ++e)
-                        tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xf);
-                for (int f = 0; f < F / 64; ++f)
-                    tma_load_2d(smem + a.off_wk + f * (d * 128), &a.tmW, 64 * f, g * d, xf);
-                for (int e = 0; e < d / 64; ++e)
-                    tma_load_3d(kb + e * (B * 128), &a.tmK, 64 * e, g, r * B, xf);
+                if (q_early) tma_load_5d(smem + a.off_q, &a.tmQ, 0, g * G, 0, r, 0, xf);
+                tma_load_3d(smem + a.off_wk, &a.tmW, 0, g * d, 0, xf);
+                tma_load_4d(kb, &a.tmK, 0, g, r * B, 0, xf);
             }
             __syncwarp();
             if (!q_early && kp > 0) ok = wait_bar(pvdone, (kp - 1) & 1u, fail, wlim);
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
-                if (!q_early)
-                    for (int e = 0; e < d / 64; ++e)
-                        tma_load_3d(smem + a.off_q + e * (128 * 128), &a.tmQ, 64 * e, g * G, r * B, xf);
+                if (!q_early) tma_load_5d(smem + a.off_q, &a.tmQ, 0, g * G, 0, r, 0, xf);
                 mbar_arrive(xf);
             }
             ++nx;
@@ -413,8 +411,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
                 mbar_arrive_expect_tx(vfull, (uint32_t)(d / 64) * (B * 128));
-                for (int e = 0; e < d / 64; ++e)
-                    tma_load_3d(smem + a.off_vb + e * (B * 128), &a.tmV, 64 * e, g, r * B, vfull);
+                tma_load_4d(smem + a.off_vb, &a.tmV, 0, g, r * B, 0, vfull);
             }
             ++nv;
             ++kp;
@@ -892,6 +889,8 @@ bool fused_supported(const hybrid_cfg &c)
     if (c.block_size != 32) return false;
     const int G = c.n_q_heads / c.n_kv_heads;
     if (G * c.block_size > 128) return false;
+    // a unit's Q arrives as one box of 128 / G tokens x G heads
+    if (128 % G != 0) return false;
     const FLayout L = make_flayout(c.head_dim, c.feat_dim, c.block_size);
     const int NCH = c.feat_dim / 32;
     // a ring shorter than a unit stages the output in first-half slots that no
@@ -910,19 +909,26 @@ cudaError_t launch_fused(const hybrid_cfg &c, const void *Q, const void *K, cons
         const int d = c.head_dim, F = c.feat_dim, B = c.block_size, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
         const int G = Hq / Hkv;
         const cuuint64_t rows = (cuuint64_t)n_req * B;
+        const cuuint64_t P = (cuuint64_t)d / 64;
+        // Q: [panel][request][token][head][64]; a box of G heads x 128 / G tokens
+        const cuuint64_t dq5[5] = {64, (cuuint64_t)Hq, (cuuint64_t)B, (cuuint64_t)n_req, P};
+        const cuuint64_t sq5[4] = {(cuuint64_t)d * 2, (cuuint64_t)Hq * d * 2, (cuuint64_t)B * Hq * d * 2, 128};
+        const cuuint32_t bq5[5] = {64, (cuuint32_t)G, (cuuint32_t)(128 / G), 1, (cuuint32_t)P};
+        // K, V: [panel][row][head][64], a box of B rows of one head
+        const cuuint64_t dv[4] = {64, (cuuint64_t)Hkv, rows, P};
+        const cuuint64_t sv[3] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2, 128};
+        const cuuint32_t bv[4] = {64, 1, (cuuint32_t)B, (cuuint32_t)P};
+        // W: [panel][row][64], a box of d rows
+        const cuuint64_t dw[3] = {64, (cuuint64_t)Hkv * d, (cuuint64_t)F / 64};
+        const cuuint64_t sw[2] = {(cuuint64_t)F * 2, 128};
+        const cuuint32_t bw[3] = {64, (cuuint32_t)d, (cuuint32_t)F / 64};
+        // O: one box per staged slot
         const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)Hq, rows};
         const cuuint64_t sq[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hq * d * 2};
-        const cuuint32_t bq[3] = {64, (cuuint32_t)G, (cuuint32_t)B};
-        const cuuint64_t dv[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, rows};
-        const cuuint64_t sv[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
-        const cuuint32_t bv[3] = {64, 1, (cuuint32_t)B};
-        const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
-        const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
-        const cuuint32_t bw[2] = {64, (cuuint32_t)d};
         const cuuint32_t bo[3] = {64, (cuuint32_t)G, (cuuint32_t)(d == 128 ? B : B / 2)};
-        if (!encode_bf16(&a.tmQ, Q, 3, dq, sq, bq) || !encode_bf16(&a.tmK, K, 3, dv, sv, bv) ||
-            !encode_bf16(&a.tmV, V, 3, dv, sv, bv) ||
-            !encode_bf16(&a.tmW, W, 2, dw, sw, bw) || !encode_bf16(&a.tmO, O, 3, dq, sq, bo))
+        if (!encode_bf16(&a.tmQ, Q, 5, dq5, sq5, bq5) || !encode_bf16(&a.tmK, K, 4, dv, sv, bv) ||
+            !encode_bf16(&a.tmV, V, 4, dv, sv, bv) ||
+            !encode_bf16(&a.tmW, W, 3, dw, sw, bw) || !encode_bf16(&a.tmO, O, 3, dq, sq, bo))
             return cudaErrorInvalidValue;
     }
     a.alpha = alpha;
