@@ -47,7 +47,8 @@ constexpr int kOneCtaPerSm = 118 * 1024;
 constexpr uint32_t kColDSp = 256, kColDSm = 384;
 
 struct CommitArgs {
-    CUtensorMap tmV, tmW;   // V [n*T][Hkv][d], W [Hkv*d][F]; 128-byte swizzle
+    CUtensorMap tmV, tmW;   // V [n*T][Hkv][d], W [Hkv*d][F]; 128-byte swizzle, 64-element panels
+                            // as the outermost box dimension (one copy for all of them)
     const bf16 *K;
     void *const *states;
     unsigned *err;
@@ -190,7 +191,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
             if (__any_sync(0xffffffffu, !ok)) break;
             if (lane == 0) {
                 mbar_arrive_expect_tx(wfull, (uint32_t)(F / 64) * atom);
-                for (int f = 0; f < F / 64; ++f) tma_load_2d(wsm + f * atom, &a.tmW, 64 * f, g * d, wfull);
+                tma_load_3d(wsm, &a.tmW, 0, g * d, 0, wfull);
             }
             ++nw;
             for (int j = 0; j < n_chunks; ++j, ++cc) {
@@ -202,9 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
                 if (__any_sync(0xffffffffu, !ok)) break;
                 if (lane == 0) {
                     mbar_arrive_expect_tx(&cfull[b], vbytes);
-                    for (int e = 0; e < d / 64; ++e)
-                        tma_load_3d(cb + atom + e * (kChunk * 128), &a.tmV, 64 * e, g, (int)tok0 + j * kChunk,
-                                    &cfull[b]);
+                    tma_load_4d(cb + atom, &a.tmV, 0, g, (int)tok0 + j * kChunk, 0, &cfull[b]);
                 }
                 ++nv;
                 kt_store(kr, d, cb, lane);
@@ -465,13 +464,14 @@ bool fill_commit_args(const hybrid_cfg &c, const void *K, const void *V, long lo
 {
     const CLayout L = make_clayout(c.head_dim, c.feat_dim);
     const int d = c.head_dim, F = c.feat_dim, Hkv = c.n_kv_heads;
-    const cuuint64_t dv[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, (cuuint64_t)rows};
-    const cuuint64_t sv[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
-    const cuuint32_t bv[3] = {64, 1, (cuuint32_t)kChunk};
-    const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
-    const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
-    const cuuint32_t bw[2] = {64, (cuuint32_t)d};
-    if (!encode_bf16(&a.tmV, V, 3, dv, sv, bv) || !encode_bf16(&a.tmW, W, 2, dw, sw, bw)) return false;
+    // V: [panel][row][head][64], a box of kChunk rows of one head; W: [panel][row][64]
+    const cuuint64_t dv[4] = {64, (cuuint64_t)Hkv, (cuuint64_t)rows, (cuuint64_t)d / 64};
+    const cuuint64_t sv[3] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2, 128};
+    const cuuint32_t bv[4] = {64, 1, (cuuint32_t)kChunk, (cuuint32_t)d / 64};
+    const cuuint64_t dw[3] = {64, (cuuint64_t)Hkv * d, (cuuint64_t)F / 64};
+    const cuuint64_t sw[2] = {(cuuint64_t)F * 2, 128};
+    const cuuint32_t bw[3] = {64, (cuuint32_t)d, (cuuint32_t)F / 64};
+    if (!encode_bf16(&a.tmV, V, 4, dv, sv, bv) || !encode_bf16(&a.tmW, W, 3, dw, sw, bw)) return false;
     a.K = static_cast<const bf16 *>(K);
     a.states = states;
     a.err = err;
