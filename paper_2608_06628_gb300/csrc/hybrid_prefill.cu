@@ -265,19 +265,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
                 if (p.first) {
                     if (s > 0 && !wait_bar(wfree, (s - 1) & 1u, fail)) break;
                     mbar_arrive_expect_tx(wfull, (uint32_t)(F / 64) * tile);
-                    for (int f = 0; f < F / 64; ++f) tma_load_2d(smem + a.off_w + f * tile, &a.tmW, 64 * f, g * d, wfull);
+                    tma_load_3d(smem + a.off_w, &a.tmW, 0, g * d, 0, wfull);
                     ++nw;
                     ++s;
                 }
                 if (i > 0 && !wait_bar(kfree, (i - 1) & 1u, fail)) break;
                 mbar_arrive_expect_tx(kfull, (uint32_t)(d / 64) * kAtom);
-                for (int e = 0; e < d / 64; ++e) tma_load_3d(smem + a.off_k + e * kAtom, &a.tmK, 64 * e, g, row0, kfull);
+                tma_load_4d(smem + a.off_k, &a.tmK, 0, g, row0, 0, kfull);
                 ++nk;
                 const int vb = i & 1;
                 if (i >= 2 && !wait_bar(&vfree[vb], ((i - 2) >> 1) & 1u, fail)) break;
                 mbar_arrive_expect_tx(&vfull[vb], (uint32_t)(d / 64) * kAtom);
-                for (int e = 0; e < d / 64; ++e)
-                    tma_load_3d(smem + a.off_v + vb * 2 * kAtom + e * kAtom, &a.tmV, 64 * e, g, row0, &vfull[vb]);
+                tma_load_4d(smem + a.off_v + vb * 2 * kAtom, &a.tmV, 0, g, row0, 0, &vfull[vb]);
                 ++nv;
                 ++i;
             }
@@ -580,14 +579,16 @@ bool fill_prefill_args(const hybrid_cfg &c, const void *K, const void *V, long l
 {
     const PLayout L = make_playout(c.head_dim, c.feat_dim);
     const int d = c.head_dim, F = c.feat_dim, Hkv = c.n_kv_heads;
-    const cuuint64_t dk[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, (cuuint64_t)rows};
-    const cuuint64_t sk[2] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2};
-    const cuuint32_t bk[3] = {64, 1, (cuuint32_t)kCT};
-    const cuuint64_t dw[2] = {(cuuint64_t)F, (cuuint64_t)Hkv * d};
-    const cuuint64_t sw[1] = {(cuuint64_t)F * 2};
-    const cuuint32_t bw[2] = {64, (cuuint32_t)d};
-    if (!encode_bf16(&a.tmK, K, 3, dk, sk, bk) || !encode_bf16(&a.tmV, V, 3, dk, sk, bk) ||
-        !encode_bf16(&a.tmW, W, 2, dw, sw, bw))
+    // K, V: [panel][row][head][64], a box of kCT rows of one head; W: [panel][row][64]
+    // (the 64-element panels as the outermost box dimension: one copy for all of them)
+    const cuuint64_t dk[4] = {64, (cuuint64_t)Hkv, (cuuint64_t)rows, (cuuint64_t)d / 64};
+    const cuuint64_t sk[3] = {(cuuint64_t)d * 2, (cuuint64_t)Hkv * d * 2, 128};
+    const cuuint32_t bk[4] = {64, 1, (cuuint32_t)kCT, (cuuint32_t)d / 64};
+    const cuuint64_t dw[3] = {64, (cuuint64_t)Hkv * d, (cuuint64_t)F / 64};
+    const cuuint64_t sw[2] = {(cuuint64_t)F * 2, 128};
+    const cuuint32_t bw[3] = {64, (cuuint32_t)d, (cuuint32_t)F / 64};
+    if (!encode_bf16(&a.tmK, K, 4, dk, sk, bk) || !encode_bf16(&a.tmV, V, 4, dk, sk, bk) ||
+        !encode_bf16(&a.tmW, W, 3, dw, sw, bw))
         return false;
     a.states = states;
     a.err = err;
