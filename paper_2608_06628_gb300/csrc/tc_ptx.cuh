@@ -137,6 +137,20 @@ __device__ __forceinline__ void tma_load_5d(void *dst, const void *tmap, int c0,
         "l"(tmap), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4), "r"(smem_u32(bar))
         : "memory");
 }
+// Prefetch of a tensor-map box into L2: nothing lands in shared memory and no barrier is
+// signalled, so it binds no value (the later load reads whatever L2 then holds).
+__device__ __forceinline__ void tma_prefetch_4d(const void *tmap, int c0, int c1, int c2, int c3)
+{
+    asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(tmap), "r"(c0),
+                 "r"(c1), "r"(c2), "r"(c3)
+                 : "memory");
+}
+__device__ __forceinline__ void tma_prefetch_5d(const void *tmap, int c0, int c1, int c2, int c3, int c4)
+{
+    asm volatile("cp.async.bulk.prefetch.tensor.5d.L2.global.tile [%0, {%1, %2, %3, %4, %5}];" ::"l"(tmap), "r"(c0),
+                 "r"(c1), "r"(c2), "r"(c3), "r"(c4)
+                 : "memory");
+}
 
 // Tiled tensor copy shared -> global through a tensor map (bulk-group completion).
 __device__ __forceinline__ void tma_store_3d(const void *tmap, int c0, int c1, int c2, const void *src)
