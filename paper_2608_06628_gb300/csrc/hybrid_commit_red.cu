@@ -49,6 +49,7 @@ constexpr uint32_t kColDSp = 256, kColDSm = 384;
 struct CommitArgs {
     CUtensorMap tmV, tmW;   // V [n*T][Hkv][d], W [Hkv*d][F]; 128-byte swizzle, 64-element panels
                             // as the outermost box dimension (one copy for all of them)
+    CUtensorMap tmK;        // K as V (used only to prefetch K into L2; K is read by the warps)
     const bf16 *K;
     void *const *states;
     unsigned *err;
@@ -170,6 +171,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_commit_red(const __grid_constan
     __syncthreads();
     tc_fence_after();
     if (tid == 0) griddep_launch_dependents();
+    // the first chunks of K and V of the CTA's first units into L2 while the previous kernel
+    // drains: a prefetch brings no value into the SM, so it needs no ordering after it
+    if (tid == 64)
+        for (int u = u_begin; u < u_end && u < u_begin + 2; ++u) {
+            const int Tu = unit_len(a, u), g = (u / a.n_pass) % a.Hkv;
+            const int tok0 = (int)unit_tok0(a, u);
+            for (int j = 0; j * kChunk < Tu && j < 2; ++j) {
+                tma_prefetch_4d(&a.tmK, 0, g, tok0 + j * kChunk, 0);
+                tma_prefetch_4d(&a.tmV, 0, g, tok0 + j * kChunk, 0);
+            }
+        }
     griddep_wait();
     const uint32_t tmem = *tmem_holder;
     uint8_t *wsm = smem + a.off_w;
@@ -471,7 +483,9 @@ bool fill_commit_args(const hybrid_cfg &c, const void *K, const void *V, long lo
     const cuuint64_t dw[3] = {64, (cuuint64_t)Hkv * d, (cuuint64_t)F / 64};
     const cuuint64_t sw[2] = {(cuuint64_t)F * 2, 128};
     const cuuint32_t bw[3] = {64, (cuuint32_t)d, (cuuint32_t)F / 64};
-    if (!encode_bf16(&a.tmV, V, 4, dv, sv, bv) || !encode_bf16(&a.tmW, W, 3, dw, sw, bw)) return false;
+    if (!encode_bf16(&a.tmV, V, 4, dv, sv, bv) || !encode_bf16(&a.tmK, K, 4, dv, sv, bv) ||
+        !encode_bf16(&a.tmW, W, 3, dw, sw, bw))
+        return false;
     a.K = static_cast<const bf16 *>(K);
     a.states = states;
     a.err = err;

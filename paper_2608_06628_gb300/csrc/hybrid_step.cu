@@ -224,7 +224,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
     // the Q, K and V boxes of the CTA's units into L2 while the previous kernel drains: a
     // prefetch brings no value into the SM, so it needs no ordering after that kernel
     if (tid == 64)
-        for (int u = u_begin; u < u_end && u < u_begin + 2; ++u) {
+        for (int u = u_begin; u < u_end && u < u_begin + 4; ++u) {
             const int r = u / a.Hkv, g = u % a.Hkv;
             tma_prefetch_5d(&a.tmQ, 0, g * G, 0, r, 0);
             tma_prefetch_4d(&a.tmK, 0, g, r * B, 0);
