@@ -207,6 +207,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tc(const __grid_constant__
     }
     __syncthreads();
     tc_fence_after();
+    // launched with programmatic stream serialisation: the set-up above may run while the
+    // previous kernel of the stream drains, and so may L2 prefetches of the first unit's Q, K
+    // and V (a prefetch binds no value); nothing below reads global memory before that kernel
+    // has completed
+    if (tid == 0) griddep_launch_dependents();
+    if (tid == 32 && u_begin < u_end) {
+        const int r = u_begin / a.Hkv, g = u_begin % a.Hkv;
+        if (kSpread) tma_prefetch_5d(&a.tmQ, 0, g, 0, r * (B / 16), 0);
+        tma_prefetch_4d(&a.tmK, 0, g, r * B, 0);
+        tma_prefetch_4d(&a.tmV, 0, g, r * B, 0);
+    }
+    griddep_wait();
     const uint32_t tmem = *tmem_holder;
 
     // the first unit from u on whose state pointer is usable (u_end if none); each
@@ -776,8 +788,17 @@ cudaError_t launch_attn_tc(const hybrid_cfg &c, const void *Q, const void *K, co
     if (e != cudaSuccess) return e;
     a.n_units = n_req * c.n_kv_heads;
     const int grid = a.n_units < pipe::sm_count() ? a.n_units : pipe::sm_count();
-    kern<<<grid, kThreads, L.bytes, st>>>(a);
-    return cudaGetLastError();
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid);
+    lc.blockDim = dim3(kThreads);
+    lc.dynamicSmemBytes = L.bytes;
+    lc.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 1;
+    return cudaLaunchKernelEx(&lc, kern, a);
 }
 
 }  // namespace hyb
