@@ -793,7 +793,9 @@ def run_hybrid(args, wl):
 
     e2e_bufs = [torch.empty_like(hQKV, device=dev) for _ in sets]
     e2e_sets = [dict(s, **split_qkv(b)) for s, b in zip(sets, e2e_bufs)]
-    n_e2e = 2 * n_sets
+    # a replay starts with the pipeline empty and ends by draining it (its first copy in and
+    # its last copy out overlap nothing), so one graph holds many steps
+    n_e2e = 8 * n_sets
     cin, cout = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
     g_e2e = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_e2e, stream=side):
