@@ -453,8 +453,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     // one bulk group per tile; the two output slots are freed as
                     // soon as their reductions have read them
                     for (int c = h * NCH; c < (h + 1) * NCH; ++c) {
-                        bulk_reduce_add_f32(Sg + (size_t)c * 32 * d, ring + (size_t)((q + c) % NS) * chunk_bytes,
-                                            chunk_bytes);
+                        bulk_s2g(Sg + (size_t)c * 32 * d, ring + (size_t)((q + c) % NS) * chunk_bytes, chunk_bytes);
                         bulk_commit();
                     }
                     if (h == ocm / NCH) {
@@ -837,9 +836,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
 
             {
                 // ---- state update: S^T += dS^T for a feature half as soon as the readout
-                // has consumed its tiles (first half now, second after R-): dS^T rows go
-                // into the tiles' slots and the storer adds them into the state by
-                // bulk reductions (float32 add at L2)
+                // has consumed its tiles (first half now, second after R-): each tile's slot
+                // still holds the tile as read, dS^T is added to it there (float32), and the
+                // storer writes the tiles back with plain bulk stores
                 const int e = row;
 #pragma unroll 1
                 for (int h = 0; h < 2; ++h) {
@@ -848,17 +847,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                     tc_fence_after();
                     const uint32_t src = tmem + (h == 0 ? kCmDSp : kCmDSm) + lane_off;
                     auto upd = [&](int k) {
-                        // the readout has consumed the tile: its slot now takes dS^T,
-                        // which the storer adds into the state in global memory
+                        // the readout has consumed the tile: S^T + dS^T replaces it in its
+                        // slot, and the storer writes it over the state in global memory
                         uint8_t *rowp = ring + (size_t)((q + h * NCH + k) % NS) * chunk_bytes + e * 128;
                         float v[32];
                         tmem_ld32(src + 32 * k, v);
                         tmem_wait_ld();
                         if (!bad2 && e < d) {
 #pragma unroll
-                            for (int gq = 0; gq < 8; ++gq)
-                                *reinterpret_cast<float4 *>(rowp + ((gq ^ (e & 7)) << 4)) =
-                                    make_float4(v[4 * gq], v[4 * gq + 1], v[4 * gq + 2], v[4 * gq + 3]);
+                            for (int gq = 0; gq < 8; ++gq) {
+                                float4 *p4 = reinterpret_cast<float4 *>(rowp + ((gq ^ (e & 7)) << 4));
+                                const float4 s4 = *p4;
+                                *p4 = make_float4(s4.x + v[4 * gq], s4.y + v[4 * gq + 1], s4.z + v[4 * gq + 2],
+                                                  s4.w + v[4 * gq + 3]);
+                            }
                         }
                     };
 #pragma unroll 1
