@@ -16,8 +16,8 @@
 //              operand image, see hybrid.h).
 //   warp 1     MMA issuer (one thread); owns the Tensor Memory allocation.
 //   warp 2     producer: TMA of Q, W, K and V.
-//   warp 3     storer: bulk reduce-adds of the dS^T tiles into the state, the
-//              store of z, and TMA stores of the output tile.
+//   warp 3     storer: bulk stores of the updated state tiles and of z, and TMA
+//              stores of the output tile.
 //   warps 4-11 math: two threads per query row (one per TMEM lane and "part");
 //              a part owns every other 32-feature chunk of each half of phi.
 //
@@ -41,11 +41,13 @@
 //
 // Tensor Memory: [D | phi | dS+ | dS-].  phi+ is parked in the dS- columns
 // while R+ reads it; phi- replaces U in the phi columns.  Once a half's tiles
-// have been read out, their ring slots take that half's dS^T rows and the
-// storer adds them into the state in global memory by bulk reduce-adds (the
-// float32 add happens at L2), so the SM never writes a state tile back.  V, P'
-// and phi(K) share the Q region once g1 has consumed Q, so all 2F/32 state
-// tiles of a unit fit in the ring.
+// have been read out, each still sits in its ring slot as read: the math warps
+// add that half's dS^T rows to it there (float32) and the storer writes the
+// tiles back over the state with plain bulk stores (a bulk reduce-add at L2
+// would do the same add, but with every SM committing at once L2 takes 2.8 TB/s
+// of added data, against ~6 TB/s of plain stores).  V, P' and phi(K) share the
+// Q region once g1 has consumed Q, so all 2F/32 state tiles of a unit fit in
+// the ring.
 //
 // MMA cost note: on this part a tcgen05.mma with M = 128 costs its issuing thread
 // about the same time for any N up to 128-256, so contractions are shaped for few,
@@ -168,8 +170,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
     const int NCH = F / 32;          // 32-feature chunks (state tiles) per half of phi
     const int NC = 2 * NCH;          // state tiles per unit
     // the output tile is staged in the slots of tiles ocm, ocm + 1 of its unit:
-    // the first two second-half tiles (their increments are reduce-added before
-    // the epilogue), so the next unit's first-half tiles, needed first, can enter
+    // the first two second-half tiles (their updated copies are stored before the
+    // epilogue), so the next unit's first-half tiles, needed first, can enter
     // the ring early; if a unit has more tiles than the ring, first-half tiles
     // that no later tile of the unit reuses
     const int ocm = NC > NS ? NC - NS : NCH;
@@ -451,13 +453,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
                 for (int h = 0; h < 2 && ok; ++h) {
                     if (!wait_bar(&tready[h], kp & 1u, fail, wlim)) { ok = false; break; }
                     // one bulk group per tile; the two output slots are freed as
-                    // soon as their reductions have read them
+                    // soon as their stores have read them
                     for (int c = h * NCH; c < (h + 1) * NCH; ++c) {
                         bulk_s2g(Sg + (size_t)c * 32 * d, ring + (size_t)((q + c) % NS) * chunk_bytes, chunk_bytes);
                         bulk_commit();
                     }
                     if (h == ocm / NCH) {
-                        // the output slots may be written once their reductions have read them
+                        // the output slots may be written once their stores have read them
                         if ((h + 1) * NCH - (ocm + 2) >= 2) bulk_wait_read_2();
                         else bulk_wait_read_all();
                         mbar_arrive(ofree);
