@@ -201,6 +201,36 @@ def test_tied_keys(wl):
     assert_parity(got, want, wl.io_dtype, "tied keys", units="out")
 
 
+# Sec. 3.1's two forms of the cross-block branch: the recurrent state (S, z) built by
+# the CUDA commits and read by the CUDA step, against the oracle's token-by-token sum
+# over the explicit prefix (lin_num = sum_t (phi(q) . phi(k_t)) v_t, Eq. 1's quadratic
+# form with the Hedgehog map), which never forms a state
+EQ1_WL = [(W_("eq1_gqa_bf16", BF16, 3, 8, 2, 128, 128, 32, 53), [0, 64, 160]),
+          (W_("eq1_f256_g1_bf16", BF16, 3, 2, 2, 128, 256, 64, 54), [128, 0, 192])]
+
+
+@pytest.mark.parametrize("wl,plen", EQ1_WL, ids=[w.name for w, _ in EQ1_WL])
+def test_state_route_matches_quadratic_prefix_form(wl, plen):
+    pair = Pair(wl, tracked=[])
+    plen = np.asarray(plen)
+    P_max = int(plen.max())
+    Kp = torch.zeros((wl.n_req, max(P_max, 1), wl.Hkv, wl.d), dtype=wl.io_dtype)
+    Vp = torch.zeros_like(Kp)
+    for b in range(P_max // wl.B):
+        reqs = np.nonzero(plen > b * wl.B)[0]
+        K, V = wk.prefix_kv(wl, b, pair.dev)
+        idx = torch.as_tensor(reqs, device=pair.dev)
+        pair.commit(K[idx], V[idx], reqs)
+        Kp[reqs, b * wl.B:(b + 1) * wl.B] = K[idx].cpu()
+        Vp[reqs, b * wl.B:(b + 1) * wl.B] = V[idx].cpu()
+    Q, K, V = wk.block_qkv(wl, "eq1", pair.dev)
+    O = torch.empty_like(Q)
+    H.hybrid_block_attn(pair.cfg, Q, K, V, pair.W, pair.alpha, pair.ptrs, wl.n_req, O)
+    H.hybrid_check()
+    want = pair.orc.block_attn_prefix(h64(Q), h64(K), h64(V), pair.W64, pair.alpha64, h64(Kp), h64(Vp), plen)
+    assert_parity(h64(O), want, wl.io_dtype, "state route vs prefix form", units="out")
+
+
 def test_permuted_and_subset_pointer_arrays():
     """A batch may list any subset of states in any order: the output of a
     request depends only on its own state pointer."""
