@@ -6,13 +6,17 @@
 //
 // Work unit = (request r, state head g): the G*B query rows of the unit share one
 // state.  Warp roles (12 warps):
-//   warp 0     ring producer: per unit Q (TMA) and then the F/32 pairs of state
-//              tiles (phi+ tile c with phi- tile c, 1-D bulk copies) into an
-//              NS-slot ring of 2 d x 128-byte slots (the state layout is the MMA
-//              operand image, see hybrid.h); z beside the ring
+//   warp 0     ring producer: per unit Q (one TMA box of 128 rows, those beyond
+//              G B zero-filled) and then the F/32 pairs of state tiles (phi+ tile
+//              c with phi- tile c, 1-D bulk copies) into an NS-slot ring of 2 d x
+//              128-byte slots (the state layout is the MMA operand image, see
+//              hybrid.h); z beside the ring
 //   warp 1     MMA issuer A; owns the Tensor Memory allocation:
 //              U = Q W, the phi+ readout, P'V
-//   warp 2     producer: TMA of W, K and V, and the TMA stores of the output tile
+//   warp 2     producer: TMA of W, K and V (one box each), and the TMA store of
+//              the output tile
+// Before its grid-dependency wait a CTA prefetches the Q, K and V boxes of its
+// first units into L2 while the previous kernel drains.
 //   warp 3     MMA issuer B: the scores Q K^T (K, as loaded, is the K-major
 //              operand), the phi- readout
 //   warps 4-11 math: two threads per query row (one warp per TMEM lane quarter
