@@ -652,7 +652,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fused(const __grid_constant__ F
             // and P' absorb the factor (phi- x sp/sn, P' = w sp e^s).  This needs the
             // unshifted softmax mass w sp e^(s) inside float range; a warp with any row
             // beyond e^60 rescales phi+ exactly once sigma is known (phase C).  Padding
-            // lanes (stale Q rows) do not count.
+            // lanes (rows beyond the unit's G B query rows) do not count.
             const bool fast = __all_sync(0xffffffffu, !valid || !(lw + ms * a.scale + __logf(sp) > 60.f));
             if (fast) {
                 tmem_wait_st();

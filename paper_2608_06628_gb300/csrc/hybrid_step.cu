@@ -537,7 +537,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_step(const __grid_constant__ St
             }
             // fast: w sp e^(max s) <= w F e^(max s) stays below e^60 for every valid row of
             // the warp, so phi+ and phi- are released unnormalised as soon as they are
-            // written (padding lanes, whose Q rows are stale, never hold a warp back)
+            // written (padding lanes, the rows beyond the unit's G B query rows, never
+            // hold a warp back)
             const bool fast = __all_sync(0xffffffffu, !valid || !(lw + ms * a.scale + log_f > 60.f));
 
             // ---- phase B: phi+ then phi- into Tensor Memory, with their sums and
