@@ -4,11 +4,14 @@
   from the tensors the synthetic inputs actually have and from the library's own
   state size, against bench.algorithmic_bytes;
 * the DRAM-traffic record: keyed by a hash of the kernel's sources that ignores
-  comments and whitespace, and dropped (null) as soon as the code changes.
+  comments and whitespace, and dropped (null) as soon as the code changes;
+* the reference arm's JSON line (the oracle on the host cores) and its rank rule.
 """
 import json
 import os
 import shutil
+import subprocess
+import sys
 
 import bench
 from paper_2608_06628_gb300 import build as B
@@ -76,3 +79,45 @@ def test_committed_traffic_records_are_consistent():
         assert rec["bytes_per_launch"] == rec["dram_read"] + rec["dram_write"], name
         ratio = rec["bytes_per_launch"] / rec["algorithmic_bytes"]
         assert abs(ratio - rec["traffic_over_algorithmic"]) < 1e-3, name
+
+
+def _run_bench(args, env_extra=None):
+    env = dict(os.environ, **(env_extra or {}))
+    env.pop("CUDA_VISIBLE_DEVICES", None)
+    return subprocess.run([sys.executable, "bench.py", *args], cwd=bench.ROOT, env=env,
+                          capture_output=True, text=True, timeout=600)
+
+
+def test_reference_arm_prints_one_contract_line():
+    """bench.py --impl reference (the fp64 oracle on the host cores) prints one
+    JSON line with the keys the driver reads, on the arm's own metric and config."""
+    B.build()
+    out = _run_bench(["--impl", "reference", "--config", "c1_fp32_tiny", "--steps", "2", "--warmup", "3"])
+    assert out.returncode == 0, out.stderr[-2000:]
+    lines = [l for l in out.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, out.stdout
+    line = json.loads(lines[0])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+                "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config",
+                "cpu_baseline", "e2e"):
+        assert key in line, key
+    assert line["impl"] == "reference" and line["metric"] == bench.METRIC
+    assert line["steps"] == 2 and line["warmup"] == 3 and line["n_gpus"] == 1
+    assert line["higher_is_better"] is True and line["unit"] == "tokens/s" and line["value"] > 0
+    assert line["config"]["workload"] == "c1_fp32_tiny"
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == line["value"] and cb["sample"]
+    assert line["e2e"] == {"value": line["value"], "unit": "tokens/s",
+                           "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
+def test_reference_arm_other_ranks_exit_without_work():
+    out = _run_bench(["--impl", "reference", "--config", "c1_fp32_tiny", "--steps", "2", "--warmup", "3"],
+                     {"RANK": "1", "LOCAL_RANK": "1", "WORLD_SIZE": "2"})
+    assert out.returncode == 0, out.stderr[-2000:]
+    assert out.stdout.strip() == ""
+
+
+def test_warmup_below_three_is_refused():
+    out = _run_bench(["--impl", "reference", "--config", "c1_fp32_tiny", "--steps", "1", "--warmup", "2"])
+    assert out.returncode != 0 and "warmup" in out.stderr
