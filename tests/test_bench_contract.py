@@ -5,13 +5,15 @@
   state size, against bench.algorithmic_bytes;
 * the DRAM-traffic record: keyed by a hash of the kernel's sources that ignores
   comments and whitespace, and dropped (null) as soon as the code changes;
-* the reference arm's JSON line (the oracle on the host cores) and its rank rule.
+* the reference arm's JSON line (the oracle on the host cores) and its rank rule;
+* the clocks record, parsed from nvidia-smi's CSV.
 """
 import json
 import os
 import shutil
 import subprocess
 import sys
+import time
 
 import bench
 from paper_2608_06628_gb300 import build as B
@@ -121,3 +123,33 @@ def test_reference_arm_other_ranks_exit_without_work():
 def test_warmup_below_three_is_refused():
     out = _run_bench(["--impl", "reference", "--config", "c1_fp32_tiny", "--steps", "1", "--warmup", "2"])
     assert out.returncode != 0 and "warmup" in out.stderr
+
+
+def test_clock_sampler_reads_clocks_and_throttle_reasons(tmp_path, monkeypatch):
+    """The clocks record of the bench line, from a stand-in nvidia-smi that prints
+    the queried CSV fields: median SM clock, the maximum, and every throttle reason
+    seen Active inside the window."""
+    rows = ["0, 2070, 2070, 610.5, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active",
+            "0, 1965, 2070, 1398.0, 0x0000000000000004, Not Active, Not Active, Not Active, Active",
+            "0, 2032, 2070, 1012.2, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active",
+            "0, [N/A], 2070, [N/A], [N/A], [N/A], [N/A], [N/A], [N/A]",
+            "0, 2070, 2070"]
+    fake = tmp_path / "nvidia-smi"
+    fake.write_text("#!/bin/sh\n" + "".join(f"echo '{r}'\n" for r in rows) + "exec sleep 30\n")
+    fake.chmod(0o755)
+    monkeypatch.setenv("PATH", f"{tmp_path}{os.pathsep}{os.environ['PATH']}")
+    t0 = time.time()
+    cs = bench.ClockSampler(None)
+    cs.start()
+    deadline = time.time() + 20
+    while len(cs.samples) < 3 and time.time() < deadline:
+        time.sleep(0.05)
+    cs.stop()
+    t1 = time.time()
+    assert len(cs.samples) == 3   # the unparsable and short rows are skipped
+    s = cs.summary(t0, t1)
+    assert s["sm_mhz"] == 2032.0 and s["sm_max_mhz"] == 2070.0
+    assert s["reasons"] == ["sw_power_cap"] and s["samples"] == 3
+    # a window with no samples says so instead of reporting a clock
+    far = cs.summary(t1 + 100, t1 + 101)
+    assert far["sm_mhz"] is None and far["samples"] == 0
