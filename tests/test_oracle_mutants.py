@@ -3,7 +3,8 @@
 
 This shows that the pins constrain every part of the oracle: the feature map,
 its W orientation, the softmax scale, the gate, the shared normaliser, the
-commit, the GQA head mapping and the in-block mask.  Mutants run in a
+commit, the GQA head mapping, the in-block mask, the per-head and per-request
+indexing of every route and the training form's forward and gradients.  Mutants run in a
 subprocess, so a mutant that crashes counts as caught without harming the
 test process.
 """
@@ -60,6 +61,27 @@ MUTANTS = [
     ("train dalpha without the sigmoid slope", "dalpha[h] = a * w * (1.0 - w);", "dalpha[h] = a;"),
     ("train state gradient of own block", "dS[(size_t)f * d + e] += phi[f] * dN[e];",
      "dS[(size_t)f * d + e] += phi[f] * dN[(e + 1) % d];"),
+    # head and request indexing of the inference routes
+    ("commit uses state head 0's W", "const double *Wg = c->W ? c->W + (size_t)g * d * F : NULL;\n    for (int t = 0; t < c->T; ++t) {",
+     "const double *Wg = c->W ? c->W + (size_t)0 * g * d * F : NULL;\n    for (int t = 0; t < c->T; ++t) {"),
+    ("step uses state head 0's W", "const double *Wg = c->W ? c->W + (size_t)g * d * F : NULL;\n\n    double *u = scratch;",
+     "const double *Wg = c->W ? c->W + (size_t)0 * g * d * F : NULL;\n\n    double *u = scratch;"),
+    ("commit into state head 0", "double *S = c->S + ((size_t)r * c->Hkv + g) * P2 * d;\n    double *z = c->z",
+     "double *S = c->S + ((size_t)r * c->Hkv + 0 * g) * P2 * d;\n    double *z = c->z"),
+    ("prefix values of the mirrored head", "const double *vt = c->Vp + (((size_t)r * c->P_max + t) * c->Hkv + g) * d;",
+     "const double *vt = c->Vp + (((size_t)r * c->P_max + t) * c->Hkv + (c->Hkv - 1 - g)) * d;"),
+    ("prefix kernel over phi+ only", "for (int f = 0; f < P2; ++f) kern += phi_q[f] * phi_k[f];",
+     "for (int f = 0; f < P2 / 2; ++f) kern += phi_q[f] * phi_k[f];"),
+    ("state readout over phi+ only", "for (int f = 0; f < P2; ++f) {\n        for (int e = 0; e < d; ++e) lin_num[e] += phi_q[f] * S[(size_t)f * d + e];",
+     "for (int f = 0; f < P2 / 2; ++f) {\n        for (int e = 0; e < d; ++e) lin_num[e] += phi_q[f] * S[(size_t)f * d + e];"),
+    ("block keys of the next request", "const size_t kv0 = ((size_t)r * B * c->Hkv + g) * d;",
+     "const size_t kv0 = ((size_t)((r + 1) % c->n_req) * B * c->Hkv + g) * d;"),
+    ("query row reversed", "const double *q = c->Q + (((size_t)r * B + i) * c->Hq + h) * d;",
+     "const double *q = c->Q + (((size_t)r * B + (B - 1 - i)) * c->Hq + h) * d;"),
+    ("output of the next query head", "merge(w, sm_num, sm_den, lin_num, lin_den, d, c->O + (((size_t)r * B + i) * c->Hq + h) * d);",
+     "merge(w, sm_num, sm_den, lin_num, lin_den, d, c->O + (((size_t)r * B + i) * c->Hq + (h + 1) % c->Hq) * d);"),
+    ("gate of the first head of the group", "const double w = gate(c->alpha[h]);\n\n    for (int i = 0; i < B; ++i) {",
+     "const double w = gate(c->alpha[g * (c->Hq / c->Hkv)]);\n\n    for (int i = 0; i < B; ++i) {"),
 ]
 
 
