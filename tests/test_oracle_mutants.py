@@ -80,6 +80,10 @@ MUTANTS = [
      "const double *q = c->Q + (((size_t)r * B + (B - 1 - i)) * c->Hq + h) * d;"),
     ("output of the next query head", "merge(w, sm_num, sm_den, lin_num, lin_den, d, c->O + (((size_t)r * B + i) * c->Hq + h) * d);",
      "merge(w, sm_num, sm_den, lin_num, lin_den, d, c->O + (((size_t)r * B + i) * c->Hq + (h + 1) % c->Hq) * d);"),
+    ("feature map with head 0's W", "const double *Wg = W + (size_t)(h / group) * d * F;",
+     "const double *Wg = W + (size_t)0 * (h / group) * d * F;"),
+    ("feature map W by head modulo", "const double *Wg = W + (size_t)(h / group) * d * F;",
+     "const double *Wg = W + (size_t)(h % n_kv_heads) * d * F;"),
     ("gate of the first head of the group", "const double w = gate(c->alpha[h]);\n\n    for (int i = 0; i < B; ++i) {",
      "const double w = gate(c->alpha[g * (c->Hq / c->Hkv)]);\n\n    for (int i = 0; i < B; ++i) {"),
 ]
