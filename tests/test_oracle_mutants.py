@@ -61,6 +61,16 @@ MUTANTS = [
     ("train dalpha without the sigmoid slope", "dalpha[h] = a * w * (1.0 - w);", "dalpha[h] = a;"),
     ("train state gradient of own block", "dS[(size_t)f * d + e] += phi[f] * dN[e];",
      "dS[(size_t)f * d + e] += phi[f] * dN[(e + 1) % d];"),
+    ("train backward query heads of group 0", "const int h = g * G + hl;", "const int h = hl;"),
+    ("train backward drops the key-side W gradient", "phi_backward_add(k, phi, gphi, d, F, du, dW);",
+     "if (0) phi_backward_add(k, phi, gphi, d, F, du, dW);"),
+    ("train backward drops the query-side W gradient", "phi_backward_add(q, phi, gphi, d, F, du, dW);",
+     "if (0) phi_backward_add(q, phi, gphi, d, F, du, dW);"),
+    ("train dalpha without the softmax denominator", "dw += dD * sm_den;", "dw += 0.0 * sm_den;"),
+    ("train backward prefix state includes its own block", "const size_t t0 = (size_t)s * c->L + (size_t)(n - 1) * B;",
+     "const size_t t0 = (size_t)s * c->L + (size_t)n * B;"),
+    ("train forward every sequence reads the first", "const size_t t0 = (size_t)s * c->L + (size_t)n * B;   /* first token of block n */",
+     "const size_t t0 = (size_t)0 * s * c->L + (size_t)n * B;   /* first token of block n */"),
     # head and request indexing of the inference routes
     ("commit uses state head 0's W", "const double *Wg = c->W ? c->W + (size_t)g * d * F : NULL;\n    for (int t = 0; t < c->T; ++t) {",
      "const double *Wg = c->W ? c->W + (size_t)0 * g * d * F : NULL;\n    for (int t = 0; t < c->T; ++t) {"),
