@@ -194,3 +194,31 @@ def test_debug_arm_wait_timeout_host_checks(L):
     assert L.hybrid_debug_arm_wait_timeout(10_000_000_001) == H.HYBRID_ERR_INVALID_ARG
     assert L.hybrid_debug_arm_wait_timeout(1_000_000) == H.HYBRID_OK
     assert L.hybrid_debug_arm_wait_timeout(0) == H.HYBRID_OK
+
+
+def test_state_pool_slots_and_pointer_arrays(L):
+    """The slab allocator behind a ragged batch (host memory here; the pointer
+    arithmetic is the same on the device): one slot per request, each the
+    library's state size, 16-byte aligned, and a batch is any subset of slots in
+    any order."""
+    import torch
+    from paper_2608_06628_gb300.state_pool import StatePool
+    c = cfg(d=128, F=128, Hq=16, Hkv=4)
+    pool = StatePool(c, 5, "cpu")
+    sb = H.hybrid_state_bytes(c)
+    assert pool.slot_bytes == sb == 4 * (2 * 128 * 128 + 2 * 128) * 4
+    assert pool.slab.numel() * 4 == 5 * sb
+    assert all(pool.slot_ptr(i) % 16 == 0 for i in range(5))
+    order = [3, 0, 4]
+    ptrs = pool.ptr_array(order)
+    assert ptrs.dtype == torch.int64 and ptrs.tolist() == [pool.slot_ptr(i) for i in order]
+    assert pool.all_ptrs().tolist() == [pool.base + i * sb for i in range(5)]
+    # slot views alias the slab and do not overlap
+    for i in range(5):
+        pool.slot_view(i).fill_(float(i))
+    for i in range(5):
+        v = pool.slot_view(i)
+        assert v.data_ptr() == pool.slot_ptr(i) and v.numel() * 4 == sb
+        assert bool((v == float(i)).all())
+    with pytest.raises(ValueError):
+        StatePool(cfg(d=96), 1, "cpu")
