@@ -222,3 +222,48 @@ def test_state_pool_slots_and_pointer_arrays(L):
         assert bool((v == float(i)).all())
     with pytest.raises(ValueError):
         StatePool(cfg(d=96), 1, "cpu")
+
+
+def declared_signatures():
+    """name -> (return type, list of parameter declarations), from include/*.h
+    (comments removed)."""
+    sigs = {}
+    for hdr in sorted(os.listdir(os.path.join(ROOT, "include"))):
+        if not hdr.endswith(".h"):
+            continue
+        text = open(os.path.join(ROOT, "include", hdr)).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", "", text)
+        for m in re.finditer(r"([A-Za-z_][\w \t*]*?)\s*\b(hybrid_[a-z_]+)\s*\(([^;{]*?)\)\s*;", text, re.S):
+            args = " ".join(m.group(3).split())
+            sigs[m.group(2)] = (" ".join(m.group(1).split()),
+                                [] if args in ("", "void") else [a.strip() for a in args.split(",")])
+    return sigs
+
+
+def _ctype_of(decl):
+    if "*" in decl or decl.startswith("cudaStream_t"):
+        return "pointer"
+    kind = decl.rsplit(" ", 1)[0].replace("const ", "")
+    return {"int": ctypes.c_int, "size_t": ctypes.c_size_t, "unsigned long long": ctypes.c_ulonglong,
+            "hybrid_status": ctypes.c_int}[kind]
+
+
+def test_binding_argtypes_match_the_header(L):
+    """Every exported entry point is bound with its declared return type and one
+    ctypes argument per declared parameter, of the declared kind (a pointer or
+    stream as a pointer, int, size_t, unsigned long long), so the binding cannot
+    drift from include/hybrid.h."""
+    sigs = declared_signatures()
+    assert set(sigs) == set(H.EXPORTED)
+    restypes = {"hybrid_status": ctypes.c_int, "size_t": ctypes.c_size_t, "const char *": ctypes.c_char_p}
+    for name, (ret, params) in sigs.items():
+        assert getattr(L, name).restype is restypes[ret], (name, ret)
+        argtypes = getattr(L, name).argtypes
+        assert len(argtypes) == len(params), name
+        for decl, at in zip(params, argtypes):
+            want = _ctype_of(decl)
+            if want == "pointer":
+                assert at is ctypes.c_void_p or issubclass(at, ctypes._Pointer), (name, decl, at)
+            else:
+                assert at is want, (name, decl, at)
