@@ -267,3 +267,56 @@ def test_binding_argtypes_match_the_header(L):
                 assert at is ctypes.c_void_p or issubclass(at, ctypes._Pointer), (name, decl, at)
             else:
                 assert at is want, (name, decl, at)
+
+
+# (entry point, argument roles after cfg): "p16"/"p8"/"p4" a pointer that must be
+# 16/8/4-byte aligned, "n" the request or row count, "i:<v>" another int, "s" the stream
+_POINTER_ARGS = {
+    "hybrid_state_init": ["p8", "n", "s"],
+    "hybrid_feature_map": ["p16", "n", "i:4", "p16", "p16", "s"],
+    "hybrid_block_attn": ["p16", "p16", "p16", "p16", "p4", "p8", "n", "p16", "s"],
+    "hybrid_block_attn_commit": ["p16", "p16", "p16", "p16", "p4", "p8", "n", "p16", "s"],
+    "hybrid_block_attn_commit_logical": ["p16", "p16", "p16", "p16", "p4", "p4", "p4", "n", "p16", "s"],
+    "hybrid_commit_block": ["p16", "p16", "i:32", "p16", "p8", "n", "s"],
+    "hybrid_state_unpack": ["p8", "n", "p4", "p4", "s"],
+    "hybrid_state_pack": ["p4", "p4", "p8", "n", "s"],
+}
+
+
+def _args(roles, override=None):
+    base = 1 << 20
+    out = []
+    for i, r in enumerate(roles):
+        if override and i in override:
+            out.append(override[i])
+        elif r.startswith("p"):
+            out.append(base + 4096 * i)
+        elif r == "n":
+            out.append(1)
+        elif r.startswith("i:"):
+            out.append(int(r[2:]))
+        else:
+            out.append(None)
+    return out
+
+
+@pytest.mark.parametrize("name", sorted(_POINTER_ARGS))
+def test_every_pointer_argument_is_checked_on_host(L, name):
+    """Each pointer argument of each entry point, made null or misaligned in turn
+    (every other argument valid), is rejected with HYBRID_ERR_INVALID_ARG before
+    the device is touched; with no requests every pointer may be null."""
+    c = cfg(d=128, F=128, Hq=16, Hkv=4, Bs=32)
+    roles = _POINTER_ARGS[name]
+    assert len(roles) + 1 == len(getattr(L, name).argtypes)
+    fn = getattr(L, name)
+    for i, r in enumerate(roles):
+        if not r.startswith("p"):
+            continue
+        align = int(r[1:])
+        base = _args(roles)[i]
+        assert fn(ctypes.byref(c), *_args(roles, {i: None})) == H.HYBRID_ERR_INVALID_ARG, (name, i, "null")
+        assert fn(ctypes.byref(c), *_args(roles, {i: base + align // 2})) == H.HYBRID_ERR_INVALID_ARG, (name, i)
+    if name == "hybrid_block_attn_commit_logical":
+        return   # with no requests it still looks up its scratch (a set-up call), which needs a device
+    empty = {i: (0 if r == "n" else None) for i, r in enumerate(roles) if r == "n" or r.startswith("p")}
+    assert fn(ctypes.byref(c), *_args(roles, empty)) == H.HYBRID_OK
