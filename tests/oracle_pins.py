@@ -510,6 +510,34 @@ def pin_train_backward_saturated_gate(orc):
     assert dalpha[1] == 0.0 and np.all(np.isfinite(dW)), "saturated gate"
 
 
+def pin_thread_count_changes_nothing(orc):
+    """The oracle fans independent (request, head) units out over threads; every
+    route gives the same bits on 1 thread and on 7 (more threads than units for
+    some calls, fewer for others), so no unit is skipped, repeated or shares
+    scratch with another."""
+    p = _random_problem(_rng(41), n_req=5, B=3, Hq=4, Hkv=2, d=6, F=3, P_max=4)
+    S1, z1 = orc.empty_state(5, 2, 6, 3)
+    S7, z7 = orc.empty_state(5, 2, 6, 3)
+    orc.commit(p["Kp"], p["Vp"], p["W"], S1, z1, n_threads=1)
+    orc.commit(p["Kp"], p["Vp"], p["W"], S7, z7, n_threads=7)
+    _close(S7, S1, rtol=0, atol=0, what="commit S")
+    _close(z7, z1, rtol=0, atol=0, what="commit z")
+    args = (p["Q"], p["K"], p["V"], p["W"], p["alpha"])
+    _close(orc.block_attn(*args, S1, z1, n_threads=7), orc.block_attn(*args, S1, z1, n_threads=1),
+           rtol=0, atol=0, what="state route")
+    _close(orc.block_attn_prefix(*args, p["Kp"], p["Vp"], p["prefix_len"], n_threads=7),
+           orc.block_attn_prefix(*args, p["Kp"], p["Vp"], p["prefix_len"], n_threads=1),
+           rtol=0, atol=0, what="prefix route")
+    t = _train_problem(_rng(42), n_seq=3, n_blk=3, B=2, Hq=4, Hkv=2, d=4, F=3)
+    targs = (t["Q"], t["K"], t["V"], t["W"], t["alpha"])
+    _close(orc.train_forward(*targs, t["B"], n_threads=7), orc.train_forward(*targs, t["B"], n_threads=1),
+           rtol=0, atol=0, what="training forward")
+    g7 = orc.train_backward(*targs, t["dO"], t["B"], n_threads=7)
+    g1 = orc.train_backward(*targs, t["dO"], t["B"], n_threads=1)
+    for a, b, what in zip(g7, g1, ("dW", "dalpha")):
+        _close(a, b, rtol=0, atol=0, what=f"training {what}")
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]
 
 

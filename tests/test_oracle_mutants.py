@@ -71,6 +71,9 @@ MUTANTS = [
      "const size_t t0 = (size_t)s * c->L + (size_t)n * B;"),
     ("train forward every sequence reads the first", "const size_t t0 = (size_t)s * c->L + (size_t)n * B;   /* first token of block n */",
      "const size_t t0 = (size_t)0 * s * c->L + (size_t)n * B;   /* first token of block n */"),
+    ("fan-out: threads after the first start one unit late",
+     "for (long u = a->tid; u < a->n_units; u += a->n_threads) {",
+     "for (long u = a->tid + (a->tid > 0); u < a->n_units; u += a->n_threads) {"),
     # head and request indexing of the inference routes
     ("commit uses state head 0's W", "const double *Wg = c->W ? c->W + (size_t)g * d * F : NULL;\n    for (int t = 0; t < c->T; ++t) {",
      "const double *Wg = c->W ? c->W + (size_t)0 * g * d * F : NULL;\n    for (int t = 0; t < c->T; ++t) {"),
