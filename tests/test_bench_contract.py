@@ -153,3 +153,22 @@ def test_clock_sampler_reads_clocks_and_throttle_reasons(tmp_path, monkeypatch):
     # a window with no samples says so instead of reporting a clock
     far = cs.summary(t1 + 100, t1 + 101)
     assert far["sm_mhz"] is None and far["samples"] == 0
+
+
+def test_algorithmic_bytes_of_the_context_configurations():
+    """The per-call bytes the c2, c4 and c5 context lines divide by, from the
+    shapes alone: Q and O once, K and V once, every state once per direction,
+    W, alpha and the pointer array."""
+    for wl, step, commit in ((wk.C2, None, None), (wk.C4, 84_934_976, 144_179_456),
+                             (wk.C5, 1_351_616_576, 2_299_529_216)):
+        n, Bk, Hq, Hkv, d, F = wl.n_req, wl.B, wl.Hq, wl.Hkv, wl.d, wl.F
+        q, kv = n * Bk * Hq * d * 2, n * Bk * Hkv * d * 2
+        state = n * Hkv * (2 * F * d + 2 * F) * 4
+        w = Hkv * d * F * 2
+        ab = bench.algorithmic_bytes(wl, 2)
+        assert ab["attn"] == 2 * q + 2 * kv + state + w + 4 * Hq + 8 * n, wl.name
+        assert ab["commit"] == 2 * kv + 2 * state + w + 8 * n, wl.name
+        assert ab["fused"] == ab["attn"] + state, wl.name
+        if step is not None:
+            assert (ab["attn"], ab["commit"]) == (step, commit), wl.name
+    assert bench.algorithmic_bytes(wk.C2, 2)["fused"] == 38_535_296
